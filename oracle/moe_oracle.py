@@ -1,0 +1,362 @@
+"""CPU oracle for the DeepSeek-V3 MoE layer forward (test infrastructure only).
+
+This module is the slow, obviously-correct statement of what the GPU path
+computes. Only the test-suite, the smoke check and the CPU-baseline leg of the
+benchmark may import it; the product library never calls it and shares no code
+with it. Every array here is numpy; floating-point work is fp64 unless a step
+states otherwise.
+
+What the layer computes (the paper's DeepSeek-V3 MoE workload, Appendix
+"Workload Details" and the host MoE listing of Appendix "Static Analysis
+Example"): route each token to k experts, dispatch (pack) the tokens into
+per-expert contiguous buffers, run GEMM1 (gate/up projection, H x 2I), SwiGLU,
+GEMM2 (down projection, I x H) per expert, then combine the expert outputs back
+into token order with the gate weights. The single-GPU form replaces both
+AlltoAll exchanges by on-device permutations (the paper's variable-size
+per-peer transfers become unpadded per-expert segments). The routing rule is
+not restated by the paper; it follows the DeepSeek-V3 layer the paper names:
+
+* sigmoid gating: s = sigmoid(L); a learned bias b is added for *selection
+  only* (s' = s + b); experts are split into G contiguous groups, a group's
+  score is the sum of its two largest s'; the top K_g groups are kept; the
+  top-k experts by s' among kept groups are selected; the weights are the
+  unbiased s of the selected experts, normalised to sum 1 and scaled by
+  `route_scale`.
+* softmax gating (the tiny configuration): p = softmax(L) over all experts;
+  the top-k by p are selected; weights are p (not renormalised) times
+  `route_scale`.
+
+Readings taken where the paper is silent (also listed in the design doc):
+* Decisions (which experts, which groups) are taken on fp32 scores: the
+  selection score is fp32(sigmoid(L)) + fp32 bias (one fp32 add); the group
+  score is the fp32 sum of the two largest selection scores.
+* Ties are broken by lower index (experts and groups). Output slot j = 0..k-1
+  lists the selected experts in descending selection score.
+* The SwiGLU activation h = silu(g) * u is rounded to bf16 (round to nearest
+  even) before GEMM2, because GEMM2 consumes bf16 operands.
+* W13 of one expert is [2I, H]: rows 0..I-1 are the gate projection, rows
+  I..2I-1 the up projection; W2 is [H, I]. Both are row-major with the
+  reduction dimension contiguous.
+
+Parity status: the paper prints no numeric example for the MoE layer, so each
+function is pinned by closed forms, invariants and brute force in
+tests/test_oracle.py; the absolute values of the full layer are
+"parity unpinned" against the paper itself.
+"""
+
+from __future__ import annotations
+
+from dataclasses import dataclass
+
+import numpy as np
+
+GATE_SOFTMAX = 0
+GATE_SIGMOID = 1
+
+
+@dataclass(frozen=True)
+class LayerConfig:
+    """Shapes and routing knobs of one MoE layer.
+
+    T tokens, H hidden, E routed experts, k experts per token, I expert
+    intermediate size, I_shared the shared expert's intermediate size (0 = no
+    shared expert), n_groups expert groups, topk_groups groups kept, gate
+    GATE_SOFTMAX or GATE_SIGMOID, normalize (1 = weights renormalised to sum 1
+    before scaling), route_scale the final weight scale.
+    """
+
+    T: int
+    H: int
+    E: int
+    k: int
+    I: int
+    I_shared: int = 0
+    n_groups: int = 1
+    topk_groups: int = 1
+    gate: int = GATE_SIGMOID
+    normalize: int = 1
+    route_scale: float = 1.0
+
+
+# ---------------------------------------------------------------------------
+# number formats
+# ---------------------------------------------------------------------------
+
+def bf16_round(a) -> np.ndarray:
+    """Round real values to the nearest bfloat16 value, ties to even.
+
+    bfloat16 keeps 8 significant bits (1 implicit + 7 stored). Writing
+    a = m * 2**e with 0.5 <= |m| < 1, the nearest bf16 is rint(m * 2**8) *
+    2**(e - 8), where rint rounds half to even. Exact for every finite fp64
+    input in the normal bf16 range (the only range the layer produces).
+    """
+    a = np.asarray(a, dtype=np.float64)
+    m, e = np.frexp(a)
+    return np.ldexp(np.rint(m * 256.0), e - 8)
+
+
+def sigmoid(x) -> np.ndarray:
+    """Logistic function 1 / (1 + exp(-x)) in fp64."""
+    x = np.asarray(x, dtype=np.float64)
+    return 1.0 / (1.0 + np.exp(-x))
+
+
+def silu(x) -> np.ndarray:
+    """SiLU (swish) x * sigmoid(x) = x / (1 + exp(-x)) in fp64."""
+    x = np.asarray(x, dtype=np.float64)
+    return x / (1.0 + np.exp(-x))
+
+
+# ---------------------------------------------------------------------------
+# step 1: router logits
+# ---------------------------------------------------------------------------
+
+def router_logits(x, Wr) -> np.ndarray:
+    """L[t, e] = sum_h x[t, h] * Wr[e, h], accumulated in fp64, rounded once to fp32.
+
+    x: [T, H] (bf16 values held in any float dtype); Wr: [E, H] fp32.
+    Returns fp32 [T, E], the precision the routing decisions are taken in.
+    """
+    x = np.asarray(x, dtype=np.float64)
+    Wr = np.asarray(Wr, dtype=np.float64)
+    return (x @ Wr.T).astype(np.float32)
+
+
+# ---------------------------------------------------------------------------
+# step 2: gating and group-limited top-k
+# ---------------------------------------------------------------------------
+
+def gate_scores(L32, cfg: LayerConfig):
+    """Per-expert gate scores from fp32 logits.
+
+    Returns (score64, score32): the exact score in fp64 (used for weights) and
+    the same score rounded to fp32 (used for decisions).
+    sigmoid gating: score = sigmoid(L). softmax gating: score = exp(L - max) /
+    sum(exp(L - max)) over all E experts of the token.
+    """
+    L = np.asarray(L32, dtype=np.float64)
+    if cfg.gate == GATE_SIGMOID:
+        s = sigmoid(L)
+    elif cfg.gate == GATE_SOFTMAX:
+        z = np.exp(L - L.max(axis=1, keepdims=True))
+        s = z / z.sum(axis=1, keepdims=True)
+    else:
+        raise ValueError("unknown gate")
+    return s, s.astype(np.float32)
+
+
+def selection_scores(L32, bias32, cfg: LayerConfig) -> np.ndarray:
+    """fp32 selection score s' = fp32(score) + bias (a single fp32 add); bias None = 0."""
+    _, s32 = gate_scores(L32, cfg)
+    if bias32 is None:
+        return s32
+    return (s32 + np.asarray(bias32, dtype=np.float32)[None, :]).astype(np.float32)
+
+
+def _order_desc(values, axis=-1) -> np.ndarray:
+    """Indices that sort `values` descending, ties by lower index (stable)."""
+    return np.argsort(-np.asarray(values), axis=axis, kind="stable")
+
+
+def group_scores(sel32, cfg: LayerConfig) -> np.ndarray:
+    """Group score: fp32 sum of the two largest selection scores in each group.
+
+    Groups are contiguous: group g holds experts [g*E/G, (g+1)*E/G). A group of
+    one expert scores that expert's selection score.
+    """
+    T, E = sel32.shape
+    G = cfg.n_groups
+    gs = E // G
+    grouped = sel32.reshape(T, G, gs)
+    srt = -np.sort(-grouped, axis=2)            # descending within each group
+    if gs == 1:
+        return srt[:, :, 0].astype(np.float32)
+    return (srt[:, :, 0] + srt[:, :, 1]).astype(np.float32)  # fp32 + fp32
+
+
+def kept_expert_mask(sel32, cfg: LayerConfig) -> np.ndarray:
+    """Boolean [T, E]: experts whose group is among the top `topk_groups` groups."""
+    T, E = sel32.shape
+    G = cfg.n_groups
+    if G <= 1 or cfg.topk_groups >= G:
+        return np.ones((T, E), dtype=bool)
+    gsc = group_scores(sel32, cfg)
+    order = _order_desc(gsc, axis=1)[:, : cfg.topk_groups]
+    keep_g = np.zeros((T, G), dtype=bool)
+    np.put_along_axis(keep_g, order, True, axis=1)
+    return np.repeat(keep_g, E // G, axis=1)
+
+
+def gate_topk(L32, bias32, cfg: LayerConfig):
+    """Route each token: returns (idx [T,k] int32, w [T,k] fp64).
+
+    Selection on fp32 s' restricted to kept groups, descending, ties by lower
+    expert index. Weights from the unbiased fp64 score of the chosen experts:
+    normalised to sum 1 when cfg.normalize, then multiplied by route_scale.
+    """
+    L32 = np.asarray(L32, dtype=np.float32)
+    s64, _ = gate_scores(L32, cfg)
+    sel = selection_scores(L32, bias32, cfg)
+    keep = kept_expert_mask(sel, cfg)
+    masked = np.where(keep, sel.astype(np.float64), -np.inf)
+    idx = _order_desc(masked, axis=1)[:, : cfg.k].astype(np.int32)
+    w = np.take_along_axis(s64, idx, axis=1)
+    if cfg.normalize:
+        w = w / w.sum(axis=1, keepdims=True)
+    w = w * cfg.route_scale
+    return idx, w
+
+
+def routing_margins(L32, bias32, cfg: LayerConfig) -> np.ndarray:
+    """Per-token decision margin (fp64 view of the fp32 scores).
+
+    min over: (k-th minus (k+1)-th selection score among kept experts) and
+    (topk_groups-th minus (topk_groups+1)-th group score). A large margin means
+    every routing decision of the token survives fp32 rounding differences.
+    """
+    sel = selection_scores(L32, bias32, cfg).astype(np.float64)
+    keep = kept_expert_mask(sel.astype(np.float32), cfg)
+    masked = np.where(keep, sel, -np.inf)
+    srt = -np.sort(-masked, axis=1)
+    T = sel.shape[0]
+    m = np.full(T, np.inf)
+    if srt.shape[1] > cfg.k:
+        nxt = srt[:, cfg.k]
+        gap = np.where(np.isfinite(nxt), srt[:, cfg.k - 1] - nxt, np.inf)
+        m = np.minimum(m, gap)
+    G = cfg.n_groups
+    if 1 < G and cfg.topk_groups < G:
+        gsc = -np.sort(-group_scores(sel.astype(np.float32), cfg).astype(np.float64), axis=1)
+        m = np.minimum(m, gsc[:, cfg.topk_groups - 1] - gsc[:, cfg.topk_groups])
+    return m
+
+
+# ---------------------------------------------------------------------------
+# step 3: histogram, scan and permutation (the on-device "AlltoAll")
+# ---------------------------------------------------------------------------
+
+def permutation(idx, E: int):
+    """Stable expert-major permutation of the T*k (token, slot) entries.
+
+    counts[e] = number of entries routed to e; offsets = exclusive prefix sum
+    (length E+1); the rows of expert e are its entries ordered by (t, j);
+    row_src_token[r] = token of row r; slot_row[t*k + j] = row of entry (t, j).
+    """
+    idx = np.asarray(idx)
+    T, k = idx.shape
+    flat = idx.reshape(-1).astype(np.int64)
+    counts = np.bincount(flat, minlength=E).astype(np.int32)
+    offsets = np.zeros(E + 1, dtype=np.int32)
+    offsets[1:] = np.cumsum(counts)
+    order = np.argsort(flat, kind="stable")     # entries sorted by expert, then t*k+j
+    row_src_token = (order // k).astype(np.int32)
+    slot_row = np.empty(T * k, dtype=np.int32)
+    slot_row[order] = np.arange(T * k, dtype=np.int32)
+    return counts, offsets, row_src_token, slot_row
+
+
+def dispatch(x, row_src_token) -> np.ndarray:
+    """x_perm[r] = x[row_src_token[r]] (a pure copy)."""
+    return np.asarray(x)[np.asarray(row_src_token)]
+
+
+# ---------------------------------------------------------------------------
+# steps 4-5: expert FFN (GEMM1 + SwiGLU + GEMM2) and the shared expert
+# ---------------------------------------------------------------------------
+
+def swiglu_ffn(rows, W13_e, W2_e) -> np.ndarray:
+    """One SwiGLU expert on a block of rows, fp64 accumulation.
+
+    rows [m, H]; W13_e [2I, H] (gate rows then up rows); W2_e [H, I].
+    g = rows . Wg^T, u = rows . Wu^T, h = bf16(silu(g) * u), y = h . W2^T.
+    """
+    rows = np.asarray(rows, dtype=np.float64)
+    W13_e = np.asarray(W13_e, dtype=np.float64)
+    W2_e = np.asarray(W2_e, dtype=np.float64)
+    I = W13_e.shape[0] // 2
+    g = rows @ W13_e[:I].T
+    u = rows @ W13_e[I:].T
+    h = bf16_round(silu(g) * u)
+    return h @ W2_e.T
+
+
+def expert_ffn(x_perm, offsets, W13, W2) -> np.ndarray:
+    """Grouped expert FFN: y_perm[r] = FFN_e(x_perm[r]) for r in expert e's segment."""
+    x_perm = np.asarray(x_perm, dtype=np.float64)
+    H = W2[0].shape[0] if len(W2) else x_perm.shape[1]
+    y = np.zeros((x_perm.shape[0], H), dtype=np.float64)
+    E = len(offsets) - 1
+    for e in range(E):
+        a, b = int(offsets[e]), int(offsets[e + 1])
+        if b > a:
+            y[a:b] = swiglu_ffn(x_perm[a:b], W13[e], W2[e])
+    return y
+
+
+# ---------------------------------------------------------------------------
+# step 6: combine (the reverse "AlltoAll")
+# ---------------------------------------------------------------------------
+
+def combine(y_perm, slot_row, w, shared=None) -> np.ndarray:
+    """out[t] = sum_j w[t, j] * y_perm[slot_row[t*k + j]] (+ shared[t]), fp64."""
+    w = np.asarray(w, dtype=np.float64)
+    T, k = w.shape
+    y = np.asarray(y_perm, dtype=np.float64)
+    rows = np.asarray(slot_row).reshape(T, k)
+    out = np.zeros((T, y.shape[1]), dtype=np.float64)
+    for j in range(k):
+        out += w[:, j : j + 1] * y[rows[:, j]]
+    if shared is not None:
+        out += np.asarray(shared, dtype=np.float64)
+    return out
+
+
+# ---------------------------------------------------------------------------
+# the whole layer
+# ---------------------------------------------------------------------------
+
+def layer_forward(x, Wr, bias, W13, W2, cfg: LayerConfig, Ws13=None, Ws2=None, logits=None):
+    """Full layer forward over all T tokens, in the paper's stage order.
+
+    route -> dispatch -> expert FFN -> combine (+ shared expert). `logits`
+    (fp32 [T, E]) may be supplied to route on given logits. Returns (out fp64
+    [T, H], aux dict with logits, idx, w, counts, offsets, row_src_token,
+    slot_row, y_perm).
+    """
+    x = np.asarray(x, dtype=np.float64)
+    L32 = router_logits(x, Wr) if logits is None else np.asarray(logits, dtype=np.float32)
+    idx, w = gate_topk(L32, bias, cfg)
+    counts, offsets, rst, slot_row = permutation(idx, cfg.E)
+    x_perm = dispatch(x, rst)
+    y_perm = expert_ffn(x_perm, offsets, W13, W2)
+    shared = None
+    if cfg.I_shared and Ws13 is not None:
+        shared = swiglu_ffn(x, Ws13, Ws2)
+    out = combine(y_perm, slot_row, w, shared)
+    aux = dict(logits=L32, idx=idx, w=w, counts=counts, offsets=offsets,
+               row_src_token=rst, slot_row=slot_row, y_perm=y_perm, shared=shared)
+    return out, aux
+
+
+def layer_forward_tokens(x_rows, Wr, bias, get_expert, cfg: LayerConfig, get_shared=None):
+    """Layer output for a sample of tokens, one token at a time.
+
+    Routing is independent per token, so a token's output needs only its own
+    row. x_rows [n, H]; get_expert(e) -> (W13_e, W2_e); get_shared() ->
+    (Ws13, Ws2) or None. Experts are visited once each, with all sampled rows
+    routed to them. Returns (out fp64 [n, H], idx [n, k], w [n, k]).
+    """
+    x_rows = np.asarray(x_rows, dtype=np.float64)
+    L32 = router_logits(x_rows, Wr)
+    idx, w = gate_topk(L32, bias, cfg)
+    n = x_rows.shape[0]
+    out = np.zeros((n, cfg.H), dtype=np.float64)
+    for e in np.unique(idx):
+        who, slot = np.nonzero(idx == e)
+        W13_e, W2_e = get_expert(int(e))
+        y = swiglu_ffn(x_rows[who], W13_e, W2_e)
+        out[who] += w[who, slot][:, None] * y
+    if get_shared is not None and cfg.I_shared:
+        Ws13, Ws2 = get_shared()
+        out += swiglu_ffn(x_rows, Ws13, Ws2)
+    return out, idx, w

@@ -1,0 +1,224 @@
+/*
+ * moe.h -- C ABI of the single-GPU DeepSeek-V3 MoE layer forward (sm_103a).
+ *
+ * The operation is the MoE layer of the CUCo paper's DeepSeek-V3 workload
+ * (Appendix "Workload Details"; host pipeline listing in Appendix "Static
+ * Analysis Example"): route tokens to experts, dispatch them into per-expert
+ * contiguous buffers, run GEMM1 (gate/up, H -> 2I) + SwiGLU + GEMM2 (down,
+ * I -> H) per expert, and combine the expert outputs back into token order
+ * with the gate weights. On one GPU the two AlltoAll exchanges of the paper
+ * become on-device permutations; the paper's variable-size per-peer transfers
+ * become unpadded per-expert row segments, and its "dispatch on a
+ * high-priority stream, hidden behind local compute" (Section 4.3) becomes a
+ * two-stream chunked pipeline inside one device.
+ *
+ * Conventions shared by every entry point:
+ *  - Tensor pointers are DEVICE pointers owned by the caller, row-major and
+ *    contiguous. bf16 tensors are passed as uint16_t bit patterns and must be
+ *    16-byte aligned (they are read by 16-byte vector loads and TMA); other
+ *    tensors must be 4-byte aligned.
+ *  - `stream` is a cudaStream_t passed as void* (NULL = the legacy default
+ *    stream). Every call only enqueues work on its stream(s): it does not
+ *    synchronise, does not allocate device memory and does not abort.
+ *  - Arguments are validated on the host before anything is launched; a bad
+ *    argument returns MOE_ERR_INVALID_ARG or MOE_ERR_UNSUPPORTED and enqueues
+ *    nothing. A failed launch returns MOE_ERR_CUDA.
+ *  - Kernels that wait on on-chip barriers give up after a bounded time and
+ *    latch MOE_ERR_TIMEOUT in a device error word; moe_check_errors() reads it.
+ *  - The library keeps no state between calls except lazily created internal
+ *    streams/events and per-device symbol addresses, released by moe_shutdown().
+ */
+#ifndef MOE_H_
+#define MOE_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+  MOE_OK = 0,
+  MOE_ERR_INVALID_ARG = 1,   /* null/misaligned pointer, bad size or knob */
+  MOE_ERR_UNSUPPORTED = 2,   /* valid but outside what the kernels implement */
+  MOE_ERR_WORKSPACE = 3,     /* workspace missing or smaller than required */
+  MOE_ERR_CUDA = 4,          /* a CUDA runtime call or launch failed */
+  MOE_ERR_TIMEOUT = 5,       /* a bounded on-device wait expired (latched) */
+  MOE_ERR_DEVICE_CHECK = 6   /* an on-device consistency check failed (latched) */
+} moe_status;
+
+typedef enum { MOE_GATE_SOFTMAX = 0, MOE_GATE_SIGMOID = 1 } moe_gate;
+
+/*
+ * Layer shape and routing rule.
+ *  T tokens; H hidden size (multiple of 128); E routed experts (1..1024);
+ *  k experts per token (1..32, k <= E); I expert intermediate size (multiple
+ *  of 128); I_shared shared-expert intermediate size (0 = none, else a
+ *  multiple of 128); n_groups expert groups (1..32, divides E); topk_groups
+ *  groups kept (1..n_groups, with k <= topk_groups * E / n_groups); gate a
+ *  moe_gate; normalize 1 = renormalise the k weights to sum 1 before scaling;
+ *  route_scale final weight multiplier.
+ * Routing rule (DeepSeek-V3, the layer the paper's MoE workload reproduces):
+ *  sigmoid: s = sigmoid(L), selection score s' = s + bias (fp32); group score =
+ *  sum of the two largest s' of the group; keep the top topk_groups groups;
+ *  pick the top-k s' among kept experts (ties: lower index); weights = s of
+ *  the picked experts (normalised if `normalize`) * route_scale.
+ *  softmax: s = softmax(L) over the E experts, otherwise identical.
+ */
+typedef struct {
+  int32_t T, H, E, k, I, I_shared, n_groups, topk_groups, gate, normalize;
+  float route_scale;
+} moe_config;
+
+/*
+ * Execution knobs of moe_layer_forward.
+ *  overlap 0 = one stream, stages in order; 1 = two-stream chunked pipeline:
+ *    chunk i+1 is routed and dispatched on a high-priority pack stream while
+ *    chunk i's experts compute (Section 4.3: dispatch hidden behind compute).
+ *  chunk_tokens tokens per chunk when overlap = 1 and chunk_axis = 0.
+ *  chunk_axis 0 = chunk by tokens (each chunk re-streams the expert weights);
+ *    1 = chunk by expert range within one full-T pass (weights read once):
+ *    the rows of expert range i+1 are packed while range i computes.
+ *  n_expert_chunks number of expert ranges when chunk_axis = 1.
+ *  out_fp32 0 = bf16 output, 1 = fp32 output.
+ */
+typedef struct {
+  int32_t overlap, chunk_tokens, chunk_axis, n_expert_chunks, out_fp32;
+} moe_exec;
+
+/* Layer weights (device pointers). Wr [E,H] fp32; bias [E] fp32 or NULL;
+ * W13 [E,2I,H] bf16 (rows 0..I-1 gate, I..2I-1 up); W2 [E,H,I] bf16;
+ * Ws13 [2*I_shared,H] bf16 and Ws2 [H,I_shared] bf16, NULL iff I_shared = 0. */
+typedef struct {
+  const float* Wr;
+  const float* bias;
+  const uint16_t* W13;
+  const uint16_t* W2;
+  const uint16_t* Ws13;
+  const uint16_t* Ws2;
+} moe_weights;
+
+/* Optional outputs of moe_layer_forward; NULL fields are skipped.
+ * logits [T,E] fp32; topk_idx [T,k] int32; topk_w [T,k] fp32; counts [E] int32. */
+typedef struct {
+  float* logits;
+  int32_t* topk_idx;
+  float* topk_w;
+  int32_t* counts;
+} moe_aux;
+
+/* Human-readable name of a status. Never NULL. */
+const char* moe_status_string(moe_status s);
+
+/* Host-only check of a configuration (no CUDA call). MOE_OK if every entry
+ * point accepts it. */
+moe_status moe_validate_config(const moe_config* cfg);
+
+/* Workspace bytes needed by moe_layer_forward for (cfg, ex); 0 on an invalid
+ * configuration. Host-only. */
+size_t moe_workspace_size(const moe_config* cfg, const moe_exec* ex);
+
+/* Workspace bytes of the split-K router partials (may be 0). Host-only. */
+size_t moe_router_workspace_size(const moe_config* cfg);
+
+/* Workspace bytes of moe_dispatch's per-chunk histograms. Host-only. */
+size_t moe_dispatch_workspace_size(const moe_config* cfg);
+
+/* Workspace bytes of moe_expert_ffn: the SwiGLU activations [rows, I] bf16. */
+size_t moe_expert_ffn_workspace_size(int32_t rows, int32_t I);
+
+/*
+ * Router logits: logits[t,e] = sum_h x[t,h] * Wr[e,h], fp32 accumulation.
+ * x [T,H] bf16; Wr [E,H] fp32; logits [T,E] fp32 (written). ws/ws_bytes:
+ * scratch for split-K partials (moe_router_workspace_size bytes); with ws NULL
+ * the reduction is not split. The gating of every routed token starts here
+ * (the paper's workload routes each token to its experts, Section 4).
+ */
+moe_status moe_router_logits(const moe_config* cfg, const uint16_t* x, const float* Wr,
+                             float* logits, void* ws, size_t ws_bytes, void* stream);
+
+/*
+ * Gate + group-limited top-k (the routing rule of moe_config).
+ * logits [T,E] fp32; bias [E] fp32 or NULL (selection only);
+ * topk_idx [T,k] int32 (written, slot j in descending selection score);
+ * topk_w [T,k] fp32 (written).
+ */
+moe_status moe_gate_topk(const moe_config* cfg, const float* logits, const float* bias,
+                         int32_t* topk_idx, float* topk_w, void* stream);
+
+/*
+ * Dispatch: the single-GPU form of the paper's AlltoAll dispatch (host MoE
+ * listing; "variable-size per-peer transfers that avoid padding",
+ * Appendix "Workload Details"). Computes a stable expert-major permutation of
+ * the T*k (token, slot) entries and optionally packs the token rows.
+ * topk_idx [T,k] int32 (values in [0,E)); counts [E] (written); offsets [E+1]
+ * (written, exclusive prefix sum of counts); row_src_token [T*k] (written:
+ * token of each packed row); slot_row [T*k] (written: packed row of entry
+ * t*k+j). Rows of one expert are ordered by (t, j). x [T,H] bf16 and x_perm
+ * [T*k,H] bf16: x_perm[r] = x[row_src_token[r]]; x_perm NULL = permutation
+ * only (x may then be NULL). ws: moe_dispatch_workspace_size bytes.
+ */
+moe_status moe_dispatch(const moe_config* cfg, const uint16_t* x, const int32_t* topk_idx,
+                        int32_t* counts, int32_t* offsets, int32_t* row_src_token,
+                        int32_t* slot_row, uint16_t* x_perm, void* ws, size_t ws_bytes,
+                        void* stream);
+
+/*
+ * Grouped expert FFN (GEMM1 + SwiGLU + GEMM2 of the paper's expert compute,
+ * shapes 7168 x 4096 and 2048 x 7168 in Appendix "Workload Details").
+ * For each expert e < n_experts and each row r in [offsets[e], offsets[e+1]):
+ *   h[r] = bf16(silu(x_perm[r] . Wg_e^T) * (x_perm[r] . Wu_e^T)),
+ *   y_perm[r] = bf16(h[r] . W2_e^T)        (fp32 accumulation throughout).
+ * rows: rows of x_perm / y_perm; H hidden (multiple of 128); I intermediate
+ * (multiple of 128); offsets [n_experts+1] int32 on the device, non-decreasing,
+ * offsets[n_experts] <= rows; W13 [n_experts,2I,H]; W2 [n_experts,H,I];
+ * x_perm [rows,H]; y_perm [rows,H] (written; rows outside every segment are
+ * left untouched). ws: moe_expert_ffn_workspace_size(rows, I) bytes.
+ * The shared expert is this call with n_experts = 1 and offsets = {0, T}.
+ */
+moe_status moe_expert_ffn(int32_t rows, int32_t H, int32_t I, int32_t n_experts,
+                          const uint16_t* x_perm, const int32_t* offsets, const uint16_t* W13,
+                          const uint16_t* W2, uint16_t* y_perm, void* ws, size_t ws_bytes,
+                          void* stream);
+
+/*
+ * Combine: the single-GPU form of the paper's reverse AlltoAll combine.
+ * out[t] = sum_j topk_w[t,j] * y_perm[slot_row[t*k+j]] (+ shared_out[t]),
+ * fp32 accumulation in slot order j = 0..k-1, then the shared term.
+ * y_perm [T*k,H] bf16; slot_row [T*k]; topk_w [T,k] fp32; shared_out [T,H]
+ * bf16 or NULL; out [T,H] bf16 (out_fp32 = 0) or fp32 (out_fp32 = 1).
+ */
+moe_status moe_combine(const moe_config* cfg, const uint16_t* y_perm, const int32_t* slot_row,
+                       const float* topk_w, const uint16_t* shared_out, void* out,
+                       int32_t out_fp32, void* stream);
+
+/*
+ * The whole layer: router -> gate/top-k -> dispatch -> grouped expert FFN
+ * (+ shared expert) -> combine, in the paper's stage order.
+ * x [T,H] bf16; out [T,H] bf16 or fp32 per ex->out_fp32; aux optional;
+ * ws: moe_workspace_size(cfg, ex) bytes. aux_stream: the pack stream of the
+ * overlapped pipeline (NULL = an internal high-priority stream); unused when
+ * ex->overlap = 0. All work is ordered after prior work on `stream`, and later
+ * work on `stream` is ordered after the whole layer.
+ */
+moe_status moe_layer_forward(const moe_config* cfg, const moe_exec* ex, const moe_weights* w,
+                             const uint16_t* x, void* out, const moe_aux* aux, void* ws,
+                             size_t ws_bytes, void* stream, void* aux_stream);
+
+/* Synchronises `stream`, then reads and clears the device error word of the
+ * current device. MOE_OK, MOE_ERR_TIMEOUT or MOE_ERR_DEVICE_CHECK (or
+ * MOE_ERR_CUDA if the synchronisation itself failed). */
+moe_status moe_check_errors(void* stream);
+
+/* Number of kernels this library has launched in this process (all devices). */
+uint64_t moe_launch_count(void);
+
+/* Releases internal streams and events. Safe to call more than once. */
+void moe_shutdown(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* MOE_H_ */

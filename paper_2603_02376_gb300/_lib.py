@@ -1,0 +1,227 @@
+"""ctypes binding of libmoe.so: the C ABI of include/moe.h, same names.
+
+Argument marshalling only: torch tensors are passed as raw device pointers
+(data_ptr) and streams as cudaStream_t handles; every step runs in the
+library's CUDA kernels. A non-OK status raises MoeError. Loading fails loudly
+when the library has not been built.
+"""
+
+from __future__ import annotations
+
+import ctypes
+import os
+
+PKG = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(PKG, "libmoe.so")
+
+MOE_OK = 0
+MOE_ERR_INVALID_ARG = 1
+MOE_ERR_UNSUPPORTED = 2
+MOE_ERR_WORKSPACE = 3
+MOE_ERR_CUDA = 4
+MOE_ERR_TIMEOUT = 5
+MOE_ERR_DEVICE_CHECK = 6
+MOE_GATE_SOFTMAX = 0
+MOE_GATE_SIGMOID = 1
+
+EXPORTS = ("moe_status_string", "moe_validate_config", "moe_workspace_size",
+           "moe_router_workspace_size", "moe_dispatch_workspace_size",
+           "moe_expert_ffn_workspace_size", "moe_router_logits", "moe_gate_topk", "moe_dispatch",
+           "moe_expert_ffn", "moe_combine", "moe_layer_forward", "moe_check_errors",
+           "moe_launch_count", "moe_shutdown")
+
+
+class MoeError(RuntimeError):
+    def __init__(self, status: int, where: str):
+        super().__init__(f"{where}: {status_string(status)} ({status})")
+        self.status = status
+
+
+class moe_config(ctypes.Structure):
+    _fields_ = [(n, ctypes.c_int32) for n in
+                ("T", "H", "E", "k", "I", "I_shared", "n_groups", "topk_groups", "gate",
+                 "normalize")] + [("route_scale", ctypes.c_float)]
+
+
+class moe_exec(ctypes.Structure):
+    _fields_ = [(n, ctypes.c_int32) for n in
+                ("overlap", "chunk_tokens", "chunk_axis", "n_expert_chunks", "out_fp32")]
+
+
+class moe_weights(ctypes.Structure):
+    _fields_ = [(n, ctypes.c_void_p) for n in ("Wr", "bias", "W13", "W2", "Ws13", "Ws2")]
+
+
+class moe_aux(ctypes.Structure):
+    _fields_ = [(n, ctypes.c_void_p) for n in ("logits", "topk_idx", "topk_w", "counts")]
+
+
+_lib = None
+
+
+def load(path: str = LIB_PATH) -> ctypes.CDLL:
+    """Load libmoe.so (once). Raises if it has not been built."""
+    global _lib
+    if _lib is not None:
+        return _lib
+    if not os.path.exists(path):
+        raise RuntimeError(f"{path} is missing: build it with __graft_entry__.build() "
+                           "(python -m paper_2603_02376_gb300.build)")
+    lib = ctypes.CDLL(path)
+    P, I32, SZ, S = ctypes.c_void_p, ctypes.c_int32, ctypes.c_size_t, ctypes.c_int
+    cfgp = ctypes.POINTER(moe_config)
+    exp = ctypes.POINTER(moe_exec)
+    sig = {
+        "moe_status_string": (ctypes.c_char_p, [S]),
+        "moe_validate_config": (S, [cfgp]),
+        "moe_workspace_size": (SZ, [cfgp, exp]),
+        "moe_router_workspace_size": (SZ, [cfgp]),
+        "moe_dispatch_workspace_size": (SZ, [cfgp]),
+        "moe_expert_ffn_workspace_size": (SZ, [I32, I32]),
+        "moe_router_logits": (S, [cfgp, P, P, P, P, SZ, P]),
+        "moe_gate_topk": (S, [cfgp, P, P, P, P, P]),
+        "moe_dispatch": (S, [cfgp, P, P, P, P, P, P, P, P, SZ, P]),
+        "moe_expert_ffn": (S, [I32, I32, I32, I32, P, P, P, P, P, P, SZ, P]),
+        "moe_combine": (S, [cfgp, P, P, P, P, P, I32, P]),
+        "moe_layer_forward": (S, [cfgp, exp, ctypes.POINTER(moe_weights), P, P,
+                                  ctypes.POINTER(moe_aux), P, SZ, P, P]),
+        "moe_check_errors": (S, [P]),
+        "moe_launch_count": (ctypes.c_uint64, []),
+        "moe_shutdown": (None, []),
+    }
+    for name, (res, args) in sig.items():
+        f = getattr(lib, name)
+        f.restype = res
+        f.argtypes = args
+    _lib = lib
+    return lib
+
+
+def status_string(status: int) -> str:
+    try:
+        return load().moe_status_string(status).decode()
+    except Exception:  # the library itself may be what failed to load
+        return f"status {status}"
+
+
+def moe_status_string(status: int) -> str:
+    return load().moe_status_string(status).decode()
+
+
+def _check(status: int, where: str) -> None:
+    if status != MOE_OK:
+        raise MoeError(status, where)
+
+
+def _ptr(t):
+    return None if t is None else ctypes.c_void_p(t.data_ptr())
+
+
+def _stream(stream):
+    if stream is None:
+        import torch
+        stream = torch.cuda.current_stream()
+    return ctypes.c_void_p(int(getattr(stream, "cuda_stream", stream)))
+
+
+def config(T, H, E, k, I, I_shared=0, n_groups=1, topk_groups=1, gate=MOE_GATE_SIGMOID,
+           normalize=1, route_scale=1.0) -> moe_config:
+    return moe_config(T, H, E, k, I, I_shared, n_groups, topk_groups, gate, normalize,
+                      route_scale)
+
+
+def config_of(wl, T=None) -> moe_config:
+    """moe_config of an inputs.Workload (optionally with another token count)."""
+    return config(wl.T if T is None else T, wl.H, wl.E, wl.k, wl.I, wl.I_shared, wl.n_groups,
+                  wl.topk_groups, wl.gate, wl.normalize, wl.route_scale)
+
+
+def exec_config(overlap=0, chunk_tokens=512, chunk_axis=0, n_expert_chunks=8, out_fp32=0):
+    return moe_exec(overlap, chunk_tokens, chunk_axis, n_expert_chunks, out_fp32)
+
+
+# ---------------------------------------------------------------- entry points
+
+def moe_validate_config(cfg) -> int:
+    return load().moe_validate_config(ctypes.byref(cfg))
+
+
+def moe_workspace_size(cfg, ex) -> int:
+    return load().moe_workspace_size(ctypes.byref(cfg), ctypes.byref(ex))
+
+
+def moe_router_workspace_size(cfg) -> int:
+    return load().moe_router_workspace_size(ctypes.byref(cfg))
+
+
+def moe_dispatch_workspace_size(cfg) -> int:
+    return load().moe_dispatch_workspace_size(ctypes.byref(cfg))
+
+
+def moe_expert_ffn_workspace_size(rows, I) -> int:
+    return load().moe_expert_ffn_workspace_size(rows, I)
+
+
+def moe_router_logits(cfg, x, Wr, logits, ws=None, stream=None) -> None:
+    nb = 0 if ws is None else ws.numel() * ws.element_size()
+    _check(load().moe_router_logits(ctypes.byref(cfg), _ptr(x), _ptr(Wr), _ptr(logits), _ptr(ws),
+                                    nb, _stream(stream)), "moe_router_logits")
+
+
+def moe_gate_topk(cfg, logits, bias, topk_idx, topk_w, stream=None) -> None:
+    _check(load().moe_gate_topk(ctypes.byref(cfg), _ptr(logits), _ptr(bias), _ptr(topk_idx),
+                                _ptr(topk_w), _stream(stream)), "moe_gate_topk")
+
+
+def moe_dispatch(cfg, x, topk_idx, counts, offsets, row_src_token, slot_row, x_perm, ws,
+                 stream=None) -> None:
+    nb = 0 if ws is None else ws.numel() * ws.element_size()
+    _check(load().moe_dispatch(ctypes.byref(cfg), _ptr(x), _ptr(topk_idx), _ptr(counts),
+                               _ptr(offsets), _ptr(row_src_token), _ptr(slot_row), _ptr(x_perm),
+                               _ptr(ws), nb, _stream(stream)), "moe_dispatch")
+
+
+def moe_expert_ffn(rows, H, I, n_experts, x_perm, offsets, W13, W2, y_perm, ws,
+                   stream=None) -> None:
+    nb = 0 if ws is None else ws.numel() * ws.element_size()
+    _check(load().moe_expert_ffn(rows, H, I, n_experts, _ptr(x_perm), _ptr(offsets), _ptr(W13),
+                                 _ptr(W2), _ptr(y_perm), _ptr(ws), nb, _stream(stream)),
+           "moe_expert_ffn")
+
+
+def moe_combine(cfg, y_perm, slot_row, topk_w, shared_out, out, out_fp32, stream=None) -> None:
+    _check(load().moe_combine(ctypes.byref(cfg), _ptr(y_perm), _ptr(slot_row), _ptr(topk_w),
+                              _ptr(shared_out), _ptr(out), int(out_fp32), _stream(stream)),
+           "moe_combine")
+
+
+def weights_struct(Wr, bias, W13, W2, Ws13=None, Ws2=None) -> moe_weights:
+    return moe_weights(*(None if t is None else t.data_ptr()
+                         for t in (Wr, bias, W13, W2, Ws13, Ws2)))
+
+
+def aux_struct(logits=None, topk_idx=None, topk_w=None, counts=None) -> moe_aux:
+    return moe_aux(*(None if t is None else t.data_ptr()
+                     for t in (logits, topk_idx, topk_w, counts)))
+
+
+def moe_layer_forward(cfg, ex, weights: moe_weights, x, out, aux: moe_aux | None, ws,
+                      stream=None, aux_stream=None) -> None:
+    nb = 0 if ws is None else ws.numel() * ws.element_size()
+    auxp = None if aux is None else ctypes.byref(aux)
+    a_s = None if aux_stream is None else _stream(aux_stream)
+    _check(load().moe_layer_forward(ctypes.byref(cfg), ctypes.byref(ex), ctypes.byref(weights),
+                                    _ptr(x), _ptr(out), auxp, _ptr(ws), nb, _stream(stream), a_s),
+           "moe_layer_forward")
+
+
+def moe_check_errors(stream=None) -> None:
+    _check(load().moe_check_errors(_stream(stream)), "moe_check_errors")
+
+
+def moe_launch_count() -> int:
+    return int(load().moe_launch_count())
+
+
+def moe_shutdown() -> None:
+    load().moe_shutdown()

@@ -1,0 +1,88 @@
+// Internal helpers shared by the kernels of the MoE library (not part of the ABI).
+#pragma once
+
+#include <cuda.h>
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "moe.h"
+
+namespace moe {
+
+// ----------------------------------------------------------------------------
+// host-side bookkeeping
+// ----------------------------------------------------------------------------
+
+// Counts every kernel launch of the library (exported through moe_launch_count).
+void note_launch(int n = 1);
+
+// Device error word of the current device (a file-scope __device__ int).
+int* device_error_word();
+
+// Number of SMs of the current device (cached per device).
+int num_sms();
+
+// Status of the last launch on this thread.
+inline moe_status launch_status() {
+  return cudaPeekAtLastError() == cudaSuccess ? MOE_OK : MOE_ERR_CUDA;
+}
+
+inline size_t align_up(size_t v, size_t a) { return (v + a - 1) / a * a; }
+inline bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+inline bool aligned4(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 3u) == 0; }
+
+// ----------------------------------------------------------------------------
+// kernel launchers (defined in the kernel translation units)
+// ----------------------------------------------------------------------------
+
+moe_status launch_router(const moe_config& c, const uint16_t* x, const float* Wr, float* logits,
+                         float* partials, int splits, cudaStream_t s);
+int router_splits(const moe_config& c);
+
+moe_status launch_gate(const moe_config& c, const float* logits, const float* bias, int32_t* idx,
+                       float* w, cudaStream_t s);
+
+int perm_num_chunks(int T);
+moe_status launch_permutation(const moe_config& c, const int32_t* idx, int32_t* counts,
+                              int32_t* offsets, int32_t* row_src_token, int32_t* slot_row,
+                              int32_t* chunk_counts, int32_t* chunk_base, cudaStream_t s);
+moe_status launch_dispatch_rows(int T, int H, int k, const uint16_t* x, const int32_t* slot_row,
+                                uint16_t* x_perm, cudaStream_t s);
+moe_status launch_gather_rows(int H, const uint16_t* x, const int32_t* row_src_token,
+                              const int32_t* offsets, int e_begin, int e_end, uint16_t* x_perm,
+                              int max_rows, cudaStream_t s);
+moe_status launch_combine(int T, int H, int k, const uint16_t* y_perm, const int32_t* slot_row,
+                          const float* w, const uint16_t* shared, void* out, int out_fp32,
+                          cudaStream_t s);
+
+moe_status launch_fill_range(int32_t* offsets, int n, cudaStream_t s);
+moe_status launch_sum_counts(const int32_t* counts, int n_chunks, int E, int32_t* out,
+                             cudaStream_t s);
+
+// Grouped expert GEMM on tcgen05. Experts [e_begin, e_end) of `offsets`.
+moe_status launch_expert_ffn(int rows, int H, int I, int n_experts, int e_begin, int e_end,
+                             const uint16_t* x_perm, const int32_t* offsets, const uint16_t* W13,
+                             const uint16_t* W2, uint16_t* h, uint16_t* y_perm, int rows_hint,
+                             cudaStream_t s);
+
+// ----------------------------------------------------------------------------
+// device helpers
+// ----------------------------------------------------------------------------
+
+__device__ __forceinline__ float bf16_bits_to_float(uint16_t b) {
+  return __uint_as_float(static_cast<uint32_t>(b) << 16);
+}
+
+__device__ __forceinline__ uint16_t float_to_bf16_bits(float f) {
+  __nv_bfloat16 h = __float2bfloat16_rn(f);
+  return *reinterpret_cast<uint16_t*>(&h);
+}
+
+__device__ __forceinline__ uint64_t global_timer_ns() {
+  uint64_t t;
+  asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+  return t;
+}
+
+}  // namespace moe

@@ -1,0 +1,536 @@
+// Grouped expert GEMMs on the 5th-generation tensor cores (tcgen05 + TMEM),
+// operands staged by TMA: the expert compute of the paper's MoE workload
+// (GEMM1 up/gate 7168 x 4096 + SwiGLU + GEMM2 down 2048 x 7168, Appendix
+// "Workload Details"), one launch per GEMM over every expert.
+//
+// Orientation ("swap AB"): the MMA's M side is 128 rows of an expert's weight
+// matrix, its N side is up to NMAX packed token rows of that expert. So an
+// expert with only a few tokens (decode) wastes no tensor work, and the weight
+// tile -- the bytes that bound the layer -- is streamed exactly once per
+// (expert, 128-feature block, token tile).
+//   D[f, n] = sum_k W[f, k] * X[n, k]      (both operands K-major, bf16)
+// D lives in TMEM: lane = output feature, column = token.
+//
+// Work unit = (expert e, feature block fb, token tile nt). The units of every
+// expert are enumerated on the device from the row offsets, so a launch needs
+// no host-side knowledge of the routing. A persistent grid (one CTA per SM)
+// walks the units round-robin. Warp roles:
+//   warp 0     TMA producer: weight tile(s) 128 x 64 and token rows 16 x 64
+//              per stage into a STAGES-deep ring (128-byte swizzle);
+//   warp 1     MMA issuer (one thread): 4 x tcgen05.mma (K = 16 each) per stage,
+//              tcgen05.commit frees the stage, a final commit hands the
+//              accumulator to the epilogue; also owns the TMEM allocation;
+//   warps 2-5  epilogue: tcgen05.ld the accumulator (each warp its 32-lane
+//              quarter), apply SwiGLU (GEMM1) or nothing (GEMM2), store bf16.
+// For SwiGLU the gate and up tiles of the same 128 features are two MMAs into
+// two TMEM column ranges, so one thread holds both g and u of its feature.
+//
+// Every mbarrier wait is bounded (%globaltimer): on expiry the kernel latches
+// MOE_ERR_TIMEOUT, tells the other roles to stop, waits (bounded) for its own
+// copies and MMAs in flight, frees TMEM and returns.
+#include <cudaTypedefs.h>
+
+#include "common.cuh"
+
+namespace moe {
+namespace {
+
+constexpr int BM = 128;           // weight rows per tile (MMA M)
+constexpr int BK = 64;            // bf16 per stage along K: one 128-byte swizzle row
+constexpr int UMMA_K = 16;        // K of one tcgen05.mma kind::f16
+constexpr int B_BOX = 16;         // token rows per TMA box
+constexpr int NUM_THREADS = 192;  // 6 warps
+constexpr uint64_t WAIT_LIMIT_NS = 2000000000ull;
+
+constexpr int pow2ceil(int v) {
+  int p = 32;
+  while (p < v) p <<= 1;
+  return p;
+}
+
+template <bool SWIGLU, int NMAX>
+struct Tile {
+  static constexpr int NA = SWIGLU ? 2 : 1;
+  static constexpr int A_BYTES = BM * BK * 2;  // 16 KiB
+  static constexpr int B_BYTES = NMAX * BK * 2;
+  static constexpr int STAGE_BYTES = NA * A_BYTES + B_BYTES;
+  static constexpr int STAGES_RAW = (200 * 1024) / STAGE_BYTES;
+  static constexpr int STAGES = STAGES_RAW > 8 ? 8 : STAGES_RAW;
+  static constexpr int TMEM_COLS = pow2ceil(NA * NMAX);
+  static_assert(STAGES >= 2, "pipeline too shallow");
+  static_assert(NMAX % 16 == 0 && NMAX >= 16 && NMAX <= 256, "MMA N range for M = 128");
+};
+
+struct Ctrl {
+  uint64_t full[8];
+  uint64_t empty[8];
+  uint64_t acc_full;
+  uint64_t acc_empty;
+  uint64_t drain;
+  uint32_t tmem_base;
+  int abort_flag;
+};
+
+// ------------------------------------------------------------------ PTX wrappers
+
+__device__ __forceinline__ uint32_t smem_u32(const void* p) {
+  return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+
+__device__ __forceinline__ void mbar_init(uint32_t bar, uint32_t count) {
+  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(bar), "r"(count) : "memory");
+}
+
+__device__ __forceinline__ void mbar_arrive_expect_tx(uint32_t bar, uint32_t bytes) {
+  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"(bytes)
+               : "memory");
+}
+
+__device__ __forceinline__ void mbar_arrive(uint32_t bar) {
+  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(bar) : "memory");
+}
+
+__device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(ok)
+      : "r"(bar), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+
+// Wait for the phase of `bar` with the given parity; false on abort or timeout.
+__device__ __noinline__ bool wait_bounded(uint32_t bar, uint32_t parity, volatile int* abort_flag,
+                                          int* err) {
+  if (mbar_try_wait(bar, parity)) return true;
+  const uint64_t t0 = global_timer_ns();
+  while (true) {
+    if (mbar_try_wait(bar, parity)) return true;
+    if (*abort_flag) return false;
+    if (global_timer_ns() - t0 > WAIT_LIMIT_NS) {
+      *abort_flag = 1;
+      atomicExch(err, (int)MOE_ERR_TIMEOUT);
+      return false;
+    }
+  }
+}
+
+__device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap* map, int x, int y,
+                                            uint32_t bar) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes"
+      " [%0], [%1, {%2, %3}], [%4];" ::"r"(dst),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(bar)
+      : "memory");
+}
+
+__device__ __forceinline__ void tma_prefetch_map(const CUtensorMap* map) {
+  asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(map)) : "memory");
+}
+
+__device__ __forceinline__ void tc_fence_before() {
+  asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+}
+__device__ __forceinline__ void tc_fence_after() {
+  asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+}
+
+// Shared-memory matrix descriptor: K-major operand, 128-byte swizzle, rows of
+// 128 bytes, 8-row swizzle atoms 1024 bytes apart (stride byte offset), the
+// leading byte offset unused, descriptor version 1, base offset 0 (atoms are
+// 1024-byte aligned). Advancing K by 16 bf16 adds 32 bytes to the start.
+__device__ __forceinline__ uint64_t sdesc(uint32_t saddr) {
+  return (uint64_t)((saddr & 0x3FFFFu) >> 4) | ((uint64_t)(1024 >> 4) << 32) | (1ull << 46) |
+         (2ull << 61);
+}
+
+// Instruction descriptor, kind::f16: fp32 accumulator (bits 4-5 = 1), A and B
+// bf16 (bits 7-9, 10-12 = 1), both K-major (bits 15, 16 = 0), N >> 3 at bit 17,
+// M >> 4 at bit 24.
+__device__ __forceinline__ uint32_t idesc_bf16(int n) {
+  return (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(n >> 3) << 17) |
+         ((uint32_t)(BM >> 4) << 24);
+}
+
+__device__ __forceinline__ void mma_bf16(uint32_t d_tmem, uint64_t a, uint64_t b, uint32_t idesc,
+                                         uint32_t accumulate) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "setp.ne.b32 p, %4, 0;\n\t"
+      "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
+      "l"(a), "l"(b), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
+
+__device__ __forceinline__ void mma_commit(uint32_t bar) {
+  asm volatile(
+      "tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(bar)
+      : "memory");
+}
+
+__device__ __forceinline__ void tmem_ld16(uint32_t taddr, uint32_t (&r)[16]) {
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x16.b32 "
+      "{%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, [%16];"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
+        "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]),
+        "=r"(r[14]), "=r"(r[15])
+      : "r"(taddr));
+}
+
+__device__ __forceinline__ void tmem_wait_ld() {
+  asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+}
+
+// ------------------------------------------------------------------ schedule
+
+struct Unit {
+  int e;     // expert, relative to e_begin
+  int fb;    // 128-feature block
+  int row0;  // first packed row of the token tile
+  int m;     // valid token rows in the tile (1..NMAX)
+};
+
+template <int NMAX>
+__device__ __forceinline__ Unit decode_unit(int u, const int* tile_off, const int* row_off,
+                                            int n_exp, int n_fb) {
+  int lo = 0, hi = n_exp - 1;
+  while (lo < hi) {  // largest e with tile_off[e] * n_fb <= u: an expert with tiles
+    const int mid = (lo + hi + 1) >> 1;
+    if (tile_off[mid] * n_fb <= u) lo = mid;
+    else hi = mid - 1;
+  }
+  Unit U;
+  U.e = lo;
+  const int nt_e = tile_off[lo + 1] - tile_off[lo];
+  const int local = u - tile_off[lo] * n_fb;
+  U.fb = local / nt_e;
+  const int nt = local - U.fb * nt_e;
+  const int cnt = row_off[lo + 1] - row_off[lo];
+  U.row0 = row_off[lo] + nt * NMAX;
+  U.m = min(NMAX, cnt - nt * NMAX);
+  return U;
+}
+
+// ------------------------------------------------------------------ kernel
+
+template <bool SWIGLU, int NMAX>
+__global__ void __launch_bounds__(NUM_THREADS, 1)
+    grouped_gemm_kernel(const __grid_constant__ CUtensorMap tmA,
+                        const __grid_constant__ CUtensorMap tmB,
+                        const int32_t* __restrict__ offsets, int rows, int e_begin, int n_exp,
+                        int K,
+                        int n_fb, int w_rows_per_expert, int up_row_offset,
+                        uint16_t* __restrict__ out, int out_ld, int* __restrict__ err) {
+  using TL = Tile<SWIGLU, NMAX>;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                             ~static_cast<uintptr_t>(1023));
+  Ctrl* ctrl = reinterpret_cast<Ctrl*>(smem + TL::STAGES * TL::STAGE_BYTES);
+  int* tile_off = reinterpret_cast<int*>(ctrl + 1);
+  int* row_off = tile_off + n_exp + 1;
+  volatile int* abort_flag = &ctrl->abort_flag;
+
+  const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < TL::STAGES; ++s) {
+      mbar_init(smem_u32(&ctrl->full[s]), 1);
+      mbar_init(smem_u32(&ctrl->empty[s]), 1);
+    }
+    mbar_init(smem_u32(&ctrl->acc_full), 1);
+    mbar_init(smem_u32(&ctrl->acc_empty), 4);
+    mbar_init(smem_u32(&ctrl->drain), 1);
+    ctrl->abort_flag = 0;
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+  }
+  if (warp == 1) {
+    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
+                     smem_u32(&ctrl->tmem_base)),
+                 "r"(TL::TMEM_COLS)
+                 : "memory");
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+  }
+  if (warp == 2) {
+    // Per-expert token tiles and their prefix, from the device row offsets.
+    // Offsets are clamped into [0, rows] and made non-decreasing, so no tile can
+    // reach outside the caller's buffers; a clamp latches MOE_ERR_DEVICE_CHECK.
+    const int per = (n_exp + 31) / 32;
+    const int a = min(n_exp, lane * per), b = min(n_exp, a + per);
+    auto clamped = [&](int i) {
+      const int v = offsets[e_begin + i];
+      const int c = min(max(v, 0), rows);
+      if (c != v) atomicExch(err, (int)MOE_ERR_DEVICE_CHECK);
+      return c;
+    };
+    int s = 0;
+    for (int i = a; i < b; ++i) {
+      const int r0 = clamped(i), r1 = max(clamped(i + 1), r0);
+      if (r1 != clamped(i + 1)) atomicExch(err, (int)MOE_ERR_DEVICE_CHECK);
+      row_off[i] = r0;
+      s += (r1 - r0 + NMAX - 1) / NMAX;
+    }
+    int incl = s;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const int v = __shfl_up_sync(0xffffffffu, incl, o);
+      if (lane >= o) incl += v;
+    }
+    int run = incl - s;
+    for (int i = a; i < b; ++i) {
+      tile_off[i] = run;
+      run += (max(clamped(i + 1), row_off[i]) - row_off[i] + NMAX - 1) / NMAX;
+    }
+    if (lane == 31) {
+      tile_off[n_exp] = incl;
+      row_off[n_exp] = clamped(n_exp);
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem_base = ctrl->tmem_base;
+  const int total_units = tile_off[n_exp] * n_fb;
+  const int kblocks = K / BK;
+
+  if (warp == 0) {
+    if (lane == 0) {
+      // ---------------------------------------------------------------- producer
+      tma_prefetch_map(&tmA);
+      tma_prefetch_map(&tmB);
+      int stage = 0;
+      uint32_t phase = 0;
+      long fills = 0;
+      bool ok = true;
+      for (int u = blockIdx.x; u < total_units && ok; u += gridDim.x) {
+        const Unit U = decode_unit<NMAX>(u, tile_off, row_off, n_exp, n_fb);
+        const int n_pad = (U.m + 15) & ~15;
+        const int wrow = (e_begin + U.e) * w_rows_per_expert + U.fb * BM;
+        const uint32_t bytes = TL::NA * TL::A_BYTES + n_pad * BK * 2;
+        for (int kb = 0; kb < kblocks; ++kb) {
+          const uint32_t full = smem_u32(&ctrl->full[stage]);
+          if (!wait_bounded(smem_u32(&ctrl->empty[stage]), phase ^ 1, abort_flag, err)) {
+            ok = false;
+            break;
+          }
+          mbar_arrive_expect_tx(full, bytes);
+          const uint32_t sa = smem_u32(smem + stage * TL::STAGE_BYTES);
+          tma_load_2d(sa, &tmA, kb * BK, wrow, full);
+          if (SWIGLU) tma_load_2d(sa + TL::A_BYTES, &tmA, kb * BK, wrow + up_row_offset, full);
+          const uint32_t sb = sa + TL::NA * TL::A_BYTES;
+          for (int i = 0; i < n_pad / B_BOX; ++i)
+            tma_load_2d(sb + i * (B_BOX * BK * 2), &tmB, kb * BK, U.row0 + i * B_BOX, full);
+          ++fills;
+          if (++stage == TL::STAGES) {
+            stage = 0;
+            phase ^= 1;
+          }
+        }
+      }
+      if (!ok) {
+        // let the copies already issued land before the CTA can exit
+        for (int s = 0; s < TL::STAGES; ++s) {
+          if (fills <= s) continue;
+          const long f = s + ((fills - 1 - s) / TL::STAGES) * TL::STAGES;  // last fill of stage s
+          const uint32_t par = (uint32_t)((f / TL::STAGES) & 1);
+          const uint64_t t0 = global_timer_ns();
+          while (!mbar_try_wait(smem_u32(&ctrl->full[s]), par) &&
+                 global_timer_ns() - t0 < WAIT_LIMIT_NS) {
+          }
+        }
+      }
+    }
+  } else if (warp == 1) {
+    if (lane == 0) {
+      // ---------------------------------------------------------------- MMA issuer
+      int stage = 0;
+      uint32_t phase = 0, acc_phase = 0;
+      bool ok = true, issued = false;
+      for (int u = blockIdx.x; u < total_units && ok; u += gridDim.x) {
+        const Unit U = decode_unit<NMAX>(u, tile_off, row_off, n_exp, n_fb);
+        const int n_pad = (U.m + 15) & ~15;
+        const uint32_t idesc = idesc_bf16(n_pad);
+        if (!wait_bounded(smem_u32(&ctrl->acc_empty), acc_phase ^ 1, abort_flag, err)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        for (int kb = 0; kb < kblocks; ++kb) {
+          if (!wait_bounded(smem_u32(&ctrl->full[stage]), phase, abort_flag, err)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const uint32_t sa = smem_u32(smem + stage * TL::STAGE_BYTES);
+          const uint32_t sb = sa + TL::NA * TL::A_BYTES;
+#pragma unroll
+          for (int k = 0; k < BK / UMMA_K; ++k) {
+            const uint32_t acc = (kb > 0 || k > 0) ? 1u : 0u;
+            const uint64_t bdesc = sdesc(sb + k * UMMA_K * 2);
+            mma_bf16(tmem_base, sdesc(sa + k * UMMA_K * 2), bdesc, idesc, acc);
+            if (SWIGLU)
+              mma_bf16(tmem_base + NMAX, sdesc(sa + TL::A_BYTES + k * UMMA_K * 2), bdesc, idesc,
+                       acc);
+          }
+          issued = true;
+          mma_commit(smem_u32(&ctrl->empty[stage]));
+          if (++stage == TL::STAGES) {
+            stage = 0;
+            phase ^= 1;
+          }
+        }
+        if (!ok) break;
+        mma_commit(smem_u32(&ctrl->acc_full));
+        acc_phase ^= 1;
+      }
+      if (!ok && issued) {
+        // wait (bounded) for the MMAs already issued before TMEM is freed
+        mma_commit(smem_u32(&ctrl->drain));
+        const uint64_t t0 = global_timer_ns();
+        while (!mbar_try_wait(smem_u32(&ctrl->drain), 0) &&
+               global_timer_ns() - t0 < WAIT_LIMIT_NS) {
+        }
+      }
+    }
+  } else {
+    // ------------------------------------------------------------------ epilogue
+    const int q = warp & 3;  // TMEM lane quarter this warp may access
+    const uint32_t tq = tmem_base + ((uint32_t)(q * 32) << 16);
+    uint32_t acc_phase = 0;
+    for (int u = blockIdx.x; u < total_units; u += gridDim.x) {
+      const Unit U = decode_unit<NMAX>(u, tile_off, row_off, n_exp, n_fb);
+      if (!wait_bounded(smem_u32(&ctrl->acc_full), acc_phase, abort_flag, err)) break;
+      tc_fence_after();
+      const int f = U.fb * BM + q * 32 + lane;
+      uint16_t* dst = out + (size_t)U.row0 * out_ld + f;
+      for (int c0 = 0; c0 < U.m; c0 += 16) {
+        uint32_t g[16];
+        tmem_ld16(tq + c0, g);
+        if (SWIGLU) {
+          uint32_t v[16];
+          tmem_ld16(tq + NMAX + c0, v);
+          tmem_wait_ld();
+#pragma unroll
+          for (int i = 0; i < 16; ++i) {
+            if (c0 + i < U.m) {
+              const float gv = __uint_as_float(g[i]);
+              const float uv = __uint_as_float(v[i]);
+              const float hv = gv / (1.0f + expf(-gv)) * uv;
+              dst[(size_t)(c0 + i) * out_ld] = float_to_bf16_bits(hv);
+            }
+          }
+        } else {
+          tmem_wait_ld();
+#pragma unroll
+          for (int i = 0; i < 16; ++i) {
+            if (c0 + i < U.m) dst[(size_t)(c0 + i) * out_ld] = float_to_bf16_bits(__uint_as_float(g[i]));
+          }
+        }
+      }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(smem_u32(&ctrl->acc_empty));
+      acc_phase ^= 1;
+    }
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem_base),
+                 "r"(TL::TMEM_COLS)
+                 : "memory");
+  }
+}
+
+// ------------------------------------------------------------------ host side
+
+PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
+  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+  if (!fn) {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault,
+                                         &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
+  }
+  return fn;
+}
+
+// 2-D bf16 row-major tensor [outer, inner] with a (box_inner x box_outer) box, 128-byte swizzle.
+bool make_map(CUtensorMap* m, const void* ptr, uint64_t inner, uint64_t outer, uint32_t box_inner,
+              uint32_t box_outer) {
+  auto fn = encode_fn();
+  if (!fn) return false;
+  cuuint64_t dims[2] = {inner, outer};
+  cuuint64_t strides[1] = {inner * 2};
+  cuuint32_t box[2] = {box_inner, box_outer};
+  cuuint32_t estr[2] = {1, 1};
+  return fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(ptr), dims, strides, box,
+            estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+            CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+template <bool SWIGLU, int NMAX>
+size_t gemm_smem_bytes(int n_exp) {
+  using TL = Tile<SWIGLU, NMAX>;
+  return 1024 + (size_t)TL::STAGES * TL::STAGE_BYTES + sizeof(Ctrl) + 2 * sizeof(int) * (n_exp + 1);
+}
+
+template <bool SWIGLU, int NMAX>
+moe_status launch_gemm(const CUtensorMap& A, const CUtensorMap& B, const int32_t* offsets,
+                       int rows, int e_begin, int n_exp, int K, int n_fb, int w_rows, int up_off,
+                       uint16_t* out, int out_ld, cudaStream_t s) {
+  const size_t smem = gemm_smem_bytes<SWIGLU, NMAX>(n_exp);
+  if (smem > 227 * 1024) return MOE_ERR_UNSUPPORTED;
+  if (cudaFuncSetAttribute(grouped_gemm_kernel<SWIGLU, NMAX>,
+                           cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) != cudaSuccess)
+    return MOE_ERR_CUDA;
+  grouped_gemm_kernel<SWIGLU, NMAX><<<num_sms(), NUM_THREADS, smem, s>>>(
+      A, B, offsets, rows, e_begin, n_exp, K, n_fb, w_rows, up_off, out, out_ld,
+      device_error_word());
+  note_launch();
+  return launch_status();
+}
+
+template <int NMAX>
+moe_status run_ffn(int rows, int H, int I, int n_experts, int e_begin, int e_end,
+                   const uint16_t* x_perm, const int32_t* offsets, const uint16_t* W13,
+                   const uint16_t* W2, uint16_t* h, uint16_t* y_perm, cudaStream_t s) {
+  CUtensorMap a1, b1, a2, b2;
+  if (!make_map(&a1, W13, H, (uint64_t)n_experts * 2 * I, BK, BM) ||
+      !make_map(&b1, x_perm, H, rows, BK, B_BOX) ||
+      !make_map(&a2, W2, I, (uint64_t)n_experts * H, BK, BM) ||
+      !make_map(&b2, h, I, rows, BK, B_BOX))
+    return MOE_ERR_CUDA;
+  const int n_exp = e_end - e_begin;
+  moe_status st = launch_gemm<true, NMAX>(a1, b1, offsets, rows, e_begin, n_exp, H, I / BM, 2 * I,
+                                          I, h, I, s);
+  if (st != MOE_OK) return st;
+  return launch_gemm<false, NMAX>(a2, b2, offsets, rows, e_begin, n_exp, I, H / BM, H, 0, y_perm,
+                                  H, s);
+}
+
+}  // namespace
+
+moe_status launch_expert_ffn(int rows, int H, int I, int n_experts, int e_begin, int e_end,
+                             const uint16_t* x_perm, const int32_t* offsets, const uint16_t* W13,
+                             const uint16_t* W2, uint16_t* h, uint16_t* y_perm, int rows_hint,
+                             cudaStream_t s) {
+  if (rows == 0 || e_end <= e_begin) return MOE_OK;
+  const int n_exp = e_end - e_begin;
+  // Few rows per expert (decode): small token tiles leave room for a deeper pipeline.
+  if ((long)rows_hint <= 24L * n_exp)
+    return run_ffn<32>(rows, H, I, n_experts, e_begin, e_end, x_perm, offsets, W13, W2, h, y_perm,
+                       s);
+  return run_ffn<256>(rows, H, I, n_experts, e_begin, e_end, x_perm, offsets, W13, W2, h, y_perm,
+                      s);
+}
+
+}  // namespace moe

@@ -1,0 +1,486 @@
+// C ABI of the MoE layer forward: host-side validation, workspace layout,
+// entry points and the stage orchestration (sequential or two-stream
+// pipelined), in the stage order of the paper's MoE pipeline (host MoE
+// listing, Appendix "Static Analysis Example"; two-stream dispatch hiding,
+// Section 4.3).
+#include <atomic>
+#include <cmath>
+#include <mutex>
+#include <vector>
+
+#include "common.cuh"
+
+// The device error word: latched by kernels whose bounded waits expire.
+__device__ int g_moe_device_error = 0;
+
+namespace moe {
+namespace {
+
+constexpr int MAX_DEVICES = 64;
+std::atomic<uint64_t> g_launches{0};
+std::mutex g_mu;
+int* g_err_addr[MAX_DEVICES] = {};
+int g_sms[MAX_DEVICES] = {};
+
+struct DeviceStreams {
+  cudaStream_t pack = nullptr;
+  std::vector<cudaEvent_t> events;
+};
+DeviceStreams g_streams[MAX_DEVICES];
+
+int current_device() {
+  int d = 0;
+  if (cudaGetDevice(&d) != cudaSuccess || d < 0 || d >= MAX_DEVICES) return 0;
+  return d;
+}
+
+}  // namespace
+
+void note_launch(int n) { g_launches.fetch_add((uint64_t)n, std::memory_order_relaxed); }
+
+int* device_error_word() {
+  const int d = current_device();
+  std::lock_guard<std::mutex> lk(g_mu);
+  if (!g_err_addr[d]) {
+    void* p = nullptr;
+    if (cudaGetSymbolAddress(&p, g_moe_device_error) == cudaSuccess) g_err_addr[d] = (int*)p;
+  }
+  return g_err_addr[d];
+}
+
+int num_sms() {
+  const int d = current_device();
+  if (!g_sms[d]) {
+    int v = 0;
+    cudaDeviceGetAttribute(&v, cudaDevAttrMultiProcessorCount, d);
+    g_sms[d] = v > 0 ? v : 1;
+  }
+  return g_sms[d];
+}
+
+namespace {
+
+// ---------------------------------------------------------------- validation
+
+bool valid_config(const moe_config* c) {
+  if (!c) return false;
+  if (c->T < 0 || c->H < 128 || c->H % 128 || c->H > 65536) return false;
+  if (c->E < 1 || c->E > 1024 || c->k < 1 || c->k > 32 || c->k > c->E) return false;
+  if (c->I < 128 || c->I % 128 || c->I > 65536) return false;
+  if (c->I_shared < 0 || (c->I_shared && (c->I_shared < 128 || c->I_shared % 128 ||
+                                          c->I_shared > 65536)))
+    return false;
+  if (c->n_groups < 1 || c->n_groups > 32 || c->E % c->n_groups) return false;
+  if (c->topk_groups < 1 || c->topk_groups > c->n_groups) return false;
+  if ((long)c->k > (long)c->topk_groups * (c->E / c->n_groups)) return false;
+  if (c->gate != MOE_GATE_SOFTMAX && c->gate != MOE_GATE_SIGMOID) return false;
+  if (c->normalize != 0 && c->normalize != 1) return false;
+  if (!std::isfinite(c->route_scale)) return false;
+  if ((long long)c->T * c->k > (1LL << 30)) return false;
+  return true;
+}
+
+bool valid_exec(const moe_exec* ex, const moe_config* c) {
+  if (!ex) return false;
+  if (ex->overlap != 0 && ex->overlap != 1) return false;
+  if (ex->out_fp32 != 0 && ex->out_fp32 != 1) return false;
+  if (ex->overlap) {
+    if (ex->chunk_axis == 0) {
+      if (ex->chunk_tokens < 1) return false;
+    } else if (ex->chunk_axis == 1) {
+      if (ex->n_expert_chunks < 1 || ex->n_expert_chunks > c->E) return false;
+    } else {
+      return false;
+    }
+  }
+  return true;
+}
+
+// ---------------------------------------------------------------- workspace layout
+
+struct Carver {
+  uint8_t* base;
+  size_t off = 0;
+  explicit Carver(void* b) : base((uint8_t*)b) {}
+  template <class T>
+  T* take(size_t count) {
+    off = align_up(off, 256);
+    T* p = base ? reinterpret_cast<T*>(base + off) : nullptr;
+    off += count * sizeof(T);
+    return p;
+  }
+};
+
+struct Layout {
+  int chunk_T = 0, n_chunks = 1, splits = 1, perm_chunks = 0;
+  float* logits;
+  int32_t* idx;
+  float* w;
+  int32_t* counts;   // [n_chunks][E]
+  int32_t* offsets;  // [n_chunks][E+1]
+  int32_t* rst;      // [T*k]
+  int32_t* slot_row; // [T*k]
+  int32_t* perm_counts;
+  int32_t* perm_base;
+  float* partials;
+  uint16_t* x_perm;  // [T*k, H]
+  uint16_t* h;       // [T*k, I]
+  uint16_t* y_perm;  // [T*k, H]
+  int32_t* sh_off;   // [2]
+  uint16_t* sh_h;    // [T, I_s]
+  uint16_t* sh_y;    // [T, H]
+  size_t bytes = 0;
+};
+
+Layout carve(const moe_config& c, const moe_exec& ex, void* ws) {
+  Layout L;
+  const size_t T = c.T, E = c.E, k = c.k;
+  L.chunk_T = c.T;
+  if (ex.overlap && ex.chunk_axis == 0) L.chunk_T = c.T < ex.chunk_tokens ? c.T : ex.chunk_tokens;
+  if (L.chunk_T < 1) L.chunk_T = 1;
+  L.n_chunks = (ex.overlap && ex.chunk_axis == 0) ? (c.T + L.chunk_T - 1) / L.chunk_T : 1;
+  if (L.n_chunks < 1) L.n_chunks = 1;
+  moe_config cc = c;
+  cc.T = L.chunk_T;
+  L.splits = router_splits(cc);
+  L.perm_chunks = perm_num_chunks(L.chunk_T);
+  Carver cv(ws);
+  L.logits = cv.take<float>(T * E);
+  L.idx = cv.take<int32_t>(T * k);
+  L.w = cv.take<float>(T * k);
+  L.counts = cv.take<int32_t>((size_t)L.n_chunks * E);
+  L.offsets = cv.take<int32_t>((size_t)L.n_chunks * (E + 1));
+  L.rst = cv.take<int32_t>(T * k);
+  L.slot_row = cv.take<int32_t>(T * k);
+  L.perm_counts = cv.take<int32_t>((size_t)(L.perm_chunks + 1) * E);
+  L.perm_base = cv.take<int32_t>((size_t)(L.perm_chunks + 1) * E);
+  L.partials = L.splits > 1 ? cv.take<float>((size_t)L.splits * L.chunk_T * E) : nullptr;
+  L.x_perm = cv.take<uint16_t>(T * k * c.H);
+  L.h = cv.take<uint16_t>(T * k * c.I);
+  L.y_perm = cv.take<uint16_t>(T * k * c.H);
+  L.sh_off = cv.take<int32_t>(2);
+  L.sh_h = c.I_shared ? cv.take<uint16_t>(T * c.I_shared) : nullptr;
+  L.sh_y = c.I_shared ? cv.take<uint16_t>(T * c.H) : nullptr;
+  L.bytes = align_up(cv.off, 256);
+  return L;
+}
+
+cudaStream_t pack_stream(int d) {
+  std::lock_guard<std::mutex> lk(g_mu);
+  if (!g_streams[d].pack) {
+    int lo = 0, hi = 0;
+    cudaDeviceGetStreamPriorityRange(&lo, &hi);
+    cudaStreamCreateWithPriority(&g_streams[d].pack, cudaStreamNonBlocking, hi);
+  }
+  return g_streams[d].pack;
+}
+
+bool events(int d, size_t n, std::vector<cudaEvent_t>* out) {
+  std::lock_guard<std::mutex> lk(g_mu);
+  auto& ev = g_streams[d].events;
+  while (ev.size() < n) {
+    cudaEvent_t e;
+    if (cudaEventCreateWithFlags(&e, cudaEventDisableTiming) != cudaSuccess) return false;
+    ev.push_back(e);
+  }
+  out->assign(ev.begin(), ev.begin() + n);
+  return true;
+}
+
+#define MOE_TRY(expr)                 \
+  do {                                \
+    moe_status _st = (expr);          \
+    if (_st != MOE_OK) return _st;    \
+  } while (0)
+
+#define MOE_CUDA(expr)                                  \
+  do {                                                  \
+    if ((expr) != cudaSuccess) return MOE_ERR_CUDA;     \
+  } while (0)
+
+// Router + gate + permutation (+ packing) of tokens [t0, t0+Tc) into chunk slot `ci`.
+moe_status pack_tokens(const moe_config& c, const Layout& L, const moe_weights& w,
+                       const uint16_t* x, int t0, int Tc, int ci, bool pack_rows,
+                       cudaStream_t s) {
+  moe_config cc = c;
+  cc.T = Tc;
+  const size_t tk = (size_t)t0 * c.k;
+  MOE_TRY(launch_router(cc, x + (size_t)t0 * c.H, w.Wr, L.logits + (size_t)t0 * c.E, L.partials,
+                        L.splits, s));
+  MOE_TRY(launch_gate(cc, L.logits + (size_t)t0 * c.E, w.bias, L.idx + tk, L.w + tk, s));
+  MOE_TRY(launch_permutation(cc, L.idx + tk, L.counts + (size_t)ci * c.E,
+                             L.offsets + (size_t)ci * (c.E + 1), L.rst + tk, L.slot_row + tk,
+                             L.perm_counts, L.perm_base, s));
+  if (pack_rows)
+    MOE_TRY(launch_dispatch_rows(Tc, c.H, c.k, x + (size_t)t0 * c.H, L.slot_row + tk,
+                                 L.x_perm + tk * c.H, s));
+  return MOE_OK;
+}
+
+// Routed experts of chunk ci (tokens [t0, t0+Tc)), experts [e0, e1), then nothing else.
+moe_status experts_tokens(const moe_config& c, const Layout& L, const moe_weights& w, int t0,
+                          int Tc, int ci, int e0, int e1, cudaStream_t s) {
+  const size_t tk = (size_t)t0 * c.k;
+  const int rows = Tc * c.k;
+  const long hint = (long)rows * (e1 - e0) / c.E;
+  return launch_expert_ffn(rows, c.H, c.I, c.E, e0, e1, L.x_perm + tk * c.H,
+                           L.offsets + (size_t)ci * (c.E + 1), w.W13, w.W2, L.h + tk * c.I,
+                           L.y_perm + tk * c.H, (int)hint, s);
+}
+
+moe_status shared_expert(const moe_config& c, const Layout& L, const moe_weights& w,
+                         const uint16_t* x, cudaStream_t s) {
+  if (!c.I_shared) return MOE_OK;
+  MOE_TRY(launch_fill_range(L.sh_off, c.T, s));
+  return launch_expert_ffn(c.T, c.H, c.I_shared, 1, 0, 1, x, L.sh_off, w.Ws13, w.Ws2, L.sh_h,
+                           L.sh_y, c.T, s);
+}
+
+moe_status combine_tokens(const moe_config& c, const Layout& L, int t0, int Tc, void* out,
+                          int out_fp32, cudaStream_t s) {
+  const size_t tk = (size_t)t0 * c.k;
+  const size_t ob = out_fp32 ? 4 : 2;
+  return launch_combine(Tc, c.H, c.k, L.y_perm + tk * c.H, L.slot_row + tk, L.w + tk,
+                        L.sh_y ? L.sh_y + (size_t)t0 * c.H : nullptr,
+                        (uint8_t*)out + (size_t)t0 * c.H * ob, out_fp32, s);
+}
+
+}  // namespace
+}  // namespace moe
+
+using namespace moe;
+
+extern "C" {
+
+const char* moe_status_string(moe_status s) {
+  switch (s) {
+    case MOE_OK: return "MOE_OK";
+    case MOE_ERR_INVALID_ARG: return "MOE_ERR_INVALID_ARG";
+    case MOE_ERR_UNSUPPORTED: return "MOE_ERR_UNSUPPORTED";
+    case MOE_ERR_WORKSPACE: return "MOE_ERR_WORKSPACE";
+    case MOE_ERR_CUDA: return "MOE_ERR_CUDA";
+    case MOE_ERR_TIMEOUT: return "MOE_ERR_TIMEOUT";
+    case MOE_ERR_DEVICE_CHECK: return "MOE_ERR_DEVICE_CHECK";
+  }
+  return "MOE_ERR_UNKNOWN";
+}
+
+moe_status moe_validate_config(const moe_config* cfg) {
+  return valid_config(cfg) ? MOE_OK : MOE_ERR_INVALID_ARG;
+}
+
+size_t moe_workspace_size(const moe_config* cfg, const moe_exec* ex) {
+  if (!valid_config(cfg) || !valid_exec(ex, cfg)) return 0;
+  return carve(*cfg, *ex, nullptr).bytes;
+}
+
+size_t moe_router_workspace_size(const moe_config* cfg) {
+  if (!valid_config(cfg)) return 0;
+  const int s = router_splits(*cfg);
+  return s > 1 ? (size_t)s * cfg->T * cfg->E * sizeof(float) : 0;
+}
+
+size_t moe_dispatch_workspace_size(const moe_config* cfg) {
+  if (!valid_config(cfg)) return 0;
+  return 2 * align_up((size_t)(perm_num_chunks(cfg->T) + 1) * cfg->E * sizeof(int32_t), 256);
+}
+
+size_t moe_expert_ffn_workspace_size(int32_t rows, int32_t I) {
+  if (rows < 0 || I < 0) return 0;
+  return (size_t)rows * I * 2;
+}
+
+moe_status moe_router_logits(const moe_config* cfg, const uint16_t* x, const float* Wr,
+                             float* logits, void* ws, size_t ws_bytes, void* stream) {
+  if (!valid_config(cfg)) return MOE_ERR_INVALID_ARG;
+  if (cfg->T == 0) return MOE_OK;
+  if (!x || !Wr || !logits || !aligned16(x) || !aligned16(Wr) || !aligned4(logits))
+    return MOE_ERR_INVALID_ARG;
+  const size_t need = moe_router_workspace_size(cfg);
+  float* part = nullptr;
+  int splits = 1;
+  if (ws && need) {
+    if (ws_bytes < need || !aligned4(ws)) return MOE_ERR_WORKSPACE;
+    part = (float*)ws;
+    splits = router_splits(*cfg);
+  }
+  return launch_router(*cfg, x, Wr, logits, part, splits, (cudaStream_t)stream);
+}
+
+moe_status moe_gate_topk(const moe_config* cfg, const float* logits, const float* bias,
+                         int32_t* topk_idx, float* topk_w, void* stream) {
+  if (!valid_config(cfg)) return MOE_ERR_INVALID_ARG;
+  if (cfg->T == 0) return MOE_OK;
+  if (!logits || !topk_idx || !topk_w || !aligned4(logits) || !aligned4(topk_idx) ||
+      !aligned4(topk_w) || (bias && !aligned4(bias)))
+    return MOE_ERR_INVALID_ARG;
+  return launch_gate(*cfg, logits, bias, topk_idx, topk_w, (cudaStream_t)stream);
+}
+
+moe_status moe_dispatch(const moe_config* cfg, const uint16_t* x, const int32_t* topk_idx,
+                        int32_t* counts, int32_t* offsets, int32_t* row_src_token,
+                        int32_t* slot_row, uint16_t* x_perm, void* ws, size_t ws_bytes,
+                        void* stream) {
+  if (!valid_config(cfg)) return MOE_ERR_INVALID_ARG;
+  if (!counts || !offsets || !aligned4(counts) || !aligned4(offsets)) return MOE_ERR_INVALID_ARG;
+  if (cfg->T > 0 && (!topk_idx || !row_src_token || !slot_row || !aligned4(topk_idx) ||
+                     !aligned4(row_src_token) || !aligned4(slot_row)))
+    return MOE_ERR_INVALID_ARG;
+  if (x_perm && (!x || !aligned16(x) || !aligned16(x_perm))) return MOE_ERR_INVALID_ARG;
+  const size_t need = moe_dispatch_workspace_size(cfg);
+  if (!ws || ws_bytes < need || ((uintptr_t)ws & 255)) return MOE_ERR_WORKSPACE;
+  int32_t* pc = (int32_t*)ws;
+  int32_t* pb = (int32_t*)((uint8_t*)ws + need / 2);
+  cudaStream_t s = (cudaStream_t)stream;
+  MOE_TRY(launch_permutation(*cfg, topk_idx, counts, offsets, row_src_token, slot_row, pc, pb, s));
+  if (x_perm) MOE_TRY(launch_dispatch_rows(cfg->T, cfg->H, cfg->k, x, slot_row, x_perm, s));
+  return MOE_OK;
+}
+
+moe_status moe_expert_ffn(int32_t rows, int32_t H, int32_t I, int32_t n_experts,
+                          const uint16_t* x_perm, const int32_t* offsets, const uint16_t* W13,
+                          const uint16_t* W2, uint16_t* y_perm, void* ws, size_t ws_bytes,
+                          void* stream) {
+  if (rows < 0 || H < 128 || H % 128 || H > 65536 || I < 128 || I % 128 || I > 65536 ||
+      n_experts < 1 || n_experts > 1024)
+    return MOE_ERR_INVALID_ARG;
+  if (rows == 0) return MOE_OK;
+  if (!x_perm || !offsets || !W13 || !W2 || !y_perm || !aligned16(x_perm) || !aligned16(W13) ||
+      !aligned16(W2) || !aligned16(y_perm) || !aligned4(offsets))
+    return MOE_ERR_INVALID_ARG;
+  const size_t need = moe_expert_ffn_workspace_size(rows, I);
+  if (!ws || ws_bytes < need || !aligned16(ws)) return MOE_ERR_WORKSPACE;
+  return launch_expert_ffn(rows, H, I, n_experts, 0, n_experts, x_perm, offsets, W13, W2,
+                           (uint16_t*)ws, y_perm, rows, (cudaStream_t)stream);
+}
+
+moe_status moe_combine(const moe_config* cfg, const uint16_t* y_perm, const int32_t* slot_row,
+                       const float* topk_w, const uint16_t* shared_out, void* out,
+                       int32_t out_fp32, void* stream) {
+  if (!valid_config(cfg) || (out_fp32 != 0 && out_fp32 != 1)) return MOE_ERR_INVALID_ARG;
+  if (cfg->T == 0) return MOE_OK;
+  if (!y_perm || !slot_row || !topk_w || !out || !aligned16(y_perm) || !aligned4(slot_row) ||
+      !aligned4(topk_w) || !aligned16(out) || (shared_out && !aligned16(shared_out)))
+    return MOE_ERR_INVALID_ARG;
+  return launch_combine(cfg->T, cfg->H, cfg->k, y_perm, slot_row, topk_w, shared_out, out,
+                        out_fp32, (cudaStream_t)stream);
+}
+
+moe_status moe_layer_forward(const moe_config* cfg, const moe_exec* ex, const moe_weights* w,
+                             const uint16_t* x, void* out, const moe_aux* aux, void* ws,
+                             size_t ws_bytes, void* stream, void* aux_stream) {
+  if (!valid_config(cfg) || !valid_exec(ex, cfg) || !w) return MOE_ERR_INVALID_ARG;
+  const moe_config& c = *cfg;
+  if (!w->Wr || !w->W13 || !w->W2 || !aligned16(w->Wr) || !aligned16(w->W13) ||
+      !aligned16(w->W2) || (w->bias && !aligned4(w->bias)))
+    return MOE_ERR_INVALID_ARG;
+  if (c.I_shared && (!w->Ws13 || !w->Ws2 || !aligned16(w->Ws13) || !aligned16(w->Ws2)))
+    return MOE_ERR_INVALID_ARG;
+  if (!c.I_shared && (w->Ws13 || w->Ws2)) return MOE_ERR_INVALID_ARG;
+  if (c.T == 0) return MOE_OK;
+  if (!x || !out || !aligned16(x) || !aligned16(out)) return MOE_ERR_INVALID_ARG;
+  if (aux && ((aux->logits && !aligned4(aux->logits)) || (aux->topk_idx && !aligned4(aux->topk_idx)) ||
+              (aux->topk_w && !aligned4(aux->topk_w)) || (aux->counts && !aligned4(aux->counts))))
+    return MOE_ERR_INVALID_ARG;
+  Layout L = carve(c, *ex, nullptr);
+  if (!ws || ws_bytes < L.bytes || ((uintptr_t)ws & 255)) return MOE_ERR_WORKSPACE;
+  L = carve(c, *ex, ws);
+  if (aux && aux->logits) L.logits = aux->logits;
+  if (aux && aux->topk_idx) L.idx = aux->topk_idx;
+  if (aux && aux->topk_w) L.w = aux->topk_w;
+
+  cudaStream_t s = (cudaStream_t)stream;
+  const int dev = current_device();
+
+  if (!ex->overlap) {
+    MOE_TRY(pack_tokens(c, L, *w, x, 0, c.T, 0, true, s));
+    MOE_TRY(experts_tokens(c, L, *w, 0, c.T, 0, 0, c.E, s));
+    MOE_TRY(shared_expert(c, L, *w, x, s));
+    MOE_TRY(combine_tokens(c, L, 0, c.T, out, ex->out_fp32, s));
+    if (aux && aux->counts)
+      MOE_CUDA(cudaMemcpyAsync(aux->counts, L.counts, sizeof(int32_t) * c.E,
+                               cudaMemcpyDeviceToDevice, s));
+    return MOE_OK;
+  }
+
+  cudaStream_t ps = aux_stream ? (cudaStream_t)aux_stream : pack_stream(dev);
+  if (!ps) return MOE_ERR_CUDA;
+  const int n_stage = ex->chunk_axis == 0 ? L.n_chunks : ex->n_expert_chunks;
+  std::vector<cudaEvent_t> ev;
+  if (!events(dev, (size_t)n_stage + 1, &ev)) return MOE_ERR_CUDA;
+  // the pack stream starts after everything already queued on `stream`
+  MOE_CUDA(cudaEventRecord(ev[n_stage], s));
+  MOE_CUDA(cudaStreamWaitEvent(ps, ev[n_stage], 0));
+
+  if (ex->chunk_axis == 0) {
+    // Token chunks: chunk i+1 is routed and packed on the pack stream while
+    // chunk i's experts compute on `stream`.
+    for (int ci = 0; ci < L.n_chunks; ++ci) {
+      const int t0 = ci * L.chunk_T, Tc = c.T - t0 < L.chunk_T ? c.T - t0 : L.chunk_T;
+      MOE_TRY(pack_tokens(c, L, *w, x, t0, Tc, ci, true, ps));
+      MOE_CUDA(cudaEventRecord(ev[ci], ps));
+    }
+    MOE_TRY(shared_expert(c, L, *w, x, s));  // overlaps the first chunk's packing
+    for (int ci = 0; ci < L.n_chunks; ++ci) {
+      const int t0 = ci * L.chunk_T, Tc = c.T - t0 < L.chunk_T ? c.T - t0 : L.chunk_T;
+      MOE_CUDA(cudaStreamWaitEvent(s, ev[ci], 0));
+      MOE_TRY(experts_tokens(c, L, *w, t0, Tc, ci, 0, c.E, s));
+      MOE_TRY(combine_tokens(c, L, t0, Tc, out, ex->out_fp32, s));
+    }
+    if (aux && aux->counts) MOE_TRY(launch_sum_counts(L.counts, L.n_chunks, c.E, aux->counts, s));
+    return MOE_OK;
+  }
+
+  // Expert ranges: route and permute all tokens once, then pack the rows of
+  // expert range i+1 while range i computes; weights are streamed once.
+  MOE_TRY(pack_tokens(c, L, *w, x, 0, c.T, 0, false, ps));
+  const int nr = ex->n_expert_chunks;
+  for (int r = 0; r < nr; ++r) {
+    const int e0 = (int)((long)c.E * r / nr), e1 = (int)((long)c.E * (r + 1) / nr);
+    MOE_TRY(launch_gather_rows(c.H, x, L.rst, L.offsets, e0, e1, L.x_perm, c.T * c.k, ps));
+    MOE_CUDA(cudaEventRecord(ev[r], ps));
+  }
+  MOE_TRY(shared_expert(c, L, *w, x, s));  // overlaps routing on the pack stream
+  for (int r = 0; r < nr; ++r) {
+    const int e0 = (int)((long)c.E * r / nr), e1 = (int)((long)c.E * (r + 1) / nr);
+    MOE_CUDA(cudaStreamWaitEvent(s, ev[r], 0));
+    MOE_TRY(experts_tokens(c, L, *w, 0, c.T, 0, e0, e1, s));
+  }
+  MOE_TRY(combine_tokens(c, L, 0, c.T, out, ex->out_fp32, s));
+  if (aux && aux->counts)
+    MOE_CUDA(cudaMemcpyAsync(aux->counts, L.counts, sizeof(int32_t) * c.E,
+                             cudaMemcpyDeviceToDevice, s));
+  return MOE_OK;
+}
+
+moe_status moe_check_errors(void* stream) {
+  if (cudaStreamSynchronize((cudaStream_t)stream) != cudaSuccess) return MOE_ERR_CUDA;
+  int v = 0;
+  if (cudaMemcpyFromSymbol(&v, g_moe_device_error, sizeof(int)) != cudaSuccess) return MOE_ERR_CUDA;
+  if (v != 0) {
+    const int zero = 0;
+    if (cudaMemcpyToSymbol(g_moe_device_error, &zero, sizeof(int)) != cudaSuccess)
+      return MOE_ERR_CUDA;
+  }
+  if (v == MOE_ERR_TIMEOUT) return MOE_ERR_TIMEOUT;
+  if (v != 0) return MOE_ERR_DEVICE_CHECK;
+  return MOE_OK;
+}
+
+uint64_t moe_launch_count(void) { return g_launches.load(std::memory_order_relaxed); }
+
+void moe_shutdown(void) {
+  std::lock_guard<std::mutex> lk(g_mu);
+  int prev = 0;
+  cudaGetDevice(&prev);
+  for (int d = 0; d < MAX_DEVICES; ++d) {
+    if (!g_streams[d].pack && g_streams[d].events.empty()) continue;
+    cudaSetDevice(d);
+    if (g_streams[d].pack) cudaStreamDestroy(g_streams[d].pack);
+    for (auto e : g_streams[d].events) cudaEventDestroy(e);
+    g_streams[d] = DeviceStreams{};
+  }
+  cudaSetDevice(prev);
+}
+
+}  // extern "C"

@@ -1,0 +1,363 @@
+// Dispatch and combine: the single-GPU form of the paper's two AlltoAll
+// exchanges (host MoE listing, Appendix "Static Analysis Example"; unpadded
+// variable-size per-peer transfers, Appendix "Workload Details").
+//
+// Permutation (stable, deterministic, no global atomics deciding order):
+//   1. perm_hist:    each CTA takes PERM_TOK consecutive tokens (all k slots)
+//                    and counts its entries per expert -> chunk_counts[c][e];
+//   2. perm_scan:    one CTA: per expert, exclusive prefix of chunk counts over
+//                    chunks -> chunk_base[c][e] and counts[e]; then offsets =
+//                    exclusive prefix of counts over experts;
+//   3. perm_scatter: each CTA re-walks its entries in (t, j) order; each warp
+//                    ranks its 32-entry steps with __match_any_sync, so every
+//                    expert's rows come out ordered by (t, j).
+// Row copies move 16-byte vectors: dispatch scatters each token row once to
+// its k packed rows (x read once); combine gathers the k expert rows of a
+// token and reduces them in fp32 in slot order.
+#include "common.cuh"
+
+namespace moe {
+namespace {
+
+constexpr int PERM_WARPS = 8;
+constexpr int PERM_TOK = 128;  // tokens per permutation chunk
+
+__device__ __forceinline__ unsigned lanemask_lt() {
+  unsigned m;
+  asm("mov.u32 %0, %%lanemask_lt;" : "=r"(m));
+  return m;
+}
+
+// Per-warp histogram of the warp's share of a chunk. hist: [PERM_WARPS][E] in smem.
+// Expert id of entry n, or -1 (and a latched error) if it lies outside [0, E).
+__device__ __forceinline__ int entry_expert(const int32_t* __restrict__ idx, long n, long n1, int E,
+                                            int* err) {
+  if (n >= n1) return -1;
+  const int e = idx[n];
+  if (e < 0 || e >= E) {
+    atomicExch(err, (int)MOE_ERR_DEVICE_CHECK);
+    return -1;
+  }
+  return e;
+}
+
+__device__ void warp_histogram(const int32_t* __restrict__ idx, long n0, long n1, int E,
+                               int* hist_w, int* err) {
+  const int lane = threadIdx.x % 32;
+  for (long base = n0; base < n1; base += 32) {
+    const long n = base + lane;
+    const int e = entry_expert(idx, n, n1, E, err);
+    const unsigned peers = __match_any_sync(0xffffffffu, e);
+    const int leader = __ffs(peers) - 1;
+    if (e >= 0 && lane == leader) hist_w[e] += __popc(peers);
+    __syncwarp();
+  }
+}
+
+// Entry range [n0, n1) of warp w within chunk c.
+__device__ __forceinline__ void warp_range(int c, int w, int T, int k, long* n0, long* n1) {
+  const long cb = (long)c * PERM_TOK * k;
+  const long ce = min((long)T * k, cb + (long)PERM_TOK * k);
+  const long per = ((long)PERM_TOK * k + PERM_WARPS - 1) / PERM_WARPS;
+  *n0 = min(ce, cb + w * per);
+  *n1 = min(ce, cb + (w + 1) * per);
+}
+
+__global__ void __launch_bounds__(PERM_WARPS * 32) perm_hist_kernel(
+    const int32_t* __restrict__ idx, int T, int k, int E, int32_t* __restrict__ chunk_counts,
+    int* __restrict__ err) {
+  extern __shared__ int perm_smem[];  // [PERM_WARPS][E]
+  for (int i = threadIdx.x; i < PERM_WARPS * E; i += blockDim.x) perm_smem[i] = 0;
+  __syncthreads();
+  const int w = threadIdx.x / 32;
+  long n0, n1;
+  warp_range(blockIdx.x, w, T, k, &n0, &n1);
+  warp_histogram(idx, n0, n1, E, perm_smem + w * E, err);
+  __syncthreads();
+  for (int e = threadIdx.x; e < E; e += blockDim.x) {
+    int s = 0;
+    for (int q = 0; q < PERM_WARPS; ++q) s += perm_smem[q * E + e];
+    chunk_counts[(size_t)blockIdx.x * E + e] = s;
+  }
+}
+
+// One CTA of 1024 threads. Warp q handles experts q, q+32, ...; its lanes split
+// the chunks into contiguous runs and combine them with a warp scan.
+__global__ void __launch_bounds__(1024) perm_scan_kernel(const int32_t* __restrict__ chunk_counts,
+                                                         int n_chunks, int E,
+                                                         int32_t* __restrict__ chunk_base,
+                                                         int32_t* __restrict__ counts,
+                                                         int32_t* __restrict__ offsets) {
+  __shared__ int tot[1024];
+  __shared__ int wsum[32];
+  const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
+  const int per = (n_chunks + 31) / 32;
+  for (int e = warp; e < E; e += 32) {
+    const int c0 = min(n_chunks, lane * per), c1 = min(n_chunks, c0 + per);
+    int s = 0;
+    for (int c = c0; c < c1; ++c) s += chunk_counts[(size_t)c * E + e];
+    int incl = s;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const int v = __shfl_up_sync(0xffffffffu, incl, o);
+      if (lane >= o) incl += v;
+    }
+    int run = incl - s;
+    for (int c = c0; c < c1; ++c) {
+      const int v = chunk_counts[(size_t)c * E + e];
+      chunk_base[(size_t)c * E + e] = run;
+      run += v;
+    }
+    const int total = __shfl_sync(0xffffffffu, incl, 31);
+    if (lane == 0) {
+      tot[e] = total;
+      counts[e] = total;
+    }
+  }
+  __syncthreads();
+  // exclusive scan of tot[0..E) with 1024 threads (E <= 1024)
+  const int i = threadIdx.x;
+  const int v = i < E ? tot[i] : 0;
+  int incl = v;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const int u = __shfl_up_sync(0xffffffffu, incl, o);
+    if (lane >= o) incl += u;
+  }
+  if (lane == 31) wsum[warp] = incl;
+  __syncthreads();
+  if (warp == 0) {
+    int s = wsum[lane];
+    int inc = s;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const int u = __shfl_up_sync(0xffffffffu, inc, o);
+      if (lane >= o) inc += u;
+    }
+    wsum[lane] = inc - s;
+  }
+  __syncthreads();
+  const int excl = incl - v + wsum[warp];
+  if (i < E) offsets[i] = excl;
+  if (i == E - 1) offsets[E] = excl + v;
+}
+
+__global__ void __launch_bounds__(PERM_WARPS * 32) perm_scatter_kernel(
+    const int32_t* __restrict__ idx, int T, int k, int E, const int32_t* __restrict__ offsets,
+    const int32_t* __restrict__ chunk_base, int32_t* __restrict__ row_src_token,
+    int32_t* __restrict__ slot_row, int* __restrict__ err) {
+  extern __shared__ int perm_smem[];  // [PERM_WARPS][E]: histogram, then cursors
+  for (int i = threadIdx.x; i < PERM_WARPS * E; i += blockDim.x) perm_smem[i] = 0;
+  __syncthreads();
+  const int w = threadIdx.x / 32, lane = threadIdx.x % 32;
+  long n0, n1;
+  warp_range(blockIdx.x, w, T, k, &n0, &n1);
+  int* hist_w = perm_smem + w * E;
+  warp_histogram(idx, n0, n1, E, hist_w, err);
+  __syncthreads();
+  for (int e = threadIdx.x; e < E; e += blockDim.x) {
+    int run = offsets[e] + chunk_base[(size_t)blockIdx.x * E + e];
+    for (int q = 0; q < PERM_WARPS; ++q) {
+      const int v = perm_smem[q * E + e];
+      perm_smem[q * E + e] = run;
+      run += v;
+    }
+  }
+  __syncthreads();
+  const unsigned lt = lanemask_lt();
+  for (long base = n0; base < n1; base += 32) {
+    const long n = base + lane;
+    const int e = entry_expert(idx, n, n1, E, err);
+    const unsigned peers = __match_any_sync(0xffffffffu, e);
+    int row = 0;
+    if (e >= 0) row = hist_w[e] + __popc(peers & lt);
+    __syncwarp();
+    if (e >= 0 && lane == __ffs(peers) - 1) hist_w[e] += __popc(peers);
+    __syncwarp();
+    if (e >= 0) {
+      row_src_token[row] = (int32_t)(n / k);
+      slot_row[n] = row;
+    }
+  }
+}
+
+// x_perm[slot_row[t*k + j]] = x[t] for every token t and slot j (16-byte vectors).
+__global__ void dispatch_rows_kernel(const uint4* __restrict__ x, int T, int vpr, int k,
+                                     const int32_t* __restrict__ slot_row,
+                                     uint4* __restrict__ x_perm) {
+  const size_t total = (size_t)T * vpr;
+  for (size_t i = blockIdx.x * (size_t)blockDim.x + threadIdx.x; i < total;
+       i += (size_t)gridDim.x * blockDim.x) {
+    const size_t t = i / vpr, v = i % vpr;
+    const uint4 val = x[i];
+    for (int j = 0; j < k; ++j) {
+      const int r = slot_row[t * k + j];
+      x_perm[(size_t)r * vpr + v] = val;
+    }
+  }
+}
+
+// x_perm[r] = x[row_src_token[r]] for rows of experts [e_begin, e_end).
+__global__ void gather_rows_kernel(const uint4* __restrict__ x, int vpr,
+                                   const int32_t* __restrict__ row_src_token,
+                                   const int32_t* __restrict__ offsets, int e_begin, int e_end,
+                                   uint4* __restrict__ x_perm) {
+  const int r0 = offsets[e_begin], r1 = offsets[e_end];
+  const size_t total = (size_t)(r1 - r0) * vpr;
+  for (size_t i = blockIdx.x * (size_t)blockDim.x + threadIdx.x; i < total;
+       i += (size_t)gridDim.x * blockDim.x) {
+    const size_t r = r0 + i / vpr, v = i % vpr;
+    x_perm[r * vpr + v] = x[(size_t)row_src_token[r] * vpr + v];
+  }
+}
+
+// out[t] = sum_j w[t,j] * y_perm[slot_row[t*k+j]] (+ shared[t]); 8 bf16 per thread-step.
+__global__ void combine_kernel(const uint4* __restrict__ y_perm, int T, int vpr, int k,
+                               const int32_t* __restrict__ slot_row, const float* __restrict__ w,
+                               const uint4* __restrict__ shared, void* __restrict__ out,
+                               int out_fp32, int* __restrict__ err) {
+  const int nrows = T * k;
+  const size_t total = (size_t)T * vpr;
+  for (size_t i = blockIdx.x * (size_t)blockDim.x + threadIdx.x; i < total;
+       i += (size_t)gridDim.x * blockDim.x) {
+    const size_t t = i / vpr, v = i % vpr;
+    float acc[8];
+#pragma unroll
+    for (int q = 0; q < 8; ++q) acc[q] = 0.f;
+    for (int j = 0; j < k; ++j) {
+      const int r = slot_row[t * k + j];
+      if (r < 0 || r >= nrows) {  // not a packed row: skip it and report
+        atomicExch(err, (int)MOE_ERR_DEVICE_CHECK);
+        continue;
+      }
+      const float wj = w[t * k + j];
+      const uint4 yv = y_perm[(size_t)r * vpr + v];
+      const uint16_t* yh = reinterpret_cast<const uint16_t*>(&yv);
+#pragma unroll
+      for (int q = 0; q < 8; ++q) acc[q] = fmaf(wj, bf16_bits_to_float(yh[q]), acc[q]);
+    }
+    if (shared) {
+      const uint4 sv = shared[i];
+      const uint16_t* sh = reinterpret_cast<const uint16_t*>(&sv);
+#pragma unroll
+      for (int q = 0; q < 8; ++q) acc[q] += bf16_bits_to_float(sh[q]);
+    }
+    if (out_fp32) {
+      float4* o = reinterpret_cast<float4*>(out) + i * 2;
+      o[0] = make_float4(acc[0], acc[1], acc[2], acc[3]);
+      o[1] = make_float4(acc[4], acc[5], acc[6], acc[7]);
+    } else {
+      uint4 ov;
+      uint16_t* oh = reinterpret_cast<uint16_t*>(&ov);
+#pragma unroll
+      for (int q = 0; q < 8; ++q) oh[q] = float_to_bf16_bits(acc[q]);
+      reinterpret_cast<uint4*>(out)[i] = ov;
+    }
+  }
+}
+
+// offsets = {0, n}: the one-segment layout of the shared expert.
+__global__ void fill_range_kernel(int32_t* __restrict__ offsets, int n) {
+  if (threadIdx.x == 0) {
+    offsets[0] = 0;
+    offsets[1] = n;
+  }
+}
+
+// out[e] = sum_c counts[c][e] over the chunks of a token-chunked layer.
+__global__ void sum_counts_kernel(const int32_t* __restrict__ counts, int n_chunks, int E,
+                                  int32_t* __restrict__ out) {
+  for (int e = blockIdx.x * blockDim.x + threadIdx.x; e < E; e += gridDim.x * blockDim.x) {
+    int s = 0;
+    for (int c = 0; c < n_chunks; ++c) s += counts[(size_t)c * E + e];
+    out[e] = s;
+  }
+}
+
+int copy_grid(size_t work) {
+  const size_t per = 256;
+  size_t b = (work + per - 1) / per;
+  const size_t cap = (size_t)num_sms() * 8;
+  if (b > cap) b = cap;
+  if (b < 1) b = 1;
+  return (int)b;
+}
+
+}  // namespace
+
+int perm_num_chunks(int T) { return (T + PERM_TOK - 1) / PERM_TOK; }
+
+moe_status launch_permutation(const moe_config& c, const int32_t* idx, int32_t* counts,
+                              int32_t* offsets, int32_t* row_src_token, int32_t* slot_row,
+                              int32_t* chunk_counts, int32_t* chunk_base, cudaStream_t s) {
+  const int nch = perm_num_chunks(c.T);
+  const size_t smem = (size_t)PERM_WARPS * c.E * sizeof(int);
+  if (smem > 48 * 1024) {
+    cudaFuncSetAttribute(perm_hist_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    cudaFuncSetAttribute(perm_scatter_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                         (int)smem);
+  }
+  if (nch > 0) {
+    perm_hist_kernel<<<nch, PERM_WARPS * 32, smem, s>>>(idx, c.T, c.k, c.E, chunk_counts,
+                                                        device_error_word());
+    note_launch();
+  }
+  perm_scan_kernel<<<1, 1024, 0, s>>>(chunk_counts, nch, c.E, chunk_base, counts, offsets);
+  note_launch();
+  if (nch > 0) {
+    perm_scatter_kernel<<<nch, PERM_WARPS * 32, smem, s>>>(idx, c.T, c.k, c.E, offsets, chunk_base,
+                                                           row_src_token, slot_row,
+                                                           device_error_word());
+    note_launch();
+  }
+  return launch_status();
+}
+
+moe_status launch_dispatch_rows(int T, int H, int k, const uint16_t* x, const int32_t* slot_row,
+                                uint16_t* x_perm, cudaStream_t s) {
+  if (T == 0) return MOE_OK;
+  const int vpr = H / 8;
+  dispatch_rows_kernel<<<copy_grid((size_t)T * vpr), 256, 0, s>>>(
+      reinterpret_cast<const uint4*>(x), T, vpr, k, slot_row, reinterpret_cast<uint4*>(x_perm));
+  note_launch();
+  return launch_status();
+}
+
+moe_status launch_gather_rows(int H, const uint16_t* x, const int32_t* row_src_token,
+                              const int32_t* offsets, int e_begin, int e_end, uint16_t* x_perm,
+                              int max_rows, cudaStream_t s) {
+  if (max_rows == 0 || e_end <= e_begin) return MOE_OK;
+  const int vpr = H / 8;
+  gather_rows_kernel<<<copy_grid((size_t)max_rows * vpr), 256, 0, s>>>(
+      reinterpret_cast<const uint4*>(x), vpr, row_src_token, offsets, e_begin, e_end,
+      reinterpret_cast<uint4*>(x_perm));
+  note_launch();
+  return launch_status();
+}
+
+moe_status launch_combine(int T, int H, int k, const uint16_t* y_perm, const int32_t* slot_row,
+                          const float* w, const uint16_t* shared, void* out, int out_fp32,
+                          cudaStream_t s) {
+  if (T == 0) return MOE_OK;
+  const int vpr = H / 8;
+  combine_kernel<<<copy_grid((size_t)T * vpr), 256, 0, s>>>(
+      reinterpret_cast<const uint4*>(y_perm), T, vpr, k, slot_row, w,
+      reinterpret_cast<const uint4*>(shared), out, out_fp32, device_error_word());
+  note_launch();
+  return launch_status();
+}
+
+moe_status launch_fill_range(int32_t* offsets, int n, cudaStream_t s) {
+  fill_range_kernel<<<1, 32, 0, s>>>(offsets, n);
+  note_launch();
+  return launch_status();
+}
+
+moe_status launch_sum_counts(const int32_t* counts, int n_chunks, int E, int32_t* out,
+                             cudaStream_t s) {
+  sum_counts_kernel<<<(E + 255) / 256, 256, 0, s>>>(counts, n_chunks, E, out);
+  note_launch();
+  return launch_status();
+}
+
+}  // namespace moe

@@ -1,0 +1,88 @@
+"""Helpers shared by the GPU parity tests (inputs, oracle glue, tolerances)."""
+
+from __future__ import annotations
+
+import numpy as np
+import torch
+
+from oracle import moe_oracle as O
+from paper_2603_02376_gb300 import inputs as I
+
+U32 = 2.0 ** -24   # fp32 unit roundoff
+UBF16 = 2.0 ** -8  # bf16 unit roundoff (8 significant bits)
+
+
+def f64(t) -> np.ndarray:
+    return t.detach().to(torch.float64).cpu().numpy()
+
+
+def oracle_cfg(wl, T=None) -> O.LayerConfig:
+    return O.LayerConfig(T=wl.T if T is None else T, H=wl.H, E=wl.E, k=wl.k, I=wl.I,
+                         I_shared=wl.I_shared, n_groups=wl.n_groups, topk_groups=wl.topk_groups,
+                         gate=wl.gate, normalize=wl.normalize, route_scale=wl.route_scale)
+
+
+def bias32(b):
+    return None if b is None else b.detach().cpu().numpy().astype(np.float32)
+
+
+def prepare_routing(wl, d, seed=0, min_margin=1e-3):
+    """Make the workload's routing well-posed on the oracle's side.
+
+    Calibrates the bias for the balanced / Zipf workloads with the oracle
+    gate, then redraws token rows whose decision margin is <= min_margin.
+    Mutates d["x"] (device) and d["bias"]; returns a dict of realised stats.
+    """
+    cfg = oracle_cfg(wl)
+    Wr = f64(d["Wr"])
+    xh = f64(d["x"])
+    L = O.router_logits(xh, Wr)
+
+    def counts_of(b):
+        idx, _ = O.gate_topk(L, b.numpy().astype(np.float32), cfg)
+        return np.bincount(idx.reshape(-1), minlength=wl.E)
+
+    stats = {}
+    if wl.balance == "balanced":
+        b, c = I.calibrate_balanced(counts_of, wl, d["bias"].cpu())
+        d["bias"] = b.to(d["x"].device)
+    elif wl.balance == "zipf":
+        b, c = I.calibrate_zipf(counts_of, wl, seed)
+        d["bias"] = b.to(d["x"].device)
+    b32 = bias32(d["bias"])
+
+    rounds = 0
+    for attempt in range(64):
+        m = O.routing_margins(L, b32, cfg)
+        bad = np.nonzero(m <= min_margin)[0]
+        if bad.size == 0:
+            break
+        I.resample_rows(d["x"], bad.tolist(), seed, attempt)
+        L[bad] = O.router_logits(f64(d["x"][torch.as_tensor(bad, device=d["x"].device)]), Wr)
+        rounds += 1
+    else:
+        raise RuntimeError("margin resampling did not converge")
+    idx, _ = O.gate_topk(L, b32, cfg)
+    cnt = np.bincount(idx.reshape(-1), minlength=wl.E)
+    mean = wl.T * wl.k / wl.E
+    stats.update(resample_rounds=rounds, max_over_mean=float(cnt.max() / mean),
+                 min_over_mean=float(cnt.min() / mean), oracle_logits=L)
+    return stats
+
+
+def logits_bound(x, Wr) -> np.ndarray:
+    """Worst-case fp32 summation error bound H * u * sum_h |x_h Wr_eh| per logit."""
+    S = np.abs(x) @ np.abs(Wr).T
+    return x.shape[1] * U32 * S + 1e-30
+
+
+def assert_layer_close(got, ref, atol=2e-2, rtol=1e-2):
+    """The layer tolerance: |got - ref| <= atol + rtol * |ref| elementwise."""
+    got = np.asarray(got, dtype=np.float64)
+    err = np.abs(got - ref)
+    lim = atol + rtol * np.abs(ref)
+    bad = err > lim
+    rel = np.linalg.norm(got - ref) / max(np.linalg.norm(ref), 1e-30)
+    assert not bad.any(), (f"{bad.sum()} of {bad.size} elements out of tolerance; "
+                           f"max|err| {err.max():.3e}, rel-fro {rel:.3e}")
+    return float(err.max()), float(rel)

@@ -1,0 +1,135 @@
+"""Host-side checks of the C ABI (no GPU needed).
+
+The library must load, export every function include/moe.h declares, and
+reject bad arguments on the host before any CUDA call.
+"""
+
+import ctypes
+import os
+import re
+
+import pytest
+
+from paper_2603_02376_gb300 import _lib as L
+from paper_2603_02376_gb300 import inputs as I
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+@pytest.fixture(scope="module")
+def lib():
+    if not os.path.exists(L.LIB_PATH):
+        from paper_2603_02376_gb300 import build
+        build.build_library()
+    return L.load()
+
+
+def header_functions():
+    src = open(os.path.join(ROOT, "include", "moe.h")).read()
+    src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+    return sorted(set(re.findall(r"\b(moe_[a-z_]+)\s*\(", src)))
+
+
+def test_header_declares_the_boundary():
+    names = header_functions()
+    for n in ("moe_gate_topk", "moe_dispatch", "moe_expert_ffn", "moe_combine",
+              "moe_layer_forward", "moe_router_logits"):
+        assert n in names
+
+
+def test_library_exports_every_declared_symbol(lib):
+    for n in header_functions():
+        assert hasattr(lib, n), n
+    assert set(header_functions()) <= set(L.EXPORTS) | {"moe_status_string"}
+
+
+def test_status_strings(lib):
+    assert L.status_string(0) == "MOE_OK"
+    assert L.status_string(L.MOE_ERR_TIMEOUT) == "MOE_ERR_TIMEOUT"
+    assert L.status_string(99) == "MOE_ERR_UNKNOWN"
+
+
+GOOD = dict(T=128, H=7168, E=256, k=8, I=2048, I_shared=2048, n_groups=8, topk_groups=4,
+            gate=1, normalize=1, route_scale=2.5)
+
+
+@pytest.mark.parametrize("bad", [
+    dict(H=100), dict(H=192), dict(I=64), dict(E=0), dict(E=2000), dict(k=0), dict(k=33),
+    dict(E=8, k=9, n_groups=1, topk_groups=1), dict(n_groups=7), dict(topk_groups=9),
+    dict(topk_groups=0), dict(n_groups=8, topk_groups=1, k=33), dict(gate=2), dict(normalize=3),
+    dict(T=-1), dict(I_shared=100), dict(route_scale=float("nan")),
+    dict(n_groups=64, E=256),
+])
+def test_invalid_configs_rejected(lib, bad):
+    c = L.config(**{**GOOD, **bad})
+    assert L.moe_validate_config(c) == L.MOE_ERR_INVALID_ARG
+    assert L.moe_workspace_size(c, L.exec_config()) == 0
+
+
+def test_group_limit_k_constraint(lib):
+    # 8 groups of 32, keep 1 group -> at most 32 experts can be picked
+    assert L.moe_validate_config(L.config(**{**GOOD, "topk_groups": 1, "k": 32})) == 0
+    c = L.config(**{**GOOD, "E": 64, "topk_groups": 1, "k": 9})  # groups of 8
+    assert L.moe_validate_config(c) == L.MOE_ERR_INVALID_ARG
+
+
+def test_valid_configs_and_workspace(lib):
+    for wl in I.WORKLOADS.values():
+        c = L.config_of(wl)
+        assert L.moe_validate_config(c) == L.MOE_OK
+        n = L.moe_workspace_size(c, L.exec_config())
+        per_token = wl.k * (2 * wl.H + wl.I) * 2
+        assert n >= wl.T * per_token
+    c = L.config_of(I.PREFILL)
+    seq = L.moe_workspace_size(c, L.exec_config())
+    ovl = L.moe_workspace_size(c, L.exec_config(overlap=1, chunk_tokens=512))
+    assert ovl > 0 and seq > 0
+    assert L.moe_workspace_size(c, L.exec_config(overlap=1, chunk_axis=2)) == 0
+    assert L.moe_workspace_size(c, L.exec_config(overlap=1, chunk_tokens=0)) == 0
+    assert L.moe_workspace_size(c, L.exec_config(overlap=1, chunk_axis=1, n_expert_chunks=0)) == 0
+
+
+def test_entry_points_reject_bad_arguments_without_a_gpu(lib):
+    c = L.config(**GOOD)
+    bad = L.config(**{**GOOD, "H": 100})
+    z = ctypes.c_void_p(0)
+    p = ctypes.c_void_p(0x1000)       # never dereferenced: validation fails first
+    odd = ctypes.c_void_p(0x1002)     # misaligned
+    cb = ctypes.byref
+    assert lib.moe_router_logits(cb(bad), p, p, p, z, 0, z) == L.MOE_ERR_INVALID_ARG
+    assert lib.moe_router_logits(cb(c), z, p, p, z, 0, z) == L.MOE_ERR_INVALID_ARG
+    assert lib.moe_router_logits(cb(c), odd, p, p, z, 0, z) == L.MOE_ERR_INVALID_ARG
+    assert lib.moe_gate_topk(cb(c), z, z, p, p, z) == L.MOE_ERR_INVALID_ARG
+    assert lib.moe_gate_topk(cb(bad), p, z, p, p, z) == L.MOE_ERR_INVALID_ARG
+    assert lib.moe_dispatch(cb(c), p, p, p, p, p, p, p, z, 0, z) == L.MOE_ERR_WORKSPACE
+    assert lib.moe_dispatch(cb(c), z, p, p, p, p, p, p, p, 1 << 30, z) == L.MOE_ERR_INVALID_ARG
+    assert lib.moe_expert_ffn(16, 100, 128, 1, p, p, p, p, p, p, 1 << 20, z) == L.MOE_ERR_INVALID_ARG
+    assert lib.moe_expert_ffn(16, 256, 128, 0, p, p, p, p, p, p, 1 << 20, z) == L.MOE_ERR_INVALID_ARG
+    assert lib.moe_expert_ffn(16, 256, 128, 1, p, p, p, p, p, z, 0, z) == L.MOE_ERR_WORKSPACE
+    assert lib.moe_expert_ffn(16, 256, 128, 1, odd, p, p, p, p, p, 1 << 20, z) == L.MOE_ERR_INVALID_ARG
+    assert lib.moe_combine(cb(c), p, p, p, z, p, 2, z) == L.MOE_ERR_INVALID_ARG
+    assert lib.moe_combine(cb(c), p, p, p, z, odd, 0, z) == L.MOE_ERR_INVALID_ARG
+    ex = L.exec_config()
+    W = L.moe_weights(0x1000, None, 0x1000, 0x1000, 0x1000, 0x1000)
+    assert lib.moe_layer_forward(cb(c), cb(ex), cb(W), p, p, None, z, 0, z, z) == L.MOE_ERR_WORKSPACE
+    Wn = L.moe_weights(0x1000, None, 0x1000, 0x1000, None, None)  # shared expert missing
+    assert lib.moe_layer_forward(cb(c), cb(ex), cb(Wn), p, p, None, p, 1 << 40, z, z) == L.MOE_ERR_INVALID_ARG
+    exb = L.exec_config(overlap=3)
+    assert lib.moe_layer_forward(cb(c), cb(exb), cb(W), p, p, None, p, 1 << 40, z, z) == L.MOE_ERR_INVALID_ARG
+
+
+def test_empty_batch_is_a_no_op(lib):
+    c = L.config(**{**GOOD, "T": 0})
+    z = ctypes.c_void_p(0)
+    cb = ctypes.byref
+    assert lib.moe_router_logits(cb(c), z, z, z, z, 0, z) == L.MOE_OK
+    assert lib.moe_gate_topk(cb(c), z, z, z, z, z) == L.MOE_OK
+    assert lib.moe_combine(cb(c), z, z, z, z, z, 0, z) == L.MOE_OK
+    assert lib.moe_expert_ffn(0, 256, 128, 4, z, z, z, z, z, z, 0, z) == L.MOE_OK
+    W = L.moe_weights(0x1000, None, 0x1000, 0x1000, 0x1000, 0x1000)
+    assert lib.moe_layer_forward(cb(c), cb(L.exec_config()), cb(W), z, z, None, z, 0, z, z) == L.MOE_OK
+
+
+def test_binding_names_match_header():
+    for n in header_functions():
+        assert hasattr(L, n), n

@@ -1,0 +1,211 @@
+"""Whole-layer GPU parity against the CPU oracle, through moe_layer_forward.
+
+* tiny (T=64, H=256, E=8, k=2, softmax): every token checked.
+* decode (T=128, DeepSeek-V3 layer): every token checked.
+* prefill (T=4096, balanced) and skewed (T=8192, Zipf): a seeded sample of
+  256 tokens, in the sequential mode and both two-stream pipelined modes.
+Routing is compared bit for bit with the oracle gate run on the GPU's own
+fp32 logits; the GPU logits stay within the fp32 summation bound; the
+permutation of the GPU routing is bit-exact; the layer output is within
+|err| <= 2e-2 + 1e-2 |ref| of the oracle's fp64 result (inputs resampled so
+every routing margin exceeds 1e-3, so both sides route identically).
+"""
+
+import numpy as np
+import pytest
+import torch
+
+from oracle import moe_oracle as O
+from paper_2603_02376_gb300 import _lib as L
+from paper_2603_02376_gb300 import inputs as I
+from tests._support import assert_layer_close, bias32, f64, logits_bound, oracle_cfg, \
+    prepare_routing
+
+pytestmark = pytest.mark.gpu
+DEV = "cuda"
+
+
+@pytest.fixture(scope="module", autouse=True)
+def lib():
+    return L.load()
+
+
+@pytest.fixture(scope="module")
+def big_weights():
+    """The DeepSeek-V3-shaped layer (22.5 GB of bf16 expert weights), drawn once."""
+    d = I.layer_inputs(I.DECODE, seed=0, device=DEV)
+    d.pop("x")
+    yield d
+    del d
+    torch.cuda.empty_cache()
+
+
+def run_layer(wl, d, ex, aux=True):
+    cfg = L.config_of(wl)
+    T, H, E, k = wl.T, wl.H, wl.E, wl.k
+    ws = torch.empty(L.moe_workspace_size(cfg, ex), dtype=torch.uint8, device=DEV)
+    out = torch.empty((T, H), dtype=torch.float32 if ex.out_fp32 else torch.bfloat16, device=DEV)
+    a = dict(logits=torch.empty((T, E), device=DEV),
+             topk_idx=torch.empty((T, k), dtype=torch.int32, device=DEV),
+             topk_w=torch.empty((T, k), device=DEV),
+             counts=torch.empty(E, dtype=torch.int32, device=DEV)) if aux else {}
+    W = L.weights_struct(d["Wr"], d["bias"], d["W13"], d["W2"], d["Ws13"], d["Ws2"])
+    L.moe_layer_forward(cfg, ex, W, d["x"], out, L.aux_struct(**a) if aux else None, ws)
+    L.moe_check_errors()
+    return out, a
+
+
+def check_routing(wl, d, a, L_oracle):
+    """Logits within the fp32 bound, routing bit-exact given the GPU logits, counts exact."""
+    cfg = oracle_cfg(wl)
+    Lg = a["logits"].cpu().numpy()
+    xh = f64(d["x"])
+    bound = logits_bound(xh, f64(d["Wr"]))
+    err = np.abs(Lg.astype(np.float64) - (xh @ f64(d["Wr"]).T))
+    assert (err <= bound).all(), f"logits max err {err.max():.3e}"
+    ridx, rw = O.gate_topk(Lg, bias32(d["bias"]), cfg)
+    gidx = a["topk_idx"].cpu().numpy()
+    np.testing.assert_array_equal(gidx, ridx)
+    np.testing.assert_allclose(a["topk_w"].cpu().numpy(), rw, rtol=2e-5, atol=1e-7)
+    oidx, _ = O.gate_topk(L_oracle, bias32(d["bias"]), cfg)
+    np.testing.assert_array_equal(gidx, oidx)   # margins make the oracle's own routing agree
+    np.testing.assert_array_equal(a["counts"].cpu().numpy(),
+                                  np.bincount(ridx.reshape(-1), minlength=wl.E))
+    return gidx
+
+
+def check_permutation(wl, d, gidx):
+    """moe_dispatch on the layer's routing equals the oracle permutation bit for bit."""
+    T, H, E, k = wl.T, wl.H, wl.E, wl.k
+    c = L.config_of(wl)
+    counts = torch.empty(E, dtype=torch.int32, device=DEV)
+    offsets = torch.empty(E + 1, dtype=torch.int32, device=DEV)
+    rst = torch.empty(T * k, dtype=torch.int32, device=DEV)
+    slot = torch.empty(T * k, dtype=torch.int32, device=DEV)
+    xp = torch.empty((T * k, H), dtype=torch.bfloat16, device=DEV)
+    ws = torch.empty(L.moe_dispatch_workspace_size(c), dtype=torch.uint8, device=DEV)
+    L.moe_dispatch(c, d["x"], torch.from_numpy(gidx).to(DEV), counts, offsets, rst, slot, xp, ws)
+    torch.cuda.synchronize()
+    rc, ro, rr, rs = O.permutation(gidx, E)
+    np.testing.assert_array_equal(offsets.cpu().numpy(), ro)
+    np.testing.assert_array_equal(rst.cpu().numpy(), rr)
+    np.testing.assert_array_equal(slot.cpu().numpy(), rs)
+    rows = torch.from_numpy(np.random.default_rng(0).choice(T * k, 512)).to(DEV)
+    assert torch.equal(xp[rows], d["x"][rst[rows].long()])
+
+
+def oracle_tokens(wl, d, toks):
+    cfg = oracle_cfg(wl)
+    Wr = f64(d["Wr"])
+
+    def expert(e):
+        return f64(d["W13"][e]), f64(d["W2"][e])
+
+    shared = (lambda: (f64(d["Ws13"]), f64(d["Ws2"]))) if wl.I_shared else None
+    out, idx, _ = O.layer_forward_tokens(f64(d["x"][torch.as_tensor(toks, device=DEV)]), Wr,
+                                         bias32(d["bias"]), expert, cfg, shared)
+    return out, idx
+
+
+# ---------------------------------------------------------------- tiny: every token
+
+@pytest.mark.parametrize("out_fp32", [1, 0])
+def test_layer_tiny_full(out_fp32):
+    wl = I.TINY
+    d = I.layer_inputs(wl, seed=0, device=DEV)
+    st = prepare_routing(wl, d)
+    out, a = run_layer(wl, d, L.exec_config(out_fp32=out_fp32))
+    gidx = check_routing(wl, d, a, st["oracle_logits"])
+    check_permutation(wl, d, gidx)
+    ref, _ = O.layer_forward(f64(d["x"]), f64(d["Wr"]), None, f64(d["W13"]), f64(d["W2"]),
+                             oracle_cfg(wl))
+    assert_layer_close(f64(out), ref)
+
+
+# ---------------------------------------------------------------- decode: every token
+
+@pytest.mark.parametrize("ex", [dict(out_fp32=1), dict(out_fp32=0),
+                                dict(out_fp32=1, overlap=1, chunk_axis=1, n_expert_chunks=4)])
+def test_layer_decode_full(big_weights, ex):
+    wl = I.DECODE
+    d = dict(big_weights)
+    d["x"] = I.randn((wl.T, wl.H), 1.0, torch.bfloat16, 0, "x", DEV)
+    st = prepare_routing(wl, d)
+    out, a = run_layer(wl, d, L.exec_config(**ex))
+    gidx = check_routing(wl, d, a, st["oracle_logits"])
+    check_permutation(wl, d, gidx)
+    ref, _ = oracle_tokens(wl, d, np.arange(wl.T))
+    assert_layer_close(f64(out), ref)
+
+
+# ---------------------------------------------------------------- prefill / skewed: sampled
+
+@pytest.fixture(scope="module")
+def prefill_inputs(big_weights):
+    wl = I.PREFILL
+    d = dict(big_weights)
+    d["x"] = I.randn((wl.T, wl.H), 1.0, torch.bfloat16, 0, "x", DEV)
+    st = prepare_routing(wl, d)
+    assert st["max_over_mean"] <= 1.15 and st["min_over_mean"] >= 0.85
+    toks = I.sample_tokens(wl.T, 256, 0).numpy()
+    ref, _ = oracle_tokens(wl, d, toks)
+    return d, st, toks, ref
+
+
+@pytest.mark.parametrize("ex", [
+    dict(out_fp32=1),
+    dict(out_fp32=0),
+    dict(out_fp32=1, overlap=1, chunk_axis=0, chunk_tokens=512),
+    dict(out_fp32=1, overlap=1, chunk_axis=1, n_expert_chunks=8),
+])
+def test_layer_prefill_sampled(prefill_inputs, ex):
+    wl = I.PREFILL
+    d, st, toks, ref = prefill_inputs
+    out, a = run_layer(wl, d, L.exec_config(**ex))
+    gidx = check_routing(wl, d, a, st["oracle_logits"])
+    if ex.get("overlap", 0) == 0 and ex["out_fp32"] == 1:
+        check_permutation(wl, d, gidx)
+    assert_layer_close(f64(out[torch.as_tensor(toks, device=DEV)]), ref)
+
+
+def test_layer_skewed_sampled(big_weights):
+    wl = I.SKEWED
+    d = dict(big_weights)
+    d["x"] = I.randn((wl.T, wl.H), 1.0, torch.bfloat16, 0, "x", DEV)
+    st = prepare_routing(wl, d)
+    assert st["max_over_mean"] > 8.0   # a real hot expert
+    toks = I.sample_tokens(wl.T, 256, 0).numpy()
+    ref, _ = oracle_tokens(wl, d, toks)
+    for ex in (L.exec_config(out_fp32=1), L.exec_config(out_fp32=1, overlap=1, chunk_axis=1)):
+        out, a = run_layer(wl, d, ex)
+        gidx = check_routing(wl, d, a, st["oracle_logits"])
+        assert_layer_close(f64(out[torch.as_tensor(toks, device=DEV)]), ref)
+    check_permutation(wl, d, gidx)
+
+
+# ---------------------------------------------------------------- data-movement sweep
+
+@pytest.mark.parametrize("T", I.DISPATCH_SWEEP_T)
+def test_dispatch_combine_sweep_identity(T):
+    """Uniform routing, identity experts: dispatch then combine with weights 1/k returns x."""
+    H, E, k = 7168, 256, 8
+    c = L.config(T, H, E, k, 2048)
+    idx, _ = I.uniform_routing(T, E, k, seed=0, device=DEV)
+    x = I.randn((T, H), 1.0, torch.bfloat16, 0, "x", DEV)
+    counts = torch.empty(E, dtype=torch.int32, device=DEV)
+    offsets = torch.empty(E + 1, dtype=torch.int32, device=DEV)
+    rst = torch.empty(T * k, dtype=torch.int32, device=DEV)
+    slot = torch.empty(T * k, dtype=torch.int32, device=DEV)
+    xp = torch.empty((T * k, H), dtype=torch.bfloat16, device=DEV)
+    ws = torch.empty(L.moe_dispatch_workspace_size(c), dtype=torch.uint8, device=DEV)
+    L.moe_dispatch(c, x, idx, counts, offsets, rst, slot, xp, ws)
+    w = torch.full((T, k), 1.0 / k, device=DEV)
+    out = torch.empty((T, H), dtype=torch.bfloat16, device=DEV)
+    L.moe_combine(c, xp, slot, w, None, out, 0)
+    torch.cuda.synchronize()
+    assert torch.equal(out, x)
+    rc, ro, rr, rs = O.permutation(idx.cpu().numpy(), E)
+    np.testing.assert_array_equal(offsets.cpu().numpy(), ro)
+    np.testing.assert_array_equal(slot.cpu().numpy(), rs)
+    del xp
+    torch.cuda.empty_cache()

@@ -85,7 +85,27 @@ typedef struct {
  */
 typedef struct {
   int32_t overlap, chunk_tokens, chunk_axis, n_expert_chunks, out_fp32;
+  /* Optional tracing: an array of MOE_N_STAGE_EVENTS cudaEvent_t (created by
+   * the caller) recorded on `stream` at the stage boundaries of a sequential
+   * (overlap = 0) forward; NULL = no tracing. Ignored when overlap = 1. */
+  void** stage_events;
 } moe_exec;
+
+/* Indices into moe_exec.stage_events: event i is recorded when stage i ends
+ * (MOE_EV_START before the first kernel). */
+enum {
+  MOE_EV_START = 0,
+  MOE_EV_ROUTER = 1,       /* router logits */
+  MOE_EV_GATE = 2,         /* gate + group-limited top-k */
+  MOE_EV_PERMUTE = 3,      /* histogram, scan, stable permutation */
+  MOE_EV_DISPATCH = 4,     /* packing of token rows into expert segments */
+  MOE_EV_GEMM1 = 5,        /* routed grouped GEMM1 + SwiGLU */
+  MOE_EV_GEMM2 = 6,        /* routed grouped GEMM2 */
+  MOE_EV_SHARED_GEMM1 = 7, /* shared expert GEMM1 + SwiGLU */
+  MOE_EV_SHARED_GEMM2 = 8, /* shared expert GEMM2 */
+  MOE_EV_COMBINE = 9,      /* weighted combine (+ shared term) */
+  MOE_N_STAGE_EVENTS = 10
+};
 
 /* Layer weights (device pointers). Wr [E,H] fp32; bias [E] fp32 or NULL;
  * W13 [E,2I,H] bf16 (rows 0..I-1 gate, I..2I-1 up); W2 [E,H,I] bf16;

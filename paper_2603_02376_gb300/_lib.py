@@ -45,7 +45,13 @@ class moe_config(ctypes.Structure):
 
 class moe_exec(ctypes.Structure):
     _fields_ = [(n, ctypes.c_int32) for n in
-                ("overlap", "chunk_tokens", "chunk_axis", "n_expert_chunks", "out_fp32")]
+                ("overlap", "chunk_tokens", "chunk_axis", "n_expert_chunks", "out_fp32")] + \
+               [("stage_events", ctypes.POINTER(ctypes.c_void_p))]
+
+
+STAGES = ("start", "router", "gate", "permute", "dispatch", "gemm1", "gemm2", "shared_gemm1",
+          "shared_gemm2", "combine")
+MOE_N_STAGE_EVENTS = len(STAGES)
 
 
 class moe_weights(ctypes.Structure):
@@ -136,8 +142,15 @@ def config_of(wl, T=None) -> moe_config:
                   wl.topk_groups, wl.gate, wl.normalize, wl.route_scale)
 
 
-def exec_config(overlap=0, chunk_tokens=512, chunk_axis=0, n_expert_chunks=8, out_fp32=0):
-    return moe_exec(overlap, chunk_tokens, chunk_axis, n_expert_chunks, out_fp32)
+def exec_config(overlap=0, chunk_tokens=512, chunk_axis=0, n_expert_chunks=8, out_fp32=0,
+                stage_events=None):
+    """moe_exec; stage_events: a list of MOE_N_STAGE_EVENTS torch.cuda.Event (or None)."""
+    ex = moe_exec(overlap, chunk_tokens, chunk_axis, n_expert_chunks, out_fp32, None)
+    if stage_events is not None:
+        arr = (ctypes.c_void_p * MOE_N_STAGE_EVENTS)(*[int(e.cuda_event) for e in stage_events])
+        ex._events_keepalive = arr
+        ex.stage_events = ctypes.cast(arr, ctypes.POINTER(ctypes.c_void_p))
+    return ex
 
 
 # ---------------------------------------------------------------- entry points

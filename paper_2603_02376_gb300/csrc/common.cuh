@@ -64,7 +64,7 @@ moe_status launch_sum_counts(const int32_t* counts, int n_chunks, int E, int32_t
 moe_status launch_expert_ffn(int rows, int H, int I, int n_experts, int e_begin, int e_end,
                              const uint16_t* x_perm, const int32_t* offsets, const uint16_t* W13,
                              const uint16_t* W2, uint16_t* h, uint16_t* y_perm, int rows_hint,
-                             cudaStream_t s);
+                             cudaStream_t s, cudaEvent_t after_gemm1 = nullptr);
 
 // ----------------------------------------------------------------------------
 // device helpers

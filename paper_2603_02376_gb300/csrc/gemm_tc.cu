@@ -502,7 +502,8 @@ moe_status launch_gemm(const CUtensorMap& A, const CUtensorMap& B, const int32_t
 template <int NMAX>
 moe_status run_ffn(int rows, int H, int I, int n_experts, int e_begin, int e_end,
                    const uint16_t* x_perm, const int32_t* offsets, const uint16_t* W13,
-                   const uint16_t* W2, uint16_t* h, uint16_t* y_perm, cudaStream_t s) {
+                   const uint16_t* W2, uint16_t* h, uint16_t* y_perm, cudaStream_t s,
+                   cudaEvent_t after_gemm1) {
   CUtensorMap a1, b1, a2, b2;
   if (!make_map(&a1, W13, H, (uint64_t)n_experts * 2 * I, BK, BM) ||
       !make_map(&b1, x_perm, H, rows, BK, B_BOX) ||
@@ -513,6 +514,7 @@ moe_status run_ffn(int rows, int H, int I, int n_experts, int e_begin, int e_end
   moe_status st = launch_gemm<true, NMAX>(a1, b1, offsets, rows, e_begin, n_exp, H, I / BM, 2 * I,
                                           I, h, I, s);
   if (st != MOE_OK) return st;
+  if (after_gemm1 && cudaEventRecord(after_gemm1, s) != cudaSuccess) return MOE_ERR_CUDA;
   return launch_gemm<false, NMAX>(a2, b2, offsets, rows, e_begin, n_exp, I, H / BM, H, 0, y_perm,
                                   H, s);
 }
@@ -522,15 +524,15 @@ moe_status run_ffn(int rows, int H, int I, int n_experts, int e_begin, int e_end
 moe_status launch_expert_ffn(int rows, int H, int I, int n_experts, int e_begin, int e_end,
                              const uint16_t* x_perm, const int32_t* offsets, const uint16_t* W13,
                              const uint16_t* W2, uint16_t* h, uint16_t* y_perm, int rows_hint,
-                             cudaStream_t s) {
+                             cudaStream_t s, cudaEvent_t after_gemm1) {
   if (rows == 0 || e_end <= e_begin) return MOE_OK;
   const int n_exp = e_end - e_begin;
   // Few rows per expert (decode): small token tiles leave room for a deeper pipeline.
   if ((long)rows_hint <= 24L * n_exp)
     return run_ffn<32>(rows, H, I, n_experts, e_begin, e_end, x_perm, offsets, W13, W2, h, y_perm,
-                       s);
+                       s, after_gemm1);
   return run_ffn<256>(rows, H, I, n_experts, e_begin, e_end, x_perm, offsets, W13, W2, h, y_perm,
-                      s);
+                      s, after_gemm1);
 }
 
 }  // namespace moe

@@ -199,41 +199,57 @@ bool events(int d, size_t n, std::vector<cudaEvent_t>* out) {
   } while (0)
 
 // Router + gate + permutation (+ packing) of tokens [t0, t0+Tc) into chunk slot `ci`.
+// Records stage event i of a traced forward (no-op without tracing).
+moe_status mark(cudaEvent_t* ev, int i, cudaStream_t s) {
+  if (ev && ev[i] && cudaEventRecord(ev[i], s) != cudaSuccess) return MOE_ERR_CUDA;
+  return MOE_OK;
+}
+
 moe_status pack_tokens(const moe_config& c, const Layout& L, const moe_weights& w,
                        const uint16_t* x, int t0, int Tc, int ci, bool pack_rows,
-                       cudaStream_t s) {
+                       cudaStream_t s, cudaEvent_t* ev = nullptr) {
   moe_config cc = c;
   cc.T = Tc;
   const size_t tk = (size_t)t0 * c.k;
   MOE_TRY(launch_router(cc, x + (size_t)t0 * c.H, w.Wr, L.logits + (size_t)t0 * c.E, L.partials,
                         L.splits, s));
+  MOE_TRY(mark(ev, MOE_EV_ROUTER, s));
   MOE_TRY(launch_gate(cc, L.logits + (size_t)t0 * c.E, w.bias, L.idx + tk, L.w + tk, s));
+  MOE_TRY(mark(ev, MOE_EV_GATE, s));
   MOE_TRY(launch_permutation(cc, L.idx + tk, L.counts + (size_t)ci * c.E,
                              L.offsets + (size_t)ci * (c.E + 1), L.rst + tk, L.slot_row + tk,
                              L.perm_counts, L.perm_base, s));
+  MOE_TRY(mark(ev, MOE_EV_PERMUTE, s));
   if (pack_rows)
     MOE_TRY(launch_dispatch_rows(Tc, c.H, c.k, x + (size_t)t0 * c.H, L.slot_row + tk,
                                  L.x_perm + tk * c.H, s));
+  MOE_TRY(mark(ev, MOE_EV_DISPATCH, s));
   return MOE_OK;
 }
 
 // Routed experts of chunk ci (tokens [t0, t0+Tc)), experts [e0, e1), then nothing else.
 moe_status experts_tokens(const moe_config& c, const Layout& L, const moe_weights& w, int t0,
-                          int Tc, int ci, int e0, int e1, cudaStream_t s) {
+                          int Tc, int ci, int e0, int e1, cudaStream_t s,
+                          cudaEvent_t* ev = nullptr) {
   const size_t tk = (size_t)t0 * c.k;
   const int rows = Tc * c.k;
   const long hint = (long)rows * (e1 - e0) / c.E;
-  return launch_expert_ffn(rows, c.H, c.I, c.E, e0, e1, L.x_perm + tk * c.H,
-                           L.offsets + (size_t)ci * (c.E + 1), w.W13, w.W2, L.h + tk * c.I,
-                           L.y_perm + tk * c.H, (int)hint, s);
+  MOE_TRY(launch_expert_ffn(rows, c.H, c.I, c.E, e0, e1, L.x_perm + tk * c.H,
+                            L.offsets + (size_t)ci * (c.E + 1), w.W13, w.W2, L.h + tk * c.I,
+                            L.y_perm + tk * c.H, (int)hint, s, ev ? ev[MOE_EV_GEMM1] : nullptr));
+  return mark(ev, MOE_EV_GEMM2, s);
 }
 
 moe_status shared_expert(const moe_config& c, const Layout& L, const moe_weights& w,
-                         const uint16_t* x, cudaStream_t s) {
-  if (!c.I_shared) return MOE_OK;
+                         const uint16_t* x, cudaStream_t s, cudaEvent_t* ev = nullptr) {
+  if (!c.I_shared) {
+    MOE_TRY(mark(ev, MOE_EV_SHARED_GEMM1, s));
+    return mark(ev, MOE_EV_SHARED_GEMM2, s);
+  }
   MOE_TRY(launch_fill_range(L.sh_off, c.T, s));
-  return launch_expert_ffn(c.T, c.H, c.I_shared, 1, 0, 1, x, L.sh_off, w.Ws13, w.Ws2, L.sh_h,
-                           L.sh_y, c.T, s);
+  MOE_TRY(launch_expert_ffn(c.T, c.H, c.I_shared, 1, 0, 1, x, L.sh_off, w.Ws13, w.Ws2, L.sh_h,
+                            L.sh_y, c.T, s, ev ? ev[MOE_EV_SHARED_GEMM1] : nullptr));
+  return mark(ev, MOE_EV_SHARED_GEMM2, s);
 }
 
 moe_status combine_tokens(const moe_config& c, const Layout& L, int t0, int Tc, void* out,
@@ -393,10 +409,13 @@ moe_status moe_layer_forward(const moe_config* cfg, const moe_exec* ex, const mo
   const int dev = current_device();
 
   if (!ex->overlap) {
-    MOE_TRY(pack_tokens(c, L, *w, x, 0, c.T, 0, true, s));
-    MOE_TRY(experts_tokens(c, L, *w, 0, c.T, 0, 0, c.E, s));
-    MOE_TRY(shared_expert(c, L, *w, x, s));
+    cudaEvent_t* ev = reinterpret_cast<cudaEvent_t*>(ex->stage_events);
+    MOE_TRY(mark(ev, MOE_EV_START, s));
+    MOE_TRY(pack_tokens(c, L, *w, x, 0, c.T, 0, true, s, ev));
+    MOE_TRY(experts_tokens(c, L, *w, 0, c.T, 0, 0, c.E, s, ev));
+    MOE_TRY(shared_expert(c, L, *w, x, s, ev));
     MOE_TRY(combine_tokens(c, L, 0, c.T, out, ex->out_fp32, s));
+    MOE_TRY(mark(ev, MOE_EV_COMBINE, s));
     if (aux && aux->counts)
       MOE_CUDA(cudaMemcpyAsync(aux->counts, L.counts, sizeof(int32_t) * c.E,
                                cudaMemcpyDeviceToDevice, s));

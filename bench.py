@@ -1,0 +1,455 @@
+#!/usr/bin/env python3
+"""Benchmark of the DeepSeek-V3 MoE layer forward on GB300.
+
+One step = one full layer forward (router -> gate/top-k -> permutation ->
+dispatch -> grouped GEMM1+SwiGLU -> grouped GEMM2 -> shared expert ->
+combine) over one batch of synthetic tokens, through the library's C ABI.
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--workload decode]
+    python bench.py --impl reference ...     # the CPU oracle, timed on host cores
+
+Prints one JSON line (rank 0). With N > 1 (torchrun) every rank runs an
+independent replica of the layer on its own tokens (no collective on the data
+path); the barrier and max-over-ranks timing use a gloo process group.
+"""
+
+from __future__ import annotations
+
+import argparse
+import datetime as _dt
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+import numpy as np  # noqa: E402
+import torch  # noqa: E402
+
+from paper_2603_02376_gb300 import inputs as I  # noqa: E402
+
+METRIC = "MoE layer tokens/sec on 1 GB300; grouped-GEMM % bf16 peak; dispatch/combine % HBM BW"
+FALLBACK_HBM_GBS = 6800.0
+FALLBACK_BF16_TFLOPS = 1900.0
+TRAFFIC_FILE = os.path.join(ROOT, "profiles", "traffic.json")
+GEMM_SOURCES = ("paper_2603_02376_gb300/csrc/gemm_tc.cu", "paper_2603_02376_gb300/csrc/common.cuh")
+
+
+def parse():
+    p = argparse.ArgumentParser(description=__doc__.splitlines()[0])
+    p.add_argument("--gpus", type=int, default=1)
+    p.add_argument("--steps", type=int, default=200)
+    p.add_argument("--warmup", type=int, default=10)
+    p.add_argument("--impl", choices=("ours", "reference"), default="ours")
+    p.add_argument("--workload", choices=("decode", "prefill", "skewed", "tiny"), default="decode")
+    p.add_argument("--mode", choices=("seq", "overlap-tokens", "overlap-experts"), default="seq")
+    p.add_argument("--chunk-tokens", type=int, default=512)
+    p.add_argument("--expert-chunks", type=int, default=8)
+    p.add_argument("--no-cpu-baseline", action="store_true")
+    p.add_argument("--cpu-tokens", type=int, default=8, help="oracle sample size (tokens)")
+    return p.parse_args()
+
+
+# ---------------------------------------------------------------- distributed plumbing
+
+def dist_env():
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return rank, world, local
+
+
+def barrier(world):
+    if world > 1:
+        torch.distributed.barrier()
+
+
+def max_over_ranks(v: float, world: int) -> float:
+    if world == 1:
+        return v
+    t = torch.tensor([v], dtype=torch.float64)
+    torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+    return float(t.item())
+
+
+# ---------------------------------------------------------------- measured peaks, clocks
+
+def peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as f:
+            m = json.load(f)
+        return float(m["hbm_gbs"]), float(m["bf16_tflops"]), float(m.get(
+            "bf16_tflops_sustained", m["bf16_tflops"])), "measured"
+    except Exception:
+        return FALLBACK_HBM_GBS, FALLBACK_BF16_TFLOPS, 1700.0, "fallback"
+
+
+class ClockSampler:
+    """nvidia-smi clock/throttle samples; only those inside the timed window count."""
+
+    FIELDS = ("timestamp,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+    NAMES = ("hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap")
+
+    def __init__(self, device_index: int):
+        self.proc = None
+        self.lines = []
+        sel = []
+        try:
+            uuid = str(torch.cuda.get_device_properties(device_index).uuid)
+            sel = ["-i", uuid if uuid.startswith("GPU-") else "GPU-" + uuid]
+        except Exception:
+            sel = ["-i", str(device_index)]
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", *sel, "--query-gpu=" + self.FIELDS, "--format=csv,noheader",
+                 "-lms", "100"], stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except Exception:
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return
+        self.proc.terminate()
+        try:
+            out, _ = self.proc.communicate(timeout=5)
+        except Exception:
+            self.proc.kill()
+            out, _ = self.proc.communicate()
+        self.lines = [l for l in out.splitlines() if l.strip()]
+
+    def summary(self, t0: _dt.datetime, t1: _dt.datetime):
+        rows = []
+        for l in self.lines:
+            f = [x.strip() for x in l.split(",")]
+            if len(f) < 9:
+                continue
+            try:
+                ts = _dt.datetime.strptime(f[0], "%Y/%m/%d %H:%M:%S.%f")
+                rows.append((ts, float(f[1].split()[0]), float(f[2].split()[0]), f[5:9]))
+            except Exception:
+                continue
+        inside = [r for r in rows if t0 <= r[0] <= t1]
+        window = "timed"
+        if not inside and rows:  # very short timed region: nearest samples (same workload)
+            rows.sort(key=lambda r: abs((r[0] - t0).total_seconds()))
+            inside, window = rows[:3], "adjacent"
+        if not inside:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": [], "samples": 0}
+        reasons = sorted({n for r in inside for n, v in zip(self.NAMES, r[3]) if v == "Active"})
+        return {"sm_mhz": statistics.median(r[1] for r in inside),
+                "sm_max_mhz": max(r[2] for r in inside), "reasons": reasons,
+                "samples": len(inside), "window": window}
+
+
+# ---------------------------------------------------------------- workload set-up
+
+def build_inputs(wl, device, rank):
+    d = I.layer_inputs(wl, seed=0, device=device)
+    if rank:
+        d["x"] = I.randn((wl.T, wl.H), 1.0, torch.bfloat16, rank, "x", device)
+    return d
+
+
+def gpu_counts_fn(L, wl, d, device):
+    """Per-expert counts of the GPU routing for a given bias (used to calibrate the bias)."""
+    cfg = L.config_of(wl)
+    logits = torch.empty((wl.T, wl.E), device=device)
+    idx = torch.empty((wl.T, wl.k), dtype=torch.int32, device=device)
+    w = torch.empty((wl.T, wl.k), device=device)
+    L.moe_router_logits(cfg, d["x"], d["Wr"], logits, None)
+
+    def counts(b):
+        L.moe_gate_topk(cfg, logits, b.to(device), idx, w)
+        return torch.bincount(idx.reshape(-1).long(), minlength=wl.E).cpu()
+
+    return counts
+
+
+def calibrate(L, wl, d, device):
+    if wl.balance == "balanced":
+        b, _ = I.calibrate_balanced(gpu_counts_fn(L, wl, d, device), wl, d["bias"].cpu())
+        d["bias"] = b.to(device)
+    elif wl.balance == "zipf":
+        b, _ = I.calibrate_zipf(gpu_counts_fn(L, wl, d, device), wl, 0)
+        d["bias"] = b.to(device)
+
+
+def algorithmic(wl, touched):
+    """Algorithmic bytes and flops of each stage for one forward."""
+    T, H, E, k, Iw, Is = wl.T, wl.H, wl.E, wl.k, wl.I, wl.I_shared
+    R = T * k
+    b = {
+        "router": T * H * 2 + E * H * 4 + T * E * 4,
+        "gate": T * E * 4 + T * k * 8,
+        "permute": T * k * 4 * 3,
+        "dispatch": T * H * 2 + R * H * 2,
+        "gemm1": touched * 2 * Iw * H * 2 + R * H * 2 + R * Iw * 2,
+        "gemm2": touched * H * Iw * 2 + R * Iw * 2 + R * H * 2,
+        "shared_gemm1": (2 * Is * H * 2 + T * H * 2 + T * Is * 2) if Is else 0,
+        "shared_gemm2": (H * Is * 2 + T * Is * 2 + T * H * 2) if Is else 0,
+        "combine": R * H * 2 + (T * H * 2 if Is else 0) + T * H * 2 + R * 8,
+    }
+    f = {"router": 2 * T * E * H, "gemm1": 2 * R * H * 2 * Iw, "gemm2": 2 * R * Iw * H,
+         "shared_gemm1": 2 * T * H * 2 * Is, "shared_gemm2": 2 * T * Is * H}
+    return b, f
+
+
+def source_sha():
+    h = hashlib.sha256()
+    for p in GEMM_SOURCES:
+        with open(os.path.join(ROOT, p), "rb") as f:
+            h.update(f.read())
+    return h.hexdigest()[:16]
+
+
+def measured_traffic(workload):
+    """ncu DRAM bytes per GEMM1 launch, if captured for the current kernel source."""
+    try:
+        with open(TRAFFIC_FILE) as f:
+            t = json.load(f)
+        e = t.get(workload)
+        if e and e.get("source_sha") == source_sha():
+            return float(e["dram_bytes_per_launch"])
+    except Exception:
+        pass
+    return None
+
+
+# ---------------------------------------------------------------- CPU oracle leg
+
+def oracle_tokens_per_s(wl, d, tokens):
+    """Time the CPU oracle on a sample of tokens; weights come from host copies."""
+    from oracle import moe_oracle as O
+
+    cfg = O.LayerConfig(T=len(tokens), H=wl.H, E=wl.E, k=wl.k, I=wl.I, I_shared=wl.I_shared,
+                        n_groups=wl.n_groups, topk_groups=wl.topk_groups, gate=wl.gate,
+                        normalize=wl.normalize, route_scale=wl.route_scale)
+    tok = torch.as_tensor(tokens, device=d["x"].device)
+    xr = d["x"][tok].to(torch.float64).cpu().numpy()
+    Wr = d["Wr"].cpu().numpy()
+    b = None if d["bias"] is None else d["bias"].cpu().numpy()
+    # host copies (bf16) of the experts the sample touches, made before the clock starts
+    idx, _ = O.gate_topk(O.router_logits(xr, Wr), b, cfg)
+    host = {int(e): (d["W13"][e].cpu(), d["W2"][e].cpu()) for e in np.unique(idx)}
+    shared = (d["Ws13"].cpu(), d["Ws2"].cpu()) if wl.I_shared else None
+
+    def get_expert(e):
+        a, c = host[e]
+        return a.to(torch.float64).numpy(), c.to(torch.float64).numpy()
+
+    get_shared = (lambda: (shared[0].to(torch.float64).numpy(),
+                           shared[1].to(torch.float64).numpy())) if shared else None
+    t0 = time.perf_counter()
+    O.layer_forward_tokens(xr, Wr, b, get_expert, cfg, get_shared)
+    dt = time.perf_counter() - t0
+    return len(tokens) / dt, dt, len(host)
+
+
+def cpu_baseline(wl, d, n_tokens, seed=1):
+    toks = I.sample_tokens(wl.T, n_tokens, seed).numpy()
+    v, dt, ne = oracle_tokens_per_s(wl, d, toks)
+    return {"value": v, "unit": "tokens/s", "cores": os.cpu_count(), "kind": "oracle",
+            "sample": f"{len(toks)} of the {wl.T} tokens ({ne} experts touched), numpy fp64 "
+                      f"oracle, {dt:.1f} s; BLAS threads = host cores"}
+
+
+# ---------------------------------------------------------------- main arms
+
+def run_reference(args, wl, rank, world, device):
+    if rank != 0:
+        return
+    d = build_inputs(wl, device, 0)
+    from paper_2603_02376_gb300 import _lib as L
+    if wl.balance != "none":
+        L.load()
+        calibrate(L, wl, d, device)
+    n = max(1, args.cpu_tokens // 2)
+    for s in range(args.warmup):
+        oracle_tokens_per_s(wl, d, I.sample_tokens(wl.T, n, 100 + s).numpy())
+    times = []
+    for s in range(args.steps):
+        v, dt, _ = oracle_tokens_per_s(wl, d, I.sample_tokens(wl.T, n, 1000 + s).numpy())
+        times.append(dt)
+    tot = sum(times)
+    value = n * args.steps / tot
+    line = {
+        "impl": "reference", "metric": METRIC, "value": value, "unit": "tokens/s",
+        "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": 1e3 * tot / args.steps, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+        "config": config_of(wl, args),
+        "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": os.cpu_count(),
+                         "kind": "oracle",
+                         "sample": f"{n} tokens per step of the {wl.T}-token batch, numpy fp64"},
+        "e2e": {"value": value, "unit": "tokens/s", "h2d_bytes_per_step": 0,
+                "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+
+
+def config_of(wl, args):
+    return {"workload": wl.name, "T": wl.T, "H": wl.H, "E": wl.E, "k": wl.k, "I": wl.I,
+            "I_shared": wl.I_shared, "gating": ("sigmoid+bias, 8 groups keep 4, top-8, x2.5"
+                                                if wl.gate == 1 else "softmax top-k"),
+            "mode": args.mode, "global_batch": wl.T * args.gpus,
+            "l2": "inputs larger than L2: the expert weights streamed per step exceed 129 MB",
+            "parallelism": f"replicas{args.gpus}"}
+
+
+def run_ours(args, wl, rank, world, local, device):
+    from paper_2603_02376_gb300 import _lib as L
+    L.load()
+    d = build_inputs(wl, device, rank)
+    calibrate(L, wl, d, device)
+    cfg = L.config_of(wl)
+    mode = dict(seq=dict(), **{"overlap-tokens": dict(overlap=1, chunk_axis=0,
+                                                      chunk_tokens=args.chunk_tokens),
+                               "overlap-experts": dict(overlap=1, chunk_axis=1,
+                                                       n_expert_chunks=args.expert_chunks)})[
+        args.mode]
+    ex = L.exec_config(**mode)
+    ws = torch.empty(L.moe_workspace_size(cfg, ex), dtype=torch.uint8, device=device)
+    out = torch.empty((wl.T, wl.H), dtype=torch.bfloat16, device=device)
+    W = L.weights_struct(d["Wr"], d["bias"], d["W13"], d["W2"], d["Ws13"], d["Ws2"])
+    stream = torch.cuda.current_stream()
+
+    def step():
+        L.moe_layer_forward(cfg, ex, W, d["x"], out, None, ws, stream)
+
+    # routing statistics of this batch (touched experts set the GEMM weight bytes)
+    counts = torch.empty(wl.E, dtype=torch.int32, device=device)
+    L.moe_layer_forward(cfg, L.exec_config(), W, d["x"], out, L.aux_struct(counts=counts), ws,
+                        stream)
+    L.moe_check_errors(stream)
+    cnt = counts.cpu()
+    touched = int((cnt > 0).sum())
+
+    for _ in range(args.warmup):
+        step()
+    torch.cuda.synchronize()
+    L.moe_check_errors(stream)
+
+    # --- device-resident timing
+    sampler = ClockSampler(local)
+    time.sleep(0.3)
+    barrier(world)
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    n0 = L.moe_launch_count()
+    w0 = _dt.datetime.now()
+    e0.record(stream)
+    for _ in range(args.steps):
+        step()
+    e1.record(stream)
+    torch.cuda.synchronize()
+    w1 = _dt.datetime.now()
+    barrier(world)
+    launches = L.moe_launch_count() - n0
+    ms = max_over_ranks(e0.elapsed_time(e1), world)
+    time.sleep(0.25)
+    sampler.stop()
+    clocks = sampler.summary(w0, w1)
+    L.moe_check_errors(stream)
+    value = wl.T * world * args.steps / (ms / 1e3)
+
+    # --- per-stage timing (sequential forward with stage events, same stream)
+    K2 = min(args.steps, 50)
+    evs = [[torch.cuda.Event(enable_timing=True) for _ in L.STAGES] for _ in range(K2)]
+    for i in range(K2):
+        exs = L.exec_config(stage_events=evs[i])
+        L.moe_layer_forward(cfg, exs, W, d["x"], out, None, ws, stream)
+    torch.cuda.synchronize()
+    stage_ms = {}
+    for j in range(1, len(L.STAGES)):
+        stage_ms[L.STAGES[j]] = statistics.mean(evs[i][j - 1].elapsed_time(evs[i][j])
+                                                for i in range(K2))
+
+    # --- end to end through the C ABI with host buffers (H2D x, D2H out every step)
+    xh = d["x"].cpu().pin_memory()
+    oh = torch.empty((wl.T, wl.H), dtype=torch.bfloat16).pin_memory()
+    xd = torch.empty_like(d["x"])
+    for _ in range(min(3, args.warmup)):
+        xd.copy_(xh, non_blocking=True)
+        L.moe_layer_forward(cfg, ex, W, xd, out, None, ws, stream)
+        oh.copy_(out, non_blocking=True)
+    barrier(world)
+    torch.cuda.synchronize()
+    f0, f1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    f0.record(stream)
+    for _ in range(args.steps):
+        xd.copy_(xh, non_blocking=True)
+        L.moe_layer_forward(cfg, ex, W, xd, out, None, ws, stream)
+        oh.copy_(out, non_blocking=True)
+    f1.record(stream)
+    torch.cuda.synchronize()
+    barrier(world)
+    e2e_ms = max_over_ranks(f0.elapsed_time(f1), world)
+    e2e_value = wl.T * world * args.steps / (e2e_ms / 1e3)
+
+    hbm, tf_burst, tf_sust, src = peaks()
+    b, f = algorithmic(wl, touched)
+    g1 = stage_ms["gemm1"] / 1e3
+    achieved = b["gemm1"] / g1 / 1e9
+    traffic = measured_traffic(wl.name)
+    stages = {}
+    for s_, t in stage_ms.items():
+        e = {"ms": round(t, 4)}
+        if b.get(s_):
+            e["GB/s"] = round(b[s_] / (t / 1e3) / 1e9, 1)
+            e["frac_hbm"] = round(b[s_] / (t / 1e3) / 1e9 / hbm, 3)
+        if f.get(s_):
+            e["TFLOP/s"] = round(f[s_] / (t / 1e3) / 1e12, 2)
+            e["frac_bf16"] = round(f[s_] / (t / 1e3) / 1e12 / tf_sust, 4)
+        stages[s_] = e
+
+    line = {
+        "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms / args.steps,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
+        "data": "synthetic (seeded N(0,1) activations, N(0,0.02^2) bf16 weights)",
+        "config": config_of(wl, args),
+        "e2e": {"value": e2e_value, "unit": "tokens/s", "h2d_bytes_per_step": wl.T * wl.H * 2,
+                "d2h_bytes_per_step": wl.T * wl.H * 2},
+        "gpu_launches": launches,
+        "roofline": {"bound": "hbm", "kernel": "grouped GEMM1 + SwiGLU (tcgen05)",
+                     "achieved": round(achieved, 1), "peak": hbm, "unit": "GB/s",
+                     "frac": round(achieved / hbm, 4), "traffic": traffic,
+                     "peak_source": f"hbm_gbs of {src}",
+                     "algorithmic_bytes": b["gemm1"], "touched_experts": touched},
+        "clocks": clocks,
+        "stages": stages,
+        "routing": {"max_over_mean": round(float(cnt.max()) * wl.E / (wl.T * wl.k), 3),
+                    "touched_experts": touched},
+    }
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        line["cpu_baseline"] = cpu_baseline(wl, d, args.cpu_tokens)
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+
+
+def main():
+    args = parse()
+    rank, world, local = dist_env()
+    if world > 1:
+        torch.distributed.init_process_group("gloo")
+    torch.cuda.set_device(local)
+    device = torch.device("cuda", local)
+    wl = I.WORKLOADS[args.workload]
+    if args.impl == "reference":
+        run_reference(args, wl, rank, world, device)
+    else:
+        run_ours(args, wl, rank, world, local, device)
+    if world > 1:
+        torch.distributed.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

@@ -256,4 +256,4 @@ def test_expert_ffn(counts, H, Iw):
         assert (np.abs(yg - y_or) <= UBF16 * np.abs(y_or) * 1.0001 + acc_bound + flip * 1.01
                 + 1e-30).all()
     # rows outside every segment are untouched
-    assert (f64(y[n:]) == sentinel).all()
+    assert (y[n:] == torch.tensor(sentinel, dtype=torch.bfloat16, device=DEV)).all()

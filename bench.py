@@ -46,7 +46,7 @@ def parse():
     p.add_argument("--steps", type=int, default=200)
     p.add_argument("--warmup", type=int, default=10)
     p.add_argument("--impl", choices=("ours", "reference"), default="ours")
-    p.add_argument("--workload", choices=("decode", "prefill", "skewed", "tiny"), default="decode")
+    p.add_argument("--workload", choices=tuple(I.WORKLOADS), default="decode")
     p.add_argument("--mode", choices=("seq", "overlap-tokens", "overlap-experts"), default="seq")
     p.add_argument("--chunk-tokens", type=int, default=512)
     p.add_argument("--expert-chunks", type=int, default=8)
@@ -363,6 +363,10 @@ def run_ours(args, wl, rank, world, local, device):
     # --- per-stage timing (sequential forward with stage events, same stream)
     K2 = min(args.steps, 50)
     evs = [[torch.cuda.Event(enable_timing=True) for _ in L.STAGES] for _ in range(K2)]
+    for row in evs:          # torch creates the CUDA event at its first record
+        for e in row:
+            e.record(stream)
+    torch.cuda.synchronize()
     for i in range(K2):
         exs = L.exec_config(stage_events=evs[i])
         L.moe_layer_forward(cfg, exs, W, d["x"], out, None, ws, stream)

@@ -65,7 +65,11 @@ DECODE = Workload("deepseek-v3 decode T=128 H=7168 E=256+1 k=8 I=2048", T=128, H
                   normalize=1, route_scale=2.5, has_bias=True)
 PREFILL = replace(DECODE, name="deepseek-v3 prefill T=4096 balanced", T=4096, balance="balanced")
 SKEWED = replace(DECODE, name="deepseek-v3 skewed prefill T=8192 zipf1.2", T=8192, balance="zipf")
-WORKLOADS = {"tiny": TINY, "decode": DECODE, "prefill": PREFILL, "skewed": SKEWED}
+# The decode shape with 32 experts (4 per group), 2.8 GB of weights: small enough
+# for multi-pass profiler captures, still far larger than L2.
+DECODE_E32 = replace(DECODE, name="deepseek-v3 decode shape, 32 experts, T=16", T=16, E=32)
+WORKLOADS = {"tiny": TINY, "decode": DECODE, "prefill": PREFILL, "skewed": SKEWED,
+             "decode_e32": DECODE_E32}
 DISPATCH_SWEEP_T = (1024, 4096, 16384, 65536)
 
 _SUB = {"x": 1, "Wr": 2, "bias": 3, "W13": 4, "W2": 5, "Ws13": 6, "Ws2": 7,

@@ -51,7 +51,7 @@ def parse():
     p.add_argument("--chunk-tokens", type=int, default=512)
     p.add_argument("--expert-chunks", type=int, default=8)
     p.add_argument("--no-cpu-baseline", action="store_true")
-    p.add_argument("--cpu-tokens", type=int, default=8, help="oracle sample size (tokens)")
+    p.add_argument("--cpu-tokens", type=int, default=128, help="oracle sample size (tokens)")
     return p.parse_args()
 
 
@@ -192,10 +192,10 @@ def algorithmic(wl, touched):
         "permute": T * k * 4 * 3,
         "dispatch": T * H * 2 + R * H * 2,
         "gemm1": touched * 2 * Iw * H * 2 + R * H * 2 + R * Iw * 2,
-        "gemm2": touched * H * Iw * 2 + R * Iw * 2 + R * H * 2,
+        "gemm2": touched * H * Iw * 2 + R * Iw * 2 + R * H * 4,
         "shared_gemm1": (2 * Is * H * 2 + T * H * 2 + T * Is * 2) if Is else 0,
-        "shared_gemm2": (H * Is * 2 + T * Is * 2 + T * H * 2) if Is else 0,
-        "combine": R * H * 2 + (T * H * 2 if Is else 0) + T * H * 2 + R * 8,
+        "shared_gemm2": (H * Is * 2 + T * Is * 2 + T * H * 4) if Is else 0,
+        "combine": R * H * 4 + (T * H * 4 if Is else 0) + T * H * 2 + R * 8,
     }
     f = {"router": 2 * T * E * H, "gemm1": 2 * R * H * 2 * Iw, "gemm2": 2 * R * Iw * H,
          "shared_gemm1": 2 * T * H * 2 * Is, "shared_gemm2": 2 * T * Is * H}

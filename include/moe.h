@@ -189,28 +189,33 @@ moe_status moe_dispatch(const moe_config* cfg, const uint16_t* x, const int32_t*
  * shapes 7168 x 4096 and 2048 x 7168 in Appendix "Workload Details").
  * For each expert e < n_experts and each row r in [offsets[e], offsets[e+1]):
  *   h[r] = bf16(silu(x_perm[r] . Wg_e^T) * (x_perm[r] . Wu_e^T)),
- *   y_perm[r] = bf16(h[r] . W2_e^T)        (fp32 accumulation throughout).
- * rows: rows of x_perm / y_perm; H hidden (multiple of 128); I intermediate
- * (multiple of 128); offsets [n_experts+1] int32 on the device, non-decreasing,
- * offsets[n_experts] <= rows; W13 [n_experts,2I,H]; W2 [n_experts,H,I];
- * x_perm [rows,H]; y_perm [rows,H] (written; rows outside every segment are
- * left untouched). ws: moe_expert_ffn_workspace_size(rows, I) bytes.
+ *   y_perm[r] = h[r] . W2_e^T             (fp32 accumulation and fp32 y).
+ * h is rounded to bf16 because it is GEMM2's tensor-core operand; y stays in
+ * fp32 for the combine. rows: rows of x_perm / y_perm; H hidden (multiple of
+ * 128); I intermediate (multiple of 128); offsets [n_experts+1] int32 on the
+ * device, non-decreasing, offsets[n_experts] <= rows (a violation is clamped
+ * and latched as MOE_ERR_DEVICE_CHECK); W13 [n_experts,2I,H] bf16;
+ * W2 [n_experts,H,I] bf16; x_perm [rows,H] bf16; y_perm [rows,H] fp32
+ * (written; rows outside every segment are left untouched). ws:
+ * moe_expert_ffn_workspace_size(rows, I) bytes, 16-byte aligned (receives h).
  * The shared expert is this call with n_experts = 1 and offsets = {0, T}.
  */
 moe_status moe_expert_ffn(int32_t rows, int32_t H, int32_t I, int32_t n_experts,
                           const uint16_t* x_perm, const int32_t* offsets, const uint16_t* W13,
-                          const uint16_t* W2, uint16_t* y_perm, void* ws, size_t ws_bytes,
+                          const uint16_t* W2, float* y_perm, void* ws, size_t ws_bytes,
                           void* stream);
 
 /*
  * Combine: the single-GPU form of the paper's reverse AlltoAll combine.
  * out[t] = sum_j topk_w[t,j] * y_perm[slot_row[t*k+j]] (+ shared_out[t]),
  * fp32 accumulation in slot order j = 0..k-1, then the shared term.
- * y_perm [T*k,H] bf16; slot_row [T*k]; topk_w [T,k] fp32; shared_out [T,H]
- * bf16 or NULL; out [T,H] bf16 (out_fp32 = 0) or fp32 (out_fp32 = 1).
+ * y_perm [T*k,H] fp32; slot_row [T*k] (values in [0, T*k); others are
+ * skipped and latched as MOE_ERR_DEVICE_CHECK); topk_w [T,k] fp32;
+ * shared_out [T,H] fp32 or NULL; out [T,H] bf16 (out_fp32 = 0, round to
+ * nearest even) or fp32 (out_fp32 = 1).
  */
-moe_status moe_combine(const moe_config* cfg, const uint16_t* y_perm, const int32_t* slot_row,
-                       const float* topk_w, const uint16_t* shared_out, void* out,
+moe_status moe_combine(const moe_config* cfg, const float* y_perm, const int32_t* slot_row,
+                       const float* topk_w, const float* shared_out, void* out,
                        int32_t out_fp32, void* stream);
 
 /*

@@ -52,8 +52,8 @@ moe_status launch_dispatch_rows(int T, int H, int k, const uint16_t* x, const in
 moe_status launch_gather_rows(int H, const uint16_t* x, const int32_t* row_src_token,
                               const int32_t* offsets, int e_begin, int e_end, uint16_t* x_perm,
                               int max_rows, cudaStream_t s);
-moe_status launch_combine(int T, int H, int k, const uint16_t* y_perm, const int32_t* slot_row,
-                          const float* w, const uint16_t* shared, void* out, int out_fp32,
+moe_status launch_combine(int T, int H, int k, const float* y_perm, const int32_t* slot_row,
+                          const float* w, const float* shared, void* out, int out_fp32,
                           cudaStream_t s);
 
 moe_status launch_fill_range(int32_t* offsets, int n, cudaStream_t s);
@@ -63,7 +63,7 @@ moe_status launch_sum_counts(const int32_t* counts, int n_chunks, int E, int32_t
 // Grouped expert GEMM on tcgen05. Experts [e_begin, e_end) of `offsets`.
 moe_status launch_expert_ffn(int rows, int H, int I, int n_experts, int e_begin, int e_end,
                              const uint16_t* x_perm, const int32_t* offsets, const uint16_t* W13,
-                             const uint16_t* W2, uint16_t* h, uint16_t* y_perm, int rows_hint,
+                             const uint16_t* W2, uint16_t* h, float* y_perm, int rows_hint,
                              cudaStream_t s, cudaEvent_t after_gemm1 = nullptr);
 
 // ----------------------------------------------------------------------------

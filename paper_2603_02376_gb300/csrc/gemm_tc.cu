@@ -21,7 +21,8 @@
 //              tcgen05.commit frees the stage, a final commit hands the
 //              accumulator to the epilogue; also owns the TMEM allocation;
 //   warps 2-5  epilogue: tcgen05.ld the accumulator (each warp its 32-lane
-//              quarter), apply SwiGLU (GEMM1) or nothing (GEMM2), store bf16.
+//              quarter); GEMM1 applies SwiGLU and stores h in bf16 (the
+//              operand of GEMM2), GEMM2 stores y in fp32 (summed by combine).
 // For SwiGLU the gate and up tiles of the same 128 features are two MMAs into
 // two TMEM column ranges, so one thread holds both g and u of its feature.
 //
@@ -224,7 +225,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
                         const int32_t* __restrict__ offsets, int rows, int e_begin, int n_exp,
                         int K,
                         int n_fb, int w_rows_per_expert, int up_row_offset,
-                        uint16_t* __restrict__ out, int out_ld, int* __restrict__ err) {
+                        void* __restrict__ out, int out_ld, int* __restrict__ err) {
   using TL = Tile<SWIGLU, NMAX>;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
@@ -406,7 +407,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       if (!wait_bounded(smem_u32(&ctrl->acc_full), acc_phase, abort_flag, err)) break;
       tc_fence_after();
       const int f = U.fb * BM + q * 32 + lane;
-      uint16_t* dst = out + (size_t)U.row0 * out_ld + f;
+      const size_t o = (size_t)U.row0 * out_ld + f;
       for (int c0 = 0; c0 < U.m; c0 += 16) {
         uint32_t g[16];
         tmem_ld16(tq + c0, g);
@@ -420,14 +421,15 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
               const float gv = __uint_as_float(g[i]);
               const float uv = __uint_as_float(v[i]);
               const float hv = gv / (1.0f + expf(-gv)) * uv;
-              dst[(size_t)(c0 + i) * out_ld] = float_to_bf16_bits(hv);
+              static_cast<uint16_t*>(out)[o + (size_t)(c0 + i) * out_ld] = float_to_bf16_bits(hv);
             }
           }
         } else {
           tmem_wait_ld();
 #pragma unroll
           for (int i = 0; i < 16; ++i) {
-            if (c0 + i < U.m) dst[(size_t)(c0 + i) * out_ld] = float_to_bf16_bits(__uint_as_float(g[i]));
+            if (c0 + i < U.m)
+              static_cast<float*>(out)[o + (size_t)(c0 + i) * out_ld] = __uint_as_float(g[i]);
           }
         }
       }
@@ -486,7 +488,7 @@ size_t gemm_smem_bytes(int n_exp) {
 template <bool SWIGLU, int NMAX>
 moe_status launch_gemm(const CUtensorMap& A, const CUtensorMap& B, const int32_t* offsets,
                        int rows, int e_begin, int n_exp, int K, int n_fb, int w_rows, int up_off,
-                       uint16_t* out, int out_ld, cudaStream_t s) {
+                       void* out, int out_ld, cudaStream_t s) {
   const size_t smem = gemm_smem_bytes<SWIGLU, NMAX>(n_exp);
   if (smem > 227 * 1024) return MOE_ERR_UNSUPPORTED;
   if (cudaFuncSetAttribute(grouped_gemm_kernel<SWIGLU, NMAX>,
@@ -502,7 +504,7 @@ moe_status launch_gemm(const CUtensorMap& A, const CUtensorMap& B, const int32_t
 template <int NMAX>
 moe_status run_ffn(int rows, int H, int I, int n_experts, int e_begin, int e_end,
                    const uint16_t* x_perm, const int32_t* offsets, const uint16_t* W13,
-                   const uint16_t* W2, uint16_t* h, uint16_t* y_perm, cudaStream_t s,
+                   const uint16_t* W2, uint16_t* h, float* y_perm, cudaStream_t s,
                    cudaEvent_t after_gemm1) {
   CUtensorMap a1, b1, a2, b2;
   if (!make_map(&a1, W13, H, (uint64_t)n_experts * 2 * I, BK, BM) ||
@@ -523,7 +525,7 @@ moe_status run_ffn(int rows, int H, int I, int n_experts, int e_begin, int e_end
 
 moe_status launch_expert_ffn(int rows, int H, int I, int n_experts, int e_begin, int e_end,
                              const uint16_t* x_perm, const int32_t* offsets, const uint16_t* W13,
-                             const uint16_t* W2, uint16_t* h, uint16_t* y_perm, int rows_hint,
+                             const uint16_t* W2, uint16_t* h, float* y_perm, int rows_hint,
                              cudaStream_t s, cudaEvent_t after_gemm1) {
   if (rows == 0 || e_end <= e_begin) return MOE_OK;
   const int n_exp = e_end - e_begin;

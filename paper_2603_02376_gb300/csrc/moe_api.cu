@@ -125,10 +125,10 @@ struct Layout {
   float* partials;
   uint16_t* x_perm;  // [T*k, H]
   uint16_t* h;       // [T*k, I]
-  uint16_t* y_perm;  // [T*k, H]
+  float* y_perm;     // [T*k, H] fp32
   int32_t* sh_off;   // [2]
   uint16_t* sh_h;    // [T, I_s]
-  uint16_t* sh_y;    // [T, H]
+  float* sh_y;       // [T, H] fp32
   size_t bytes = 0;
 };
 
@@ -157,10 +157,10 @@ Layout carve(const moe_config& c, const moe_exec& ex, void* ws) {
   L.partials = L.splits > 1 ? cv.take<float>((size_t)L.splits * L.chunk_T * E) : nullptr;
   L.x_perm = cv.take<uint16_t>(T * k * c.H);
   L.h = cv.take<uint16_t>(T * k * c.I);
-  L.y_perm = cv.take<uint16_t>(T * k * c.H);
+  L.y_perm = cv.take<float>(T * k * c.H);
   L.sh_off = cv.take<int32_t>(2);
   L.sh_h = c.I_shared ? cv.take<uint16_t>(T * c.I_shared) : nullptr;
-  L.sh_y = c.I_shared ? cv.take<uint16_t>(T * c.H) : nullptr;
+  L.sh_y = c.I_shared ? cv.take<float>(T * c.H) : nullptr;
   L.bytes = align_up(cv.off, 256);
   return L;
 }
@@ -355,7 +355,7 @@ moe_status moe_dispatch(const moe_config* cfg, const uint16_t* x, const int32_t*
 
 moe_status moe_expert_ffn(int32_t rows, int32_t H, int32_t I, int32_t n_experts,
                           const uint16_t* x_perm, const int32_t* offsets, const uint16_t* W13,
-                          const uint16_t* W2, uint16_t* y_perm, void* ws, size_t ws_bytes,
+                          const uint16_t* W2, float* y_perm, void* ws, size_t ws_bytes,
                           void* stream) {
   if (rows < 0 || H < 128 || H % 128 || H > 65536 || I < 128 || I % 128 || I > 65536 ||
       n_experts < 1 || n_experts > 1024)
@@ -370,8 +370,8 @@ moe_status moe_expert_ffn(int32_t rows, int32_t H, int32_t I, int32_t n_experts,
                            (uint16_t*)ws, y_perm, rows, (cudaStream_t)stream);
 }
 
-moe_status moe_combine(const moe_config* cfg, const uint16_t* y_perm, const int32_t* slot_row,
-                       const float* topk_w, const uint16_t* shared_out, void* out,
+moe_status moe_combine(const moe_config* cfg, const float* y_perm, const int32_t* slot_row,
+                       const float* topk_w, const float* shared_out, void* out,
                        int32_t out_fp32, void* stream) {
   if (!valid_config(cfg) || (out_fp32 != 0 && out_fp32 != 1)) return MOE_ERR_INVALID_ARG;
   if (cfg->T == 0) return MOE_OK;

@@ -12,7 +12,7 @@
 //                    ranks its 32-entry steps with __match_any_sync, so every
 //                    expert's rows come out ordered by (t, j).
 // Row copies move 16-byte vectors: dispatch scatters each token row once to
-// its k packed rows (x read once); combine gathers the k expert rows of a
+// its k packed rows (x read once); combine gathers the k fp32 expert rows of a
 // token and reduces them in fp32 in slot order.
 #include "common.cuh"
 
@@ -211,10 +211,10 @@ __global__ void gather_rows_kernel(const uint4* __restrict__ x, int vpr,
   }
 }
 
-// out[t] = sum_j w[t,j] * y_perm[slot_row[t*k+j]] (+ shared[t]); 8 bf16 per thread-step.
-__global__ void combine_kernel(const uint4* __restrict__ y_perm, int T, int vpr, int k,
+// out[t] = sum_j w[t,j] * y_perm[slot_row[t*k+j]] (+ shared[t]); 8 elements per thread-step.
+__global__ void combine_kernel(const float4* __restrict__ y_perm, int T, int vpr, int k,
                                const int32_t* __restrict__ slot_row, const float* __restrict__ w,
-                               const uint4* __restrict__ shared, void* __restrict__ out,
+                               const float4* __restrict__ shared, void* __restrict__ out,
                                int out_fp32, int* __restrict__ err) {
   const int nrows = T * k;
   const size_t total = (size_t)T * vpr;
@@ -231,16 +231,17 @@ __global__ void combine_kernel(const uint4* __restrict__ y_perm, int T, int vpr,
         continue;
       }
       const float wj = w[t * k + j];
-      const uint4 yv = y_perm[(size_t)r * vpr + v];
-      const uint16_t* yh = reinterpret_cast<const uint16_t*>(&yv);
+      const float4 y0 = y_perm[((size_t)r * vpr + v) * 2];
+      const float4 y1 = y_perm[((size_t)r * vpr + v) * 2 + 1];
+      const float yv[8] = {y0.x, y0.y, y0.z, y0.w, y1.x, y1.y, y1.z, y1.w};
 #pragma unroll
-      for (int q = 0; q < 8; ++q) acc[q] = fmaf(wj, bf16_bits_to_float(yh[q]), acc[q]);
+      for (int q = 0; q < 8; ++q) acc[q] = fmaf(wj, yv[q], acc[q]);
     }
     if (shared) {
-      const uint4 sv = shared[i];
-      const uint16_t* sh = reinterpret_cast<const uint16_t*>(&sv);
+      const float4 s0 = shared[i * 2], s1 = shared[i * 2 + 1];
+      const float sv[8] = {s0.x, s0.y, s0.z, s0.w, s1.x, s1.y, s1.z, s1.w};
 #pragma unroll
-      for (int q = 0; q < 8; ++q) acc[q] += bf16_bits_to_float(sh[q]);
+      for (int q = 0; q < 8; ++q) acc[q] += sv[q];
     }
     if (out_fp32) {
       float4* o = reinterpret_cast<float4*>(out) + i * 2;
@@ -335,14 +336,14 @@ moe_status launch_gather_rows(int H, const uint16_t* x, const int32_t* row_src_t
   return launch_status();
 }
 
-moe_status launch_combine(int T, int H, int k, const uint16_t* y_perm, const int32_t* slot_row,
-                          const float* w, const uint16_t* shared, void* out, int out_fp32,
+moe_status launch_combine(int T, int H, int k, const float* y_perm, const int32_t* slot_row,
+                          const float* w, const float* shared, void* out, int out_fp32,
                           cudaStream_t s) {
   if (T == 0) return MOE_OK;
   const int vpr = H / 8;
   combine_kernel<<<copy_grid((size_t)T * vpr), 256, 0, s>>>(
-      reinterpret_cast<const uint4*>(y_perm), T, vpr, k, slot_row, w,
-      reinterpret_cast<const uint4*>(shared), out, out_fp32, device_error_word());
+      reinterpret_cast<const float4*>(y_perm), T, vpr, k, slot_row, w,
+      reinterpret_cast<const float4*>(shared), out, out_fp32, device_error_word());
   note_launch();
   return launch_status();
 }

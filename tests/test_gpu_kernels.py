@@ -4,8 +4,8 @@ Routing indices, counts, offsets and the permutation are compared bit for
 bit; floating-point outputs within bounds derived from their arithmetic:
 fp32 logits within the worst-case summation bound H*u*sum|x*Wr|; the
 SwiGLU activations h equal the oracle's bf16-rounded h except for rare
-one-ulp flips; GEMM outputs within bf16 rounding (2^-8 relative) of the fp64
-result; combine within (k+1) fp32 roundings (+ bf16 output rounding).
+one-ulp flips; fp32 GEMM2 outputs within the fp32 summation bound of the
+fp64 result; combine within (k+1) fp32 roundings (+ bf16 output rounding).
 """
 
 import numpy as np
@@ -153,10 +153,10 @@ def test_combine(T, H, k, E, shared, out_fp32):
     idx_h = routing(T, E, k, 11 * T + k)
     _, _, _, slot_h = O.permutation(idx_h, E)
     c = L.config(T, H, E, k, 128)
-    y = rand_bf16((T * k, H), 6)
+    y = rand_bf16((T * k, H), 6).float() * 1.37
     rng = np.random.default_rng(3)
     w_h = rng.uniform(0, 1, (T, k)).astype(np.float32)
-    sh = rand_bf16((T, H), 7) if shared else None
+    sh = rand_bf16((T, H), 7).float() * 0.71 if shared else None
     out = torch.empty((T, H), dtype=torch.float32 if out_fp32 else torch.bfloat16, device=DEV)
     L.moe_combine(c, y, torch.from_numpy(slot_h).to(DEV), torch.from_numpy(w_h).to(DEV), sh, out,
                   out_fp32)
@@ -184,15 +184,16 @@ def test_dispatch_identity_combine_roundtrip():
     ws = torch.empty(L.moe_dispatch_workspace_size(c), dtype=torch.uint8, device=DEV)
     L.moe_dispatch(c, x, idx, counts, offsets, rst, slot, xp, ws)
     w = torch.full((T, k), 1.0 / k, device=DEV)
+    yp = xp.float()   # identity experts: y = x_perm (fp32 expert outputs)
     out = torch.empty((T, H), dtype=torch.float32, device=DEV)
-    L.moe_combine(c, xp, slot, w, None, out, 1)
+    L.moe_combine(c, yp, slot, w, None, out, 1)
     outb = torch.empty((T, H), dtype=torch.bfloat16, device=DEV)
-    L.moe_combine(c, xp, slot, w, None, outb, 0)
+    L.moe_combine(c, yp, slot, w, None, outb, 0)
     torch.cuda.synchronize()
     assert torch.equal(out, x.float())
     assert torch.equal(outb, x)
     w1 = torch.ones((T, k), device=DEV)
-    L.moe_combine(c, xp, slot, w1, None, out, 1)
+    L.moe_combine(c, yp, slot, w1, None, out, 1)
     torch.cuda.synchronize()
     assert torch.equal(out, x.float() * k)
 
@@ -222,7 +223,7 @@ def test_expert_ffn(counts, H, Iw):
     rows, offs, xp, W13, W2 = ffn_case(counts, H, Iw, seed=len(counts) + H)
     E = len(counts)
     sentinel = -12345.0
-    y = torch.full((rows, H), sentinel, dtype=torch.bfloat16, device=DEV)
+    y = torch.full((rows, H), sentinel, dtype=torch.float32, device=DEV)
     ws = torch.zeros(L.moe_expert_ffn_workspace_size(rows, Iw), dtype=torch.uint8, device=DEV)
     L.moe_expert_ffn(rows, H, Iw, E, xp, torch.from_numpy(offs).to(DEV), W13, W2, y, ws)
     L.moe_check_errors()
@@ -251,17 +252,15 @@ def test_expert_ffn(counts, H, Iw):
                                               + dsilu * dg * du) * (1 + 2.0 ** -7)) * 1.0001
         assert (diff <= lim + 1e-30).all(), f"expert {e}: h outside one ulp + fp32 bound"
         assert (diff == 0).mean() > 0.98, f"expert {e}: too many h rounding flips"
-        # GEMM2 given the GPU's own h: bf16 rounding of y plus the fp32 summation bound
+        # GEMM2 given the GPU's own h: fp32 output, within the fp32 summation bound
         y_ref = hg @ We2.T
         acc_bound = Iw * 2.0 ** -24 * (np.abs(hg) @ np.abs(We2).T)
         yg = f64(y[a:b])
         err = np.abs(yg - y_ref)
-        assert (err <= UBF16 * np.abs(y_ref) * 1.0001 + acc_bound + 1e-30).all(), \
-            f"expert {e}: max err {err.max():.3e}"
+        assert (err <= acc_bound + 1e-30).all(), f"expert {e}: max err {err.max():.3e}"
         # end to end against the oracle's own h: the h flips above are the only extra term
         y_or = h_ref @ We2.T
         flip = np.abs(hg - h_ref) @ np.abs(We2).T
-        assert (np.abs(yg - y_or) <= UBF16 * np.abs(y_or) * 1.0001 + acc_bound + flip * 1.01
-                + 1e-30).all()
+        assert (np.abs(yg - y_or) <= acc_bound + flip * 1.0001 + 1e-30).all()
     # rows outside every segment are untouched
-    assert (y[n:] == torch.tensor(sentinel, dtype=torch.bfloat16, device=DEV)).all()
+    assert (y[n:] == sentinel).all()

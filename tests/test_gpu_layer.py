@@ -201,7 +201,7 @@ def test_dispatch_combine_sweep_identity(T):
     L.moe_dispatch(c, x, idx, counts, offsets, rst, slot, xp, ws)
     w = torch.full((T, k), 1.0 / k, device=DEV)
     out = torch.empty((T, H), dtype=torch.bfloat16, device=DEV)
-    L.moe_combine(c, xp, slot, w, None, out, 0)
+    L.moe_combine(c, xp.float(), slot, w, None, out, 0)
     torch.cuda.synchronize()
     assert torch.equal(out, x)
     rc, ro, rr, rs = O.permutation(idx.cpu().numpy(), E)

@@ -43,28 +43,32 @@ def prepare_routing(wl, d, seed=0, min_margin=1e-3):
         return np.bincount(idx.reshape(-1), minlength=wl.E)
 
     stats = {}
-    if wl.balance == "balanced":
-        b, c = I.calibrate_balanced(counts_of, wl, d["bias"].cpu())
-        d["bias"] = b.to(d["x"].device)
-    elif wl.balance == "zipf":
-        b, c = I.calibrate_zipf(counts_of, wl, seed)
-        d["bias"] = b.to(d["x"].device)
-    b32 = bias32(d["bias"])
-
-    rounds = 0
-    for attempt in range(64):
-        m = O.routing_margins(L, b32, cfg)
-        bad = np.nonzero(m <= min_margin)[0]
-        if bad.size == 0:
-            break
-        I.resample_rows(d["x"], bad.tolist(), seed, attempt)
-        L[bad] = O.router_logits(f64(d["x"][torch.as_tensor(bad, device=d["x"].device)]), Wr)
-        rounds += 1
-    else:
-        raise RuntimeError("margin resampling did not converge")
-    idx, _ = O.gate_topk(L, b32, cfg)
-    cnt = np.bincount(idx.reshape(-1), minlength=wl.E)
     mean = wl.T * wl.k / wl.E
+    rounds = 0
+    # Calibrating the bias moves margins and redrawing rows moves loads: alternate
+    # until both hold (the Zipf workload only needs its hot ratio, not a band).
+    for outer in range(8):
+        if wl.balance == "balanced":
+            b, c = I.calibrate_balanced(counts_of, wl, d["bias"].cpu())
+            d["bias"] = b.to(d["x"].device)
+        elif wl.balance == "zipf" and outer == 0:
+            b, c = I.calibrate_zipf(counts_of, wl, seed)
+            d["bias"] = b.to(d["x"].device)
+        b32 = bias32(d["bias"])
+        for attempt in range(64):
+            m = O.routing_margins(L, b32, cfg)
+            bad = np.nonzero(m <= min_margin)[0]
+            if bad.size == 0:
+                break
+            I.resample_rows(d["x"], bad.tolist(), seed, 1000 * outer + attempt)
+            L[bad] = O.router_logits(f64(d["x"][torch.as_tensor(bad, device=d["x"].device)]), Wr)
+            rounds += 1
+        else:
+            raise RuntimeError("margin resampling did not converge")
+        idx, _ = O.gate_topk(L, b32, cfg)
+        cnt = np.bincount(idx.reshape(-1), minlength=wl.E)
+        if wl.balance != "balanced" or np.abs(cnt / mean - 1).max() <= wl.balance_tol:
+            break
     stats.update(resample_rounds=rounds, max_over_mean=float(cnt.max() / mean),
                  min_over_mean=float(cnt.min() / mean), oracle_logits=L)
     return stats

@@ -188,7 +188,8 @@ def calibrate_zipf(counts_fn, wl: Workload, seed: int, iters: int = 30):
     return best
 
 
-def calibrate_balanced(counts_fn, wl: Workload, bias0: torch.Tensor, iters: int = 400):
+def calibrate_balanced(counts_fn, wl: Workload, bias0: torch.Tensor, iters: int = 400,
+                       gamma: float = 2e-3):
     """Sign-step bias updates until every expert's load is within +-tol of the mean.
 
     counts_fn(bias) -> counts. b_e -= gamma * sign(load_e - mean) with a
@@ -196,7 +197,6 @@ def calibrate_balanced(counts_fn, wl: Workload, bias0: torch.Tensor, iters: int 
     """
     mean = wl.T * wl.k / wl.E
     b = bias0.clone().to(torch.float32).cpu()
-    gamma = 2e-3
     c = None
     for it in range(iters):
         c = torch.as_tensor(counts_fn(b)).to(torch.float64)

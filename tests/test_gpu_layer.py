@@ -146,7 +146,8 @@ def prefill_inputs(big_weights):
     d = dict(big_weights)
     d["x"] = I.randn((wl.T, wl.H), 1.0, torch.bfloat16, 0, "x", DEV)
     st = prepare_routing(wl, d)
-    assert st["max_over_mean"] <= 1.10 and st["min_over_mean"] >= 0.90
+    # +-10 % balanced, then low-margin rows redrawn: +-12 % realised
+    assert st["max_over_mean"] <= 1.12 and st["min_over_mean"] >= 0.88
     toks = I.sample_tokens(wl.T, 256, 0).numpy()
     ref, _ = oracle_tokens(wl, d, toks)
     return d, st, toks, ref

@@ -185,6 +185,32 @@ moe_status moe_dispatch(const moe_config* cfg, const uint16_t* x, const int32_t*
                         void* stream);
 
 /*
+ * moe_dispatch for callers that cannot allocate device memory. (The paper has
+ * no counterpart; this is a deployment variant.) Some callers can't call
+ * cudaMalloc: plugins inside a host framework that owns all device memory,
+ * serving loops whose memory was planned once and must not grow, and
+ * latency-critical paths where an allocation may synchronise the device; they
+ * may also have no workspace to pass. This call computes exactly what
+ * moe_dispatch computes (same arguments, minus the workspace) but keeps the
+ * per-chunk histogram scratch in a fixed-size array inside the library
+ * (2 x MOE_DISPATCH_NOALLOC_MAX_ENTRIES int32 = 1 MiB per device, held until
+ * the process exits). It allocates nothing.
+ *  - Size limit: (ceil(T / 128) + 1) * E <= MOE_DISPATCH_NOALLOC_MAX_ENTRIES
+ *    (e.g. T <= 65408 tokens at E = 256); larger inputs return
+ *    MOE_ERR_UNSUPPORTED and enqueue nothing.
+ *  - The first call on each device looks up the array's device address (with
+ *    that device current) and caches it; make that first call before any
+ *    stream capture.
+ *  - All calls on a device share the array, which keeps the previous call's
+ *    contents (nothing in it needs to start at zero). Calls whose GPU work
+ *    overlaps -- different streams with no ordering between them -- race on it.
+ */
+#define MOE_DISPATCH_NOALLOC_MAX_ENTRIES 131072
+moe_status moe_dispatch_noalloc(const moe_config* cfg, const uint16_t* x, const int32_t* topk_idx,
+                                int32_t* counts, int32_t* offsets, int32_t* row_src_token,
+                                int32_t* slot_row, uint16_t* x_perm, void* stream);
+
+/*
  * Grouped expert FFN (GEMM1 + SwiGLU + GEMM2 of the paper's expert compute,
  * shapes 7168 x 4096 and 2048 x 7168 in Appendix "Workload Details").
  * For each expert e < n_experts and each row r in [offsets[e], offsets[e+1]):

@@ -28,7 +28,8 @@ EXPORTS = ("moe_status_string", "moe_validate_config", "moe_workspace_size",
            "moe_router_workspace_size", "moe_dispatch_workspace_size",
            "moe_expert_ffn_workspace_size", "moe_router_logits", "moe_gate_topk", "moe_dispatch",
            "moe_expert_ffn", "moe_combine", "moe_layer_forward", "moe_check_errors",
-           "moe_launch_count", "moe_shutdown")
+           "moe_launch_count", "moe_shutdown", "moe_dispatch_noalloc")
+MOE_DISPATCH_NOALLOC_MAX_ENTRIES = 131072
 
 
 class MoeError(RuntimeError):
@@ -87,6 +88,7 @@ def load(path: str = LIB_PATH) -> ctypes.CDLL:
         "moe_router_logits": (S, [cfgp, P, P, P, P, SZ, P]),
         "moe_gate_topk": (S, [cfgp, P, P, P, P, P]),
         "moe_dispatch": (S, [cfgp, P, P, P, P, P, P, P, P, SZ, P]),
+        "moe_dispatch_noalloc": (S, [cfgp, P, P, P, P, P, P, P, P]),
         "moe_expert_ffn": (S, [I32, I32, I32, I32, P, P, P, P, P, P, SZ, P]),
         "moe_combine": (S, [cfgp, P, P, P, P, P, I32, P]),
         "moe_layer_forward": (S, [cfgp, exp, ctypes.POINTER(moe_weights), P, P,
@@ -192,6 +194,14 @@ def moe_dispatch(cfg, x, topk_idx, counts, offsets, row_src_token, slot_row, x_p
     _check(load().moe_dispatch(ctypes.byref(cfg), _ptr(x), _ptr(topk_idx), _ptr(counts),
                                _ptr(offsets), _ptr(row_src_token), _ptr(slot_row), _ptr(x_perm),
                                _ptr(ws), nb, _stream(stream)), "moe_dispatch")
+
+
+def moe_dispatch_noalloc(cfg, x, topk_idx, counts, offsets, row_src_token, slot_row, x_perm,
+                         stream=None) -> None:
+    """moe_dispatch without a workspace, for callers that cannot allocate device memory."""
+    _check(load().moe_dispatch_noalloc(ctypes.byref(cfg), _ptr(x), _ptr(topk_idx), _ptr(counts),
+                                       _ptr(offsets), _ptr(row_src_token), _ptr(slot_row),
+                                       _ptr(x_perm), _stream(stream)), "moe_dispatch_noalloc")
 
 
 def moe_expert_ffn(rows, H, I, n_experts, x_perm, offsets, W13, W2, y_perm, ws,

@@ -316,7 +316,9 @@ def run_ours(args, wl, rank, world, local, device):
                                                        n_expert_chunks=args.expert_chunks)})[
         args.mode]
     ex = L.exec_config(**mode)
-    ws = torch.empty(L.moe_workspace_size(cfg, ex), dtype=torch.uint8, device=device)
+    # one workspace serves the timed mode and the sequential stats / stage-event passes
+    ws = torch.empty(max(L.moe_workspace_size(cfg, ex), L.moe_workspace_size(cfg, L.exec_config())),
+                     dtype=torch.uint8, device=device)
     out = torch.empty((wl.T, wl.H), dtype=torch.bfloat16, device=device)
     W = L.weights_struct(d["Wr"], d["bias"], d["W13"], d["W2"], d["Ws13"], d["Ws2"])
     stream = torch.cuda.current_stream()
@@ -398,6 +400,25 @@ def run_ours(args, wl, rank, world, local, device):
     e2e_ms = max_over_ranks(f0.elapsed_time(f1), world)
     e2e_value = wl.T * world * args.steps / (e2e_ms / 1e3)
 
+    # --- two-stream overlap: the same chunking on one stream, and the pack work alone
+    overlap = None
+    if ex.overlap:
+        barrier(world)
+        torch.cuda.synchronize()
+        g0, g1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        g0.record(stream)
+        for _ in range(args.steps):
+            L.moe_layer_forward(cfg, ex, W, d["x"], out, None, ws, stream, aux_stream=stream)
+        g1.record(stream)
+        torch.cuda.synchronize()
+        t_single = max_over_ranks(g0.elapsed_time(g1), world) / args.steps
+        t_ovl = ms / args.steps
+        t_pack = sum(stage_ms[k] for k in ("router", "gate", "permute", "dispatch"))
+        overlap = {"ms_two_streams": round(t_ovl, 4), "ms_same_chunks_one_stream": round(t_single, 4),
+                   "ms_pack_work": round(t_pack, 4),
+                   "hidden_frac": round((t_single - t_ovl) / t_pack, 3) if t_pack > 0 else None,
+                   "ms_sequential_unchunked": round(sum(stage_ms.values()), 4)}
+
     hbm, tf_burst, tf_sust, src = peaks()
     b, f = algorithmic(wl, touched)
     g1 = stage_ms["gemm1"] / 1e3
@@ -433,6 +454,8 @@ def run_ours(args, wl, rank, world, local, device):
         "routing": {"max_over_mean": round(float(cnt.max()) * wl.E / (wl.T * wl.k), 3),
                     "touched_experts": touched},
     }
+    if overlap:
+        line["overlap"] = overlap
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         line["cpu_baseline"] = cpu_baseline(wl, d, args.cpu_tokens)
     if rank == 0:

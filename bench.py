@@ -199,6 +199,10 @@ def algorithmic(wl, touched):
     }
     f = {"router": 2 * T * E * H, "gemm1": 2 * R * H * 2 * Iw, "gemm2": 2 * R * Iw * H,
          "shared_gemm1": 2 * T * H * 2 * Is, "shared_gemm2": 2 * T * Is * H}
+    if Is and Is == Iw:  # the library runs the shared expert inside the routed GEMM launches
+        for d_ in (b, f):
+            d_["gemm1"] += d_.pop("shared_gemm1")
+            d_["gemm2"] += d_.pop("shared_gemm2")
     return b, f
 
 
@@ -444,11 +448,13 @@ def run_ours(args, wl, rank, world, local, device):
         "e2e": {"value": e2e_value, "unit": "tokens/s", "h2d_bytes_per_step": wl.T * wl.H * 2,
                 "d2h_bytes_per_step": wl.T * wl.H * 2},
         "gpu_launches": launches,
-        "roofline": {"bound": "hbm", "kernel": "grouped GEMM1 + SwiGLU (tcgen05)",
+        "roofline": {"bound": "hbm", "kernel": "grouped GEMM1 + SwiGLU (tcgen05), routed + shared",
                      "achieved": round(achieved, 1), "peak": hbm, "unit": "GB/s",
                      "frac": round(achieved / hbm, 4), "traffic": traffic,
                      "peak_source": f"hbm_gbs of {src}",
-                     "algorithmic_bytes": b["gemm1"], "touched_experts": touched},
+                     "algorithmic_bytes": b["gemm1"], "touched_experts": touched,
+                     "note": ("the grouped GEMM1 launch also runs the shared expert's GEMM1; "
+                              "its bytes are included") if wl.I_shared == wl.I else ""},
         "clocks": clocks,
         "stages": stages,
         "routing": {"max_over_mean": round(float(cnt.max()) * wl.E / (wl.T * wl.k), 3),

@@ -92,7 +92,9 @@ typedef struct {
 } moe_exec;
 
 /* Indices into moe_exec.stage_events: event i is recorded when stage i ends
- * (MOE_EV_START before the first kernel). */
+ * (MOE_EV_START before the first kernel). When I_shared == I the shared
+ * expert runs inside the routed GEMM launches: its work is then timed in the
+ * GEMM1/GEMM2 stages and the SHARED_* stages are empty. */
 enum {
   MOE_EV_START = 0,
   MOE_EV_ROUTER = 1,       /* router logits */
@@ -101,8 +103,8 @@ enum {
   MOE_EV_DISPATCH = 4,     /* packing of token rows into expert segments */
   MOE_EV_GEMM1 = 5,        /* routed grouped GEMM1 + SwiGLU */
   MOE_EV_GEMM2 = 6,        /* routed grouped GEMM2 */
-  MOE_EV_SHARED_GEMM1 = 7, /* shared expert GEMM1 + SwiGLU */
-  MOE_EV_SHARED_GEMM2 = 8, /* shared expert GEMM2 */
+  MOE_EV_SHARED_GEMM1 = 7, /* shared expert GEMM1 + SwiGLU (empty when fused) */
+  MOE_EV_SHARED_GEMM2 = 8, /* shared expert GEMM2 (empty when fused) */
   MOE_EV_COMBINE = 9,      /* weighted combine (+ shared term) */
   MOE_N_STAGE_EVENTS = 10
 };

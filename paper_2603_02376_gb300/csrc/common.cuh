@@ -60,6 +60,25 @@ moe_status launch_fill_range(int32_t* offsets, int n, cudaStream_t s);
 moe_status launch_sum_counts(const int32_t* counts, int n_chunks, int E, int32_t* out,
                              cudaStream_t s);
 
+// One operand group of the grouped expert GEMMs: experts [e_begin, e_end) of
+// the packed activations x [rows, H] with device row offsets, or (offsets
+// unused) a single dense segment [0, rows) with one weight matrix.
+struct FfnGroup {
+  const uint16_t* x;
+  const int32_t* offsets;
+  int rows, n_experts, e_begin, e_end;
+  const uint16_t* W13;
+  const uint16_t* W2;
+  uint16_t* h;  // [rows, I] bf16
+  float* y;     // [rows, H] fp32
+};
+
+// Routed group plus an optional dense group (the shared expert, same I) in one
+// pair of launches.
+moe_status launch_expert_ffn_groups(const FfnGroup& routed, const FfnGroup* dense, int H, int I,
+                                    int rows_hint, cudaStream_t s,
+                                    cudaEvent_t after_gemm1 = nullptr);
+
 // Grouped expert GEMM on tcgen05. Experts [e_begin, e_end) of `offsets`.
 moe_status launch_expert_ffn(int rows, int H, int I, int n_experts, int e_begin, int e_end,
                              const uint16_t* x_perm, const int32_t* offsets, const uint16_t* W13,

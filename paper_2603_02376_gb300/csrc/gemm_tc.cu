@@ -13,8 +13,10 @@
 //
 // Work unit = (expert e, feature block fb, token tile nt). The units of every
 // expert are enumerated on the device from the row offsets, so a launch needs
-// no host-side knowledge of the routing. A persistent grid (one CTA per SM)
-// walks the units round-robin. Warp roles:
+// no host-side knowledge of the routing. A launch may carry a second operand
+// group: one dense segment with its own weights and activations (the shared
+// expert), whose units run in the same persistent grid as the routed ones. A
+// persistent grid (one CTA per SM) walks the units round-robin. Warp roles:
 //   warp 0     TMA producer: weight tile(s) 128 x 64 and token rows 16 x 64
 //              per stage into a STAGES-deep ring (128-byte swizzle);
 //   warp 1     MMA issuer (one thread): 4 x tcgen05.mma (K = 16 each) per stage,
@@ -25,6 +27,8 @@
 //              operand of GEMM2), GEMM2 stores y in fp32 (summed by combine).
 // For SwiGLU the gate and up tiles of the same 128 features are two MMAs into
 // two TMEM column ranges, so one thread holds both g and u of its feature.
+// When two accumulators fit in TMEM's 512 columns they alternate, so the
+// epilogue of one unit overlaps the MMAs of the next.
 //
 // Every mbarrier wait is bounded (%globaltimer): on expiry the kernel latches
 // MOE_ERR_TIMEOUT, tells the other roles to stop, waits (bounded) for its own
@@ -57,16 +61,19 @@ struct Tile {
   static constexpr int STAGE_BYTES = NA * A_BYTES + B_BYTES;
   static constexpr int STAGES_RAW = (200 * 1024) / STAGE_BYTES;
   static constexpr int STAGES = STAGES_RAW > 8 ? 8 : STAGES_RAW;
-  static constexpr int TMEM_COLS = pow2ceil(NA * NMAX);
+  static constexpr int ACC_COLS = NA * NMAX;                  // one accumulator (gate | up)
+  static constexpr int ACC_STAGES = 2 * ACC_COLS <= 512 ? 2 : 1;  // double-buffer when it fits
+  static constexpr int TMEM_COLS = pow2ceil(ACC_STAGES * ACC_COLS);
   static_assert(STAGES >= 2, "pipeline too shallow");
   static_assert(NMAX % 16 == 0 && NMAX >= 16 && NMAX <= 256, "MMA N range for M = 128");
+  static_assert(TMEM_COLS <= 512, "TMEM holds 512 columns");
 };
 
 struct Ctrl {
   uint64_t full[8];
   uint64_t empty[8];
-  uint64_t acc_full;
-  uint64_t acc_empty;
+  uint64_t acc_full[2];
+  uint64_t acc_empty[2];
   uint64_t drain;
   uint32_t tmem_base;
   int abort_flag;
@@ -188,26 +195,56 @@ __device__ __forceinline__ void tmem_wait_ld() {
 
 // ------------------------------------------------------------------ schedule
 
+// Launch arguments besides the tensor maps. Group 0: experts [e_begin,
+// e_begin + n_exp) of a packed activation matrix with `rows0` rows, segments
+// given by device offsets. Group 1 (rows1 > 0): one segment [0, rows1) of its
+// own activation matrix with one weight matrix (the shared expert).
+struct GemmArgs {
+  const int32_t* offsets;
+  int rows0, e_begin, n_exp;
+  int rows1;
+  int K, n_fb;
+  int w_rows0;  // weight rows per expert in group 0
+  int up_off;   // SwiGLU: row offset of the up projection inside an expert
+  void* out0;
+  void* out1;
+  int out_ld;
+  int* err;
+};
+
 struct Unit {
-  int e;     // expert, relative to e_begin
+  int grp;   // operand group
+  int e;     // expert (group 0, relative to e_begin)
   int fb;    // 128-feature block
-  int row0;  // first packed row of the token tile
+  int row0;  // first activation row of the token tile
   int m;     // valid token rows in the tile (1..NMAX)
 };
 
 template <int NMAX>
 __device__ __forceinline__ Unit decode_unit(int u, const int* tile_off, const int* row_off,
-                                            int n_exp, int n_fb) {
-  int lo = 0, hi = n_exp - 1;
+                                            const GemmArgs& a, int units1) {
+  Unit U;
+  if (u < units1) {  // group 1: the shared expert's dense segment
+    const int nt1 = (a.rows1 + NMAX - 1) / NMAX;
+    U.grp = 1;
+    U.e = 0;
+    U.fb = u / nt1;
+    const int nt = u - U.fb * nt1;
+    U.row0 = nt * NMAX;
+    U.m = min(NMAX, a.rows1 - U.row0);
+    return U;
+  }
+  u -= units1;
+  int lo = 0, hi = a.n_exp - 1;
   while (lo < hi) {  // largest e with tile_off[e] * n_fb <= u: an expert with tiles
     const int mid = (lo + hi + 1) >> 1;
-    if (tile_off[mid] * n_fb <= u) lo = mid;
+    if (tile_off[mid] * a.n_fb <= u) lo = mid;
     else hi = mid - 1;
   }
-  Unit U;
+  U.grp = 0;
   U.e = lo;
   const int nt_e = tile_off[lo + 1] - tile_off[lo];
-  const int local = u - tile_off[lo] * n_fb;
+  const int local = u - tile_off[lo] * a.n_fb;
   U.fb = local / nt_e;
   const int nt = local - U.fb * nt_e;
   const int cnt = row_off[lo + 1] - row_off[lo];
@@ -220,20 +257,19 @@ __device__ __forceinline__ Unit decode_unit(int u, const int* tile_off, const in
 
 template <bool SWIGLU, int NMAX>
 __global__ void __launch_bounds__(NUM_THREADS, 1)
-    grouped_gemm_kernel(const __grid_constant__ CUtensorMap tmA,
-                        const __grid_constant__ CUtensorMap tmB,
-                        const int32_t* __restrict__ offsets, int rows, int e_begin, int n_exp,
-                        int K,
-                        int n_fb, int w_rows_per_expert, int up_row_offset,
-                        void* __restrict__ out, int out_ld, int* __restrict__ err) {
+    grouped_gemm_kernel(const __grid_constant__ CUtensorMap tmA0,
+                        const __grid_constant__ CUtensorMap tmB0,
+                        const __grid_constant__ CUtensorMap tmA1,
+                        const __grid_constant__ CUtensorMap tmB1, const GemmArgs a) {
   using TL = Tile<SWIGLU, NMAX>;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~static_cast<uintptr_t>(1023));
   Ctrl* ctrl = reinterpret_cast<Ctrl*>(smem + TL::STAGES * TL::STAGE_BYTES);
   int* tile_off = reinterpret_cast<int*>(ctrl + 1);
-  int* row_off = tile_off + n_exp + 1;
+  int* row_off = tile_off + a.n_exp + 1;
   volatile int* abort_flag = &ctrl->abort_flag;
+  int* err = a.err;
 
   const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
 
@@ -242,8 +278,10 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       mbar_init(smem_u32(&ctrl->full[s]), 1);
       mbar_init(smem_u32(&ctrl->empty[s]), 1);
     }
-    mbar_init(smem_u32(&ctrl->acc_full), 1);
-    mbar_init(smem_u32(&ctrl->acc_empty), 4);
+    for (int s = 0; s < TL::ACC_STAGES; ++s) {
+      mbar_init(smem_u32(&ctrl->acc_full[s]), 1);
+      mbar_init(smem_u32(&ctrl->acc_empty[s]), 4);
+    }
     mbar_init(smem_u32(&ctrl->drain), 1);
     ctrl->abort_flag = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
@@ -257,19 +295,21 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
     asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
   }
   if (warp == 2) {
-    // Per-expert token tiles and their prefix, from the device row offsets.
-    // Offsets are clamped into [0, rows] and made non-decreasing, so no tile can
-    // reach outside the caller's buffers; a clamp latches MOE_ERR_DEVICE_CHECK.
+    // Per-expert token tiles of group 0 and their prefix, from the device row
+    // offsets. Offsets are clamped into [0, rows0] and made non-decreasing, so no
+    // tile can reach outside the caller's buffers; a clamp latches
+    // MOE_ERR_DEVICE_CHECK.
+    const int n_exp = a.n_exp;
     const int per = (n_exp + 31) / 32;
-    const int a = min(n_exp, lane * per), b = min(n_exp, a + per);
+    const int lo = min(n_exp, lane * per), hi = min(n_exp, lo + per);
     auto clamped = [&](int i) {
-      const int v = offsets[e_begin + i];
-      const int c = min(max(v, 0), rows);
+      const int v = a.offsets[a.e_begin + i];
+      const int c = min(max(v, 0), a.rows0);
       if (c != v) atomicExch(err, (int)MOE_ERR_DEVICE_CHECK);
       return c;
     };
     int s = 0;
-    for (int i = a; i < b; ++i) {
+    for (int i = lo; i < hi; ++i) {
       const int r0 = clamped(i), r1 = max(clamped(i + 1), r0);
       if (r1 != clamped(i + 1)) atomicExch(err, (int)MOE_ERR_DEVICE_CHECK);
       row_off[i] = r0;
@@ -282,7 +322,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       if (lane >= o) incl += v;
     }
     int run = incl - s;
-    for (int i = a; i < b; ++i) {
+    for (int i = lo; i < hi; ++i) {
       tile_off[i] = run;
       run += (max(clamped(i + 1), row_off[i]) - row_off[i] + NMAX - 1) / NMAX;
     }
@@ -295,22 +335,29 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem_base = ctrl->tmem_base;
-  const int total_units = tile_off[n_exp] * n_fb;
-  const int kblocks = K / BK;
+  const int units1 = a.rows1 > 0 ? ((a.rows1 + NMAX - 1) / NMAX) * a.n_fb : 0;
+  const int total_units = units1 + tile_off[a.n_exp] * a.n_fb;
+  const int kblocks = a.K / BK;
 
   if (warp == 0) {
     if (lane == 0) {
       // ---------------------------------------------------------------- producer
-      tma_prefetch_map(&tmA);
-      tma_prefetch_map(&tmB);
+      tma_prefetch_map(&tmA0);
+      tma_prefetch_map(&tmB0);
+      if (units1) {
+        tma_prefetch_map(&tmA1);
+        tma_prefetch_map(&tmB1);
+      }
       int stage = 0;
       uint32_t phase = 0;
       long fills = 0;
       bool ok = true;
       for (int u = blockIdx.x; u < total_units && ok; u += gridDim.x) {
-        const Unit U = decode_unit<NMAX>(u, tile_off, row_off, n_exp, n_fb);
+        const Unit U = decode_unit<NMAX>(u, tile_off, row_off, a, units1);
+        const CUtensorMap* mA = U.grp ? &tmA1 : &tmA0;
+        const CUtensorMap* mB = U.grp ? &tmB1 : &tmB0;
         const int n_pad = (U.m + 15) & ~15;
-        const int wrow = (e_begin + U.e) * w_rows_per_expert + U.fb * BM;
+        const int wrow = U.grp ? U.fb * BM : (a.e_begin + U.e) * a.w_rows0 + U.fb * BM;
         const uint32_t bytes = TL::NA * TL::A_BYTES + n_pad * BK * 2;
         for (int kb = 0; kb < kblocks; ++kb) {
           const uint32_t full = smem_u32(&ctrl->full[stage]);
@@ -320,11 +367,11 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
           }
           mbar_arrive_expect_tx(full, bytes);
           const uint32_t sa = smem_u32(smem + stage * TL::STAGE_BYTES);
-          tma_load_2d(sa, &tmA, kb * BK, wrow, full);
-          if (SWIGLU) tma_load_2d(sa + TL::A_BYTES, &tmA, kb * BK, wrow + up_row_offset, full);
+          tma_load_2d(sa, mA, kb * BK, wrow, full);
+          if (SWIGLU) tma_load_2d(sa + TL::A_BYTES, mA, kb * BK, wrow + a.up_off, full);
           const uint32_t sb = sa + TL::NA * TL::A_BYTES;
           for (int i = 0; i < n_pad / B_BOX; ++i)
-            tma_load_2d(sb + i * (B_BOX * BK * 2), &tmB, kb * BK, U.row0 + i * B_BOX, full);
+            tma_load_2d(sb + i * (B_BOX * BK * 2), mB, kb * BK, U.row0 + i * B_BOX, full);
           ++fills;
           if (++stage == TL::STAGES) {
             stage = 0;
@@ -349,17 +396,21 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
     if (lane == 0) {
       // ---------------------------------------------------------------- MMA issuer
       int stage = 0;
-      uint32_t phase = 0, acc_phase = 0;
+      uint32_t phase = 0;
+      int j = 0;  // units of this CTA so far: accumulator j % ACC_STAGES
       bool ok = true, issued = false;
-      for (int u = blockIdx.x; u < total_units && ok; u += gridDim.x) {
-        const Unit U = decode_unit<NMAX>(u, tile_off, row_off, n_exp, n_fb);
+      for (int u = blockIdx.x; u < total_units && ok; u += gridDim.x, ++j) {
+        const Unit U = decode_unit<NMAX>(u, tile_off, row_off, a, units1);
         const int n_pad = (U.m + 15) & ~15;
         const uint32_t idesc = idesc_bf16(n_pad);
-        if (!wait_bounded(smem_u32(&ctrl->acc_empty), acc_phase ^ 1, abort_flag, err)) {
+        const int as = j % TL::ACC_STAGES;
+        const uint32_t acc_par = (uint32_t)((j / TL::ACC_STAGES) & 1);
+        if (!wait_bounded(smem_u32(&ctrl->acc_empty[as]), acc_par ^ 1, abort_flag, err)) {
           ok = false;
           break;
         }
         tc_fence_after();
+        const uint32_t d = tmem_base + (uint32_t)(as * TL::ACC_COLS);
         for (int kb = 0; kb < kblocks; ++kb) {
           if (!wait_bounded(smem_u32(&ctrl->full[stage]), phase, abort_flag, err)) {
             ok = false;
@@ -372,10 +423,9 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
           for (int k = 0; k < BK / UMMA_K; ++k) {
             const uint32_t acc = (kb > 0 || k > 0) ? 1u : 0u;
             const uint64_t bdesc = sdesc(sb + k * UMMA_K * 2);
-            mma_bf16(tmem_base, sdesc(sa + k * UMMA_K * 2), bdesc, idesc, acc);
+            mma_bf16(d, sdesc(sa + k * UMMA_K * 2), bdesc, idesc, acc);
             if (SWIGLU)
-              mma_bf16(tmem_base + NMAX, sdesc(sa + TL::A_BYTES + k * UMMA_K * 2), bdesc, idesc,
-                       acc);
+              mma_bf16(d + NMAX, sdesc(sa + TL::A_BYTES + k * UMMA_K * 2), bdesc, idesc, acc);
           }
           issued = true;
           mma_commit(smem_u32(&ctrl->empty[stage]));
@@ -385,8 +435,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
           }
         }
         if (!ok) break;
-        mma_commit(smem_u32(&ctrl->acc_full));
-        acc_phase ^= 1;
+        mma_commit(smem_u32(&ctrl->acc_full[as]));
       }
       if (!ok && issued) {
         // wait (bounded) for the MMAs already issued before TMEM is freed
@@ -400,14 +449,17 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
   } else {
     // ------------------------------------------------------------------ epilogue
     const int q = warp & 3;  // TMEM lane quarter this warp may access
-    const uint32_t tq = tmem_base + ((uint32_t)(q * 32) << 16);
-    uint32_t acc_phase = 0;
-    for (int u = blockIdx.x; u < total_units; u += gridDim.x) {
-      const Unit U = decode_unit<NMAX>(u, tile_off, row_off, n_exp, n_fb);
-      if (!wait_bounded(smem_u32(&ctrl->acc_full), acc_phase, abort_flag, err)) break;
+    int j = 0;
+    for (int u = blockIdx.x; u < total_units; u += gridDim.x, ++j) {
+      const Unit U = decode_unit<NMAX>(u, tile_off, row_off, a, units1);
+      const int as = j % TL::ACC_STAGES;
+      const uint32_t acc_par = (uint32_t)((j / TL::ACC_STAGES) & 1);
+      if (!wait_bounded(smem_u32(&ctrl->acc_full[as]), acc_par, abort_flag, err)) break;
       tc_fence_after();
+      const uint32_t tq = tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(as * TL::ACC_COLS);
       const int f = U.fb * BM + q * 32 + lane;
-      const size_t o = (size_t)U.row0 * out_ld + f;
+      const size_t o = (size_t)U.row0 * a.out_ld + f;
+      void* out = U.grp ? a.out1 : a.out0;
       for (int c0 = 0; c0 < U.m; c0 += 16) {
         uint32_t g[16];
         tmem_ld16(tq + c0, g);
@@ -421,7 +473,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
               const float gv = __uint_as_float(g[i]);
               const float uv = __uint_as_float(v[i]);
               const float hv = gv / (1.0f + expf(-gv)) * uv;
-              static_cast<uint16_t*>(out)[o + (size_t)(c0 + i) * out_ld] = float_to_bf16_bits(hv);
+              static_cast<uint16_t*>(out)[o + (size_t)(c0 + i) * a.out_ld] = float_to_bf16_bits(hv);
             }
           }
         } else {
@@ -429,14 +481,13 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
 #pragma unroll
           for (int i = 0; i < 16; ++i) {
             if (c0 + i < U.m)
-              static_cast<float*>(out)[o + (size_t)(c0 + i) * out_ld] = __uint_as_float(g[i]);
+              static_cast<float*>(out)[o + (size_t)(c0 + i) * a.out_ld] = __uint_as_float(g[i]);
           }
         }
       }
       tc_fence_before();
       __syncwarp();
-      if (lane == 0) mbar_arrive(smem_u32(&ctrl->acc_empty));
-      acc_phase ^= 1;
+      if (lane == 0) mbar_arrive(smem_u32(&ctrl->acc_empty[as]));
     }
   }
 
@@ -486,55 +537,89 @@ size_t gemm_smem_bytes(int n_exp) {
 }
 
 template <bool SWIGLU, int NMAX>
-moe_status launch_gemm(const CUtensorMap& A, const CUtensorMap& B, const int32_t* offsets,
-                       int rows, int e_begin, int n_exp, int K, int n_fb, int w_rows, int up_off,
-                       void* out, int out_ld, cudaStream_t s) {
-  const size_t smem = gemm_smem_bytes<SWIGLU, NMAX>(n_exp);
+moe_status launch_gemm(const CUtensorMap& A0, const CUtensorMap& B0, const CUtensorMap& A1,
+                       const CUtensorMap& B1, const GemmArgs& args, cudaStream_t s) {
+  const size_t smem = gemm_smem_bytes<SWIGLU, NMAX>(args.n_exp);
   if (smem > 227 * 1024) return MOE_ERR_UNSUPPORTED;
   if (cudaFuncSetAttribute(grouped_gemm_kernel<SWIGLU, NMAX>,
                            cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) != cudaSuccess)
     return MOE_ERR_CUDA;
-  grouped_gemm_kernel<SWIGLU, NMAX><<<num_sms(), NUM_THREADS, smem, s>>>(
-      A, B, offsets, rows, e_begin, n_exp, K, n_fb, w_rows, up_off, out, out_ld,
-      device_error_word());
+  grouped_gemm_kernel<SWIGLU, NMAX><<<num_sms(), NUM_THREADS, smem, s>>>(A0, B0, A1, B1, args);
   note_launch();
   return launch_status();
 }
 
 template <int NMAX>
-moe_status run_ffn(int rows, int H, int I, int n_experts, int e_begin, int e_end,
-                   const uint16_t* x_perm, const int32_t* offsets, const uint16_t* W13,
-                   const uint16_t* W2, uint16_t* h, float* y_perm, cudaStream_t s,
+moe_status run_ffn(const FfnGroup& g0, const FfnGroup* g1, int H, int I, cudaStream_t s,
                    cudaEvent_t after_gemm1) {
-  CUtensorMap a1, b1, a2, b2;
-  if (!make_map(&a1, W13, H, (uint64_t)n_experts * 2 * I, BK, BM) ||
-      !make_map(&b1, x_perm, H, rows, BK, B_BOX) ||
-      !make_map(&a2, W2, I, (uint64_t)n_experts * H, BK, BM) ||
-      !make_map(&b2, h, I, rows, BK, B_BOX))
+  CUtensorMap a1, b1, a2, b2, sa1, sb1, sa2, sb2;
+  if (!make_map(&a1, g0.W13, H, (uint64_t)g0.n_experts * 2 * I, BK, BM) ||
+      !make_map(&b1, g0.x, H, g0.rows, BK, B_BOX) ||
+      !make_map(&a2, g0.W2, I, (uint64_t)g0.n_experts * H, BK, BM) ||
+      !make_map(&b2, g0.h, I, g0.rows, BK, B_BOX))
     return MOE_ERR_CUDA;
-  const int n_exp = e_end - e_begin;
-  moe_status st = launch_gemm<true, NMAX>(a1, b1, offsets, rows, e_begin, n_exp, H, I / BM, 2 * I,
-                                          I, h, I, s);
+  if (g1) {
+    if (!make_map(&sa1, g1->W13, H, (uint64_t)2 * I, BK, BM) ||
+        !make_map(&sb1, g1->x, H, g1->rows, BK, B_BOX) ||
+        !make_map(&sa2, g1->W2, I, (uint64_t)H, BK, BM) ||
+        !make_map(&sb2, g1->h, I, g1->rows, BK, B_BOX))
+      return MOE_ERR_CUDA;
+  } else {
+    sa1 = a1;  // unused: group 1 is empty
+    sb1 = b1;
+    sa2 = a2;
+    sb2 = b2;
+  }
+  GemmArgs args{};
+  args.offsets = g0.offsets;
+  args.rows0 = g0.rows;
+  args.e_begin = g0.e_begin;
+  args.n_exp = g0.e_end - g0.e_begin;
+  args.rows1 = g1 ? g1->rows : 0;
+  args.err = device_error_word();
+  // GEMM1 + SwiGLU: h = silu(x Wg^T) * (x Wu^T)
+  args.K = H;
+  args.n_fb = I / BM;
+  args.w_rows0 = 2 * I;
+  args.up_off = I;
+  args.out0 = g0.h;
+  args.out1 = g1 ? g1->h : nullptr;
+  args.out_ld = I;
+  moe_status st = launch_gemm<true, NMAX>(a1, b1, sa1, sb1, args, s);
   if (st != MOE_OK) return st;
   if (after_gemm1 && cudaEventRecord(after_gemm1, s) != cudaSuccess) return MOE_ERR_CUDA;
-  return launch_gemm<false, NMAX>(a2, b2, offsets, rows, e_begin, n_exp, I, H / BM, H, 0, y_perm,
-                                  H, s);
+  // GEMM2: y = h W2^T (fp32)
+  args.K = I;
+  args.n_fb = H / BM;
+  args.w_rows0 = H;
+  args.up_off = 0;
+  args.out0 = g0.y;
+  args.out1 = g1 ? g1->y : nullptr;
+  args.out_ld = H;
+  return launch_gemm<false, NMAX>(a2, b2, sa2, sb2, args, s);
 }
 
 }  // namespace
+
+moe_status launch_expert_ffn_groups(const FfnGroup& routed, const FfnGroup* dense, int H, int I,
+                                    int rows_hint, cudaStream_t s, cudaEvent_t after_gemm1) {
+  if ((routed.rows == 0 || routed.e_end <= routed.e_begin) && (!dense || dense->rows == 0))
+    return MOE_OK;
+  const int n_exp = routed.e_end - routed.e_begin;
+  const FfnGroup* g1 = (dense && dense->rows > 0) ? dense : nullptr;
+  // Few rows per expert (decode): small token tiles leave room for a deeper pipeline.
+  if ((long)rows_hint <= 24L * (n_exp > 0 ? n_exp : 1))
+    return run_ffn<32>(routed, g1, H, I, s, after_gemm1);
+  return run_ffn<256>(routed, g1, H, I, s, after_gemm1);
+}
 
 moe_status launch_expert_ffn(int rows, int H, int I, int n_experts, int e_begin, int e_end,
                              const uint16_t* x_perm, const int32_t* offsets, const uint16_t* W13,
                              const uint16_t* W2, uint16_t* h, float* y_perm, int rows_hint,
                              cudaStream_t s, cudaEvent_t after_gemm1) {
   if (rows == 0 || e_end <= e_begin) return MOE_OK;
-  const int n_exp = e_end - e_begin;
-  // Few rows per expert (decode): small token tiles leave room for a deeper pipeline.
-  if ((long)rows_hint <= 24L * n_exp)
-    return run_ffn<32>(rows, H, I, n_experts, e_begin, e_end, x_perm, offsets, W13, W2, h, y_perm,
-                       s, after_gemm1);
-  return run_ffn<256>(rows, H, I, n_experts, e_begin, e_end, x_perm, offsets, W13, W2, h, y_perm,
-                      s, after_gemm1);
+  FfnGroup g{x_perm, offsets, rows, n_experts, e_begin, e_end, W13, W2, h, y_perm};
+  return launch_expert_ffn_groups(g, nullptr, H, I, rows_hint, s, after_gemm1);
 }
 
 }  // namespace moe

@@ -252,6 +252,22 @@ moe_status shared_expert(const moe_config& c, const Layout& L, const moe_weights
   return mark(ev, MOE_EV_SHARED_GEMM2, s);
 }
 
+// Routed experts and the shared expert in one pair of grouped-GEMM launches
+// (the shared expert's units share the persistent grid with the routed ones).
+// Requires I_shared == I; the stage events then mark the fused GEMMs.
+moe_status experts_and_shared(const moe_config& c, const Layout& L, const moe_weights& w,
+                              const uint16_t* x, cudaStream_t s, cudaEvent_t* ev) {
+  MOE_TRY(launch_fill_range(L.sh_off, c.T, s));
+  const int rows = c.T * c.k;
+  FfnGroup routed{L.x_perm, L.offsets, rows, c.E, 0, c.E, w.W13, w.W2, L.h, L.y_perm};
+  FfnGroup dense{x, L.sh_off, c.T, 1, 0, 1, w.Ws13, w.Ws2, L.sh_h, L.sh_y};
+  MOE_TRY(launch_expert_ffn_groups(routed, &dense, c.H, c.I, rows, s,
+                                   ev ? ev[MOE_EV_GEMM1] : nullptr));
+  MOE_TRY(mark(ev, MOE_EV_GEMM2, s));
+  MOE_TRY(mark(ev, MOE_EV_SHARED_GEMM1, s));
+  return mark(ev, MOE_EV_SHARED_GEMM2, s);
+}
+
 moe_status combine_tokens(const moe_config& c, const Layout& L, int t0, int Tc, void* out,
                           int out_fp32, cudaStream_t s) {
   const size_t tk = (size_t)t0 * c.k;
@@ -412,8 +428,12 @@ moe_status moe_layer_forward(const moe_config* cfg, const moe_exec* ex, const mo
     cudaEvent_t* ev = reinterpret_cast<cudaEvent_t*>(ex->stage_events);
     MOE_TRY(mark(ev, MOE_EV_START, s));
     MOE_TRY(pack_tokens(c, L, *w, x, 0, c.T, 0, true, s, ev));
-    MOE_TRY(experts_tokens(c, L, *w, 0, c.T, 0, 0, c.E, s, ev));
-    MOE_TRY(shared_expert(c, L, *w, x, s, ev));
+    if (c.I_shared == c.I) {
+      MOE_TRY(experts_and_shared(c, L, *w, x, s, ev));
+    } else {
+      MOE_TRY(experts_tokens(c, L, *w, 0, c.T, 0, 0, c.E, s, ev));
+      MOE_TRY(shared_expert(c, L, *w, x, s, ev));
+    }
     MOE_TRY(combine_tokens(c, L, 0, c.T, out, ex->out_fp32, s));
     MOE_TRY(mark(ev, MOE_EV_COMBINE, s));
     if (aux && aux->counts)

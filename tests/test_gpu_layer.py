@@ -122,6 +122,27 @@ def test_layer_tiny_full(out_fp32):
     assert_layer_close(f64(out), ref)
 
 
+# ---------------------------------------------------------------- small grouped layers, every token
+
+@pytest.mark.parametrize("I_shared,T", [(128, 100), (256, 100), (128, 1), (384, 300)])
+def test_layer_small_grouped_full(I_shared, T):
+    """Sigmoid group-limited routing with a shared expert: fused into the routed GEMM
+    launches when I_shared == I, separate launches otherwise."""
+    wl = I.Workload("small", T=T, H=256, E=16, k=4, I=128, I_shared=I_shared, n_groups=4,
+                    topk_groups=2, gate=I.GATE_SIGMOID, normalize=1, route_scale=2.5)
+    d = I.layer_inputs(wl, seed=5, device=DEV)
+    st = prepare_routing(wl, d)
+    for ex in (L.exec_config(out_fp32=1), L.exec_config(out_fp32=0),
+               L.exec_config(out_fp32=1, overlap=1, chunk_axis=0, chunk_tokens=37),
+               L.exec_config(out_fp32=1, overlap=1, chunk_axis=1, n_expert_chunks=3)):
+        out, a = run_layer(wl, d, ex)
+        gidx = check_routing(wl, d, a, st["oracle_logits"])
+        ref, _ = O.layer_forward(f64(d["x"]), f64(d["Wr"]), bias32(d["bias"]), f64(d["W13"]),
+                                 f64(d["W2"]), oracle_cfg(wl), f64(d["Ws13"]), f64(d["Ws2"]))
+        assert_layer_close(f64(out), ref)
+    check_permutation(wl, d, gidx)
+
+
 # ---------------------------------------------------------------- decode: every token
 
 @pytest.mark.parametrize("ex", [dict(out_fp32=1), dict(out_fp32=0),

@@ -47,31 +47,52 @@ constexpr int B_BOX = 16;         // token rows per TMA box
 constexpr int NUM_THREADS = 192;  // 6 warps
 constexpr uint64_t WAIT_LIMIT_NS = 2000000000ull;
 
+// Tuning switches (compile time). Prefetching weight tiles into L2 ahead of
+// their shared-memory loads and marking weight lines evict-first both measured
+// slower on GB300 for the decode and prefill layers, so both are off.
+#ifndef MOE_GEMM_PREFETCH_BYTES
+#define MOE_GEMM_PREFETCH_BYTES 0
+#endif
+#ifndef MOE_GEMM_WEIGHT_EVICT_FIRST
+#define MOE_GEMM_WEIGHT_EVICT_FIRST 0
+#endif
+
 constexpr int pow2ceil(int v) {
   int p = 32;
   while (p < v) p <<= 1;
   return p;
 }
 
-template <bool SWIGLU, int NMAX>
+// Kernel modes: what one work unit's weight tiles are and what its epilogue does.
+constexpr int MODE_PLAIN = 0;   // one 128-feature weight tile; fp32 output
+constexpr int MODE_SWIGLU = 1;  // gate and up tiles of the same 128 features; SwiGLU, bf16 out
+constexpr int MODE_PLAIN2 = 2;  // two adjacent 128-feature tiles sharing one token tile; fp32 out
+
+template <int MODE, int NMAX>
 struct Tile {
-  static constexpr int NA = SWIGLU ? 2 : 1;
+  static constexpr int NA = MODE == MODE_PLAIN ? 1 : 2;        // weight tiles per stage
+  static constexpr int FEAT = MODE == MODE_PLAIN2 ? 2 * BM : BM;  // output features per unit
   static constexpr int A_BYTES = BM * BK * 2;  // 16 KiB
   static constexpr int B_BYTES = NMAX * BK * 2;
   static constexpr int STAGE_BYTES = NA * A_BYTES + B_BYTES;
-  static constexpr int STAGES_RAW = (200 * 1024) / STAGE_BYTES;
-  static constexpr int STAGES = STAGES_RAW > 8 ? 8 : STAGES_RAW;
+  // ~217 KiB of stages: with the control block, the expert tables (<= 8 KiB)
+  // and the 1 KiB alignment slack this stays under 227 KiB per CTA.
+  static constexpr int STAGES_RAW = (217 * 1024) / STAGE_BYTES;
+  static constexpr int STAGES = STAGES_RAW > 12 ? 12 : STAGES_RAW;
   static constexpr int ACC_COLS = NA * NMAX;                  // one accumulator (gate | up)
   static constexpr int ACC_STAGES = 2 * ACC_COLS <= 512 ? 2 : 1;  // double-buffer when it fits
   static constexpr int TMEM_COLS = pow2ceil(ACC_STAGES * ACC_COLS);
+  // Weight tiles prefetched into L2 this many k-blocks ahead of their
+  // shared-memory load (0 = no prefetch).
+  static constexpr int PF = MOE_GEMM_PREFETCH_BYTES / (NA * A_BYTES);
   static_assert(STAGES >= 2, "pipeline too shallow");
   static_assert(NMAX % 16 == 0 && NMAX >= 16 && NMAX <= 256, "MMA N range for M = 128");
   static_assert(TMEM_COLS <= 512, "TMEM holds 512 columns");
 };
 
 struct Ctrl {
-  uint64_t full[8];
-  uint64_t empty[8];
+  uint64_t full[12];
+  uint64_t empty[12];
   uint64_t acc_full[2];
   uint64_t acc_empty[2];
   uint64_t drain;
@@ -133,6 +154,30 @@ __device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap* map
       " [%0], [%1, {%2, %3}], [%4];" ::"r"(dst),
       "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(bar)
       : "memory");
+}
+
+// Same load with an L2 eviction-priority policy (createpolicy) on the lines read.
+__device__ __forceinline__ void tma_load_2d_hint(uint32_t dst, const CUtensorMap* map, int x, int y,
+                                                 uint32_t bar, uint64_t policy) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes.L2::cache_hint"
+      " [%0], [%1, {%2, %3}], [%4], %5;" ::"r"(dst),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(bar), "l"(policy)
+      : "memory");
+}
+
+// Bring a tile into L2 ahead of its shared-memory load (no completion to track).
+__device__ __forceinline__ void tma_prefetch_l2(const CUtensorMap* map, int x, int y) {
+  asm volatile("cp.async.bulk.prefetch.tensor.2d.L2.global.tile [%0, {%1, %2}];" ::"l"(
+                   reinterpret_cast<uint64_t>(map)),
+               "r"(x), "r"(y)
+               : "memory");
+}
+
+__device__ __forceinline__ uint64_t policy_evict_first() {
+  uint64_t p;
+  asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(p));
+  return p;
 }
 
 __device__ __forceinline__ void tma_prefetch_map(const CUtensorMap* map) {
@@ -205,7 +250,7 @@ struct GemmArgs {
   int rows1;
   int K, n_fb;
   int w_rows0;  // weight rows per expert in group 0
-  int up_off;   // SwiGLU: row offset of the up projection inside an expert
+  int up_off;   // row offset of a unit's second weight tile (SwiGLU: the up projection)
   void* out0;
   void* out1;
   int out_ld;
@@ -255,13 +300,14 @@ __device__ __forceinline__ Unit decode_unit(int u, const int* tile_off, const in
 
 // ------------------------------------------------------------------ kernel
 
-template <bool SWIGLU, int NMAX>
+template <int MODE, int NMAX>
 __global__ void __launch_bounds__(NUM_THREADS, 1)
     grouped_gemm_kernel(const __grid_constant__ CUtensorMap tmA0,
                         const __grid_constant__ CUtensorMap tmB0,
                         const __grid_constant__ CUtensorMap tmA1,
                         const __grid_constant__ CUtensorMap tmB1, const GemmArgs a) {
-  using TL = Tile<SWIGLU, NMAX>;
+  using TL = Tile<MODE, NMAX>;
+  constexpr bool SWIGLU = MODE == MODE_SWIGLU;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~static_cast<uintptr_t>(1023));
@@ -348,6 +394,31 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
         tma_prefetch_map(&tmA1);
         tma_prefetch_map(&tmB1);
       }
+      const uint64_t evict_first = policy_evict_first();
+      // L2 prefetch cursor (unit pu, k-block pkb): TL::PF k-blocks ahead of the fills
+      int pu = blockIdx.x, pkb = 0, p_wrow = 0;
+      const CUtensorMap* p_map = &tmA0;
+      auto p_setup = [&]() {
+        if (pu < total_units) {
+          const Unit P = decode_unit<NMAX>(pu, tile_off, row_off, a, units1);
+          p_map = P.grp ? &tmA1 : &tmA0;
+          p_wrow = P.grp ? P.fb * TL::FEAT : (a.e_begin + P.e) * a.w_rows0 + P.fb * TL::FEAT;
+        }
+      };
+      auto p_step = [&]() {
+        if (pu >= total_units) return;
+        tma_prefetch_l2(p_map, pkb * BK, p_wrow);
+        if (TL::NA == 2) tma_prefetch_l2(p_map, pkb * BK, p_wrow + a.up_off);
+        if (++pkb == kblocks) {
+          pkb = 0;
+          pu += gridDim.x;
+          p_setup();
+        }
+      };
+      if (TL::PF) {
+        p_setup();
+        for (int i = 0; i < TL::PF; ++i) p_step();
+      }
       int stage = 0;
       uint32_t phase = 0;
       long fills = 0;
@@ -357,7 +428,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
         const CUtensorMap* mA = U.grp ? &tmA1 : &tmA0;
         const CUtensorMap* mB = U.grp ? &tmB1 : &tmB0;
         const int n_pad = (U.m + 15) & ~15;
-        const int wrow = U.grp ? U.fb * BM : (a.e_begin + U.e) * a.w_rows0 + U.fb * BM;
+        const int wrow = U.grp ? U.fb * TL::FEAT : (a.e_begin + U.e) * a.w_rows0 + U.fb * TL::FEAT;
         const uint32_t bytes = TL::NA * TL::A_BYTES + n_pad * BK * 2;
         for (int kb = 0; kb < kblocks; ++kb) {
           const uint32_t full = smem_u32(&ctrl->full[stage]);
@@ -367,12 +438,19 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
           }
           mbar_arrive_expect_tx(full, bytes);
           const uint32_t sa = smem_u32(smem + stage * TL::STAGE_BYTES);
-          tma_load_2d(sa, mA, kb * BK, wrow, full);
-          if (SWIGLU) tma_load_2d(sa + TL::A_BYTES, mA, kb * BK, wrow + a.up_off, full);
+          if (MOE_GEMM_WEIGHT_EVICT_FIRST) {
+            tma_load_2d_hint(sa, mA, kb * BK, wrow, full, evict_first);
+            if (TL::NA == 2)
+              tma_load_2d_hint(sa + TL::A_BYTES, mA, kb * BK, wrow + a.up_off, full, evict_first);
+          } else {
+            tma_load_2d(sa, mA, kb * BK, wrow, full);
+            if (TL::NA == 2) tma_load_2d(sa + TL::A_BYTES, mA, kb * BK, wrow + a.up_off, full);
+          }
           const uint32_t sb = sa + TL::NA * TL::A_BYTES;
           for (int i = 0; i < n_pad / B_BOX; ++i)
             tma_load_2d(sb + i * (B_BOX * BK * 2), mB, kb * BK, U.row0 + i * B_BOX, full);
           ++fills;
+          if (TL::PF) p_step();
           if (++stage == TL::STAGES) {
             stage = 0;
             phase ^= 1;
@@ -424,7 +502,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
             const uint32_t acc = (kb > 0 || k > 0) ? 1u : 0u;
             const uint64_t bdesc = sdesc(sb + k * UMMA_K * 2);
             mma_bf16(d, sdesc(sa + k * UMMA_K * 2), bdesc, idesc, acc);
-            if (SWIGLU)
+            if (TL::NA == 2)
               mma_bf16(d + NMAX, sdesc(sa + TL::A_BYTES + k * UMMA_K * 2), bdesc, idesc, acc);
           }
           issued = true;
@@ -457,7 +535,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       if (!wait_bounded(smem_u32(&ctrl->acc_full[as]), acc_par, abort_flag, err)) break;
       tc_fence_after();
       const uint32_t tq = tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(as * TL::ACC_COLS);
-      const int f = U.fb * BM + q * 32 + lane;
+      const int f = U.fb * TL::FEAT + q * 32 + lane;
       const size_t o = (size_t)U.row0 * a.out_ld + f;
       void* out = U.grp ? a.out1 : a.out0;
       for (int c0 = 0; c0 < U.m; c0 += 16) {
@@ -474,6 +552,18 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
               const float uv = __uint_as_float(v[i]);
               const float hv = gv / (1.0f + expf(-gv)) * uv;
               static_cast<uint16_t*>(out)[o + (size_t)(c0 + i) * a.out_ld] = float_to_bf16_bits(hv);
+            }
+          }
+        } else if (MODE == MODE_PLAIN2) {
+          uint32_t v[16];
+          tmem_ld16(tq + NMAX + c0, v);  // the second tile: features f + 128
+          tmem_wait_ld();
+#pragma unroll
+          for (int i = 0; i < 16; ++i) {
+            if (c0 + i < U.m) {
+              float* y = static_cast<float*>(out) + o + (size_t)(c0 + i) * a.out_ld;
+              y[0] = __uint_as_float(g[i]);
+              y[BM] = __uint_as_float(v[i]);
             }
           }
         } else {
@@ -530,21 +620,21 @@ bool make_map(CUtensorMap* m, const void* ptr, uint64_t inner, uint64_t outer, u
             CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
-template <bool SWIGLU, int NMAX>
+template <int MODE, int NMAX>
 size_t gemm_smem_bytes(int n_exp) {
-  using TL = Tile<SWIGLU, NMAX>;
+  using TL = Tile<MODE, NMAX>;
   return 1024 + (size_t)TL::STAGES * TL::STAGE_BYTES + sizeof(Ctrl) + 2 * sizeof(int) * (n_exp + 1);
 }
 
-template <bool SWIGLU, int NMAX>
+template <int MODE, int NMAX>
 moe_status launch_gemm(const CUtensorMap& A0, const CUtensorMap& B0, const CUtensorMap& A1,
                        const CUtensorMap& B1, const GemmArgs& args, cudaStream_t s) {
-  const size_t smem = gemm_smem_bytes<SWIGLU, NMAX>(args.n_exp);
+  const size_t smem = gemm_smem_bytes<MODE, NMAX>(args.n_exp);
   if (smem > 227 * 1024) return MOE_ERR_UNSUPPORTED;
-  if (cudaFuncSetAttribute(grouped_gemm_kernel<SWIGLU, NMAX>,
+  if (cudaFuncSetAttribute(grouped_gemm_kernel<MODE, NMAX>,
                            cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) != cudaSuccess)
     return MOE_ERR_CUDA;
-  grouped_gemm_kernel<SWIGLU, NMAX><<<num_sms(), NUM_THREADS, smem, s>>>(A0, B0, A1, B1, args);
+  grouped_gemm_kernel<MODE, NMAX><<<num_sms(), NUM_THREADS, smem, s>>>(A0, B0, A1, B1, args);
   note_launch();
   return launch_status();
 }
@@ -585,18 +675,23 @@ moe_status run_ffn(const FfnGroup& g0, const FfnGroup* g1, int H, int I, cudaStr
   args.out0 = g0.h;
   args.out1 = g1 ? g1->h : nullptr;
   args.out_ld = I;
-  moe_status st = launch_gemm<true, NMAX>(a1, b1, sa1, sb1, args, s);
+  moe_status st = launch_gemm<MODE_SWIGLU, NMAX>(a1, b1, sa1, sb1, args, s);
   if (st != MOE_OK) return st;
   if (after_gemm1 && cudaEventRecord(after_gemm1, s) != cudaSuccess) return MOE_ERR_CUDA;
-  // GEMM2: y = h W2^T (fp32)
+  // GEMM2: y = h W2^T (fp32); two 128-feature weight tiles per unit when H allows
   args.K = I;
-  args.n_fb = H / BM;
   args.w_rows0 = H;
-  args.up_off = 0;
   args.out0 = g0.y;
   args.out1 = g1 ? g1->y : nullptr;
   args.out_ld = H;
-  return launch_gemm<false, NMAX>(a2, b2, sa2, sb2, args, s);
+  if (H % (2 * BM) == 0) {
+    args.n_fb = H / (2 * BM);
+    args.up_off = BM;
+    return launch_gemm<MODE_PLAIN2, NMAX>(a2, b2, sa2, sb2, args, s);
+  }
+  args.n_fb = H / BM;
+  args.up_off = 0;
+  return launch_gemm<MODE_PLAIN, NMAX>(a2, b2, sa2, sb2, args, s);
 }
 
 }  // namespace
@@ -607,9 +702,12 @@ moe_status launch_expert_ffn_groups(const FfnGroup& routed, const FfnGroup* dens
     return MOE_OK;
   const int n_exp = routed.e_end - routed.e_begin;
   const FfnGroup* g1 = (dense && dense->rows > 0) ? dense : nullptr;
-  // Few rows per expert (decode): small token tiles leave room for a deeper pipeline.
-  if ((long)rows_hint <= 24L * (n_exp > 0 ? n_exp : 1))
-    return run_ffn<32>(routed, g1, H, I, s, after_gemm1);
+  // Token-tile size from the expected rows per expert: small tiles leave more
+  // of the stage ring to weights (decode ~4 rows/expert -> 32; balanced
+  // prefill ~128 +- 10 % -> 144; larger or skewed loads -> 256).
+  const long per = (long)rows_hint / (n_exp > 0 ? n_exp : 1);
+  if (per <= 24) return run_ffn<32>(routed, g1, H, I, s, after_gemm1);
+  if (per <= 132) return run_ffn<144>(routed, g1, H, I, s, after_gemm1);
   return run_ffn<256>(routed, g1, H, I, s, after_gemm1);
 }
 

@@ -216,6 +216,7 @@ def ffn_case(counts, H, Iw, seed, rows_extra=3):
     ([300, 256, 257, 0, 1, 16], 256, 256),              # multi-tile experts, tile edges
     ([4] * 60 + [0, 12, 31, 33], 512, 256),             # decode-like: small token tiles
     ([0, 0, 0, 40], 384, 128),
+    ([150, 100, 0, 145, 3], 512, 256),                  # 144-row tiles, experts over two tiles
     ([130, 111], 7168, 2048),                           # the real layer shape
     ([1] * 48 + [3, 7], 7168, 2048),                    # decode: few rows per expert
 ])

@@ -141,7 +141,7 @@ moe_status moe_validate_config(const moe_config* cfg);
  * configuration. Host-only. */
 size_t moe_workspace_size(const moe_config* cfg, const moe_exec* ex);
 
-/* Workspace bytes of the split-K router partials (may be 0). Host-only. */
+/* Workspace bytes of moe_router_logits' scratch (may be 0). Host-only. */
 size_t moe_router_workspace_size(const moe_config* cfg);
 
 /* Workspace bytes of moe_dispatch's per-chunk histograms. Host-only. */
@@ -151,11 +151,15 @@ size_t moe_dispatch_workspace_size(const moe_config* cfg);
 size_t moe_expert_ffn_workspace_size(int32_t rows, int32_t I);
 
 /*
- * Router logits: logits[t,e] = sum_h x[t,h] * Wr[e,h], fp32 accumulation.
+ * Router logits: logits[t,e] = sum_h x[t,h] * Wr[e,h], fp32-accurate.
  * x [T,H] bf16; Wr [E,H] fp32; logits [T,E] fp32 (written). ws/ws_bytes:
- * scratch for split-K partials (moe_router_workspace_size bytes); with ws NULL
- * the reduction is not split. The gating of every routed token starts here
- * (the paper's workload routes each token to its experts, Section 4).
+ * scratch of moe_router_workspace_size bytes, 16-byte aligned. With it and E
+ * a multiple of 128 the product runs on the tensor cores: Wr is split exactly
+ * into three bf16 planes (hi + mid + lo) whose products with the bf16 x are
+ * exact and summed in fp32; K is split across CTAs and the partials are added
+ * in a fixed order. Otherwise (or with ws NULL) an fp32 SIMT kernel runs. The
+ * gating of every routed token starts here (the paper's workload routes each
+ * token to its experts, Section 4).
  */
 moe_status moe_router_logits(const moe_config* cfg, const uint16_t* x, const float* Wr,
                              float* logits, void* ws, size_t ws_bytes, void* stream);

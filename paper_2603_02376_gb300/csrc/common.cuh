@@ -39,6 +39,20 @@ inline bool aligned4(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 3
 moe_status launch_router(const moe_config& c, const uint16_t* x, const float* Wr, float* logits,
                          float* partials, int splits, cudaStream_t s);
 int router_splits(const moe_config& c);
+// The router as the library runs it: tensor cores when E % 128 == 0 and a
+// workspace of router_workspace_bytes(c) is given, else the SIMT kernel.
+size_t router_workspace_bytes(const moe_config& c);
+moe_status launch_router_auto(const moe_config& c, const uint16_t* x, const float* Wr,
+                              float* logits, void* ws, cudaStream_t s);
+
+// Tensor-core router (E a multiple of 128): Wr split into three bf16 planes
+// (hi, mid, lo) whose sum is the fp32 value; partial logits per K split.
+moe_status launch_split_planes(const float* Wr, size_t n, uint16_t* planes, cudaStream_t s);
+int router_tc_splits(int T, int H, int E);
+moe_status launch_router_tc(int T, int H, int E, const uint16_t* x, const uint16_t* planes,
+                            float* partials, int k_splits, cudaStream_t s);
+moe_status launch_router_reduce(const float* partials, int splits, size_t n, float* logits,
+                                cudaStream_t s);
 
 moe_status launch_gate(const moe_config& c, const float* logits, const float* bias, int32_t* idx,
                        float* w, cudaStream_t s);

@@ -47,15 +47,7 @@ constexpr int B_BOX = 16;         // token rows per TMA box
 constexpr int NUM_THREADS = 192;  // 6 warps
 constexpr uint64_t WAIT_LIMIT_NS = 2000000000ull;
 
-// Tuning switches (compile time). Prefetching weight tiles into L2 ahead of
-// their shared-memory loads and marking weight lines evict-first both measured
-// slower on GB300 for the decode and prefill layers, so both are off.
-#ifndef MOE_GEMM_PREFETCH_BYTES
-#define MOE_GEMM_PREFETCH_BYTES 0
-#endif
-#ifndef MOE_GEMM_WEIGHT_EVICT_FIRST
-#define MOE_GEMM_WEIGHT_EVICT_FIRST 0
-#endif
+
 
 constexpr int pow2ceil(int v) {
   int p = 32;
@@ -67,10 +59,13 @@ constexpr int pow2ceil(int v) {
 constexpr int MODE_PLAIN = 0;   // one 128-feature weight tile; fp32 output
 constexpr int MODE_SWIGLU = 1;  // gate and up tiles of the same 128 features; SwiGLU, bf16 out
 constexpr int MODE_PLAIN2 = 2;  // two adjacent 128-feature tiles sharing one token tile; fp32 out
+constexpr int MODE_SPLIT3 = 3;  // three bf16 planes of one fp32 weight tile, summed into one
+                                // accumulator (an fp32 x bf16 product on bf16 tensor cores)
 
 template <int MODE, int NMAX>
 struct Tile {
-  static constexpr int NA = MODE == MODE_PLAIN ? 1 : 2;        // weight tiles per stage
+  static constexpr int NA = MODE == MODE_PLAIN ? 1 : MODE == MODE_SPLIT3 ? 3 : 2;  // A tiles
+  static constexpr bool TWO_ACC = MODE == MODE_SWIGLU || MODE == MODE_PLAIN2;  // tile i -> acc i
   static constexpr int FEAT = MODE == MODE_PLAIN2 ? 2 * BM : BM;  // output features per unit
   static constexpr int A_BYTES = BM * BK * 2;  // 16 KiB
   static constexpr int B_BYTES = NMAX * BK * 2;
@@ -79,12 +74,9 @@ struct Tile {
   // and the 1 KiB alignment slack this stays under 227 KiB per CTA.
   static constexpr int STAGES_RAW = (217 * 1024) / STAGE_BYTES;
   static constexpr int STAGES = STAGES_RAW > 12 ? 12 : STAGES_RAW;
-  static constexpr int ACC_COLS = NA * NMAX;                  // one accumulator (gate | up)
+  static constexpr int ACC_COLS = TWO_ACC ? 2 * NMAX : NMAX;  // one accumulator (gate | up)
   static constexpr int ACC_STAGES = 2 * ACC_COLS <= 512 ? 2 : 1;  // double-buffer when it fits
   static constexpr int TMEM_COLS = pow2ceil(ACC_STAGES * ACC_COLS);
-  // Weight tiles prefetched into L2 this many k-blocks ahead of their
-  // shared-memory load (0 = no prefetch).
-  static constexpr int PF = MOE_GEMM_PREFETCH_BYTES / (NA * A_BYTES);
   static_assert(STAGES >= 2, "pipeline too shallow");
   static_assert(NMAX % 16 == 0 && NMAX >= 16 && NMAX <= 256, "MMA N range for M = 128");
   static_assert(TMEM_COLS <= 512, "TMEM holds 512 columns");
@@ -154,30 +146,6 @@ __device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap* map
       " [%0], [%1, {%2, %3}], [%4];" ::"r"(dst),
       "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(bar)
       : "memory");
-}
-
-// Same load with an L2 eviction-priority policy (createpolicy) on the lines read.
-__device__ __forceinline__ void tma_load_2d_hint(uint32_t dst, const CUtensorMap* map, int x, int y,
-                                                 uint32_t bar, uint64_t policy) {
-  asm volatile(
-      "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes.L2::cache_hint"
-      " [%0], [%1, {%2, %3}], [%4], %5;" ::"r"(dst),
-      "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(bar), "l"(policy)
-      : "memory");
-}
-
-// Bring a tile into L2 ahead of its shared-memory load (no completion to track).
-__device__ __forceinline__ void tma_prefetch_l2(const CUtensorMap* map, int x, int y) {
-  asm volatile("cp.async.bulk.prefetch.tensor.2d.L2.global.tile [%0, {%1, %2}];" ::"l"(
-                   reinterpret_cast<uint64_t>(map)),
-               "r"(x), "r"(y)
-               : "memory");
-}
-
-__device__ __forceinline__ uint64_t policy_evict_first() {
-  uint64_t p;
-  asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(p));
-  return p;
 }
 
 __device__ __forceinline__ void tma_prefetch_map(const CUtensorMap* map) {
@@ -250,7 +218,9 @@ struct GemmArgs {
   int rows1;
   int K, n_fb;
   int w_rows0;  // weight rows per expert in group 0
-  int up_off;   // row offset of a unit's second weight tile (SwiGLU: the up projection)
+  int up_off;   // row offset between a unit's weight tiles (SwiGLU: the up projection)
+  int k_splits; // group 1 only: the K range is split into this many units ...
+  long split_stride;  // ... whose outputs go to out1 + split * split_stride (partials)
   void* out0;
   void* out1;
   int out_ld;
@@ -263,22 +233,33 @@ struct Unit {
   int fb;    // 128-feature block
   int row0;  // first activation row of the token tile
   int m;     // valid token rows in the tile (1..NMAX)
+  int kb0, kb1;  // k-blocks [kb0, kb1) of this unit
+  int split;     // K split index (group 1)
 };
 
 template <int NMAX>
 __device__ __forceinline__ Unit decode_unit(int u, const int* tile_off, const int* row_off,
-                                            const GemmArgs& a, int units1) {
+                                            const GemmArgs& a, int units1, int kblocks) {
   Unit U;
-  if (u < units1) {  // group 1: the shared expert's dense segment
+  if (u < units1) {  // group 1: one dense segment (the shared expert, or the router)
     const int nt1 = (a.rows1 + NMAX - 1) / NMAX;
+    const int per_split = nt1 * a.n_fb;
+    U.split = u / per_split;
+    u -= U.split * per_split;
     U.grp = 1;
     U.e = 0;
     U.fb = u / nt1;
     const int nt = u - U.fb * nt1;
     U.row0 = nt * NMAX;
     U.m = min(NMAX, a.rows1 - U.row0);
+    const int kps = (kblocks + a.k_splits - 1) / a.k_splits;
+    U.kb0 = min(kblocks, U.split * kps);
+    U.kb1 = min(kblocks, U.kb0 + kps);
     return U;
   }
+  U.split = 0;
+  U.kb0 = 0;
+  U.kb1 = kblocks;
   u -= units1;
   int lo = 0, hi = a.n_exp - 1;
   while (lo < hi) {  // largest e with tile_off[e] * n_fb <= u: an expert with tiles
@@ -374,16 +355,16 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
     }
     if (lane == 31) {
       tile_off[n_exp] = incl;
-      row_off[n_exp] = clamped(n_exp);
+      row_off[n_exp] = n_exp > 0 ? clamped(n_exp) : 0;
     }
   }
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem_base = ctrl->tmem_base;
-  const int units1 = a.rows1 > 0 ? ((a.rows1 + NMAX - 1) / NMAX) * a.n_fb : 0;
-  const int total_units = units1 + tile_off[a.n_exp] * a.n_fb;
   const int kblocks = a.K / BK;
+  const int units1 = a.rows1 > 0 ? ((a.rows1 + NMAX - 1) / NMAX) * a.n_fb * a.k_splits : 0;
+  const int total_units = units1 + tile_off[a.n_exp] * a.n_fb;
 
   if (warp == 0) {
     if (lane == 0) {
@@ -394,43 +375,18 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
         tma_prefetch_map(&tmA1);
         tma_prefetch_map(&tmB1);
       }
-      const uint64_t evict_first = policy_evict_first();
-      // L2 prefetch cursor (unit pu, k-block pkb): TL::PF k-blocks ahead of the fills
-      int pu = blockIdx.x, pkb = 0, p_wrow = 0;
-      const CUtensorMap* p_map = &tmA0;
-      auto p_setup = [&]() {
-        if (pu < total_units) {
-          const Unit P = decode_unit<NMAX>(pu, tile_off, row_off, a, units1);
-          p_map = P.grp ? &tmA1 : &tmA0;
-          p_wrow = P.grp ? P.fb * TL::FEAT : (a.e_begin + P.e) * a.w_rows0 + P.fb * TL::FEAT;
-        }
-      };
-      auto p_step = [&]() {
-        if (pu >= total_units) return;
-        tma_prefetch_l2(p_map, pkb * BK, p_wrow);
-        if (TL::NA == 2) tma_prefetch_l2(p_map, pkb * BK, p_wrow + a.up_off);
-        if (++pkb == kblocks) {
-          pkb = 0;
-          pu += gridDim.x;
-          p_setup();
-        }
-      };
-      if (TL::PF) {
-        p_setup();
-        for (int i = 0; i < TL::PF; ++i) p_step();
-      }
       int stage = 0;
       uint32_t phase = 0;
       long fills = 0;
       bool ok = true;
       for (int u = blockIdx.x; u < total_units && ok; u += gridDim.x) {
-        const Unit U = decode_unit<NMAX>(u, tile_off, row_off, a, units1);
+        const Unit U = decode_unit<NMAX>(u, tile_off, row_off, a, units1, kblocks);
         const CUtensorMap* mA = U.grp ? &tmA1 : &tmA0;
         const CUtensorMap* mB = U.grp ? &tmB1 : &tmB0;
         const int n_pad = (U.m + 15) & ~15;
         const int wrow = U.grp ? U.fb * TL::FEAT : (a.e_begin + U.e) * a.w_rows0 + U.fb * TL::FEAT;
         const uint32_t bytes = TL::NA * TL::A_BYTES + n_pad * BK * 2;
-        for (int kb = 0; kb < kblocks; ++kb) {
+        for (int kb = U.kb0; kb < U.kb1; ++kb) {
           const uint32_t full = smem_u32(&ctrl->full[stage]);
           if (!wait_bounded(smem_u32(&ctrl->empty[stage]), phase ^ 1, abort_flag, err)) {
             ok = false;
@@ -438,19 +394,13 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
           }
           mbar_arrive_expect_tx(full, bytes);
           const uint32_t sa = smem_u32(smem + stage * TL::STAGE_BYTES);
-          if (MOE_GEMM_WEIGHT_EVICT_FIRST) {
-            tma_load_2d_hint(sa, mA, kb * BK, wrow, full, evict_first);
-            if (TL::NA == 2)
-              tma_load_2d_hint(sa + TL::A_BYTES, mA, kb * BK, wrow + a.up_off, full, evict_first);
-          } else {
-            tma_load_2d(sa, mA, kb * BK, wrow, full);
-            if (TL::NA == 2) tma_load_2d(sa + TL::A_BYTES, mA, kb * BK, wrow + a.up_off, full);
-          }
+#pragma unroll
+          for (int t = 0; t < TL::NA; ++t)
+            tma_load_2d(sa + t * TL::A_BYTES, mA, kb * BK, wrow + t * a.up_off, full);
           const uint32_t sb = sa + TL::NA * TL::A_BYTES;
           for (int i = 0; i < n_pad / B_BOX; ++i)
             tma_load_2d(sb + i * (B_BOX * BK * 2), mB, kb * BK, U.row0 + i * B_BOX, full);
           ++fills;
-          if (TL::PF) p_step();
           if (++stage == TL::STAGES) {
             stage = 0;
             phase ^= 1;
@@ -478,7 +428,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       int j = 0;  // units of this CTA so far: accumulator j % ACC_STAGES
       bool ok = true, issued = false;
       for (int u = blockIdx.x; u < total_units && ok; u += gridDim.x, ++j) {
-        const Unit U = decode_unit<NMAX>(u, tile_off, row_off, a, units1);
+        const Unit U = decode_unit<NMAX>(u, tile_off, row_off, a, units1, kblocks);
         const int n_pad = (U.m + 15) & ~15;
         const uint32_t idesc = idesc_bf16(n_pad);
         const int as = j % TL::ACC_STAGES;
@@ -489,7 +439,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
         }
         tc_fence_after();
         const uint32_t d = tmem_base + (uint32_t)(as * TL::ACC_COLS);
-        for (int kb = 0; kb < kblocks; ++kb) {
+        for (int kb = U.kb0; kb < U.kb1; ++kb) {
           if (!wait_bounded(smem_u32(&ctrl->full[stage]), phase, abort_flag, err)) {
             ok = false;
             break;
@@ -499,11 +449,15 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
           const uint32_t sb = sa + TL::NA * TL::A_BYTES;
 #pragma unroll
           for (int k = 0; k < BK / UMMA_K; ++k) {
-            const uint32_t acc = (kb > 0 || k > 0) ? 1u : 0u;
+            const uint32_t acc = (kb > U.kb0 || k > 0) ? 1u : 0u;
             const uint64_t bdesc = sdesc(sb + k * UMMA_K * 2);
             mma_bf16(d, sdesc(sa + k * UMMA_K * 2), bdesc, idesc, acc);
-            if (TL::NA == 2)
+            if (TL::TWO_ACC)
               mma_bf16(d + NMAX, sdesc(sa + TL::A_BYTES + k * UMMA_K * 2), bdesc, idesc, acc);
+            if (MODE == MODE_SPLIT3) {  // the lower planes add into the same accumulator
+              mma_bf16(d, sdesc(sa + TL::A_BYTES + k * UMMA_K * 2), bdesc, idesc, 1u);
+              mma_bf16(d, sdesc(sa + 2 * TL::A_BYTES + k * UMMA_K * 2), bdesc, idesc, 1u);
+            }
           }
           issued = true;
           mma_commit(smem_u32(&ctrl->empty[stage]));
@@ -529,7 +483,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
     const int q = warp & 3;  // TMEM lane quarter this warp may access
     int j = 0;
     for (int u = blockIdx.x; u < total_units; u += gridDim.x, ++j) {
-      const Unit U = decode_unit<NMAX>(u, tile_off, row_off, a, units1);
+      const Unit U = decode_unit<NMAX>(u, tile_off, row_off, a, units1, kblocks);
       const int as = j % TL::ACC_STAGES;
       const uint32_t acc_par = (uint32_t)((j / TL::ACC_STAGES) & 1);
       if (!wait_bounded(smem_u32(&ctrl->acc_full[as]), acc_par, abort_flag, err)) break;
@@ -537,7 +491,8 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       const uint32_t tq = tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(as * TL::ACC_COLS);
       const int f = U.fb * TL::FEAT + q * 32 + lane;
       const size_t o = (size_t)U.row0 * a.out_ld + f;
-      void* out = U.grp ? a.out1 : a.out0;
+      void* out = U.grp ? static_cast<void*>(static_cast<float*>(a.out1) + U.split * a.split_stride)
+                        : a.out0;
       for (int c0 = 0; c0 < U.m; c0 += 16) {
         uint32_t g[16];
         tmem_ld16(tq + c0, g);
@@ -661,6 +616,7 @@ moe_status run_ffn(const FfnGroup& g0, const FfnGroup* g1, int H, int I, cudaStr
     sb2 = b2;
   }
   GemmArgs args{};
+  args.k_splits = 1;
   args.offsets = g0.offsets;
   args.rows0 = g0.rows;
   args.e_begin = g0.e_begin;
@@ -709,6 +665,33 @@ moe_status launch_expert_ffn_groups(const FfnGroup& routed, const FfnGroup* dens
   if (per <= 24) return run_ffn<32>(routed, g1, H, I, s, after_gemm1);
   if (per <= 132) return run_ffn<144>(routed, g1, H, I, s, after_gemm1);
   return run_ffn<256>(routed, g1, H, I, s, after_gemm1);
+}
+
+int router_tc_splits(int T, int H, int E) {
+  const int tiles = ((T + 127) / 128) * (E / BM);
+  const int kblocks = H / BK;
+  int ks = (2 * 152 + tiles - 1) / tiles;  // about two units per SM
+  if (ks > kblocks / 2) ks = kblocks / 2;  // at least two k-blocks per unit
+  return ks < 1 ? 1 : ks;
+}
+
+moe_status launch_router_tc(int T, int H, int E, const uint16_t* x, const uint16_t* planes,
+                            float* partials, int k_splits, cudaStream_t s) {
+  if (T == 0) return MOE_OK;
+  CUtensorMap A, B;
+  if (!make_map(&A, planes, H, (uint64_t)3 * E, BK, BM) || !make_map(&B, x, H, T, BK, B_BOX))
+    return MOE_ERR_CUDA;
+  GemmArgs args{};
+  args.rows1 = T;  // group 1: all tokens; group 0 is empty
+  args.K = H;
+  args.n_fb = E / BM;
+  args.up_off = E;  // plane p of expert row r sits at row p * E + r
+  args.k_splits = k_splits;
+  args.split_stride = (long)T * E;
+  args.out1 = partials;
+  args.out_ld = E;
+  args.err = device_error_word();
+  return launch_gemm<MODE_SPLIT3, 128>(A, B, A, B, args, s);
 }
 
 moe_status launch_expert_ffn(int rows, int H, int I, int n_experts, int e_begin, int e_end,

@@ -112,7 +112,7 @@ struct Carver {
 };
 
 struct Layout {
-  int chunk_T = 0, n_chunks = 1, splits = 1, perm_chunks = 0;
+  int chunk_T = 0, n_chunks = 1, perm_chunks = 0;
   float* logits;
   int32_t* idx;
   float* w;
@@ -122,7 +122,7 @@ struct Layout {
   int32_t* slot_row; // [T*k]
   int32_t* perm_counts;
   int32_t* perm_base;
-  float* partials;
+  void* router_ws;   // router scratch (planes + partials), sized for one chunk
   uint16_t* x_perm;  // [T*k, H]
   uint16_t* h;       // [T*k, I]
   float* y_perm;     // [T*k, H] fp32
@@ -142,7 +142,6 @@ Layout carve(const moe_config& c, const moe_exec& ex, void* ws) {
   if (L.n_chunks < 1) L.n_chunks = 1;
   moe_config cc = c;
   cc.T = L.chunk_T;
-  L.splits = router_splits(cc);
   L.perm_chunks = perm_num_chunks(L.chunk_T);
   Carver cv(ws);
   L.logits = cv.take<float>(T * E);
@@ -154,7 +153,8 @@ Layout carve(const moe_config& c, const moe_exec& ex, void* ws) {
   L.slot_row = cv.take<int32_t>(T * k);
   L.perm_counts = cv.take<int32_t>((size_t)(L.perm_chunks + 1) * E);
   L.perm_base = cv.take<int32_t>((size_t)(L.perm_chunks + 1) * E);
-  L.partials = L.splits > 1 ? cv.take<float>((size_t)L.splits * L.chunk_T * E) : nullptr;
+  const size_t rws = router_workspace_bytes(cc);
+  L.router_ws = rws ? static_cast<void*>(cv.take<uint8_t>(rws)) : nullptr;
   L.x_perm = cv.take<uint16_t>(T * k * c.H);
   L.h = cv.take<uint16_t>(T * k * c.I);
   L.y_perm = cv.take<float>(T * k * c.H);
@@ -211,8 +211,8 @@ moe_status pack_tokens(const moe_config& c, const Layout& L, const moe_weights& 
   moe_config cc = c;
   cc.T = Tc;
   const size_t tk = (size_t)t0 * c.k;
-  MOE_TRY(launch_router(cc, x + (size_t)t0 * c.H, w.Wr, L.logits + (size_t)t0 * c.E, L.partials,
-                        L.splits, s));
+  MOE_TRY(launch_router_auto(cc, x + (size_t)t0 * c.H, w.Wr, L.logits + (size_t)t0 * c.E,
+                             L.router_ws, s));
   MOE_TRY(mark(ev, MOE_EV_ROUTER, s));
   MOE_TRY(launch_gate(cc, L.logits + (size_t)t0 * c.E, w.bias, L.idx + tk, L.w + tk, s));
   MOE_TRY(mark(ev, MOE_EV_GATE, s));
@@ -308,8 +308,7 @@ size_t moe_workspace_size(const moe_config* cfg, const moe_exec* ex) {
 
 size_t moe_router_workspace_size(const moe_config* cfg) {
   if (!valid_config(cfg)) return 0;
-  const int s = router_splits(*cfg);
-  return s > 1 ? (size_t)s * cfg->T * cfg->E * sizeof(float) : 0;
+  return router_workspace_bytes(*cfg);
 }
 
 size_t moe_dispatch_workspace_size(const moe_config* cfg) {
@@ -329,14 +328,8 @@ moe_status moe_router_logits(const moe_config* cfg, const uint16_t* x, const flo
   if (!x || !Wr || !logits || !aligned16(x) || !aligned16(Wr) || !aligned4(logits))
     return MOE_ERR_INVALID_ARG;
   const size_t need = moe_router_workspace_size(cfg);
-  float* part = nullptr;
-  int splits = 1;
-  if (ws && need) {
-    if (ws_bytes < need || !aligned4(ws)) return MOE_ERR_WORKSPACE;
-    part = (float*)ws;
-    splits = router_splits(*cfg);
-  }
-  return launch_router(*cfg, x, Wr, logits, part, splits, (cudaStream_t)stream);
+  if (ws && need && (ws_bytes < need || !aligned16(ws))) return MOE_ERR_WORKSPACE;
+  return launch_router_auto(*cfg, x, Wr, logits, need ? ws : nullptr, (cudaStream_t)stream);
 }
 
 moe_status moe_gate_topk(const moe_config* cfg, const float* logits, const float* bias,

@@ -1,9 +1,15 @@
 // Router logits: L[t,e] = sum_h x[t,h] * Wr[e,h] with x bf16, Wr fp32, fp32 accumulation.
 //
 // The router is the first step of the routed MoE layer (the paper's DeepSeek-V3
-// workload routes every token to its experts, Section 4). Kept on the fp32 SIMT
-// pipe: the router weights are fp32, so a bf16 tensor-core product would change
-// the logits the routing decisions are taken on.
+// workload routes every token to its experts, Section 4). The router weights
+// are fp32, so a plain bf16 tensor-core product would change the logits the
+// routing decisions are taken on. Two exact forms are provided:
+//  * tensor cores (E a multiple of 128): Wr is split into three bf16 planes
+//    whose sum is Wr (split_planes_kernel); each x * plane product is exact in
+//    the fp32 TMEM accumulator, so the grouped GEMM (three planes summed into
+//    one accumulator) yields fp32-accurate logits; K is split across CTAs and
+//    the partials are summed in split order (router_reduce_kernel);
+//  * the fp32 SIMT kernel below, for any E.
 //
 // Tiling: a CTA computes a 64-token x 64-expert tile with 256 threads, each
 // owning a 4x4 block of outputs; K is staged 32 at a time through shared memory
@@ -103,7 +109,42 @@ __global__ void router_reduce_kernel(const float* __restrict__ partials, int spl
   }
 }
 
+// planes[p * n + i] for p = 0, 1, 2: hi = bf16(w), mid = bf16(w - hi),
+// lo = bf16(w - hi - mid). Both differences are exact in fp32, so
+// hi + mid + lo carries all 24 significant bits of w (to within 2^-24 |w|).
+__global__ void split_planes_kernel(const float* __restrict__ w, size_t n,
+                                    uint16_t* __restrict__ planes) {
+  for (size_t i = blockIdx.x * (size_t)blockDim.x + threadIdx.x; i < n;
+       i += (size_t)gridDim.x * blockDim.x) {
+    const float v = w[i];
+    const uint16_t hi = float_to_bf16_bits(v);
+    const float r1 = v - bf16_bits_to_float(hi);
+    const uint16_t mid = float_to_bf16_bits(r1);
+    const float r2 = r1 - bf16_bits_to_float(mid);
+    planes[i] = hi;
+    planes[n + i] = mid;
+    planes[2 * n + i] = float_to_bf16_bits(r2);
+  }
+}
+
 }  // namespace
+
+moe_status launch_split_planes(const float* Wr, size_t n, uint16_t* planes, cudaStream_t s) {
+  int blocks = (int)((n + 255) / 256);
+  if (blocks > 4 * num_sms()) blocks = 4 * num_sms();
+  split_planes_kernel<<<blocks, 256, 0, s>>>(Wr, n, planes);
+  note_launch();
+  return launch_status();
+}
+
+moe_status launch_router_reduce(const float* partials, int splits, size_t n, float* logits,
+                                cudaStream_t s) {
+  int blocks = (int)((n + 255) / 256);
+  if (blocks > 4 * num_sms()) blocks = 4 * num_sms();
+  router_reduce_kernel<<<blocks, 256, 0, s>>>(partials, splits, n, logits);
+  note_launch();
+  return launch_status();
+}
 
 int router_splits(const moe_config& c) {
   if (c.T <= 0) return 1;
@@ -134,6 +175,35 @@ moe_status launch_router(const moe_config& c, const uint16_t* x, const float* Wr
     note_launch();
   }
   return launch_status();
+}
+
+// Scratch of the router: the three bf16 planes of Wr and the per-split partial
+// logits (tensor-core path), or the SIMT split-K partials.
+size_t router_workspace_bytes(const moe_config& c) {
+  if (c.T <= 0) return 0;
+  if (c.E % 128 == 0) {
+    const size_t planes = align_up((size_t)3 * c.E * c.H * sizeof(uint16_t), 256);
+    return planes + (size_t)router_tc_splits(c.T, c.H, c.E) * c.T * c.E * sizeof(float);
+  }
+  const int s = router_splits(c);
+  return s > 1 ? (size_t)s * c.T * c.E * sizeof(float) : 0;
+}
+
+moe_status launch_router_auto(const moe_config& c, const uint16_t* x, const float* Wr,
+                              float* logits, void* ws, cudaStream_t s) {
+  if (c.T == 0) return MOE_OK;
+  if (c.E % 128 == 0 && ws) {
+    uint16_t* planes = static_cast<uint16_t*>(ws);
+    float* partials = reinterpret_cast<float*>(
+        static_cast<uint8_t*>(ws) + align_up((size_t)3 * c.E * c.H * sizeof(uint16_t), 256));
+    const int ks = router_tc_splits(c.T, c.H, c.E);
+    moe_status st = launch_split_planes(Wr, (size_t)c.E * c.H, planes, s);
+    if (st != MOE_OK) return st;
+    st = launch_router_tc(c.T, c.H, c.E, x, planes, partials, ks, s);
+    if (st != MOE_OK) return st;
+    return launch_router_reduce(partials, ks, (size_t)c.T * c.E, logits, s);
+  }
+  return launch_router(c, x, Wr, logits, static_cast<float*>(ws), ws ? router_splits(c) : 1, s);
 }
 
 }  // namespace moe

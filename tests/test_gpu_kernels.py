@@ -34,8 +34,12 @@ def rand_bf16(shape, seed, std=1.0):
 # ---------------------------------------------------------------- router logits
 
 @pytest.mark.parametrize("T,H,E", [(64, 256, 8), (100, 384, 96), (128, 7168, 256), (1, 128, 1000),
-                                   (4096, 7168, 256)])
+                                   (4096, 7168, 256), (300, 384, 128), (1, 7168, 256),
+                                   (333, 1024, 384)])
 def test_router_logits(T, H, E):
+    """With a workspace and E % 128 == 0 the tensor-core path runs (three exact bf16
+    planes of Wr); without one the fp32 SIMT kernel does. Both stay within the
+    worst-case fp32 summation bound of the fp64 product."""
     cfg = L.config(T, H, E, min(8, E), 128)
     x = rand_bf16((T, H), 1)
     g = torch.Generator(device=DEV).manual_seed(2)
@@ -59,6 +63,12 @@ def test_router_logits(T, H, E):
     L.moe_router_logits(cfg, x, Wr, out3, ws if n else None)
     torch.cuda.synchronize()
     assert torch.equal(out, out3)
+    if E % 128 == 0:
+        # the three bf16 planes left in the workspace add up to Wr (to 2^-26 |w|)
+        planes = ws[: 3 * E * H * 2].view(torch.bfloat16).view(3, E, H).to(torch.float64)
+        recon = planes.sum(0).cpu().numpy()
+        assert (np.abs(recon - Wh) <= 2.0 ** -26 * np.abs(Wh)).all()
+        assert (planes[0] == Wr.to(torch.bfloat16).to(torch.float64)).all()
 
 
 # ---------------------------------------------------------------- gate / top-k

@@ -68,7 +68,9 @@ def check_routing(wl, d, a, L_oracle):
     np.testing.assert_array_equal(gidx, ridx)
     np.testing.assert_allclose(a["topk_w"].cpu().numpy(), rw, rtol=2e-5, atol=1e-7)
     oidx, _ = O.gate_topk(L_oracle, bias32(d["bias"]), cfg)
-    np.testing.assert_array_equal(gidx, oidx)   # margins make the oracle's own routing agree
+    # The margins (k-th vs (k+1)-th score, kept-group boundary) make the oracle's own
+    # routing pick the same experts; their order among the k slots is not margin-protected.
+    np.testing.assert_array_equal(np.sort(gidx, 1), np.sort(oidx, 1))
     np.testing.assert_array_equal(a["counts"].cpu().numpy(),
                                   np.bincount(ridx.reshape(-1), minlength=wl.E))
     return gidx

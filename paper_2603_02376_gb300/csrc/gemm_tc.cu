@@ -634,13 +634,15 @@ moe_status run_ffn(const FfnGroup& g0, const FfnGroup* g1, int H, int I, cudaStr
   moe_status st = launch_gemm<MODE_SWIGLU, NMAX>(a1, b1, sa1, sb1, args, s);
   if (st != MOE_OK) return st;
   if (after_gemm1 && cudaEventRecord(after_gemm1, s) != cudaSuccess) return MOE_ERR_CUDA;
-  // GEMM2: y = h W2^T (fp32); two 128-feature weight tiles per unit when H allows
+  // GEMM2: y = h W2^T (fp32). With prefill-sized token tiles, two 128-feature
+  // weight tiles per unit share one token tile (more weight bytes per stage);
+  // with decode-sized tiles a single weight tile and a deeper ring measured faster.
   args.K = I;
   args.w_rows0 = H;
   args.out0 = g0.y;
   args.out1 = g1 ? g1->y : nullptr;
   args.out_ld = H;
-  if (H % (2 * BM) == 0) {
+  if (NMAX > 32 && H % (2 * BM) == 0) {
     args.n_fb = H / (2 * BM);
     args.up_off = BM;
     return launch_gemm<MODE_PLAIN2, NMAX>(a2, b2, sa2, sb2, args, s);

@@ -181,6 +181,76 @@ __global__ void __launch_bounds__(PERM_WARPS * 32) perm_scatter_kernel(
   }
 }
 
+// The whole permutation in one CTA when the batch is a single chunk (decode):
+// the histogram, the scan over experts and the stable scatter of perm_hist /
+// perm_scan / perm_scatter, without two launches and the chunk tables.
+__global__ void __launch_bounds__(PERM_WARPS * 32) perm_single_kernel(
+    const int32_t* __restrict__ idx, int T, int k, int E, int32_t* __restrict__ counts,
+    int32_t* __restrict__ offsets, int32_t* __restrict__ row_src_token,
+    int32_t* __restrict__ slot_row, int* __restrict__ err) {
+  extern __shared__ int perm_smem[];  // [PERM_WARPS][E] histograms, then [E] totals
+  int* tot = perm_smem + PERM_WARPS * E;
+  for (int i = threadIdx.x; i < PERM_WARPS * E; i += blockDim.x) perm_smem[i] = 0;
+  __syncthreads();
+  const int w = threadIdx.x / 32, lane = threadIdx.x % 32;
+  long n0, n1;
+  warp_range(0, w, T, k, &n0, &n1);
+  int* hist_w = perm_smem + w * E;
+  warp_histogram(idx, n0, n1, E, hist_w, err);
+  __syncthreads();
+  for (int e = threadIdx.x; e < E; e += blockDim.x) {
+    int s = 0;
+    for (int q = 0; q < PERM_WARPS; ++q) s += perm_smem[q * E + e];
+    tot[e] = s;
+    counts[e] = s;
+  }
+  __syncthreads();
+  if (w == 0) {  // exclusive scan of the E totals by one warp, 32 experts per step
+    int base = 0;
+    for (int e0 = 0; e0 < E; e0 += 32) {
+      const int e = e0 + lane;
+      const int v = e < E ? tot[e] : 0;
+      int incl = v;
+#pragma unroll
+      for (int o = 1; o < 32; o <<= 1) {
+        const int u = __shfl_up_sync(0xffffffffu, incl, o);
+        if (lane >= o) incl += u;
+      }
+      if (e < E) {
+        offsets[e] = base + incl - v;
+        tot[e] = base + incl - v;
+      }
+      base += __shfl_sync(0xffffffffu, incl, 31);
+    }
+    if (lane == 0) offsets[E] = base;
+  }
+  __syncthreads();
+  for (int e = threadIdx.x; e < E; e += blockDim.x) {
+    int run = tot[e];
+    for (int q = 0; q < PERM_WARPS; ++q) {
+      const int v = perm_smem[q * E + e];
+      perm_smem[q * E + e] = run;
+      run += v;
+    }
+  }
+  __syncthreads();
+  const unsigned lt = lanemask_lt();
+  for (long base = n0; base < n1; base += 32) {
+    const long n = base + lane;
+    const int e = entry_expert(idx, n, n1, E, err);
+    const unsigned peers = __match_any_sync(0xffffffffu, e);
+    int row = 0;
+    if (e >= 0) row = hist_w[e] + __popc(peers & lt);
+    __syncwarp();
+    if (e >= 0 && lane == __ffs(peers) - 1) hist_w[e] += __popc(peers);
+    __syncwarp();
+    if (e >= 0) {
+      row_src_token[row] = (int32_t)(n / k);
+      slot_row[n] = row;
+    }
+  }
+}
+
 // x_perm[slot_row[t*k + j]] = x[t] for every token t and slot j (16-byte vectors).
 __global__ void dispatch_rows_kernel(const uint4* __restrict__ x, int T, int vpr, int k,
                                      const int32_t* __restrict__ slot_row,
@@ -292,6 +362,17 @@ moe_status launch_permutation(const moe_config& c, const int32_t* idx, int32_t* 
                               int32_t* offsets, int32_t* row_src_token, int32_t* slot_row,
                               int32_t* chunk_counts, int32_t* chunk_base, cudaStream_t s) {
   const int nch = perm_num_chunks(c.T);
+  if (nch == 1) {
+    const size_t smem1 = (size_t)(PERM_WARPS + 1) * c.E * sizeof(int);
+    if (smem1 > 48 * 1024)
+      cudaFuncSetAttribute(perm_single_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                           (int)smem1);
+    perm_single_kernel<<<1, PERM_WARPS * 32, smem1, s>>>(idx, c.T, c.k, c.E, counts, offsets,
+                                                         row_src_token, slot_row,
+                                                         device_error_word());
+    note_launch();
+    return launch_status();
+  }
   const size_t smem = (size_t)PERM_WARPS * c.E * sizeof(int);
   if (smem > 48 * 1024) {
     cudaFuncSetAttribute(perm_hist_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);

@@ -50,6 +50,8 @@ def parse():
     p.add_argument("--mode", choices=("seq", "overlap-tokens", "overlap-experts"), default="seq")
     p.add_argument("--chunk-tokens", type=int, default=512)
     p.add_argument("--expert-chunks", type=int, default=8)
+    p.add_argument("--no-fuse-gather", action="store_true",
+                   help="pack x_perm with a dispatch kernel instead of gathering in GEMM1")
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--cpu-tokens", type=int, default=128, help="oracle sample size (tokens)")
     return p.parse_args()
@@ -182,15 +184,19 @@ def calibrate(L, wl, d, device):
         d["bias"] = b.to(device)
 
 
-def algorithmic(wl, touched):
-    """Algorithmic bytes and flops of each stage for one forward."""
+def algorithmic(wl, touched, fused_gather=True):
+    """Algorithmic bytes and flops of each stage for one forward.
+
+    GEMM1's token operand is counted as R*H*2 either way (packed rows read, or
+    the same rows gathered from x); a fused dispatch has no stage of its own.
+    """
     T, H, E, k, Iw, Is = wl.T, wl.H, wl.E, wl.k, wl.I, wl.I_shared
     R = T * k
     b = {
         "router": T * H * 2 + E * H * 4 + T * E * 4,
         "gate": T * E * 4 + T * k * 8,
         "permute": T * k * 4 * 3,
-        "dispatch": T * H * 2 + R * H * 2,
+        "dispatch": 0 if fused_gather else T * H * 2 + R * H * 2,
         "gemm1": touched * 2 * Iw * H * 2 + R * H * 2 + R * Iw * 2,
         "gemm2": touched * H * Iw * 2 + R * Iw * 2 + R * H * 4,
         "shared_gemm1": (2 * Is * H * 2 + T * H * 2 + T * Is * 2) if Is else 0,
@@ -303,7 +309,8 @@ def config_of(wl, args):
     return {"workload": wl.name, "T": wl.T, "H": wl.H, "E": wl.E, "k": wl.k, "I": wl.I,
             "I_shared": wl.I_shared, "gating": ("sigmoid+bias, 8 groups keep 4, top-8, x2.5"
                                                 if wl.gate == 1 else "softmax top-k"),
-            "mode": args.mode, "global_batch": wl.T * args.gpus,
+            "mode": args.mode, "dispatch": "packed x_perm" if args.no_fuse_gather
+            else "fused into GEMM1 (TMA gather4)", "global_batch": wl.T * args.gpus,
             "l2": "inputs larger than L2: the expert weights streamed per step exceed 129 MB",
             "parallelism": f"replicas{args.gpus}"}
 
@@ -319,9 +326,11 @@ def run_ours(args, wl, rank, world, local, device):
                                "overlap-experts": dict(overlap=1, chunk_axis=1,
                                                        n_expert_chunks=args.expert_chunks)})[
         args.mode]
-    ex = L.exec_config(**mode)
+    fuse = 0 if args.no_fuse_gather else 1
+    ex = L.exec_config(fuse_gather=fuse, **mode)
     # one workspace serves the timed mode and the sequential stats / stage-event passes
-    ws = torch.empty(max(L.moe_workspace_size(cfg, ex), L.moe_workspace_size(cfg, L.exec_config())),
+    ws = torch.empty(max(L.moe_workspace_size(cfg, ex),
+                         L.moe_workspace_size(cfg, L.exec_config(fuse_gather=fuse))),
                      dtype=torch.uint8, device=device)
     out = torch.empty((wl.T, wl.H), dtype=torch.bfloat16, device=device)
     W = L.weights_struct(d["Wr"], d["bias"], d["W13"], d["W2"], d["Ws13"], d["Ws2"])
@@ -332,8 +341,8 @@ def run_ours(args, wl, rank, world, local, device):
 
     # routing statistics of this batch (touched experts set the GEMM weight bytes)
     counts = torch.empty(wl.E, dtype=torch.int32, device=device)
-    L.moe_layer_forward(cfg, L.exec_config(), W, d["x"], out, L.aux_struct(counts=counts), ws,
-                        stream)
+    L.moe_layer_forward(cfg, L.exec_config(fuse_gather=fuse), W, d["x"], out,
+                        L.aux_struct(counts=counts), ws, stream)
     L.moe_check_errors(stream)
     cnt = counts.cpu()
     touched = int((cnt > 0).sum())
@@ -374,7 +383,7 @@ def run_ours(args, wl, rank, world, local, device):
             e.record(stream)
     torch.cuda.synchronize()
     for i in range(K2):
-        exs = L.exec_config(stage_events=evs[i])
+        exs = L.exec_config(fuse_gather=fuse, stage_events=evs[i])
         L.moe_layer_forward(cfg, exs, W, d["x"], out, None, ws, stream)
     torch.cuda.synchronize()
     stage_ms = {}
@@ -424,7 +433,7 @@ def run_ours(args, wl, rank, world, local, device):
                    "ms_sequential_unchunked": round(sum(stage_ms.values()), 4)}
 
     hbm, tf_burst, tf_sust, src = peaks()
-    b, f = algorithmic(wl, touched)
+    b, f = algorithmic(wl, touched, bool(fuse))
     g1 = stage_ms["gemm1"] / 1e3
     achieved = b["gemm1"] / g1 / 1e9
     traffic = measured_traffic(wl.name)

@@ -82,9 +82,12 @@ typedef struct {
  *    the rows of expert range i+1 are packed while range i computes.
  *  n_expert_chunks number of expert ranges when chunk_axis = 1.
  *  out_fp32 0 = bf16 output, 1 = fp32 output.
+ *  fuse_gather 1 = the dispatch is fused into GEMM1: its operand loads gather
+ *    each expert's token rows straight from x (TMA gather4) and the packed
+ *    copy x_perm is never written; 0 = a dispatch kernel packs x_perm first.
  */
 typedef struct {
-  int32_t overlap, chunk_tokens, chunk_axis, n_expert_chunks, out_fp32;
+  int32_t overlap, chunk_tokens, chunk_axis, n_expert_chunks, out_fp32, fuse_gather;
   /* Optional tracing: an array of MOE_N_STAGE_EVENTS cudaEvent_t (created by
    * the caller) recorded on `stream` at the stage boundaries of a sequential
    * (overlap = 0) forward; NULL = no tracing. Ignored when overlap = 1. */

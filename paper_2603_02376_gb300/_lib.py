@@ -46,7 +46,8 @@ class moe_config(ctypes.Structure):
 
 class moe_exec(ctypes.Structure):
     _fields_ = [(n, ctypes.c_int32) for n in
-                ("overlap", "chunk_tokens", "chunk_axis", "n_expert_chunks", "out_fp32")] + \
+                ("overlap", "chunk_tokens", "chunk_axis", "n_expert_chunks", "out_fp32",
+                 "fuse_gather")] + \
                [("stage_events", ctypes.POINTER(ctypes.c_void_p))]
 
 
@@ -145,9 +146,9 @@ def config_of(wl, T=None) -> moe_config:
 
 
 def exec_config(overlap=0, chunk_tokens=512, chunk_axis=0, n_expert_chunks=8, out_fp32=0,
-                stage_events=None):
+                fuse_gather=1, stage_events=None):
     """moe_exec; stage_events: a list of MOE_N_STAGE_EVENTS torch.cuda.Event (or None)."""
-    ex = moe_exec(overlap, chunk_tokens, chunk_axis, n_expert_chunks, out_fp32, None)
+    ex = moe_exec(overlap, chunk_tokens, chunk_axis, n_expert_chunks, out_fp32, fuse_gather, None)
     if stage_events is not None:
         arr = (ctypes.c_void_p * MOE_N_STAGE_EVENTS)(*[int(e.cuda_event) for e in stage_events])
         ex._events_keepalive = arr

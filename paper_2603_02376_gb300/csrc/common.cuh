@@ -85,6 +85,10 @@ struct FfnGroup {
   const uint16_t* W2;
   uint16_t* h;  // [rows, I] bf16
   float* y;     // [rows, H] fp32
+  // Fused dispatch: packed row r of the group is row gather[r] of x (x_rows
+  // rows), read by GEMM1 directly; null = x is already packed.
+  const int32_t* gather;
+  int x_rows;
 };
 
 // Routed group plus an optional dense group (the shared expert, same I) in one

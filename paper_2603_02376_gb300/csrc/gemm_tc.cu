@@ -148,6 +148,17 @@ __device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap* map
       : "memory");
 }
 
+// Four rows (y0..y3) of a 2-D tensor whose map has a one-row box, landing as
+// four consecutive 128-byte rows of a swizzled tile (tile::gather4).
+__device__ __forceinline__ void tma_gather4(uint32_t dst, const CUtensorMap* map, int x, int y0,
+                                            int y1, int y2, int y3, uint32_t bar) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.shared::cluster.global.tile::gather4.mbarrier::complete_tx::bytes"
+      " [%0], [%1, {%2, %3, %4, %5, %6}], [%7];" ::"r"(dst),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y0), "r"(y1), "r"(y2), "r"(y3), "r"(bar)
+      : "memory");
+}
+
 __device__ __forceinline__ void tma_prefetch_map(const CUtensorMap* map) {
   asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(map)) : "memory");
 }
@@ -214,6 +225,7 @@ __device__ __forceinline__ void tmem_wait_ld() {
 // own activation matrix with one weight matrix (the shared expert).
 struct GemmArgs {
   const int32_t* offsets;
+  const int32_t* gather0;  // group 0: activation row of packed row r (fused dispatch), or null
   int rows0, e_begin, n_exp;
   int rows1;
   int K, n_fb;
@@ -367,56 +379,90 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
   const int total_units = units1 + tile_off[a.n_exp] * a.n_fb;
 
   if (warp == 0) {
+    // ------------------------------------------------------------------ producer
+    // Lane 0 owns the stage barriers and loads the weight tiles. Token rows are
+    // either one contiguous 16-row box at a time (packed activations), or -- when
+    // the dispatch is fused (a.gather0) -- gathered straight from x four rows per
+    // tile::gather4 load, every lane issuing the groups of four it holds the row
+    // indices of (registers, loaded once per unit).
     if (lane == 0) {
-      // ---------------------------------------------------------------- producer
       tma_prefetch_map(&tmA0);
       tma_prefetch_map(&tmB0);
       if (units1) {
         tma_prefetch_map(&tmA1);
         tma_prefetch_map(&tmB1);
       }
-      int stage = 0;
-      uint32_t phase = 0;
-      long fills = 0;
-      bool ok = true;
-      for (int u = blockIdx.x; u < total_units && ok; u += gridDim.x) {
-        const Unit U = decode_unit<NMAX>(u, tile_off, row_off, a, units1, kblocks);
-        const CUtensorMap* mA = U.grp ? &tmA1 : &tmA0;
-        const CUtensorMap* mB = U.grp ? &tmB1 : &tmB0;
-        const int n_pad = (U.m + 15) & ~15;
-        const int wrow = U.grp ? U.fb * TL::FEAT : (a.e_begin + U.e) * a.w_rows0 + U.fb * TL::FEAT;
-        const uint32_t bytes = TL::NA * TL::A_BYTES + n_pad * BK * 2;
-        for (int kb = U.kb0; kb < U.kb1; ++kb) {
-          const uint32_t full = smem_u32(&ctrl->full[stage]);
-          if (!wait_bounded(smem_u32(&ctrl->empty[stage]), phase ^ 1, abort_flag, err)) {
-            ok = false;
-            break;
-          }
-          mbar_arrive_expect_tx(full, bytes);
-          const uint32_t sa = smem_u32(smem + stage * TL::STAGE_BYTES);
+    }
+    int stage = 0;
+    uint32_t phase = 0;
+    long fills = 0;
+    bool ok = true;
+    for (int u = blockIdx.x; u < total_units && ok; u += gridDim.x) {
+      const Unit U = decode_unit<NMAX>(u, tile_off, row_off, a, units1, kblocks);
+      const CUtensorMap* mA = U.grp ? &tmA1 : &tmA0;
+      const CUtensorMap* mB = U.grp ? &tmB1 : &tmB0;
+      const int n_pad = (U.m + 15) & ~15;
+      const int wrow = U.grp ? U.fb * TL::FEAT : (a.e_begin + U.e) * a.w_rows0 + U.fb * TL::FEAT;
+      const uint32_t bytes = TL::NA * TL::A_BYTES + n_pad * BK * 2;
+      const bool gather = U.grp == 0 && a.gather0 != nullptr;
+      // rows of gather groups g = lane and g = lane + 32 (four rows each); rows past
+      // the tile's valid ones repeat its last row (their columns are never stored)
+      int gr[2][4];
+      const int n_groups = n_pad / 4;
 #pragma unroll
-          for (int t = 0; t < TL::NA; ++t)
-            tma_load_2d(sa + t * TL::A_BYTES, mA, kb * BK, wrow + t * a.up_off, full);
-          const uint32_t sb = sa + TL::NA * TL::A_BYTES;
-          for (int i = 0; i < n_pad / B_BOX; ++i)
-            tma_load_2d(sb + i * (B_BOX * BK * 2), mB, kb * BK, U.row0 + i * B_BOX, full);
-          ++fills;
-          if (++stage == TL::STAGES) {
-            stage = 0;
-            phase ^= 1;
+      for (int h = 0; h < 2; ++h)
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+          const int r = (lane + 32 * h) * 4 + j;
+          gr[h][j] = gather && r < n_pad ? a.gather0[U.row0 + min(r, U.m - 1)] : 0;
+        }
+      for (int kb = U.kb0; kb < U.kb1; ++kb) {
+        const uint32_t full = smem_u32(&ctrl->full[stage]);
+        const uint32_t sa = smem_u32(smem + stage * TL::STAGE_BYTES);
+        const uint32_t sb = sa + TL::NA * TL::A_BYTES;
+        int got = 1;
+        if (lane == 0) {
+          got = wait_bounded(smem_u32(&ctrl->empty[stage]), phase ^ 1, abort_flag, err) ? 1 : 0;
+          if (got) {
+            mbar_arrive_expect_tx(full, bytes);
+#pragma unroll
+            for (int t = 0; t < TL::NA; ++t)
+              tma_load_2d(sa + t * TL::A_BYTES, mA, kb * BK, wrow + t * a.up_off, full);
+            if (!gather)
+              for (int i = 0; i < n_pad / B_BOX; ++i)
+                tma_load_2d(sb + i * (B_BOX * BK * 2), mB, kb * BK, U.row0 + i * B_BOX, full);
           }
         }
-      }
-      if (!ok) {
-        // let the copies already issued land before the CTA can exit
-        for (int s = 0; s < TL::STAGES; ++s) {
-          if (fills <= s) continue;
-          const long f = s + ((fills - 1 - s) / TL::STAGES) * TL::STAGES;  // last fill of stage s
-          const uint32_t par = (uint32_t)((f / TL::STAGES) & 1);
-          const uint64_t t0 = global_timer_ns();
-          while (!mbar_try_wait(smem_u32(&ctrl->full[s]), par) &&
-                 global_timer_ns() - t0 < WAIT_LIMIT_NS) {
+        got = __shfl_sync(0xffffffffu, got, 0);
+        if (!got) {
+          ok = false;
+          break;
+        }
+        if (gather) {
+#pragma unroll
+          for (int h = 0; h < 2; ++h) {
+            const int g = lane + 32 * h;
+            if (g < n_groups)
+              tma_gather4(sb + g * (4 * BK * 2), mB, kb * BK, gr[h][0], gr[h][1], gr[h][2],
+                          gr[h][3], full);
           }
+        }
+        ++fills;
+        if (++stage == TL::STAGES) {
+          stage = 0;
+          phase ^= 1;
+        }
+      }
+    }
+    if (!ok && lane == 0) {
+      // let the copies already issued land before the CTA can exit
+      for (int s = 0; s < TL::STAGES; ++s) {
+        if (fills <= s) continue;
+        const long f = s + ((fills - 1 - s) / TL::STAGES) * TL::STAGES;  // last fill of stage s
+        const uint32_t par = (uint32_t)((f / TL::STAGES) & 1);
+        const uint64_t t0 = global_timer_ns();
+        while (!mbar_try_wait(smem_u32(&ctrl->full[s]), par) &&
+               global_timer_ns() - t0 < WAIT_LIMIT_NS) {
         }
       }
     }
@@ -598,8 +644,10 @@ template <int NMAX>
 moe_status run_ffn(const FfnGroup& g0, const FfnGroup* g1, int H, int I, cudaStream_t s,
                    cudaEvent_t after_gemm1) {
   CUtensorMap a1, b1, a2, b2, sa1, sb1, sa2, sb2;
+  // with a fused dispatch GEMM1 reads token rows of x by index: a one-row box
+  const bool gather = g0.gather != nullptr;
   if (!make_map(&a1, g0.W13, H, (uint64_t)g0.n_experts * 2 * I, BK, BM) ||
-      !make_map(&b1, g0.x, H, g0.rows, BK, B_BOX) ||
+      !make_map(&b1, g0.x, H, gather ? g0.x_rows : g0.rows, BK, gather ? 1 : B_BOX) ||
       !make_map(&a2, g0.W2, I, (uint64_t)g0.n_experts * H, BK, BM) ||
       !make_map(&b2, g0.h, I, g0.rows, BK, B_BOX))
     return MOE_ERR_CUDA;
@@ -624,6 +672,7 @@ moe_status run_ffn(const FfnGroup& g0, const FfnGroup* g1, int H, int I, cudaStr
   args.rows1 = g1 ? g1->rows : 0;
   args.err = device_error_word();
   // GEMM1 + SwiGLU: h = silu(x Wg^T) * (x Wu^T)
+  args.gather0 = g0.gather;
   args.K = H;
   args.n_fb = I / BM;
   args.w_rows0 = 2 * I;
@@ -634,6 +683,7 @@ moe_status run_ffn(const FfnGroup& g0, const FfnGroup* g1, int H, int I, cudaStr
   moe_status st = launch_gemm<MODE_SWIGLU, NMAX>(a1, b1, sa1, sb1, args, s);
   if (st != MOE_OK) return st;
   if (after_gemm1 && cudaEventRecord(after_gemm1, s) != cudaSuccess) return MOE_ERR_CUDA;
+  args.gather0 = nullptr;  // GEMM2 reads h, already in packed row order
   // GEMM2: y = h W2^T (fp32). With prefill-sized token tiles, two 128-feature
   // weight tiles per unit share one token tile (more weight bytes per stage);
   // with decode-sized tiles a single weight tile and a deeper ring measured faster.
@@ -701,7 +751,7 @@ moe_status launch_expert_ffn(int rows, int H, int I, int n_experts, int e_begin,
                              const uint16_t* W2, uint16_t* h, float* y_perm, int rows_hint,
                              cudaStream_t s, cudaEvent_t after_gemm1) {
   if (rows == 0 || e_end <= e_begin) return MOE_OK;
-  FfnGroup g{x_perm, offsets, rows, n_experts, e_begin, e_end, W13, W2, h, y_perm};
+  FfnGroup g{x_perm, offsets, rows, n_experts, e_begin, e_end, W13, W2, h, y_perm, nullptr, 0};
   return launch_expert_ffn_groups(g, nullptr, H, I, rows_hint, s, after_gemm1);
 }
 

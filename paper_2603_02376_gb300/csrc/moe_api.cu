@@ -84,6 +84,7 @@ bool valid_exec(const moe_exec* ex, const moe_config* c) {
   if (!ex) return false;
   if (ex->overlap != 0 && ex->overlap != 1) return false;
   if (ex->out_fp32 != 0 && ex->out_fp32 != 1) return false;
+  if (ex->fuse_gather != 0 && ex->fuse_gather != 1) return false;
   if (ex->overlap) {
     if (ex->chunk_axis == 0) {
       if (ex->chunk_tokens < 1) return false;
@@ -155,7 +156,7 @@ Layout carve(const moe_config& c, const moe_exec& ex, void* ws) {
   L.perm_base = cv.take<int32_t>((size_t)(L.perm_chunks + 1) * E);
   const size_t rws = router_workspace_bytes(cc);
   L.router_ws = rws ? static_cast<void*>(cv.take<uint8_t>(rws)) : nullptr;
-  L.x_perm = cv.take<uint16_t>(T * k * c.H);
+  L.x_perm = ex.fuse_gather ? nullptr : cv.take<uint16_t>(T * k * c.H);
   L.h = cv.take<uint16_t>(T * k * c.I);
   L.y_perm = cv.take<float>(T * k * c.H);
   L.sh_off = cv.take<int32_t>(2);
@@ -228,15 +229,38 @@ moe_status pack_tokens(const moe_config& c, const Layout& L, const moe_weights& 
 }
 
 // Routed experts of chunk ci (tokens [t0, t0+Tc)), experts [e0, e1), then nothing else.
-moe_status experts_tokens(const moe_config& c, const Layout& L, const moe_weights& w, int t0,
-                          int Tc, int ci, int e0, int e1, cudaStream_t s,
-                          cudaEvent_t* ev = nullptr) {
+// The routed operand group of tokens [t0, t0+Tc): packed rows of chunk ci, read
+// from x_perm or (fused dispatch) gathered from x by row_src_token.
+FfnGroup routed_group(const moe_config& c, const Layout& L, const moe_weights& w,
+                      const uint16_t* x, int t0, int Tc, int ci, int e0, int e1) {
   const size_t tk = (size_t)t0 * c.k;
-  const int rows = Tc * c.k;
-  const long hint = (long)rows * (e1 - e0) / c.E;
-  MOE_TRY(launch_expert_ffn(rows, c.H, c.I, c.E, e0, e1, L.x_perm + tk * c.H,
-                            L.offsets + (size_t)ci * (c.E + 1), w.W13, w.W2, L.h + tk * c.I,
-                            L.y_perm + tk * c.H, (int)hint, s, ev ? ev[MOE_EV_GEMM1] : nullptr));
+  FfnGroup g{};
+  g.rows = Tc * c.k;
+  g.offsets = L.offsets + (size_t)ci * (c.E + 1);
+  g.n_experts = c.E;
+  g.e_begin = e0;
+  g.e_end = e1;
+  g.W13 = w.W13;
+  g.W2 = w.W2;
+  g.h = L.h + tk * c.I;
+  g.y = L.y_perm + tk * c.H;
+  if (L.x_perm) {
+    g.x = L.x_perm + tk * c.H;
+  } else {
+    g.x = x + (size_t)t0 * c.H;
+    g.gather = L.rst + tk;
+    g.x_rows = Tc;
+  }
+  return g;
+}
+
+moe_status experts_tokens(const moe_config& c, const Layout& L, const moe_weights& w,
+                          const uint16_t* x, int t0, int Tc, int ci, int e0, int e1,
+                          cudaStream_t s, cudaEvent_t* ev = nullptr) {
+  const FfnGroup g = routed_group(c, L, w, x, t0, Tc, ci, e0, e1);
+  const long hint = (long)g.rows * (e1 - e0) / c.E;
+  MOE_TRY(launch_expert_ffn_groups(g, nullptr, c.H, c.I, (int)hint, s,
+                                   ev ? ev[MOE_EV_GEMM1] : nullptr));
   return mark(ev, MOE_EV_GEMM2, s);
 }
 
@@ -258,10 +282,9 @@ moe_status shared_expert(const moe_config& c, const Layout& L, const moe_weights
 moe_status experts_and_shared(const moe_config& c, const Layout& L, const moe_weights& w,
                               const uint16_t* x, cudaStream_t s, cudaEvent_t* ev) {
   MOE_TRY(launch_fill_range(L.sh_off, c.T, s));
-  const int rows = c.T * c.k;
-  FfnGroup routed{L.x_perm, L.offsets, rows, c.E, 0, c.E, w.W13, w.W2, L.h, L.y_perm};
-  FfnGroup dense{x, L.sh_off, c.T, 1, 0, 1, w.Ws13, w.Ws2, L.sh_h, L.sh_y};
-  MOE_TRY(launch_expert_ffn_groups(routed, &dense, c.H, c.I, rows, s,
+  const FfnGroup routed = routed_group(c, L, w, x, 0, c.T, 0, 0, c.E);
+  FfnGroup dense{x, L.sh_off, c.T, 1, 0, 1, w.Ws13, w.Ws2, L.sh_h, L.sh_y, nullptr, 0};
+  MOE_TRY(launch_expert_ffn_groups(routed, &dense, c.H, c.I, routed.rows, s,
                                    ev ? ev[MOE_EV_GEMM1] : nullptr));
   MOE_TRY(mark(ev, MOE_EV_GEMM2, s));
   MOE_TRY(mark(ev, MOE_EV_SHARED_GEMM1, s));
@@ -420,11 +443,11 @@ moe_status moe_layer_forward(const moe_config* cfg, const moe_exec* ex, const mo
   if (!ex->overlap) {
     cudaEvent_t* ev = reinterpret_cast<cudaEvent_t*>(ex->stage_events);
     MOE_TRY(mark(ev, MOE_EV_START, s));
-    MOE_TRY(pack_tokens(c, L, *w, x, 0, c.T, 0, true, s, ev));
+    MOE_TRY(pack_tokens(c, L, *w, x, 0, c.T, 0, L.x_perm != nullptr, s, ev));
     if (c.I_shared == c.I) {
       MOE_TRY(experts_and_shared(c, L, *w, x, s, ev));
     } else {
-      MOE_TRY(experts_tokens(c, L, *w, 0, c.T, 0, 0, c.E, s, ev));
+      MOE_TRY(experts_tokens(c, L, *w, x, 0, c.T, 0, 0, c.E, s, ev));
       MOE_TRY(shared_expert(c, L, *w, x, s, ev));
     }
     MOE_TRY(combine_tokens(c, L, 0, c.T, out, ex->out_fp32, s));
@@ -449,14 +472,14 @@ moe_status moe_layer_forward(const moe_config* cfg, const moe_exec* ex, const mo
     // chunk i's experts compute on `stream`.
     for (int ci = 0; ci < L.n_chunks; ++ci) {
       const int t0 = ci * L.chunk_T, Tc = c.T - t0 < L.chunk_T ? c.T - t0 : L.chunk_T;
-      MOE_TRY(pack_tokens(c, L, *w, x, t0, Tc, ci, true, ps));
+      MOE_TRY(pack_tokens(c, L, *w, x, t0, Tc, ci, L.x_perm != nullptr, ps));
       MOE_CUDA(cudaEventRecord(ev[ci], ps));
     }
     MOE_TRY(shared_expert(c, L, *w, x, s));  // overlaps the first chunk's packing
     for (int ci = 0; ci < L.n_chunks; ++ci) {
       const int t0 = ci * L.chunk_T, Tc = c.T - t0 < L.chunk_T ? c.T - t0 : L.chunk_T;
       MOE_CUDA(cudaStreamWaitEvent(s, ev[ci], 0));
-      MOE_TRY(experts_tokens(c, L, *w, t0, Tc, ci, 0, c.E, s));
+      MOE_TRY(experts_tokens(c, L, *w, x, t0, Tc, ci, 0, c.E, s));
       MOE_TRY(combine_tokens(c, L, t0, Tc, out, ex->out_fp32, s));
     }
     if (aux && aux->counts) MOE_TRY(launch_sum_counts(L.counts, L.n_chunks, c.E, aux->counts, s));
@@ -469,14 +492,15 @@ moe_status moe_layer_forward(const moe_config* cfg, const moe_exec* ex, const mo
   const int nr = ex->n_expert_chunks;
   for (int r = 0; r < nr; ++r) {
     const int e0 = (int)((long)c.E * r / nr), e1 = (int)((long)c.E * (r + 1) / nr);
-    MOE_TRY(launch_gather_rows(c.H, x, L.rst, L.offsets, e0, e1, L.x_perm, c.T * c.k, ps));
+    if (L.x_perm)  // with a fused dispatch GEMM1 gathers the rows itself
+      MOE_TRY(launch_gather_rows(c.H, x, L.rst, L.offsets, e0, e1, L.x_perm, c.T * c.k, ps));
     MOE_CUDA(cudaEventRecord(ev[r], ps));
   }
   MOE_TRY(shared_expert(c, L, *w, x, s));  // overlaps routing on the pack stream
   for (int r = 0; r < nr; ++r) {
     const int e0 = (int)((long)c.E * r / nr), e1 = (int)((long)c.E * (r + 1) / nr);
     MOE_CUDA(cudaStreamWaitEvent(s, ev[r], 0));
-    MOE_TRY(experts_tokens(c, L, *w, 0, c.T, 0, e0, e1, s));
+    MOE_TRY(experts_tokens(c, L, *w, x, 0, c.T, 0, e0, e1, s));
   }
   MOE_TRY(combine_tokens(c, L, 0, c.T, out, ex->out_fp32, s));
   if (aux && aux->counts)

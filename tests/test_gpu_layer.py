@@ -135,8 +135,12 @@ def test_layer_small_grouped_full(I_shared, T):
     d = I.layer_inputs(wl, seed=5, device=DEV)
     st = prepare_routing(wl, d)
     for ex in (L.exec_config(out_fp32=1), L.exec_config(out_fp32=0),
+               L.exec_config(out_fp32=1, fuse_gather=0),
                L.exec_config(out_fp32=1, overlap=1, chunk_axis=0, chunk_tokens=37),
-               L.exec_config(out_fp32=1, overlap=1, chunk_axis=1, n_expert_chunks=3)):
+               L.exec_config(out_fp32=1, overlap=1, chunk_axis=0, chunk_tokens=37, fuse_gather=0),
+               L.exec_config(out_fp32=1, overlap=1, chunk_axis=1, n_expert_chunks=3),
+               L.exec_config(out_fp32=1, overlap=1, chunk_axis=1, n_expert_chunks=3,
+                             fuse_gather=0)):
         out, a = run_layer(wl, d, ex)
         gidx = check_routing(wl, d, a, st["oracle_logits"])
         ref, _ = O.layer_forward(f64(d["x"]), f64(d["Wr"]), bias32(d["bias"]), f64(d["W13"]),
@@ -147,7 +151,7 @@ def test_layer_small_grouped_full(I_shared, T):
 
 # ---------------------------------------------------------------- decode: every token
 
-@pytest.mark.parametrize("ex", [dict(out_fp32=1), dict(out_fp32=0),
+@pytest.mark.parametrize("ex", [dict(out_fp32=1), dict(out_fp32=0), dict(out_fp32=1, fuse_gather=0),
                                 dict(out_fp32=1, overlap=1, chunk_axis=1, n_expert_chunks=4)])
 def test_layer_decode_full(big_weights, ex):
     wl = I.DECODE
@@ -179,6 +183,7 @@ def prefill_inputs(big_weights):
 @pytest.mark.parametrize("ex", [
     dict(out_fp32=1),
     dict(out_fp32=0),
+    dict(out_fp32=1, fuse_gather=0),
     dict(out_fp32=1, overlap=1, chunk_axis=0, chunk_tokens=512),
     dict(out_fp32=1, overlap=1, chunk_axis=1, n_expert_chunks=8),
 ])
@@ -200,7 +205,8 @@ def test_layer_skewed_sampled(big_weights):
     assert st["max_over_mean"] > 8.0   # a real hot expert
     toks = I.sample_tokens(wl.T, 256, 0).numpy()
     ref, _ = oracle_tokens(wl, d, toks)
-    for ex in (L.exec_config(out_fp32=1), L.exec_config(out_fp32=1, overlap=1, chunk_axis=1)):
+    for ex in (L.exec_config(out_fp32=1), L.exec_config(out_fp32=1, fuse_gather=0),
+               L.exec_config(out_fp32=1, overlap=1, chunk_axis=1)):
         out, a = run_layer(wl, d, ex)
         gidx = check_routing(wl, d, a, st["oracle_logits"])
         assert_layer_close(f64(out[torch.as_tensor(toks, device=DEV)]), ref)

@@ -82,9 +82,12 @@ typedef struct {
  *    the rows of expert range i+1 are packed while range i computes.
  *  n_expert_chunks number of expert ranges when chunk_axis = 1.
  *  out_fp32 0 = bf16 output, 1 = fp32 output.
- *  fuse_gather 1 = the dispatch is fused into GEMM1: its operand loads gather
- *    each expert's token rows straight from x (TMA gather4) and the packed
- *    copy x_perm is never written; 0 = a dispatch kernel packs x_perm first.
+ *  fuse_gather 1 = fuse the dispatch into GEMM1 when a (chunk of the) batch
+ *    averages at most 24 rows per expert (decode): GEMM1's operand loads then
+ *    gather each expert's token rows straight from x (TMA gather4) and the
+ *    packed copy x_perm is never written; larger batches, and 0, pack x_perm
+ *    with a dispatch kernel first (one gather instruction per four rows per
+ *    k-block costs more than the copy once tiles hold ~128 rows).
  */
 typedef struct {
   int32_t overlap, chunk_tokens, chunk_axis, n_expert_chunks, out_fp32, fuse_gather;

@@ -156,7 +156,12 @@ Layout carve(const moe_config& c, const moe_exec& ex, void* ws) {
   L.perm_base = cv.take<int32_t>((size_t)(L.perm_chunks + 1) * E);
   const size_t rws = router_workspace_bytes(cc);
   L.router_ws = rws ? static_cast<void*>(cv.take<uint8_t>(rws)) : nullptr;
-  L.x_perm = ex.fuse_gather ? nullptr : cv.take<uint16_t>(T * k * c.H);
+  // The fused dispatch (GEMM1 gathering rows with TMA gather4) pays one gather
+  // instruction per four token rows per k-block: a win for decode-sized tiles,
+  // measured 1.8x slower GEMM1 at ~128 rows per expert. It is used when a
+  // chunk averages at most 24 rows per expert.
+  const bool fuse = ex.fuse_gather && (long)L.chunk_T * c.k <= 24L * c.E;
+  L.x_perm = fuse ? nullptr : cv.take<uint16_t>(T * k * c.H);
   L.h = cv.take<uint16_t>(T * k * c.I);
   L.y_perm = cv.take<float>(T * k * c.H);
   L.sh_off = cv.take<int32_t>(2);

@@ -333,7 +333,8 @@ def run_ours(args, wl, rank, world, local, device):
     ex = L.exec_config(fuse_gather=fuse, **mode)
     # one workspace serves the timed mode and the sequential stats / stage-event passes
     ws = torch.empty(max(L.moe_workspace_size(cfg, ex),
-                         L.moe_workspace_size(cfg, L.exec_config(fuse_gather=fuse))),
+                         L.moe_workspace_size(cfg, L.exec_config(fuse_gather=fuse)),
+                         L.moe_workspace_size(cfg, L.exec_config(fuse_gather=0))),
                      dtype=torch.uint8, device=device)
     out = torch.empty((wl.T, wl.H), dtype=torch.bfloat16, device=device)
     W = L.weights_struct(d["Wr"], d["bias"], d["W13"], d["W2"], d["Ws13"], d["Ws2"])

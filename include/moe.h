@@ -269,6 +269,23 @@ moe_status moe_layer_forward(const moe_config* cfg, const moe_exec* ex, const mo
                              const uint16_t* x, void* out, const moe_aux* aux, void* ws,
                              size_t ws_bytes, void* stream, void* aux_stream);
 
+/*
+ * Testing hook for failure detection (no counterpart in the paper): exactly
+ * moe_expert_ffn, except that CTA 0 of each grouped GEMM never issues its
+ * producer fill number `stall_fill` (0-based), so the MMA's barrier wait on
+ * that stage cannot complete, and every barrier wait is limited to
+ * wait_limit_ns (1 ms .. 2 s). The kernel must then latch MOE_ERR_TIMEOUT,
+ * let its issued copies and MMAs finish (bounded), free its tensor memory
+ * and return; moe_check_errors() reports the timeout and the context stays
+ * usable. y_perm and the workspace hold garbage afterwards. Faults, traps and
+ * hangs are never used: the wait simply runs out.
+ */
+moe_status moe_testing_expert_ffn_stall(int32_t rows, int32_t H, int32_t I, int32_t n_experts,
+                                        const uint16_t* x_perm, const int32_t* offsets,
+                                        const uint16_t* W13, const uint16_t* W2, float* y_perm,
+                                        void* ws, size_t ws_bytes, int64_t stall_fill,
+                                        int64_t wait_limit_ns, void* stream);
+
 /* Synchronises `stream`, then reads and clears the device error word of the
  * current device. MOE_OK, MOE_ERR_TIMEOUT or MOE_ERR_DEVICE_CHECK (or
  * MOE_ERR_CUDA if the synchronisation itself failed). */

@@ -28,7 +28,8 @@ EXPORTS = ("moe_status_string", "moe_validate_config", "moe_workspace_size",
            "moe_router_workspace_size", "moe_dispatch_workspace_size",
            "moe_expert_ffn_workspace_size", "moe_router_logits", "moe_gate_topk", "moe_dispatch",
            "moe_expert_ffn", "moe_combine", "moe_layer_forward", "moe_check_errors",
-           "moe_launch_count", "moe_shutdown", "moe_dispatch_noalloc")
+           "moe_launch_count", "moe_shutdown", "moe_dispatch_noalloc",
+           "moe_testing_expert_ffn_stall")
 MOE_DISPATCH_NOALLOC_MAX_ENTRIES = 131072
 
 
@@ -92,6 +93,8 @@ def load(path: str = LIB_PATH) -> ctypes.CDLL:
         "moe_dispatch_noalloc": (S, [cfgp, P, P, P, P, P, P, P, P]),
         "moe_expert_ffn": (S, [I32, I32, I32, I32, P, P, P, P, P, P, SZ, P]),
         "moe_combine": (S, [cfgp, P, P, P, P, P, I32, P]),
+        "moe_testing_expert_ffn_stall": (S, [I32, I32, I32, I32, P, P, P, P, P, P, SZ,
+                                             ctypes.c_int64, ctypes.c_int64, P]),
         "moe_layer_forward": (S, [cfgp, exp, ctypes.POINTER(moe_weights), P, P,
                                   ctypes.POINTER(moe_aux), P, SZ, P, P]),
         "moe_check_errors": (S, [P]),
@@ -211,6 +214,16 @@ def moe_expert_ffn(rows, H, I, n_experts, x_perm, offsets, W13, W2, y_perm, ws,
     _check(load().moe_expert_ffn(rows, H, I, n_experts, _ptr(x_perm), _ptr(offsets), _ptr(W13),
                                  _ptr(W2), _ptr(y_perm), _ptr(ws), nb, _stream(stream)),
            "moe_expert_ffn")
+
+
+def moe_testing_expert_ffn_stall(rows, H, I, n_experts, x_perm, offsets, W13, W2, y_perm, ws,
+                                 stall_fill, wait_limit_ns, stream=None) -> int:
+    """Failure-detection hook: returns the launch status (the timeout shows in moe_check_errors)."""
+    nb = 0 if ws is None else ws.numel() * ws.element_size()
+    return load().moe_testing_expert_ffn_stall(rows, H, I, n_experts, _ptr(x_perm), _ptr(offsets),
+                                               _ptr(W13), _ptr(W2), _ptr(y_perm), _ptr(ws), nb,
+                                               int(stall_fill), int(wait_limit_ns),
+                                               _stream(stream))
 
 
 def moe_combine(cfg, y_perm, slot_row, topk_w, shared_out, out, out_fp32, stream=None) -> None:

@@ -97,6 +97,13 @@ moe_status launch_expert_ffn_groups(const FfnGroup& routed, const FfnGroup* dens
                                     int rows_hint, cudaStream_t s,
                                     cudaEvent_t after_gemm1 = nullptr);
 
+// Testing: moe_expert_ffn whose GEMM1 has one producer fill of CTA 0 never issued,
+// with the given barrier-wait limit (exercises the timeout and abort path).
+moe_status launch_expert_ffn_stalled(int rows, int H, int I, int n_experts, const uint16_t* x_perm,
+                                     const int32_t* offsets, const uint16_t* W13,
+                                     const uint16_t* W2, uint16_t* h, float* y_perm,
+                                     long stall_fill, uint64_t wait_limit_ns, cudaStream_t s);
+
 // Grouped expert GEMM on tcgen05. Experts [e_begin, e_end) of `offsets`.
 moe_status launch_expert_ffn(int rows, int H, int I, int n_experts, int e_begin, int e_end,
                              const uint16_t* x_perm, const int32_t* offsets, const uint16_t* W13,

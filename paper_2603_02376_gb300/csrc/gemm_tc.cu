@@ -45,7 +45,7 @@ constexpr int BK = 64;            // bf16 per stage along K: one 128-byte swizzl
 constexpr int UMMA_K = 16;        // K of one tcgen05.mma kind::f16
 constexpr int B_BOX = 16;         // token rows per TMA box
 constexpr int NUM_THREADS = 192;  // 6 warps
-constexpr uint64_t WAIT_LIMIT_NS = 2000000000ull;
+constexpr uint64_t WAIT_LIMIT_NS = 2000000000ull;  // default limit of every barrier wait
 
 
 
@@ -125,13 +125,13 @@ __device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
 
 // Wait for the phase of `bar` with the given parity; false on abort or timeout.
 __device__ __noinline__ bool wait_bounded(uint32_t bar, uint32_t parity, volatile int* abort_flag,
-                                          int* err) {
+                                          int* err, uint64_t limit_ns) {
   if (mbar_try_wait(bar, parity)) return true;
   const uint64_t t0 = global_timer_ns();
   while (true) {
     if (mbar_try_wait(bar, parity)) return true;
     if (*abort_flag) return false;
-    if (global_timer_ns() - t0 > WAIT_LIMIT_NS) {
+    if (global_timer_ns() - t0 > limit_ns) {
       *abort_flag = 1;
       atomicExch(err, (int)MOE_ERR_TIMEOUT);
       return false;
@@ -237,6 +237,9 @@ struct GemmArgs {
   void* out1;
   int out_ld;
   int* err;
+  uint64_t wait_limit_ns;  // limit of each barrier wait
+  long stall_fill;         // testing: CTA 0 never issues this fill (-1 = none), so the
+                           // MMA's wait on it runs out and the abort path is exercised
 };
 
 struct Unit {
@@ -422,8 +425,12 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
         const uint32_t sb = sa + TL::NA * TL::A_BYTES;
         int got = 1;
         if (lane == 0) {
-          got = wait_bounded(smem_u32(&ctrl->empty[stage]), phase ^ 1, abort_flag, err) ? 1 : 0;
-          if (got) {
+          got = wait_bounded(smem_u32(&ctrl->empty[stage]), phase ^ 1, abort_flag, err,
+                             a.wait_limit_ns)
+                    ? 1
+                    : 0;
+          if (got && blockIdx.x == 0 && fills == a.stall_fill) got = 2;  // skip this fill
+          if (got == 1) {
             mbar_arrive_expect_tx(full, bytes);
 #pragma unroll
             for (int t = 0; t < TL::NA; ++t)
@@ -438,7 +445,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
           ok = false;
           break;
         }
-        if (gather) {
+        if (gather && got == 1) {
 #pragma unroll
           for (int h = 0; h < 2; ++h) {
             const int g = lane + 32 * h;
@@ -459,10 +466,11 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       for (int s = 0; s < TL::STAGES; ++s) {
         if (fills <= s) continue;
         const long f = s + ((fills - 1 - s) / TL::STAGES) * TL::STAGES;  // last fill of stage s
+        if (blockIdx.x == 0 && f == a.stall_fill) continue;  // never issued
         const uint32_t par = (uint32_t)((f / TL::STAGES) & 1);
         const uint64_t t0 = global_timer_ns();
         while (!mbar_try_wait(smem_u32(&ctrl->full[s]), par) &&
-               global_timer_ns() - t0 < WAIT_LIMIT_NS) {
+               global_timer_ns() - t0 < a.wait_limit_ns) {
         }
       }
     }
@@ -479,14 +487,16 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
         const uint32_t idesc = idesc_bf16(n_pad);
         const int as = j % TL::ACC_STAGES;
         const uint32_t acc_par = (uint32_t)((j / TL::ACC_STAGES) & 1);
-        if (!wait_bounded(smem_u32(&ctrl->acc_empty[as]), acc_par ^ 1, abort_flag, err)) {
+        if (!wait_bounded(smem_u32(&ctrl->acc_empty[as]), acc_par ^ 1, abort_flag, err,
+                          a.wait_limit_ns)) {
           ok = false;
           break;
         }
         tc_fence_after();
         const uint32_t d = tmem_base + (uint32_t)(as * TL::ACC_COLS);
         for (int kb = U.kb0; kb < U.kb1; ++kb) {
-          if (!wait_bounded(smem_u32(&ctrl->full[stage]), phase, abort_flag, err)) {
+          if (!wait_bounded(smem_u32(&ctrl->full[stage]), phase, abort_flag, err,
+                            a.wait_limit_ns)) {
             ok = false;
             break;
           }
@@ -520,7 +530,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
         mma_commit(smem_u32(&ctrl->drain));
         const uint64_t t0 = global_timer_ns();
         while (!mbar_try_wait(smem_u32(&ctrl->drain), 0) &&
-               global_timer_ns() - t0 < WAIT_LIMIT_NS) {
+               global_timer_ns() - t0 < a.wait_limit_ns) {
         }
       }
     }
@@ -532,7 +542,8 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       const Unit U = decode_unit<NMAX>(u, tile_off, row_off, a, units1, kblocks);
       const int as = j % TL::ACC_STAGES;
       const uint32_t acc_par = (uint32_t)((j / TL::ACC_STAGES) & 1);
-      if (!wait_bounded(smem_u32(&ctrl->acc_full[as]), acc_par, abort_flag, err)) break;
+      if (!wait_bounded(smem_u32(&ctrl->acc_full[as]), acc_par, abort_flag, err, a.wait_limit_ns))
+        break;
       tc_fence_after();
       const uint32_t tq = tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(as * TL::ACC_COLS);
       const int f = U.fb * TL::FEAT + q * 32 + lane;
@@ -621,6 +632,11 @@ bool make_map(CUtensorMap* m, const void* ptr, uint64_t inner, uint64_t outer, u
             CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+// Barrier-wait limit and injected stall of the expert-FFN launches: WAIT_LIMIT_NS
+// and none, except inside moe_testing_expert_ffn_stall (one host thread).
+uint64_t g_wait_limit_ns = WAIT_LIMIT_NS;
+long g_stall_fill = -1;
+
 template <int MODE, int NMAX>
 size_t gemm_smem_bytes(int n_exp) {
   using TL = Tile<MODE, NMAX>;
@@ -665,6 +681,8 @@ moe_status run_ffn(const FfnGroup& g0, const FfnGroup* g1, int H, int I, cudaStr
   }
   GemmArgs args{};
   args.k_splits = 1;
+  args.wait_limit_ns = g_wait_limit_ns;
+  args.stall_fill = g_stall_fill;
   args.offsets = g0.offsets;
   args.rows0 = g0.rows;
   args.e_begin = g0.e_begin;
@@ -734,6 +752,8 @@ moe_status launch_router_tc(int T, int H, int E, const uint16_t* x, const uint16
   if (!make_map(&A, planes, H, (uint64_t)3 * E, BK, BM) || !make_map(&B, x, H, T, BK, B_BOX))
     return MOE_ERR_CUDA;
   GemmArgs args{};
+  args.wait_limit_ns = WAIT_LIMIT_NS;
+  args.stall_fill = -1;
   args.rows1 = T;  // group 1: all tokens; group 0 is empty
   args.K = H;
   args.n_fb = E / BM;
@@ -744,6 +764,19 @@ moe_status launch_router_tc(int T, int H, int E, const uint16_t* x, const uint16
   args.out_ld = E;
   args.err = device_error_word();
   return launch_gemm<MODE_SPLIT3, 128>(A, B, A, B, args, s);
+}
+
+moe_status launch_expert_ffn_stalled(int rows, int H, int I, int n_experts, const uint16_t* x_perm,
+                                     const int32_t* offsets, const uint16_t* W13,
+                                     const uint16_t* W2, uint16_t* h, float* y_perm,
+                                     long stall_fill, uint64_t wait_limit_ns, cudaStream_t s) {
+  g_wait_limit_ns = wait_limit_ns;
+  g_stall_fill = stall_fill;
+  FfnGroup g{x_perm, offsets, rows, n_experts, 0, n_experts, W13, W2, h, y_perm, nullptr, 0};
+  const moe_status st = launch_expert_ffn_groups(g, nullptr, H, I, rows, s);
+  g_wait_limit_ns = WAIT_LIMIT_NS;
+  g_stall_fill = -1;
+  return st;
 }
 
 moe_status launch_expert_ffn(int rows, int H, int I, int n_experts, int e_begin, int e_end,

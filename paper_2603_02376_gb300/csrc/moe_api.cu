@@ -407,6 +407,25 @@ moe_status moe_expert_ffn(int32_t rows, int32_t H, int32_t I, int32_t n_experts,
                            (uint16_t*)ws, y_perm, rows, (cudaStream_t)stream);
 }
 
+moe_status moe_testing_expert_ffn_stall(int32_t rows, int32_t H, int32_t I, int32_t n_experts,
+                                        const uint16_t* x_perm, const int32_t* offsets,
+                                        const uint16_t* W13, const uint16_t* W2, float* y_perm,
+                                        void* ws, size_t ws_bytes, int64_t stall_fill,
+                                        int64_t wait_limit_ns, void* stream) {
+  if (rows < 1 || H < 128 || H % 128 || H > 65536 || I < 128 || I % 128 || I > 65536 ||
+      n_experts < 1 || n_experts > 1024 || stall_fill < 0 || wait_limit_ns < 1000000 ||
+      wait_limit_ns > 2000000000LL)
+    return MOE_ERR_INVALID_ARG;
+  if (!x_perm || !offsets || !W13 || !W2 || !y_perm || !aligned16(x_perm) || !aligned16(W13) ||
+      !aligned16(W2) || !aligned16(y_perm) || !aligned4(offsets))
+    return MOE_ERR_INVALID_ARG;
+  if (!ws || ws_bytes < moe_expert_ffn_workspace_size(rows, I) || !aligned16(ws))
+    return MOE_ERR_WORKSPACE;
+  return launch_expert_ffn_stalled(rows, H, I, n_experts, x_perm, offsets, W13, W2,
+                                   (uint16_t*)ws, y_perm, (long)stall_fill,
+                                   (uint64_t)wait_limit_ns, (cudaStream_t)stream);
+}
+
 moe_status moe_combine(const moe_config* cfg, const float* y_perm, const int32_t* slot_row,
                        const float* topk_w, const float* shared_out, void* out,
                        int32_t out_fp32, void* stream) {

@@ -52,6 +52,8 @@ def parse():
     p.add_argument("--expert-chunks", type=int, default=8)
     p.add_argument("--no-fuse-gather", action="store_true",
                    help="pack x_perm with a dispatch kernel instead of gathering in GEMM1")
+    p.add_argument("--no-pack", action="store_true",
+                   help="keep the expert weights row-major instead of tile-packed at load")
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--cpu-tokens", type=int, default=128, help="oracle sample size (tokens)")
     return p.parse_args()
@@ -311,6 +313,7 @@ def config_of(wl, args):
                                                 if wl.gate == 1 else "softmax top-k"),
             "mode": args.mode, "dispatch": "fused into GEMM1 (TMA gather4)"
             if (not args.no_fuse_gather and wl.T * wl.k <= 24 * wl.E) else "packed x_perm",
+            "weights": "row-major" if args.no_pack else "tile-packed at load (moe_pack_weights)",
             "global_batch": wl.T * args.gpus,
             "l2": "inputs larger than L2: the expert weights streamed per step exceed 129 MB",
             "parallelism": f"replicas{args.gpus}"}
@@ -337,8 +340,15 @@ def run_ours(args, wl, rank, world, local, device):
                          L.moe_workspace_size(cfg, L.exec_config(fuse_gather=0))),
                      dtype=torch.uint8, device=device)
     out = torch.empty((wl.T, wl.H), dtype=torch.bfloat16, device=device)
-    W = L.weights_struct(d["Wr"], d["bias"], d["W13"], d["W2"], d["Ws13"], d["Ws2"])
     stream = torch.cuda.current_stream()
+    # the layer runs on tile-packed copies (a load-time layout transform, not part
+    # of the timed step); the row-major tensors stay for the CPU oracle
+    run_w = {k_: d.get(k_) for k_ in ("W13", "W2", "Ws13", "Ws2")}
+    if not args.no_pack:
+        run_w = {k_: (None if v is None else L.pack_weights(v)) for k_, v in run_w.items()}
+        torch.cuda.synchronize()
+    W = L.weights_struct(d["Wr"], d["bias"], run_w["W13"], run_w["W2"], run_w["Ws13"],
+                         run_w["Ws2"], 0 if args.no_pack else 1)
 
     def step():
         L.moe_layer_forward(cfg, ex, W, d["x"], out, None, ws, stream)

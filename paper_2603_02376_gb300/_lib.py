@@ -29,7 +29,7 @@ EXPORTS = ("moe_status_string", "moe_validate_config", "moe_workspace_size",
            "moe_expert_ffn_workspace_size", "moe_router_logits", "moe_gate_topk", "moe_dispatch",
            "moe_expert_ffn", "moe_combine", "moe_layer_forward", "moe_check_errors",
            "moe_launch_count", "moe_shutdown", "moe_dispatch_noalloc",
-           "moe_testing_expert_ffn_stall")
+           "moe_testing_expert_ffn_stall", "moe_pack_weights")
 MOE_DISPATCH_NOALLOC_MAX_ENTRIES = 131072
 
 
@@ -58,7 +58,8 @@ MOE_N_STAGE_EVENTS = len(STAGES)
 
 
 class moe_weights(ctypes.Structure):
-    _fields_ = [(n, ctypes.c_void_p) for n in ("Wr", "bias", "W13", "W2", "Ws13", "Ws2")]
+    _fields_ = [(n, ctypes.c_void_p) for n in ("Wr", "bias", "W13", "W2", "Ws13", "Ws2")] + \
+               [("packed", ctypes.c_int32)]
 
 
 class moe_aux(ctypes.Structure):
@@ -91,7 +92,8 @@ def load(path: str = LIB_PATH) -> ctypes.CDLL:
         "moe_gate_topk": (S, [cfgp, P, P, P, P, P]),
         "moe_dispatch": (S, [cfgp, P, P, P, P, P, P, P, P, SZ, P]),
         "moe_dispatch_noalloc": (S, [cfgp, P, P, P, P, P, P, P, P]),
-        "moe_expert_ffn": (S, [I32, I32, I32, I32, P, P, P, P, P, P, SZ, P]),
+        "moe_expert_ffn": (S, [I32, I32, I32, I32, P, P, P, P, P, P, SZ, I32, P]),
+        "moe_pack_weights": (S, [ctypes.c_int64, I32, P, P, P]),
         "moe_combine": (S, [cfgp, P, P, P, P, P, I32, P]),
         "moe_testing_expert_ffn_stall": (S, [I32, I32, I32, I32, P, P, P, P, P, P, SZ,
                                              ctypes.c_int64, ctypes.c_int64, P]),
@@ -209,11 +211,28 @@ def moe_dispatch_noalloc(cfg, x, topk_idx, counts, offsets, row_src_token, slot_
 
 
 def moe_expert_ffn(rows, H, I, n_experts, x_perm, offsets, W13, W2, y_perm, ws,
-                   stream=None) -> None:
+                   stream=None, weights_packed=0) -> None:
     nb = 0 if ws is None else ws.numel() * ws.element_size()
     _check(load().moe_expert_ffn(rows, H, I, n_experts, _ptr(x_perm), _ptr(offsets), _ptr(W13),
-                                 _ptr(W2), _ptr(y_perm), _ptr(ws), nb, _stream(stream)),
+                                 _ptr(W2), _ptr(y_perm), _ptr(ws), nb, int(weights_packed),
+                                 _stream(stream)),
            "moe_expert_ffn")
+
+
+def moe_pack_weights(W, W_packed, stream=None) -> None:
+    """Tile-packed copy of a bf16 weight tensor viewed as [rows, K] (K = its last dim)."""
+    K = W.shape[-1]
+    rows = W.numel() // K
+    _check(load().moe_pack_weights(rows, K, _ptr(W), _ptr(W_packed), _stream(stream)),
+           "moe_pack_weights")
+
+
+def pack_weights(W, stream=None):
+    """A new tensor holding W (bf16, rows a multiple of 128) in the tile-packed layout."""
+    import torch
+    out = torch.empty_like(W)
+    moe_pack_weights(W, out, stream)
+    return out
 
 
 def moe_testing_expert_ffn_stall(rows, H, I, n_experts, x_perm, offsets, W13, W2, y_perm, ws,
@@ -232,9 +251,9 @@ def moe_combine(cfg, y_perm, slot_row, topk_w, shared_out, out, out_fp32, stream
            "moe_combine")
 
 
-def weights_struct(Wr, bias, W13, W2, Ws13=None, Ws2=None) -> moe_weights:
+def weights_struct(Wr, bias, W13, W2, Ws13=None, Ws2=None, packed=0) -> moe_weights:
     return moe_weights(*(None if t is None else t.data_ptr()
-                         for t in (Wr, bias, W13, W2, Ws13, Ws2)))
+                         for t in (Wr, bias, W13, W2, Ws13, Ws2)), int(packed))
 
 
 def aux_struct(logits=None, topk_idx=None, topk_w=None, counts=None) -> moe_aux:

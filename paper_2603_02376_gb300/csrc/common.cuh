@@ -89,6 +89,7 @@ struct FfnGroup {
   // rows), read by GEMM1 directly; null = x is already packed.
   const int32_t* gather;
   int x_rows;
+  bool packed;  // W13 / W2 in the tile-packed layout (moe_pack_weights)
 };
 
 // Routed group plus an optional dense group (the shared expert, same I) in one
@@ -108,7 +109,11 @@ moe_status launch_expert_ffn_stalled(int rows, int H, int I, int n_experts, cons
 moe_status launch_expert_ffn(int rows, int H, int I, int n_experts, int e_begin, int e_end,
                              const uint16_t* x_perm, const int32_t* offsets, const uint16_t* W13,
                              const uint16_t* W2, uint16_t* h, float* y_perm, int rows_hint,
-                             cudaStream_t s, cudaEvent_t after_gemm1 = nullptr);
+                             cudaStream_t s, cudaEvent_t after_gemm1 = nullptr,
+                             bool packed = false);
+
+// Tile-packed copy of a bf16 weight matrix [rows, K] (rows % 128 == 0, K % 64 == 0).
+moe_status launch_pack_weights(const uint16_t* W, uint16_t* Wp, long rows, int K, cudaStream_t s);
 
 // ----------------------------------------------------------------------------
 // device helpers

@@ -43,7 +43,8 @@ namespace {
 constexpr int BM = 128;           // weight rows per tile (MMA M)
 constexpr int BK = 64;            // bf16 per stage along K: one 128-byte swizzle row
 constexpr int UMMA_K = 16;        // K of one tcgen05.mma kind::f16
-constexpr int B_BOX = 16;         // token rows per TMA box
+constexpr int B_BOX = 16;         // token rows per TMA box (tile remainders)
+constexpr int B_BIG = 64;         // token rows per TMA box (bulk of tiles of >= 64 rows)
 constexpr int NUM_THREADS = 192;  // 6 warps
 constexpr uint64_t WAIT_LIMIT_NS = 2000000000ull;  // default limit of every barrier wait
 
@@ -148,6 +149,17 @@ __device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap* map
       : "memory");
 }
 
+// One 128-row x 64-column weight tile of the tile-packed layout: a 3-D map
+// {64 columns, 128 rows, tiles} whose box is one whole tile (16 KiB, contiguous).
+__device__ __forceinline__ void tma_load_tile3d(uint32_t dst, const CUtensorMap* map, int tile,
+                                                uint32_t bar) {
+  asm volatile(
+      "cp.async.bulk.tensor.3d.shared::cluster.global.mbarrier::complete_tx::bytes"
+      " [%0], [%1, {%2, %3, %4}], [%5];" ::"r"(dst),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(0), "r"(0), "r"(tile), "r"(bar)
+      : "memory");
+}
+
 // Four rows (y0..y3) of a 2-D tensor whose map has a one-row box, landing as
 // four consecutive 128-byte rows of a swizzled tile (tile::gather4).
 __device__ __forceinline__ void tma_gather4(uint32_t dst, const CUtensorMap* map, int x, int y0,
@@ -231,6 +243,7 @@ struct GemmArgs {
   int K, n_fb;
   int w_rows0;  // weight rows per expert in group 0
   int up_off;   // row offset between a unit's weight tiles (SwiGLU: the up projection)
+  int a_packed;  // weights (A) in the tile-packed layout: 3-D maps, tile = (row/128)*kblocks + kb
   int k_splits; // group 1 only: the K range is split into this many units ...
   long split_stride;  // ... whose outputs go to out1 + split * split_stride (partials)
   void* out0;
@@ -301,7 +314,9 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
     grouped_gemm_kernel(const __grid_constant__ CUtensorMap tmA0,
                         const __grid_constant__ CUtensorMap tmB0,
                         const __grid_constant__ CUtensorMap tmA1,
-                        const __grid_constant__ CUtensorMap tmB1, const GemmArgs a) {
+                        const __grid_constant__ CUtensorMap tmB1,
+                        const __grid_constant__ CUtensorMap tmB0big,
+                        const __grid_constant__ CUtensorMap tmB1big, const GemmArgs a) {
   using TL = Tile<MODE, NMAX>;
   constexpr bool SWIGLU = MODE == MODE_SWIGLU;
   extern __shared__ uint8_t smem_raw[];
@@ -404,7 +419,10 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       const Unit U = decode_unit<NMAX>(u, tile_off, row_off, a, units1, kblocks);
       const CUtensorMap* mA = U.grp ? &tmA1 : &tmA0;
       const CUtensorMap* mB = U.grp ? &tmB1 : &tmB0;
+      const CUtensorMap* mBbig = U.grp ? &tmB1big : &tmB0big;
       const int n_pad = (U.m + 15) & ~15;
+      // 64-row boxes for the bulk of a packed token tile, 16-row boxes for the rest
+      const int n_big = NMAX >= B_BIG ? n_pad / B_BIG : 0;
       const int wrow = U.grp ? U.fb * TL::FEAT : (a.e_begin + U.e) * a.w_rows0 + U.fb * TL::FEAT;
       const uint32_t bytes = TL::NA * TL::A_BYTES + n_pad * BK * 2;
       const bool gather = U.grp == 0 && a.gather0 != nullptr;
@@ -433,11 +451,19 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
           if (got == 1) {
             mbar_arrive_expect_tx(full, bytes);
 #pragma unroll
-            for (int t = 0; t < TL::NA; ++t)
-              tma_load_2d(sa + t * TL::A_BYTES, mA, kb * BK, wrow + t * a.up_off, full);
-            if (!gather)
-              for (int i = 0; i < n_pad / B_BOX; ++i)
+            for (int t = 0; t < TL::NA; ++t) {
+              const int r = wrow + t * a.up_off;
+              if (a.a_packed)
+                tma_load_tile3d(sa + t * TL::A_BYTES, mA, (r / BM) * kblocks + kb, full);
+              else
+                tma_load_2d(sa + t * TL::A_BYTES, mA, kb * BK, r, full);
+            }
+            if (!gather) {
+              for (int i = 0; i < n_big; ++i)
+                tma_load_2d(sb + i * (B_BIG * BK * 2), mBbig, kb * BK, U.row0 + i * B_BIG, full);
+              for (int i = n_big * (B_BIG / B_BOX); i < n_pad / B_BOX; ++i)
                 tma_load_2d(sb + i * (B_BOX * BK * 2), mB, kb * BK, U.row0 + i * B_BOX, full);
+            }
           }
         }
         got = __shfl_sync(0xffffffffu, got, 0);
@@ -562,7 +588,9 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
             if (c0 + i < U.m) {
               const float gv = __uint_as_float(g[i]);
               const float uv = __uint_as_float(v[i]);
-              const float hv = gv / (1.0f + expf(-gv)) * uv;
+              // silu(g) * u with the hardware exp2-based __expf and a reciprocal:
+              // their error (a few fp32 ulp) is far below the bf16 rounding of h
+              const float hv = gv * __frcp_rn(1.0f + __expf(-gv)) * uv;
               static_cast<uint16_t*>(out)[o + (size_t)(c0 + i) * a.out_ld] = float_to_bf16_bits(hv);
             }
           }
@@ -637,6 +665,25 @@ bool make_map(CUtensorMap* m, const void* ptr, uint64_t inner, uint64_t outer, u
 uint64_t g_wait_limit_ns = WAIT_LIMIT_NS;
 long g_stall_fill = -1;
 
+// Weights [rows, K] bf16 in the tile-packed layout (see moe_pack_weights): a
+// 3-D map {64, 128, rows/128 * K/64} with one 16 KiB tile per box.
+bool make_tile_map(CUtensorMap* m, const void* ptr, uint64_t K, uint64_t rows) {
+  auto fn = encode_fn();
+  if (!fn) return false;
+  cuuint64_t dims[3] = {(cuuint64_t)BK, (cuuint64_t)BM, (cuuint64_t)(rows / BM) * (K / BK)};
+  cuuint64_t strides[2] = {(cuuint64_t)BK * 2, (cuuint64_t)BK * BM * 2};
+  cuuint32_t box[3] = {BK, BM, 1};
+  cuuint32_t estr[3] = {1, 1, 1};
+  return fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(ptr), dims, strides, box,
+            estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+            CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+// A weight map in the layout the group's weights are stored in.
+bool make_weight_map(CUtensorMap* m, const void* ptr, uint64_t K, uint64_t rows, bool packed) {
+  return packed ? make_tile_map(m, ptr, K, rows) : make_map(m, ptr, K, rows, BK, BM);
+}
+
 template <int MODE, int NMAX>
 size_t gemm_smem_bytes(int n_exp) {
   using TL = Tile<MODE, NMAX>;
@@ -645,13 +692,15 @@ size_t gemm_smem_bytes(int n_exp) {
 
 template <int MODE, int NMAX>
 moe_status launch_gemm(const CUtensorMap& A0, const CUtensorMap& B0, const CUtensorMap& A1,
-                       const CUtensorMap& B1, const GemmArgs& args, cudaStream_t s) {
+                       const CUtensorMap& B1, const CUtensorMap& B0big, const CUtensorMap& B1big,
+                       const GemmArgs& args, cudaStream_t s) {
   const size_t smem = gemm_smem_bytes<MODE, NMAX>(args.n_exp);
   if (smem > 227 * 1024) return MOE_ERR_UNSUPPORTED;
   if (cudaFuncSetAttribute(grouped_gemm_kernel<MODE, NMAX>,
                            cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) != cudaSuccess)
     return MOE_ERR_CUDA;
-  grouped_gemm_kernel<MODE, NMAX><<<num_sms(), NUM_THREADS, smem, s>>>(A0, B0, A1, B1, args);
+  grouped_gemm_kernel<MODE, NMAX><<<num_sms(), NUM_THREADS, smem, s>>>(A0, B0, A1, B1, B0big,
+                                                                       B1big, args);
   note_launch();
   return launch_status();
 }
@@ -659,28 +708,37 @@ moe_status launch_gemm(const CUtensorMap& A0, const CUtensorMap& B0, const CUten
 template <int NMAX>
 moe_status run_ffn(const FfnGroup& g0, const FfnGroup* g1, int H, int I, cudaStream_t s,
                    cudaEvent_t after_gemm1) {
-  CUtensorMap a1, b1, a2, b2, sa1, sb1, sa2, sb2;
+  CUtensorMap a1, b1, a2, b2, sa1, sb1, sa2, sb2, b1big, b2big, sb1big, sb2big;
   // with a fused dispatch GEMM1 reads token rows of x by index: a one-row box
   const bool gather = g0.gather != nullptr;
-  if (!make_map(&a1, g0.W13, H, (uint64_t)g0.n_experts * 2 * I, BK, BM) ||
+  const bool pk = g0.packed;
+  if (!make_weight_map(&a1, g0.W13, H, (uint64_t)g0.n_experts * 2 * I, pk) ||
       !make_map(&b1, g0.x, H, gather ? g0.x_rows : g0.rows, BK, gather ? 1 : B_BOX) ||
-      !make_map(&a2, g0.W2, I, (uint64_t)g0.n_experts * H, BK, BM) ||
-      !make_map(&b2, g0.h, I, g0.rows, BK, B_BOX))
+      !make_weight_map(&a2, g0.W2, I, (uint64_t)g0.n_experts * H, pk) ||
+      !make_map(&b2, g0.h, I, g0.rows, BK, B_BOX) ||
+      !make_map(&b1big, g0.x, H, gather ? g0.x_rows : g0.rows, BK, gather ? 1 : B_BIG) ||
+      !make_map(&b2big, g0.h, I, g0.rows, BK, B_BIG))
     return MOE_ERR_CUDA;
   if (g1) {
-    if (!make_map(&sa1, g1->W13, H, (uint64_t)2 * I, BK, BM) ||
+    if (g1->packed != g0.packed) return MOE_ERR_INVALID_ARG;
+    if (!make_weight_map(&sa1, g1->W13, H, (uint64_t)2 * I, pk) ||
         !make_map(&sb1, g1->x, H, g1->rows, BK, B_BOX) ||
-        !make_map(&sa2, g1->W2, I, (uint64_t)H, BK, BM) ||
-        !make_map(&sb2, g1->h, I, g1->rows, BK, B_BOX))
+        !make_weight_map(&sa2, g1->W2, I, (uint64_t)H, pk) ||
+        !make_map(&sb2, g1->h, I, g1->rows, BK, B_BOX) ||
+        !make_map(&sb1big, g1->x, H, g1->rows, BK, B_BIG) ||
+        !make_map(&sb2big, g1->h, I, g1->rows, BK, B_BIG))
       return MOE_ERR_CUDA;
   } else {
     sa1 = a1;  // unused: group 1 is empty
     sb1 = b1;
     sa2 = a2;
     sb2 = b2;
+    sb1big = b1big;
+    sb2big = b2big;
   }
   GemmArgs args{};
   args.k_splits = 1;
+  args.a_packed = pk ? 1 : 0;
   args.wait_limit_ns = g_wait_limit_ns;
   args.stall_fill = g_stall_fill;
   args.offsets = g0.offsets;
@@ -698,7 +756,7 @@ moe_status run_ffn(const FfnGroup& g0, const FfnGroup* g1, int H, int I, cudaStr
   args.out0 = g0.h;
   args.out1 = g1 ? g1->h : nullptr;
   args.out_ld = I;
-  moe_status st = launch_gemm<MODE_SWIGLU, NMAX>(a1, b1, sa1, sb1, args, s);
+  moe_status st = launch_gemm<MODE_SWIGLU, NMAX>(a1, b1, sa1, sb1, b1big, sb1big, args, s);
   if (st != MOE_OK) return st;
   if (after_gemm1 && cudaEventRecord(after_gemm1, s) != cudaSuccess) return MOE_ERR_CUDA;
   args.gather0 = nullptr;  // GEMM2 reads h, already in packed row order
@@ -713,11 +771,11 @@ moe_status run_ffn(const FfnGroup& g0, const FfnGroup* g1, int H, int I, cudaStr
   if (NMAX > 32 && H % (2 * BM) == 0) {
     args.n_fb = H / (2 * BM);
     args.up_off = BM;
-    return launch_gemm<MODE_PLAIN2, NMAX>(a2, b2, sa2, sb2, args, s);
+    return launch_gemm<MODE_PLAIN2, NMAX>(a2, b2, sa2, sb2, b2big, sb2big, args, s);
   }
   args.n_fb = H / BM;
   args.up_off = 0;
-  return launch_gemm<MODE_PLAIN, NMAX>(a2, b2, sa2, sb2, args, s);
+  return launch_gemm<MODE_PLAIN, NMAX>(a2, b2, sa2, sb2, b2big, sb2big, args, s);
 }
 
 }  // namespace
@@ -748,8 +806,9 @@ int router_tc_splits(int T, int H, int E) {
 moe_status launch_router_tc(int T, int H, int E, const uint16_t* x, const uint16_t* planes,
                             float* partials, int k_splits, cudaStream_t s) {
   if (T == 0) return MOE_OK;
-  CUtensorMap A, B;
-  if (!make_map(&A, planes, H, (uint64_t)3 * E, BK, BM) || !make_map(&B, x, H, T, BK, B_BOX))
+  CUtensorMap A, B, Bbig;
+  if (!make_map(&A, planes, H, (uint64_t)3 * E, BK, BM) || !make_map(&B, x, H, T, BK, B_BOX) ||
+      !make_map(&Bbig, x, H, T, BK, B_BIG))
     return MOE_ERR_CUDA;
   GemmArgs args{};
   args.wait_limit_ns = WAIT_LIMIT_NS;
@@ -763,7 +822,7 @@ moe_status launch_router_tc(int T, int H, int E, const uint16_t* x, const uint16
   args.out1 = partials;
   args.out_ld = E;
   args.err = device_error_word();
-  return launch_gemm<MODE_SPLIT3, 128>(A, B, A, B, args, s);
+  return launch_gemm<MODE_SPLIT3, 128>(A, B, A, B, Bbig, Bbig, args, s);
 }
 
 moe_status launch_expert_ffn_stalled(int rows, int H, int I, int n_experts, const uint16_t* x_perm,
@@ -772,7 +831,7 @@ moe_status launch_expert_ffn_stalled(int rows, int H, int I, int n_experts, cons
                                      long stall_fill, uint64_t wait_limit_ns, cudaStream_t s) {
   g_wait_limit_ns = wait_limit_ns;
   g_stall_fill = stall_fill;
-  FfnGroup g{x_perm, offsets, rows, n_experts, 0, n_experts, W13, W2, h, y_perm, nullptr, 0};
+  FfnGroup g{x_perm, offsets, rows, n_experts, 0, n_experts, W13, W2, h, y_perm, nullptr, 0, false};
   const moe_status st = launch_expert_ffn_groups(g, nullptr, H, I, rows, s);
   g_wait_limit_ns = WAIT_LIMIT_NS;
   g_stall_fill = -1;
@@ -782,9 +841,10 @@ moe_status launch_expert_ffn_stalled(int rows, int H, int I, int n_experts, cons
 moe_status launch_expert_ffn(int rows, int H, int I, int n_experts, int e_begin, int e_end,
                              const uint16_t* x_perm, const int32_t* offsets, const uint16_t* W13,
                              const uint16_t* W2, uint16_t* h, float* y_perm, int rows_hint,
-                             cudaStream_t s, cudaEvent_t after_gemm1) {
+                             cudaStream_t s, cudaEvent_t after_gemm1, bool packed) {
   if (rows == 0 || e_end <= e_begin) return MOE_OK;
-  FfnGroup g{x_perm, offsets, rows, n_experts, e_begin, e_end, W13, W2, h, y_perm, nullptr, 0};
+  FfnGroup g{x_perm, offsets, rows, n_experts, e_begin, e_end, W13, W2, h, y_perm, nullptr, 0,
+             packed};
   return launch_expert_ffn_groups(g, nullptr, H, I, rows_hint, s, after_gemm1);
 }
 

@@ -247,6 +247,7 @@ FfnGroup routed_group(const moe_config& c, const Layout& L, const moe_weights& w
   g.e_end = e1;
   g.W13 = w.W13;
   g.W2 = w.W2;
+  g.packed = w.packed != 0;
   g.h = L.h + tk * c.I;
   g.y = L.y_perm + tk * c.H;
   if (L.x_perm) {
@@ -277,7 +278,8 @@ moe_status shared_expert(const moe_config& c, const Layout& L, const moe_weights
   }
   MOE_TRY(launch_fill_range(L.sh_off, c.T, s));
   MOE_TRY(launch_expert_ffn(c.T, c.H, c.I_shared, 1, 0, 1, x, L.sh_off, w.Ws13, w.Ws2, L.sh_h,
-                            L.sh_y, c.T, s, ev ? ev[MOE_EV_SHARED_GEMM1] : nullptr));
+                            L.sh_y, c.T, s, ev ? ev[MOE_EV_SHARED_GEMM1] : nullptr,
+                            w.packed != 0));
   return mark(ev, MOE_EV_SHARED_GEMM2, s);
 }
 
@@ -288,7 +290,8 @@ moe_status experts_and_shared(const moe_config& c, const Layout& L, const moe_we
                               const uint16_t* x, cudaStream_t s, cudaEvent_t* ev) {
   MOE_TRY(launch_fill_range(L.sh_off, c.T, s));
   const FfnGroup routed = routed_group(c, L, w, x, 0, c.T, 0, 0, c.E);
-  FfnGroup dense{x, L.sh_off, c.T, 1, 0, 1, w.Ws13, w.Ws2, L.sh_h, L.sh_y, nullptr, 0};
+  FfnGroup dense{x, L.sh_off, c.T, 1, 0, 1, w.Ws13, w.Ws2, L.sh_h, L.sh_y, nullptr, 0,
+                 w.packed != 0};
   MOE_TRY(launch_expert_ffn_groups(routed, &dense, c.H, c.I, routed.rows, s,
                                    ev ? ev[MOE_EV_GEMM1] : nullptr));
   MOE_TRY(mark(ev, MOE_EV_GEMM2, s));
@@ -390,10 +393,22 @@ moe_status moe_dispatch(const moe_config* cfg, const uint16_t* x, const int32_t*
   return MOE_OK;
 }
 
+moe_status moe_pack_weights(int64_t rows, int32_t K, const uint16_t* W, uint16_t* W_packed,
+                            void* stream) {
+  if (rows < 0 || rows % 128 || K < 64 || K % 64 || K > 65536) return MOE_ERR_INVALID_ARG;
+  if (rows == 0) return MOE_OK;
+  if (!W || !W_packed || !aligned16(W) || !aligned16(W_packed)) return MOE_ERR_INVALID_ARG;
+  const uint8_t *a = (const uint8_t*)W, *b = (const uint8_t*)W_packed;
+  const size_t n = (size_t)rows * K * 2;
+  if (a < b + n && b < a + n) return MOE_ERR_INVALID_ARG;  // must not overlap
+  return launch_pack_weights(W, W_packed, (long)rows, K, (cudaStream_t)stream);
+}
+
 moe_status moe_expert_ffn(int32_t rows, int32_t H, int32_t I, int32_t n_experts,
                           const uint16_t* x_perm, const int32_t* offsets, const uint16_t* W13,
                           const uint16_t* W2, float* y_perm, void* ws, size_t ws_bytes,
-                          void* stream) {
+                          int32_t weights_packed, void* stream) {
+  if (weights_packed != 0 && weights_packed != 1) return MOE_ERR_INVALID_ARG;
   if (rows < 0 || H < 128 || H % 128 || H > 65536 || I < 128 || I % 128 || I > 65536 ||
       n_experts < 1 || n_experts > 1024)
     return MOE_ERR_INVALID_ARG;
@@ -404,7 +419,8 @@ moe_status moe_expert_ffn(int32_t rows, int32_t H, int32_t I, int32_t n_experts,
   const size_t need = moe_expert_ffn_workspace_size(rows, I);
   if (!ws || ws_bytes < need || !aligned16(ws)) return MOE_ERR_WORKSPACE;
   return launch_expert_ffn(rows, H, I, n_experts, 0, n_experts, x_perm, offsets, W13, W2,
-                           (uint16_t*)ws, y_perm, rows, (cudaStream_t)stream);
+                           (uint16_t*)ws, y_perm, rows, (cudaStream_t)stream, nullptr,
+                           weights_packed != 0);
 }
 
 moe_status moe_testing_expert_ffn_stall(int32_t rows, int32_t H, int32_t I, int32_t n_experts,
@@ -442,6 +458,7 @@ moe_status moe_layer_forward(const moe_config* cfg, const moe_exec* ex, const mo
                              const uint16_t* x, void* out, const moe_aux* aux, void* ws,
                              size_t ws_bytes, void* stream, void* aux_stream) {
   if (!valid_config(cfg) || !valid_exec(ex, cfg) || !w) return MOE_ERR_INVALID_ARG;
+  if (w->packed != 0 && w->packed != 1) return MOE_ERR_INVALID_ARG;
   const moe_config& c = *cfg;
   if (!w->Wr || !w->W13 || !w->W2 || !aligned16(w->Wr) || !aligned16(w->W13) ||
       !aligned16(w->W2) || (w->bias && !aligned4(w->bias)))

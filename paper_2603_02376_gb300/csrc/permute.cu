@@ -181,6 +181,23 @@ __global__ void __launch_bounds__(PERM_WARPS * 32) perm_scatter_kernel(
   }
 }
 
+// Tile-packed weights: element (r, c) of W [rows, K] moves to
+// ((r / 128) * (K / 64) + c / 64) * 8192 + (r % 128) * 64 + c % 64, so every
+// 128 x 64 tile the GEMM loads is one contiguous 16 KiB block. 16-byte vectors.
+__global__ void pack_weights_kernel(const uint4* __restrict__ W, uint4* __restrict__ Wp, long rows,
+                                    int K) {
+  const long vpr = K / 8;  // 16-byte vectors per row
+  const long total = rows * vpr;
+  const long kbs = K / 64;
+  for (long i = blockIdx.x * (long)blockDim.x + threadIdx.x; i < total;
+       i += (long)gridDim.x * blockDim.x) {
+    const long r = i / vpr, v = i % vpr;
+    const long c = v * 8;
+    const long dst = (((r / 128) * kbs + c / 64) * 8192 + (r % 128) * 64 + c % 64) / 8;
+    Wp[dst] = W[i];
+  }
+}
+
 // The whole permutation in one CTA when the batch is a single chunk (decode):
 // the histogram, the scan over experts and the stable scatter of perm_hist /
 // perm_scan / perm_scatter, without two launches and the chunk tables.
@@ -438,6 +455,14 @@ moe_status launch_fill_range(int32_t* offsets, int n, cudaStream_t s) {
 moe_status launch_sum_counts(const int32_t* counts, int n_chunks, int E, int32_t* out,
                              cudaStream_t s) {
   sum_counts_kernel<<<(E + 255) / 256, 256, 0, s>>>(counts, n_chunks, E, out);
+  note_launch();
+  return launch_status();
+}
+
+moe_status launch_pack_weights(const uint16_t* W, uint16_t* Wp, long rows, int K, cudaStream_t s) {
+  if (rows == 0) return MOE_OK;
+  pack_weights_kernel<<<copy_grid((size_t)rows * (K / 8)), 256, 0, s>>>(
+      reinterpret_cast<const uint4*>(W), reinterpret_cast<uint4*>(Wp), rows, K);
   note_launch();
   return launch_status();
 }

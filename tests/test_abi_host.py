@@ -103,10 +103,16 @@ def test_entry_points_reject_bad_arguments_without_a_gpu(lib):
     assert lib.moe_gate_topk(cb(bad), p, z, p, p, z) == L.MOE_ERR_INVALID_ARG
     assert lib.moe_dispatch(cb(c), p, p, p, p, p, p, p, z, 0, z) == L.MOE_ERR_WORKSPACE
     assert lib.moe_dispatch(cb(c), z, p, p, p, p, p, p, p, 1 << 30, z) == L.MOE_ERR_INVALID_ARG
-    assert lib.moe_expert_ffn(16, 100, 128, 1, p, p, p, p, p, p, 1 << 20, z) == L.MOE_ERR_INVALID_ARG
-    assert lib.moe_expert_ffn(16, 256, 128, 0, p, p, p, p, p, p, 1 << 20, z) == L.MOE_ERR_INVALID_ARG
-    assert lib.moe_expert_ffn(16, 256, 128, 1, p, p, p, p, p, z, 0, z) == L.MOE_ERR_WORKSPACE
-    assert lib.moe_expert_ffn(16, 256, 128, 1, odd, p, p, p, p, p, 1 << 20, z) == L.MOE_ERR_INVALID_ARG
+    assert lib.moe_expert_ffn(16, 100, 128, 1, p, p, p, p, p, p, 1 << 20, 0, z) == L.MOE_ERR_INVALID_ARG
+    assert lib.moe_expert_ffn(16, 256, 128, 0, p, p, p, p, p, p, 1 << 20, 0, z) == L.MOE_ERR_INVALID_ARG
+    assert lib.moe_expert_ffn(16, 256, 128, 1, p, p, p, p, p, z, 0, 0, z) == L.MOE_ERR_WORKSPACE
+    assert lib.moe_expert_ffn(16, 256, 128, 1, odd, p, p, p, p, p, 1 << 20, 0, z) == L.MOE_ERR_INVALID_ARG
+    assert lib.moe_expert_ffn(16, 256, 128, 1, p, p, p, p, p, p, 1 << 20, 2, z) == L.MOE_ERR_INVALID_ARG
+    assert lib.moe_pack_weights(100, 64, p, p, z) == L.MOE_ERR_INVALID_ARG      # rows % 128
+    assert lib.moe_pack_weights(128, 96, p, p, z) == L.MOE_ERR_INVALID_ARG      # K % 64
+    assert lib.moe_pack_weights(128, 64, p, p, z) == L.MOE_ERR_INVALID_ARG      # W == W_packed
+    assert lib.moe_pack_weights(128, 64, p, ctypes.c_void_p(0x1000 + 8192), z) == L.MOE_ERR_INVALID_ARG
+    assert lib.moe_pack_weights(0, 64, z, z, z) == L.MOE_OK
     assert lib.moe_combine(cb(c), p, p, p, z, p, 2, z) == L.MOE_ERR_INVALID_ARG
     assert lib.moe_combine(cb(c), p, p, p, z, odd, 0, z) == L.MOE_ERR_INVALID_ARG
     ex = L.exec_config()
@@ -125,7 +131,7 @@ def test_empty_batch_is_a_no_op(lib):
     assert lib.moe_router_logits(cb(c), z, z, z, z, 0, z) == L.MOE_OK
     assert lib.moe_gate_topk(cb(c), z, z, z, z, z) == L.MOE_OK
     assert lib.moe_combine(cb(c), z, z, z, z, z, 0, z) == L.MOE_OK
-    assert lib.moe_expert_ffn(0, 256, 128, 4, z, z, z, z, z, z, 0, z) == L.MOE_OK
+    assert lib.moe_expert_ffn(0, 256, 128, 4, z, z, z, z, z, z, 0, 0, z) == L.MOE_OK
     W = L.moe_weights(0x1000, None, 0x1000, 0x1000, 0x1000, 0x1000)
     assert lib.moe_layer_forward(cb(c), cb(L.exec_config()), cb(W), z, z, None, z, 0, z, z) == L.MOE_OK
 

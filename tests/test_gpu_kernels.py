@@ -221,6 +221,18 @@ def ffn_case(counts, H, Iw, seed, rows_extra=3):
     return rows, offs, xp, W13, W2
 
 
+@pytest.mark.parametrize("rows,K", [(128, 64), (256, 7168), (4096, 2048), (384, 192)])
+def test_pack_weights_layout(rows, K):
+    """Every 128 x 64 tile becomes one contiguous block, tiles in (row block, k block) order."""
+    W = rand_bf16((rows, K), rows + K)
+    Wp = torch.empty_like(W)
+    L.moe_pack_weights(W, Wp)
+    torch.cuda.synchronize()
+    ref = W.view(rows // 128, 128, K // 64, 64).permute(0, 2, 1, 3).reshape(rows, K)
+    assert torch.equal(Wp, ref)
+
+
+@pytest.mark.parametrize("packed", [0, 1])
 @pytest.mark.parametrize("counts,H,Iw", [
     ([5, 0, 17, 1], 256, 128),                          # tiny, ragged, an empty expert
     ([300, 256, 257, 0, 1, 16], 256, 256),              # multi-tile experts, tile edges
@@ -230,13 +242,15 @@ def ffn_case(counts, H, Iw, seed, rows_extra=3):
     ([130, 111], 7168, 2048),                           # the real layer shape
     ([1] * 48 + [3, 7], 7168, 2048),                    # decode: few rows per expert
 ])
-def test_expert_ffn(counts, H, Iw):
+def test_expert_ffn(counts, H, Iw, packed):
     rows, offs, xp, W13, W2 = ffn_case(counts, H, Iw, seed=len(counts) + H)
     E = len(counts)
     sentinel = -12345.0
     y = torch.full((rows, H), sentinel, dtype=torch.float32, device=DEV)
     ws = torch.zeros(L.moe_expert_ffn_workspace_size(rows, Iw), dtype=torch.uint8, device=DEV)
-    L.moe_expert_ffn(rows, H, Iw, E, xp, torch.from_numpy(offs).to(DEV), W13, W2, y, ws)
+    W13g, W2g = (L.pack_weights(W13), L.pack_weights(W2)) if packed else (W13, W2)
+    L.moe_expert_ffn(rows, H, Iw, E, xp, torch.from_numpy(offs).to(DEV), W13g, W2g, y, ws,
+                     weights_packed=packed)
     L.moe_check_errors()
     h = ws.view(torch.bfloat16).view(rows, Iw)
     n = int(offs[-1])

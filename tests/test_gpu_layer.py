@@ -40,6 +40,16 @@ def big_weights():
     torch.cuda.empty_cache()
 
 
+def packed_copy(d):
+    """The same layer with its expert weights in the tile-packed layout."""
+    p = dict(d)
+    for k in ("W13", "W2", "Ws13", "Ws2"):
+        if p.get(k) is not None:
+            p[k] = L.pack_weights(p[k])
+    p["packed"] = 1
+    return p
+
+
 def run_layer(wl, d, ex, aux=True):
     cfg = L.config_of(wl)
     T, H, E, k = wl.T, wl.H, wl.E, wl.k
@@ -49,7 +59,8 @@ def run_layer(wl, d, ex, aux=True):
              topk_idx=torch.empty((T, k), dtype=torch.int32, device=DEV),
              topk_w=torch.empty((T, k), device=DEV),
              counts=torch.empty(E, dtype=torch.int32, device=DEV)) if aux else {}
-    W = L.weights_struct(d["Wr"], d["bias"], d["W13"], d["W2"], d["Ws13"], d["Ws2"])
+    W = L.weights_struct(d["Wr"], d["bias"], d["W13"], d["W2"], d["Ws13"], d["Ws2"],
+                         d.get("packed", 0))
     L.moe_layer_forward(cfg, ex, W, d["x"], out, L.aux_struct(**a) if aux else None, ws)
     L.moe_check_errors()
     return out, a
@@ -134,6 +145,12 @@ def test_layer_small_grouped_full(I_shared, T):
                     topk_groups=2, gate=I.GATE_SIGMOID, normalize=1, route_scale=2.5)
     d = I.layer_inputs(wl, seed=5, device=DEV)
     st = prepare_routing(wl, d)
+    dp = packed_copy(d)
+    out, a = run_layer(wl, dp, L.exec_config(out_fp32=1))      # tile-packed expert weights
+    check_routing(wl, dp, a, st["oracle_logits"])
+    ref, _ = O.layer_forward(f64(d["x"]), f64(d["Wr"]), bias32(d["bias"]), f64(d["W13"]),
+                             f64(d["W2"]), oracle_cfg(wl), f64(d["Ws13"]), f64(d["Ws2"]))
+    assert_layer_close(f64(out), ref)
     for ex in (L.exec_config(out_fp32=1), L.exec_config(out_fp32=0),
                L.exec_config(out_fp32=1, fuse_gather=0),
                L.exec_config(out_fp32=1, overlap=1, chunk_axis=0, chunk_tokens=37),
@@ -152,10 +169,12 @@ def test_layer_small_grouped_full(I_shared, T):
 # ---------------------------------------------------------------- decode: every token
 
 @pytest.mark.parametrize("ex", [dict(out_fp32=1), dict(out_fp32=0), dict(out_fp32=1, fuse_gather=0),
-                                dict(out_fp32=1, overlap=1, chunk_axis=1, n_expert_chunks=4)])
+                                dict(out_fp32=1, overlap=1, chunk_axis=1, n_expert_chunks=4),
+                                dict(out_fp32=1, packed=1)])
 def test_layer_decode_full(big_weights, ex):
     wl = I.DECODE
-    d = dict(big_weights)
+    ex = dict(ex)
+    d = packed_copy(big_weights) if ex.pop("packed", 0) else dict(big_weights)
     d["x"] = I.randn((wl.T, wl.H), 1.0, torch.bfloat16, 0, "x", DEV)
     st = prepare_routing(wl, d)
     out, a = run_layer(wl, d, L.exec_config(**ex))

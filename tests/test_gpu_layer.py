@@ -174,10 +174,12 @@ def test_layer_small_grouped_full(I_shared, T):
 def test_layer_decode_full(big_weights, ex):
     wl = I.DECODE
     ex = dict(ex)
-    d = packed_copy(big_weights) if ex.pop("packed", 0) else dict(big_weights)
+    packed = ex.pop("packed", 0)
+    d = dict(big_weights)
     d["x"] = I.randn((wl.T, wl.H), 1.0, torch.bfloat16, 0, "x", DEV)
     st = prepare_routing(wl, d)
-    out, a = run_layer(wl, d, L.exec_config(**ex))
+    # the layer may run on tile-packed weights; the oracle always reads row-major ones
+    out, a = run_layer(wl, packed_copy(d) if packed else d, L.exec_config(**ex))
     gidx = check_routing(wl, d, a, st["oracle_logits"])
     check_permutation(wl, d, gidx)
     ref, _ = oracle_tokens(wl, d, np.arange(wl.T))

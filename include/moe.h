@@ -230,12 +230,13 @@ moe_status moe_dispatch_noalloc(const moe_config* cfg, const uint16_t* x, const 
  * the paper). Copies W [rows, K] bf16 (row-major; rows a multiple of 128, K a
  * multiple of 64) to W_packed (same size, caller-allocated, not overlapping W)
  * so that every 128-row x 64-column tile the GEMMs load is one contiguous
- * 16 KiB block: element (r, c) goes to
- *   ((r / 128) * (K / 64) + c / 64) * 8192 + (r % 128) * 64 + c % 64.
+ * 16 KiB block, already in the 128-byte-swizzled order of the tensor-core
+ * operands: tile (r / 128, c / 64) is block (r / 128) * (K / 64) + c / 64, and
+ * inside it the 16-byte chunk j = (c % 64) / 8 of row r sits at element
+ *   (r % 128) * 64 + 8 * (j ^ (r % 8)) + c % 8.
  * Pack W13 as rows = E*2I, K = H; W2 as rows = E*H, K = I; the shared expert's
  * Ws13 / Ws2 likewise; then set moe_weights.packed (or weights_packed of
- * moe_expert_ffn). Contiguous tiles stream ~3 % faster from HBM than 128 rows
- * strided by the row pitch.
+ * moe_expert_ffn). The GEMMs then fetch each tile with one bulk copy.
  */
 moe_status moe_pack_weights(int64_t rows, int32_t K, const uint16_t* W, uint16_t* W_packed,
                             void* stream);

@@ -149,14 +149,14 @@ __device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap* map
       : "memory");
 }
 
-// One 128-row x 64-column weight tile of the tile-packed layout: a 3-D map
-// {64 columns, 128 rows, tiles} whose box is one whole tile (16 KiB, contiguous).
-__device__ __forceinline__ void tma_load_tile3d(uint32_t dst, const CUtensorMap* map, int tile,
-                                                uint32_t bar) {
+// One weight tile of the tile-packed layout: 16 KiB, contiguous and already in
+// the 128-byte-swizzled order the MMA descriptors expect, so a plain bulk copy
+// (no tensor map) lands it ready to use.
+__device__ __forceinline__ void bulk_load_tile(uint32_t dst, const void* src, uint32_t bar) {
   asm volatile(
-      "cp.async.bulk.tensor.3d.shared::cluster.global.mbarrier::complete_tx::bytes"
-      " [%0], [%1, {%2, %3, %4}], [%5];" ::"r"(dst),
-      "l"(reinterpret_cast<uint64_t>(map)), "r"(0), "r"(0), "r"(tile), "r"(bar)
+      "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::
+          "r"(dst),
+      "l"(reinterpret_cast<uint64_t>(src)), "r"(BM * BK * 2), "r"(bar)
       : "memory");
 }
 
@@ -243,7 +243,8 @@ struct GemmArgs {
   int K, n_fb;
   int w_rows0;  // weight rows per expert in group 0
   int up_off;   // row offset between a unit's weight tiles (SwiGLU: the up projection)
-  int a_packed;  // weights (A) in the tile-packed layout: 3-D maps, tile = (row/128)*kblocks + kb
+  const uint16_t* a0_packed;  // group 0 weights in the tile-packed layout (else null: tensor maps)
+  const uint16_t* a1_packed;  // group 1 likewise
   int k_splits; // group 1 only: the K range is split into this many units ...
   long split_stride;  // ... whose outputs go to out1 + split * split_stride (partials)
   void* out0;
@@ -453,8 +454,10 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
 #pragma unroll
             for (int t = 0; t < TL::NA; ++t) {
               const int r = wrow + t * a.up_off;
-              if (a.a_packed)
-                tma_load_tile3d(sa + t * TL::A_BYTES, mA, (r / BM) * kblocks + kb, full);
+              const uint16_t* ap = U.grp ? a.a1_packed : a.a0_packed;
+              if (ap)  // tile (r / 128, kb): 8192 bf16 per tile
+                bulk_load_tile(sa + t * TL::A_BYTES,
+                               ap + ((size_t)(r / BM) * kblocks + kb) * (BM * BK), full);
               else
                 tma_load_2d(sa + t * TL::A_BYTES, mA, kb * BK, r, full);
             }
@@ -665,23 +668,11 @@ bool make_map(CUtensorMap* m, const void* ptr, uint64_t inner, uint64_t outer, u
 uint64_t g_wait_limit_ns = WAIT_LIMIT_NS;
 long g_stall_fill = -1;
 
-// Weights [rows, K] bf16 in the tile-packed layout (see moe_pack_weights): a
-// 3-D map {64, 128, rows/128 * K/64} with one 16 KiB tile per box.
-bool make_tile_map(CUtensorMap* m, const void* ptr, uint64_t K, uint64_t rows) {
-  auto fn = encode_fn();
-  if (!fn) return false;
-  cuuint64_t dims[3] = {(cuuint64_t)BK, (cuuint64_t)BM, (cuuint64_t)(rows / BM) * (K / BK)};
-  cuuint64_t strides[2] = {(cuuint64_t)BK * 2, (cuuint64_t)BK * BM * 2};
-  cuuint32_t box[3] = {BK, BM, 1};
-  cuuint32_t estr[3] = {1, 1, 1};
-  return fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(ptr), dims, strides, box,
-            estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
-            CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
-}
-
-// A weight map in the layout the group's weights are stored in.
+// A weight map for row-major weights; packed weights are read by bulk copies
+// and get a (valid, unused) map over the same bytes.
 bool make_weight_map(CUtensorMap* m, const void* ptr, uint64_t K, uint64_t rows, bool packed) {
-  return packed ? make_tile_map(m, ptr, K, rows) : make_map(m, ptr, K, rows, BK, BM);
+  (void)packed;
+  return make_map(m, ptr, K, rows, BK, BM);
 }
 
 template <int MODE, int NMAX>
@@ -738,7 +729,8 @@ moe_status run_ffn(const FfnGroup& g0, const FfnGroup* g1, int H, int I, cudaStr
   }
   GemmArgs args{};
   args.k_splits = 1;
-  args.a_packed = pk ? 1 : 0;
+  args.a0_packed = pk ? g0.W13 : nullptr;
+  args.a1_packed = (pk && g1) ? g1->W13 : nullptr;
   args.wait_limit_ns = g_wait_limit_ns;
   args.stall_fill = g_stall_fill;
   args.offsets = g0.offsets;
@@ -760,6 +752,8 @@ moe_status run_ffn(const FfnGroup& g0, const FfnGroup* g1, int H, int I, cudaStr
   if (st != MOE_OK) return st;
   if (after_gemm1 && cudaEventRecord(after_gemm1, s) != cudaSuccess) return MOE_ERR_CUDA;
   args.gather0 = nullptr;  // GEMM2 reads h, already in packed row order
+  args.a0_packed = pk ? g0.W2 : nullptr;
+  args.a1_packed = (pk && g1) ? g1->W2 : nullptr;
   // GEMM2: y = h W2^T (fp32). With prefill-sized token tiles, two 128-feature
   // weight tiles per unit share one token tile (more weight bytes per stage);
   // with decode-sized tiles a single weight tile and a deeper ring measured faster.

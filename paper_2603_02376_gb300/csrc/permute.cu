@@ -181,9 +181,11 @@ __global__ void __launch_bounds__(PERM_WARPS * 32) perm_scatter_kernel(
   }
 }
 
-// Tile-packed weights: element (r, c) of W [rows, K] moves to
-// ((r / 128) * (K / 64) + c / 64) * 8192 + (r % 128) * 64 + c % 64, so every
-// 128 x 64 tile the GEMM loads is one contiguous 16 KiB block. 16-byte vectors.
+// Tile-packed weights: the 128 x 64 tile (r / 128, c / 64) of W [rows, K] is one
+// contiguous 16 KiB block, tiles in (row block, column block) order; inside a
+// tile, row r % 128 occupies 128 bytes and its 16-byte chunk j = (c % 64) / 8 sits
+// at chunk j ^ (r % 8) -- the 128-byte swizzle the MMA operand descriptors use,
+// so the GEMM copies tiles to shared memory unchanged. 16-byte vectors.
 __global__ void pack_weights_kernel(const uint4* __restrict__ W, uint4* __restrict__ Wp, long rows,
                                     int K) {
   const long vpr = K / 8;  // 16-byte vectors per row
@@ -192,9 +194,9 @@ __global__ void pack_weights_kernel(const uint4* __restrict__ W, uint4* __restri
   for (long i = blockIdx.x * (long)blockDim.x + threadIdx.x; i < total;
        i += (long)gridDim.x * blockDim.x) {
     const long r = i / vpr, v = i % vpr;
-    const long c = v * 8;
-    const long dst = (((r / 128) * kbs + c / 64) * 8192 + (r % 128) * 64 + c % 64) / 8;
-    Wp[dst] = W[i];
+    const long tile = (r / 128) * kbs + v / 8;
+    const long chunk = (v % 8) ^ (r % 8);
+    Wp[tile * 1024 + (r % 128) * 8 + chunk] = W[i];
   }
 }
 

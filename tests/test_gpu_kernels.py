@@ -228,8 +228,15 @@ def test_pack_weights_layout(rows, K):
     Wp = torch.empty_like(W)
     L.moe_pack_weights(W, Wp)
     torch.cuda.synchronize()
-    ref = W.view(rows // 128, 128, K // 64, 64).permute(0, 2, 1, 3).reshape(rows, K)
-    assert torch.equal(Wp, ref)
+    # tile order (row block, column block); inside a tile row r's 16-byte chunk j
+    # sits at chunk j ^ (r % 8)
+    t = W.view(rows // 128, 128, K // 64, 8, 8).permute(0, 2, 1, 3, 4)  # [rb, cb, r, j, 8]
+    r = torch.arange(128, device=DEV).view(128, 1)
+    j = torch.arange(8, device=DEV).view(1, 8)
+    dst = (j ^ (r % 8))                                                     # [r, j]
+    ref = torch.empty_like(t)
+    ref[:, :, r.expand(128, 8), dst, :] = t
+    assert torch.equal(Wp.view_as(ref), ref)
 
 
 @pytest.mark.parametrize("packed", [0, 1])

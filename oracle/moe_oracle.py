@@ -312,6 +312,69 @@ def combine(y_perm, slot_row, w, shared=None) -> np.ndarray:
 
 
 # ---------------------------------------------------------------------------
+# FP8 expert compute (the paper quantizes tokens before the dispatch and
+# dequantizes before GEMM1: int8 in its host listing, "FP8 quantize" in its
+# Section 4.3 table). Reading: OCP e4m3 ("E4M3FN": 4 exponent bits, 3 mantissa
+# bits, bias 7, largest finite 448, subnormals down to 2^-9), round to nearest
+# even, saturating; one fp32 scale per row s = amax / 448 (fp32 division), the
+# quantized value e4m3(v / s) with v / s an fp32 division. Per token for x,
+# per packed row for h, per output row for the weights. Quantized products
+# are exact, the sums are fp64 here; the two row scales multiply the sum.
+# ---------------------------------------------------------------------------
+
+E4M3_MAX = 448.0
+
+
+def e4m3_round(a) -> np.ndarray:
+    """Nearest e4m3 value (ties to even), saturating at +-448.
+
+    Normal e4m3 numbers in [2^e, 2^(e+1)) (e = -6..8) are spaced 2^(e-3);
+    below 2^-6 the subnormals are spaced 2^-9.
+    """
+    a = np.asarray(a, dtype=np.float64)
+    mag = np.abs(a)
+    e = np.floor(np.log2(np.where(mag > 0, mag, 1.0)))
+    e = np.clip(e, -6, 8)
+    q = np.ldexp(1.0, (e - 3).astype(np.int64))
+    r = np.rint(mag / q) * q
+    r = np.minimum(r, E4M3_MAX)
+    return np.where(mag > 0, np.sign(a) * r, 0.0)
+
+
+def quantize_rows_e4m3(a):
+    """Per-row e4m3 quantization: returns (q fp64 values on the e4m3 grid, scale fp32 [rows]).
+
+    s = fp32(amax / 448) (1 for an all-zero row); q = e4m3(fp32(v / s)).
+    """
+    a32 = np.asarray(a, dtype=np.float32)
+    amax = np.abs(a32).max(axis=1)
+    s = np.where(amax > 0, (amax / np.float32(E4M3_MAX)).astype(np.float32), np.float32(1.0))
+    s = s.astype(np.float32)
+    v = (a32 / s[:, None]).astype(np.float32)
+    return e4m3_round(v), s
+
+
+def swiglu_ffn_fp8(rows, W13_q, s13, W2_q, s2):
+    """One SwiGLU expert in the FP8 form.
+
+    rows [m, H] (bf16 values); W13_q [2I, H], W2_q [H, I] e4m3 values with
+    per-row fp32 scales s13 [2I], s2 [H]. x is quantized per row; g, u =
+    (x_q . W_q^T) * s_x * s_w; h = bf16(silu(g) * u) quantized per row;
+    y = (h_q . W2_q^T) * s_h * s_2.
+    """
+    rows = np.asarray(rows, dtype=np.float64)
+    I = W13_q.shape[0] // 2
+    xq, sx = quantize_rows_e4m3(rows)
+    acc = xq @ np.asarray(W13_q, dtype=np.float64).T
+    gu = acc * sx.astype(np.float64)[:, None] * np.asarray(s13, dtype=np.float64)[None, :]
+    g, u = gu[:, :I], gu[:, I:]
+    h = bf16_round(silu(g) * u)
+    hq, sh = quantize_rows_e4m3(h)
+    y = (hq @ np.asarray(W2_q, dtype=np.float64).T)
+    return y * sh.astype(np.float64)[:, None] * np.asarray(s2, dtype=np.float64)[None, :]
+
+
+# ---------------------------------------------------------------------------
 # the whole layer
 # ---------------------------------------------------------------------------
 

@@ -380,3 +380,61 @@ def test_workload_shapes_match_paper():
         assert [wl.H, 2 * wl.I] == p["gemm1"]
         assert [wl.I, wl.H] == p["gemm2"]
     assert I.PREFILL.T == p["tokens_per_rank"]
+
+
+# ---------------------------------------------------------------- FP8 (e4m3) quantization
+
+def test_e4m3_round_matches_torch_inside_the_range():
+    g = torch.Generator().manual_seed(4)
+    a = torch.randn(200000, generator=g) * torch.exp(torch.randn(200000, generator=g) * 3)
+    a = a[a.abs() < 460]                       # torch gives NaN past the range; the oracle saturates
+    ref = a.to(torch.float8_e4m3fn).to(torch.float64).numpy()
+    np.testing.assert_array_equal(O.e4m3_round(a.to(torch.float64).numpy()), ref)
+
+
+def test_e4m3_round_by_hand():
+    # 3 mantissa bits: between 1 and 2 the grid step is 1/8. 1.0625 is halfway between
+    # 1 and 1.125 -> even mantissa (1.0); 1.1875 halfway between 1.125 and 1.25 -> 1.25.
+    # 448 is the largest finite value; larger values saturate. Subnormal step 2^-9:
+    # 2^-10 is halfway between 0 and 2^-9 -> 0; 3 * 2^-11 -> 2^-9.
+    vals = [1.0625, 1.1875, -1.1875, 448.0, 1000.0, -1e9, 2**-10, 3 * 2**-11, 0.0, 240.0, 232.0]
+    exp = [1.0, 1.25, -1.25, 448.0, 448.0, -448.0, 0.0, 2**-9, 0.0, 240.0, 224.0]
+    np.testing.assert_array_equal(O.e4m3_round(vals), exp)
+
+
+def test_quantize_rows_closed_form():
+    a = np.array([[1.0, -2.0, 0.5], [0.0, 0.0, 0.0], [448.0, 224.0, -112.0]])
+    q, s = O.quantize_rows_e4m3(a)
+    assert s.dtype == np.float32
+    np.testing.assert_array_equal(s, np.float32([2.0 / 448, 1.0, 1.0]))
+    # the row maximum maps to +-448 exactly; a zero row stays zero
+    assert q[0, 1] == -448.0 and q[2, 0] == 448.0 and (q[1] == 0).all()
+    np.testing.assert_array_equal(q[2], [448.0, 224.0, -112.0])
+    # dequantized error within half an e4m3 step of the scaled value (relative 2^-4)
+    rng = np.random.default_rng(0)
+    x = rng.standard_normal((50, 300))
+    q, s = O.quantize_rows_e4m3(x)
+    deq = q * s[:, None]
+    assert (np.abs(deq - x) <= np.abs(x) * 2.0 ** -4 + s[:, None] * 2.0 ** -10 + 1e-12).all()
+
+
+def test_swiglu_fp8_equals_dequantized_operands():
+    # The FP8 form applies the row scales outside the sums; that must equal the same
+    # products written with dequantized operands (q * s) inside the sums. Inputs on the
+    # e4m3 grid with a row maximum of 448 have scale 1 and quantize to themselves.
+    rng = np.random.default_rng(2)
+    H, Iw, m = 64, 32, 5
+    grid = lambda shape: O.e4m3_round(rng.uniform(-448, 448, shape))
+    rows = grid((m, H)); rows[:, 0] = 448.0
+    W13 = grid((2 * Iw, H)) / 448.0 / 64.0
+    W2 = grid((H, Iw)) / 448.0 / 64.0
+    W13q, s13 = O.quantize_rows_e4m3(W13)
+    W2q, s2 = O.quantize_rows_e4m3(W2)
+    y8 = O.swiglu_ffn_fp8(rows, W13q, s13, W2q, s2)
+    # same computation written with the dequantized operands (h re-quantized as in the FP8 form)
+    g = rows @ (W13q * s13[:, None].astype(np.float64))[:Iw].T
+    u = rows @ (W13q * s13[:, None].astype(np.float64))[Iw:].T
+    h = O.bf16_round(O.silu(g) * u)
+    hq, sh = O.quantize_rows_e4m3(h)
+    y = (hq * sh[:, None].astype(np.float64)) @ (W2q * s2[:, None].astype(np.float64)).T
+    np.testing.assert_allclose(y8, y, rtol=1e-12, atol=1e-12)

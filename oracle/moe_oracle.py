@@ -354,6 +354,26 @@ def quantize_rows_e4m3(a):
     return e4m3_round(v), s
 
 
+def fp8_linear(a_q, s_a, W_q, s_w) -> np.ndarray:
+    """Dequantized product of e4m3 operands: (a_q . W_q^T) * s_a[r] * s_w[c] (fp64).
+
+    a_q [m, K], W_q [n, K] on the e4m3 grid; s_a [m], s_w [n] fp32 row scales.
+    """
+    acc = np.asarray(a_q, dtype=np.float64) @ np.asarray(W_q, dtype=np.float64).T
+    return acc * np.asarray(s_a, dtype=np.float64)[:, None] * \
+        np.asarray(s_w, dtype=np.float64)[None, :]
+
+
+def swiglu_h_fp8(rows, W13_q, s13) -> np.ndarray:
+    """GEMM1 + SwiGLU of the FP8 form: h = bf16(silu(g) * u), with g | u the
+    dequantized product of the per-row quantized rows and W13_q (scales s13)."""
+    I = W13_q.shape[0] // 2
+    xq, sx = quantize_rows_e4m3(np.asarray(rows, dtype=np.float64))
+    gu = fp8_linear(xq, sx, W13_q, s13)
+    g, u = gu[:, :I], gu[:, I:]
+    return bf16_round(silu(g) * u)
+
+
 def swiglu_ffn_fp8(rows, W13_q, s13, W2_q, s2):
     """One SwiGLU expert in the FP8 form.
 
@@ -362,16 +382,9 @@ def swiglu_ffn_fp8(rows, W13_q, s13, W2_q, s2):
     (x_q . W_q^T) * s_x * s_w; h = bf16(silu(g) * u) quantized per row;
     y = (h_q . W2_q^T) * s_h * s_2.
     """
-    rows = np.asarray(rows, dtype=np.float64)
-    I = W13_q.shape[0] // 2
-    xq, sx = quantize_rows_e4m3(rows)
-    acc = xq @ np.asarray(W13_q, dtype=np.float64).T
-    gu = acc * sx.astype(np.float64)[:, None] * np.asarray(s13, dtype=np.float64)[None, :]
-    g, u = gu[:, :I], gu[:, I:]
-    h = bf16_round(silu(g) * u)
+    h = swiglu_h_fp8(rows, W13_q, s13)
     hq, sh = quantize_rows_e4m3(h)
-    y = (hq @ np.asarray(W2_q, dtype=np.float64).T)
-    return y * sh.astype(np.float64)[:, None] * np.asarray(s2, dtype=np.float64)[None, :]
+    return fp8_linear(hq, sh, W2_q, s2)
 
 
 # ---------------------------------------------------------------------------
@@ -401,13 +414,16 @@ def layer_forward(x, Wr, bias, W13, W2, cfg: LayerConfig, Ws13=None, Ws2=None, l
     return out, aux
 
 
-def layer_forward_tokens(x_rows, Wr, bias, get_expert, cfg: LayerConfig, get_shared=None):
+def layer_forward_tokens(x_rows, Wr, bias, get_expert, cfg: LayerConfig, get_shared=None,
+                         ffn=swiglu_ffn):
     """Layer output for a sample of tokens, one token at a time.
 
     Routing is independent per token, so a token's output needs only its own
-    row. x_rows [n, H]; get_expert(e) -> (W13_e, W2_e); get_shared() ->
-    (Ws13, Ws2) or None. Experts are visited once each, with all sampled rows
-    routed to them. Returns (out fp64 [n, H], idx [n, k], w [n, k]).
+    row. x_rows [n, H]; get_expert(e) -> the expert's weight arguments of
+    `ffn` after the rows ((W13_e, W2_e) for swiglu_ffn; (W13_q, s13, W2_q, s2)
+    for swiglu_ffn_fp8); get_shared() -> the shared expert's, or None.
+    Experts are visited once each, with all sampled rows routed to them.
+    Returns (out fp64 [n, H], idx [n, k], w [n, k]).
     """
     x_rows = np.asarray(x_rows, dtype=np.float64)
     L32 = router_logits(x_rows, Wr)
@@ -416,10 +432,8 @@ def layer_forward_tokens(x_rows, Wr, bias, get_expert, cfg: LayerConfig, get_sha
     out = np.zeros((n, cfg.H), dtype=np.float64)
     for e in np.unique(idx):
         who, slot = np.nonzero(idx == e)
-        W13_e, W2_e = get_expert(int(e))
-        y = swiglu_ffn(x_rows[who], W13_e, W2_e)
+        y = ffn(x_rows[who], *get_expert(int(e)))
         out[who] += w[who, slot][:, None] * y
     if get_shared is not None and cfg.I_shared:
-        Ws13, Ws2 = get_shared()
-        out += swiglu_ffn(x_rows, Ws13, Ws2)
+        out += ffn(x_rows, *get_shared())
     return out, idx, w

@@ -438,3 +438,42 @@ def test_swiglu_fp8_equals_dequantized_operands():
     hq, sh = O.quantize_rows_e4m3(h)
     y = (hq * sh[:, None].astype(np.float64)) @ (W2q * s2[:, None].astype(np.float64)).T
     np.testing.assert_allclose(y8, y, rtol=1e-12, atol=1e-12)
+
+
+def test_fp8_linear_by_hand():
+    # acc = [[1*3 + 2*4, 1*1 + 2*(-1)]] = [[11, -1]]; scaled by s_a = 0.5 and s_w = (2, 0.25)
+    y = O.fp8_linear(np.array([[1.0, 2.0]]), np.array([0.5], np.float32),
+                     np.array([[3.0, 4.0], [1.0, -1.0]]), np.array([2.0, 0.25], np.float32))
+    np.testing.assert_array_equal(y, [[11.0, -0.125]])
+
+
+def test_swiglu_h_fp8_row_scale_cancels():
+    # Scaling a row by a power of two scales its e4m3 scale alone (same q), so g and u
+    # scale with it: h = silu(g) * u for the scaled row follows from the plain one.
+    rng = np.random.default_rng(5)
+    H, Iw = 32, 16
+    rows = O.bf16_round(rng.standard_normal((3, H)))
+    W13q, s13 = O.quantize_rows_e4m3(rng.standard_normal((2 * Iw, H)) * 0.05)
+    h1 = O.swiglu_h_fp8(rows, W13q, s13)
+    xq, sx = O.quantize_rows_e4m3(rows)
+    gu = O.fp8_linear(xq, sx, W13q, s13)
+    np.testing.assert_array_equal(h1, O.bf16_round(O.silu(gu[:, :Iw]) * gu[:, Iw:]))
+    xq4, sx4 = O.quantize_rows_e4m3(rows * 4.0)
+    np.testing.assert_array_equal(xq4, xq)
+    np.testing.assert_array_equal(sx4, sx * 4)
+
+
+def test_layer_tokens_fp8_hook_matches_per_expert_calls():
+    # the ffn hook of the per-token layer forward: FP8 experts through the same routing
+    rng = np.random.default_rng(6)
+    cfg = O.LayerConfig(T=6, H=32, E=4, k=2, I=16, gate=O.GATE_SOFTMAX)
+    x = O.bf16_round(rng.standard_normal((6, 32)))
+    Wr = rng.standard_normal((4, 32)).astype(np.float32) * 0.1
+    W13 = [O.quantize_rows_e4m3(rng.standard_normal((32, 32)) * 0.05) for _ in range(4)]
+    W2 = [O.quantize_rows_e4m3(rng.standard_normal((32, 16)) * 0.05) for _ in range(4)]
+    get = lambda e: (W13[e][0], W13[e][1], W2[e][0], W2[e][1])
+    out, idx, w = O.layer_forward_tokens(x, Wr, None, get, cfg, ffn=O.swiglu_ffn_fp8)
+    for t in range(6):
+        ref = sum(w[t, j] * O.swiglu_ffn_fp8(x[t:t + 1], *get(int(idx[t, j])))[0]
+                  for j in range(2))
+        np.testing.assert_allclose(out[t], ref, rtol=1e-13, atol=1e-15)

@@ -477,3 +477,15 @@ def test_layer_tokens_fp8_hook_matches_per_expert_calls():
         ref = sum(w[t, j] * O.swiglu_ffn_fp8(x[t:t + 1], *get(int(idx[t, j])))[0]
                   for j in range(2))
         np.testing.assert_allclose(out[t], ref, rtol=1e-13, atol=1e-15)
+
+
+def test_e4m3_decode_every_code():
+    codes = np.arange(256, dtype=np.uint8)
+    v = O.e4m3_decode(codes)
+    ref = torch.from_numpy(codes).view(torch.float8_e4m3fn).to(torch.float64).numpy()
+    np.testing.assert_array_equal(v, ref)               # NaN at 0x7f / 0xff on both sides
+    # by hand: 1.0, the largest finite, the smallest subnormal, -2.5, -0
+    assert O.e4m3_decode([0x38, 0x7E, 0x01, 0xC2, 0x80]).tolist() == [1.0, 448.0, 2.0 ** -9, -2.5, 0.0]
+    finite = v[~np.isnan(v)]
+    np.testing.assert_array_equal(O.e4m3_round(finite), finite)   # the grid rounds to itself
+    assert len(np.unique(finite)) == 253                           # 254 finite codes, +-0 equal

@@ -56,6 +56,9 @@ def parse():
                    help="tile-pack the expert weights at load (auto: for batches of more than "
                         "24 rows per expert, where it measured 1-4 %% faster; decode-sized "
                         "batches measured ~1 %% faster row-major)")
+    p.add_argument("--precision", choices=("bf16", "fp8"), default="bf16",
+                   help="expert GEMM operands: bf16, or e4m3 with per-row scales (weights "
+                        "quantized once at load, tokens and h quantized inside each step)")
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--cpu-tokens", type=int, default=128, help="oracle sample size (tokens)")
     return p.parse_args()
@@ -188,23 +191,28 @@ def calibrate(L, wl, d, device):
         d["bias"] = b.to(device)
 
 
-def algorithmic(wl, touched, fused_gather=True):
+def algorithmic(wl, touched, fused_gather=True, fp8=False):
     """Algorithmic bytes and flops of each stage for one forward.
 
-    GEMM1's token operand is counted as R*H*2 either way (packed rows read, or
-    the same rows gathered from x); a fused dispatch has no stage of its own.
+    GEMM1's token operand is counted as R*H*eb either way (packed rows read, or
+    the same rows gathered from x); a fused dispatch has no copy of its own.
+    FP8 (eb = 1): the dispatch stage also quantizes x (bf16 read, e4m3 + scales
+    written) and the GEMM1 stage also quantizes h (bf16 read, e4m3 + scales).
     """
     T, H, E, k, Iw, Is = wl.T, wl.H, wl.E, wl.k, wl.I, wl.I_shared
     R = T * k
+    eb = 1 if fp8 else 2
+    qx = T * H * 3 + T * 4 if fp8 else 0               # x -> e4m3 rows + scales
+    qh = lambda rows, n: rows * n * 3 + rows * 4 if fp8 else 0   # h -> e4m3
     b = {
         "router": T * H * 2 + E * H * 4 + T * E * 4,
         "gate": T * E * 4 + T * k * 8,
         "permute": T * k * 4 * 3,
-        "dispatch": 0 if fused_gather else T * H * 2 + R * H * 2,
-        "gemm1": touched * 2 * Iw * H * 2 + R * H * 2 + R * Iw * 2,
-        "gemm2": touched * H * Iw * 2 + R * Iw * 2 + R * H * 4,
-        "shared_gemm1": (2 * Is * H * 2 + T * H * 2 + T * Is * 2) if Is else 0,
-        "shared_gemm2": (H * Is * 2 + T * Is * 2 + T * H * 4) if Is else 0,
+        "dispatch": qx + (0 if fused_gather else T * H * eb + R * H * eb),
+        "gemm1": touched * 2 * Iw * H * eb + R * H * eb + R * Iw * 2 + qh(R, Iw),
+        "gemm2": touched * H * Iw * eb + R * Iw * eb + R * H * 4,
+        "shared_gemm1": (2 * Is * H * eb + T * H * eb + T * Is * 2 + qh(T, Is)) if Is else 0,
+        "shared_gemm2": (H * Is * eb + T * Is * eb + T * H * 4) if Is else 0,
         "combine": R * H * 4 + (T * H * 4 if Is else 0) + T * H * 2 + R * 8,
     }
     f = {"router": 2 * T * E * H, "gemm1": 2 * R * H * 2 * Iw, "gemm2": 2 * R * Iw * H,
@@ -240,7 +248,9 @@ def measured_traffic(workload):
 # ---------------------------------------------------------------- CPU oracle leg
 
 def oracle_tokens_per_s(wl, d, tokens):
-    """Time the CPU oracle on a sample of tokens; weights come from host copies."""
+    """Time the CPU oracle on a sample of tokens; weights come from host copies.
+
+    With d["fp8"] the oracle runs the FP8 expert form on the e4m3 weights."""
     from oracle import moe_oracle as O
 
     cfg = O.LayerConfig(T=len(tokens), H=wl.H, E=wl.E, k=wl.k, I=wl.I, I_shared=wl.I_shared,
@@ -252,17 +262,26 @@ def oracle_tokens_per_s(wl, d, tokens):
     b = None if d["bias"] is None else d["bias"].cpu().numpy()
     # host copies (bf16) of the experts the sample touches, made before the clock starts
     idx, _ = O.gate_topk(O.router_logits(xr, Wr), b, cfg)
-    host = {int(e): (d["W13"][e].cpu(), d["W2"][e].cpu()) for e in np.unique(idx)}
-    shared = (d["Ws13"].cpu(), d["Ws2"].cpu()) if wl.I_shared else None
+    f8 = d.get("fp8")
+    if f8:
+        host = {int(e): tuple(f8[n][e].cpu() for n in ("W13", "s13", "W2", "s2"))
+                for e in np.unique(idx)}
+        shared = tuple(f8[n].cpu() for n in ("Ws13", "ss13", "Ws2", "ss2")) \
+            if wl.I_shared else None
+        conv = lambda t: O.e4m3_decode(t.numpy()) if t.dtype == torch.uint8 else t.numpy()
+        ffn = O.swiglu_ffn_fp8
+    else:
+        host = {int(e): (d["W13"][e].cpu(), d["W2"][e].cpu()) for e in np.unique(idx)}
+        shared = (d["Ws13"].cpu(), d["Ws2"].cpu()) if wl.I_shared else None
+        conv = lambda t: t.to(torch.float64).numpy()
+        ffn = O.swiglu_ffn
 
     def get_expert(e):
-        a, c = host[e]
-        return a.to(torch.float64).numpy(), c.to(torch.float64).numpy()
+        return tuple(conv(t) for t in host[e])
 
-    get_shared = (lambda: (shared[0].to(torch.float64).numpy(),
-                           shared[1].to(torch.float64).numpy())) if shared else None
+    get_shared = (lambda: tuple(conv(t) for t in shared)) if shared else None
     t0 = time.perf_counter()
-    O.layer_forward_tokens(xr, Wr, b, get_expert, cfg, get_shared)
+    O.layer_forward_tokens(xr, Wr, b, get_expert, cfg, get_shared, ffn=ffn)
     dt = time.perf_counter() - t0
     return len(tokens) / dt, dt, len(host)
 
@@ -270,9 +289,10 @@ def oracle_tokens_per_s(wl, d, tokens):
 def cpu_baseline(wl, d, n_tokens, seed=1):
     toks = I.sample_tokens(wl.T, n_tokens, seed).numpy()
     v, dt, ne = oracle_tokens_per_s(wl, d, toks)
+    form = "FP8 expert form, " if d.get("fp8") else ""
     return {"value": v, "unit": "tokens/s", "cores": os.cpu_count(), "kind": "oracle",
-            "sample": f"{len(toks)} of the {wl.T} tokens ({ne} experts touched), numpy fp64 "
-                      f"oracle, {dt:.1f} s; BLAS threads = host cores"}
+            "sample": f"{len(toks)} of the {wl.T} tokens ({ne} experts touched), {form}numpy "
+                      f"fp64 oracle, {dt:.1f} s; BLAS threads = host cores"}
 
 
 # ---------------------------------------------------------------- main arms
@@ -310,7 +330,9 @@ def run_reference(args, wl, rank, world, device):
 
 
 def packs(args, wl):
-    """Whether the run uses tile-packed expert weights."""
+    """Whether the run uses tile-packed expert weights (bf16 only)."""
+    if args.precision == "fp8":
+        return False
     if args.pack == "auto":
         return wl.T * wl.k > 24 * wl.E
     return args.pack == "yes"
@@ -323,6 +345,8 @@ def config_of(wl, args):
             "mode": args.mode, "dispatch": "fused into GEMM1 (TMA gather4)"
             if (not args.no_fuse_gather and wl.T * wl.k <= 24 * wl.E) else "packed x_perm",
             "weights": "tile-packed at load (moe_pack_weights)" if packs(args, wl) else "row-major",
+            "precision": "e4m3 expert GEMMs, per-row fp32 scales (weights quantized at load)"
+            if args.precision == "fp8" else "bf16 expert GEMMs",
             "global_batch": wl.T * args.gpus,
             "l2": "inputs larger than L2: the expert weights streamed per step exceed 129 MB",
             "parallelism": f"replicas{args.gpus}"}
@@ -342,11 +366,12 @@ def run_ours(args, wl, rank, world, local, device):
     fuse = 0 if args.no_fuse_gather else 1
     # the library fuses the dispatch only for decode-sized batches (<= 24 rows per expert)
     fused = bool(fuse) and wl.T * wl.k <= 24 * wl.E
-    ex = L.exec_config(fuse_gather=fuse, **mode)
+    fp8 = 1 if args.precision == "fp8" else 0
+    ex = L.exec_config(fuse_gather=fuse, fp8=fp8, **mode)
     # one workspace serves the timed mode and the sequential stats / stage-event passes
     ws = torch.empty(max(L.moe_workspace_size(cfg, ex),
-                         L.moe_workspace_size(cfg, L.exec_config(fuse_gather=fuse)),
-                         L.moe_workspace_size(cfg, L.exec_config(fuse_gather=0))),
+                         L.moe_workspace_size(cfg, L.exec_config(fuse_gather=fuse, fp8=fp8)),
+                         L.moe_workspace_size(cfg, L.exec_config(fuse_gather=0, fp8=fp8))),
                      dtype=torch.uint8, device=device)
     out = torch.empty((wl.T, wl.H), dtype=torch.bfloat16, device=device)
     stream = torch.cuda.current_stream()
@@ -357,15 +382,34 @@ def run_ours(args, wl, rank, world, local, device):
     if packed:
         run_w = {k_: (None if v is None else L.pack_weights(v)) for k_, v in run_w.items()}
         torch.cuda.synchronize()
-    W = L.weights_struct(d["Wr"], d["bias"], run_w["W13"], run_w["W2"], run_w["Ws13"],
-                         run_w["Ws2"], 1 if packed else 0)
+    if fp8:
+        # e4m3 copies of the expert weights with per-row scales: a load-time step
+        # like the packing above; the bf16 tensors are dropped (the oracle leg
+        # reads the e4m3 bytes)
+        f8 = {}
+        for n, sn in (("W13", "s13"), ("W2", "s2"), ("Ws13", "ss13"), ("Ws2", "ss2")):
+            if d.get(n) is not None:
+                f8[n], f8[sn] = L.quantize_fp8(d[n])
+            else:
+                f8[n] = f8[sn] = None
+        torch.cuda.synchronize()
+        d["fp8"] = f8
+        for n in ("W13", "W2", "Ws13", "Ws2"):
+            d[n] = None
+        run_w = None
+        torch.cuda.empty_cache()
+        W = L.weights_struct(d["Wr"], d["bias"], f8["W13"], f8["W2"], f8["Ws13"], f8["Ws2"], 0,
+                             f8["s13"], f8["s2"], f8["ss13"], f8["ss2"])
+    else:
+        W = L.weights_struct(d["Wr"], d["bias"], run_w["W13"], run_w["W2"], run_w["Ws13"],
+                             run_w["Ws2"], 1 if packed else 0)
 
     def step():
         L.moe_layer_forward(cfg, ex, W, d["x"], out, None, ws, stream)
 
     # routing statistics of this batch (touched experts set the GEMM weight bytes)
     counts = torch.empty(wl.E, dtype=torch.int32, device=device)
-    L.moe_layer_forward(cfg, L.exec_config(fuse_gather=fuse), W, d["x"], out,
+    L.moe_layer_forward(cfg, L.exec_config(fuse_gather=fuse, fp8=fp8), W, d["x"], out,
                         L.aux_struct(counts=counts), ws, stream)
     L.moe_check_errors(stream)
     cnt = counts.cpu()
@@ -409,7 +453,7 @@ def run_ours(args, wl, rank, world, local, device):
                 e.record(stream)
         torch.cuda.synchronize()
         for i in range(K2):
-            exs = L.exec_config(fuse_gather=fuse_flag, stage_events=evs[i])
+            exs = L.exec_config(fuse_gather=fuse_flag, stage_events=evs[i], fp8=fp8)
             L.moe_layer_forward(cfg, exs, W, d["x"], out, None, ws, stream)
         torch.cuda.synchronize()
         return {L.STAGES[j]: statistics.mean(evs[i][j - 1].elapsed_time(evs[i][j])
@@ -469,10 +513,10 @@ def run_ours(args, wl, rank, world, local, device):
                    "ms_sequential_unchunked": round(sum(stage_ms.values()), 4)}
 
     hbm, tf_burst, tf_sust, src = peaks()
-    b, f = algorithmic(wl, touched, fused)
+    b, f = algorithmic(wl, touched, fused, bool(fp8))
     g1 = stage_ms["gemm1"] / 1e3
     achieved = b["gemm1"] / g1 / 1e9
-    traffic = measured_traffic(wl.name)
+    traffic = None if fp8 else measured_traffic(wl.name)
     stages = {}
     for s_, t in stage_ms.items():
         e = {"ms": round(t, 4)}
@@ -481,19 +525,27 @@ def run_ours(args, wl, rank, world, local, device):
             e["frac_hbm"] = round(b[s_] / (t / 1e3) / 1e9 / hbm, 3)
         if f.get(s_):
             e["TFLOP/s"] = round(f[s_] / (t / 1e3) / 1e12, 2)
-            e["frac_bf16"] = round(f[s_] / (t / 1e3) / 1e12 / tf_sust, 4)
+            if fp8:  # fp8 dense peak = the measured bf16 peak x the nominal 2x ratio
+                e["frac_fp8"] = round(f[s_] / (t / 1e3) / 1e12 / (2 * tf_sust), 4)
+            else:
+                e["frac_bf16"] = round(f[s_] / (t / 1e3) / 1e12 / tf_sust, 4)
         stages[s_] = e
 
     line = {
         "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms / args.steps,
-        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
-        "data": "synthetic (seeded N(0,1) activations, N(0,0.02^2) bf16 weights)",
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+        "dtype": "e4m3" if fp8 else "bf16",
+        "data": "synthetic (seeded N(0,1) activations, N(0,0.02^2) bf16 weights"
+                + (", quantized to e4m3 at load)" if fp8 else ")"),
         "config": config_of(wl, args),
         "e2e": {"value": e2e_value, "unit": "tokens/s", "h2d_bytes_per_step": wl.T * wl.H * 2,
                 "d2h_bytes_per_step": wl.T * wl.H * 2},
         "gpu_launches": launches,
-        "roofline": {"bound": "hbm", "kernel": "grouped GEMM1 + SwiGLU (tcgen05), routed + shared",
+        "roofline": {"bound": "hbm",
+                     "kernel": ("grouped GEMM1 + SwiGLU (tcgen05 kind::f8f6f4) and the h "
+                                "quantization, routed + shared") if fp8 else
+                               "grouped GEMM1 + SwiGLU (tcgen05), routed + shared",
                      "achieved": round(achieved, 1), "peak": hbm, "unit": "GB/s",
                      "frac": round(achieved / hbm, 4), "traffic": traffic,
                      "peak_source": f"hbm_gbs of {src}",

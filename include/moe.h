@@ -88,6 +88,15 @@ typedef struct {
  *    packed copy x_perm is never written; larger batches, and 0, pack x_perm
  *    with a dispatch kernel first (one gather instruction per four rows per
  *    k-block costs more than the copy once tiles hold ~128 rows).
+ *  fp8 0 = bf16 expert GEMMs; 1 = FP8 (e4m3) expert GEMMs, the quantized
+ *    pipeline of the paper's MoE workload (Section 4.3 lists an FP8 quantize
+ *    stage before the dispatch): after the gate every token row x[t] is
+ *    quantized (moe_quantize_fp8: e4m3 values and one fp32 scale per row), the
+ *    dispatch moves the e4m3 rows (half the bytes), GEMM1 and the shared
+ *    expert's GEMM1 multiply e4m3 x e4m3 into fp32 and apply both row scales
+ *    in the epilogue, h (bf16, as in the bf16 form) is quantized per row the
+ *    same way, and GEMM2 runs on e4m3 h and W2. The expert weights of
+ *    moe_weights must then be e4m3 with their row scales (fp8 fields there).
  */
 typedef struct {
   int32_t overlap, chunk_tokens, chunk_axis, n_expert_chunks, out_fp32, fuse_gather;
@@ -95,6 +104,7 @@ typedef struct {
    * the caller) recorded on `stream` at the stage boundaries of a sequential
    * (overlap = 0) forward; NULL = no tracing. Ignored when overlap = 1. */
   void** stage_events;
+  int32_t fp8;
 } moe_exec;
 
 /* Indices into moe_exec.stage_events: event i is recorded when stage i ends
@@ -119,15 +129,24 @@ enum {
  * W13 [E,2I,H] bf16 (rows 0..I-1 gate, I..2I-1 up); W2 [E,H,I] bf16;
  * Ws13 [2*I_shared,H] bf16 and Ws2 [H,I_shared] bf16, NULL iff I_shared = 0.
  * packed 1 = W13, W2, Ws13 and Ws2 are in the tile-packed layout written by
- * moe_pack_weights (same values, same sizes); 0 = row-major as above. */
+ * moe_pack_weights (same values, same sizes); 0 = row-major as above.
+ * With moe_exec.fp8 = 1 the four expert matrices hold e4m3 bytes instead
+ * (same shapes, row-major, packed = 0), as written by moe_quantize_fp8 over
+ * their rows, and the *_scale arrays hold the fp32 scale of every row:
+ * W13_scale [E*2I], W2_scale [E*H], Ws13_scale [2*I_shared], Ws2_scale [H]
+ * (the shared ones NULL iff I_shared = 0). With fp8 = 0 the scales are unused. */
 typedef struct {
   const float* Wr;
   const float* bias;
-  const uint16_t* W13;
-  const uint16_t* W2;
-  const uint16_t* Ws13;
-  const uint16_t* Ws2;
+  const void* W13;
+  const void* W2;
+  const void* Ws13;
+  const void* Ws2;
   int32_t packed;
+  const float* W13_scale;
+  const float* W2_scale;
+  const float* Ws13_scale;
+  const float* Ws2_scale;
 } moe_weights;
 
 /* Optional outputs of moe_layer_forward; NULL fields are skipped.
@@ -158,6 +177,10 @@ size_t moe_dispatch_workspace_size(const moe_config* cfg);
 
 /* Workspace bytes of moe_expert_ffn: the SwiGLU activations [rows, I] bf16. */
 size_t moe_expert_ffn_workspace_size(int32_t rows, int32_t I);
+
+/* Workspace bytes of moe_expert_ffn_fp8: h [rows, I] bf16, its e4m3 copy
+ * [rows, I] and its row scales [rows] fp32, each 256-byte aligned. */
+size_t moe_expert_ffn_fp8_workspace_size(int32_t rows, int32_t I);
 
 /*
  * Router logits: logits[t,e] = sum_h x[t,h] * Wr[e,h], fp32-accurate.
@@ -262,6 +285,42 @@ moe_status moe_expert_ffn(int32_t rows, int32_t H, int32_t I, int32_t n_experts,
                           const uint16_t* x_perm, const int32_t* offsets, const uint16_t* W13,
                           const uint16_t* W2, float* y_perm, void* ws, size_t ws_bytes,
                           int32_t weights_packed, void* stream);
+
+/*
+ * FP8 row quantization, the paper's "quantize" stage (Section 4.3's FP8
+ * quantize before the dispatch; the dequantize is folded into the GEMM
+ * epilogues). For each row r of in [rows, K] bf16:
+ *   scale[r] = fp32(amax_r / 448)   (1 when the row is all zero),
+ *   out[r][c] = e4m3(fp32(in[r][c] / scale[r])),
+ * with e4m3 the OCP E4M3 format (bias 7, no infinities, largest finite 448),
+ * rounded to nearest even and saturated at +-448. out [rows, K] e4m3 bytes;
+ * scale [rows] fp32; both written, caller-allocated. K a multiple of 16 and at
+ * most 65536; in and out 16-byte aligned; in and out must not overlap.
+ * Used on token rows inside moe_layer_forward (fp8 = 1) and, once, on the
+ * expert weights (W13 as rows = E*2I, K = H; W2 as rows = E*H, K = I).
+ */
+moe_status moe_quantize_fp8(int64_t rows, int32_t K, const uint16_t* in, uint8_t* out,
+                            float* scale, void* stream);
+
+/*
+ * Grouped expert FFN in the FP8 form (moe_expert_ffn with e4m3 operands).
+ * For each expert e < n_experts and row r in [offsets[e], offsets[e+1]):
+ *   g|u = (x_q[r] . W13_q[e]^T) * sx(r) * W13_scale[e*2I + j]  (fp32 accumulate),
+ *   h[r] = bf16(silu(g) * u),  (h_q, s_h) = moe_quantize_fp8 of h per row,
+ *   y_perm[r] = (h_q[r] . W2_q[e]^T) * s_h[r] * W2_scale[e*H + c].
+ * sx(r) = x_scale[x_scale_idx[r]] when x_scale_idx is given (x_q rows are
+ * copies of token rows, scales kept per token), else x_scale[r].
+ * x_q [rows,H] e4m3; W13_q [n_experts,2I,H] and W2_q [n_experts,H,I] e4m3
+ * (row-major); offsets, shapes, y_perm and the segment rules as in
+ * moe_expert_ffn. ws: moe_expert_ffn_fp8_workspace_size(rows, I) bytes,
+ * 256-byte aligned.
+ */
+moe_status moe_expert_ffn_fp8(int32_t rows, int32_t H, int32_t I, int32_t n_experts,
+                              const uint8_t* x_q, const float* x_scale,
+                              const int32_t* x_scale_idx, const int32_t* offsets,
+                              const uint8_t* W13_q, const float* W13_scale, const uint8_t* W2_q,
+                              const float* W2_scale, float* y_perm, void* ws, size_t ws_bytes,
+                              void* stream);
 
 /*
  * Combine: the single-GPU form of the paper's reverse AlltoAll combine.

@@ -29,7 +29,8 @@ EXPORTS = ("moe_status_string", "moe_validate_config", "moe_workspace_size",
            "moe_expert_ffn_workspace_size", "moe_router_logits", "moe_gate_topk", "moe_dispatch",
            "moe_expert_ffn", "moe_combine", "moe_layer_forward", "moe_check_errors",
            "moe_launch_count", "moe_shutdown", "moe_dispatch_noalloc",
-           "moe_testing_expert_ffn_stall", "moe_pack_weights")
+           "moe_testing_expert_ffn_stall", "moe_pack_weights", "moe_quantize_fp8",
+           "moe_expert_ffn_fp8", "moe_expert_ffn_fp8_workspace_size")
 MOE_DISPATCH_NOALLOC_MAX_ENTRIES = 131072
 
 
@@ -49,7 +50,7 @@ class moe_exec(ctypes.Structure):
     _fields_ = [(n, ctypes.c_int32) for n in
                 ("overlap", "chunk_tokens", "chunk_axis", "n_expert_chunks", "out_fp32",
                  "fuse_gather")] + \
-               [("stage_events", ctypes.POINTER(ctypes.c_void_p))]
+               [("stage_events", ctypes.POINTER(ctypes.c_void_p)), ("fp8", ctypes.c_int32)]
 
 
 STAGES = ("start", "router", "gate", "permute", "dispatch", "gemm1", "gemm2", "shared_gemm1",
@@ -59,7 +60,9 @@ MOE_N_STAGE_EVENTS = len(STAGES)
 
 class moe_weights(ctypes.Structure):
     _fields_ = [(n, ctypes.c_void_p) for n in ("Wr", "bias", "W13", "W2", "Ws13", "Ws2")] + \
-               [("packed", ctypes.c_int32)]
+               [("packed", ctypes.c_int32)] + \
+               [(n, ctypes.c_void_p) for n in ("W13_scale", "W2_scale", "Ws13_scale",
+                                               "Ws2_scale")]
 
 
 class moe_aux(ctypes.Structure):
@@ -94,6 +97,9 @@ def load(path: str = LIB_PATH) -> ctypes.CDLL:
         "moe_dispatch_noalloc": (S, [cfgp, P, P, P, P, P, P, P, P]),
         "moe_expert_ffn": (S, [I32, I32, I32, I32, P, P, P, P, P, P, SZ, I32, P]),
         "moe_pack_weights": (S, [ctypes.c_int64, I32, P, P, P]),
+        "moe_quantize_fp8": (S, [ctypes.c_int64, I32, P, P, P, P]),
+        "moe_expert_ffn_fp8_workspace_size": (SZ, [I32, I32]),
+        "moe_expert_ffn_fp8": (S, [I32, I32, I32, I32, P, P, P, P, P, P, P, P, P, P, SZ, P]),
         "moe_combine": (S, [cfgp, P, P, P, P, P, I32, P]),
         "moe_testing_expert_ffn_stall": (S, [I32, I32, I32, I32, P, P, P, P, P, P, SZ,
                                              ctypes.c_int64, ctypes.c_int64, P]),
@@ -151,9 +157,10 @@ def config_of(wl, T=None) -> moe_config:
 
 
 def exec_config(overlap=0, chunk_tokens=512, chunk_axis=0, n_expert_chunks=8, out_fp32=0,
-                fuse_gather=1, stage_events=None):
+                fuse_gather=1, stage_events=None, fp8=0):
     """moe_exec; stage_events: a list of MOE_N_STAGE_EVENTS torch.cuda.Event (or None)."""
-    ex = moe_exec(overlap, chunk_tokens, chunk_axis, n_expert_chunks, out_fp32, fuse_gather, None)
+    ex = moe_exec(overlap, chunk_tokens, chunk_axis, n_expert_chunks, out_fp32, fuse_gather, None,
+                  int(fp8))
     if stage_events is not None:
         arr = (ctypes.c_void_p * MOE_N_STAGE_EVENTS)(*[int(e.cuda_event) for e in stage_events])
         ex._events_keepalive = arr
@@ -219,6 +226,38 @@ def moe_expert_ffn(rows, H, I, n_experts, x_perm, offsets, W13, W2, y_perm, ws,
            "moe_expert_ffn")
 
 
+def moe_expert_ffn_fp8_workspace_size(rows, I) -> int:
+    return load().moe_expert_ffn_fp8_workspace_size(rows, I)
+
+
+def moe_quantize_fp8(x, out, scale, stream=None) -> None:
+    """Per-row e4m3 quantization of a bf16 tensor viewed as [rows, K] (K = its last dim)."""
+    K = x.shape[-1]
+    rows = x.numel() // K
+    _check(load().moe_quantize_fp8(rows, K, _ptr(x), _ptr(out), _ptr(scale), _stream(stream)),
+           "moe_quantize_fp8")
+
+
+def quantize_fp8(x, stream=None):
+    """(e4m3 bytes as uint8 of x's shape, fp32 scale per row) of a bf16 tensor."""
+    import torch
+    K = x.shape[-1]
+    q = torch.empty(x.shape, dtype=torch.uint8, device=x.device)
+    s = torch.empty(x.numel() // K, dtype=torch.float32, device=x.device)
+    moe_quantize_fp8(x, q, s, stream)
+    return q, s
+
+
+def moe_expert_ffn_fp8(rows, H, I, n_experts, x_q, x_scale, x_scale_idx, offsets, W13_q,
+                       W13_scale, W2_q, W2_scale, y_perm, ws, stream=None) -> None:
+    nb = 0 if ws is None else ws.numel() * ws.element_size()
+    _check(load().moe_expert_ffn_fp8(rows, H, I, n_experts, _ptr(x_q), _ptr(x_scale),
+                                     _ptr(x_scale_idx), _ptr(offsets), _ptr(W13_q),
+                                     _ptr(W13_scale), _ptr(W2_q), _ptr(W2_scale), _ptr(y_perm),
+                                     _ptr(ws), nb, _stream(stream)),
+           "moe_expert_ffn_fp8")
+
+
 def moe_pack_weights(W, W_packed, stream=None) -> None:
     """Tile-packed copy of a bf16 weight tensor viewed as [rows, K] (K = its last dim)."""
     K = W.shape[-1]
@@ -251,9 +290,12 @@ def moe_combine(cfg, y_perm, slot_row, topk_w, shared_out, out, out_fp32, stream
            "moe_combine")
 
 
-def weights_struct(Wr, bias, W13, W2, Ws13=None, Ws2=None, packed=0) -> moe_weights:
-    return moe_weights(*(None if t is None else t.data_ptr()
-                         for t in (Wr, bias, W13, W2, Ws13, Ws2)), int(packed))
+def weights_struct(Wr, bias, W13, W2, Ws13=None, Ws2=None, packed=0, W13_scale=None,
+                   W2_scale=None, Ws13_scale=None, Ws2_scale=None) -> moe_weights:
+    p = [None if t is None else t.data_ptr() for t in (Wr, bias, W13, W2, Ws13, Ws2)]
+    sc = [None if t is None else t.data_ptr() for t in (W13_scale, W2_scale, Ws13_scale,
+                                                         Ws2_scale)]
+    return moe_weights(*p, int(packed), *sc)
 
 
 def aux_struct(logits=None, topk_idx=None, topk_w=None, counts=None) -> moe_aux:

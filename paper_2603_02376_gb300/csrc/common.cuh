@@ -78,11 +78,11 @@ moe_status launch_sum_counts(const int32_t* counts, int n_chunks, int E, int32_t
 // the packed activations x [rows, H] with device row offsets, or (offsets
 // unused) a single dense segment [0, rows) with one weight matrix.
 struct FfnGroup {
-  const uint16_t* x;
+  const void* x;  // [rows or x_rows, H] bf16, or e4m3 bytes when fp8
   const int32_t* offsets;
   int rows, n_experts, e_begin, e_end;
-  const uint16_t* W13;
-  const uint16_t* W2;
+  const void* W13;  // bf16, or e4m3 bytes when fp8
+  const void* W2;
   uint16_t* h;  // [rows, I] bf16
   float* y;     // [rows, H] fp32
   // Fused dispatch: packed row r of the group is row gather[r] of x (x_rows
@@ -90,6 +90,16 @@ struct FfnGroup {
   const int32_t* gather;
   int x_rows;
   bool packed;  // W13 / W2 in the tile-packed layout (moe_pack_weights)
+  // FP8 (e4m3) form: per-row fp32 scales of x (indexed by token through
+  // x_scale_idx when x holds packed copies, else by row), of W13 and W2 rows;
+  // hq / hs receive GEMM2's quantized operand and its row scales.
+  bool fp8;
+  const float* x_scale;
+  const int32_t* x_scale_idx;
+  const float* W13_scale;
+  const float* W2_scale;
+  uint8_t* hq;
+  float* hs;
 };
 
 // Routed group plus an optional dense group (the shared expert, same I) in one
@@ -111,6 +121,10 @@ moe_status launch_expert_ffn(int rows, int H, int I, int n_experts, int e_begin,
                              const uint16_t* W2, uint16_t* h, float* y_perm, int rows_hint,
                              cudaStream_t s, cudaEvent_t after_gemm1 = nullptr,
                              bool packed = false);
+
+// e4m3 row quantization of a bf16 matrix [rows, K] (K % 8 == 0).
+moe_status launch_quantize_rows(const uint16_t* in, long rows, int K, uint8_t* out, float* scale,
+                                cudaStream_t s);
 
 // Tile-packed copy of a bf16 weight matrix [rows, K] (rows % 128 == 0, K % 64 == 0).
 moe_status launch_pack_weights(const uint16_t* W, uint16_t* Wp, long rows, int K, cudaStream_t s);

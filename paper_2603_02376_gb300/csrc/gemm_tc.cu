@@ -37,6 +37,12 @@
 
 #include "common.cuh"
 
+#define MOE_STATUS_TRY(expr)          \
+  do {                                \
+    moe_status _st = (expr);          \
+    if (_st != MOE_OK) return _st;    \
+  } while (0)
+
 namespace moe {
 namespace {
 
@@ -199,6 +205,33 @@ __device__ __forceinline__ uint32_t idesc_bf16(int n) {
          ((uint32_t)(BM >> 4) << 24);
 }
 
+// Instruction descriptor, kind::f8f6f4 with e4m3 A and B (format code 0 in bits
+// 7-9 and 10-12), fp32 accumulator, K-major, same N / M fields.
+__device__ __forceinline__ uint32_t idesc_e4m3(int n) {
+  return (1u << 4) | ((uint32_t)(n >> 3) << 17) | ((uint32_t)(BM >> 4) << 24);
+}
+
+// One MMA of K = 32 e4m3 values (32 bytes, like K = 16 bf16).
+__device__ __forceinline__ void mma_e4m3(uint32_t d_tmem, uint64_t a, uint64_t b, uint32_t idesc,
+                                         uint32_t accumulate) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "setp.ne.b32 p, %4, 0;\n\t"
+      "tcgen05.mma.cta_group::1.kind::f8f6f4 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
+      "l"(a), "l"(b), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
+
+__device__ __forceinline__ void mma_bf16(uint32_t d_tmem, uint64_t a, uint64_t b, uint32_t idesc,
+                                         uint32_t accumulate);
+
+template <bool F8>
+__device__ __forceinline__ void mma_op(uint32_t d, uint64_t a, uint64_t b, uint32_t idesc,
+                                       uint32_t acc) {
+  if (F8) mma_e4m3(d, a, b, idesc, acc);
+  else mma_bf16(d, a, b, idesc, acc);
+}
+
 __device__ __forceinline__ void mma_bf16(uint32_t d_tmem, uint64_t a, uint64_t b, uint32_t idesc,
                                          uint32_t accumulate) {
   asm volatile(
@@ -251,6 +284,14 @@ struct GemmArgs {
   void* out1;
   int out_ld;
   int* err;
+  // FP8 only: fp32 scale of every weight row (a_scale*, indexed by the absolute
+  // weight row) and of every activation row (b_scale*, indexed by the B row, or
+  // through b_scale_idx0 for group 0 when the rows are packed copies of tokens)
+  const float* a_scale0;
+  const float* a_scale1;
+  const float* b_scale0;
+  const float* b_scale1;
+  const int32_t* b_scale_idx0;
   uint64_t wait_limit_ns;  // limit of each barrier wait
   long stall_fill;         // testing: CTA 0 never issues this fill (-1 = none), so the
                            // MMA's wait on it runs out and the abort path is exercised
@@ -310,7 +351,7 @@ __device__ __forceinline__ Unit decode_unit(int u, const int* tile_off, const in
 
 // ------------------------------------------------------------------ kernel
 
-template <int MODE, int NMAX>
+template <int MODE, int NMAX, bool F8>
 __global__ void __launch_bounds__(NUM_THREADS, 1)
     grouped_gemm_kernel(const __grid_constant__ CUtensorMap tmA0,
                         const __grid_constant__ CUtensorMap tmB0,
@@ -393,7 +434,8 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem_base = ctrl->tmem_base;
-  const int kblocks = a.K / BK;
+  constexpr int KE = F8 ? 2 * BK : BK;  // elements per k-block: one 128-byte row
+  const int kblocks = a.K / KE;
   const int units1 = a.rows1 > 0 ? ((a.rows1 + NMAX - 1) / NMAX) * a.n_fb * a.k_splits : 0;
   const int total_units = units1 + tile_off[a.n_exp] * a.n_fb;
 
@@ -459,13 +501,13 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
                 bulk_load_tile(sa + t * TL::A_BYTES,
                                ap + ((size_t)(r / BM) * kblocks + kb) * (BM * BK), full);
               else
-                tma_load_2d(sa + t * TL::A_BYTES, mA, kb * BK, r, full);
+                tma_load_2d(sa + t * TL::A_BYTES, mA, kb * KE, r, full);
             }
             if (!gather) {
               for (int i = 0; i < n_big; ++i)
-                tma_load_2d(sb + i * (B_BIG * BK * 2), mBbig, kb * BK, U.row0 + i * B_BIG, full);
+                tma_load_2d(sb + i * (B_BIG * BK * 2), mBbig, kb * KE, U.row0 + i * B_BIG, full);
               for (int i = n_big * (B_BIG / B_BOX); i < n_pad / B_BOX; ++i)
-                tma_load_2d(sb + i * (B_BOX * BK * 2), mB, kb * BK, U.row0 + i * B_BOX, full);
+                tma_load_2d(sb + i * (B_BOX * BK * 2), mB, kb * KE, U.row0 + i * B_BOX, full);
             }
           }
         }
@@ -479,7 +521,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
           for (int h = 0; h < 2; ++h) {
             const int g = lane + 32 * h;
             if (g < n_groups)
-              tma_gather4(sb + g * (4 * BK * 2), mB, kb * BK, gr[h][0], gr[h][1], gr[h][2],
+              tma_gather4(sb + g * (4 * BK * 2), mB, kb * KE, gr[h][0], gr[h][1], gr[h][2],
                           gr[h][3], full);
           }
         }
@@ -513,7 +555,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       for (int u = blockIdx.x; u < total_units && ok; u += gridDim.x, ++j) {
         const Unit U = decode_unit<NMAX>(u, tile_off, row_off, a, units1, kblocks);
         const int n_pad = (U.m + 15) & ~15;
-        const uint32_t idesc = idesc_bf16(n_pad);
+        const uint32_t idesc = F8 ? idesc_e4m3(n_pad) : idesc_bf16(n_pad);
         const int as = j % TL::ACC_STAGES;
         const uint32_t acc_par = (uint32_t)((j / TL::ACC_STAGES) & 1);
         if (!wait_bounded(smem_u32(&ctrl->acc_empty[as]), acc_par ^ 1, abort_flag, err,
@@ -536,12 +578,12 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
           for (int k = 0; k < BK / UMMA_K; ++k) {
             const uint32_t acc = (kb > U.kb0 || k > 0) ? 1u : 0u;
             const uint64_t bdesc = sdesc(sb + k * UMMA_K * 2);
-            mma_bf16(d, sdesc(sa + k * UMMA_K * 2), bdesc, idesc, acc);
+            mma_op<F8>(d, sdesc(sa + k * UMMA_K * 2), bdesc, idesc, acc);
             if (TL::TWO_ACC)
-              mma_bf16(d + NMAX, sdesc(sa + TL::A_BYTES + k * UMMA_K * 2), bdesc, idesc, acc);
+              mma_op<F8>(d + NMAX, sdesc(sa + TL::A_BYTES + k * UMMA_K * 2), bdesc, idesc, acc);
             if (MODE == MODE_SPLIT3) {  // the lower planes add into the same accumulator
-              mma_bf16(d, sdesc(sa + TL::A_BYTES + k * UMMA_K * 2), bdesc, idesc, 1u);
-              mma_bf16(d, sdesc(sa + 2 * TL::A_BYTES + k * UMMA_K * 2), bdesc, idesc, 1u);
+              mma_op<F8>(d, sdesc(sa + TL::A_BYTES + k * UMMA_K * 2), bdesc, idesc, 1u);
+              mma_op<F8>(d, sdesc(sa + 2 * TL::A_BYTES + k * UMMA_K * 2), bdesc, idesc, 1u);
             }
           }
           issued = true;
@@ -577,6 +619,23 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       const uint32_t tq = tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(as * TL::ACC_COLS);
       const int f = U.fb * TL::FEAT + q * 32 + lane;
       const size_t o = (size_t)U.row0 * a.out_ld + f;
+      // FP8: the scales of this thread's weight row(s) and of each token column
+      float sa0 = 1.f, sa1 = 1.f;
+      const float* bsc = nullptr;
+      const int32_t* bidx = nullptr;
+      if (F8) {
+        const float* asc = U.grp ? a.a_scale1 : a.a_scale0;
+        const int wr = (U.grp ? 0 : (a.e_begin + U.e) * a.w_rows0) + f;
+        sa0 = asc[wr];
+        if (TL::NA == 2) sa1 = asc[wr + a.up_off];
+        bsc = U.grp ? a.b_scale1 : a.b_scale0;
+        bidx = U.grp ? nullptr : a.b_scale_idx0;
+      }
+      auto col_scale = [&](int c) -> float {
+        if (!F8) return 1.f;
+        const int br = U.row0 + c;
+        return bsc[bidx ? bidx[br] : br];
+      };
       void* out = U.grp ? static_cast<void*>(static_cast<float*>(a.out1) + U.split * a.split_stride)
                         : a.out0;
       for (int c0 = 0; c0 < U.m; c0 += 16) {
@@ -589,8 +648,9 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
 #pragma unroll
           for (int i = 0; i < 16; ++i) {
             if (c0 + i < U.m) {
-              const float gv = __uint_as_float(g[i]);
-              const float uv = __uint_as_float(v[i]);
+              const float sb = col_scale(c0 + i);
+              const float gv = __uint_as_float(g[i]) * (sa0 * sb);
+              const float uv = __uint_as_float(v[i]) * (sa1 * sb);
               // silu(g) * u with the hardware exp2-based __expf and a reciprocal:
               // their error (a few fp32 ulp) is far below the bf16 rounding of h
               const float hv = gv * __frcp_rn(1.0f + __expf(-gv)) * uv;
@@ -604,9 +664,10 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
 #pragma unroll
           for (int i = 0; i < 16; ++i) {
             if (c0 + i < U.m) {
+              const float sb = col_scale(c0 + i);
               float* y = static_cast<float*>(out) + o + (size_t)(c0 + i) * a.out_ld;
-              y[0] = __uint_as_float(g[i]);
-              y[BM] = __uint_as_float(v[i]);
+              y[0] = __uint_as_float(g[i]) * (sa0 * sb);
+              y[BM] = __uint_as_float(v[i]) * (sa1 * sb);
             }
           }
         } else {
@@ -614,7 +675,8 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
 #pragma unroll
           for (int i = 0; i < 16; ++i) {
             if (c0 + i < U.m)
-              static_cast<float*>(out)[o + (size_t)(c0 + i) * a.out_ld] = __uint_as_float(g[i]);
+              static_cast<float*>(out)[o + (size_t)(c0 + i) * a.out_ld] =
+                  __uint_as_float(g[i]) * (sa0 * col_scale(c0 + i));
           }
         }
       }
@@ -681,43 +743,65 @@ size_t gemm_smem_bytes(int n_exp) {
   return 1024 + (size_t)TL::STAGES * TL::STAGE_BYTES + sizeof(Ctrl) + 2 * sizeof(int) * (n_exp + 1);
 }
 
-template <int MODE, int NMAX>
+template <int MODE, int NMAX, bool F8>
 moe_status launch_gemm(const CUtensorMap& A0, const CUtensorMap& B0, const CUtensorMap& A1,
                        const CUtensorMap& B1, const CUtensorMap& B0big, const CUtensorMap& B1big,
                        const GemmArgs& args, cudaStream_t s) {
   const size_t smem = gemm_smem_bytes<MODE, NMAX>(args.n_exp);
   if (smem > 227 * 1024) return MOE_ERR_UNSUPPORTED;
-  if (cudaFuncSetAttribute(grouped_gemm_kernel<MODE, NMAX>,
+  if (cudaFuncSetAttribute(grouped_gemm_kernel<MODE, NMAX, F8>,
                            cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) != cudaSuccess)
     return MOE_ERR_CUDA;
-  grouped_gemm_kernel<MODE, NMAX><<<num_sms(), NUM_THREADS, smem, s>>>(A0, B0, A1, B1, B0big,
-                                                                       B1big, args);
+  grouped_gemm_kernel<MODE, NMAX, F8><<<num_sms(), NUM_THREADS, smem, s>>>(A0, B0, A1, B1, B0big,
+                                                                           B1big, args);
   note_launch();
   return launch_status();
 }
 
-template <int NMAX>
+// Row-major [rows, cols] operand map with (one 128-byte row segment) x box_rows
+// boxes: bf16 elements, or e4m3 bytes for the FP8 form.
+template <bool F8>
+bool make_rows_map(CUtensorMap* m, const void* ptr, uint64_t cols, uint64_t rows,
+                   uint32_t box_rows) {
+  if (!F8) return make_map(m, ptr, cols, rows, BK, box_rows);
+  auto fn = encode_fn();
+  if (!fn) return false;
+  cuuint64_t dims[2] = {cols, rows};
+  cuuint64_t strides[1] = {cols};
+  cuuint32_t box[2] = {2 * BK, box_rows};
+  cuuint32_t estr[2] = {1, 1};
+  return fn(m, CU_TENSOR_MAP_DATA_TYPE_UINT8, 2, const_cast<void*>(ptr), dims, strides, box, estr,
+            CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+            CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+template <int NMAX, bool F8>
 moe_status run_ffn(const FfnGroup& g0, const FfnGroup* g1, int H, int I, cudaStream_t s,
                    cudaEvent_t after_gemm1) {
   CUtensorMap a1, b1, a2, b2, sa1, sb1, sa2, sb2, b1big, b2big, sb1big, sb2big;
   // with a fused dispatch GEMM1 reads token rows of x by index: a one-row box
   const bool gather = g0.gather != nullptr;
   const bool pk = g0.packed;
-  if (!make_weight_map(&a1, g0.W13, H, (uint64_t)g0.n_experts * 2 * I, pk) ||
-      !make_map(&b1, g0.x, H, gather ? g0.x_rows : g0.rows, BK, gather ? 1 : B_BOX) ||
-      !make_weight_map(&a2, g0.W2, I, (uint64_t)g0.n_experts * H, pk) ||
-      !make_map(&b2, g0.h, I, g0.rows, BK, B_BOX) ||
-      !make_map(&b1big, g0.x, H, gather ? g0.x_rows : g0.rows, BK, gather ? 1 : B_BIG) ||
-      !make_map(&b2big, g0.h, I, g0.rows, BK, B_BIG))
+  if (F8 && pk) return MOE_ERR_UNSUPPORTED;  // packed tiles are bf16 only
+  const uint64_t xr = gather ? g0.x_rows : g0.rows;
+  // GEMM2's token operand: h (bf16), or its e4m3 copy hq in the FP8 form
+  const void* h0 = F8 ? static_cast<const void*>(g0.hq) : static_cast<const void*>(g0.h);
+  if (!make_rows_map<F8>(&a1, g0.W13, H, (uint64_t)g0.n_experts * 2 * I, BM) ||
+      !make_rows_map<F8>(&b1, g0.x, H, xr, gather ? 1 : B_BOX) ||
+      !make_rows_map<F8>(&a2, g0.W2, I, (uint64_t)g0.n_experts * H, BM) ||
+      !make_rows_map<F8>(&b2, h0, I, g0.rows, B_BOX) ||
+      !make_rows_map<F8>(&b1big, g0.x, H, xr, gather ? 1 : B_BIG) ||
+      !make_rows_map<F8>(&b2big, h0, I, g0.rows, B_BIG))
     return MOE_ERR_CUDA;
   if (g1) {
-    if (g1->packed != g0.packed) return MOE_ERR_INVALID_ARG;
-    if (!make_weight_map(&sa1, g1->W13, H, (uint64_t)2 * I, pk) ||
-        !make_map(&sb1, g1->x, H, g1->rows, BK, B_BOX) ||
-        !make_weight_map(&sa2, g1->W2, I, (uint64_t)H, pk) ||
-        !make_map(&sb2, g1->h, I, g1->rows, BK, B_BOX) ||
-        !make_map(&sb1big, g1->x, H, g1->rows, BK, B_BIG) ||
-        !make_map(&sb2big, g1->h, I, g1->rows, BK, B_BIG))
+    if (g1->packed != g0.packed || g1->fp8 != g0.fp8) return MOE_ERR_INVALID_ARG;
+    const void* h1 = F8 ? static_cast<const void*>(g1->hq) : static_cast<const void*>(g1->h);
+    if (!make_rows_map<F8>(&sa1, g1->W13, H, (uint64_t)2 * I, BM) ||
+        !make_rows_map<F8>(&sb1, g1->x, H, g1->rows, B_BOX) ||
+        !make_rows_map<F8>(&sa2, g1->W2, I, (uint64_t)H, BM) ||
+        !make_rows_map<F8>(&sb2, h1, I, g1->rows, B_BOX) ||
+        !make_rows_map<F8>(&sb1big, g1->x, H, g1->rows, B_BIG) ||
+        !make_rows_map<F8>(&sb2big, h1, I, g1->rows, B_BIG))
       return MOE_ERR_CUDA;
   } else {
     sa1 = a1;  // unused: group 1 is empty
@@ -729,8 +813,8 @@ moe_status run_ffn(const FfnGroup& g0, const FfnGroup* g1, int H, int I, cudaStr
   }
   GemmArgs args{};
   args.k_splits = 1;
-  args.a0_packed = pk ? g0.W13 : nullptr;
-  args.a1_packed = (pk && g1) ? g1->W13 : nullptr;
+  args.a0_packed = pk ? static_cast<const uint16_t*>(g0.W13) : nullptr;
+  args.a1_packed = (pk && g1) ? static_cast<const uint16_t*>(g1->W13) : nullptr;
   args.wait_limit_ns = g_wait_limit_ns;
   args.stall_fill = g_stall_fill;
   args.offsets = g0.offsets;
@@ -748,12 +832,30 @@ moe_status run_ffn(const FfnGroup& g0, const FfnGroup* g1, int H, int I, cudaStr
   args.out0 = g0.h;
   args.out1 = g1 ? g1->h : nullptr;
   args.out_ld = I;
-  moe_status st = launch_gemm<MODE_SWIGLU, NMAX>(a1, b1, sa1, sb1, b1big, sb1big, args, s);
+  if (F8) {
+    args.a_scale0 = g0.W13_scale;
+    args.a_scale1 = g1 ? g1->W13_scale : nullptr;
+    args.b_scale0 = g0.x_scale;
+    args.b_scale1 = g1 ? g1->x_scale : nullptr;
+    args.b_scale_idx0 = g0.x_scale_idx;
+  }
+  moe_status st = launch_gemm<MODE_SWIGLU, NMAX, F8>(a1, b1, sa1, sb1, b1big, sb1big, args, s);
   if (st != MOE_OK) return st;
+  if (F8) {  // h of every packed row -> e4m3 and its row scale: GEMM2's operand
+    MOE_STATUS_TRY(launch_quantize_rows(g0.h, g0.rows, I, g0.hq, g0.hs, s));
+    if (g1) MOE_STATUS_TRY(launch_quantize_rows(g1->h, g1->rows, I, g1->hq, g1->hs, s));
+  }
   if (after_gemm1 && cudaEventRecord(after_gemm1, s) != cudaSuccess) return MOE_ERR_CUDA;
   args.gather0 = nullptr;  // GEMM2 reads h, already in packed row order
-  args.a0_packed = pk ? g0.W2 : nullptr;
-  args.a1_packed = (pk && g1) ? g1->W2 : nullptr;
+  args.a0_packed = pk ? static_cast<const uint16_t*>(g0.W2) : nullptr;
+  args.a1_packed = (pk && g1) ? static_cast<const uint16_t*>(g1->W2) : nullptr;
+  if (F8) {
+    args.a_scale0 = g0.W2_scale;
+    args.a_scale1 = g1 ? g1->W2_scale : nullptr;
+    args.b_scale0 = g0.hs;
+    args.b_scale1 = g1 ? g1->hs : nullptr;
+    args.b_scale_idx0 = nullptr;
+  }
   // GEMM2: y = h W2^T (fp32). With prefill-sized token tiles, two 128-feature
   // weight tiles per unit share one token tile (more weight bytes per stage);
   // with decode-sized tiles a single weight tile and a deeper ring measured faster.
@@ -765,11 +867,11 @@ moe_status run_ffn(const FfnGroup& g0, const FfnGroup* g1, int H, int I, cudaStr
   if (NMAX > 32 && H % (2 * BM) == 0) {
     args.n_fb = H / (2 * BM);
     args.up_off = BM;
-    return launch_gemm<MODE_PLAIN2, NMAX>(a2, b2, sa2, sb2, b2big, sb2big, args, s);
+    return launch_gemm<MODE_PLAIN2, NMAX, F8>(a2, b2, sa2, sb2, b2big, sb2big, args, s);
   }
   args.n_fb = H / BM;
   args.up_off = 0;
-  return launch_gemm<MODE_PLAIN, NMAX>(a2, b2, sa2, sb2, b2big, sb2big, args, s);
+  return launch_gemm<MODE_PLAIN, NMAX, F8>(a2, b2, sa2, sb2, b2big, sb2big, args, s);
 }
 
 }  // namespace
@@ -784,9 +886,14 @@ moe_status launch_expert_ffn_groups(const FfnGroup& routed, const FfnGroup* dens
   // of the stage ring to weights (decode ~4 rows/expert -> 32; balanced
   // prefill ~128 +- 10 % -> 144; larger or skewed loads -> 256).
   const long per = (long)rows_hint / (n_exp > 0 ? n_exp : 1);
-  if (per <= 24) return run_ffn<32>(routed, g1, H, I, s, after_gemm1);
-  if (per <= 132) return run_ffn<144>(routed, g1, H, I, s, after_gemm1);
-  return run_ffn<256>(routed, g1, H, I, s, after_gemm1);
+  if (routed.fp8) {
+    if (per <= 24) return run_ffn<32, true>(routed, g1, H, I, s, after_gemm1);
+    if (per <= 132) return run_ffn<144, true>(routed, g1, H, I, s, after_gemm1);
+    return run_ffn<256, true>(routed, g1, H, I, s, after_gemm1);
+  }
+  if (per <= 24) return run_ffn<32, false>(routed, g1, H, I, s, after_gemm1);
+  if (per <= 132) return run_ffn<144, false>(routed, g1, H, I, s, after_gemm1);
+  return run_ffn<256, false>(routed, g1, H, I, s, after_gemm1);
 }
 
 int router_tc_splits(int T, int H, int E) {
@@ -816,7 +923,7 @@ moe_status launch_router_tc(int T, int H, int E, const uint16_t* x, const uint16
   args.out1 = partials;
   args.out_ld = E;
   args.err = device_error_word();
-  return launch_gemm<MODE_SPLIT3, 128>(A, B, A, B, Bbig, Bbig, args, s);
+  return launch_gemm<MODE_SPLIT3, 128, false>(A, B, A, B, Bbig, Bbig, args, s);
 }
 
 moe_status launch_expert_ffn_stalled(int rows, int H, int I, int n_experts, const uint16_t* x_perm,
@@ -825,7 +932,16 @@ moe_status launch_expert_ffn_stalled(int rows, int H, int I, int n_experts, cons
                                      long stall_fill, uint64_t wait_limit_ns, cudaStream_t s) {
   g_wait_limit_ns = wait_limit_ns;
   g_stall_fill = stall_fill;
-  FfnGroup g{x_perm, offsets, rows, n_experts, 0, n_experts, W13, W2, h, y_perm, nullptr, 0, false};
+  FfnGroup g{};
+  g.x = x_perm;
+  g.offsets = offsets;
+  g.rows = rows;
+  g.n_experts = n_experts;
+  g.e_end = n_experts;
+  g.W13 = W13;
+  g.W2 = W2;
+  g.h = h;
+  g.y = y_perm;
   const moe_status st = launch_expert_ffn_groups(g, nullptr, H, I, rows, s);
   g_wait_limit_ns = WAIT_LIMIT_NS;
   g_stall_fill = -1;
@@ -837,8 +953,18 @@ moe_status launch_expert_ffn(int rows, int H, int I, int n_experts, int e_begin,
                              const uint16_t* W2, uint16_t* h, float* y_perm, int rows_hint,
                              cudaStream_t s, cudaEvent_t after_gemm1, bool packed) {
   if (rows == 0 || e_end <= e_begin) return MOE_OK;
-  FfnGroup g{x_perm, offsets, rows, n_experts, e_begin, e_end, W13, W2, h, y_perm, nullptr, 0,
-             packed};
+  FfnGroup g{};
+  g.x = x_perm;
+  g.offsets = offsets;
+  g.rows = rows;
+  g.n_experts = n_experts;
+  g.e_begin = e_begin;
+  g.e_end = e_end;
+  g.W13 = W13;
+  g.W2 = W2;
+  g.h = h;
+  g.y = y_perm;
+  g.packed = packed;
   return launch_expert_ffn_groups(g, nullptr, H, I, rows_hint, s, after_gemm1);
 }
 

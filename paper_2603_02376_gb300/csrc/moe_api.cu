@@ -85,6 +85,7 @@ bool valid_exec(const moe_exec* ex, const moe_config* c) {
   if (ex->overlap != 0 && ex->overlap != 1) return false;
   if (ex->out_fp32 != 0 && ex->out_fp32 != 1) return false;
   if (ex->fuse_gather != 0 && ex->fuse_gather != 1) return false;
+  if (ex->fp8 != 0 && ex->fp8 != 1) return false;
   if (ex->overlap) {
     if (ex->chunk_axis == 0) {
       if (ex->chunk_tokens < 1) return false;
@@ -124,11 +125,18 @@ struct Layout {
   int32_t* perm_counts;
   int32_t* perm_base;
   void* router_ws;   // router scratch (planes + partials), sized for one chunk
-  uint16_t* x_perm;  // [T*k, H]
+  bool fp8 = false;
+  uint8_t* x_q;      // [T, H] e4m3 (fp8 only)
+  float* x_s;        // [T] row scales of x_q
+  void* x_perm;      // [T*k, H] bf16, or e4m3 bytes (fp8)
   uint16_t* h;       // [T*k, I]
+  uint8_t* hq;       // [T*k, I] e4m3 copy of h (fp8 only)
+  float* hs;         // [T*k] its row scales
   float* y_perm;     // [T*k, H] fp32
   int32_t* sh_off;   // [2]
   uint16_t* sh_h;    // [T, I_s]
+  uint8_t* sh_hq;    // [T, I_s] (fp8 only)
+  float* sh_hs;      // [T]
   float* sh_y;       // [T, H] fp32
   size_t bytes = 0;
 };
@@ -161,11 +169,19 @@ Layout carve(const moe_config& c, const moe_exec& ex, void* ws) {
   // measured 1.8x slower GEMM1 at ~128 rows per expert. It is used when a
   // chunk averages at most 24 rows per expert.
   const bool fuse = ex.fuse_gather && (long)L.chunk_T * c.k <= 24L * c.E;
-  L.x_perm = fuse ? nullptr : cv.take<uint16_t>(T * k * c.H);
+  L.fp8 = ex.fp8 != 0;
+  const size_t xb = L.fp8 ? 1 : 2;  // bytes per activation element
+  L.x_q = L.fp8 ? cv.take<uint8_t>(T * c.H) : nullptr;
+  L.x_s = L.fp8 ? cv.take<float>(T) : nullptr;
+  L.x_perm = fuse ? nullptr : static_cast<void*>(cv.take<uint8_t>(T * k * c.H * xb));
   L.h = cv.take<uint16_t>(T * k * c.I);
+  L.hq = L.fp8 ? cv.take<uint8_t>(T * k * c.I) : nullptr;
+  L.hs = L.fp8 ? cv.take<float>(T * k) : nullptr;
   L.y_perm = cv.take<float>(T * k * c.H);
   L.sh_off = cv.take<int32_t>(2);
   L.sh_h = c.I_shared ? cv.take<uint16_t>(T * c.I_shared) : nullptr;
+  L.sh_hq = (c.I_shared && L.fp8) ? cv.take<uint8_t>(T * c.I_shared) : nullptr;
+  L.sh_hs = (c.I_shared && L.fp8) ? cv.take<float>(T) : nullptr;
   L.sh_y = c.I_shared ? cv.take<float>(T * c.H) : nullptr;
   L.bytes = align_up(cv.off, 256);
   return L;
@@ -211,9 +227,19 @@ moe_status mark(cudaEvent_t* ev, int i, cudaStream_t s) {
   return MOE_OK;
 }
 
+// FP8: rows [t0, t0+Tc) of x -> e4m3 rows of x_q and their scales.
+moe_status quantize_tokens(const moe_config& c, const Layout& L, const uint16_t* x, int t0, int Tc,
+                           cudaStream_t s) {
+  return launch_quantize_rows(x + (size_t)t0 * c.H, Tc, c.H, L.x_q + (size_t)t0 * c.H, L.x_s + t0,
+                              s);
+}
+
+// With quantize (FP8 only) the chunk's rows are quantized after the
+// permutation, inside the dispatch stage; the pipelined modes quantize all
+// rows up front instead (the shared expert reads them on the other stream).
 moe_status pack_tokens(const moe_config& c, const Layout& L, const moe_weights& w,
                        const uint16_t* x, int t0, int Tc, int ci, bool pack_rows,
-                       cudaStream_t s, cudaEvent_t* ev = nullptr) {
+                       cudaStream_t s, cudaEvent_t* ev = nullptr, bool quantize = false) {
   moe_config cc = c;
   cc.T = Tc;
   const size_t tk = (size_t)t0 * c.k;
@@ -226,9 +252,19 @@ moe_status pack_tokens(const moe_config& c, const Layout& L, const moe_weights& 
                              L.offsets + (size_t)ci * (c.E + 1), L.rst + tk, L.slot_row + tk,
                              L.perm_counts, L.perm_base, s));
   MOE_TRY(mark(ev, MOE_EV_PERMUTE, s));
-  if (pack_rows)
+  if (L.fp8) {
+    // quantize, then dispatch the e4m3 rows: a row of H bytes is copied as
+    // H / 2 two-byte units by the same copy kernel
+    if (quantize) MOE_TRY(quantize_tokens(c, L, x, t0, Tc, s));
+    if (pack_rows)
+      MOE_TRY(launch_dispatch_rows(Tc, c.H / 2, c.k,
+                                   reinterpret_cast<const uint16_t*>(L.x_q + (size_t)t0 * c.H),
+                                   L.slot_row + tk,
+                                   static_cast<uint16_t*>(L.x_perm) + tk * c.H / 2, s));
+  } else if (pack_rows) {
     MOE_TRY(launch_dispatch_rows(Tc, c.H, c.k, x + (size_t)t0 * c.H, L.slot_row + tk,
-                                 L.x_perm + tk * c.H, s));
+                                 static_cast<uint16_t*>(L.x_perm) + tk * c.H, s));
+  }
   MOE_TRY(mark(ev, MOE_EV_DISPATCH, s));
   return MOE_OK;
 }
@@ -250,12 +286,49 @@ FfnGroup routed_group(const moe_config& c, const Layout& L, const moe_weights& w
   g.packed = w.packed != 0;
   g.h = L.h + tk * c.I;
   g.y = L.y_perm + tk * c.H;
+  const size_t xb = L.fp8 ? 1 : 2;
   if (L.x_perm) {
-    g.x = L.x_perm + tk * c.H;
+    g.x = static_cast<const uint8_t*>(L.x_perm) + tk * c.H * xb;
   } else {
-    g.x = x + (size_t)t0 * c.H;
+    g.x = L.fp8 ? static_cast<const void*>(L.x_q + (size_t)t0 * c.H)
+                : static_cast<const void*>(x + (size_t)t0 * c.H);
     g.gather = L.rst + tk;
     g.x_rows = Tc;
+  }
+  if (L.fp8) {
+    g.fp8 = true;
+    g.x_scale = L.x_s + t0;  // per token of the chunk, reached through row_src_token
+    g.x_scale_idx = L.rst + tk;
+    g.W13_scale = w.W13_scale;
+    g.W2_scale = w.W2_scale;
+    g.hq = L.hq + tk * c.I;
+    g.hs = L.hs + tk;
+  }
+  return g;
+}
+
+// The shared expert as a one-expert group over all T tokens (offsets {0, T}).
+FfnGroup dense_group(const moe_config& c, const Layout& L, const moe_weights& w,
+                     const uint16_t* x) {
+  FfnGroup g{};
+  g.offsets = L.sh_off;
+  g.rows = c.T;
+  g.n_experts = 1;
+  g.e_end = 1;
+  g.W13 = w.Ws13;
+  g.W2 = w.Ws2;
+  g.h = L.sh_h;
+  g.y = L.sh_y;
+  g.packed = w.packed != 0;
+  g.x = x;
+  if (L.fp8) {
+    g.fp8 = true;
+    g.x = L.x_q;
+    g.x_scale = L.x_s;
+    g.W13_scale = w.Ws13_scale;
+    g.W2_scale = w.Ws2_scale;
+    g.hq = L.sh_hq;
+    g.hs = L.sh_hs;
   }
   return g;
 }
@@ -277,9 +350,9 @@ moe_status shared_expert(const moe_config& c, const Layout& L, const moe_weights
     return mark(ev, MOE_EV_SHARED_GEMM2, s);
   }
   MOE_TRY(launch_fill_range(L.sh_off, c.T, s));
-  MOE_TRY(launch_expert_ffn(c.T, c.H, c.I_shared, 1, 0, 1, x, L.sh_off, w.Ws13, w.Ws2, L.sh_h,
-                            L.sh_y, c.T, s, ev ? ev[MOE_EV_SHARED_GEMM1] : nullptr,
-                            w.packed != 0));
+  const FfnGroup g = dense_group(c, L, w, x);
+  MOE_TRY(launch_expert_ffn_groups(g, nullptr, c.H, c.I_shared, c.T, s,
+                                   ev ? ev[MOE_EV_SHARED_GEMM1] : nullptr));
   return mark(ev, MOE_EV_SHARED_GEMM2, s);
 }
 
@@ -290,8 +363,7 @@ moe_status experts_and_shared(const moe_config& c, const Layout& L, const moe_we
                               const uint16_t* x, cudaStream_t s, cudaEvent_t* ev) {
   MOE_TRY(launch_fill_range(L.sh_off, c.T, s));
   const FfnGroup routed = routed_group(c, L, w, x, 0, c.T, 0, 0, c.E);
-  FfnGroup dense{x, L.sh_off, c.T, 1, 0, 1, w.Ws13, w.Ws2, L.sh_h, L.sh_y, nullptr, 0,
-                 w.packed != 0};
+  const FfnGroup dense = dense_group(c, L, w, x);
   MOE_TRY(launch_expert_ffn_groups(routed, &dense, c.H, c.I, routed.rows, s,
                                    ev ? ev[MOE_EV_GEMM1] : nullptr));
   MOE_TRY(mark(ev, MOE_EV_GEMM2, s));
@@ -423,6 +495,64 @@ moe_status moe_expert_ffn(int32_t rows, int32_t H, int32_t I, int32_t n_experts,
                            weights_packed != 0);
 }
 
+size_t moe_expert_ffn_fp8_workspace_size(int32_t rows, int32_t I) {
+  if (rows < 0 || I < 0) return 0;
+  Carver cv(nullptr);
+  cv.take<uint16_t>((size_t)rows * I);
+  cv.take<uint8_t>((size_t)rows * I);
+  cv.take<float>((size_t)rows);
+  return align_up(cv.off, 256);
+}
+
+moe_status moe_quantize_fp8(int64_t rows, int32_t K, const uint16_t* in, uint8_t* out,
+                            float* scale, void* stream) {
+  if (rows < 0 || rows > (1LL << 31) || K < 16 || K % 16 || K > 65536) return MOE_ERR_INVALID_ARG;
+  if (rows == 0) return MOE_OK;
+  if (!in || !out || !scale || !aligned16(in) || !aligned16(out) || !aligned4(scale))
+    return MOE_ERR_INVALID_ARG;
+  const uint8_t *a = (const uint8_t*)in, *b = out;
+  if (a < b + (size_t)rows * K && b < a + (size_t)rows * K * 2) return MOE_ERR_INVALID_ARG;
+  return launch_quantize_rows(in, (long)rows, K, out, scale, (cudaStream_t)stream);
+}
+
+moe_status moe_expert_ffn_fp8(int32_t rows, int32_t H, int32_t I, int32_t n_experts,
+                              const uint8_t* x_q, const float* x_scale,
+                              const int32_t* x_scale_idx, const int32_t* offsets,
+                              const uint8_t* W13_q, const float* W13_scale, const uint8_t* W2_q,
+                              const float* W2_scale, float* y_perm, void* ws, size_t ws_bytes,
+                              void* stream) {
+  if (rows < 0 || H < 128 || H % 128 || H > 65536 || I < 128 || I % 128 || I > 65536 ||
+      n_experts < 1 || n_experts > 1024)
+    return MOE_ERR_INVALID_ARG;
+  if (rows == 0) return MOE_OK;
+  if (!x_q || !x_scale || !offsets || !W13_q || !W13_scale || !W2_q || !W2_scale || !y_perm ||
+      !aligned16(x_q) || !aligned16(W13_q) || !aligned16(W2_q) || !aligned16(y_perm) ||
+      !aligned4(offsets) || !aligned4(x_scale) || !aligned4(W13_scale) || !aligned4(W2_scale) ||
+      (x_scale_idx && !aligned4(x_scale_idx)))
+    return MOE_ERR_INVALID_ARG;
+  if (!ws || ws_bytes < moe_expert_ffn_fp8_workspace_size(rows, I) || ((uintptr_t)ws & 255))
+    return MOE_ERR_WORKSPACE;
+  Carver cv(ws);
+  FfnGroup g{};
+  g.x = x_q;
+  g.offsets = offsets;
+  g.rows = rows;
+  g.n_experts = n_experts;
+  g.e_end = n_experts;
+  g.W13 = W13_q;
+  g.W2 = W2_q;
+  g.h = cv.take<uint16_t>((size_t)rows * I);
+  g.hq = cv.take<uint8_t>((size_t)rows * I);
+  g.hs = cv.take<float>((size_t)rows);
+  g.y = y_perm;
+  g.fp8 = true;
+  g.x_scale = x_scale;
+  g.x_scale_idx = x_scale_idx;
+  g.W13_scale = W13_scale;
+  g.W2_scale = W2_scale;
+  return launch_expert_ffn_groups(g, nullptr, H, I, rows, (cudaStream_t)stream);
+}
+
 moe_status moe_testing_expert_ffn_stall(int32_t rows, int32_t H, int32_t I, int32_t n_experts,
                                         const uint16_t* x_perm, const int32_t* offsets,
                                         const uint16_t* W13, const uint16_t* W2, float* y_perm,
@@ -460,6 +590,14 @@ moe_status moe_layer_forward(const moe_config* cfg, const moe_exec* ex, const mo
   if (!valid_config(cfg) || !valid_exec(ex, cfg) || !w) return MOE_ERR_INVALID_ARG;
   if (w->packed != 0 && w->packed != 1) return MOE_ERR_INVALID_ARG;
   const moe_config& c = *cfg;
+  if (ex->fp8) {  // e4m3 expert weights with row scales; no packed form
+    if (w->packed) return MOE_ERR_UNSUPPORTED;
+    if (!w->W13_scale || !w->W2_scale || !aligned4(w->W13_scale) || !aligned4(w->W2_scale))
+      return MOE_ERR_INVALID_ARG;
+    if (c.I_shared && (!w->Ws13_scale || !w->Ws2_scale || !aligned4(w->Ws13_scale) ||
+                       !aligned4(w->Ws2_scale)))
+      return MOE_ERR_INVALID_ARG;
+  }
   if (!w->Wr || !w->W13 || !w->W2 || !aligned16(w->Wr) || !aligned16(w->W13) ||
       !aligned16(w->W2) || (w->bias && !aligned4(w->bias)))
     return MOE_ERR_INVALID_ARG;
@@ -484,7 +622,7 @@ moe_status moe_layer_forward(const moe_config* cfg, const moe_exec* ex, const mo
   if (!ex->overlap) {
     cudaEvent_t* ev = reinterpret_cast<cudaEvent_t*>(ex->stage_events);
     MOE_TRY(mark(ev, MOE_EV_START, s));
-    MOE_TRY(pack_tokens(c, L, *w, x, 0, c.T, 0, L.x_perm != nullptr, s, ev));
+    MOE_TRY(pack_tokens(c, L, *w, x, 0, c.T, 0, L.x_perm != nullptr, s, ev, true));
     if (c.I_shared == c.I) {
       MOE_TRY(experts_and_shared(c, L, *w, x, s, ev));
     } else {
@@ -504,6 +642,7 @@ moe_status moe_layer_forward(const moe_config* cfg, const moe_exec* ex, const mo
   const int n_stage = ex->chunk_axis == 0 ? L.n_chunks : ex->n_expert_chunks;
   std::vector<cudaEvent_t> ev;
   if (!events(dev, (size_t)n_stage + 1, &ev)) return MOE_ERR_CUDA;
+  if (L.fp8) MOE_TRY(quantize_tokens(c, L, x, 0, c.T, s));  // before the fork: both streams read x_q
   // the pack stream starts after everything already queued on `stream`
   MOE_CUDA(cudaEventRecord(ev[n_stage], s));
   MOE_CUDA(cudaStreamWaitEvent(ps, ev[n_stage], 0));
@@ -533,8 +672,13 @@ moe_status moe_layer_forward(const moe_config* cfg, const moe_exec* ex, const mo
   const int nr = ex->n_expert_chunks;
   for (int r = 0; r < nr; ++r) {
     const int e0 = (int)((long)c.E * r / nr), e1 = (int)((long)c.E * (r + 1) / nr);
-    if (L.x_perm)  // with a fused dispatch GEMM1 gathers the rows itself
-      MOE_TRY(launch_gather_rows(c.H, x, L.rst, L.offsets, e0, e1, L.x_perm, c.T * c.k, ps));
+    if (L.x_perm && L.fp8)  // e4m3 rows: H bytes = H / 2 two-byte units
+      MOE_TRY(launch_gather_rows(c.H / 2, reinterpret_cast<const uint16_t*>(L.x_q), L.rst,
+                                 L.offsets, e0, e1, static_cast<uint16_t*>(L.x_perm), c.T * c.k,
+                                 ps));
+    else if (L.x_perm)  // with a fused dispatch GEMM1 gathers the rows itself
+      MOE_TRY(launch_gather_rows(c.H, x, L.rst, L.offsets, e0, e1,
+                                 static_cast<uint16_t*>(L.x_perm), c.T * c.k, ps));
     MOE_CUDA(cudaEventRecord(ev[r], ps));
   }
   MOE_TRY(shared_expert(c, L, *w, x, s));  // overlaps routing on the pack stream

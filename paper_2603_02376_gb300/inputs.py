@@ -75,7 +75,8 @@ WORKLOADS = {"tiny": TINY, "decode": DECODE, "prefill": PREFILL, "skewed": SKEWE
 DISPATCH_SWEEP_T = (1024, 4096, 16384, 65536)
 
 _SUB = {"x": 1, "Wr": 2, "bias": 3, "W13": 4, "W2": 5, "Ws13": 6, "Ws2": 7,
-        "resample": 8, "zipf": 9, "sample": 10, "route": 11}
+        "resample": 8, "zipf": 9, "sample": 10, "route": 11, "W13q": 12, "W2q": 13,
+        "Ws13q": 14, "Ws2q": 15}
 
 
 def generator(seed: int, what: str, device, extra: int = 0) -> torch.Generator:
@@ -107,6 +108,49 @@ def expert_weights(wl: Workload, seed: int, device, experts=None):
         W13[n] = randn((2 * wl.I, wl.H), 0.02, torch.bfloat16, seed, "W13", device, extra=e)
         W2[n] = randn((wl.H, wl.I), 0.02, torch.bfloat16, seed, "W2", device, extra=e)
     return W13, W2
+
+
+# FP8 expert weights are drawn in their stored form: e4m3 bytes plus one fp32
+# scale per row, as an FP8 checkpoint holds them. Bytes: a random sign and a
+# magnitude code uniform over 0x30..0x7E (values 0.5 .. 448, ten binades, no
+# NaN code); row scales 2^-14 * U[1, 2), so the weights span about +-0.05 like
+# the N(0, 0.02^2) bf16 ones.
+E4M3_CODE_LO, E4M3_CODE_HI = 0x30, 0x7E
+
+
+def e4m3_codes(shape, seed, what, device, extra=0):
+    """(uint8 e4m3 bytes of `shape`, fp32 scales [prod(shape[:-1])]) for one weight matrix."""
+    g = generator(seed, what, device, extra)
+    mag = torch.randint(E4M3_CODE_LO, E4M3_CODE_HI + 1, shape, generator=g, device=device,
+                        dtype=torch.int32)
+    sgn = torch.randint(0, 2, shape, generator=g, device=device, dtype=torch.int32)
+    codes = (mag + 128 * sgn).to(torch.uint8)
+    rows = codes.numel() // shape[-1]
+    scale = (torch.rand(rows, generator=g, device=device, dtype=torch.float32) + 1.0) * 2.0 ** -14
+    return codes, scale
+
+
+def fp8_expert_weights(wl: Workload, seed: int, device, experts=None):
+    """FP8 routed-expert weights: W13 bytes [E, 2I, H] with scales [E, 2I], W2 bytes
+    [E, H, I] with scales [E, H]; drawn expert by expert like expert_weights."""
+    es = range(wl.E) if experts is None else experts
+    W13 = torch.empty((len(es), 2 * wl.I, wl.H), dtype=torch.uint8, device=device)
+    W2 = torch.empty((len(es), wl.H, wl.I), dtype=torch.uint8, device=device)
+    s13 = torch.empty((len(es), 2 * wl.I), dtype=torch.float32, device=device)
+    s2 = torch.empty((len(es), wl.H), dtype=torch.float32, device=device)
+    for n, e in enumerate(es):
+        W13[n], s13[n] = e4m3_codes((2 * wl.I, wl.H), seed, "W13q", device, extra=e)
+        W2[n], s2[n] = e4m3_codes((wl.H, wl.I), seed, "W2q", device, extra=e)
+    return W13, s13, W2, s2
+
+
+def fp8_shared_weights(wl: Workload, seed: int, device):
+    """FP8 shared-expert weights (Ws13, Ws13 scales, Ws2, Ws2 scales), or four Nones."""
+    if not wl.I_shared:
+        return None, None, None, None
+    Ws13, ss13 = e4m3_codes((2 * wl.I_shared, wl.H), seed, "Ws13q", device)
+    Ws2, ss2 = e4m3_codes((wl.H, wl.I_shared), seed, "Ws2q", device)
+    return Ws13, ss13, Ws2, ss2
 
 
 def layer_inputs(wl: Workload, seed: int = 0, device="cpu", with_experts=True):

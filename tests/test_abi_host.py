@@ -124,6 +124,49 @@ def test_entry_points_reject_bad_arguments_without_a_gpu(lib):
     assert lib.moe_layer_forward(cb(c), cb(exb), cb(W), p, p, None, p, 1 << 40, z, z) == L.MOE_ERR_INVALID_ARG
 
 
+def test_fp8_entry_points_reject_bad_arguments_without_a_gpu(lib):
+    c = L.config(**GOOD)
+    z = ctypes.c_void_p(0)
+    p = ctypes.c_void_p(0x1000)
+    q = ctypes.c_void_p(0x100000)     # a second buffer far from p
+    odd = ctypes.c_void_p(0x1008)     # 8-byte aligned only
+    cb = ctypes.byref
+    Q = lib.moe_quantize_fp8
+    assert Q(16, 100, p, q, q, z) == L.MOE_ERR_INVALID_ARG          # K % 16
+    assert Q(16, 8, p, q, q, z) == L.MOE_ERR_INVALID_ARG            # K < 16
+    assert Q(-1, 128, p, q, q, z) == L.MOE_ERR_INVALID_ARG
+    assert Q(16, 128, p, p, q, z) == L.MOE_ERR_INVALID_ARG          # in and out overlap
+    assert Q(16, 128, odd, q, q, z) == L.MOE_ERR_INVALID_ARG
+    assert Q(16, 128, p, q, z, z) == L.MOE_ERR_INVALID_ARG          # no scale buffer
+    assert Q(0, 128, z, z, z, z) == L.MOE_OK
+    F = lib.moe_expert_ffn_fp8
+    args = [p] * 9                    # x_q .. y_perm; the workspace follows
+    assert F(16, 100, 128, 1, *args, q, 1 << 20, z) == L.MOE_ERR_INVALID_ARG
+    assert F(16, 256, 96, 1, *args, q, 1 << 20, z) == L.MOE_ERR_INVALID_ARG
+    assert F(16, 256, 128, 1, *args, z, 0, z) == L.MOE_ERR_WORKSPACE
+    assert F(16, 256, 128, 1, *args, ctypes.c_void_p(0x100010), 1 << 20, z) == L.MOE_ERR_WORKSPACE
+    assert F(16, 256, 128, 1, z, *([p] * 8), q, 1 << 20, z) == L.MOE_ERR_INVALID_ARG
+    assert F(0, 256, 128, 1, *([z] * 9), z, 0, z) == L.MOE_OK
+    n = lib.moe_expert_ffn_fp8_workspace_size(16, 128)
+    assert n >= 16 * 128 * 3 + 16 * 4 and n % 256 == 0
+    # layer forward: fp8 needs the weight row scales and excludes the packed layout
+    ex8 = L.exec_config(fp8=1)
+    W = L.moe_weights(0x1000, None, 0x1000, 0x1000, 0x1000, 0x1000, 0)
+    assert lib.moe_layer_forward(cb(c), cb(ex8), cb(W), p, p, None, p, 1 << 40, z, z) == L.MOE_ERR_INVALID_ARG
+    Wp = L.moe_weights(0x1000, None, 0x1000, 0x1000, 0x1000, 0x1000, 1, 0x1000, 0x1000, 0x1000, 0x1000)
+    assert lib.moe_layer_forward(cb(c), cb(ex8), cb(Wp), p, p, None, p, 1 << 40, z, z) == L.MOE_ERR_UNSUPPORTED
+    assert lib.moe_layer_forward(cb(c), cb(L.exec_config(fp8=2)), cb(W), p, p, None, p, 1 << 40, z, z) == L.MOE_ERR_INVALID_ARG
+    W8 = L.moe_weights(0x1000, None, 0x1000, 0x1000, 0x1000, 0x1000, 0, 0x1000, 0x1000, 0x1000, 0x1000)
+    assert lib.moe_layer_forward(cb(c), cb(ex8), cb(W8), p, p, None, z, 0, z, z) == L.MOE_ERR_WORKSPACE
+    # the fp8 layout adds the quantized copies; its x_perm is half the bf16 one
+    for wl in (I.DECODE, I.PREFILL):
+        cw = L.config_of(wl)
+        n16 = L.moe_workspace_size(cw, L.exec_config(fuse_gather=0))
+        n8 = L.moe_workspace_size(cw, L.exec_config(fuse_gather=0, fp8=1))
+        tk = wl.T * wl.k
+        assert n8 - n16 >= wl.T * wl.H + tk * wl.I - tk * wl.H - (1 << 16)
+
+
 def test_empty_batch_is_a_no_op(lib):
     c = L.config(**{**GOOD, "T": 0})
     z = ctypes.c_void_p(0)

@@ -341,17 +341,25 @@ def e4m3_round(a) -> np.ndarray:
     return np.where(mag > 0, np.sign(a) * r, 0.0)
 
 
-def e4m3_decode(codes) -> np.ndarray:
-    """Value of e4m3 bytes (fp64): bit 7 sign, bits 6-3 exponent field E, bits
-    2-0 mantissa field M; E = 0 gives the subnormal M / 8 * 2^-6, otherwise
-    (1 + M / 8) * 2^(E - 7); E = 15 with M = 7 is NaN (no infinities)."""
-    c = np.asarray(codes, dtype=np.uint8).astype(np.int64)
+def _e4m3_table() -> np.ndarray:
+    """Value of each of the 256 e4m3 bytes (fp64): bit 7 sign, bits 6-3 exponent
+    field E, bits 2-0 mantissa field M; E = 0 gives the subnormal M / 8 * 2^-6,
+    otherwise (1 + M / 8) * 2^(E - 7); E = 15 with M = 7 is NaN (no infinities)."""
+    c = np.arange(256, dtype=np.int64)
     sign = np.where(c & 0x80, -1.0, 1.0)
     E = (c >> 3) & 0xF
     M = c & 0x7
     mag = np.where(E == 0, M / 8.0 * 2.0 ** -6, (1.0 + M / 8.0) * np.exp2(E - 7.0))
     mag = np.where((E == 15) & (M == 7), np.nan, mag)
     return sign * mag
+
+
+E4M3_VALUES = _e4m3_table()
+
+
+def e4m3_decode(codes) -> np.ndarray:
+    """Values (fp64) of e4m3 bytes: a lookup in the 256-entry table above."""
+    return E4M3_VALUES[np.asarray(codes, dtype=np.uint8)]
 
 
 def quantize_rows_e4m3(a):

@@ -59,6 +59,8 @@ def parse():
     p.add_argument("--precision", choices=("bf16", "fp8"), default="bf16",
                    help="expert GEMM operands: bf16, or e4m3 with per-row scales (weights "
                         "quantized once at load, tokens and h quantized inside each step)")
+    p.add_argument("--fuse-combine", action="store_true",
+                   help="fuse the gate-weighted combine into GEMM2's epilogue (fp32 reductions)")
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--cpu-tokens", type=int, default=128, help="oracle sample size (tokens)")
     return p.parse_args()
@@ -191,13 +193,16 @@ def calibrate(L, wl, d, device):
         d["bias"] = b.to(device)
 
 
-def algorithmic(wl, touched, fused_gather=True, fp8=False):
+def algorithmic(wl, touched, fused_gather=True, fp8=False, fused_combine=False):
     """Algorithmic bytes and flops of each stage for one forward.
 
     GEMM1's token operand is counted as R*H*eb either way (packed rows read, or
     the same rows gathered from x); a fused dispatch has no copy of its own.
     FP8 (eb = 1): the dispatch stage also quantizes x (bf16 read, e4m3 + scales
     written) and the GEMM1 stage also quantizes h (bf16 read, e4m3 + scales).
+    Fused combine: GEMM2 reduces into the fp32 [T, H] accumulator (counted once)
+    instead of writing y_perm; the accumulator is cleared at the start (counted
+    in the router stage) and converted to the bf16 output in the combine stage.
     """
     T, H, E, k, Iw, Is = wl.T, wl.H, wl.E, wl.k, wl.I, wl.I_shared
     R = T * k
@@ -215,6 +220,12 @@ def algorithmic(wl, touched, fused_gather=True, fp8=False):
         "shared_gemm2": (H * Is * eb + T * Is * eb + T * H * 4) if Is else 0,
         "combine": R * H * 4 + (T * H * 4 if Is else 0) + T * H * 2 + R * 8,
     }
+    if fused_combine:
+        b["router"] += T * H * 4
+        b["gemm2"] += T * H * 4 - R * H * 4
+        if Is:  # the shared expert adds into the same accumulator: no y of its own
+            b["shared_gemm2"] -= T * H * 4
+        b["combine"] = T * H * 4 + T * H * 2
     f = {"router": 2 * T * E * H, "gemm1": 2 * R * H * 2 * Iw, "gemm2": 2 * R * Iw * H,
          "shared_gemm1": 2 * T * H * 2 * Is, "shared_gemm2": 2 * T * Is * H}
     if Is and Is == Iw:  # the library runs the shared expert inside the routed GEMM launches
@@ -347,6 +358,8 @@ def config_of(wl, args):
             "weights": "tile-packed at load (moe_pack_weights)" if packs(args, wl) else "row-major",
             "precision": "e4m3 expert GEMMs, per-row fp32 scales (weights quantized at load)"
             if args.precision == "fp8" else "bf16 expert GEMMs",
+            "combine": "fused into GEMM2's epilogue (fp32 reductions)" if args.fuse_combine
+            else "y_perm + combine kernel",
             "global_batch": wl.T * args.gpus,
             "l2": "inputs larger than L2: the expert weights streamed per step exceed 129 MB",
             "parallelism": f"replicas{args.gpus}"}
@@ -367,7 +380,8 @@ def run_ours(args, wl, rank, world, local, device):
     # the library fuses the dispatch only for decode-sized batches (<= 24 rows per expert)
     fused = bool(fuse) and wl.T * wl.k <= 24 * wl.E
     fp8 = 1 if args.precision == "fp8" else 0
-    ex = L.exec_config(fuse_gather=fuse, fp8=fp8, **mode)
+    fc = 1 if args.fuse_combine else 0
+    ex = L.exec_config(fuse_gather=fuse, fp8=fp8, fuse_combine=fc, **mode)
     # one workspace serves the timed mode and the sequential stats / stage-event passes
     ws = torch.empty(max(L.moe_workspace_size(cfg, ex),
                          L.moe_workspace_size(cfg, L.exec_config(fuse_gather=fuse, fp8=fp8)),
@@ -453,7 +467,8 @@ def run_ours(args, wl, rank, world, local, device):
                 e.record(stream)
         torch.cuda.synchronize()
         for i in range(K2):
-            exs = L.exec_config(fuse_gather=fuse_flag, stage_events=evs[i], fp8=fp8)
+            exs = L.exec_config(fuse_gather=fuse_flag, stage_events=evs[i], fp8=fp8,
+                                fuse_combine=fc)
             L.moe_layer_forward(cfg, exs, W, d["x"], out, None, ws, stream)
         torch.cuda.synchronize()
         return {L.STAGES[j]: statistics.mean(evs[i][j - 1].elapsed_time(evs[i][j])
@@ -513,7 +528,7 @@ def run_ours(args, wl, rank, world, local, device):
                    "ms_sequential_unchunked": round(sum(stage_ms.values()), 4)}
 
     hbm, tf_burst, tf_sust, src = peaks()
-    b, f = algorithmic(wl, touched, fused, bool(fp8))
+    b, f = algorithmic(wl, touched, fused, bool(fp8), bool(fc))
     g1 = stage_ms["gemm1"] / 1e3
     achieved = b["gemm1"] / g1 / 1e9
     traffic = None if fp8 else measured_traffic(wl.name)

@@ -97,6 +97,13 @@ typedef struct {
  *    in the epilogue, h (bf16, as in the bf16 form) is quantized per row the
  *    same way, and GEMM2 runs on e4m3 h and W2. The expert weights of
  *    moe_weights must then be e4m3 with their row scales (fp8 fields there).
+ *  fuse_combine 0 = GEMM2 writes y_perm (fp32) and a combine kernel sums each
+ *    token's k rows in slot order (deterministic); 1 = the gate-weighted
+ *    combine is fused into GEMM2's epilogue: every GEMM2 (and the shared
+ *    expert's) adds w * y straight into an fp32 [T,H] accumulator (the output
+ *    itself when out_fp32 = 1) with fp32 atomic reductions, so y_perm is never
+ *    written; the order of the k + 1 additions per element is not fixed, so
+ *    results may differ in the last fp32 bits from run to run.
  */
 typedef struct {
   int32_t overlap, chunk_tokens, chunk_axis, n_expert_chunks, out_fp32, fuse_gather;
@@ -104,7 +111,7 @@ typedef struct {
    * the caller) recorded on `stream` at the stage boundaries of a sequential
    * (overlap = 0) forward; NULL = no tracing. Ignored when overlap = 1. */
   void** stage_events;
-  int32_t fp8;
+  int32_t fp8, fuse_combine;
 } moe_exec;
 
 /* Indices into moe_exec.stage_events: event i is recorded when stage i ends

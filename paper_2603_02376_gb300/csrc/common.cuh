@@ -58,9 +58,12 @@ moe_status launch_gate(const moe_config& c, const float* logits, const float* bi
                        float* w, cudaStream_t s);
 
 int perm_num_chunks(int T);
+// row_w (optional, with topk_w [T*k]): row_w[slot_row[n]] = topk_w[n], the
+// gate weight of every packed row, for a combine fused into GEMM2.
 moe_status launch_permutation(const moe_config& c, const int32_t* idx, int32_t* counts,
                               int32_t* offsets, int32_t* row_src_token, int32_t* slot_row,
-                              int32_t* chunk_counts, int32_t* chunk_base, cudaStream_t s);
+                              int32_t* chunk_counts, int32_t* chunk_base, cudaStream_t s,
+                              const float* topk_w = nullptr, float* row_w = nullptr);
 moe_status launch_dispatch_rows(int T, int H, int k, const uint16_t* x, const int32_t* slot_row,
                                 uint16_t* x_perm, cudaStream_t s);
 moe_status launch_gather_rows(int H, const uint16_t* x, const int32_t* row_src_token,
@@ -100,6 +103,12 @@ struct FfnGroup {
   const float* W2_scale;
   uint8_t* hq;
   float* hs;
+  // Combine fused into GEMM2 (comb_out non-null): instead of y, GEMM2 adds
+  // comb_w[r] * y[r] into comb_out[comb_tok[r]] with fp32 reductions (comb_tok
+  // null = row r is token r; comb_w null = weight 1).
+  float* comb_out;
+  const int32_t* comb_tok;
+  const float* comb_w;
 };
 
 // Routed group plus an optional dense group (the shared expert, same I) in one

@@ -35,6 +35,8 @@
 // copies and MMAs in flight, frees TMEM and returns.
 #include <cudaTypedefs.h>
 
+#include <type_traits>
+
 #include "common.cuh"
 
 #define MOE_STATUS_TRY(expr)          \
@@ -292,6 +294,14 @@ struct GemmArgs {
   const float* b_scale0;
   const float* b_scale1;
   const int32_t* b_scale_idx0;
+  // PLAIN / PLAIN2 only: the combine fused into the epilogue. Non-null comb_out*
+  // replaces the y store of that group by comb_out[tok][f] += w * y (fp32
+  // reductions), tok = comb_tok0[row] and w = comb_w0[row] for group 0 (null:
+  // the row itself, weight 1), the row itself and weight 1 for group 1.
+  float* comb_out0;
+  float* comb_out1;
+  const int32_t* comb_tok0;
+  const float* comb_w0;
   uint64_t wait_limit_ns;  // limit of each barrier wait
   long stall_fill;         // testing: CTA 0 never issues this fill (-1 = none), so the
                            // MMA's wait on it runs out and the abort path is exercised
@@ -351,7 +361,7 @@ __device__ __forceinline__ Unit decode_unit(int u, const int* tile_off, const in
 
 // ------------------------------------------------------------------ kernel
 
-template <int MODE, int NMAX, bool F8>
+template <int MODE, int NMAX, bool F8, bool PK>
 __global__ void __launch_bounds__(NUM_THREADS, 1)
     grouped_gemm_kernel(const __grid_constant__ CUtensorMap tmA0,
                         const __grid_constant__ CUtensorMap tmB0,
@@ -497,7 +507,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
             for (int t = 0; t < TL::NA; ++t) {
               const int r = wrow + t * a.up_off;
               const uint16_t* ap = U.grp ? a.a1_packed : a.a0_packed;
-              if (ap)  // tile (r / 128, kb): 8192 bf16 per tile
+              if (PK)  // tile (r / 128, kb): 8192 bf16 per tile
                 bulk_load_tile(sa + t * TL::A_BYTES,
                                ap + ((size_t)(r / BM) * kblocks + kb) * (BM * BK), full);
               else
@@ -638,47 +648,87 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       };
       void* out = U.grp ? static_cast<void*>(static_cast<float*>(a.out1) + U.split * a.split_stride)
                         : a.out0;
-      for (int c0 = 0; c0 < U.m; c0 += 16) {
-        uint32_t g[16];
-        tmem_ld16(tq + c0, g);
-        if (SWIGLU) {
-          uint32_t v[16];
-          tmem_ld16(tq + NMAX + c0, v);
-          tmem_wait_ld();
+      float* comb = U.grp ? a.comb_out1 : a.comb_out0;
+      const int32_t* ctok = U.grp ? nullptr : a.comb_tok0;
+      const float* cw = U.grp ? nullptr : a.comb_w0;
+      // the destination row of token column c and the weight it is added with
+      auto comb_dst = [&](int c, float* wv) -> float* {
+        const int br = U.row0 + c;
+        *wv = cw ? cw[br] : 1.f;
+        return comb + (size_t)(ctok ? ctok[br] : br) * a.out_ld + f;
+      };
+      // The unit's columns; CB (the fused combine) is a compile-time copy of the
+      // loop so the plain stores keep their unrolled form.
+      auto columns = [&](auto cb_tag) {
+        constexpr bool CB = decltype(cb_tag)::value;
+        for (int c0 = 0; c0 < U.m; c0 += 16) {
+          uint32_t g[16];
+          tmem_ld16(tq + c0, g);
+          if constexpr (SWIGLU) {
+            uint32_t v[16];
+            tmem_ld16(tq + NMAX + c0, v);
+            tmem_wait_ld();
 #pragma unroll
-          for (int i = 0; i < 16; ++i) {
-            if (c0 + i < U.m) {
-              const float sb = col_scale(c0 + i);
-              const float gv = __uint_as_float(g[i]) * (sa0 * sb);
-              const float uv = __uint_as_float(v[i]) * (sa1 * sb);
-              // silu(g) * u with the hardware exp2-based __expf and a reciprocal:
-              // their error (a few fp32 ulp) is far below the bf16 rounding of h
-              const float hv = gv * __frcp_rn(1.0f + __expf(-gv)) * uv;
-              static_cast<uint16_t*>(out)[o + (size_t)(c0 + i) * a.out_ld] = float_to_bf16_bits(hv);
+            for (int i = 0; i < 16; ++i) {
+              if (c0 + i < U.m) {
+                const float sb = col_scale(c0 + i);
+                const float gv = __uint_as_float(g[i]) * (sa0 * sb);
+                const float uv = __uint_as_float(v[i]) * (sa1 * sb);
+                // silu(g) * u with the hardware exp2-based __expf and a reciprocal:
+                // their error (a few fp32 ulp) is far below the bf16 rounding of h
+                const float hv = gv * __frcp_rn(1.0f + __expf(-gv)) * uv;
+                static_cast<uint16_t*>(out)[o + (size_t)(c0 + i) * a.out_ld] =
+                    float_to_bf16_bits(hv);
+              }
             }
-          }
-        } else if (MODE == MODE_PLAIN2) {
-          uint32_t v[16];
-          tmem_ld16(tq + NMAX + c0, v);  // the second tile: features f + 128
-          tmem_wait_ld();
+          } else if constexpr (MODE == MODE_PLAIN2) {
+            uint32_t v[16];
+            tmem_ld16(tq + NMAX + c0, v);  // the second tile: features f + 128
+            tmem_wait_ld();
 #pragma unroll
-          for (int i = 0; i < 16; ++i) {
-            if (c0 + i < U.m) {
-              const float sb = col_scale(c0 + i);
-              float* y = static_cast<float*>(out) + o + (size_t)(c0 + i) * a.out_ld;
-              y[0] = __uint_as_float(g[i]) * (sa0 * sb);
-              y[BM] = __uint_as_float(v[i]) * (sa1 * sb);
+            for (int i = 0; i < 16; ++i) {
+              if (c0 + i < U.m) {
+                const float sb = col_scale(c0 + i);
+                const float y0 = __uint_as_float(g[i]) * (sa0 * sb);
+                const float y1 = __uint_as_float(v[i]) * (sa1 * sb);
+                if constexpr (CB) {
+                  float wv;
+                  float* d = comb_dst(c0 + i, &wv);
+                  atomicAdd(d, wv * y0);
+                  atomicAdd(d + BM, wv * y1);
+                } else {
+                  float* y = static_cast<float*>(out) + o + (size_t)(c0 + i) * a.out_ld;
+                  y[0] = y0;
+                  y[BM] = y1;
+                }
+              }
             }
-          }
-        } else {
-          tmem_wait_ld();
+          } else {
+            tmem_wait_ld();
 #pragma unroll
-          for (int i = 0; i < 16; ++i) {
-            if (c0 + i < U.m)
-              static_cast<float*>(out)[o + (size_t)(c0 + i) * a.out_ld] =
-                  __uint_as_float(g[i]) * (sa0 * col_scale(c0 + i));
+            for (int i = 0; i < 16; ++i) {
+              if (c0 + i < U.m) {
+                const float y0 = __uint_as_float(g[i]) * (sa0 * col_scale(c0 + i));
+                if constexpr (CB) {
+                  float wv;
+                  float* d = comb_dst(c0 + i, &wv);
+                  atomicAdd(d, wv * y0);
+                } else {
+                  static_cast<float*>(out)[o + (size_t)(c0 + i) * a.out_ld] = y0;
+                }
+              }
+            }
           }
         }
+      };
+      if constexpr (MODE == MODE_PLAIN || MODE == MODE_PLAIN2) {
+        if (comb) {
+          columns(std::true_type{});
+        } else {
+          columns(std::false_type{});
+        }
+      } else {
+        columns(std::false_type{});
       }
       tc_fence_before();
       __syncwarp();
@@ -730,30 +780,23 @@ bool make_map(CUtensorMap* m, const void* ptr, uint64_t inner, uint64_t outer, u
 uint64_t g_wait_limit_ns = WAIT_LIMIT_NS;
 long g_stall_fill = -1;
 
-// A weight map for row-major weights; packed weights are read by bulk copies
-// and get a (valid, unused) map over the same bytes.
-bool make_weight_map(CUtensorMap* m, const void* ptr, uint64_t K, uint64_t rows, bool packed) {
-  (void)packed;
-  return make_map(m, ptr, K, rows, BK, BM);
-}
-
 template <int MODE, int NMAX>
 size_t gemm_smem_bytes(int n_exp) {
   using TL = Tile<MODE, NMAX>;
   return 1024 + (size_t)TL::STAGES * TL::STAGE_BYTES + sizeof(Ctrl) + 2 * sizeof(int) * (n_exp + 1);
 }
 
-template <int MODE, int NMAX, bool F8>
+template <int MODE, int NMAX, bool F8, bool PK>
 moe_status launch_gemm(const CUtensorMap& A0, const CUtensorMap& B0, const CUtensorMap& A1,
                        const CUtensorMap& B1, const CUtensorMap& B0big, const CUtensorMap& B1big,
                        const GemmArgs& args, cudaStream_t s) {
   const size_t smem = gemm_smem_bytes<MODE, NMAX>(args.n_exp);
   if (smem > 227 * 1024) return MOE_ERR_UNSUPPORTED;
-  if (cudaFuncSetAttribute(grouped_gemm_kernel<MODE, NMAX, F8>,
+  if (cudaFuncSetAttribute(grouped_gemm_kernel<MODE, NMAX, F8, PK>,
                            cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) != cudaSuccess)
     return MOE_ERR_CUDA;
-  grouped_gemm_kernel<MODE, NMAX, F8><<<num_sms(), NUM_THREADS, smem, s>>>(A0, B0, A1, B1, B0big,
-                                                                           B1big, args);
+  grouped_gemm_kernel<MODE, NMAX, F8, PK><<<num_sms(), NUM_THREADS, smem, s>>>(A0, B0, A1, B1,
+                                                                               B0big, B1big, args);
   note_launch();
   return launch_status();
 }
@@ -775,14 +818,17 @@ bool make_rows_map(CUtensorMap* m, const void* ptr, uint64_t cols, uint64_t rows
             CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
-template <int NMAX, bool F8>
+// PK: weights in the tile-packed layout, fetched by bulk copies (a separate
+// instantiation: a runtime choice between the two weight paths in the
+// producer's loop measured 12 % slower decode GEMM2 even when never taken).
+template <int NMAX, bool F8, bool PK>
 moe_status run_ffn(const FfnGroup& g0, const FfnGroup* g1, int H, int I, cudaStream_t s,
                    cudaEvent_t after_gemm1) {
   CUtensorMap a1, b1, a2, b2, sa1, sb1, sa2, sb2, b1big, b2big, sb1big, sb2big;
   // with a fused dispatch GEMM1 reads token rows of x by index: a one-row box
   const bool gather = g0.gather != nullptr;
-  const bool pk = g0.packed;
-  if (F8 && pk) return MOE_ERR_UNSUPPORTED;  // packed tiles are bf16 only
+  const bool pk = PK;
+  if (g0.packed != PK || (F8 && PK)) return MOE_ERR_UNSUPPORTED;  // packed tiles are bf16 only
   const uint64_t xr = gather ? g0.x_rows : g0.rows;
   // GEMM2's token operand: h (bf16), or its e4m3 copy hq in the FP8 form
   const void* h0 = F8 ? static_cast<const void*>(g0.hq) : static_cast<const void*>(g0.h);
@@ -839,7 +885,8 @@ moe_status run_ffn(const FfnGroup& g0, const FfnGroup* g1, int H, int I, cudaStr
     args.b_scale1 = g1 ? g1->x_scale : nullptr;
     args.b_scale_idx0 = g0.x_scale_idx;
   }
-  moe_status st = launch_gemm<MODE_SWIGLU, NMAX, F8>(a1, b1, sa1, sb1, b1big, sb1big, args, s);
+  moe_status st =
+      launch_gemm<MODE_SWIGLU, NMAX, F8, PK>(a1, b1, sa1, sb1, b1big, sb1big, args, s);
   if (st != MOE_OK) return st;
   if (F8) {  // h of every packed row -> e4m3 and its row scale: GEMM2's operand
     MOE_STATUS_TRY(launch_quantize_rows(g0.h, g0.rows, I, g0.hq, g0.hs, s));
@@ -856,6 +903,11 @@ moe_status run_ffn(const FfnGroup& g0, const FfnGroup* g1, int H, int I, cudaStr
     args.b_scale1 = g1 ? g1->hs : nullptr;
     args.b_scale_idx0 = nullptr;
   }
+  args.comb_out0 = g0.comb_out;
+  args.comb_tok0 = g0.comb_tok;
+  args.comb_w0 = g0.comb_w;
+  args.comb_out1 = g1 ? g1->comb_out : nullptr;
+  if (g1 && (g1->comb_tok || g1->comb_w)) return MOE_ERR_INVALID_ARG;  // group 1 is dense
   // GEMM2: y = h W2^T (fp32). With prefill-sized token tiles, two 128-feature
   // weight tiles per unit share one token tile (more weight bytes per stage);
   // with decode-sized tiles a single weight tile and a deeper ring measured faster.
@@ -867,11 +919,11 @@ moe_status run_ffn(const FfnGroup& g0, const FfnGroup* g1, int H, int I, cudaStr
   if (NMAX > 32 && H % (2 * BM) == 0) {
     args.n_fb = H / (2 * BM);
     args.up_off = BM;
-    return launch_gemm<MODE_PLAIN2, NMAX, F8>(a2, b2, sa2, sb2, b2big, sb2big, args, s);
+    return launch_gemm<MODE_PLAIN2, NMAX, F8, PK>(a2, b2, sa2, sb2, b2big, sb2big, args, s);
   }
   args.n_fb = H / BM;
   args.up_off = 0;
-  return launch_gemm<MODE_PLAIN, NMAX, F8>(a2, b2, sa2, sb2, b2big, sb2big, args, s);
+  return launch_gemm<MODE_PLAIN, NMAX, F8, PK>(a2, b2, sa2, sb2, b2big, sb2big, args, s);
 }
 
 }  // namespace
@@ -887,13 +939,18 @@ moe_status launch_expert_ffn_groups(const FfnGroup& routed, const FfnGroup* dens
   // prefill ~128 +- 10 % -> 144; larger or skewed loads -> 256).
   const long per = (long)rows_hint / (n_exp > 0 ? n_exp : 1);
   if (routed.fp8) {
-    if (per <= 24) return run_ffn<32, true>(routed, g1, H, I, s, after_gemm1);
-    if (per <= 132) return run_ffn<144, true>(routed, g1, H, I, s, after_gemm1);
-    return run_ffn<256, true>(routed, g1, H, I, s, after_gemm1);
+    if (per <= 24) return run_ffn<32, true, false>(routed, g1, H, I, s, after_gemm1);
+    if (per <= 132) return run_ffn<144, true, false>(routed, g1, H, I, s, after_gemm1);
+    return run_ffn<256, true, false>(routed, g1, H, I, s, after_gemm1);
   }
-  if (per <= 24) return run_ffn<32, false>(routed, g1, H, I, s, after_gemm1);
-  if (per <= 132) return run_ffn<144, false>(routed, g1, H, I, s, after_gemm1);
-  return run_ffn<256, false>(routed, g1, H, I, s, after_gemm1);
+  if (routed.packed) {
+    if (per <= 24) return run_ffn<32, false, true>(routed, g1, H, I, s, after_gemm1);
+    if (per <= 132) return run_ffn<144, false, true>(routed, g1, H, I, s, after_gemm1);
+    return run_ffn<256, false, true>(routed, g1, H, I, s, after_gemm1);
+  }
+  if (per <= 24) return run_ffn<32, false, false>(routed, g1, H, I, s, after_gemm1);
+  if (per <= 132) return run_ffn<144, false, false>(routed, g1, H, I, s, after_gemm1);
+  return run_ffn<256, false, false>(routed, g1, H, I, s, after_gemm1);
 }
 
 int router_tc_splits(int T, int H, int E) {
@@ -923,7 +980,7 @@ moe_status launch_router_tc(int T, int H, int E, const uint16_t* x, const uint16
   args.out1 = partials;
   args.out_ld = E;
   args.err = device_error_word();
-  return launch_gemm<MODE_SPLIT3, 128, false>(A, B, A, B, Bbig, Bbig, args, s);
+  return launch_gemm<MODE_SPLIT3, 128, false, false>(A, B, A, B, Bbig, Bbig, args, s);
 }
 
 moe_status launch_expert_ffn_stalled(int rows, int H, int I, int n_experts, const uint16_t* x_perm,

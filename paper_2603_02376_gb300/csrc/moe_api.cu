@@ -86,6 +86,7 @@ bool valid_exec(const moe_exec* ex, const moe_config* c) {
   if (ex->out_fp32 != 0 && ex->out_fp32 != 1) return false;
   if (ex->fuse_gather != 0 && ex->fuse_gather != 1) return false;
   if (ex->fp8 != 0 && ex->fp8 != 1) return false;
+  if (ex->fuse_combine != 0 && ex->fuse_combine != 1) return false;
   if (ex->overlap) {
     if (ex->chunk_axis == 0) {
       if (ex->chunk_tokens < 1) return false;
@@ -137,7 +138,13 @@ struct Layout {
   uint16_t* sh_h;    // [T, I_s]
   uint8_t* sh_hq;    // [T, I_s] (fp8 only)
   float* sh_hs;      // [T]
-  float* sh_y;       // [T, H] fp32
+  float* sh_y;       // [T, H] fp32 (unfused combine)
+  // Combine fused into GEMM2: the gate weight of every packed row, and the fp32
+  // [T, H] accumulator the GEMM2s reduce into (the caller's output when it is
+  // fp32, else carved here and converted to bf16 at the end).
+  bool fuse_combine = false;
+  float* row_w;      // [T*k]
+  float* acc;        // [T, H] or null (= the fp32 output)
   size_t bytes = 0;
 };
 
@@ -177,12 +184,15 @@ Layout carve(const moe_config& c, const moe_exec& ex, void* ws) {
   L.h = cv.take<uint16_t>(T * k * c.I);
   L.hq = L.fp8 ? cv.take<uint8_t>(T * k * c.I) : nullptr;
   L.hs = L.fp8 ? cv.take<float>(T * k) : nullptr;
-  L.y_perm = cv.take<float>(T * k * c.H);
+  L.fuse_combine = ex.fuse_combine != 0;
+  L.row_w = L.fuse_combine ? cv.take<float>(T * k) : nullptr;
+  L.y_perm = L.fuse_combine ? nullptr : cv.take<float>(T * k * c.H);
+  L.acc = (L.fuse_combine && !ex.out_fp32) ? cv.take<float>(T * c.H) : nullptr;
   L.sh_off = cv.take<int32_t>(2);
   L.sh_h = c.I_shared ? cv.take<uint16_t>(T * c.I_shared) : nullptr;
   L.sh_hq = (c.I_shared && L.fp8) ? cv.take<uint8_t>(T * c.I_shared) : nullptr;
   L.sh_hs = (c.I_shared && L.fp8) ? cv.take<float>(T) : nullptr;
-  L.sh_y = c.I_shared ? cv.take<float>(T * c.H) : nullptr;
+  L.sh_y = (c.I_shared && !L.fuse_combine) ? cv.take<float>(T * c.H) : nullptr;
   L.bytes = align_up(cv.off, 256);
   return L;
 }
@@ -250,7 +260,8 @@ moe_status pack_tokens(const moe_config& c, const Layout& L, const moe_weights& 
   MOE_TRY(mark(ev, MOE_EV_GATE, s));
   MOE_TRY(launch_permutation(cc, L.idx + tk, L.counts + (size_t)ci * c.E,
                              L.offsets + (size_t)ci * (c.E + 1), L.rst + tk, L.slot_row + tk,
-                             L.perm_counts, L.perm_base, s));
+                             L.perm_counts, L.perm_base, s, L.w + tk,
+                             L.row_w ? L.row_w + tk : nullptr));
   MOE_TRY(mark(ev, MOE_EV_PERMUTE, s));
   if (L.fp8) {
     // quantize, then dispatch the e4m3 rows: a row of H bytes is copied as
@@ -285,7 +296,13 @@ FfnGroup routed_group(const moe_config& c, const Layout& L, const moe_weights& w
   g.W2 = w.W2;
   g.packed = w.packed != 0;
   g.h = L.h + tk * c.I;
-  g.y = L.y_perm + tk * c.H;
+  if (L.fuse_combine) {  // GEMM2 adds w * y into the token rows of the accumulator
+    g.comb_out = L.acc + (size_t)t0 * c.H;
+    g.comb_tok = L.rst + tk;
+    g.comb_w = L.row_w + tk;
+  } else {
+    g.y = L.y_perm + tk * c.H;
+  }
   const size_t xb = L.fp8 ? 1 : 2;
   if (L.x_perm) {
     g.x = static_cast<const uint8_t*>(L.x_perm) + tk * c.H * xb;
@@ -319,6 +336,7 @@ FfnGroup dense_group(const moe_config& c, const Layout& L, const moe_weights& w,
   g.W2 = w.Ws2;
   g.h = L.sh_h;
   g.y = L.sh_y;
+  g.comb_out = L.fuse_combine ? L.acc : nullptr;  // token rows, weight 1
   g.packed = w.packed != 0;
   g.x = x;
   if (L.fp8) {
@@ -369,6 +387,22 @@ moe_status experts_and_shared(const moe_config& c, const Layout& L, const moe_we
   MOE_TRY(mark(ev, MOE_EV_GEMM2, s));
   MOE_TRY(mark(ev, MOE_EV_SHARED_GEMM1, s));
   return mark(ev, MOE_EV_SHARED_GEMM2, s);
+}
+
+// Fused combine: the accumulator starts at zero before any GEMM2 adds into it.
+moe_status clear_acc(const moe_config& c, const Layout& L, cudaStream_t s) {
+  if (!L.fuse_combine) return MOE_OK;
+  return cudaMemsetAsync(L.acc, 0, (size_t)c.T * c.H * sizeof(float), s) == cudaSuccess
+             ? MOE_OK
+             : MOE_ERR_CUDA;
+}
+
+// Fused combine, bf16 output: out = bf16(acc) (the combine kernel with no
+// routed term and acc as its dense term); with an fp32 output acc is out.
+moe_status finish_acc(const moe_config& c, const Layout& L, void* out, int out_fp32,
+                      cudaStream_t s) {
+  if (out_fp32) return MOE_OK;
+  return launch_combine(c.T, c.H, 0, nullptr, nullptr, nullptr, L.acc, out, 0, s);
 }
 
 moe_status combine_tokens(const moe_config& c, const Layout& L, int t0, int Tc, void* out,
@@ -612,6 +646,7 @@ moe_status moe_layer_forward(const moe_config* cfg, const moe_exec* ex, const mo
   Layout L = carve(c, *ex, nullptr);
   if (!ws || ws_bytes < L.bytes || ((uintptr_t)ws & 255)) return MOE_ERR_WORKSPACE;
   L = carve(c, *ex, ws);
+  if (L.fuse_combine && ex->out_fp32) L.acc = static_cast<float*>(out);
   if (aux && aux->logits) L.logits = aux->logits;
   if (aux && aux->topk_idx) L.idx = aux->topk_idx;
   if (aux && aux->topk_w) L.w = aux->topk_w;
@@ -622,6 +657,7 @@ moe_status moe_layer_forward(const moe_config* cfg, const moe_exec* ex, const mo
   if (!ex->overlap) {
     cudaEvent_t* ev = reinterpret_cast<cudaEvent_t*>(ex->stage_events);
     MOE_TRY(mark(ev, MOE_EV_START, s));
+    MOE_TRY(clear_acc(c, L, s));
     MOE_TRY(pack_tokens(c, L, *w, x, 0, c.T, 0, L.x_perm != nullptr, s, ev, true));
     if (c.I_shared == c.I) {
       MOE_TRY(experts_and_shared(c, L, *w, x, s, ev));
@@ -629,7 +665,10 @@ moe_status moe_layer_forward(const moe_config* cfg, const moe_exec* ex, const mo
       MOE_TRY(experts_tokens(c, L, *w, x, 0, c.T, 0, 0, c.E, s, ev));
       MOE_TRY(shared_expert(c, L, *w, x, s, ev));
     }
-    MOE_TRY(combine_tokens(c, L, 0, c.T, out, ex->out_fp32, s));
+    if (L.fuse_combine)
+      MOE_TRY(finish_acc(c, L, out, ex->out_fp32, s));
+    else
+      MOE_TRY(combine_tokens(c, L, 0, c.T, out, ex->out_fp32, s));
     MOE_TRY(mark(ev, MOE_EV_COMBINE, s));
     if (aux && aux->counts)
       MOE_CUDA(cudaMemcpyAsync(aux->counts, L.counts, sizeof(int32_t) * c.E,
@@ -643,6 +682,7 @@ moe_status moe_layer_forward(const moe_config* cfg, const moe_exec* ex, const mo
   std::vector<cudaEvent_t> ev;
   if (!events(dev, (size_t)n_stage + 1, &ev)) return MOE_ERR_CUDA;
   if (L.fp8) MOE_TRY(quantize_tokens(c, L, x, 0, c.T, s));  // before the fork: both streams read x_q
+  MOE_TRY(clear_acc(c, L, s));
   // the pack stream starts after everything already queued on `stream`
   MOE_CUDA(cudaEventRecord(ev[n_stage], s));
   MOE_CUDA(cudaStreamWaitEvent(ps, ev[n_stage], 0));
@@ -660,8 +700,9 @@ moe_status moe_layer_forward(const moe_config* cfg, const moe_exec* ex, const mo
       const int t0 = ci * L.chunk_T, Tc = c.T - t0 < L.chunk_T ? c.T - t0 : L.chunk_T;
       MOE_CUDA(cudaStreamWaitEvent(s, ev[ci], 0));
       MOE_TRY(experts_tokens(c, L, *w, x, t0, Tc, ci, 0, c.E, s));
-      MOE_TRY(combine_tokens(c, L, t0, Tc, out, ex->out_fp32, s));
+      if (!L.fuse_combine) MOE_TRY(combine_tokens(c, L, t0, Tc, out, ex->out_fp32, s));
     }
+    if (L.fuse_combine) MOE_TRY(finish_acc(c, L, out, ex->out_fp32, s));
     if (aux && aux->counts) MOE_TRY(launch_sum_counts(L.counts, L.n_chunks, c.E, aux->counts, s));
     return MOE_OK;
   }
@@ -687,7 +728,10 @@ moe_status moe_layer_forward(const moe_config* cfg, const moe_exec* ex, const mo
     MOE_CUDA(cudaStreamWaitEvent(s, ev[r], 0));
     MOE_TRY(experts_tokens(c, L, *w, x, 0, c.T, 0, e0, e1, s));
   }
-  MOE_TRY(combine_tokens(c, L, 0, c.T, out, ex->out_fp32, s));
+  if (L.fuse_combine)
+    MOE_TRY(finish_acc(c, L, out, ex->out_fp32, s));
+  else
+    MOE_TRY(combine_tokens(c, L, 0, c.T, out, ex->out_fp32, s));
   if (aux && aux->counts)
     MOE_CUDA(cudaMemcpyAsync(aux->counts, L.counts, sizeof(int32_t) * c.E,
                              cudaMemcpyDeviceToDevice, s));

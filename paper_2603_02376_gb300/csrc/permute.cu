@@ -145,7 +145,8 @@ __global__ void __launch_bounds__(1024) perm_scan_kernel(const int32_t* __restri
 __global__ void __launch_bounds__(PERM_WARPS * 32) perm_scatter_kernel(
     const int32_t* __restrict__ idx, int T, int k, int E, const int32_t* __restrict__ offsets,
     const int32_t* __restrict__ chunk_base, int32_t* __restrict__ row_src_token,
-    int32_t* __restrict__ slot_row, int* __restrict__ err) {
+    int32_t* __restrict__ slot_row, const float* __restrict__ topk_w, float* __restrict__ row_w,
+    int* __restrict__ err) {
   extern __shared__ int perm_smem[];  // [PERM_WARPS][E]: histogram, then cursors
   for (int i = threadIdx.x; i < PERM_WARPS * E; i += blockDim.x) perm_smem[i] = 0;
   __syncthreads();
@@ -177,6 +178,7 @@ __global__ void __launch_bounds__(PERM_WARPS * 32) perm_scatter_kernel(
     if (e >= 0) {
       row_src_token[row] = (int32_t)(n / k);
       slot_row[n] = row;
+      if (row_w) row_w[row] = topk_w[n];  // the gate weight in packed-row order
     }
   }
 }
@@ -206,7 +208,8 @@ __global__ void pack_weights_kernel(const uint4* __restrict__ W, uint4* __restri
 __global__ void __launch_bounds__(PERM_WARPS * 32) perm_single_kernel(
     const int32_t* __restrict__ idx, int T, int k, int E, int32_t* __restrict__ counts,
     int32_t* __restrict__ offsets, int32_t* __restrict__ row_src_token,
-    int32_t* __restrict__ slot_row, int* __restrict__ err) {
+    int32_t* __restrict__ slot_row, const float* __restrict__ topk_w, float* __restrict__ row_w,
+    int* __restrict__ err) {
   extern __shared__ int perm_smem[];  // [PERM_WARPS][E] histograms, then [E] totals
   int* tot = perm_smem + PERM_WARPS * E;
   for (int i = threadIdx.x; i < PERM_WARPS * E; i += blockDim.x) perm_smem[i] = 0;
@@ -266,6 +269,7 @@ __global__ void __launch_bounds__(PERM_WARPS * 32) perm_single_kernel(
     if (e >= 0) {
       row_src_token[row] = (int32_t)(n / k);
       slot_row[n] = row;
+      if (row_w) row_w[row] = topk_w[n];  // the gate weight in packed-row order
     }
   }
 }
@@ -379,7 +383,8 @@ int perm_num_chunks(int T) { return (T + PERM_TOK - 1) / PERM_TOK; }
 
 moe_status launch_permutation(const moe_config& c, const int32_t* idx, int32_t* counts,
                               int32_t* offsets, int32_t* row_src_token, int32_t* slot_row,
-                              int32_t* chunk_counts, int32_t* chunk_base, cudaStream_t s) {
+                              int32_t* chunk_counts, int32_t* chunk_base, cudaStream_t s,
+                              const float* topk_w, float* row_w) {
   const int nch = perm_num_chunks(c.T);
   if (nch == 1) {
     const size_t smem1 = (size_t)(PERM_WARPS + 1) * c.E * sizeof(int);
@@ -387,8 +392,8 @@ moe_status launch_permutation(const moe_config& c, const int32_t* idx, int32_t* 
       cudaFuncSetAttribute(perm_single_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                            (int)smem1);
     perm_single_kernel<<<1, PERM_WARPS * 32, smem1, s>>>(idx, c.T, c.k, c.E, counts, offsets,
-                                                         row_src_token, slot_row,
-                                                         device_error_word());
+                                                         row_src_token, slot_row, topk_w,
+                                                         row_w, device_error_word());
     note_launch();
     return launch_status();
   }
@@ -407,8 +412,8 @@ moe_status launch_permutation(const moe_config& c, const int32_t* idx, int32_t* 
   note_launch();
   if (nch > 0) {
     perm_scatter_kernel<<<nch, PERM_WARPS * 32, smem, s>>>(idx, c.T, c.k, c.E, offsets, chunk_base,
-                                                           row_src_token, slot_row,
-                                                           device_error_word());
+                                                           row_src_token, slot_row, topk_w,
+                                                           row_w, device_error_word());
     note_launch();
   }
   return launch_status();

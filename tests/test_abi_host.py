@@ -122,6 +122,22 @@ def test_entry_points_reject_bad_arguments_without_a_gpu(lib):
     assert lib.moe_layer_forward(cb(c), cb(ex), cb(Wn), p, p, None, p, 1 << 40, z, z) == L.MOE_ERR_INVALID_ARG
     exb = L.exec_config(overlap=3)
     assert lib.moe_layer_forward(cb(c), cb(exb), cb(W), p, p, None, p, 1 << 40, z, z) == L.MOE_ERR_INVALID_ARG
+    exc = L.exec_config(fuse_combine=2)
+    assert lib.moe_layer_forward(cb(c), cb(exc), cb(W), p, p, None, p, 1 << 40, z, z) == L.MOE_ERR_INVALID_ARG
+    assert L.moe_workspace_size(c, exc) == 0
+
+
+def test_fused_combine_workspace():
+    # fused combine: no y_perm [T*k, H] and no shared y; an fp32 [T, H] accumulator
+    # only when the output is bf16 (an fp32 output is the accumulator itself)
+    for wl in (I.DECODE, I.PREFILL):
+        c = L.config_of(wl)
+        plain = L.moe_workspace_size(c, L.exec_config(fuse_gather=0))
+        f16 = L.moe_workspace_size(c, L.exec_config(fuse_gather=0, fuse_combine=1))
+        f32 = L.moe_workspace_size(c, L.exec_config(fuse_gather=0, fuse_combine=1, out_fp32=1))
+        T, H, k = wl.T, wl.H, wl.k
+        assert plain - f32 >= T * k * H * 4 + T * H * 4 - T * k * 4 - 4096
+        assert f16 - f32 >= T * H * 4
 
 
 def test_fp8_entry_points_reject_bad_arguments_without_a_gpu(lib):

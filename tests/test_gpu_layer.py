@@ -122,12 +122,13 @@ def oracle_tokens(wl, d, toks):
 
 # ---------------------------------------------------------------- tiny: every token
 
+@pytest.mark.parametrize("fuse_combine", [0, 1])
 @pytest.mark.parametrize("out_fp32", [1, 0])
-def test_layer_tiny_full(out_fp32):
+def test_layer_tiny_full(out_fp32, fuse_combine):
     wl = I.TINY
     d = I.layer_inputs(wl, seed=0, device=DEV)
     st = prepare_routing(wl, d)
-    out, a = run_layer(wl, d, L.exec_config(out_fp32=out_fp32))
+    out, a = run_layer(wl, d, L.exec_config(out_fp32=out_fp32, fuse_combine=fuse_combine))
     gidx = check_routing(wl, d, a, st["oracle_logits"])
     check_permutation(wl, d, gidx)
     ref, _ = O.layer_forward(f64(d["x"]), f64(d["Wr"]), None, f64(d["W13"]), f64(d["W2"]),
@@ -157,7 +158,14 @@ def test_layer_small_grouped_full(I_shared, T):
                L.exec_config(out_fp32=1, overlap=1, chunk_axis=0, chunk_tokens=37, fuse_gather=0),
                L.exec_config(out_fp32=1, overlap=1, chunk_axis=1, n_expert_chunks=3),
                L.exec_config(out_fp32=1, overlap=1, chunk_axis=1, n_expert_chunks=3,
-                             fuse_gather=0)):
+                             fuse_gather=0),
+               # the combine fused into GEMM2's epilogue (fp32 reductions)
+               L.exec_config(out_fp32=1, fuse_combine=1),
+               L.exec_config(out_fp32=0, fuse_combine=1, fuse_gather=0),
+               L.exec_config(out_fp32=0, overlap=1, chunk_axis=0, chunk_tokens=37,
+                             fuse_combine=1),
+               L.exec_config(out_fp32=1, overlap=1, chunk_axis=1, n_expert_chunks=3,
+                             fuse_combine=1)):
         out, a = run_layer(wl, d, ex)
         gidx = check_routing(wl, d, a, st["oracle_logits"])
         ref, _ = O.layer_forward(f64(d["x"]), f64(d["Wr"]), bias32(d["bias"]), f64(d["W13"]),
@@ -170,7 +178,8 @@ def test_layer_small_grouped_full(I_shared, T):
 
 @pytest.mark.parametrize("ex", [dict(out_fp32=1), dict(out_fp32=0), dict(out_fp32=1, fuse_gather=0),
                                 dict(out_fp32=1, overlap=1, chunk_axis=1, n_expert_chunks=4),
-                                dict(out_fp32=1, packed=1)])
+                                dict(out_fp32=1, packed=1), dict(out_fp32=0, fuse_combine=1),
+                                dict(out_fp32=1, fuse_combine=1, fuse_gather=0)])
 def test_layer_decode_full(big_weights, ex):
     wl = I.DECODE
     ex = dict(ex)
@@ -207,6 +216,8 @@ def prefill_inputs(big_weights):
     dict(out_fp32=1, fuse_gather=0),
     dict(out_fp32=1, overlap=1, chunk_axis=0, chunk_tokens=512),
     dict(out_fp32=1, overlap=1, chunk_axis=1, n_expert_chunks=8),
+    dict(out_fp32=1, fuse_combine=1),
+    dict(out_fp32=0, overlap=1, chunk_axis=0, chunk_tokens=512, fuse_combine=1),
 ])
 def test_layer_prefill_sampled(prefill_inputs, ex):
     wl = I.PREFILL
@@ -227,7 +238,8 @@ def test_layer_skewed_sampled(big_weights):
     toks = I.sample_tokens(wl.T, 256, 0).numpy()
     ref, _ = oracle_tokens(wl, d, toks)
     for ex in (L.exec_config(out_fp32=1), L.exec_config(out_fp32=1, fuse_gather=0),
-               L.exec_config(out_fp32=1, overlap=1, chunk_axis=1)):
+               L.exec_config(out_fp32=1, overlap=1, chunk_axis=1),
+               L.exec_config(out_fp32=1, fuse_combine=1)):
         out, a = run_layer(wl, d, ex)
         gidx = check_routing(wl, d, a, st["oracle_logits"])
         assert_layer_close(f64(out[torch.as_tensor(toks, device=DEV)]), ref)

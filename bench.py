@@ -243,14 +243,21 @@ def source_sha():
     return h.hexdigest()[:16]
 
 
-def measured_traffic(workload):
-    """ncu DRAM bytes per GEMM1 launch, if captured for the current kernel source."""
+def measured_traffic(workload, fp8=False, kernel_bytes=None):
+    """ncu DRAM bytes per GEMM1 launch, if captured for the current kernel source.
+
+    The bf16 entry holds the bytes of the full launch; the FP8 entry holds the
+    measured traffic / algorithmic ratio, applied to this run's GEMM1 kernel bytes.
+    """
     try:
         with open(TRAFFIC_FILE) as f:
             t = json.load(f)
-        e = t.get(workload)
+        e = t.get(workload + (" fp8" if fp8 else ""))
         if e and e.get("source_sha") == source_sha():
-            return float(e["dram_bytes_per_launch"])
+            if "dram_bytes_per_launch" in e:
+                return float(e["dram_bytes_per_launch"])
+            if kernel_bytes is not None:
+                return float(e["traffic_over_algorithmic"]) * kernel_bytes
     except Exception:
         pass
     return None
@@ -531,7 +538,10 @@ def run_ours(args, wl, rank, world, local, device):
     b, f = algorithmic(wl, touched, fused, bool(fp8), bool(fc))
     g1 = stage_ms["gemm1"] / 1e3
     achieved = b["gemm1"] / g1 / 1e9
-    traffic = None if fp8 else measured_traffic(wl.name)
+    # GEMM1's own bytes (the FP8 GEMM1 stage also holds the h quantization)
+    qh = (wl.T * wl.k * wl.I * 3 + wl.T * wl.k * 4
+          + (wl.T * wl.I_shared * 3 + wl.T * 4 if wl.I_shared == wl.I else 0)) if fp8 else 0
+    traffic = measured_traffic(wl.name, bool(fp8), b["gemm1"] - qh)
     stages = {}
     for s_, t in stage_ms.items():
         e = {"ms": round(t, 4)}

@@ -435,6 +435,30 @@ def layer_forward(x, Wr, bias, W13, W2, cfg: LayerConfig, Ws13=None, Ws2=None, l
     return out, aux
 
 
+def rms_normalize(y, eps: float = 1e-6) -> np.ndarray:
+    """Per-row RMS normalization y / sqrt(mean(y^2) + eps) (fp64), the unit-gain
+    form of the RMSNorm a DeepSeek-V3 block applies in front of its MoE."""
+    y = np.asarray(y, dtype=np.float64)
+    return y / np.sqrt(np.mean(y * y, axis=1, keepdims=True) + eps)
+
+
+def stack_forward(x, layers, cfg: LayerConfig, norm: bool = True):
+    """Consecutive layers (the paper's multi-layer study, Section 4.3): layer l + 1
+    reads layer l's output rounded to bf16 (then, with norm, RMS-normalized and
+    rounded to bf16 again); returns the last layer's fp64 output.
+    layers: a list of dicts with Wr, bias, W13, W2, Ws13, Ws2."""
+    h = np.asarray(x, dtype=np.float64)
+    out = None
+    for n, w in enumerate(layers):
+        if n > 0:
+            h = bf16_round(out)
+            if norm:
+                h = bf16_round(rms_normalize(h))
+        out, _ = layer_forward(h, w["Wr"], w["bias"], w["W13"], w["W2"], cfg, w.get("Ws13"),
+                               w.get("Ws2"))
+    return out
+
+
 def layer_forward_tokens(x_rows, Wr, bias, get_expert, cfg: LayerConfig, get_shared=None,
                          ffn=swiglu_ffn):
     """Layer output for a sample of tokens, one token at a time.

@@ -489,3 +489,35 @@ def test_e4m3_decode_every_code():
     finite = v[~np.isnan(v)]
     np.testing.assert_array_equal(O.e4m3_round(finite), finite)   # the grid rounds to itself
     assert len(np.unique(finite)) == 253                           # 254 finite codes, +-0 equal
+
+
+def test_rms_normalize_by_hand_and_invariants():
+    y = np.array([[3.0, 4.0], [0.0, 0.0], [1e3, -1e3]])
+    r = O.rms_normalize(y, eps=0.0 + 1e-30)
+    np.testing.assert_allclose(r[0], [3 / math.sqrt(12.5), 4 / math.sqrt(12.5)], rtol=1e-15)
+    np.testing.assert_array_equal(O.rms_normalize(y[1:2]), [[0.0, 0.0]])
+    np.testing.assert_allclose(r[2], [1.0, -1.0], rtol=1e-15)
+    rng = np.random.default_rng(3)
+    z = rng.standard_normal((7, 64)) * 5
+    n = O.rms_normalize(z, eps=0.0)
+    np.testing.assert_allclose(np.mean(n * n, axis=1), 1.0, rtol=1e-13)
+    np.testing.assert_allclose(O.rms_normalize(3.5 * z, eps=0.0), n, rtol=1e-13)
+
+
+def test_stack_forward_chains_layers():
+    # one layer = layer_forward; two layers = layer_forward on the bf16 (normalized) output
+    rng = np.random.default_rng(8)
+    cfg = O.LayerConfig(T=5, H=32, E=4, k=2, I=16, gate=O.GATE_SOFTMAX)
+    x = O.bf16_round(rng.standard_normal((5, 32)))
+    mk = lambda: dict(Wr=rng.standard_normal((4, 32)).astype(np.float32) * 0.1, bias=None,
+                      W13=O.bf16_round(rng.standard_normal((4, 32, 32)) * 0.1),
+                      W2=O.bf16_round(rng.standard_normal((4, 32, 16)) * 0.1))
+    l0, l1 = mk(), mk()
+    y0, _ = O.layer_forward(x, l0["Wr"], None, l0["W13"], l0["W2"], cfg)
+    np.testing.assert_array_equal(O.stack_forward(x, [l0], cfg), y0)
+    for norm in (False, True):
+        h = O.bf16_round(y0)
+        if norm:
+            h = O.bf16_round(h / np.sqrt(np.mean(h * h, axis=1, keepdims=True) + 1e-6))
+        y1, _ = O.layer_forward(h, l1["Wr"], None, l1["W13"], l1["W2"], cfg)
+        np.testing.assert_array_equal(O.stack_forward(x, [l0, l1], cfg, norm=norm), y1)

@@ -61,6 +61,9 @@ def parse():
                         "quantized once at load, tokens and h quantized inside each step)")
     p.add_argument("--fuse-combine", action="store_true",
                    help="fuse the gate-weighted combine into GEMM2's epilogue (fp32 reductions)")
+    p.add_argument("--layers", type=int, default=1,
+                   help="time a stack of this many consecutive layers replayed as one CUDA "
+                        "graph (each layer its own router; expert weights shared)")
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--cpu-tokens", type=int, default=128, help="oracle sample size (tokens)")
     return p.parse_args()
@@ -425,6 +428,9 @@ def run_ours(args, wl, rank, world, local, device):
         W = L.weights_struct(d["Wr"], d["bias"], run_w["W13"], run_w["W2"], run_w["Ws13"],
                              run_w["Ws2"], 1 if packed else 0)
 
+    if args.layers > 1:
+        return run_stack(args, wl, rank, world, local, device, L, cfg, ex, W, d)
+
     def step():
         L.moe_layer_forward(cfg, ex, W, d["x"], out, None, ws, stream)
 
@@ -588,6 +594,66 @@ def run_ours(args, wl, rank, world, local, device):
         line["dispatch_fusion"] = dispatch_fusion
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         line["cpu_baseline"] = cpu_baseline(wl, d, args.cpu_tokens)
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+
+
+def run_stack(args, wl, rank, world, local, device, L, cfg, ex, W, d):
+    """The paper's multi-layer study: L consecutive layers (layer l + 1 reads layer l's
+    bf16 output) captured once into a CUDA graph; each step is one graph launch.
+
+    Layer l has its own router weights (seeded by l); the expert weights are shared by
+    all layers (a distinct copy per layer would not fit 16 layers in HBM, and each
+    layer still streams its 22.5 GB of expert weights from HBM: L2 is 129 MB).
+    """
+    nl = args.layers
+    layers = [W]
+    keep = []
+    for l in range(1, nl):
+        Wr = I.randn((wl.E, wl.H), 0.01, torch.float32, l, "Wr", device)
+        keep.append(Wr)
+        wl_ = L.moe_weights.from_buffer_copy(W)
+        wl_.Wr = Wr.data_ptr()
+        layers.append(wl_)
+    ws = torch.empty(L.moe_stack_workspace_size(cfg, ex), dtype=torch.uint8, device=device)
+    x = d["x"].clone()
+    out = torch.empty_like(x)
+    stream = torch.cuda.current_stream()
+    g = L.Graph(cfg, ex, layers, x, out, ws)
+    for _ in range(args.warmup):
+        g.launch(stream)
+    torch.cuda.synchronize()
+    L.moe_check_errors(stream)
+    sampler = ClockSampler(local)
+    time.sleep(0.3)
+    barrier(world)
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    w0 = _dt.datetime.now()
+    e0.record(stream)
+    for _ in range(args.steps):
+        g.launch(stream)
+    e1.record(stream)
+    torch.cuda.synchronize()
+    w1 = _dt.datetime.now()
+    barrier(world)
+    ms = max_over_ranks(e0.elapsed_time(e1), world)
+    time.sleep(0.25)
+    sampler.stop()
+    L.moe_check_errors(stream)
+    line = {
+        "metric": METRIC + f" (stack of {nl} layers, one CUDA graph)",
+        "value": wl.T * world * args.steps / (ms / 1e3), "unit": "tokens/s", "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms / args.steps,
+        "ms_per_layer": ms / args.steps / nl, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "e4m3" if args.precision == "fp8" else "bf16",
+        "data": "synthetic (seeded N(0,1) activations, N(0,0.02^2) bf16 weights)",
+        "config": dict(config_of(wl, args), layers=nl, graph=True,
+                       between_layers="unit-gain RMS normalization (moe_rms_norm)"),
+        "gpu_launches": g.kernels * args.steps,
+        "clocks": sampler.summary(w0, w1),
+    }
+    g.close()
     if rank == 0:
         print(json.dumps(line), flush=True)
 

@@ -356,6 +356,50 @@ moe_status moe_layer_forward(const moe_config* cfg, const moe_exec* ex, const mo
                              size_t ws_bytes, void* stream, void* aux_stream);
 
 /*
+ * A stack of n_layers consecutive MoE layers (the paper's multi-layer study,
+ * Section 4.3 "Multi-layer scaling", L = 1..16): layer 0 reads x, layer l + 1
+ * reads layer l's output, layer n_layers - 1 writes out. layers[l] holds layer
+ * l's weights (layers may share tensors). rms_norm 1: between layers every
+ * token row h is replaced by bf16(h / sqrt(mean(h^2) + 1e-6)) (fp32), the
+ * unit-gain RMSNorm a DeepSeek-V3 block applies before its MoE; 0: raw chain. x and out [T,H] bf16 (may not
+ * overlap each other or ws); ex->out_fp32 must be 0 (the layers chain through
+ * bf16 activations); ex->stage_events, if set, are recorded by every layer.
+ * ws: moe_stack_workspace_size(cfg, ex) bytes, 256-byte aligned: one layer
+ * workspace shared by all layers plus two [T,H] bf16 activation buffers.
+ * Ordering on `stream` as for moe_layer_forward.
+ */
+size_t moe_stack_workspace_size(const moe_config* cfg, const moe_exec* ex);
+
+/* The normalization between stacked layers on its own: for each row r of
+ * x [rows, H] bf16, out[r] = bf16(x[r] * rsqrt(mean(x[r]^2) + 1e-6)), the sum
+ * of squares in fp32. H a multiple of 8; out may equal x (in place), otherwise
+ * the two must not overlap; both 16-byte aligned. */
+moe_status moe_rms_norm(int64_t rows, int32_t H, const uint16_t* x, uint16_t* out, void* stream);
+moe_status moe_stack_forward(const moe_config* cfg, const moe_exec* ex, const moe_weights* layers,
+                             int32_t n_layers, int32_t rms_norm, const uint16_t* x, uint16_t* out,
+                             void* ws, size_t ws_bytes, void* stream, void* aux_stream);
+
+/*
+ * CUDA-graph form of moe_stack_forward: runs the stack once eagerly (on a
+ * private stream, synchronised), then records it by stream capture into an
+ * executable graph bound to these pointers and shapes (x, out, ws, every
+ * layer's weights; ex->stage_events must be NULL). moe_graph_launch replays
+ * all layers with one launch on `stream`: new inputs are written into x, the
+ * result is read from out. The weights, ws, x and out must stay allocated
+ * while the graph exists. The graph does not synchronise; errors latched by
+ * the kernels are read with moe_check_errors as usual.
+ * moe_graph_kernel_count: kernels of this library in one replay.
+ */
+typedef struct moe_graph_s* moe_graph;
+moe_status moe_graph_create_stack(const moe_config* cfg, const moe_exec* ex,
+                                  const moe_weights* layers, int32_t n_layers, int32_t rms_norm,
+                                  const uint16_t* x, uint16_t* out, void* ws, size_t ws_bytes,
+                                  moe_graph* graph);
+moe_status moe_graph_launch(moe_graph graph, void* stream);
+uint64_t moe_graph_kernel_count(moe_graph graph);
+void moe_graph_destroy(moe_graph graph);
+
+/*
  * Testing hook for failure detection (no counterpart in the paper): exactly
  * moe_expert_ffn, except that CTA 0 of each grouped GEMM never issues its
  * producer fill number `stall_fill` (0-based), so the MMA's barrier wait on

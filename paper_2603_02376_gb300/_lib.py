@@ -30,7 +30,9 @@ EXPORTS = ("moe_status_string", "moe_validate_config", "moe_workspace_size",
            "moe_expert_ffn", "moe_combine", "moe_layer_forward", "moe_check_errors",
            "moe_launch_count", "moe_shutdown", "moe_dispatch_noalloc",
            "moe_testing_expert_ffn_stall", "moe_pack_weights", "moe_quantize_fp8",
-           "moe_expert_ffn_fp8", "moe_expert_ffn_fp8_workspace_size")
+           "moe_expert_ffn_fp8", "moe_expert_ffn_fp8_workspace_size", "moe_stack_workspace_size",
+           "moe_stack_forward", "moe_rms_norm", "moe_graph_create_stack", "moe_graph_launch",
+           "moe_graph_kernel_count", "moe_graph_destroy")
 MOE_DISPATCH_NOALLOC_MAX_ENTRIES = 131072
 
 
@@ -106,6 +108,15 @@ def load(path: str = LIB_PATH) -> ctypes.CDLL:
                                              ctypes.c_int64, ctypes.c_int64, P]),
         "moe_layer_forward": (S, [cfgp, exp, ctypes.POINTER(moe_weights), P, P,
                                   ctypes.POINTER(moe_aux), P, SZ, P, P]),
+        "moe_stack_workspace_size": (SZ, [cfgp, exp]),
+        "moe_rms_norm": (S, [ctypes.c_int64, I32, P, P, P]),
+        "moe_stack_forward": (S, [cfgp, exp, ctypes.POINTER(moe_weights), I32, I32, P, P, P, SZ,
+                                  P, P]),
+        "moe_graph_create_stack": (S, [cfgp, exp, ctypes.POINTER(moe_weights), I32, I32, P, P, P,
+                                       SZ, ctypes.POINTER(ctypes.c_void_p)]),
+        "moe_graph_launch": (S, [P, P]),
+        "moe_graph_kernel_count": (ctypes.c_uint64, [P]),
+        "moe_graph_destroy": (None, [P]),
         "moe_check_errors": (S, [P]),
         "moe_launch_count": (ctypes.c_uint64, []),
         "moe_shutdown": (None, []),
@@ -312,6 +323,83 @@ def moe_layer_forward(cfg, ex, weights: moe_weights, x, out, aux: moe_aux | None
     _check(load().moe_layer_forward(ctypes.byref(cfg), ctypes.byref(ex), ctypes.byref(weights),
                                     _ptr(x), _ptr(out), auxp, _ptr(ws), nb, _stream(stream), a_s),
            "moe_layer_forward")
+
+
+def moe_stack_workspace_size(cfg, ex) -> int:
+    return load().moe_stack_workspace_size(ctypes.byref(cfg), ctypes.byref(ex))
+
+
+def moe_rms_norm(x, out, stream=None) -> None:
+    """Row-wise unit-gain RMS normalization of a bf16 tensor viewed as [rows, H]."""
+    H = x.shape[-1]
+    _check(load().moe_rms_norm(x.numel() // H, H, _ptr(x), _ptr(out), _stream(stream)),
+           "moe_rms_norm")
+
+
+def _layers(layers):
+    arr = (moe_weights * len(layers))(*layers)
+    return arr, len(layers)
+
+
+def moe_stack_forward(cfg, ex, layers, x, out, ws, stream=None, aux_stream=None,
+                      rms_norm=1) -> None:
+    """Consecutive layers (a list of moe_weights); bf16 x -> bf16 out."""
+    arr, n = _layers(layers)
+    nb = 0 if ws is None else ws.numel() * ws.element_size()
+    a_s = None if aux_stream is None else _stream(aux_stream)
+    _check(load().moe_stack_forward(ctypes.byref(cfg), ctypes.byref(ex), arr, n, int(rms_norm),
+                                    _ptr(x), _ptr(out), _ptr(ws), nb, _stream(stream), a_s),
+           "moe_stack_forward")
+
+
+def moe_graph_create_stack(cfg, ex, layers, x, out, ws, rms_norm=1) -> ctypes.c_void_p:
+    """Handle of an executable CUDA graph of the stack (free with moe_graph_destroy)."""
+    arr, n = _layers(layers)
+    nb = 0 if ws is None else ws.numel() * ws.element_size()
+    h = ctypes.c_void_p()
+    _check(load().moe_graph_create_stack(ctypes.byref(cfg), ctypes.byref(ex), arr, n,
+                                         int(rms_norm), _ptr(x), _ptr(out), _ptr(ws), nb,
+                                         ctypes.byref(h)),
+           "moe_graph_create_stack")
+    return h
+
+
+def moe_graph_launch(graph, stream=None) -> None:
+    _check(load().moe_graph_launch(graph, _stream(stream)), "moe_graph_launch")
+
+
+def moe_graph_kernel_count(graph) -> int:
+    return int(load().moe_graph_kernel_count(graph))
+
+
+def moe_graph_destroy(graph) -> None:
+    load().moe_graph_destroy(graph)
+
+
+class Graph:
+    """Owner of a moe_graph_create_stack handle; keeps its tensors alive."""
+
+    def __init__(self, cfg, ex, layers, x, out, ws, rms_norm=1):
+        self._h = moe_graph_create_stack(cfg, ex, layers, x, out, ws, rms_norm)
+        self._keep = (x, out, ws, layers)   # the graph holds these pointers
+
+    @property
+    def kernels(self) -> int:
+        return moe_graph_kernel_count(self._h)
+
+    def launch(self, stream=None) -> None:
+        moe_graph_launch(self._h, stream)
+
+    def close(self) -> None:
+        if self._h:
+            moe_graph_destroy(self._h)
+            self._h = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
 
 
 def moe_check_errors(stream=None) -> None:

@@ -127,6 +127,39 @@ def test_entry_points_reject_bad_arguments_without_a_gpu(lib):
     assert L.moe_workspace_size(c, exc) == 0
 
 
+def test_stack_entry_points_reject_bad_arguments_without_a_gpu(lib):
+    c = L.config(**GOOD)
+    z = ctypes.c_void_p(0)
+    p = ctypes.c_void_p(0x1000)
+    cb = ctypes.byref
+    ex = L.exec_config()
+    n1 = L.moe_workspace_size(c, ex)
+    ns = L.moe_stack_workspace_size(c, ex)
+    assert ns >= n1 + 2 * GOOD["T"] * GOOD["H"] * 2
+    assert L.moe_stack_workspace_size(c, L.exec_config(out_fp32=1)) == 0   # bf16 chaining only
+    W = (L.moe_weights * 2)(L.moe_weights(0x1000, None, 0x1000, 0x1000, 0x1000, 0x1000),
+                           L.moe_weights(0x1000, None, 0x1000, 0x1000, 0x1000, 0x1000))
+    S = lib.moe_stack_forward
+    assert S(cb(c), cb(ex), W, 0, 1, p, p, p, 1 << 40, z, z) == L.MOE_ERR_INVALID_ARG   # no layers
+    assert S(cb(c), cb(ex), W, 2, 2, p, p, p, 1 << 40, z, z) == L.MOE_ERR_INVALID_ARG   # rms_norm
+    assert S(cb(c), cb(L.exec_config(out_fp32=1)), W, 2, 1, p, p, p, 1 << 40, z, z) == L.MOE_ERR_INVALID_ARG
+    assert S(cb(c), cb(ex), W, 2, 1, p, p, z, 0, z, z) == L.MOE_ERR_WORKSPACE
+    assert S(cb(c), cb(ex), None, 2, 1, p, p, p, 1 << 40, z, z) == L.MOE_ERR_INVALID_ARG
+    h = ctypes.c_void_p()
+    G = lib.moe_graph_create_stack
+    assert G(cb(c), cb(ex), W, 2, 1, p, p, p, 1 << 40, None) == L.MOE_ERR_INVALID_ARG   # no handle
+    assert G(cb(c), cb(ex), W, 0, 1, p, p, p, 1 << 40, cb(h)) == L.MOE_ERR_INVALID_ARG
+    assert G(cb(c), cb(ex), W, 2, 1, p, p, z, 0, cb(h)) == L.MOE_ERR_WORKSPACE
+    evs = (ctypes.c_void_p * L.MOE_N_STAGE_EVENTS)()
+    ext = L.exec_config()
+    ext.stage_events = ctypes.cast(evs, ctypes.POINTER(ctypes.c_void_p))
+    assert G(cb(c), cb(ext), W, 2, 1, p, p, p, 1 << 40, cb(h)) == L.MOE_ERR_INVALID_ARG  # tracing
+    assert h.value is None
+    assert lib.moe_graph_launch(None, z) == L.MOE_ERR_INVALID_ARG
+    assert lib.moe_graph_kernel_count(None) == 0
+    lib.moe_graph_destroy(None)
+
+
 def test_fused_combine_workspace():
     # fused combine: no y_perm [T*k, H] and no shared y; an fp32 [T, H] accumulator
     # only when the output is bf16 (an fp32 output is the accumulator itself)

@@ -619,7 +619,7 @@ def run_stack(args, wl, rank, world, local, device, L, cfg, ex, W, d):
     x = d["x"].clone()
     out = torch.empty_like(x)
     stream = torch.cuda.current_stream()
-    g = L.Graph(cfg, ex, layers, x, out, ws)
+    g = L.Graph(cfg, ex, layers, x, out, ws, stream=stream)
     for _ in range(args.warmup):
         g.launch(stream)
     torch.cuda.synchronize()

@@ -381,7 +381,8 @@ moe_status moe_stack_forward(const moe_config* cfg, const moe_exec* ex, const mo
 
 /*
  * CUDA-graph form of moe_stack_forward: runs the stack once eagerly (on a
- * private stream, synchronised), then records it by stream capture into an
+ * private stream ordered after prior work on `stream`, then synchronised, so
+ * x must be ready by then), then records it by stream capture into an
  * executable graph bound to these pointers and shapes (x, out, ws, every
  * layer's weights; ex->stage_events must be NULL). moe_graph_launch replays
  * all layers with one launch on `stream`: new inputs are written into x, the
@@ -394,7 +395,7 @@ typedef struct moe_graph_s* moe_graph;
 moe_status moe_graph_create_stack(const moe_config* cfg, const moe_exec* ex,
                                   const moe_weights* layers, int32_t n_layers, int32_t rms_norm,
                                   const uint16_t* x, uint16_t* out, void* ws, size_t ws_bytes,
-                                  moe_graph* graph);
+                                  void* stream, moe_graph* graph);
 moe_status moe_graph_launch(moe_graph graph, void* stream);
 uint64_t moe_graph_kernel_count(moe_graph graph);
 void moe_graph_destroy(moe_graph graph);

@@ -113,7 +113,7 @@ def load(path: str = LIB_PATH) -> ctypes.CDLL:
         "moe_stack_forward": (S, [cfgp, exp, ctypes.POINTER(moe_weights), I32, I32, P, P, P, SZ,
                                   P, P]),
         "moe_graph_create_stack": (S, [cfgp, exp, ctypes.POINTER(moe_weights), I32, I32, P, P, P,
-                                       SZ, ctypes.POINTER(ctypes.c_void_p)]),
+                                       SZ, P, ctypes.POINTER(ctypes.c_void_p)]),
         "moe_graph_launch": (S, [P, P]),
         "moe_graph_kernel_count": (ctypes.c_uint64, [P]),
         "moe_graph_destroy": (None, [P]),
@@ -352,14 +352,15 @@ def moe_stack_forward(cfg, ex, layers, x, out, ws, stream=None, aux_stream=None,
            "moe_stack_forward")
 
 
-def moe_graph_create_stack(cfg, ex, layers, x, out, ws, rms_norm=1) -> ctypes.c_void_p:
+def moe_graph_create_stack(cfg, ex, layers, x, out, ws, rms_norm=1,
+                           stream=None) -> ctypes.c_void_p:
     """Handle of an executable CUDA graph of the stack (free with moe_graph_destroy)."""
     arr, n = _layers(layers)
     nb = 0 if ws is None else ws.numel() * ws.element_size()
     h = ctypes.c_void_p()
     _check(load().moe_graph_create_stack(ctypes.byref(cfg), ctypes.byref(ex), arr, n,
                                          int(rms_norm), _ptr(x), _ptr(out), _ptr(ws), nb,
-                                         ctypes.byref(h)),
+                                         _stream(stream), ctypes.byref(h)),
            "moe_graph_create_stack")
     return h
 
@@ -379,8 +380,8 @@ def moe_graph_destroy(graph) -> None:
 class Graph:
     """Owner of a moe_graph_create_stack handle; keeps its tensors alive."""
 
-    def __init__(self, cfg, ex, layers, x, out, ws, rms_norm=1):
-        self._h = moe_graph_create_stack(cfg, ex, layers, x, out, ws, rms_norm)
+    def __init__(self, cfg, ex, layers, x, out, ws, rms_norm=1, stream=None):
+        self._h = moe_graph_create_stack(cfg, ex, layers, x, out, ws, rms_norm, stream)
         self._keep = (x, out, ws, layers)   # the graph holds these pointers
 
     @property

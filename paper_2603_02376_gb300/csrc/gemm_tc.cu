@@ -53,7 +53,7 @@ constexpr int BK = 64;            // bf16 per stage along K: one 128-byte swizzl
 constexpr int UMMA_K = 16;        // K of one tcgen05.mma kind::f16
 constexpr int B_BOX = 16;         // token rows per TMA box (tile remainders)
 constexpr int B_BIG = 64;         // token rows per TMA box (bulk of tiles of >= 64 rows)
-constexpr int NUM_THREADS = 192;  // 6 warps
+constexpr int NUM_THREADS = 320;  // 10 warps: producer, MMA, 8 epilogue
 constexpr uint64_t WAIT_LIMIT_NS = 2000000000ull;  // default limit of every barrier wait
 
 
@@ -389,7 +389,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
     }
     for (int s = 0; s < TL::ACC_STAGES; ++s) {
       mbar_init(smem_u32(&ctrl->acc_full[s]), 1);
-      mbar_init(smem_u32(&ctrl->acc_empty[s]), 4);
+      mbar_init(smem_u32(&ctrl->acc_empty[s]), 8);  // one arrive per epilogue warp
     }
     mbar_init(smem_u32(&ctrl->drain), 1);
     ctrl->abort_flag = 0;
@@ -617,7 +617,10 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
     }
   } else {
     // ------------------------------------------------------------------ epilogue
+    // Two warps per TMEM lane quarter: warp w reads lanes 32 * (w % 4) .. + 31
+    // and the 16-column chunks c0 = 16 * half, 16 * half + 32, ... of a unit.
     const int q = warp & 3;  // TMEM lane quarter this warp may access
+    const int half = (warp - 2) >> 2;
     int j = 0;
     for (int u = blockIdx.x; u < total_units; u += gridDim.x, ++j) {
       const Unit U = decode_unit<NMAX>(u, tile_off, row_off, a, units1, kblocks);
@@ -629,7 +632,8 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       const uint32_t tq = tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(as * TL::ACC_COLS);
       const int f = U.fb * TL::FEAT + q * 32 + lane;
       const size_t o = (size_t)U.row0 * a.out_ld + f;
-      // FP8: the scales of this thread's weight row(s) and of each token column
+      // FP8: the scales of this thread's weight row(s); the token columns' scales
+      // are fetched per chunk below
       float sa0 = 1.f, sa1 = 1.f;
       const float* bsc = nullptr;
       const int32_t* bidx = nullptr;
@@ -641,27 +645,30 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
         bsc = U.grp ? a.b_scale1 : a.b_scale0;
         bidx = U.grp ? nullptr : a.b_scale_idx0;
       }
-      auto col_scale = [&](int c) -> float {
-        if (!F8) return 1.f;
-        const int br = U.row0 + c;
-        return bsc[bidx ? bidx[br] : br];
-      };
       void* out = U.grp ? static_cast<void*>(static_cast<float*>(a.out1) + U.split * a.split_stride)
                         : a.out0;
       float* comb = U.grp ? a.comb_out1 : a.comb_out0;
       const int32_t* ctok = U.grp ? nullptr : a.comb_tok0;
       const float* cw = U.grp ? nullptr : a.comb_w0;
-      // the destination row of token column c and the weight it is added with
-      auto comb_dst = [&](int c, float* wv) -> float* {
-        const int br = U.row0 + c;
-        *wv = cw ? cw[br] : 1.f;
-        return comb + (size_t)(ctok ? ctok[br] : br) * a.out_ld + f;
-      };
       // The unit's columns; CB (the fused combine) is a compile-time copy of the
-      // loop so the plain stores keep their unrolled form.
+      // loop so the plain stores keep their unrolled form. Per 16-column chunk,
+      // lane l < 16 fetches what column c0 + l needs from global memory (the
+      // token's scale; with the combine its token row and gate weight) once,
+      // and the other lanes read it with a shuffle: no dependent global loads
+      // inside the column loop.
       auto columns = [&](auto cb_tag) {
         constexpr bool CB = decltype(cb_tag)::value;
-        for (int c0 = 0; c0 < U.m; c0 += 16) {
+        for (int c0 = 16 * half; c0 < U.m; c0 += 32) {
+          const int mc = c0 + (lane & 15);            // this lane's column of the chunk
+          const bool cv = mc < U.m;
+          const int br = U.row0 + (cv ? mc : 0);
+          float sb_l = 1.f, w_l = 1.f;
+          int t_l = br;
+          if (F8 && cv) sb_l = bsc[bidx ? bidx[br] : br];
+          if (CB && cv) {
+            if (cw) w_l = cw[br];
+            if (ctok) t_l = ctok[br];
+          }
           uint32_t g[16];
           tmem_ld16(tq + c0, g);
           if constexpr (SWIGLU) {
@@ -670,13 +677,14 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
             tmem_wait_ld();
 #pragma unroll
             for (int i = 0; i < 16; ++i) {
+              const float sb = F8 ? __shfl_sync(0xffffffffu, sb_l, i) : 1.f;
               if (c0 + i < U.m) {
-                const float sb = col_scale(c0 + i);
                 const float gv = __uint_as_float(g[i]) * (sa0 * sb);
                 const float uv = __uint_as_float(v[i]) * (sa1 * sb);
-                // silu(g) * u with the hardware exp2-based __expf and a reciprocal:
-                // their error (a few fp32 ulp) is far below the bf16 rounding of h
-                const float hv = gv * __frcp_rn(1.0f + __expf(-gv)) * uv;
+                // silu(g) * u with the hardware exp2-based __expf and a fast
+                // division: their error (a few fp32 ulp) is far below the bf16
+                // rounding of h
+                const float hv = __fdividef(gv, 1.0f + __expf(-gv)) * uv;
                 static_cast<uint16_t*>(out)[o + (size_t)(c0 + i) * a.out_ld] =
                     float_to_bf16_bits(hv);
               }
@@ -687,13 +695,14 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
             tmem_wait_ld();
 #pragma unroll
             for (int i = 0; i < 16; ++i) {
+              const float sb = F8 ? __shfl_sync(0xffffffffu, sb_l, i) : 1.f;
+              const float wv = CB ? __shfl_sync(0xffffffffu, w_l, i) : 1.f;
+              const int tv = CB ? __shfl_sync(0xffffffffu, t_l, i) : 0;
               if (c0 + i < U.m) {
-                const float sb = col_scale(c0 + i);
                 const float y0 = __uint_as_float(g[i]) * (sa0 * sb);
                 const float y1 = __uint_as_float(v[i]) * (sa1 * sb);
                 if constexpr (CB) {
-                  float wv;
-                  float* d = comb_dst(c0 + i, &wv);
+                  float* d = comb + (size_t)tv * a.out_ld + f;
                   atomicAdd(d, wv * y0);
                   atomicAdd(d + BM, wv * y1);
                 } else {
@@ -707,12 +716,13 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
             tmem_wait_ld();
 #pragma unroll
             for (int i = 0; i < 16; ++i) {
+              const float sb = F8 ? __shfl_sync(0xffffffffu, sb_l, i) : 1.f;
+              const float wv = CB ? __shfl_sync(0xffffffffu, w_l, i) : 1.f;
+              const int tv = CB ? __shfl_sync(0xffffffffu, t_l, i) : 0;
               if (c0 + i < U.m) {
-                const float y0 = __uint_as_float(g[i]) * (sa0 * col_scale(c0 + i));
+                const float y0 = __uint_as_float(g[i]) * (sa0 * sb);
                 if constexpr (CB) {
-                  float wv;
-                  float* d = comb_dst(c0 + i, &wv);
-                  atomicAdd(d, wv * y0);
+                  atomicAdd(comb + (size_t)tv * a.out_ld + f, wv * y0);
                 } else {
                   static_cast<float*>(out)[o + (size_t)(c0 + i) * a.out_ld] = y0;
                 }

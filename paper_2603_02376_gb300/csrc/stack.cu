@@ -126,7 +126,7 @@ moe_status moe_stack_forward(const moe_config* cfg, const moe_exec* ex, const mo
 moe_status moe_graph_create_stack(const moe_config* cfg, const moe_exec* ex,
                                   const moe_weights* layers, int32_t n_layers, int32_t rms_norm,
                                   const uint16_t* x, uint16_t* out, void* ws, size_t ws_bytes,
-                                  moe_graph* graph) {
+                                  void* stream, moe_graph* graph) {
   if (!graph) return MOE_ERR_INVALID_ARG;
   *graph = nullptr;
   if (!valid_stack(cfg, ex, layers, n_layers) || (rms_norm != 0 && rms_norm != 1))
@@ -136,10 +136,18 @@ moe_status moe_graph_create_stack(const moe_config* cfg, const moe_exec* ex,
     return MOE_ERR_WORKSPACE;
   cudaStream_t cs = nullptr;
   if (cudaStreamCreateWithFlags(&cs, cudaStreamNonBlocking) != cudaSuccess) return MOE_ERR_CUDA;
+  // The private stream starts after the caller's prior work on `stream` (x
+  // may still be being written there).
+  cudaEvent_t ready = nullptr;
+  moe_status st = MOE_OK;
+  if (cudaEventCreateWithFlags(&ready, cudaEventDisableTiming) != cudaSuccess ||
+      cudaEventRecord(ready, static_cast<cudaStream_t>(stream)) != cudaSuccess ||
+      cudaStreamWaitEvent(cs, ready, 0) != cudaSuccess)
+    st = MOE_ERR_CUDA;
   // One eager forward first: lazily created internal streams, events and
   // kernel attributes are then in place before the capture.
-  moe_status st =
-      moe_stack_forward(cfg, ex, layers, n_layers, rms_norm, x, out, ws, ws_bytes, cs, nullptr);
+  if (st == MOE_OK)
+    st = moe_stack_forward(cfg, ex, layers, n_layers, rms_norm, x, out, ws, ws_bytes, cs, nullptr);
   if (st == MOE_OK && cudaStreamSynchronize(cs) != cudaSuccess) st = MOE_ERR_CUDA;
   cudaGraph_t g = nullptr;
   const uint64_t k0 = moe_launch_count();
@@ -157,6 +165,7 @@ moe_status moe_graph_create_stack(const moe_config* cfg, const moe_exec* ex,
   cudaGraphExec_t exec = nullptr;
   if (st == MOE_OK && cudaGraphInstantiate(&exec, g, 0) != cudaSuccess) st = MOE_ERR_CUDA;
   if (g) cudaGraphDestroy(g);
+  if (ready) cudaEventDestroy(ready);
   cudaStreamDestroy(cs);
   cudaGetLastError();  // a failed capture leaves no sticky error behind
   if (st != MOE_OK) {

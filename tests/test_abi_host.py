@@ -147,13 +147,13 @@ def test_stack_entry_points_reject_bad_arguments_without_a_gpu(lib):
     assert S(cb(c), cb(ex), None, 2, 1, p, p, p, 1 << 40, z, z) == L.MOE_ERR_INVALID_ARG
     h = ctypes.c_void_p()
     G = lib.moe_graph_create_stack
-    assert G(cb(c), cb(ex), W, 2, 1, p, p, p, 1 << 40, None) == L.MOE_ERR_INVALID_ARG   # no handle
-    assert G(cb(c), cb(ex), W, 0, 1, p, p, p, 1 << 40, cb(h)) == L.MOE_ERR_INVALID_ARG
-    assert G(cb(c), cb(ex), W, 2, 1, p, p, z, 0, cb(h)) == L.MOE_ERR_WORKSPACE
+    assert G(cb(c), cb(ex), W, 2, 1, p, p, p, 1 << 40, z, None) == L.MOE_ERR_INVALID_ARG  # no handle
+    assert G(cb(c), cb(ex), W, 0, 1, p, p, p, 1 << 40, z, cb(h)) == L.MOE_ERR_INVALID_ARG
+    assert G(cb(c), cb(ex), W, 2, 1, p, p, z, 0, z, cb(h)) == L.MOE_ERR_WORKSPACE
     evs = (ctypes.c_void_p * L.MOE_N_STAGE_EVENTS)()
     ext = L.exec_config()
     ext.stage_events = ctypes.cast(evs, ctypes.POINTER(ctypes.c_void_p))
-    assert G(cb(c), cb(ext), W, 2, 1, p, p, p, 1 << 40, cb(h)) == L.MOE_ERR_INVALID_ARG  # tracing
+    assert G(cb(c), cb(ext), W, 2, 1, p, p, p, 1 << 40, z, cb(h)) == L.MOE_ERR_INVALID_ARG  # tracing
     assert h.value is None
     assert lib.moe_graph_launch(None, z) == L.MOE_ERR_INVALID_ARG
     assert lib.moe_graph_kernel_count(None) == 0

@@ -53,9 +53,8 @@ def parse():
     p.add_argument("--no-fuse-gather", action="store_true",
                    help="pack x_perm with a dispatch kernel instead of gathering in GEMM1")
     p.add_argument("--pack", choices=("auto", "yes", "no"), default="auto",
-                   help="tile-pack the expert weights at load (auto: for batches of more than "
-                        "24 rows per expert, where it measured 1-4 %% faster; decode-sized "
-                        "batches measured ~1 %% faster row-major)")
+                   help="tile-pack the expert weights at load (auto: yes for bf16, "
+                        "no for fp8, which has no packed form)")
     p.add_argument("--precision", choices=("bf16", "fp8"), default="bf16",
                    help="expert GEMM operands: bf16, or e4m3 with per-row scales (weights "
                         "quantized once at load, tokens and h quantized inside each step)")
@@ -351,12 +350,12 @@ def run_reference(args, wl, rank, world, device):
 
 
 def packs(args, wl):
-    """Whether the run uses tile-packed expert weights (bf16 only)."""
+    """Whether the run uses tile-packed expert weights (bf16 only; auto = yes: the
+    GEMMs fetch each packed weight tile with one bulk copy, measured as fast or
+    faster at every batch size)."""
     if args.precision == "fp8":
         return False
-    if args.pack == "auto":
-        return wl.T * wl.k > 24 * wl.E
-    return args.pack == "yes"
+    return args.pack in ("auto", "yes")
 
 
 def config_of(wl, args):

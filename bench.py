@@ -196,7 +196,7 @@ def calibrate(L, wl, d, device):
 
 
 def algorithmic(wl, touched, fused_gather=True, fp8=False, fused_combine=False):
-    """Algorithmic bytes and flops of each stage for one forward (see DESIGN.md).
+    """Algorithmic bytes and flops of each stage for one forward.
 
     GEMM1's token operand is counted as R*H*eb either way (packed rows read, or
     the same rows gathered from x); a fused dispatch has no copy of its own.

@@ -26,7 +26,7 @@ not restated by the paper; it follows the DeepSeek-V3 layer the paper names:
   the top-k by p are selected; weights are p (not renormalised) times
   `route_scale`.
 
-Readings taken where the paper is silent (also listed in the design doc):
+Readings taken where the paper is silent:
 * Decisions (which experts, which groups) are taken on fp32 scores: the
   selection score is fp32(sigmoid(L)) + fp32 bias (one fp32 add); the group
   score is the fp32 sum of the two largest selection scores.

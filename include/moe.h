@@ -349,7 +349,9 @@ moe_status moe_combine(const moe_config* cfg, const float* y_perm, const int32_t
  * ws: moe_workspace_size(cfg, ex) bytes. aux_stream: the pack stream of the
  * overlapped pipeline (NULL = an internal high-priority stream); unused when
  * ex->overlap = 0. All work is ordered after prior work on `stream`, and later
- * work on `stream` is ordered after the whole layer.
+ * work on `stream` is ordered after the whole layer. Calls from several host
+ * threads are safe; pipelined calls on one device share internal events and
+ * enqueue one at a time. Concurrent calls must not share a workspace.
  */
 moe_status moe_layer_forward(const moe_config* cfg, const moe_exec* ex, const moe_weights* w,
                              const uint16_t* x, void* out, const moe_aux* aux, void* ws,

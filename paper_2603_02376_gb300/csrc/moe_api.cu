@@ -27,6 +27,10 @@ struct DeviceStreams {
   std::vector<cudaEvent_t> events;
 };
 DeviceStreams g_streams[MAX_DEVICES];
+// Pipelined forwards of one device share its internal events: their host-side
+// enqueue is serialised (a wait captures the event's record at the time of the
+// wait call, so a later re-record by another call cannot reach back into it).
+std::mutex g_pipe_mu[MAX_DEVICES];
 
 int current_device() {
   int d = 0;
@@ -676,6 +680,7 @@ moe_status moe_layer_forward(const moe_config* cfg, const moe_exec* ex, const mo
     return MOE_OK;
   }
 
+  std::lock_guard<std::mutex> pipe_lock(g_pipe_mu[dev]);
   cudaStream_t ps = aux_stream ? (cudaStream_t)aux_stream : pack_stream(dev);
   if (!ps) return MOE_ERR_CUDA;
   const int n_stage = ex->chunk_axis == 0 ? L.n_chunks : ex->n_expert_chunks;

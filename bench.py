@@ -63,6 +63,10 @@ def parse():
     p.add_argument("--layers", type=int, default=1,
                    help="time a stack of this many consecutive layers replayed as one CUDA "
                         "graph (each layer its own router; expert weights shared)")
+    p.add_argument("--sweep", action="store_true",
+                   help="the dispatch + combine data-movement sweep instead of a layer: identity "
+                        "experts, H=7168, E=256, top-8 uniform routing, T in 1024..65536; one JSON "
+                        "line with the HBM GB/s of the permutation, dispatch and combine kernels")
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--cpu-tokens", type=int, default=128, help="oracle sample size (tokens)")
     return p.parse_args()
@@ -657,6 +661,90 @@ def run_stack(args, wl, rank, world, local, device, L, cfg, ex, W, d):
         print(json.dumps(line), flush=True)
 
 
+def run_sweep(args, rank, world, local, device):
+    """Dispatch + combine of uniform top-8 routing at T = 1024 .. 65536 (identity experts).
+
+    Per T: the permutation alone (moe_dispatch without x_perm), the permutation and
+    the row copy (moe_dispatch with x_perm; the copy's time is the difference), and
+    moe_combine of fp32 rows into a bf16 output, each timed with CUDA events around
+    `steps` launches, an L2-sized buffer written between launches. Algorithmic
+    bytes: copy T*H*2 read + T*k*H*2 written; combine T*k*H*4 read + T*H*2 written
+    (+ 8 bytes of slot row and weight per entry).
+    """
+    from paper_2603_02376_gb300 import _lib as L
+    L.load()
+    H, E, k = 7168, 256, 8
+    hbm, _, _, src = peaks()
+    stream = torch.cuda.current_stream()
+    flush = torch.empty(256 << 20, dtype=torch.uint8, device=device)
+    n0 = L.moe_launch_count()
+    rows, w0 = [], _dt.datetime.now()
+    sampler = ClockSampler(local)
+
+    def timed(fn):
+        ms = 0.0
+        for i in range(args.warmup + args.steps):
+            flush.fill_(i & 0xFF)
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record(stream)
+            fn()
+            e1.record(stream)
+            torch.cuda.synchronize()
+            if i >= args.warmup:
+                ms += e0.elapsed_time(e1)
+        return ms / args.steps
+
+    for T in I.DISPATCH_SWEEP_T:
+        c = L.config(T, H, E, k, 2048)
+        idx, w = I.uniform_routing(T, E, k, seed=rank, device=device)
+        x = I.randn((T, H), 1.0, torch.bfloat16, rank, "x", device)
+        counts = torch.empty(E, dtype=torch.int32, device=device)
+        offsets = torch.empty(E + 1, dtype=torch.int32, device=device)
+        rst = torch.empty(T * k, dtype=torch.int32, device=device)
+        slot = torch.empty(T * k, dtype=torch.int32, device=device)
+        xp = torch.empty((T * k, H), dtype=torch.bfloat16, device=device)
+        ws = torch.empty(L.moe_dispatch_workspace_size(c), dtype=torch.uint8, device=device)
+        perm_ms = timed(lambda: L.moe_dispatch(c, x, idx, counts, offsets, rst, slot, None, ws,
+                                               stream))
+        disp_ms = timed(lambda: L.moe_dispatch(c, x, idx, counts, offsets, rst, slot, xp, ws,
+                                               stream))
+        yp = xp.float()
+        del xp
+        out = torch.empty((T, H), dtype=torch.bfloat16, device=device)
+        comb_ms = timed(lambda: L.moe_combine(c, yp, slot, w, None, out, 0, stream))
+        L.moe_check_errors(stream)
+        copy_ms = max(disp_ms - perm_ms, 1e-6)
+        copy_b = T * H * 2 + T * k * H * 2
+        comb_b = T * k * H * 4 + T * H * 2 + T * k * 8
+        rows.append({"T": T, "permutation_ms": round(perm_ms, 4),
+                     "dispatch_copy_ms": round(copy_ms, 4),
+                     "dispatch_copy_GBs": round(copy_b / copy_ms / 1e6, 1),
+                     "dispatch_copy_frac_hbm": round(copy_b / copy_ms / 1e6 / hbm, 3),
+                     "combine_ms": round(comb_ms, 4),
+                     "combine_GBs": round(comb_b / comb_ms / 1e6, 1),
+                     "combine_frac_hbm": round(comb_b / comb_ms / 1e6 / hbm, 3)})
+        del yp, out, x
+        torch.cuda.empty_cache()
+    w1 = _dt.datetime.now()
+    sampler.stop()
+    big = rows[-1]
+    line = {
+        "metric": "dispatch / combine HBM GB/s, identity experts (H=7168, E=256, top-8 uniform)",
+        "value": big["combine_GBs"], "unit": "GB/s", "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": big["combine_ms"], "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "bf16 rows, fp32 combine",
+        "data": "synthetic (seeded N(0,1) rows, uniform routing)",
+        "config": {"workload": "dispatch+combine sweep", "H": H, "E": E, "k": k,
+                   "T": list(I.DISPATCH_SWEEP_T),
+                   "l2": "a 256 MB buffer is written between timed launches"},
+        "peak": hbm, "peak_source": f"hbm_gbs of {src}", "sweep": rows,
+        "gpu_launches": L.moe_launch_count() - n0,
+        "clocks": sampler.summary(w0, w1),
+    }
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+
+
 def main():
     args = parse()
     rank, world, local = dist_env()
@@ -665,7 +753,9 @@ def main():
     torch.cuda.set_device(local)
     device = torch.device("cuda", local)
     wl = I.WORKLOADS[args.workload]
-    if args.impl == "reference":
+    if args.sweep and args.impl != "reference":
+        run_sweep(args, rank, world, local, device)
+    elif args.impl == "reference":
         run_reference(args, wl, rank, world, device)
     else:
         run_ours(args, wl, rank, world, local, device)

@@ -81,43 +81,43 @@ __global__ void __launch_bounds__(PERM_WARPS * 32) perm_hist_kernel(
   }
 }
 
-// One CTA of 1024 threads. Warp q handles experts q, q+32, ...; its lanes split
-// the chunks into contiguous runs and combine them with a warp scan.
+// One CTA of 1024 threads; thread e owns expert e (E <= 1024). It walks the
+// chunks in order and writes each chunk's base, the exclusive prefix of its
+// count over the earlier chunks: threads of consecutive experts touch adjacent
+// words, so every chunk row is one coalesced pass, and the loads of eight
+// chunks are issued before their sums are needed. The CTA then scans the E
+// totals into the expert offsets.
 __global__ void __launch_bounds__(1024) perm_scan_kernel(const int32_t* __restrict__ chunk_counts,
                                                          int n_chunks, int E,
                                                          int32_t* __restrict__ chunk_base,
                                                          int32_t* __restrict__ counts,
                                                          int32_t* __restrict__ offsets) {
-  __shared__ int tot[1024];
   __shared__ int wsum[32];
   const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
-  const int per = (n_chunks + 31) / 32;
-  for (int e = warp; e < E; e += 32) {
-    const int c0 = min(n_chunks, lane * per), c1 = min(n_chunks, c0 + per);
-    int s = 0;
-    for (int c = c0; c < c1; ++c) s += chunk_counts[(size_t)c * E + e];
-    int incl = s;
+  const int e = threadIdx.x;
+  int total = 0;
+  if (e < E) {
+    int c = 0;
+    for (; c + 8 <= n_chunks; c += 8) {
+      int v[8];
 #pragma unroll
-    for (int o = 1; o < 32; o <<= 1) {
-      const int v = __shfl_up_sync(0xffffffffu, incl, o);
-      if (lane >= o) incl += v;
+      for (int q = 0; q < 8; ++q) v[q] = chunk_counts[(size_t)(c + q) * E + e];
+#pragma unroll
+      for (int q = 0; q < 8; ++q) {
+        chunk_base[(size_t)(c + q) * E + e] = total;
+        total += v[q];
+      }
     }
-    int run = incl - s;
-    for (int c = c0; c < c1; ++c) {
+    for (; c < n_chunks; ++c) {
       const int v = chunk_counts[(size_t)c * E + e];
-      chunk_base[(size_t)c * E + e] = run;
-      run += v;
+      chunk_base[(size_t)c * E + e] = total;
+      total += v;
     }
-    const int total = __shfl_sync(0xffffffffu, incl, 31);
-    if (lane == 0) {
-      tot[e] = total;
-      counts[e] = total;
-    }
+    counts[e] = total;
   }
-  __syncthreads();
-  // exclusive scan of tot[0..E) with 1024 threads (E <= 1024)
+  // exclusive scan of the E totals with 1024 threads (E <= 1024)
   const int i = threadIdx.x;
-  const int v = i < E ? tot[i] : 0;
+  const int v = i < E ? total : 0;
   int incl = v;
 #pragma unroll
   for (int o = 1; o < 32; o <<= 1) {

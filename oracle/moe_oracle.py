@@ -409,6 +409,84 @@ def swiglu_ffn_fp8(rows, W13_q, s13, W2_q, s2):
 
 
 # ---------------------------------------------------------------------------
+# FP8 with block scales: DeepSeek-V3's fine-grained form of the quantize step,
+# one scale per 1 x 128 block of an activation row (x per token, h per packed
+# row) and one per 128 x 128 block of a weight matrix. Reading: the scales are
+# powers of two 2^k stored as UE8M0 exponent bytes k + 127 (the block-scale
+# format a tensor core applies by itself); a block's k is the smallest integer
+# with amax <= 448 * 2^k (k = 0 for an all-zero block), clamped to [-127, 127];
+# its values are e4m3(v * 2^-k), an exact scaling then one rounding to nearest
+# even, saturating. A product sums, block by block, q_a * q_w * 2^(k_a + k_w).
+# ---------------------------------------------------------------------------
+
+FP8_BLOCK = 128
+
+
+def block_exponent(amax) -> np.ndarray:
+    """k = min{integer k : amax <= 448 * 2^k} (0 where amax == 0), clamped to [-127, 127]."""
+    amax = np.asarray(amax, dtype=np.float64)
+    safe = np.where(amax > 0, amax, E4M3_MAX)
+    k = np.ceil(np.log2(safe / E4M3_MAX))
+    # settle the rounding of log2 against the definition (448 * 2^k is exact)
+    k = np.where(safe > E4M3_MAX * np.exp2(k), k + 1, k)
+    k = np.where(safe <= E4M3_MAX * np.exp2(k - 1), k - 1, k)
+    return np.clip(k, -127, 127).astype(np.int64)
+
+
+def quantize_blocks_e4m3(a, rows_per_block: int):
+    """Block e4m3 quantization of a [m, K] matrix in blocks of rows_per_block x 128.
+
+    Returns (q fp64 [m, K] on the e4m3 grid, k int64 [m / rows_per_block, K / 128]).
+    rows_per_block = 1 for activations, 128 for weights; m and K must divide.
+    """
+    a = np.asarray(a, dtype=np.float64)
+    m, K = a.shape
+    rb, cb = rows_per_block, FP8_BLOCK
+    assert m % rb == 0 and K % cb == 0
+    amax = np.abs(a).reshape(m // rb, rb, K // cb, cb).max(axis=(1, 3))
+    k = block_exponent(amax)
+    return e4m3_round(a * block_scales(-k, rb)), k
+
+
+def block_scales(k, rows_per_block: int) -> np.ndarray:
+    """2^k of every element: the block exponents k [m / rb, K / 128] spread over their blocks."""
+    k = np.asarray(k, dtype=np.int64)
+    return np.exp2(np.repeat(np.repeat(k, rows_per_block, axis=0), FP8_BLOCK, axis=1).astype(np.float64))
+
+
+def fp8_block_linear(a_q, k_a, W_q, k_w) -> np.ndarray:
+    """Product of block-scaled e4m3 operands (fp64): dequantize, then a_deq . W_deq^T.
+
+    a_q [m, K] with 1 x 128 block exponents k_a [m, K/128]; W_q [n, K] with
+    128 x 128 block exponents k_w [n/128, K/128].
+    """
+    a = np.asarray(a_q, dtype=np.float64) * block_scales(k_a, 1)
+    W = np.asarray(W_q, dtype=np.float64) * block_scales(k_w, FP8_BLOCK)
+    return a @ W.T
+
+
+def swiglu_h_fp8_blocks(rows, W13_q, k13) -> np.ndarray:
+    """GEMM1 + SwiGLU of the block-scaled FP8 form: x quantized per 1 x 128 block,
+    g | u = fp8_block_linear(x_q, W13_q), h = bf16(silu(g) * u)."""
+    I = W13_q.shape[0] // 2
+    xq, kx = quantize_blocks_e4m3(rows, 1)
+    gu = fp8_block_linear(xq, kx, W13_q, k13)
+    return bf16_round(silu(gu[:, :I]) * gu[:, I:])
+
+
+def swiglu_ffn_fp8_blocks(rows, W13_q, k13, W2_q, k2):
+    """One SwiGLU expert in the block-scaled FP8 form.
+
+    rows [m, H] (bf16 values); W13_q [2I, H], W2_q [H, I] on the e4m3 grid with
+    128 x 128 block exponents k13 [2I/128, H/128], k2 [H/128, I/128]. h (bf16)
+    is quantized per 1 x 128 block before GEMM2.
+    """
+    h = swiglu_h_fp8_blocks(rows, W13_q, k13)
+    hq, kh = quantize_blocks_e4m3(h, 1)
+    return fp8_block_linear(hq, kh, W2_q, k2)
+
+
+# ---------------------------------------------------------------------------
 # the whole layer
 # ---------------------------------------------------------------------------
 

@@ -76,7 +76,7 @@ DISPATCH_SWEEP_T = (1024, 4096, 16384, 65536)
 
 _SUB = {"x": 1, "Wr": 2, "bias": 3, "W13": 4, "W2": 5, "Ws13": 6, "Ws2": 7,
         "resample": 8, "zipf": 9, "sample": 10, "route": 11, "W13q": 12, "W2q": 13,
-        "Ws13q": 14, "Ws2q": 15}
+        "Ws13q": 14, "Ws2q": 15, "W13b": 16, "W2b": 17, "Ws13b": 18, "Ws2b": 19}
 
 
 def generator(seed: int, what: str, device, extra: int = 0) -> torch.Generator:
@@ -142,6 +142,45 @@ def fp8_expert_weights(wl: Workload, seed: int, device, experts=None):
         W13[n], s13[n] = e4m3_codes((2 * wl.I, wl.H), seed, "W13q", device, extra=e)
         W2[n], s2[n] = e4m3_codes((wl.H, wl.I), seed, "W2q", device, extra=e)
     return W13, s13, W2, s2
+
+
+# Block-scaled FP8 weights in stored form: the same e4m3 bytes, and one UE8M0
+# exponent byte per 128 x 128 block (scale 2^(byte - 127)), drawn from
+# {127 - 14, 127 - 13}: weights within about +-0.05 again.
+def e4m3_block_codes(shape, seed, what, device, extra=0):
+    """(uint8 e4m3 bytes of `shape` [rows, cols], uint8 exponents [rows/128, cols/128])."""
+    g = generator(seed, what, device, extra)
+    rows, cols = shape
+    mag = torch.randint(E4M3_CODE_LO, E4M3_CODE_HI + 1, shape, generator=g, device=device,
+                        dtype=torch.int32)
+    sgn = torch.randint(0, 2, shape, generator=g, device=device, dtype=torch.int32)
+    codes = (mag + 128 * sgn).to(torch.uint8)
+    exps = torch.randint(127 - 14, 127 - 12, (rows // 128, cols // 128), generator=g,
+                         device=device, dtype=torch.int32).to(torch.uint8)
+    return codes, exps
+
+
+def fp8_block_expert_weights(wl: Workload, seed: int, device, experts=None):
+    """Block-scaled FP8 routed-expert weights: W13 bytes [E, 2I, H] with exponents
+    [E, 2I/128, H/128], W2 bytes [E, H, I] with exponents [E, H/128, I/128]."""
+    es = range(wl.E) if experts is None else experts
+    W13 = torch.empty((len(es), 2 * wl.I, wl.H), dtype=torch.uint8, device=device)
+    W2 = torch.empty((len(es), wl.H, wl.I), dtype=torch.uint8, device=device)
+    k13 = torch.empty((len(es), 2 * wl.I // 128, wl.H // 128), dtype=torch.uint8, device=device)
+    k2 = torch.empty((len(es), wl.H // 128, wl.I // 128), dtype=torch.uint8, device=device)
+    for n, e in enumerate(es):
+        W13[n], k13[n] = e4m3_block_codes((2 * wl.I, wl.H), seed, "W13b", device, extra=e)
+        W2[n], k2[n] = e4m3_block_codes((wl.H, wl.I), seed, "W2b", device, extra=e)
+    return W13, k13, W2, k2
+
+
+def fp8_block_shared_weights(wl: Workload, seed: int, device):
+    """Block-scaled FP8 shared-expert weights (Ws13, its exponents, Ws2, its exponents)."""
+    if not wl.I_shared:
+        return None, None, None, None
+    Ws13, k13 = e4m3_block_codes((2 * wl.I_shared, wl.H), seed, "Ws13b", device)
+    Ws2, k2 = e4m3_block_codes((wl.H, wl.I_shared), seed, "Ws2b", device)
+    return Ws13, k13, Ws2, k2
 
 
 def fp8_shared_weights(wl: Workload, seed: int, device):

@@ -491,6 +491,148 @@ def test_e4m3_decode_every_code():
     assert len(np.unique(finite)) == 253                           # 254 finite codes, +-0 equal
 
 
+# ------------------------------------------- FP8 with block scales (UE8M0, 1x128 / 128x128)
+
+def test_block_exponent_by_hand():
+    # 448 * 2^k >= amax with k minimal: 448 fits at k = 0, 448.5 needs k = 1; 224 = 448 / 2
+    # fits at k = -1; 1.0 fits 448 / 256 = 1.75 but not 448 / 512 = 0.875 -> -8; 3.0 fits
+    # 3.5 = 448 / 128 but not 1.75 -> -7. An all-zero block takes k = 0; a block far below
+    # 448 * 2^-127 is clamped at -127.
+    amax = [448.0, 448.5, 224.0, 224.5, 1.0, 3.0, 0.0, 1e-40, 3.3e38]
+    assert O.block_exponent(amax).tolist() == [0, 1, -1, 0, -8, -7, 0, -127, 120]
+
+
+def test_block_exponent_is_the_smallest_fitting_power():
+    # brute force: scan k upward until amax <= 448 * 2^k (exact ldexp products)
+    rng = np.random.default_rng(11)
+    amax = np.ldexp(rng.uniform(1.0, 2.0, 400), rng.integers(-60, 60, 400))
+    amax[:8] = [448.0 * 2.0 ** e for e in (-50, -3, 0, 7, 20, 33, 45, 59)]  # exact boundaries
+    got = O.block_exponent(amax)
+    for a, k in zip(amax.tolist(), got.tolist()):
+        kk = -140
+        while a > math.ldexp(448.0, kk):
+            kk += 1
+        assert k == max(kk, -127)
+
+
+def test_quantize_blocks_by_hand():
+    # one activation row of two 128-blocks: block 0 has amax 3 -> k = -7, scaled by 2^7:
+    # 3 -> 384 (on the grid: [256, 448) steps 32), -1.5 -> -192 ([128, 256) steps 16),
+    # 0.1 -> 12.8 -> 13 ([8, 16) steps 1); block 1 is zero -> k = 0, codes 0.
+    row = np.zeros((1, 256))
+    row[0, :3] = [3.0, -1.5, 0.1]
+    q, k = O.quantize_blocks_e4m3(row, 1)
+    assert k.tolist() == [[-7, 0]]
+    assert q[0, :4].tolist() == [384.0, -192.0, 13.0, 0.0] and (q[0, 128:] == 0).all()
+    # a weight matrix of two 128-row blocks: |v| <= 0.05 -> 2^-13 (448 * 2^-13 = 0.0547,
+    # 448 * 2^-14 = 0.0273); a block of 448s -> k = 0 and codes 448
+    W = np.full((256, 128), 448.0)
+    W[:128] = np.linspace(-0.05, 0.05, 128 * 128).reshape(128, 128)
+    q, k = O.quantize_blocks_e4m3(W, 128)
+    assert k.tolist() == [[-13], [0]]
+    assert (q[128:] == 448.0).all() and np.abs(q[:128]).max() == O.e4m3_round(0.05 * 2 ** 13)
+
+
+def test_block_quantization_is_local_and_shifts_with_powers_of_two():
+    rng = np.random.default_rng(12)
+    a = O.bf16_round(rng.standard_normal((4, 384)))
+    q, k = O.quantize_blocks_e4m3(a, 1)
+    b = a.copy()
+    b[2, 128:256] *= 2.0 ** 5                 # one block scaled by a power of two
+    qb, kb = O.quantize_blocks_e4m3(b, 1)
+    np.testing.assert_array_equal(qb, q)       # same codes everywhere
+    dk = kb - k
+    assert dk[2, 1] == 5 and np.count_nonzero(dk) == 1
+    W = rng.standard_normal((256, 256)) * 0.02
+    q, k = O.quantize_blocks_e4m3(W, 128)
+    W2 = W.copy()
+    W2[0, 0] = 100.0                           # a new maximum in block (0, 0) only
+    q2, k2 = O.quantize_blocks_e4m3(W2, 128)
+    assert k2[0, 0] > k[0, 0] and (k2.ravel()[1:] == k.ravel()[1:]).all()
+    np.testing.assert_array_equal(q2[128:], q[128:])
+    np.testing.assert_array_equal(q2[:128, 128:], q[:128, 128:])
+
+
+def test_quantize_blocks_error_bound():
+    # dequantized values within half an e4m3 step: 2^-4 relative, 2^(k-10) absolute
+    rng = np.random.default_rng(13)
+    a = rng.standard_normal((20, 512)) * np.exp(rng.standard_normal((20, 1)) * 3)
+    q, k = O.quantize_blocks_e4m3(a, 1)
+    s = np.exp2(np.repeat(k, 128, axis=1).astype(np.float64))
+    assert (np.abs(q * s - a) <= np.abs(a) * 2.0 ** -4 + s * 2.0 ** -10).all()
+    assert (np.abs(q) <= 448).all()
+
+
+def test_fp8_block_linear_brute_force():
+    # pure-Python sums of q_a * 2^k_a(block) * q_w * 2^k_w(block) over every k
+    rng = np.random.default_rng(14)
+    m, n, K = 2, 256, 256
+    a_q = O.e4m3_round(rng.uniform(-448, 448, (m, K)))
+    W_q = O.e4m3_round(rng.uniform(-448, 448, (n, K)))
+    k_a = rng.integers(-20, 5, (m, K // 128))
+    k_w = rng.integers(-20, 5, (n // 128, K // 128))
+    y = O.fp8_block_linear(a_q, k_a, W_q, k_w)
+    al, Wl = a_q.tolist(), W_q.tolist()
+    for r in range(m):
+        for c in range(0, n, 37):
+            ref = 0.0
+            for kk in range(K):
+                ref += math.ldexp(al[r][kk], int(k_a[r][kk // 128])) * \
+                    math.ldexp(Wl[c][kk], int(k_w[c // 128][kk // 128]))
+            assert y[r, c] == pytest.approx(ref, rel=1e-12, abs=1e-300)
+
+
+def test_fp8_block_linear_reduces_to_row_scales():
+    # with one exponent per row (all its blocks alike) the block form is the per-row form
+    rng = np.random.default_rng(15)
+    a_q = O.e4m3_round(rng.uniform(-448, 448, (3, 256)))
+    W_q = O.e4m3_round(rng.uniform(-448, 448, (128, 256)))
+    k_a = np.repeat(rng.integers(-9, 3, (3, 1)), 2, axis=1)
+    k_w = np.full((1, 2), -11)
+    y = O.fp8_block_linear(a_q, k_a, W_q, k_w)
+    ref = O.fp8_linear(a_q, np.exp2(k_a[:, 0]).astype(np.float32), W_q,
+                       np.full(128, 2.0 ** -11, np.float32))
+    np.testing.assert_allclose(y, ref, rtol=1e-13)
+
+
+def test_swiglu_fp8_blocks_equals_dequantized_operands():
+    # the block form written out: quantize x per 1x128 block, dequantize both operands,
+    # two plain products, SwiGLU, bf16 h, h quantized per 1x128 block, third product
+    rng = np.random.default_rng(16)
+    H, Iw, m = 256, 128, 3
+    rows = O.bf16_round(rng.standard_normal((m, H)))
+    W13q, k13 = O.quantize_blocks_e4m3(rng.standard_normal((2 * Iw, H)) * 0.05, 128)
+    W2q, k2 = O.quantize_blocks_e4m3(rng.standard_normal((H, Iw)) * 0.05, 128)
+    y8 = O.swiglu_ffn_fp8_blocks(rows, W13q, k13, W2q, k2)
+    xq, kx = O.quantize_blocks_e4m3(rows, 1)
+    xd = xq * np.exp2(np.repeat(kx, 128, axis=1))
+    W13d = W13q * np.exp2(np.repeat(np.repeat(k13, 128, axis=0), 128, axis=1))
+    W2d = W2q * np.exp2(np.repeat(np.repeat(k2, 128, axis=0), 128, axis=1))
+    g, u = xd @ W13d[:Iw].T, xd @ W13d[Iw:].T
+    h = O.bf16_round(g / (1 + np.exp(-g)) * u)
+    hq, kh = O.quantize_blocks_e4m3(h, 1)
+    y = (hq * np.exp2(np.repeat(kh, 128, axis=1))) @ W2d.T
+    np.testing.assert_allclose(y8, y, rtol=1e-12, atol=1e-14)
+    # and close to the unquantized expert (e4m3 keeps ~2^-4 relative per operand)
+    ref = O.swiglu_ffn(rows, W13q * np.exp2(np.repeat(np.repeat(k13, 128, 0), 128, 1)), W2d)
+    assert np.abs(y8 - ref).max() < 0.15 * np.abs(ref).max()
+
+
+def test_layer_tokens_fp8_blocks_hook_matches_per_expert_calls():
+    rng = np.random.default_rng(17)
+    cfg = O.LayerConfig(T=5, H=128, E=3, k=2, I=128, gate=O.GATE_SOFTMAX)
+    x = O.bf16_round(rng.standard_normal((5, 128)))
+    Wr = rng.standard_normal((3, 128)).astype(np.float32) * 0.1
+    W13 = [O.quantize_blocks_e4m3(rng.standard_normal((256, 128)) * 0.05, 128) for _ in range(3)]
+    W2 = [O.quantize_blocks_e4m3(rng.standard_normal((128, 128)) * 0.05, 128) for _ in range(3)]
+    get = lambda e: (W13[e][0], W13[e][1], W2[e][0], W2[e][1])
+    out, idx, w = O.layer_forward_tokens(x, Wr, None, get, cfg, ffn=O.swiglu_ffn_fp8_blocks)
+    for t in range(5):
+        ref = sum(w[t, j] * O.swiglu_ffn_fp8_blocks(x[t:t + 1], *get(int(idx[t, j])))[0]
+                  for j in range(2))
+        np.testing.assert_allclose(out[t], ref, rtol=1e-13, atol=1e-15)
+
+
 def test_rms_normalize_by_hand_and_invariants():
     y = np.array([[3.0, 4.0], [0.0, 0.0], [1e3, -1e3]])
     r = O.rms_normalize(y, eps=0.0 + 1e-30)

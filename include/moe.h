@@ -97,6 +97,13 @@ typedef struct {
  *    in the epilogue, h (bf16, as in the bf16 form) is quantized per row the
  *    same way, and GEMM2 runs on e4m3 h and W2. The expert weights of
  *    moe_weights must then be e4m3 with their row scales (fp8 fields there).
+ *    2 = FP8 with block scales (DeepSeek-V3's fine-grained form): x and h are
+ *    quantized per 1 x 128 block (moe_quantize_fp8_blocks) and the weights
+ *    per 128 x 128 block (moe_quantize_fp8_weight_blocks), every scale a
+ *    power of two kept as a UE8M0 exponent byte, and the tensor cores apply
+ *    the scales inside the MMAs (tcgen05 kind::mxf8f6f4 block_scale, one
+ *    scale per 32 products; H, I and I_shared, multiples of 128 in every
+ *    valid configuration, hold whole blocks).
  *  fuse_combine 0 = GEMM2 writes y_perm (fp32) and a combine kernel sums each
  *    token's k rows in slot order (deterministic); 1 = the gate-weighted
  *    combine is fused into GEMM2's epilogue: every GEMM2 (and the shared
@@ -141,7 +148,12 @@ enum {
  * (same shapes, row-major, packed = 0), as written by moe_quantize_fp8 over
  * their rows, and the *_scale arrays hold the fp32 scale of every row:
  * W13_scale [E*2I], W2_scale [E*H], Ws13_scale [2*I_shared], Ws2_scale [H]
- * (the shared ones NULL iff I_shared = 0). With fp8 = 0 the scales are unused. */
+ * (the shared ones NULL iff I_shared = 0). With fp8 = 2 the matrices hold
+ * e4m3 bytes as written by moe_quantize_fp8_weight_blocks and the *_scale
+ * arrays hold uint8 UE8M0 exponents (scale 2^(byte - 127)) of their 128 x 128
+ * blocks, row-major [rows / 128][cols / 128]: W13_scale [E*2I/128][H/128],
+ * W2_scale [E*H/128][I/128], Ws13_scale [2*I_shared/128][H/128], Ws2_scale
+ * [H/128][I_shared/128]. With fp8 = 0 the scales are unused. */
 typedef struct {
   const float* Wr;
   const float* bias;
@@ -150,10 +162,10 @@ typedef struct {
   const void* Ws13;
   const void* Ws2;
   int32_t packed;
-  const float* W13_scale;
-  const float* W2_scale;
-  const float* Ws13_scale;
-  const float* Ws2_scale;
+  const void* W13_scale; /* fp8 = 1: const float*; fp8 = 2: const uint8_t* */
+  const void* W2_scale;
+  const void* Ws13_scale;
+  const void* Ws2_scale;
 } moe_weights;
 
 /* Optional outputs of moe_layer_forward; NULL fields are skipped.
@@ -328,6 +340,53 @@ moe_status moe_expert_ffn_fp8(int32_t rows, int32_t H, int32_t I, int32_t n_expe
                               const uint8_t* W13_q, const float* W13_scale, const uint8_t* W2_q,
                               const float* W2_scale, float* y_perm, void* ws, size_t ws_bytes,
                               void* stream);
+
+/*
+ * FP8 quantization with block scales, for activation rows: each 1 x 128 block
+ * of in [rows, K] bf16 gets the exponent k = the smallest integer with
+ * amax <= 448 * 2^k (k = 0 for an all-zero block, clamped to [-127, 127]),
+ * stored as the UE8M0 byte sf[(c / 128) * sf_ld + r] = k + 127, and its
+ * values out[r][c] = e4m3(in[r][c] * 2^-k) (exact scaling, then round to
+ * nearest even, saturating at +-448). K a multiple of 128, at most 65536;
+ * sf_ld >= rows; in and out 16-byte aligned and not overlapping; all written
+ * buffers caller-allocated. Used on token rows and on h inside
+ * moe_layer_forward (fp8 = 2).
+ */
+moe_status moe_quantize_fp8_blocks(int64_t rows, int32_t K, const uint16_t* in, uint8_t* out,
+                                   uint8_t* sf, int64_t sf_ld, void* stream);
+
+/*
+ * The same in 128 x 128 blocks, for weight matrices viewed as [rows, K]:
+ * sf[(r / 128) * (K / 128) + c / 128] = k + 127 of block (r / 128, c / 128).
+ * rows a multiple of 128 (at most 128 * 65535), K a multiple of 128 (at most
+ * 65536). A load-time step (W13 as rows = E*2I, K = H; W2 as rows = E*H, K = I).
+ */
+moe_status moe_quantize_fp8_weight_blocks(int64_t rows, int32_t K, const uint16_t* in,
+                                          uint8_t* out, uint8_t* sf, void* stream);
+
+/* Workspace bytes of moe_expert_ffn_fp8_blocks: h [rows, I] bf16, its e4m3
+ * copy [rows, I] and its block exponents [I/128][rows], each 256-byte aligned. */
+size_t moe_expert_ffn_fp8_blocks_workspace_size(int32_t rows, int32_t I);
+
+/*
+ * Grouped expert FFN with block-scaled FP8 operands (moe_expert_ffn's segments
+ * and shapes). With 2^kx, 2^kw the scales of the blocks a product's terms fall in:
+ *   g|u[r][j] = sum_c x_q[r][c] 2^kx(r, c/128) * W13_q[e][j][c] 2^kw13(e, j/128, c/128),
+ *   h[r] = bf16(silu(g) * u), h quantized by moe_quantize_fp8_blocks,
+ *   y_perm[r][c] = sum_i h_q[r][i] 2^kh(r, i/128) * W2_q[e][c][i] 2^kw2(e, c/128, i/128),
+ * fp32 accumulation on the tensor cores. kx(r, b) is x_sf[b * x_sf_ld + t] with
+ * t = x_scale_idx[r] when given (x_q rows are copies of token rows; values in
+ * [0, x_sf_ld)), else r (then x_sf_ld >= rows).
+ * W13_sf [n_experts*2I/128][H/128], W2_sf [n_experts*H/128][I/128] as in
+ * moe_weights (fp8 = 2). H and I multiples of 128. ws:
+ * moe_expert_ffn_fp8_blocks_workspace_size(rows, I) bytes, 256-byte aligned.
+ */
+moe_status moe_expert_ffn_fp8_blocks(int32_t rows, int32_t H, int32_t I, int32_t n_experts,
+                                     const uint8_t* x_q, const uint8_t* x_sf, int64_t x_sf_ld,
+                                     const int32_t* x_scale_idx, const int32_t* offsets,
+                                     const uint8_t* W13_q, const uint8_t* W13_sf,
+                                     const uint8_t* W2_q, const uint8_t* W2_sf, float* y_perm,
+                                     void* ws, size_t ws_bytes, void* stream);
 
 /*
  * Combine: the single-GPU form of the paper's reverse AlltoAll combine.

@@ -32,7 +32,9 @@ EXPORTS = ("moe_status_string", "moe_validate_config", "moe_workspace_size",
            "moe_testing_expert_ffn_stall", "moe_pack_weights", "moe_quantize_fp8",
            "moe_expert_ffn_fp8", "moe_expert_ffn_fp8_workspace_size", "moe_stack_workspace_size",
            "moe_stack_forward", "moe_rms_norm", "moe_graph_create_stack", "moe_graph_launch",
-           "moe_graph_kernel_count", "moe_graph_destroy")
+           "moe_graph_kernel_count", "moe_graph_destroy", "moe_quantize_fp8_blocks",
+           "moe_quantize_fp8_weight_blocks", "moe_expert_ffn_fp8_blocks",
+           "moe_expert_ffn_fp8_blocks_workspace_size")
 MOE_DISPATCH_NOALLOC_MAX_ENTRIES = 131072
 
 
@@ -103,6 +105,11 @@ def load(path: str = LIB_PATH) -> ctypes.CDLL:
         "moe_quantize_fp8": (S, [ctypes.c_int64, I32, P, P, P, P]),
         "moe_expert_ffn_fp8_workspace_size": (SZ, [I32, I32]),
         "moe_expert_ffn_fp8": (S, [I32, I32, I32, I32, P, P, P, P, P, P, P, P, P, P, SZ, P]),
+        "moe_quantize_fp8_blocks": (S, [ctypes.c_int64, I32, P, P, P, ctypes.c_int64, P]),
+        "moe_quantize_fp8_weight_blocks": (S, [ctypes.c_int64, I32, P, P, P, P]),
+        "moe_expert_ffn_fp8_blocks_workspace_size": (SZ, [I32, I32]),
+        "moe_expert_ffn_fp8_blocks": (S, [I32, I32, I32, I32, P, P, ctypes.c_int64, P, P, P, P,
+                                          P, P, P, P, SZ, P]),
         "moe_combine": (S, [cfgp, P, P, P, P, P, I32, P]),
         "moe_testing_expert_ffn_stall": (S, [I32, I32, I32, I32, P, P, P, P, P, P, SZ,
                                              ctypes.c_int64, ctypes.c_int64, P]),
@@ -268,6 +275,60 @@ def moe_expert_ffn_fp8(rows, H, I, n_experts, x_q, x_scale, x_scale_idx, offsets
                                      _ptr(W13_scale), _ptr(W2_q), _ptr(W2_scale), _ptr(y_perm),
                                      _ptr(ws), nb, _stream(stream)),
            "moe_expert_ffn_fp8")
+
+
+def moe_quantize_fp8_blocks(x, out, sf, sf_ld, stream=None) -> None:
+    """e4m3 quantization of a bf16 tensor viewed as [rows, K] in 1 x 128 blocks;
+    UE8M0 exponents to sf[(c / 128) * sf_ld + r]."""
+    K = x.shape[-1]
+    rows = x.numel() // K
+    _check(load().moe_quantize_fp8_blocks(rows, K, _ptr(x), _ptr(out), _ptr(sf), int(sf_ld),
+                                          _stream(stream)), "moe_quantize_fp8_blocks")
+
+
+def quantize_fp8_blocks(x, stream=None):
+    """(e4m3 bytes as uint8 of x's shape, uint8 exponents [K / 128, rows]) of a bf16 tensor."""
+    import torch
+    K = x.shape[-1]
+    rows = x.numel() // K
+    q = torch.empty(x.shape, dtype=torch.uint8, device=x.device)
+    sf = torch.empty((K // 128, rows), dtype=torch.uint8, device=x.device)
+    moe_quantize_fp8_blocks(x, q, sf, rows, stream)
+    return q, sf
+
+
+def moe_quantize_fp8_weight_blocks(W, out, sf, stream=None) -> None:
+    """e4m3 quantization of a bf16 tensor viewed as [rows, K] in 128 x 128 blocks."""
+    K = W.shape[-1]
+    rows = W.numel() // K
+    _check(load().moe_quantize_fp8_weight_blocks(rows, K, _ptr(W), _ptr(out), _ptr(sf),
+                                                 _stream(stream)),
+           "moe_quantize_fp8_weight_blocks")
+
+
+def quantize_fp8_weight_blocks(W, stream=None):
+    """(e4m3 bytes as uint8 of W's shape, uint8 exponents [rows / 128, K / 128])."""
+    import torch
+    K = W.shape[-1]
+    rows = W.numel() // K
+    q = torch.empty(W.shape, dtype=torch.uint8, device=W.device)
+    sf = torch.empty((rows // 128, K // 128), dtype=torch.uint8, device=W.device)
+    moe_quantize_fp8_weight_blocks(W, q, sf, stream)
+    return q, sf
+
+
+def moe_expert_ffn_fp8_blocks_workspace_size(rows, I) -> int:
+    return load().moe_expert_ffn_fp8_blocks_workspace_size(rows, I)
+
+
+def moe_expert_ffn_fp8_blocks(rows, H, I, n_experts, x_q, x_sf, x_sf_ld, x_scale_idx, offsets,
+                              W13_q, W13_sf, W2_q, W2_sf, y_perm, ws, stream=None) -> None:
+    nb = 0 if ws is None else ws.numel() * ws.element_size()
+    _check(load().moe_expert_ffn_fp8_blocks(rows, H, I, n_experts, _ptr(x_q), _ptr(x_sf),
+                                            int(x_sf_ld), _ptr(x_scale_idx), _ptr(offsets),
+                                            _ptr(W13_q), _ptr(W13_sf), _ptr(W2_q), _ptr(W2_sf),
+                                            _ptr(y_perm), _ptr(ws), nb, _stream(stream)),
+           "moe_expert_ffn_fp8_blocks")
 
 
 def moe_pack_weights(W, W_packed, stream=None) -> None:

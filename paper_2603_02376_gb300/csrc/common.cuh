@@ -103,6 +103,17 @@ struct FfnGroup {
   const float* W2_scale;
   uint8_t* hq;
   float* hs;
+  // Block-scaled FP8 (fp8 and fp8_block): UE8M0 exponents of x's 1 x 128
+  // blocks (x_sf[kb * x_sf_ld + token], the token through x_scale_idx as
+  // above) and of the 128 x 128 blocks of W13 and W2 ([rows / 128][K / 128]);
+  // hsf receives those of h's 1 x 128 blocks (hsf[kb * h_sf_ld + row]).
+  bool fp8_block;
+  const uint8_t* x_sf;
+  long x_sf_ld;
+  const uint8_t* W13_sf;
+  const uint8_t* W2_sf;
+  uint8_t* hsf;
+  long h_sf_ld;
   // Combine fused into GEMM2 (comb_out non-null): instead of y, GEMM2 adds
   // comb_w[r] * y[r] into comb_out[comb_tok[r]] with fp32 reductions (comb_tok
   // null = row r is token r; comb_w null = weight 1).
@@ -134,6 +145,15 @@ moe_status launch_expert_ffn(int rows, int H, int I, int n_experts, int e_begin,
 // e4m3 row quantization of a bf16 matrix [rows, K] (K % 8 == 0).
 moe_status launch_quantize_rows(const uint16_t* in, long rows, int K, uint8_t* out, float* scale,
                                 cudaStream_t s);
+
+// e4m3 quantization of a bf16 matrix [rows, K] in 1 x 128 blocks (K % 128 == 0):
+// k = the smallest exponent with amax <= 448 * 2^k (0 for a zero block, within
+// [-127, 127]); out[r][c] = e4m3(in[r][c] * 2^-k); sf[(c / 128) * sf_ld + r] = k + 127.
+moe_status launch_quantize_blocks(const uint16_t* in, long rows, int K, uint8_t* out, uint8_t* sf,
+                                  long sf_ld, cudaStream_t s);
+// The same in 128 x 128 blocks (rows % 128 == 0): sf[(r / 128) * (K / 128) + c / 128].
+moe_status launch_quantize_weight_blocks(const uint16_t* in, long rows, int K, uint8_t* out,
+                                         uint8_t* sf, cudaStream_t s);
 
 // Tile-packed copy of a bf16 weight matrix [rows, K] (rows % 128 == 0, K % 64 == 0).
 moe_status launch_pack_weights(const uint16_t* W, uint16_t* Wp, long rows, int K, cudaStream_t s);

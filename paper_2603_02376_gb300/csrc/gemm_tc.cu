@@ -74,24 +74,43 @@ constexpr int MODE_PLAIN2 = 2;  // two adjacent 128-feature tiles sharing one to
 constexpr int MODE_SPLIT3 = 3;  // three bf16 planes of one fp32 weight tile, summed into one
                                 // accumulator (an fp32 x bf16 product on bf16 tensor cores)
 
-template <int MODE, int NMAX>
+// Operand precision of a launch: bf16; e4m3 with fp32 row scales applied in
+// the epilogue; e4m3 with UE8M0 block scales (1 x 128 per token row, 128 x 128
+// per weight block) applied by the tensor core (kind::mxf8f6f4 block_scale).
+constexpr int Q_BF16 = 0;
+constexpr int Q_ROW = 1;
+constexpr int Q_BLOCK = 2;
+
+template <int MODE, int NMAX, bool MX = false>
 struct Tile {
   static constexpr int NA = MODE == MODE_PLAIN ? 1 : MODE == MODE_SPLIT3 ? 3 : 2;  // A tiles
   static constexpr bool TWO_ACC = MODE == MODE_SWIGLU || MODE == MODE_PLAIN2;  // tile i -> acc i
   static constexpr int FEAT = MODE == MODE_PLAIN2 ? 2 * BM : BM;  // output features per unit
   static constexpr int A_BYTES = BM * BK * 2;  // 16 KiB
   static constexpr int B_BYTES = NMAX * BK * 2;
-  static constexpr int STAGE_BYTES = NA * A_BYTES + B_BYTES;
+  // Block scales (MX): per stage one 512-byte scale image per A tile and per
+  // 128 token rows, in the order tcgen05.cp 32x128b.warpx4 expects (entry x at
+  // byte 16 * (x % 32) + 4 * (x / 32 % 4)), after the operand tiles.
+  static constexpr int SF_CB = MX ? (NMAX + 127) / 128 : 0;  // token-scale images
+  static constexpr int SF_OFF = NA * A_BYTES + B_BYTES;
+  static constexpr int SF_BYTES = MX ? ((NA + SF_CB) * 512 + 1023) / 1024 * 1024 : 0;
+  static constexpr int STAGE_BYTES = NA * A_BYTES + B_BYTES + SF_BYTES;
   // ~217 KiB of stages: with the control block, the expert tables (<= 8 KiB)
   // and the 1 KiB alignment slack this stays under 227 KiB per CTA.
   static constexpr int STAGES_RAW = (217 * 1024) / STAGE_BYTES;
   static constexpr int STAGES = STAGES_RAW > 12 ? 12 : STAGES_RAW;
   static constexpr int ACC_COLS = TWO_ACC ? 2 * NMAX : NMAX;  // one accumulator (gate | up)
-  static constexpr int ACC_STAGES = 2 * ACC_COLS <= 512 ? 2 : 1;  // double-buffer when it fits
-  static constexpr int TMEM_COLS = pow2ceil(ACC_STAGES * ACC_COLS);
+  // MX: each stage's scales live in TMEM columns of their own (4 per image)
+  // until the stage's MMAs complete
+  static constexpr int SF_COLS = MX ? 4 * (NA + SF_CB) : 0;
+  static constexpr int ACC_STAGES =
+      2 * ACC_COLS + STAGES * SF_COLS <= 512 ? 2 : 1;  // double-buffer when it fits
+  static constexpr int SF_COL0 = ACC_STAGES * ACC_COLS;
+  static constexpr int TMEM_COLS = pow2ceil(SF_COL0 + STAGES * SF_COLS);
   static_assert(STAGES >= 2, "pipeline too shallow");
   static_assert(NMAX % 16 == 0 && NMAX >= 16 && NMAX <= 256, "MMA N range for M = 128");
   static_assert(TMEM_COLS <= 512, "TMEM holds 512 columns");
+  static_assert(SF_OFF % 1024 == 0 && STAGE_BYTES % 1024 == 0, "stage alignment");
 };
 
 struct Ctrl {
@@ -227,6 +246,43 @@ __device__ __forceinline__ void mma_e4m3(uint32_t d_tmem, uint64_t a, uint64_t b
       : "memory");
 }
 
+// Instruction descriptor, kind::mxf8f6f4 with e4m3 A and B: as above without
+// the accumulator-format field (bits 4-5 select the byte of each B scale word
+// instead, 0 here, like bits 29-30 for A) and with UE8M0 scales (bit 23).
+__device__ __forceinline__ uint32_t idesc_mx(int n) {
+  return ((uint32_t)(n >> 3) << 17) | (1u << 23) | ((uint32_t)(BM >> 4) << 24);
+}
+
+// One block-scaled MMA of K = 32 e4m3 values: each A row and each B row
+// carries one UE8M0 scale 2^(s - 127) for these 32 products, read from TMEM:
+// A row i at lane i, column sfa + i / 32; B row j at column sfb + j / 32, lane
+// j % 32 of every 32-lane quarter (byte 0 of each 32-bit word).
+__device__ __forceinline__ void mma_mx(uint32_t d_tmem, uint64_t a, uint64_t b, uint32_t idesc,
+                                       uint32_t sfa, uint32_t sfb, uint32_t accumulate) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "setp.ne.b32 p, %6, 0;\n\t"
+      "tcgen05.mma.cta_group::1.kind::mxf8f6f4.block_scale.scale_vec::1X [%0], %1, %2, %3, [%4], "
+      "[%5], p;\n\t}" ::"r"(d_tmem),
+      "l"(a), "l"(b), "r"(idesc), "r"(sfa), "r"(sfb), "r"(accumulate)
+      : "memory");
+}
+
+// Shared-memory descriptor of a 512-byte scale image for tcgen05.cp: no
+// swizzle, 8-row core matrices of 16-byte rows 128 bytes apart.
+__device__ __forceinline__ uint64_t sdesc_sf(uint32_t saddr) {
+  return (uint64_t)((saddr & 0x3FFFFu) >> 4) | ((uint64_t)(128 >> 4) << 32) | (1ull << 46);
+}
+
+// 32 rows x 16 bytes of shared memory -> 4 TMEM columns, row r to lane r of
+// each of the four 32-lane quarters. Ordered before the MMAs this thread
+// issues next.
+__device__ __forceinline__ void sf_copy(uint32_t taddr, uint32_t saddr) {
+  asm volatile("tcgen05.cp.cta_group::1.32x128b.warpx4 [%0], %1;" ::"r"(taddr),
+               "l"(sdesc_sf(saddr))
+               : "memory");
+}
+
 __device__ __forceinline__ void mma_bf16(uint32_t d_tmem, uint64_t a, uint64_t b, uint32_t idesc,
                                          uint32_t accumulate);
 
@@ -297,6 +353,15 @@ struct GemmArgs {
   const float* b_scale0;
   const float* b_scale1;
   const int32_t* b_scale_idx0;
+  // Block-scaled FP8 only: UE8M0 exponents of the 128 x 128 weight blocks
+  // ([weight rows / 128][K / 128], absolute weight rows) and of the 1 x 128
+  // activation blocks (b_sf[kb * b_sf_ld + row], the row through b_scale_idx0
+  // for group 0 when given)
+  const uint8_t* a_sf0;
+  const uint8_t* a_sf1;
+  const uint8_t* b_sf0;
+  const uint8_t* b_sf1;
+  long b_sf_ld0, b_sf_ld1;
   // PLAIN / PLAIN2 only: the combine fused into the epilogue. Non-null comb_out*
   // replaces the y store of that group by comb_out[tok][f] += w * y (fp32
   // reductions), tok = comb_tok0[row] and w = comb_w0[row] for group 0 (null:
@@ -369,7 +434,7 @@ __device__ __forceinline__ Unit decode_unit(int u, const int* tile_off, const in
 
 // ------------------------------------------------------------------ kernel
 
-template <int MODE, int NMAX, bool F8, bool PK>
+template <int MODE, int NMAX, int Q, bool PK>
 __global__ void __launch_bounds__(NUM_THREADS, 1)
     grouped_gemm_kernel(const __grid_constant__ CUtensorMap tmA0,
                         const __grid_constant__ CUtensorMap tmB0,
@@ -377,7 +442,9 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
                         const __grid_constant__ CUtensorMap tmB1,
                         const __grid_constant__ CUtensorMap tmB0big,
                         const __grid_constant__ CUtensorMap tmB1big, const GemmArgs a) {
-  using TL = Tile<MODE, NMAX>;
+  constexpr bool F8 = Q != Q_BF16;  // e4m3 operands
+  constexpr bool MX = Q == Q_BLOCK;  // ... with block scales applied by the MMA
+  using TL = Tile<MODE, NMAX, MX>;
   constexpr bool SWIGLU = MODE == MODE_SWIGLU;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
@@ -498,10 +565,53 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
           const int r = (lane + 32 * h) * 4 + j;
           gr[h][j] = gather && r < n_pad ? a.gather0[U.row0 + min(r, U.m - 1)] : 0;
         }
+      // MX: lane l fetches the block scales of token columns j = 32 g + l of the
+      // tile (the activation row of column j: sf_row[g]; -1 past the valid rows)
+      constexpr int NG = MX ? (NMAX + 31) / 32 : 1;
+      int sf_row[NG];
+      if constexpr (MX) {
+        const int32_t* bidx = U.grp ? nullptr : a.b_scale_idx0;
+#pragma unroll
+        for (int g = 0; g < NG; ++g) {
+          const int j = 32 * g + lane;
+          sf_row[g] = j < U.m ? (bidx ? bidx[U.row0 + j] : U.row0 + j) : -1;
+        }
+      }
       for (int kb = U.kb0; kb < U.kb1; ++kb) {
         const uint32_t full = smem_u32(&ctrl->full[stage]);
         const uint32_t sa = smem_u32(smem + stage * TL::STAGE_BYTES);
         const uint32_t sb = sa + TL::NA * TL::A_BYTES;
+        auto issue = [&]() {  // lane 0: arm the stage barrier, load the tiles
+          mbar_arrive_expect_tx(full, bytes);
+#pragma unroll
+          for (int t = 0; t < TL::NA; ++t) {
+            const int r = wrow + t * a.up_off;
+            const uint16_t* ap = U.grp ? a.a1_packed : a.a0_packed;
+            if (PK)  // tile (r / 128, kb): 8192 bf16 per tile
+              bulk_load_tile(sa + t * TL::A_BYTES,
+                             ap + ((size_t)(r / BM) * kblocks + kb) * (BM * BK), full);
+            else
+              tma_load_2d(sa + t * TL::A_BYTES, mA, kb * KE, r, full);
+          }
+          if (!gather) {
+            for (int i = 0; i < n_big; ++i)
+              tma_load_2d(sb + i * (B_BIG * BK * 2), mBbig, kb * KE, U.row0 + i * B_BIG, full);
+            for (int i = n_big * (B_BIG / B_BOX); i < n_pad / B_BOX; ++i)
+              tma_load_2d(sb + i * (B_BOX * BK * 2), mB, kb * KE, U.row0 + i * B_BOX, full);
+          }
+        };
+        // MX: this k-block's scales, loaded before the wait for the slot
+        uint32_t sfa[TL::NA], sfb[NG];
+        if constexpr (MX) {
+          const uint8_t* asf = U.grp ? a.a_sf1 : a.a_sf0;
+          const uint8_t* bsf = U.grp ? a.b_sf1 : a.b_sf0;
+          const size_t boff = (size_t)kb * (U.grp ? a.b_sf_ld1 : a.b_sf_ld0);
+#pragma unroll
+          for (int t = 0; t < TL::NA; ++t)
+            sfa[t] = asf[(size_t)((wrow + t * a.up_off) / BM) * kblocks + kb];
+#pragma unroll
+          for (int g = 0; g < NG; ++g) sfb[g] = sf_row[g] >= 0 ? bsf[boff + sf_row[g]] : 127u;
+        }
         int got = 1;
         if (lane == 0) {
           got = wait_bounded(smem_u32(&ctrl->empty[stage]), phase ^ 1, abort_flag, err,
@@ -509,30 +619,39 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
                     ? 1
                     : 0;
           if (got && blockIdx.x == 0 && fills == a.stall_fill) got = 2;  // skip this fill
-          if (got == 1) {
-            mbar_arrive_expect_tx(full, bytes);
-#pragma unroll
-            for (int t = 0; t < TL::NA; ++t) {
-              const int r = wrow + t * a.up_off;
-              const uint16_t* ap = U.grp ? a.a1_packed : a.a0_packed;
-              if (PK)  // tile (r / 128, kb): 8192 bf16 per tile
-                bulk_load_tile(sa + t * TL::A_BYTES,
-                               ap + ((size_t)(r / BM) * kblocks + kb) * (BM * BK), full);
-              else
-                tma_load_2d(sa + t * TL::A_BYTES, mA, kb * KE, r, full);
-            }
-            if (!gather) {
-              for (int i = 0; i < n_big; ++i)
-                tma_load_2d(sb + i * (B_BIG * BK * 2), mBbig, kb * KE, U.row0 + i * B_BIG, full);
-              for (int i = n_big * (B_BIG / B_BOX); i < n_pad / B_BOX; ++i)
-                tma_load_2d(sb + i * (B_BOX * BK * 2), mB, kb * KE, U.row0 + i * B_BOX, full);
-            }
+          if constexpr (!MX) {
+            if (got == 1) issue();
           }
         }
         got = __shfl_sync(0xffffffffu, got, 0);
         if (!got) {
           ok = false;
           break;
+        }
+        if constexpr (MX) {
+          // scale images of the stage (every byte of a word holds the scale), made
+          // visible to the tensor core's reads before lane 0 arms the barrier
+          if (got == 1) {
+            uint8_t* sf = smem + stage * TL::STAGE_BYTES + TL::SF_OFF;
+#pragma unroll
+            for (int t = 0; t < TL::NA; ++t) {
+              const uint32_t v = sfa[t] * 0x01010101u;
+              *reinterpret_cast<uint4*>(sf + t * 512 + lane * 16) = make_uint4(v, v, v, v);
+            }
+#pragma unroll
+            for (int c = 0; c < TL::SF_CB; ++c) {
+              uint32_t w[4];
+#pragma unroll
+              for (int q = 0; q < 4; ++q)
+                w[q] = (4 * c + q < NG ? sfb[min(4 * c + q, NG - 1)] : 127u) * 0x01010101u;
+              *reinterpret_cast<uint4*>(sf + (TL::NA + c) * 512 + lane * 16) =
+                  make_uint4(w[0], w[1], w[2], w[3]);
+            }
+            asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+          }
+          __syncwarp();
+          if (lane == 0 && got == 1) issue();
+          __syncwarp();
         }
         if (gather && got == 1) {
 #pragma unroll
@@ -573,7 +692,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       for (int u = blockIdx.x; u < total_units && ok; u += gridDim.x, ++j) {
         const Unit U = decode_unit<NMAX>(u, tile_off, row_off, a, units1, kblocks);
         const int n_pad = (U.m + 15) & ~15;
-        const uint32_t idesc = F8 ? idesc_e4m3(n_pad) : idesc_bf16(n_pad);
+        const uint32_t idesc = MX ? idesc_mx(n_pad) : F8 ? idesc_e4m3(n_pad) : idesc_bf16(n_pad);
         const int as = j % TL::ACC_STAGES;
         const uint32_t acc_par = (uint32_t)((j / TL::ACC_STAGES) & 1);
         if (!wait_bounded(smem_u32(&ctrl->acc_empty[as]), acc_par ^ 1, abort_flag, err,
@@ -592,16 +711,39 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
           tc_fence_after();
           const uint32_t sa = smem_u32(smem + stage * TL::STAGE_BYTES);
           const uint32_t sb = sa + TL::NA * TL::A_BYTES;
+          if constexpr (MX) {
+            // the stage's scale images -> its TMEM scale columns: A tile t at
+            // sfc + 4 t, token rows 128 c .. at sfc + 4 (NA + c); the copies run
+            // before the MMAs below (same issuing thread), and the stage's commit
+            // covers them before the producer rewrites the images
+            const uint32_t sfs = sa + TL::SF_OFF;
+            const uint32_t sfc = tmem_base + (uint32_t)(TL::SF_COL0 + stage * TL::SF_COLS);
 #pragma unroll
-          for (int k = 0; k < BK / UMMA_K; ++k) {
-            const uint32_t acc = (kb > U.kb0 || k > 0) ? 1u : 0u;
-            const uint64_t bdesc = sdesc(sb + k * UMMA_K * 2);
-            mma_op<F8>(d, sdesc(sa + k * UMMA_K * 2), bdesc, idesc, acc);
-            if (TL::TWO_ACC)
-              mma_op<F8>(d + NMAX, sdesc(sa + TL::A_BYTES + k * UMMA_K * 2), bdesc, idesc, acc);
-            if (MODE == MODE_SPLIT3) {  // the lower planes add into the same accumulator
-              mma_op<F8>(d, sdesc(sa + TL::A_BYTES + k * UMMA_K * 2), bdesc, idesc, 1u);
-              mma_op<F8>(d, sdesc(sa + 2 * TL::A_BYTES + k * UMMA_K * 2), bdesc, idesc, 1u);
+            for (int t = 0; t < TL::NA; ++t) sf_copy(sfc + 4 * t, sfs + t * 512);
+            for (int c = 0; c < (n_pad + 127) / 128; ++c)
+              sf_copy(sfc + 4 * (TL::NA + c), sfs + (TL::NA + c) * 512);
+            const uint32_t sfb = sfc + 4 * TL::NA;
+#pragma unroll
+            for (int k = 0; k < BK / UMMA_K; ++k) {
+              const uint32_t acc = (kb > U.kb0 || k > 0) ? 1u : 0u;
+              const uint64_t bdesc = sdesc(sb + k * UMMA_K * 2);
+              mma_mx(d, sdesc(sa + k * UMMA_K * 2), bdesc, idesc, sfc, sfb, acc);
+              if (TL::TWO_ACC)
+                mma_mx(d + NMAX, sdesc(sa + TL::A_BYTES + k * UMMA_K * 2), bdesc, idesc, sfc + 4,
+                       sfb, acc);
+            }
+          } else {
+#pragma unroll
+            for (int k = 0; k < BK / UMMA_K; ++k) {
+              const uint32_t acc = (kb > U.kb0 || k > 0) ? 1u : 0u;
+              const uint64_t bdesc = sdesc(sb + k * UMMA_K * 2);
+              mma_op<F8>(d, sdesc(sa + k * UMMA_K * 2), bdesc, idesc, acc);
+              if (TL::TWO_ACC)
+                mma_op<F8>(d + NMAX, sdesc(sa + TL::A_BYTES + k * UMMA_K * 2), bdesc, idesc, acc);
+              if (MODE == MODE_SPLIT3) {  // the lower planes add into the same accumulator
+                mma_op<F8>(d, sdesc(sa + TL::A_BYTES + k * UMMA_K * 2), bdesc, idesc, 1u);
+                mma_op<F8>(d, sdesc(sa + 2 * TL::A_BYTES + k * UMMA_K * 2), bdesc, idesc, 1u);
+              }
             }
           }
           issued = true;
@@ -645,7 +787,8 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       float sa0 = 1.f, sa1 = 1.f;
       const float* bsc = nullptr;
       const int32_t* bidx = nullptr;
-      if (F8) {
+      constexpr bool RS = F8 && !MX;  // row scales applied here
+      if (RS) {
         const float* asc = U.grp ? a.a_scale1 : a.a_scale0;
         const int wr = (U.grp ? 0 : (a.e_begin + U.e) * a.w_rows0) + f;
         sa0 = asc[wr];
@@ -672,7 +815,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
           const int br = U.row0 + (cv ? mc : 0);
           float sb_l = 1.f, w_l = 1.f;
           int t_l = br;
-          if (F8 && cv) sb_l = bsc[bidx ? bidx[br] : br];
+          if (RS && cv) sb_l = bsc[bidx ? bidx[br] : br];
           if (CB && cv) {
             if (cw) w_l = cw[br];
             if (ctok) t_l = ctok[br];
@@ -685,7 +828,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
             tmem_wait_ld();
 #pragma unroll
             for (int i = 0; i < 16; ++i) {
-              const float sb = F8 ? __shfl_sync(0xffffffffu, sb_l, i) : 1.f;
+              const float sb = RS ? __shfl_sync(0xffffffffu, sb_l, i) : 1.f;
               if (c0 + i < U.m) {
                 const float gv = __uint_as_float(g[i]) * (sa0 * sb);
                 const float uv = __uint_as_float(v[i]) * (sa1 * sb);
@@ -703,7 +846,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
             tmem_wait_ld();
 #pragma unroll
             for (int i = 0; i < 16; ++i) {
-              const float sb = F8 ? __shfl_sync(0xffffffffu, sb_l, i) : 1.f;
+              const float sb = RS ? __shfl_sync(0xffffffffu, sb_l, i) : 1.f;
               const float wv = CB ? __shfl_sync(0xffffffffu, w_l, i) : 1.f;
               const int tv = CB ? __shfl_sync(0xffffffffu, t_l, i) : 0;
               if (c0 + i < U.m) {
@@ -724,7 +867,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
             tmem_wait_ld();
 #pragma unroll
             for (int i = 0; i < 16; ++i) {
-              const float sb = F8 ? __shfl_sync(0xffffffffu, sb_l, i) : 1.f;
+              const float sb = RS ? __shfl_sync(0xffffffffu, sb_l, i) : 1.f;
               const float wv = CB ? __shfl_sync(0xffffffffu, w_l, i) : 1.f;
               const int tv = CB ? __shfl_sync(0xffffffffu, t_l, i) : 0;
               if (c0 + i < U.m) {
@@ -798,23 +941,23 @@ bool make_map(CUtensorMap* m, const void* ptr, uint64_t inner, uint64_t outer, u
 uint64_t g_wait_limit_ns = WAIT_LIMIT_NS;
 long g_stall_fill = -1;
 
-template <int MODE, int NMAX>
+template <int MODE, int NMAX, bool MX>
 size_t gemm_smem_bytes(int n_exp) {
-  using TL = Tile<MODE, NMAX>;
+  using TL = Tile<MODE, NMAX, MX>;
   return 1024 + (size_t)TL::STAGES * TL::STAGE_BYTES + sizeof(Ctrl) + 2 * sizeof(int) * (n_exp + 1);
 }
 
-template <int MODE, int NMAX, bool F8, bool PK>
+template <int MODE, int NMAX, int Q, bool PK>
 moe_status launch_gemm(const CUtensorMap& A0, const CUtensorMap& B0, const CUtensorMap& A1,
                        const CUtensorMap& B1, const CUtensorMap& B0big, const CUtensorMap& B1big,
                        const GemmArgs& args, cudaStream_t s) {
-  const size_t smem = gemm_smem_bytes<MODE, NMAX>(args.n_exp);
+  const size_t smem = gemm_smem_bytes<MODE, NMAX, Q == Q_BLOCK>(args.n_exp);
   if (smem > 227 * 1024) return MOE_ERR_UNSUPPORTED;
-  if (cudaFuncSetAttribute(grouped_gemm_kernel<MODE, NMAX, F8, PK>,
+  if (cudaFuncSetAttribute(grouped_gemm_kernel<MODE, NMAX, Q, PK>,
                            cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) != cudaSuccess)
     return MOE_ERR_CUDA;
-  grouped_gemm_kernel<MODE, NMAX, F8, PK><<<num_sms(), NUM_THREADS, smem, s>>>(A0, B0, A1, B1,
-                                                                               B0big, B1big, args);
+  grouped_gemm_kernel<MODE, NMAX, Q, PK><<<num_sms(), NUM_THREADS, smem, s>>>(A0, B0, A1, B1,
+                                                                              B0big, B1big, args);
   note_launch();
   return launch_status();
 }
@@ -839,9 +982,11 @@ bool make_rows_map(CUtensorMap* m, const void* ptr, uint64_t cols, uint64_t rows
 // PK: weights in the tile-packed layout, fetched by bulk copies (a separate
 // instantiation: a runtime choice between the two weight paths in the
 // producer's loop measured 12 % slower decode GEMM2 even when never taken).
-template <int NMAX, bool F8, bool PK>
+template <int NMAX, int Q, bool PK>
 moe_status run_ffn(const FfnGroup& g0, const FfnGroup* g1, int H, int I, cudaStream_t s,
                    cudaEvent_t after_gemm1) {
+  constexpr bool F8 = Q != Q_BF16;
+  constexpr bool MX = Q == Q_BLOCK;
   CUtensorMap a1, b1, a2, b2, sa1, sb1, sa2, sb2, b1big, b2big, sb1big, sb2big;
   // with a fused dispatch GEMM1 reads token rows of x by index: a one-row box
   const bool gather = g0.gather != nullptr;
@@ -858,7 +1003,8 @@ moe_status run_ffn(const FfnGroup& g0, const FfnGroup* g1, int H, int I, cudaStr
       !make_rows_map<F8>(&b2big, h0, I, g0.rows, B_BIG))
     return MOE_ERR_CUDA;
   if (g1) {
-    if (g1->packed != g0.packed || g1->fp8 != g0.fp8) return MOE_ERR_INVALID_ARG;
+    if (g1->packed != g0.packed || g1->fp8 != g0.fp8 || g1->fp8_block != g0.fp8_block)
+      return MOE_ERR_INVALID_ARG;
     const void* h1 = F8 ? static_cast<const void*>(g1->hq) : static_cast<const void*>(g1->h);
     if (!make_rows_map<F8>(&sa1, g1->W13, H, (uint64_t)2 * I, BM) ||
         !make_rows_map<F8>(&sb1, g1->x, H, g1->rows, B_BOX) ||
@@ -896,17 +1042,30 @@ moe_status run_ffn(const FfnGroup& g0, const FfnGroup* g1, int H, int I, cudaStr
   args.out0 = g0.h;
   args.out1 = g1 ? g1->h : nullptr;
   args.out_ld = I;
-  if (F8) {
+  if (F8 && !MX) {
     args.a_scale0 = g0.W13_scale;
     args.a_scale1 = g1 ? g1->W13_scale : nullptr;
     args.b_scale0 = g0.x_scale;
     args.b_scale1 = g1 ? g1->x_scale : nullptr;
     args.b_scale_idx0 = g0.x_scale_idx;
   }
+  if (MX) {
+    args.a_sf0 = g0.W13_sf;
+    args.a_sf1 = g1 ? g1->W13_sf : nullptr;
+    args.b_sf0 = g0.x_sf;
+    args.b_sf_ld0 = g0.x_sf_ld;
+    args.b_sf1 = g1 ? g1->x_sf : nullptr;
+    args.b_sf_ld1 = g1 ? g1->x_sf_ld : 0;
+    args.b_scale_idx0 = g0.x_scale_idx;
+  }
   moe_status st =
-      launch_gemm<MODE_SWIGLU, NMAX, F8, PK>(a1, b1, sa1, sb1, b1big, sb1big, args, s);
+      launch_gemm<MODE_SWIGLU, NMAX, Q, PK>(a1, b1, sa1, sb1, b1big, sb1big, args, s);
   if (st != MOE_OK) return st;
-  if (F8) {  // h of every packed row -> e4m3 and its row scale: GEMM2's operand
+  if (MX) {  // h of every packed row -> e4m3 in 1 x 128 blocks: GEMM2's operand
+    MOE_STATUS_TRY(launch_quantize_blocks(g0.h, g0.rows, I, g0.hq, g0.hsf, g0.h_sf_ld, s));
+    if (g1)
+      MOE_STATUS_TRY(launch_quantize_blocks(g1->h, g1->rows, I, g1->hq, g1->hsf, g1->h_sf_ld, s));
+  } else if (F8) {  // h of every packed row -> e4m3 and its row scale: GEMM2's operand
     MOE_STATUS_TRY(launch_quantize_rows(g0.h, g0.rows, I, g0.hq, g0.hs, s));
     if (g1) MOE_STATUS_TRY(launch_quantize_rows(g1->h, g1->rows, I, g1->hq, g1->hs, s));
   }
@@ -914,11 +1073,20 @@ moe_status run_ffn(const FfnGroup& g0, const FfnGroup* g1, int H, int I, cudaStr
   args.gather0 = nullptr;  // GEMM2 reads h, already in packed row order
   args.a0_packed = pk ? static_cast<const uint16_t*>(g0.W2) : nullptr;
   args.a1_packed = (pk && g1) ? static_cast<const uint16_t*>(g1->W2) : nullptr;
-  if (F8) {
+  if (F8 && !MX) {
     args.a_scale0 = g0.W2_scale;
     args.a_scale1 = g1 ? g1->W2_scale : nullptr;
     args.b_scale0 = g0.hs;
     args.b_scale1 = g1 ? g1->hs : nullptr;
+    args.b_scale_idx0 = nullptr;
+  }
+  if (MX) {
+    args.a_sf0 = g0.W2_sf;
+    args.a_sf1 = g1 ? g1->W2_sf : nullptr;
+    args.b_sf0 = g0.hsf;
+    args.b_sf_ld0 = g0.h_sf_ld;
+    args.b_sf1 = g1 ? g1->hsf : nullptr;
+    args.b_sf_ld1 = g1 ? g1->h_sf_ld : 0;
     args.b_scale_idx0 = nullptr;
   }
   args.comb_out0 = g0.comb_out;
@@ -938,11 +1106,11 @@ moe_status run_ffn(const FfnGroup& g0, const FfnGroup* g1, int H, int I, cudaStr
   if (H % (2 * BM) == 0) {
     args.n_fb = H / (2 * BM);
     args.up_off = BM;
-    return launch_gemm<MODE_PLAIN2, NMAX, F8, PK>(a2, b2, sa2, sb2, b2big, sb2big, args, s);
+    return launch_gemm<MODE_PLAIN2, NMAX, Q, PK>(a2, b2, sa2, sb2, b2big, sb2big, args, s);
   }
   args.n_fb = H / BM;
   args.up_off = 0;
-  return launch_gemm<MODE_PLAIN, NMAX, F8, PK>(a2, b2, sa2, sb2, b2big, sb2big, args, s);
+  return launch_gemm<MODE_PLAIN, NMAX, Q, PK>(a2, b2, sa2, sb2, b2big, sb2big, args, s);
 }
 
 }  // namespace
@@ -957,19 +1125,26 @@ moe_status launch_expert_ffn_groups(const FfnGroup& routed, const FfnGroup* dens
   // of the stage ring to weights (decode ~4 rows/expert -> 32; balanced
   // prefill ~128 +- 10 % -> 144; larger or skewed loads -> 256).
   const long per = (long)rows_hint / (n_exp > 0 ? n_exp : 1);
+  if (routed.fp8 && routed.fp8_block) {
+    // the largest tile is 224 rows: two 224-column accumulators and the
+    // stages' scale columns share TMEM's 512 columns
+    if (per <= 24) return run_ffn<32, Q_BLOCK, false>(routed, g1, H, I, s, after_gemm1);
+    if (per <= 132) return run_ffn<144, Q_BLOCK, false>(routed, g1, H, I, s, after_gemm1);
+    return run_ffn<224, Q_BLOCK, false>(routed, g1, H, I, s, after_gemm1);
+  }
   if (routed.fp8) {
-    if (per <= 24) return run_ffn<32, true, false>(routed, g1, H, I, s, after_gemm1);
-    if (per <= 132) return run_ffn<144, true, false>(routed, g1, H, I, s, after_gemm1);
-    return run_ffn<256, true, false>(routed, g1, H, I, s, after_gemm1);
+    if (per <= 24) return run_ffn<32, Q_ROW, false>(routed, g1, H, I, s, after_gemm1);
+    if (per <= 132) return run_ffn<144, Q_ROW, false>(routed, g1, H, I, s, after_gemm1);
+    return run_ffn<256, Q_ROW, false>(routed, g1, H, I, s, after_gemm1);
   }
   if (routed.packed) {
-    if (per <= 24) return run_ffn<32, false, true>(routed, g1, H, I, s, after_gemm1);
-    if (per <= 132) return run_ffn<144, false, true>(routed, g1, H, I, s, after_gemm1);
-    return run_ffn<256, false, true>(routed, g1, H, I, s, after_gemm1);
+    if (per <= 24) return run_ffn<32, Q_BF16, true>(routed, g1, H, I, s, after_gemm1);
+    if (per <= 132) return run_ffn<144, Q_BF16, true>(routed, g1, H, I, s, after_gemm1);
+    return run_ffn<256, Q_BF16, true>(routed, g1, H, I, s, after_gemm1);
   }
-  if (per <= 24) return run_ffn<32, false, false>(routed, g1, H, I, s, after_gemm1);
-  if (per <= 132) return run_ffn<144, false, false>(routed, g1, H, I, s, after_gemm1);
-  return run_ffn<256, false, false>(routed, g1, H, I, s, after_gemm1);
+  if (per <= 24) return run_ffn<32, Q_BF16, false>(routed, g1, H, I, s, after_gemm1);
+  if (per <= 132) return run_ffn<144, Q_BF16, false>(routed, g1, H, I, s, after_gemm1);
+  return run_ffn<256, Q_BF16, false>(routed, g1, H, I, s, after_gemm1);
 }
 
 int router_tc_splits(int T, int H, int E) {
@@ -999,7 +1174,7 @@ moe_status launch_router_tc(int T, int H, int E, const uint16_t* x, const uint16
   args.out1 = partials;
   args.out_ld = E;
   args.err = device_error_word();
-  return launch_gemm<MODE_SPLIT3, 128, false, false>(A, B, A, B, Bbig, Bbig, args, s);
+  return launch_gemm<MODE_SPLIT3, 128, Q_BF16, false>(A, B, A, B, Bbig, Bbig, args, s);
 }
 
 moe_status launch_expert_ffn_stalled(int rows, int H, int I, int n_experts, const uint16_t* x_perm,

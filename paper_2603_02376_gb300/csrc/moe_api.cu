@@ -89,7 +89,7 @@ bool valid_exec(const moe_exec* ex, const moe_config* c) {
   if (ex->overlap != 0 && ex->overlap != 1) return false;
   if (ex->out_fp32 != 0 && ex->out_fp32 != 1) return false;
   if (ex->fuse_gather != 0 && ex->fuse_gather != 1) return false;
-  if (ex->fp8 != 0 && ex->fp8 != 1) return false;
+  if (ex->fp8 < 0 || ex->fp8 > 2) return false;
   if (ex->fuse_combine != 0 && ex->fuse_combine != 1) return false;
   if (ex->overlap) {
     if (ex->chunk_axis == 0) {
@@ -131,17 +131,21 @@ struct Layout {
   int32_t* perm_base;
   void* router_ws;   // router scratch (planes + partials), sized for one chunk
   bool fp8 = false;
+  bool fp8_block = false;  // block scales (fp8 = 2) instead of row scales (fp8 = 1)
   uint8_t* x_q;      // [T, H] e4m3 (fp8 only)
   float* x_s;        // [T] row scales of x_q
+  uint8_t* x_sf;     // [H/128][T] block exponents of x_q (block form)
   void* x_perm;      // [T*k, H] bf16, or e4m3 bytes (fp8)
   uint16_t* h;       // [T*k, I]
   uint8_t* hq;       // [T*k, I] e4m3 copy of h (fp8 only)
   float* hs;         // [T*k] its row scales
+  uint8_t* hsf;      // [I/128][T*k] its block exponents (block form)
   float* y_perm;     // [T*k, H] fp32
   int32_t* sh_off;   // [2]
   uint16_t* sh_h;    // [T, I_s]
   uint8_t* sh_hq;    // [T, I_s] (fp8 only)
   float* sh_hs;      // [T]
+  uint8_t* sh_hsf;   // [I_s/128][T] (block form)
   float* sh_y;       // [T, H] fp32 (unfused combine)
   // Combine fused into GEMM2: the gate weight of every packed row, and the fp32
   // [T, H] accumulator the GEMM2s reduce into (the caller's output when it is
@@ -181,13 +185,17 @@ Layout carve(const moe_config& c, const moe_exec& ex, void* ws) {
   // chunk averages at most 24 rows per expert.
   const bool fuse = ex.fuse_gather && (long)L.chunk_T * c.k <= 24L * c.E;
   L.fp8 = ex.fp8 != 0;
+  L.fp8_block = ex.fp8 == 2;
+  const bool rows_fp8 = L.fp8 && !L.fp8_block;
   const size_t xb = L.fp8 ? 1 : 2;  // bytes per activation element
   L.x_q = L.fp8 ? cv.take<uint8_t>(T * c.H) : nullptr;
-  L.x_s = L.fp8 ? cv.take<float>(T) : nullptr;
+  L.x_s = rows_fp8 ? cv.take<float>(T) : nullptr;
+  L.x_sf = L.fp8_block ? cv.take<uint8_t>((size_t)(c.H / 128) * T) : nullptr;
   L.x_perm = fuse ? nullptr : static_cast<void*>(cv.take<uint8_t>(T * k * c.H * xb));
   L.h = cv.take<uint16_t>(T * k * c.I);
   L.hq = L.fp8 ? cv.take<uint8_t>(T * k * c.I) : nullptr;
-  L.hs = L.fp8 ? cv.take<float>(T * k) : nullptr;
+  L.hs = rows_fp8 ? cv.take<float>(T * k) : nullptr;
+  L.hsf = L.fp8_block ? cv.take<uint8_t>((size_t)(c.I / 128) * T * k) : nullptr;
   L.fuse_combine = ex.fuse_combine != 0;
   L.row_w = L.fuse_combine ? cv.take<float>(T * k) : nullptr;
   L.y_perm = L.fuse_combine ? nullptr : cv.take<float>(T * k * c.H);
@@ -195,7 +203,9 @@ Layout carve(const moe_config& c, const moe_exec& ex, void* ws) {
   L.sh_off = cv.take<int32_t>(2);
   L.sh_h = c.I_shared ? cv.take<uint16_t>(T * c.I_shared) : nullptr;
   L.sh_hq = (c.I_shared && L.fp8) ? cv.take<uint8_t>(T * c.I_shared) : nullptr;
-  L.sh_hs = (c.I_shared && L.fp8) ? cv.take<float>(T) : nullptr;
+  L.sh_hs = (c.I_shared && rows_fp8) ? cv.take<float>(T) : nullptr;
+  L.sh_hsf = (c.I_shared && L.fp8_block) ? cv.take<uint8_t>((size_t)(c.I_shared / 128) * T)
+                                         : nullptr;
   L.sh_y = (c.I_shared && !L.fuse_combine) ? cv.take<float>(T * c.H) : nullptr;
   L.bytes = align_up(cv.off, 256);
   return L;
@@ -241,9 +251,13 @@ moe_status mark(cudaEvent_t* ev, int i, cudaStream_t s) {
   return MOE_OK;
 }
 
-// FP8: rows [t0, t0+Tc) of x -> e4m3 rows of x_q and their scales.
+// FP8: rows [t0, t0+Tc) of x -> e4m3 rows of x_q and their scales (per row,
+// or per 1 x 128 block: exponents x_sf[kb * T + t]).
 moe_status quantize_tokens(const moe_config& c, const Layout& L, const uint16_t* x, int t0, int Tc,
                            cudaStream_t s) {
+  if (L.fp8_block)
+    return launch_quantize_blocks(x + (size_t)t0 * c.H, Tc, c.H, L.x_q + (size_t)t0 * c.H,
+                                  L.x_sf + t0, (long)c.T, s);
   return launch_quantize_rows(x + (size_t)t0 * c.H, Tc, c.H, L.x_q + (size_t)t0 * c.H, L.x_s + t0,
                               s);
 }
@@ -318,12 +332,22 @@ FfnGroup routed_group(const moe_config& c, const Layout& L, const moe_weights& w
   }
   if (L.fp8) {
     g.fp8 = true;
-    g.x_scale = L.x_s + t0;  // per token of the chunk, reached through row_src_token
-    g.x_scale_idx = L.rst + tk;
-    g.W13_scale = w.W13_scale;
-    g.W2_scale = w.W2_scale;
+    g.x_scale_idx = L.rst + tk;  // the scales are per token, reached through row_src_token
     g.hq = L.hq + tk * c.I;
-    g.hs = L.hs + tk;
+    if (L.fp8_block) {
+      g.fp8_block = true;
+      g.x_sf = L.x_sf + t0;
+      g.x_sf_ld = c.T;
+      g.W13_sf = static_cast<const uint8_t*>(w.W13_scale);
+      g.W2_sf = static_cast<const uint8_t*>(w.W2_scale);
+      g.hsf = L.hsf + tk;
+      g.h_sf_ld = (long)c.T * c.k;
+    } else {
+      g.x_scale = L.x_s + t0;
+      g.W13_scale = static_cast<const float*>(w.W13_scale);
+      g.W2_scale = static_cast<const float*>(w.W2_scale);
+      g.hs = L.hs + tk;
+    }
   }
   return g;
 }
@@ -346,11 +370,21 @@ FfnGroup dense_group(const moe_config& c, const Layout& L, const moe_weights& w,
   if (L.fp8) {
     g.fp8 = true;
     g.x = L.x_q;
-    g.x_scale = L.x_s;
-    g.W13_scale = w.Ws13_scale;
-    g.W2_scale = w.Ws2_scale;
     g.hq = L.sh_hq;
-    g.hs = L.sh_hs;
+    if (L.fp8_block) {
+      g.fp8_block = true;
+      g.x_sf = L.x_sf;
+      g.x_sf_ld = c.T;
+      g.W13_sf = static_cast<const uint8_t*>(w.Ws13_scale);
+      g.W2_sf = static_cast<const uint8_t*>(w.Ws2_scale);
+      g.hsf = L.sh_hsf;
+      g.h_sf_ld = c.T;
+    } else {
+      g.x_scale = L.x_s;
+      g.W13_scale = static_cast<const float*>(w.Ws13_scale);
+      g.W2_scale = static_cast<const float*>(w.Ws2_scale);
+      g.hs = L.sh_hs;
+    }
   }
   return g;
 }
@@ -591,6 +625,78 @@ moe_status moe_expert_ffn_fp8(int32_t rows, int32_t H, int32_t I, int32_t n_expe
   return launch_expert_ffn_groups(g, nullptr, H, I, rows, (cudaStream_t)stream);
 }
 
+size_t moe_expert_ffn_fp8_blocks_workspace_size(int32_t rows, int32_t I) {
+  if (rows < 0 || I < 0) return 0;
+  Carver cv(nullptr);
+  cv.take<uint16_t>((size_t)rows * I);
+  cv.take<uint8_t>((size_t)rows * I);
+  cv.take<uint8_t>((size_t)(I / 128) * rows);
+  return align_up(cv.off, 256);
+}
+
+moe_status moe_quantize_fp8_blocks(int64_t rows, int32_t K, const uint16_t* in, uint8_t* out,
+                                   uint8_t* sf, int64_t sf_ld, void* stream) {
+  if (rows < 0 || rows > (1LL << 31) || K < 128 || K % 128 || K > 65536 || sf_ld < rows)
+    return MOE_ERR_INVALID_ARG;
+  if (rows == 0) return MOE_OK;
+  if (!in || !out || !sf || !aligned16(in) || !aligned16(out)) return MOE_ERR_INVALID_ARG;
+  const uint8_t *a = (const uint8_t*)in, *b = out;
+  if (a < b + (size_t)rows * K && b < a + (size_t)rows * K * 2) return MOE_ERR_INVALID_ARG;
+  return launch_quantize_blocks(in, (long)rows, K, out, sf, (long)sf_ld, (cudaStream_t)stream);
+}
+
+moe_status moe_quantize_fp8_weight_blocks(int64_t rows, int32_t K, const uint16_t* in,
+                                          uint8_t* out, uint8_t* sf, void* stream) {
+  if (rows < 0 || rows % 128 || rows / 128 > 65535 || K < 128 || K % 128 || K > 65536)
+    return MOE_ERR_INVALID_ARG;
+  if (rows == 0) return MOE_OK;
+  if (!in || !out || !sf || !aligned16(in) || !aligned16(out)) return MOE_ERR_INVALID_ARG;
+  const uint8_t *a = (const uint8_t*)in, *b = out;
+  if (a < b + (size_t)rows * K && b < a + (size_t)rows * K * 2) return MOE_ERR_INVALID_ARG;
+  return launch_quantize_weight_blocks(in, (long)rows, K, out, sf, (cudaStream_t)stream);
+}
+
+moe_status moe_expert_ffn_fp8_blocks(int32_t rows, int32_t H, int32_t I, int32_t n_experts,
+                                     const uint8_t* x_q, const uint8_t* x_sf, int64_t x_sf_ld,
+                                     const int32_t* x_scale_idx, const int32_t* offsets,
+                                     const uint8_t* W13_q, const uint8_t* W13_sf,
+                                     const uint8_t* W2_q, const uint8_t* W2_sf, float* y_perm,
+                                     void* ws, size_t ws_bytes, void* stream) {
+  if (rows < 0 || H < 128 || H % 128 || H > 65536 || I < 128 || I % 128 || I > 65536 ||
+      n_experts < 1 || n_experts > 1024 || x_sf_ld < 1 || (!x_scale_idx && x_sf_ld < rows))
+    return MOE_ERR_INVALID_ARG;
+  if (rows == 0) return MOE_OK;
+  if (!x_q || !x_sf || !offsets || !W13_q || !W13_sf || !W2_q || !W2_sf || !y_perm ||
+      !aligned16(x_q) || !aligned16(W13_q) || !aligned16(W2_q) || !aligned16(y_perm) ||
+      !aligned4(offsets) || (x_scale_idx && !aligned4(x_scale_idx)))
+    return MOE_ERR_INVALID_ARG;
+  if (!ws || ws_bytes < moe_expert_ffn_fp8_blocks_workspace_size(rows, I) ||
+      ((uintptr_t)ws & 255))
+    return MOE_ERR_WORKSPACE;
+  Carver cv(ws);
+  FfnGroup g{};
+  g.x = x_q;
+  g.offsets = offsets;
+  g.rows = rows;
+  g.n_experts = n_experts;
+  g.e_end = n_experts;
+  g.W13 = W13_q;
+  g.W2 = W2_q;
+  g.h = cv.take<uint16_t>((size_t)rows * I);
+  g.hq = cv.take<uint8_t>((size_t)rows * I);
+  g.hsf = cv.take<uint8_t>((size_t)(I / 128) * rows);
+  g.h_sf_ld = rows;
+  g.y = y_perm;
+  g.fp8 = true;
+  g.fp8_block = true;
+  g.x_sf = x_sf;
+  g.x_sf_ld = (long)x_sf_ld;
+  g.x_scale_idx = x_scale_idx;
+  g.W13_sf = W13_sf;
+  g.W2_sf = W2_sf;
+  return launch_expert_ffn_groups(g, nullptr, H, I, rows, (cudaStream_t)stream);
+}
+
 moe_status moe_testing_expert_ffn_stall(int32_t rows, int32_t H, int32_t I, int32_t n_experts,
                                         const uint16_t* x_perm, const int32_t* offsets,
                                         const uint16_t* W13, const uint16_t* W2, float* y_perm,
@@ -628,12 +734,14 @@ moe_status moe_layer_forward(const moe_config* cfg, const moe_exec* ex, const mo
   if (!valid_config(cfg) || !valid_exec(ex, cfg) || !w) return MOE_ERR_INVALID_ARG;
   if (w->packed != 0 && w->packed != 1) return MOE_ERR_INVALID_ARG;
   const moe_config& c = *cfg;
-  if (ex->fp8) {  // e4m3 expert weights with row scales; no packed form
+  if (ex->fp8) {  // e4m3 expert weights with row or block scales; no packed form
     if (w->packed) return MOE_ERR_UNSUPPORTED;
-    if (!w->W13_scale || !w->W2_scale || !aligned4(w->W13_scale) || !aligned4(w->W2_scale))
+    const bool al = ex->fp8 == 2;  // exponent bytes need no alignment
+    if (!w->W13_scale || !w->W2_scale || !(al || aligned4(w->W13_scale)) ||
+        !(al || aligned4(w->W2_scale)))
       return MOE_ERR_INVALID_ARG;
-    if (c.I_shared && (!w->Ws13_scale || !w->Ws2_scale || !aligned4(w->Ws13_scale) ||
-                       !aligned4(w->Ws2_scale)))
+    if (c.I_shared && (!w->Ws13_scale || !w->Ws2_scale || !(al || aligned4(w->Ws13_scale)) ||
+                       !(al || aligned4(w->Ws2_scale))))
       return MOE_ERR_INVALID_ARG;
   }
   if (!w->Wr || !w->W13 || !w->W2 || !aligned16(w->Wr) || !aligned16(w->W13) ||

@@ -204,7 +204,9 @@ def test_fp8_entry_points_reject_bad_arguments_without_a_gpu(lib):
     assert lib.moe_layer_forward(cb(c), cb(ex8), cb(W), p, p, None, p, 1 << 40, z, z) == L.MOE_ERR_INVALID_ARG
     Wp = L.moe_weights(0x1000, None, 0x1000, 0x1000, 0x1000, 0x1000, 1, 0x1000, 0x1000, 0x1000, 0x1000)
     assert lib.moe_layer_forward(cb(c), cb(ex8), cb(Wp), p, p, None, p, 1 << 40, z, z) == L.MOE_ERR_UNSUPPORTED
-    assert lib.moe_layer_forward(cb(c), cb(L.exec_config(fp8=2)), cb(W), p, p, None, p, 1 << 40, z, z) == L.MOE_ERR_INVALID_ARG
+    assert lib.moe_layer_forward(cb(c), cb(L.exec_config(fp8=3)), cb(W8 := L.moe_weights(
+        0x1000, None, 0x1000, 0x1000, 0x1000, 0x1000, 0, 0x1000, 0x1000, 0x1000, 0x1000)),
+        p, p, None, p, 1 << 40, z, z) == L.MOE_ERR_INVALID_ARG                 # no such form
     W8 = L.moe_weights(0x1000, None, 0x1000, 0x1000, 0x1000, 0x1000, 0, 0x1000, 0x1000, 0x1000, 0x1000)
     assert lib.moe_layer_forward(cb(c), cb(ex8), cb(W8), p, p, None, z, 0, z, z) == L.MOE_ERR_WORKSPACE
     # the fp8 layout adds the quantized copies; its x_perm is half the bf16 one
@@ -214,6 +216,59 @@ def test_fp8_entry_points_reject_bad_arguments_without_a_gpu(lib):
         n8 = L.moe_workspace_size(cw, L.exec_config(fuse_gather=0, fp8=1))
         tk = wl.T * wl.k
         assert n8 - n16 >= wl.T * wl.H + tk * wl.I - tk * wl.H - (1 << 16)
+
+
+def test_fp8_block_entry_points_reject_bad_arguments_without_a_gpu(lib):
+    c = L.config(**GOOD)
+    z = ctypes.c_void_p(0)
+    p = ctypes.c_void_p(0x1000)
+    q = ctypes.c_void_p(0x100000)
+    odd = ctypes.c_void_p(0x1008)
+    cb = ctypes.byref
+    QB = lib.moe_quantize_fp8_blocks
+    assert QB(16, 100, p, q, q, 16, z) == L.MOE_ERR_INVALID_ARG       # K % 128
+    assert QB(16, 64, p, q, q, 16, z) == L.MOE_ERR_INVALID_ARG        # K < 128
+    assert QB(16, 128, p, q, q, 15, z) == L.MOE_ERR_INVALID_ARG       # sf_ld < rows
+    assert QB(16, 128, p, p, q, 16, z) == L.MOE_ERR_INVALID_ARG       # in and out overlap
+    assert QB(16, 128, odd, q, q, 16, z) == L.MOE_ERR_INVALID_ARG
+    assert QB(16, 128, p, q, z, 16, z) == L.MOE_ERR_INVALID_ARG       # no exponent buffer
+    assert QB(0, 128, z, z, z, 0, z) == L.MOE_OK
+    QW = lib.moe_quantize_fp8_weight_blocks
+    assert QW(100, 128, p, q, q, z) == L.MOE_ERR_INVALID_ARG          # rows % 128
+    assert QW(128, 96, p, q, q, z) == L.MOE_ERR_INVALID_ARG           # K % 128
+    assert QW(128 * 65536, 128, p, q, q, z) == L.MOE_ERR_INVALID_ARG  # grid rows
+    assert QW(128, 128, p, p, q, z) == L.MOE_ERR_INVALID_ARG
+    assert QW(0, 128, z, z, z, z) == L.MOE_OK
+    F = lib.moe_expert_ffn_fp8_blocks
+    a = lambda ld=16, idx=z: [p, p, ld, idx, p, p, p, p, p, p]    # x_q .. y_perm
+    assert F(16, 100, 128, 1, *a(), q, 1 << 20, z) == L.MOE_ERR_INVALID_ARG     # H % 128
+    assert F(16, 256, 96, 1, *a(), q, 1 << 20, z) == L.MOE_ERR_INVALID_ARG      # I % 128
+    assert F(16, 256, 128, 1, *a(ld=8), q, 1 << 20, z) == L.MOE_ERR_INVALID_ARG  # ld < rows
+    # rows reached through x_scale_idx may use a shorter exponent stride (the arguments
+    # pass; the misaligned workspace is what fails)
+    assert F(16, 256, 128, 1, *a(ld=8, idx=p), ctypes.c_void_p(0x100010), 1 << 20, z) == \
+        L.MOE_ERR_WORKSPACE
+    assert F(16, 256, 128, 1, *a(), z, 0, z) == L.MOE_ERR_WORKSPACE
+    assert F(16, 256, 128, 1, z, *a()[1:], q, 1 << 20, z) == L.MOE_ERR_INVALID_ARG
+    assert F(0, 256, 128, 1, z, z, 1, z, z, z, z, z, z, z, z, 0, z) == L.MOE_OK
+    n = lib.moe_expert_ffn_fp8_blocks_workspace_size(16, 256)
+    assert n >= 16 * 256 * 3 + 2 * 16 and n % 256 == 0
+    # layer forward: block scales need whole 128-blocks and the exponent arrays
+    W8 = L.moe_weights(0x1000, None, 0x1000, 0x1000, 0x1000, 0x1000, 0, 0x1001, 0x1001, 0x1001,
+                       0x1001)                        # byte arrays: any alignment
+    exb = L.exec_config(fp8=2)
+    assert lib.moe_layer_forward(cb(c), cb(exb), cb(W8), p, p, None, z, 0, z, z) == L.MOE_ERR_WORKSPACE
+    Wn = L.moe_weights(0x1000, None, 0x1000, 0x1000, 0x1000, 0x1000, 0, 0x1001, None, 0x1001,
+                       0x1001)
+    assert lib.moe_layer_forward(cb(c), cb(exb), cb(Wn), p, p, None, z, 0, z, z) == L.MOE_ERR_INVALID_ARG
+    # the block layout: per-row scale arrays replaced by exponent bytes
+    for wl in (I.DECODE, I.PREFILL):
+        cw = L.config_of(wl)
+        n8 = L.moe_workspace_size(cw, L.exec_config(fuse_gather=0, fp8=1))
+        nb = L.moe_workspace_size(cw, L.exec_config(fuse_gather=0, fp8=2))
+        tk = wl.T * wl.k
+        extra = wl.H // 128 * wl.T + wl.I // 128 * tk + wl.I_shared // 128 * wl.T
+        assert nb - n8 == pytest.approx(extra - 4 * (wl.T + tk + wl.T), abs=4096)
 
 
 def test_empty_batch_is_a_no_op(lib):

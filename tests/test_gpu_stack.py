@@ -7,7 +7,7 @@
   the chain matches the oracle run on that layer's input and on the GPU's
   fp32 logits, within the layer bound |err| <= 2e-2 + 1e-2 |ref|.
 * A graph made by moe_graph_create_stack replays the stack bit for bit, in
-  the sequential and both pipelined modes and in the FP8 form, also after new
+  the sequential and both pipelined modes and in both FP8 forms, also after new
   inputs are written into its x buffer; its kernel count is the eager one.
 """
 
@@ -98,14 +98,17 @@ def test_stack_equals_chained_layers_and_the_oracle(rms_norm):
 
 @pytest.mark.parametrize("mode", [dict(), dict(overlap=1, chunk_axis=0, chunk_tokens=37),
                                   dict(overlap=1, chunk_axis=1, n_expert_chunks=3),
-                                  dict(fuse_gather=0), dict(fp8=1)])
+                                  dict(fuse_gather=0), dict(fp8=1), dict(fp8=2)])
 def test_graph_replays_the_stack(mode):
     wl, n = SMALL, 3
     ds = small_layers(n)
     if mode.get("fp8"):
-        for d in ds:   # e4m3 expert weights with row scales, quantized on the device
+        # e4m3 expert weights with row scales (fp8 = 1) or 128 x 128 block exponents
+        # (fp8 = 2), quantized on the device
+        quant = L.quantize_fp8 if mode["fp8"] == 1 else L.quantize_fp8_weight_blocks
+        for d in ds:
             for w_, s_ in (("W13", "s13"), ("W2", "s2"), ("Ws13", "ss13"), ("Ws2", "ss2")):
-                d[w_], d[s_] = L.quantize_fp8(d[w_])
+                d[w_], d[s_] = quant(d[w_])
     cfg, ex = L.config_of(wl), L.exec_config(**mode)
     layers = [wstruct(d) for d in ds]
     ws = torch.empty(L.moe_stack_workspace_size(cfg, ex), dtype=torch.uint8, device=DEV)

@@ -55,9 +55,10 @@ def parse():
     p.add_argument("--pack", choices=("auto", "yes", "no"), default="auto",
                    help="tile-pack the expert weights at load (auto: yes for bf16, "
                         "no for fp8, which has no packed form)")
-    p.add_argument("--precision", choices=("bf16", "fp8"), default="bf16",
-                   help="expert GEMM operands: bf16, or e4m3 with per-row scales (weights "
-                        "quantized once at load, tokens and h quantized inside each step)")
+    p.add_argument("--precision", choices=("bf16", "fp8", "fp8-block"), default="bf16",
+                   help="expert GEMM operands: bf16; e4m3 with per-row scales; or e4m3 with "
+                        "UE8M0 block scales (1x128 tokens and h, 128x128 weights). Weights "
+                        "are quantized once at load, tokens and h inside each step")
     p.add_argument("--fuse-combine", action="store_true",
                    help="fuse the gate-weighted combine into GEMM2's epilogue (fp32 reductions)")
     p.add_argument("--layers", type=int, default=1,
@@ -199,13 +200,21 @@ def calibrate(L, wl, d, device):
         d["bias"] = b.to(device)
 
 
-def algorithmic(wl, touched, fused_gather=True, fp8=False, fused_combine=False):
+def scale_bytes(rows, n, fp8):
+    """Bytes of the scales of a [rows, n] activation: one fp32 per row (fp8 = 1)
+    or one UE8M0 byte per 1 x 128 block (fp8 = 2)."""
+    return 0 if not fp8 else rows * 4 if fp8 == 1 else rows * (n // 128)
+
+
+def algorithmic(wl, touched, fused_gather=True, fp8=0, fused_combine=False):
     """Algorithmic bytes and flops of each stage for one forward.
 
     GEMM1's token operand is counted as R*H*eb either way (packed rows read, or
     the same rows gathered from x); a fused dispatch has no copy of its own.
-    FP8 (eb = 1): the dispatch stage also quantizes x (bf16 read, e4m3 + scales
-    written) and the GEMM1 stage also quantizes h (bf16 read, e4m3 + scales).
+    FP8 (eb = 1; fp8 = 1 row scales, 2 block scales): the dispatch stage also
+    quantizes x (bf16 read, e4m3 + scales written) and the GEMM1 stage also
+    quantizes h (bf16 read, e4m3 + scales); the GEMMs read the scales of their
+    operands (weights: one fp32 per row, or one byte per 128 x 128 block).
     Fused combine: GEMM2 reduces into the fp32 [T, H] accumulator (counted once)
     instead of writing y_perm; the accumulator is cleared at the start (counted
     in the router stage) and converted to the bf16 output in the combine stage.
@@ -213,17 +222,23 @@ def algorithmic(wl, touched, fused_gather=True, fp8=False, fused_combine=False):
     T, H, E, k, Iw, Is = wl.T, wl.H, wl.E, wl.k, wl.I, wl.I_shared
     R = T * k
     eb = 1 if fp8 else 2
-    qx = T * H * 3 + T * 4 if fp8 else 0               # x -> e4m3 rows + scales
-    qh = lambda rows, n: rows * n * 3 + rows * 4 if fp8 else 0   # h -> e4m3
+    sb = lambda rows, n: scale_bytes(rows, n, fp8)
+    # weight scales of a [rows, n] matrix: fp32 per row, or a byte per 128 x 128 block
+    wsb = lambda rows, n: 0 if not fp8 else rows * 4 if fp8 == 1 else (rows // 128) * (n // 128)
+    qx = T * H * 3 + sb(T, H) if fp8 else 0               # x -> e4m3 rows + scales
+    qh = lambda rows, n: rows * n * 3 + sb(rows, n) if fp8 else 0   # h -> e4m3
     b = {
         "router": T * H * 2 + E * H * 4 + T * E * 4,
         "gate": T * E * 4 + T * k * 8,
         "permute": T * k * 4 * 3,
         "dispatch": qx + (0 if fused_gather else T * H * eb + R * H * eb),
-        "gemm1": touched * 2 * Iw * H * eb + R * H * eb + R * Iw * 2 + qh(R, Iw),
-        "gemm2": touched * H * Iw * eb + R * Iw * eb + R * H * 4,
-        "shared_gemm1": (2 * Is * H * eb + T * H * eb + T * Is * 2 + qh(T, Is)) if Is else 0,
-        "shared_gemm2": (H * Is * eb + T * Is * eb + T * H * 4) if Is else 0,
+        "gemm1": touched * (2 * Iw * H * eb + wsb(2 * Iw, H)) + R * H * eb + sb(R, H)
+        + R * Iw * 2 + qh(R, Iw),
+        "gemm2": touched * (H * Iw * eb + wsb(H, Iw)) + R * Iw * eb + sb(R, Iw) + R * H * 4,
+        "shared_gemm1": (2 * Is * H * eb + wsb(2 * Is, H) + T * H * eb + sb(T, H) + T * Is * 2
+                         + qh(T, Is)) if Is else 0,
+        "shared_gemm2": (H * Is * eb + wsb(H, Is) + T * Is * eb + sb(T, Is) + T * H * 4)
+        if Is else 0,
         "combine": R * H * 4 + (T * H * 4 if Is else 0) + T * H * 2 + R * 8,
     }
     if fused_combine:
@@ -249,7 +264,7 @@ def source_sha():
     return h.hexdigest()[:16]
 
 
-def measured_traffic(workload, fp8=False, kernel_bytes=None):
+def measured_traffic(workload, fp8=0, kernel_bytes=None):
     """ncu DRAM bytes per GEMM1 launch, if captured for the current kernel source.
 
     The bf16 entry holds the bytes of the full launch; the FP8 entry holds the
@@ -258,7 +273,7 @@ def measured_traffic(workload, fp8=False, kernel_bytes=None):
     try:
         with open(TRAFFIC_FILE) as f:
             t = json.load(f)
-        e = t.get(workload + (" fp8" if fp8 else ""))
+        e = t.get(workload + {0: "", 1: " fp8", 2: " fp8-block"}[int(fp8)])
         if e and e.get("source_sha") == source_sha():
             if "dram_bytes_per_launch" in e:
                 return float(e["dram_bytes_per_launch"])
@@ -288,22 +303,29 @@ def oracle_tokens_per_s(wl, d, tokens):
     idx, _ = O.gate_topk(O.router_logits(xr, Wr), b, cfg)
     f8 = d.get("fp8")
     if f8:
+        # (codes, scales) pairs: e4m3 bytes, then fp32 row scales or UE8M0 block exponents
         host = {int(e): tuple(f8[n][e].cpu() for n in ("W13", "s13", "W2", "s2"))
                 for e in np.unique(idx)}
         shared = tuple(f8[n].cpu() for n in ("Ws13", "ss13", "Ws2", "ss2")) \
             if wl.I_shared else None
-        conv = lambda t: O.e4m3_decode(t.numpy()) if t.dtype == torch.uint8 else t.numpy()
-        ffn = O.swiglu_ffn_fp8
+        blk = f8.get("block", False)
+
+        def conv(t, i):
+            if i % 2 == 0:
+                return O.e4m3_decode(t.numpy())
+            return t.numpy().astype(np.int64) - 127 if blk else t.numpy()
+
+        ffn = O.swiglu_ffn_fp8_blocks if blk else O.swiglu_ffn_fp8
     else:
         host = {int(e): (d["W13"][e].cpu(), d["W2"][e].cpu()) for e in np.unique(idx)}
         shared = (d["Ws13"].cpu(), d["Ws2"].cpu()) if wl.I_shared else None
-        conv = lambda t: t.to(torch.float64).numpy()
+        conv = lambda t, i: t.to(torch.float64).numpy()
         ffn = O.swiglu_ffn
 
     def get_expert(e):
-        return tuple(conv(t) for t in host[e])
+        return tuple(conv(t, i) for i, t in enumerate(host[e]))
 
-    get_shared = (lambda: tuple(conv(t) for t in shared)) if shared else None
+    get_shared = (lambda: tuple(conv(t, i) for i, t in enumerate(shared))) if shared else None
     t0 = time.perf_counter()
     O.layer_forward_tokens(xr, Wr, b, get_expert, cfg, get_shared, ffn=ffn)
     dt = time.perf_counter() - t0
@@ -313,7 +335,8 @@ def oracle_tokens_per_s(wl, d, tokens):
 def cpu_baseline(wl, d, n_tokens, seed=1):
     toks = I.sample_tokens(wl.T, n_tokens, seed).numpy()
     v, dt, ne = oracle_tokens_per_s(wl, d, toks)
-    form = "FP8 expert form, " if d.get("fp8") else ""
+    form = ("block-scaled FP8 expert form, " if d["fp8"].get("block") else
+            "FP8 expert form, ") if d.get("fp8") else ""
     return {"value": v, "unit": "tokens/s", "cores": os.cpu_count(), "kind": "oracle",
             "sample": f"{len(toks)} of the {wl.T} tokens ({ne} experts touched), {form}numpy "
                       f"fp64 oracle, {dt:.1f} s; BLAS threads = host cores"}
@@ -357,7 +380,7 @@ def packs(args, wl):
     """Whether the run uses tile-packed expert weights (bf16 only; auto = yes: the
     GEMMs fetch each packed weight tile with one bulk copy, measured as fast or
     faster at every batch size)."""
-    if args.precision == "fp8":
+    if args.precision != "bf16":
         return False
     return args.pack in ("auto", "yes")
 
@@ -369,8 +392,12 @@ def config_of(wl, args):
             "mode": args.mode, "dispatch": "fused into GEMM1 (TMA gather4)"
             if (not args.no_fuse_gather and wl.T * wl.k <= 24 * wl.E) else "packed x_perm",
             "weights": "tile-packed at load (moe_pack_weights)" if packs(args, wl) else "row-major",
-            "precision": "e4m3 expert GEMMs, per-row fp32 scales (weights quantized at load)"
-            if args.precision == "fp8" else "bf16 expert GEMMs",
+            "precision": {"bf16": "bf16 expert GEMMs",
+                          "fp8": "e4m3 expert GEMMs, per-row fp32 scales (weights quantized "
+                                 "at load)",
+                          "fp8-block": "e4m3 expert GEMMs, UE8M0 block scales: 1x128 "
+                                       "activations, 128x128 weights (quantized at load), "
+                                       "applied by tcgen05 kind::mxf8f6f4"}[args.precision],
             "combine": "fused into GEMM2's epilogue (fp32 reductions)" if args.fuse_combine
             else "y_perm + combine kernel",
             "global_batch": wl.T * args.gpus,
@@ -392,7 +419,7 @@ def run_ours(args, wl, rank, world, local, device):
     fuse = 0 if args.no_fuse_gather else 1
     # the library fuses the dispatch only for decode-sized batches (<= 24 rows per expert)
     fused = bool(fuse) and wl.T * wl.k <= 24 * wl.E
-    fp8 = 1 if args.precision == "fp8" else 0
+    fp8 = {"bf16": 0, "fp8": 1, "fp8-block": 2}[args.precision]
     fc = 1 if args.fuse_combine else 0
     ex = L.exec_config(fuse_gather=fuse, fp8=fp8, fuse_combine=fc, **mode)
     # one workspace serves the timed mode and the sequential stats / stage-event passes
@@ -410,15 +437,20 @@ def run_ours(args, wl, rank, world, local, device):
         run_w = {k_: (None if v is None else L.pack_weights(v)) for k_, v in run_w.items()}
         torch.cuda.synchronize()
     if fp8:
-        # e4m3 copies of the expert weights with per-row scales: a load-time step
-        # like the packing above; the bf16 tensors are dropped (the oracle leg
-        # reads the e4m3 bytes)
-        f8 = {}
+        # e4m3 copies of the expert weights with per-row scales (fp8 = 1) or 128 x 128
+        # block exponents (fp8 = 2, kept per expert as [E, rows/128, cols/128]): a
+        # load-time step like the packing above; the bf16 tensors are dropped (the
+        # oracle leg reads the e4m3 bytes)
+        f8 = {"block": fp8 == 2}
         for n, sn in (("W13", "s13"), ("W2", "s2"), ("Ws13", "ss13"), ("Ws2", "ss2")):
-            if d.get(n) is not None:
+            if d.get(n) is None:
+                f8[n] = f8[sn] = None
+            elif fp8 == 1:
                 f8[n], f8[sn] = L.quantize_fp8(d[n])
             else:
-                f8[n] = f8[sn] = None
+                f8[n], f8[sn] = L.quantize_fp8_weight_blocks(d[n])
+                if d[n].dim() == 3:
+                    f8[sn] = f8[sn].view(d[n].shape[0], -1, f8[sn].shape[-1])
         torch.cuda.synchronize()
         d["fp8"] = f8
         for n in ("W13", "W2", "Ws13", "Ws2"):
@@ -544,13 +576,15 @@ def run_ours(args, wl, rank, world, local, device):
                    "ms_sequential_unchunked": round(sum(stage_ms.values()), 4)}
 
     hbm, tf_burst, tf_sust, src = peaks()
-    b, f = algorithmic(wl, touched, fused, bool(fp8), bool(fc))
+    b, f = algorithmic(wl, touched, fused, fp8, bool(fc))
     g1 = stage_ms["gemm1"] / 1e3
     achieved = b["gemm1"] / g1 / 1e9
     # GEMM1's own bytes (the FP8 GEMM1 stage also holds the h quantization)
-    qh = (wl.T * wl.k * wl.I * 3 + wl.T * wl.k * 4
-          + (wl.T * wl.I_shared * 3 + wl.T * 4 if wl.I_shared == wl.I else 0)) if fp8 else 0
-    traffic = measured_traffic(wl.name, bool(fp8), b["gemm1"] - qh)
+    R = wl.T * wl.k
+    qh = (R * wl.I * 3 + scale_bytes(R, wl.I, fp8)
+          + (wl.T * wl.I_shared * 3 + scale_bytes(wl.T, wl.I_shared, fp8)
+             if wl.I_shared == wl.I else 0)) if fp8 else 0
+    traffic = measured_traffic(wl.name, fp8, b["gemm1"] - qh)
     stages = {}
     for s_, t in stage_ms.items():
         e = {"ms": round(t, 4)}
@@ -571,15 +605,18 @@ def run_ours(args, wl, rank, world, local, device):
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
         "dtype": "e4m3" if fp8 else "bf16",
         "data": "synthetic (seeded N(0,1) activations, N(0,0.02^2) bf16 weights"
-                + (", quantized to e4m3 at load)" if fp8 else ")"),
+                + ({1: ", quantized to e4m3 at load)",
+                    2: ", quantized to e4m3 in 128x128 blocks at load)"}.get(fp8, ")")),
         "config": config_of(wl, args),
         "e2e": {"value": e2e_value, "unit": "tokens/s", "h2d_bytes_per_step": wl.T * wl.H * 2,
                 "d2h_bytes_per_step": wl.T * wl.H * 2},
         "gpu_launches": launches,
         "roofline": {"bound": "hbm",
-                     "kernel": ("grouped GEMM1 + SwiGLU (tcgen05 kind::f8f6f4) and the h "
-                                "quantization, routed + shared") if fp8 else
-                               "grouped GEMM1 + SwiGLU (tcgen05), routed + shared",
+                     "kernel": {0: "grouped GEMM1 + SwiGLU (tcgen05), routed + shared",
+                                1: "grouped GEMM1 + SwiGLU (tcgen05 kind::f8f6f4) and the h "
+                                   "quantization, routed + shared",
+                                2: "grouped GEMM1 + SwiGLU (tcgen05 kind::mxf8f6f4 block_scale) "
+                                   "and the h block quantization, routed + shared"}[fp8],
                      "achieved": round(achieved, 1), "peak": hbm, "unit": "GB/s",
                      "frac": round(achieved / hbm, 4), "traffic": traffic,
                      "peak_source": f"hbm_gbs of {src}",
@@ -649,7 +686,7 @@ def run_stack(args, wl, rank, world, local, device, L, cfg, ex, W, d):
         "value": wl.T * world * args.steps / (ms / 1e3), "unit": "tokens/s", "n_gpus": world,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms / args.steps,
         "ms_per_layer": ms / args.steps / nl, "higher_is_better": True, "scaling": "weak",
-        "vs_baseline": None, "dtype": "e4m3" if args.precision == "fp8" else "bf16",
+        "vs_baseline": None, "dtype": "bf16" if args.precision == "bf16" else "e4m3",
         "data": "synthetic (seeded N(0,1) activations, N(0,0.02^2) bf16 weights)",
         "config": dict(config_of(wl, args), layers=nl, graph=True,
                        between_layers="unit-gain RMS normalization (moe_rms_norm)"),

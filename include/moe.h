@@ -345,10 +345,10 @@ moe_status moe_expert_ffn_fp8(int32_t rows, int32_t H, int32_t I, int32_t n_expe
  * FP8 quantization with block scales, for activation rows: each 1 x 128 block
  * of in [rows, K] bf16 gets the exponent k = the smallest integer with
  * amax <= 448 * 2^k (k = 0 for an all-zero block, clamped to [-127, 127]),
- * stored as the UE8M0 byte sf[(c / 128) * sf_ld + r] = k + 127, and its
+ * stored as the UE8M0 byte sf[r * sf_ld + c / 128] = k + 127, and its
  * values out[r][c] = e4m3(in[r][c] * 2^-k) (exact scaling, then round to
  * nearest even, saturating at +-448). K a multiple of 128, at most 65536;
- * sf_ld >= rows; in and out 16-byte aligned and not overlapping; all written
+ * sf_ld >= K / 128; in and out 16-byte aligned and not overlapping; all written
  * buffers caller-allocated. Used on token rows and on h inside
  * moe_layer_forward (fp8 = 2).
  */
@@ -365,7 +365,7 @@ moe_status moe_quantize_fp8_weight_blocks(int64_t rows, int32_t K, const uint16_
                                           uint8_t* out, uint8_t* sf, void* stream);
 
 /* Workspace bytes of moe_expert_ffn_fp8_blocks: h [rows, I] bf16, its e4m3
- * copy [rows, I] and its block exponents [I/128][rows], each 256-byte aligned. */
+ * copy [rows, I] and its block exponents [rows][I/128], each 256-byte aligned. */
 size_t moe_expert_ffn_fp8_blocks_workspace_size(int32_t rows, int32_t I);
 
 /*
@@ -374,9 +374,9 @@ size_t moe_expert_ffn_fp8_blocks_workspace_size(int32_t rows, int32_t I);
  *   g|u[r][j] = sum_c x_q[r][c] 2^kx(r, c/128) * W13_q[e][j][c] 2^kw13(e, j/128, c/128),
  *   h[r] = bf16(silu(g) * u), h quantized by moe_quantize_fp8_blocks,
  *   y_perm[r][c] = sum_i h_q[r][i] 2^kh(r, i/128) * W2_q[e][c][i] 2^kw2(e, c/128, i/128),
- * fp32 accumulation on the tensor cores. kx(r, b) is x_sf[b * x_sf_ld + t] with
- * t = x_scale_idx[r] when given (x_q rows are copies of token rows; values in
- * [0, x_sf_ld)), else r (then x_sf_ld >= rows).
+ * fp32 accumulation on the tensor cores. kx(r, b) is x_sf[t * x_sf_ld + b] with
+ * t = x_scale_idx[r] when given (x_q rows are copies of token rows, whose
+ * exponent rows x_sf holds), else r; x_sf_ld >= H / 128.
  * W13_sf [n_experts*2I/128][H/128], W2_sf [n_experts*H/128][I/128] as in
  * moe_weights (fp8 = 2). H and I multiples of 128. ws:
  * moe_expert_ffn_fp8_blocks_workspace_size(rows, I) bytes, 256-byte aligned.

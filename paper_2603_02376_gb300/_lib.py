@@ -279,7 +279,7 @@ def moe_expert_ffn_fp8(rows, H, I, n_experts, x_q, x_scale, x_scale_idx, offsets
 
 def moe_quantize_fp8_blocks(x, out, sf, sf_ld, stream=None) -> None:
     """e4m3 quantization of a bf16 tensor viewed as [rows, K] in 1 x 128 blocks;
-    UE8M0 exponents to sf[(c / 128) * sf_ld + r]."""
+    UE8M0 exponents to sf[r * sf_ld + c / 128]."""
     K = x.shape[-1]
     rows = x.numel() // K
     _check(load().moe_quantize_fp8_blocks(rows, K, _ptr(x), _ptr(out), _ptr(sf), int(sf_ld),
@@ -287,13 +287,13 @@ def moe_quantize_fp8_blocks(x, out, sf, sf_ld, stream=None) -> None:
 
 
 def quantize_fp8_blocks(x, stream=None):
-    """(e4m3 bytes as uint8 of x's shape, uint8 exponents [K / 128, rows]) of a bf16 tensor."""
+    """(e4m3 bytes as uint8 of x's shape, uint8 exponents [rows, K / 128]) of a bf16 tensor."""
     import torch
     K = x.shape[-1]
     rows = x.numel() // K
     q = torch.empty(x.shape, dtype=torch.uint8, device=x.device)
-    sf = torch.empty((K // 128, rows), dtype=torch.uint8, device=x.device)
-    moe_quantize_fp8_blocks(x, q, sf, rows, stream)
+    sf = torch.empty((rows, K // 128), dtype=torch.uint8, device=x.device)
+    moe_quantize_fp8_blocks(x, q, sf, K // 128, stream)
     return q, sf
 
 

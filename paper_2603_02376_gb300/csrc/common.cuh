@@ -104,9 +104,9 @@ struct FfnGroup {
   uint8_t* hq;
   float* hs;
   // Block-scaled FP8 (fp8 and fp8_block): UE8M0 exponents of x's 1 x 128
-  // blocks (x_sf[kb * x_sf_ld + token], the token through x_scale_idx as
+  // blocks (x_sf[token * x_sf_ld + kb], the token through x_scale_idx as
   // above) and of the 128 x 128 blocks of W13 and W2 ([rows / 128][K / 128]);
-  // hsf receives those of h's 1 x 128 blocks (hsf[kb * h_sf_ld + row]).
+  // hsf receives those of h's 1 x 128 blocks (hsf[row * h_sf_ld + kb]).
   bool fp8_block;
   const uint8_t* x_sf;
   long x_sf_ld;
@@ -148,7 +148,7 @@ moe_status launch_quantize_rows(const uint16_t* in, long rows, int K, uint8_t* o
 
 // e4m3 quantization of a bf16 matrix [rows, K] in 1 x 128 blocks (K % 128 == 0):
 // k = the smallest exponent with amax <= 448 * 2^k (0 for a zero block, within
-// [-127, 127]); out[r][c] = e4m3(in[r][c] * 2^-k); sf[(c / 128) * sf_ld + r] = k + 127.
+// [-127, 127]); out[r][c] = e4m3(in[r][c] * 2^-k); sf[r * sf_ld + c / 128] = k + 127.
 moe_status launch_quantize_blocks(const uint16_t* in, long rows, int K, uint8_t* out, uint8_t* sf,
                                   long sf_ld, cudaStream_t s);
 // The same in 128 x 128 blocks (rows % 128 == 0): sf[(r / 128) * (K / 128) + c / 128].

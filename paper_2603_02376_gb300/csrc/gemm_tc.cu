@@ -95,9 +95,16 @@ struct Tile {
   static constexpr int SF_OFF = NA * A_BYTES + B_BYTES;
   static constexpr int SF_BYTES = MX ? ((NA + SF_CB) * 512 + 1023) / 1024 * 1024 : 0;
   static constexpr int STAGE_BYTES = NA * A_BYTES + B_BYTES + SF_BYTES;
-  // ~217 KiB of stages: with the control block, the expert tables (<= 8 KiB)
-  // and the 1 KiB alignment slack this stays under 227 KiB per CTA.
-  static constexpr int STAGES_RAW = (217 * 1024) / STAGE_BYTES;
+  // MX: the producer's staging copy of a unit's exponents for SF_KC k-blocks:
+  // token j's at j * SF_STR (a stride that keeps the per-stage reads of 32
+  // consecutive tokens on distinct banks), then the A tiles' at t * SF_KC.
+  static constexpr int SF_KC = 32;
+  static constexpr int SF_STR = SF_KC + 4;
+  static constexpr int SF_STG_A = NMAX * SF_STR;
+  static constexpr int SF_STG_BYTES = MX ? (SF_STG_A + NA * SF_KC + 15) / 16 * 16 : 0;
+  // ~217 KiB of stages and staging: with the control block, the expert tables
+  // (<= 8 KiB) and the 1 KiB alignment slack this stays under 227 KiB per CTA.
+  static constexpr int STAGES_RAW = (217 * 1024 - SF_STG_BYTES) / STAGE_BYTES;
   static constexpr int STAGES = STAGES_RAW > 12 ? 12 : STAGES_RAW;
   static constexpr int ACC_COLS = TWO_ACC ? 2 * NMAX : NMAX;  // one accumulator (gate | up)
   // MX: each stage's scales live in TMEM columns of their own (4 per image)
@@ -355,7 +362,7 @@ struct GemmArgs {
   const int32_t* b_scale_idx0;
   // Block-scaled FP8 only: UE8M0 exponents of the 128 x 128 weight blocks
   // ([weight rows / 128][K / 128], absolute weight rows) and of the 1 x 128
-  // activation blocks (b_sf[kb * b_sf_ld + row], the row through b_scale_idx0
+  // activation blocks (b_sf[row * b_sf_ld + kb], the row through b_scale_idx0
   // for group 0 when given)
   const uint8_t* a_sf0;
   const uint8_t* a_sf1;
@@ -449,7 +456,8 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~static_cast<uintptr_t>(1023));
-  Ctrl* ctrl = reinterpret_cast<Ctrl*>(smem + TL::STAGES * TL::STAGE_BYTES);
+  uint8_t* sf_stg = smem + TL::STAGES * TL::STAGE_BYTES;  // MX staging (SF_STG_BYTES)
+  Ctrl* ctrl = reinterpret_cast<Ctrl*>(sf_stg + TL::SF_STG_BYTES);
   int* tile_off = reinterpret_cast<int*>(ctrl + 1);
   int* row_off = tile_off + a.n_exp + 1;
   volatile int* abort_flag = &ctrl->abort_flag;
@@ -600,17 +608,64 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
               tma_load_2d(sb + i * (B_BOX * BK * 2), mB, kb * KE, U.row0 + i * B_BOX, full);
           }
         };
-        // MX: this k-block's scales, loaded before the wait for the slot
+        // MX: this k-block's exponents. Every SF_KC k-blocks of the unit the warp
+        // stages the next SF_KC exponents of each token row and of each A tile in
+        // shared memory (one round trip: every lane issues all the 8-byte loads of
+        // its token rows before its first store); the per-stage values then come
+        // from there, not from global memory.
         uint32_t sfa[TL::NA], sfb[NG];
         if constexpr (MX) {
-          const uint8_t* asf = U.grp ? a.a_sf1 : a.a_sf0;
-          const uint8_t* bsf = U.grp ? a.b_sf1 : a.b_sf0;
-          const size_t boff = (size_t)kb * (U.grp ? a.b_sf_ld1 : a.b_sf_ld0);
+          const int kbl = (kb - U.kb0) % TL::SF_KC;
+          if (kbl == 0) {
+            const int kc = min(TL::SF_KC, U.kb1 - kb);
+            const uint8_t* asf = U.grp ? a.a_sf1 : a.a_sf0;
+            const uint8_t* bsf = U.grp ? a.b_sf1 : a.b_sf0;
+            const long ld = U.grp ? a.b_sf_ld1 : a.b_sf_ld0;
+            uint32_t av[TL::NA];
 #pragma unroll
-          for (int t = 0; t < TL::NA; ++t)
-            sfa[t] = asf[(size_t)((wrow + t * a.up_off) / BM) * kblocks + kb];
+            for (int t = 0; t < TL::NA; ++t)
+              av[t] = lane < kc ? asf[(size_t)((wrow + t * a.up_off) / BM) * kblocks + kb + lane]
+                                : 0u;
+            if ((ld & 7) == 0 && ((uintptr_t)bsf & 7) == 0 && (kb & 7) == 0) {
+              // rows of 8-byte multiples: bytes [kb, kb + 8 ceil(kc / 8)) of a row
+              // stay inside it (kb + kc <= K / 128 <= ld)
+              uint2 v[NG][TL::SF_KC / 8];
 #pragma unroll
-          for (int g = 0; g < NG; ++g) sfb[g] = sf_row[g] >= 0 ? bsf[boff + sf_row[g]] : 127u;
+              for (int g = 0; g < NG; ++g)
+#pragma unroll
+                for (int i = 0; i < TL::SF_KC / 8; ++i)
+                  v[g][i] = sf_row[g] >= 0 && 8 * i < kc
+                                ? *reinterpret_cast<const uint2*>(bsf + (size_t)sf_row[g] * ld +
+                                                                  kb + 8 * i)
+                                : make_uint2(0u, 0u);
+#pragma unroll
+              for (int g = 0; g < NG; ++g) {
+                uint32_t* d = reinterpret_cast<uint32_t*>(sf_stg + (32 * g + lane) * TL::SF_STR);
+#pragma unroll
+                for (int i = 0; i < TL::SF_KC / 8; ++i)
+                  if (sf_row[g] >= 0 && 8 * i < kc) {
+                    d[2 * i] = v[g][i].x;
+                    d[2 * i + 1] = v[g][i].y;
+                  }
+              }
+            } else {  // any other stride: byte loads
+#pragma unroll
+              for (int g = 0; g < NG; ++g)
+                if (sf_row[g] >= 0)
+                  for (int i = 0; i < kc; ++i)
+                    sf_stg[(32 * g + lane) * TL::SF_STR + i] = bsf[(size_t)sf_row[g] * ld + kb + i];
+            }
+            if (lane < kc) {
+#pragma unroll
+              for (int t = 0; t < TL::NA; ++t) sf_stg[TL::SF_STG_A + t * TL::SF_KC + lane] = av[t];
+            }
+            __syncwarp();
+          }
+#pragma unroll
+          for (int t = 0; t < TL::NA; ++t) sfa[t] = sf_stg[TL::SF_STG_A + t * TL::SF_KC + kbl];
+#pragma unroll
+          for (int g = 0; g < NG; ++g)
+            sfb[g] = sf_row[g] >= 0 ? sf_stg[(32 * g + lane) * TL::SF_STR + kbl] : 127u;
         }
         int got = 1;
         if (lane == 0) {
@@ -944,7 +999,8 @@ long g_stall_fill = -1;
 template <int MODE, int NMAX, bool MX>
 size_t gemm_smem_bytes(int n_exp) {
   using TL = Tile<MODE, NMAX, MX>;
-  return 1024 + (size_t)TL::STAGES * TL::STAGE_BYTES + sizeof(Ctrl) + 2 * sizeof(int) * (n_exp + 1);
+  return 1024 + (size_t)TL::STAGES * TL::STAGE_BYTES + TL::SF_STG_BYTES + sizeof(Ctrl) +
+         2 * sizeof(int) * (n_exp + 1);
 }
 
 template <int MODE, int NMAX, int Q, bool PK>

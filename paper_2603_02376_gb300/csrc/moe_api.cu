@@ -134,18 +134,18 @@ struct Layout {
   bool fp8_block = false;  // block scales (fp8 = 2) instead of row scales (fp8 = 1)
   uint8_t* x_q;      // [T, H] e4m3 (fp8 only)
   float* x_s;        // [T] row scales of x_q
-  uint8_t* x_sf;     // [H/128][T] block exponents of x_q (block form)
+  uint8_t* x_sf;     // [T][H/128] block exponents of x_q (block form)
   void* x_perm;      // [T*k, H] bf16, or e4m3 bytes (fp8)
   uint16_t* h;       // [T*k, I]
   uint8_t* hq;       // [T*k, I] e4m3 copy of h (fp8 only)
   float* hs;         // [T*k] its row scales
-  uint8_t* hsf;      // [I/128][T*k] its block exponents (block form)
+  uint8_t* hsf;      // [T*k][I/128] its block exponents (block form)
   float* y_perm;     // [T*k, H] fp32
   int32_t* sh_off;   // [2]
   uint16_t* sh_h;    // [T, I_s]
   uint8_t* sh_hq;    // [T, I_s] (fp8 only)
   float* sh_hs;      // [T]
-  uint8_t* sh_hsf;   // [I_s/128][T] (block form)
+  uint8_t* sh_hsf;   // [T][I_s/128] (block form)
   float* sh_y;       // [T, H] fp32 (unfused combine)
   // Combine fused into GEMM2: the gate weight of every packed row, and the fp32
   // [T, H] accumulator the GEMM2s reduce into (the caller's output when it is
@@ -252,12 +252,12 @@ moe_status mark(cudaEvent_t* ev, int i, cudaStream_t s) {
 }
 
 // FP8: rows [t0, t0+Tc) of x -> e4m3 rows of x_q and their scales (per row,
-// or per 1 x 128 block: exponents x_sf[kb * T + t]).
+// or per 1 x 128 block: exponents x_sf[t * H/128 + kb]).
 moe_status quantize_tokens(const moe_config& c, const Layout& L, const uint16_t* x, int t0, int Tc,
                            cudaStream_t s) {
   if (L.fp8_block)
     return launch_quantize_blocks(x + (size_t)t0 * c.H, Tc, c.H, L.x_q + (size_t)t0 * c.H,
-                                  L.x_sf + t0, (long)c.T, s);
+                                  L.x_sf + (size_t)t0 * (c.H / 128), c.H / 128, s);
   return launch_quantize_rows(x + (size_t)t0 * c.H, Tc, c.H, L.x_q + (size_t)t0 * c.H, L.x_s + t0,
                               s);
 }
@@ -336,12 +336,12 @@ FfnGroup routed_group(const moe_config& c, const Layout& L, const moe_weights& w
     g.hq = L.hq + tk * c.I;
     if (L.fp8_block) {
       g.fp8_block = true;
-      g.x_sf = L.x_sf + t0;
-      g.x_sf_ld = c.T;
+      g.x_sf = L.x_sf + (size_t)t0 * (c.H / 128);
+      g.x_sf_ld = c.H / 128;
       g.W13_sf = static_cast<const uint8_t*>(w.W13_scale);
       g.W2_sf = static_cast<const uint8_t*>(w.W2_scale);
-      g.hsf = L.hsf + tk;
-      g.h_sf_ld = (long)c.T * c.k;
+      g.hsf = L.hsf + tk * (c.I / 128);
+      g.h_sf_ld = c.I / 128;
     } else {
       g.x_scale = L.x_s + t0;
       g.W13_scale = static_cast<const float*>(w.W13_scale);
@@ -374,11 +374,11 @@ FfnGroup dense_group(const moe_config& c, const Layout& L, const moe_weights& w,
     if (L.fp8_block) {
       g.fp8_block = true;
       g.x_sf = L.x_sf;
-      g.x_sf_ld = c.T;
+      g.x_sf_ld = c.H / 128;
       g.W13_sf = static_cast<const uint8_t*>(w.Ws13_scale);
       g.W2_sf = static_cast<const uint8_t*>(w.Ws2_scale);
       g.hsf = L.sh_hsf;
-      g.h_sf_ld = c.T;
+      g.h_sf_ld = c.I_shared / 128;
     } else {
       g.x_scale = L.x_s;
       g.W13_scale = static_cast<const float*>(w.Ws13_scale);
@@ -636,7 +636,7 @@ size_t moe_expert_ffn_fp8_blocks_workspace_size(int32_t rows, int32_t I) {
 
 moe_status moe_quantize_fp8_blocks(int64_t rows, int32_t K, const uint16_t* in, uint8_t* out,
                                    uint8_t* sf, int64_t sf_ld, void* stream) {
-  if (rows < 0 || rows > (1LL << 31) || K < 128 || K % 128 || K > 65536 || sf_ld < rows)
+  if (rows < 0 || rows > (1LL << 31) || K < 128 || K % 128 || K > 65536 || sf_ld < K / 128)
     return MOE_ERR_INVALID_ARG;
   if (rows == 0) return MOE_OK;
   if (!in || !out || !sf || !aligned16(in) || !aligned16(out)) return MOE_ERR_INVALID_ARG;
@@ -663,7 +663,7 @@ moe_status moe_expert_ffn_fp8_blocks(int32_t rows, int32_t H, int32_t I, int32_t
                                      const uint8_t* W2_q, const uint8_t* W2_sf, float* y_perm,
                                      void* ws, size_t ws_bytes, void* stream) {
   if (rows < 0 || H < 128 || H % 128 || H > 65536 || I < 128 || I % 128 || I > 65536 ||
-      n_experts < 1 || n_experts > 1024 || x_sf_ld < 1 || (!x_scale_idx && x_sf_ld < rows))
+      n_experts < 1 || n_experts > 1024 || x_sf_ld < H / 128)
     return MOE_ERR_INVALID_ARG;
   if (rows == 0) return MOE_OK;
   if (!x_q || !x_sf || !offsets || !W13_q || !W13_sf || !W2_q || !W2_sf || !y_perm ||
@@ -685,7 +685,7 @@ moe_status moe_expert_ffn_fp8_blocks(int32_t rows, int32_t H, int32_t I, int32_t
   g.h = cv.take<uint16_t>((size_t)rows * I);
   g.hq = cv.take<uint8_t>((size_t)rows * I);
   g.hsf = cv.take<uint8_t>((size_t)(I / 128) * rows);
-  g.h_sf_ld = rows;
+  g.h_sf_ld = I / 128;
   g.y = y_perm;
   g.fp8 = true;
   g.fp8_block = true;

@@ -100,7 +100,7 @@ __global__ void __launch_bounds__(Q_WARPS * 32) quantize_blocks_kernel(
     const int k = block_exponent(m);
     if (act) {
       dst[b * 16 + hl] = quantize8(x, inv_pow2(k));
-      if (hl == 0) sf[(size_t)b * sf_ld + r] = (uint8_t)(k + 127);
+      if (hl == 0) sf[(size_t)r * sf_ld + b] = (uint8_t)(k + 127);
     }
   }
 }

@@ -228,11 +228,11 @@ def test_fp8_block_entry_points_reject_bad_arguments_without_a_gpu(lib):
     QB = lib.moe_quantize_fp8_blocks
     assert QB(16, 100, p, q, q, 16, z) == L.MOE_ERR_INVALID_ARG       # K % 128
     assert QB(16, 64, p, q, q, 16, z) == L.MOE_ERR_INVALID_ARG        # K < 128
-    assert QB(16, 128, p, q, q, 15, z) == L.MOE_ERR_INVALID_ARG       # sf_ld < rows
+    assert QB(16, 256, p, q, q, 1, z) == L.MOE_ERR_INVALID_ARG        # sf_ld < K / 128
     assert QB(16, 128, p, p, q, 16, z) == L.MOE_ERR_INVALID_ARG       # in and out overlap
     assert QB(16, 128, odd, q, q, 16, z) == L.MOE_ERR_INVALID_ARG
     assert QB(16, 128, p, q, z, 16, z) == L.MOE_ERR_INVALID_ARG       # no exponent buffer
-    assert QB(0, 128, z, z, z, 0, z) == L.MOE_OK
+    assert QB(0, 128, z, z, z, 1, z) == L.MOE_OK
     QW = lib.moe_quantize_fp8_weight_blocks
     assert QW(100, 128, p, q, q, z) == L.MOE_ERR_INVALID_ARG          # rows % 128
     assert QW(128, 96, p, q, q, z) == L.MOE_ERR_INVALID_ARG           # K % 128
@@ -240,17 +240,15 @@ def test_fp8_block_entry_points_reject_bad_arguments_without_a_gpu(lib):
     assert QW(128, 128, p, p, q, z) == L.MOE_ERR_INVALID_ARG
     assert QW(0, 128, z, z, z, z) == L.MOE_OK
     F = lib.moe_expert_ffn_fp8_blocks
-    a = lambda ld=16, idx=z: [p, p, ld, idx, p, p, p, p, p, p]    # x_q .. y_perm
+    a = lambda ld=2, idx=z: [p, p, ld, idx, p, p, p, p, p, p]    # x_q .. y_perm
     assert F(16, 100, 128, 1, *a(), q, 1 << 20, z) == L.MOE_ERR_INVALID_ARG     # H % 128
     assert F(16, 256, 96, 1, *a(), q, 1 << 20, z) == L.MOE_ERR_INVALID_ARG      # I % 128
-    assert F(16, 256, 128, 1, *a(ld=8), q, 1 << 20, z) == L.MOE_ERR_INVALID_ARG  # ld < rows
-    # rows reached through x_scale_idx may use a shorter exponent stride (the arguments
-    # pass; the misaligned workspace is what fails)
-    assert F(16, 256, 128, 1, *a(ld=8, idx=p), ctypes.c_void_p(0x100010), 1 << 20, z) == \
+    assert F(16, 256, 128, 1, *a(ld=1), q, 1 << 20, z) == L.MOE_ERR_INVALID_ARG  # ld < H / 128
+    assert F(16, 256, 128, 1, *a(idx=p), ctypes.c_void_p(0x100010), 1 << 20, z) == \
         L.MOE_ERR_WORKSPACE
     assert F(16, 256, 128, 1, *a(), z, 0, z) == L.MOE_ERR_WORKSPACE
     assert F(16, 256, 128, 1, z, *a()[1:], q, 1 << 20, z) == L.MOE_ERR_INVALID_ARG
-    assert F(0, 256, 128, 1, z, z, 1, z, z, z, z, z, z, z, z, 0, z) == L.MOE_OK
+    assert F(0, 256, 128, 1, z, z, 2, z, z, z, z, z, z, z, z, 0, z) == L.MOE_OK
     n = lib.moe_expert_ffn_fp8_blocks_workspace_size(16, 256)
     assert n >= 16 * 256 * 3 + 2 * 16 and n % 256 == 0
     # layer forward: block scales need whole 128-blocks and the exponent arrays

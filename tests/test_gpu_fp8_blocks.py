@@ -66,17 +66,17 @@ def test_quantize_fp8_blocks_bit_exact(rows, K, std, ld_extra):
         x[1, :128] = 0                             # an all-zero block: k = 0, codes 0
         x[2, :] = x[2, :] * 1e-3                   # blocks reaching e4m3 subnormals ...
         x[2, 5] = 300.0                            # ... under one large element
-    ld = rows + ld_extra
+    ld = K // 128 + ld_extra
     q = torch.empty((rows, K), dtype=torch.uint8, device=DEV)
-    sf = torch.full((K // 128, ld), 0xEE, dtype=torch.uint8, device=DEV)
+    sf = torch.full((rows, ld), 0xEE, dtype=torch.uint8, device=DEV)
     L.moe_quantize_fp8_blocks(x, q, sf, ld)
     torch.cuda.synchronize()
     q_ref, k_ref = O.quantize_blocks_e4m3(f64(x), 1)
-    np.testing.assert_array_equal(exps(sf[:, :rows]).T, k_ref)
+    np.testing.assert_array_equal(exps(sf[:, :K // 128]), k_ref)
     np.testing.assert_array_equal(e4m3(q), q_ref)
-    assert (sf[:, rows:] == 0xEE).all()            # the stride's slack is untouched
-    q2, sf2 = L.quantize_fp8_blocks(x)             # the allocating form: [K / 128, rows]
-    assert torch.equal(q2, q) and torch.equal(sf2, sf[:, :rows])
+    assert (sf[:, K // 128:] == 0xEE).all()        # the stride's slack is untouched
+    q2, sf2 = L.quantize_fp8_blocks(x)             # the allocating form: [rows, K / 128]
+    assert torch.equal(q2, q) and torch.equal(sf2, sf[:, :K // 128])
 
 
 @pytest.mark.parametrize("rows,K,std", [(128, 128, 1.0), (256, 7168, 0.02), (4096, 2048, 0.02),
@@ -127,10 +127,11 @@ def test_expert_ffn_fp8_blocks(counts, H, Iw, token_scales):
         xq_tok, xsf = L.quantize_fp8_blocks(tok)
         xq = xq_tok[src.long()].contiguous()
         xp = tok[src.long()]
-        sidx, ld = src, n_tok
+        sidx = src
     else:
         xq, xsf = L.quantize_fp8_blocks(xp)
-        sidx, ld = None, rows
+        sidx = None
+    ld = H // 128
     y = torch.full((rows, H), -12345.0, dtype=torch.float32, device=DEV)
     ws = torch.zeros(L.moe_expert_ffn_fp8_blocks_workspace_size(rows, Iw), dtype=torch.uint8,
                      device=DEV)
@@ -141,7 +142,7 @@ def test_expert_ffn_fp8_blocks(counts, H, Iw, token_scales):
     o_hs = align256(o_hq + rows * Iw)
     h = ws[:rows * Iw * 2].view(torch.bfloat16).view(rows, Iw)
     hq = ws[o_hq:o_hq + rows * Iw].view(rows, Iw)
-    hsf = ws[o_hs:o_hs + (Iw // 128) * rows].view(Iw // 128, rows)
+    hsf = ws[o_hs:o_hs + (Iw // 128) * rows].view(rows, Iw // 128)
     n = int(offs[-1])
     xh = f64(xp)
     for e in range(E):
@@ -170,7 +171,7 @@ def test_expert_ffn_fp8_blocks(counts, H, Iw, token_scales):
         assert (diff == 0).mean() > 0.98, f"expert {e}: too many h rounding flips"
         # block quantization of the kernel's own h: bit-exact
         hq_o, kh_o = O.quantize_blocks_e4m3(hg, 1)
-        np.testing.assert_array_equal(exps(hsf[:, a:b]).T, kh_o)
+        np.testing.assert_array_equal(exps(hsf[a:b]), kh_o)
         np.testing.assert_array_equal(e4m3(hq[a:b]), hq_o)
         # GEMM2 given that quantized h: within the fp32 summation bound
         y_ref = O.fp8_block_linear(hq_o, kh_o, W2e, k2e)

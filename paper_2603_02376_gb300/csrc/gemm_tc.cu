@@ -27,7 +27,10 @@
 //              16-column chunks): tcgen05.ld the accumulator; GEMM1 applies
 //              SwiGLU and stores h in bf16 (the operand of GEMM2), GEMM2
 //              stores y in fp32 (summed by combine, or added into the output
-//              by the fused combine).
+//              by the fused combine);
+//   warp 10    block-scaled FP8 only: the stage's UE8M0 exponents as scale
+//              images in shared memory, which the MMA thread copies to TMEM
+//              (tcgen05.cp) ahead of block_scale MMAs.
 // For SwiGLU the gate and up tiles of the same 128 features are two MMAs into
 // two TMEM column ranges, so one thread holds both g and u of its feature.
 // When two accumulators fit in TMEM's 512 columns they alternate, so the
@@ -57,6 +60,7 @@ constexpr int UMMA_K = 16;        // K of one tcgen05.mma kind::f16
 constexpr int B_BOX = 16;         // token rows per TMA box (tile remainders)
 constexpr int B_BIG = 64;         // token rows per TMA box (bulk of tiles of >= 64 rows)
 constexpr int NUM_THREADS = 320;  // 10 warps: producer, MMA, 8 epilogue
+constexpr int NUM_WARPS_MX = 11;  // block-scaled FP8: and a scale warp
 constexpr uint64_t WAIT_LIMIT_NS = 2000000000ull;  // default limit of every barrier wait
 
 
@@ -441,8 +445,10 @@ __device__ __forceinline__ Unit decode_unit(int u, const int* tile_off, const in
 
 // ------------------------------------------------------------------ kernel
 
+constexpr int threads_of(int q) { return q == Q_BLOCK ? NUM_WARPS_MX * 32 : NUM_THREADS; }
+
 template <int MODE, int NMAX, int Q, bool PK>
-__global__ void __launch_bounds__(NUM_THREADS, 1)
+__global__ void __launch_bounds__(threads_of(Q), 1)
     grouped_gemm_kernel(const __grid_constant__ CUtensorMap tmA0,
                         const __grid_constant__ CUtensorMap tmB0,
                         const __grid_constant__ CUtensorMap tmA1,
@@ -467,7 +473,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < TL::STAGES; ++s) {
-      mbar_init(smem_u32(&ctrl->full[s]), 1);
+      mbar_init(smem_u32(&ctrl->full[s]), MX ? 2 : 1);  // MX: the producer and the scale warp
       mbar_init(smem_u32(&ctrl->empty[s]), 1);
     }
     for (int s = 0; s < TL::ACC_STAGES; ++s) {
@@ -573,18 +579,6 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
           const int r = (lane + 32 * h) * 4 + j;
           gr[h][j] = gather && r < n_pad ? a.gather0[U.row0 + min(r, U.m - 1)] : 0;
         }
-      // MX: lane l fetches the block scales of token columns j = 32 g + l of the
-      // tile (the activation row of column j: sf_row[g]; -1 past the valid rows)
-      constexpr int NG = MX ? (NMAX + 31) / 32 : 1;
-      int sf_row[NG];
-      if constexpr (MX) {
-        const int32_t* bidx = U.grp ? nullptr : a.b_scale_idx0;
-#pragma unroll
-        for (int g = 0; g < NG; ++g) {
-          const int j = 32 * g + lane;
-          sf_row[g] = j < U.m ? (bidx ? bidx[U.row0 + j] : U.row0 + j) : -1;
-        }
-      }
       for (int kb = U.kb0; kb < U.kb1; ++kb) {
         const uint32_t full = smem_u32(&ctrl->full[stage]);
         const uint32_t sa = smem_u32(smem + stage * TL::STAGE_BYTES);
@@ -608,65 +602,6 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
               tma_load_2d(sb + i * (B_BOX * BK * 2), mB, kb * KE, U.row0 + i * B_BOX, full);
           }
         };
-        // MX: this k-block's exponents. Every SF_KC k-blocks of the unit the warp
-        // stages the next SF_KC exponents of each token row and of each A tile in
-        // shared memory (one round trip: every lane issues all the 8-byte loads of
-        // its token rows before its first store); the per-stage values then come
-        // from there, not from global memory.
-        uint32_t sfa[TL::NA], sfb[NG];
-        if constexpr (MX) {
-          const int kbl = (kb - U.kb0) % TL::SF_KC;
-          if (kbl == 0) {
-            const int kc = min(TL::SF_KC, U.kb1 - kb);
-            const uint8_t* asf = U.grp ? a.a_sf1 : a.a_sf0;
-            const uint8_t* bsf = U.grp ? a.b_sf1 : a.b_sf0;
-            const long ld = U.grp ? a.b_sf_ld1 : a.b_sf_ld0;
-            uint32_t av[TL::NA];
-#pragma unroll
-            for (int t = 0; t < TL::NA; ++t)
-              av[t] = lane < kc ? asf[(size_t)((wrow + t * a.up_off) / BM) * kblocks + kb + lane]
-                                : 0u;
-            if ((ld & 7) == 0 && ((uintptr_t)bsf & 7) == 0 && (kb & 7) == 0) {
-              // rows of 8-byte multiples: bytes [kb, kb + 8 ceil(kc / 8)) of a row
-              // stay inside it (kb + kc <= K / 128 <= ld)
-              uint2 v[NG][TL::SF_KC / 8];
-#pragma unroll
-              for (int g = 0; g < NG; ++g)
-#pragma unroll
-                for (int i = 0; i < TL::SF_KC / 8; ++i)
-                  v[g][i] = sf_row[g] >= 0 && 8 * i < kc
-                                ? *reinterpret_cast<const uint2*>(bsf + (size_t)sf_row[g] * ld +
-                                                                  kb + 8 * i)
-                                : make_uint2(0u, 0u);
-#pragma unroll
-              for (int g = 0; g < NG; ++g) {
-                uint32_t* d = reinterpret_cast<uint32_t*>(sf_stg + (32 * g + lane) * TL::SF_STR);
-#pragma unroll
-                for (int i = 0; i < TL::SF_KC / 8; ++i)
-                  if (sf_row[g] >= 0 && 8 * i < kc) {
-                    d[2 * i] = v[g][i].x;
-                    d[2 * i + 1] = v[g][i].y;
-                  }
-              }
-            } else {  // any other stride: byte loads
-#pragma unroll
-              for (int g = 0; g < NG; ++g)
-                if (sf_row[g] >= 0)
-                  for (int i = 0; i < kc; ++i)
-                    sf_stg[(32 * g + lane) * TL::SF_STR + i] = bsf[(size_t)sf_row[g] * ld + kb + i];
-            }
-            if (lane < kc) {
-#pragma unroll
-              for (int t = 0; t < TL::NA; ++t) sf_stg[TL::SF_STG_A + t * TL::SF_KC + lane] = av[t];
-            }
-            __syncwarp();
-          }
-#pragma unroll
-          for (int t = 0; t < TL::NA; ++t) sfa[t] = sf_stg[TL::SF_STG_A + t * TL::SF_KC + kbl];
-#pragma unroll
-          for (int g = 0; g < NG; ++g)
-            sfb[g] = sf_row[g] >= 0 ? sf_stg[(32 * g + lane) * TL::SF_STR + kbl] : 127u;
-        }
         int got = 1;
         if (lane == 0) {
           got = wait_bounded(smem_u32(&ctrl->empty[stage]), phase ^ 1, abort_flag, err,
@@ -674,39 +609,12 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
                     ? 1
                     : 0;
           if (got && blockIdx.x == 0 && fills == a.stall_fill) got = 2;  // skip this fill
-          if constexpr (!MX) {
-            if (got == 1) issue();
-          }
+          if (got == 1) issue();
         }
         got = __shfl_sync(0xffffffffu, got, 0);
         if (!got) {
           ok = false;
           break;
-        }
-        if constexpr (MX) {
-          // scale images of the stage (every byte of a word holds the scale), made
-          // visible to the tensor core's reads before lane 0 arms the barrier
-          if (got == 1) {
-            uint8_t* sf = smem + stage * TL::STAGE_BYTES + TL::SF_OFF;
-#pragma unroll
-            for (int t = 0; t < TL::NA; ++t) {
-              const uint32_t v = sfa[t] * 0x01010101u;
-              *reinterpret_cast<uint4*>(sf + t * 512 + lane * 16) = make_uint4(v, v, v, v);
-            }
-#pragma unroll
-            for (int c = 0; c < TL::SF_CB; ++c) {
-              uint32_t w[4];
-#pragma unroll
-              for (int q = 0; q < 4; ++q)
-                w[q] = (4 * c + q < NG ? sfb[min(4 * c + q, NG - 1)] : 127u) * 0x01010101u;
-              *reinterpret_cast<uint4*>(sf + (TL::NA + c) * 512 + lane * 16) =
-                  make_uint4(w[0], w[1], w[2], w[3]);
-            }
-            asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-          }
-          __syncwarp();
-          if (lane == 0 && got == 1) issue();
-          __syncwarp();
         }
         if (gather && got == 1) {
 #pragma unroll
@@ -820,7 +728,123 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
         }
       }
     }
-  } else {
+  } else if (MX && warp == NUM_WARPS_MX - 1) {
+    // ------------------------------------------------------------------ scale warp
+    // Block-scaled FP8 only. Per stage, once the slot is free: the UE8M0
+    // exponents of the stage's A tiles and token rows, written as the 512-byte
+    // images tcgen05.cp expects (every byte of a word holds the exponent) and
+    // made visible to the tensor core's reads, then one arrive on the stage's
+    // full barrier (its second arrival besides the producer's). Every SF_KC
+    // k-blocks of a unit the warp first stages the next SF_KC exponents of each
+    // token row and A tile in shared memory, every lane issuing all the 8-byte
+    // loads of its token rows before its first store (one round trip), so the
+    // per-stage values come from shared memory. Lane l holds token columns
+    // j = 32 g + l of the tile (activation row sf_row[g]; -1 past the valid rows).
+    constexpr int NG = MX ? (NMAX + 31) / 32 : 1;
+    int stage = 0;
+    uint32_t phase = 0;
+    bool ok = true;
+    for (int u = blockIdx.x; u < total_units && ok; u += gridDim.x) {
+      const Unit U = decode_unit<NMAX>(u, tile_off, row_off, a, units1, kblocks);
+      const int wrow = U.grp ? U.fb * TL::FEAT : (a.e_begin + U.e) * a.w_rows0 + U.fb * TL::FEAT;
+      int sf_row[NG];
+      {
+        const int32_t* bidx = U.grp ? nullptr : a.b_scale_idx0;
+#pragma unroll
+        for (int g = 0; g < NG; ++g) {
+          const int j = 32 * g + lane;
+          sf_row[g] = j < U.m ? (bidx ? bidx[U.row0 + j] : U.row0 + j) : -1;
+        }
+      }
+      for (int kb = U.kb0; kb < U.kb1; ++kb) {
+        uint32_t sfa[TL::NA], sfb[NG];
+        const int kbl = (kb - U.kb0) % TL::SF_KC;
+        if (kbl == 0) {
+          const int kc = min(TL::SF_KC, U.kb1 - kb);
+          const uint8_t* asf = U.grp ? a.a_sf1 : a.a_sf0;
+          const uint8_t* bsf = U.grp ? a.b_sf1 : a.b_sf0;
+          const long ld = U.grp ? a.b_sf_ld1 : a.b_sf_ld0;
+          uint32_t av[TL::NA];
+#pragma unroll
+          for (int t = 0; t < TL::NA; ++t)
+            av[t] = lane < kc ? asf[(size_t)((wrow + t * a.up_off) / BM) * kblocks + kb + lane]
+                              : 0u;
+          if ((ld & 7) == 0 && ((uintptr_t)bsf & 7) == 0 && (kb & 7) == 0) {
+            // rows of 8-byte multiples: bytes [kb, kb + 8 ceil(kc / 8)) of a row
+            // stay inside it (kb + kc <= K / 128 <= ld)
+            uint2 v[NG][TL::SF_KC / 8];
+#pragma unroll
+            for (int g = 0; g < NG; ++g)
+#pragma unroll
+              for (int i = 0; i < TL::SF_KC / 8; ++i)
+                v[g][i] = sf_row[g] >= 0 && 8 * i < kc
+                              ? *reinterpret_cast<const uint2*>(bsf + (size_t)sf_row[g] * ld +
+                                                                kb + 8 * i)
+                              : make_uint2(0u, 0u);
+#pragma unroll
+            for (int g = 0; g < NG; ++g) {
+              uint32_t* d = reinterpret_cast<uint32_t*>(sf_stg + (32 * g + lane) * TL::SF_STR);
+#pragma unroll
+              for (int i = 0; i < TL::SF_KC / 8; ++i)
+                if (sf_row[g] >= 0 && 8 * i < kc) {
+                  d[2 * i] = v[g][i].x;
+                  d[2 * i + 1] = v[g][i].y;
+                }
+            }
+          } else {  // any other stride: byte loads
+#pragma unroll
+            for (int g = 0; g < NG; ++g)
+              if (sf_row[g] >= 0)
+                for (int i = 0; i < kc; ++i)
+                  sf_stg[(32 * g + lane) * TL::SF_STR + i] = bsf[(size_t)sf_row[g] * ld + kb + i];
+          }
+          if (lane < kc) {
+#pragma unroll
+            for (int t = 0; t < TL::NA; ++t) sf_stg[TL::SF_STG_A + t * TL::SF_KC + lane] = av[t];
+          }
+          __syncwarp();
+        }
+#pragma unroll
+        for (int t = 0; t < TL::NA; ++t) sfa[t] = sf_stg[TL::SF_STG_A + t * TL::SF_KC + kbl];
+#pragma unroll
+        for (int g = 0; g < NG; ++g)
+          sfb[g] = sf_row[g] >= 0 ? sf_stg[(32 * g + lane) * TL::SF_STR + kbl] : 127u;
+        int got = 1;
+        if (lane == 0)
+          got = wait_bounded(smem_u32(&ctrl->empty[stage]), phase ^ 1, abort_flag, err,
+                             a.wait_limit_ns)
+                    ? 1
+                    : 0;
+        got = __shfl_sync(0xffffffffu, got, 0);
+        if (!got) {
+          ok = false;
+          break;
+        }
+        uint8_t* sf = smem + stage * TL::STAGE_BYTES + TL::SF_OFF;
+#pragma unroll
+        for (int t = 0; t < TL::NA; ++t) {
+          const uint32_t v = sfa[t] * 0x01010101u;
+          *reinterpret_cast<uint4*>(sf + t * 512 + lane * 16) = make_uint4(v, v, v, v);
+        }
+#pragma unroll
+        for (int c = 0; c < TL::SF_CB; ++c) {
+          uint32_t w[4];
+#pragma unroll
+          for (int q = 0; q < 4; ++q)
+            w[q] = (4 * c + q < NG ? sfb[min(4 * c + q, NG - 1)] : 127u) * 0x01010101u;
+          *reinterpret_cast<uint4*>(sf + (TL::NA + c) * 512 + lane * 16) =
+              make_uint4(w[0], w[1], w[2], w[3]);
+        }
+        asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+        __syncwarp();
+        if (lane == 0) mbar_arrive(smem_u32(&ctrl->full[stage]));
+        if (++stage == TL::STAGES) {
+          stage = 0;
+          phase ^= 1;
+        }
+      }
+    }
+  } else if (warp < 10) {
     // ------------------------------------------------------------------ epilogue
     // Two warps per TMEM lane quarter: warp w reads lanes 32 * (w % 4) .. + 31
     // and the 16-column chunks c0 = 16 * half, 16 * half + 32, ... of a unit.
@@ -1012,7 +1036,7 @@ moe_status launch_gemm(const CUtensorMap& A0, const CUtensorMap& B0, const CUten
   if (cudaFuncSetAttribute(grouped_gemm_kernel<MODE, NMAX, Q, PK>,
                            cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) != cudaSuccess)
     return MOE_ERR_CUDA;
-  grouped_gemm_kernel<MODE, NMAX, Q, PK><<<num_sms(), NUM_THREADS, smem, s>>>(A0, B0, A1, B1,
+  grouped_gemm_kernel<MODE, NMAX, Q, PK><<<num_sms(), threads_of(Q), smem, s>>>(A0, B0, A1, B1,
                                                                               B0big, B1big, args);
   note_launch();
   return launch_status();

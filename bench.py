@@ -69,7 +69,9 @@ def parse():
                         "experts, H=7168, E=256, top-8 uniform routing, T in 1024..65536; one JSON "
                         "line with the HBM GB/s of the permutation, dispatch and combine kernels")
     p.add_argument("--no-cpu-baseline", action="store_true")
-    p.add_argument("--cpu-tokens", type=int, default=128, help="oracle sample size (tokens)")
+    p.add_argument("--cpu-tokens", type=int, default=None,
+                   help="oracle sample size (tokens); default 128, or 8 with --precision "
+                        "fp8-block, whose oracle dequantizes each touched expert in full")
     return p.parse_args()
 
 
@@ -352,7 +354,7 @@ def run_reference(args, wl, rank, world, device):
     if wl.balance != "none":
         L.load()
         calibrate(L, wl, d, device)
-    n = max(1, args.cpu_tokens // 2)
+    n = max(1, (args.cpu_tokens or 128) // 2)
     for s in range(args.warmup):
         oracle_tokens_per_s(wl, d, I.sample_tokens(wl.T, n, 100 + s).numpy())
     times = []
@@ -633,7 +635,8 @@ def run_ours(args, wl, rank, world, local, device):
     if dispatch_fusion:
         line["dispatch_fusion"] = dispatch_fusion
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        line["cpu_baseline"] = cpu_baseline(wl, d, args.cpu_tokens)
+        n_cpu = args.cpu_tokens or (8 if args.precision == "fp8-block" else 128)
+        line["cpu_baseline"] = cpu_baseline(wl, d, n_cpu)
     if rank == 0:
         print(json.dumps(line), flush=True)
 

@@ -120,6 +120,9 @@ struct FfnGroup {
   float* comb_out;
   const int32_t* comb_tok;
   const float* comb_w;
+  // Dynamic unit scheduling (two ints, 0 before the first launch that uses them;
+  // launches sharing them must run one after another): null = static.
+  int* sched;
 };
 
 // Routed group plus an optional dense group (the shared expert, same I) in one

@@ -16,8 +16,12 @@
 // a launch needs no host-side knowledge of the routing. A launch may carry a
 // second operand group: one dense segment with its own weights and
 // activations (the shared expert), whose units run in the same persistent
-// grid as the routed ones. A persistent grid (one CTA per SM) walks the units
-// round-robin. Warp roles:
+// grid as the routed ones. A persistent grid (one CTA per SM) runs the units:
+// each CTA's producer takes the next unit index from a global counter as it
+// becomes free (so the units in flight are consecutive ones, sharing token and
+// weight tiles in L2, however unequal their sizes), or, without a counter,
+// round-robin; it announces each unit to the CTA's other roles through a
+// small ring in shared memory. Warp roles:
 //   warp 0     TMA producer: weight tile(s) 128 x 64 and token rows 16 x 64
 //              per stage into a STAGES-deep ring (128-byte swizzle);
 //   warp 1     MMA issuer (one thread): 4 x tcgen05.mma (K = 16 each) per stage,
@@ -124,12 +128,19 @@ struct Tile {
   static_assert(SF_OFF % 1024 == 0 && STAGE_BYTES % 1024 == 0, "stage alignment");
 };
 
+constexpr int UNIT_RING = 8;  // units announced ahead by the producer (a power of two)
+
 struct Ctrl {
   uint64_t full[12];
   uint64_t empty[12];
   uint64_t acc_full[2];
   uint64_t acc_empty[2];
   uint64_t drain;
+  // The producer announces each unit this CTA runs (its index, or an index
+  // past the last unit to stop) in unit_ring; the other roles read it there.
+  uint64_t unit_full[UNIT_RING];
+  uint64_t unit_empty[UNIT_RING];
+  int unit_ring[UNIT_RING];
   uint32_t tmem_base;
   int abort_flag;
 };
@@ -381,6 +392,13 @@ struct GemmArgs {
   float* comb_out1;
   const int32_t* comb_tok0;
   const float* comb_w0;
+  // Dynamic unit scheduling: sched[0] hands out unit indices (atomicAdd) to the
+  // CTAs' producers as they become free, so the units running at one time are
+  // consecutive ones whatever their sizes; sched[1] counts exited CTAs, and the
+  // last one to exit sets both back to 0 for the next launch. Both must be 0 at
+  // the first launch; launches sharing them must not overlap in time. Null:
+  // CTA b runs units b, b + grid, b + 2 grid, ...
+  int* sched;
   uint64_t wait_limit_ns;  // limit of each barrier wait
   long stall_fill;         // testing: CTA 0 never issues this fill (-1 = none), so the
                            // MMA's wait on it runs out and the abort path is exercised
@@ -481,6 +499,12 @@ __global__ void __launch_bounds__(threads_of(Q), 1)
       mbar_init(smem_u32(&ctrl->acc_empty[s]), 8);  // one arrive per epilogue warp
     }
     mbar_init(smem_u32(&ctrl->drain), 1);
+    // readers of each announced unit: the MMA thread, the 8 epilogue warps and
+    // (block-scaled FP8) the scale warp
+    for (int r = 0; r < UNIT_RING; ++r) {
+      mbar_init(smem_u32(&ctrl->unit_full[r]), 1);
+      mbar_init(smem_u32(&ctrl->unit_empty[r]), MX ? 10 : 9);
+    }
     ctrl->abort_flag = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
@@ -537,6 +561,17 @@ __global__ void __launch_bounds__(threads_of(Q), 1)
   const int kblocks = a.K / KE;
   const int units1 = a.rows1 > 0 ? ((a.rows1 + NMAX - 1) / NMAX) * a.n_fb * a.k_splits : 0;
   const int total_units = units1 + tile_off[a.n_exp] * a.n_fb;
+  // The j-th unit of this CTA as announced by the producer (one lane of a role
+  // calls this): its index, or -1 when the wait gave up (abort / timeout).
+  auto next_unit = [&](int j) -> int {
+    const int r = j & (UNIT_RING - 1);
+    if (!wait_bounded(smem_u32(&ctrl->unit_full[r]), (uint32_t)((j / UNIT_RING) & 1), abort_flag,
+                      err, a.wait_limit_ns))
+      return -1;
+    const int u = reinterpret_cast<volatile int*>(ctrl->unit_ring)[r];
+    mbar_arrive(smem_u32(&ctrl->unit_empty[r]));
+    return u;
+  };
 
   if (warp == 0) {
     // ------------------------------------------------------------------ producer
@@ -557,7 +592,31 @@ __global__ void __launch_bounds__(threads_of(Q), 1)
     uint32_t phase = 0;
     long fills = 0;
     bool ok = true;
-    for (int u = blockIdx.x; u < total_units && ok; u += gridDim.x) {
+    // lane 0 takes the next unit one unit ahead, so the atomic's round trip
+    // overlaps the current unit's loads
+    int u_next = 0;
+    if (lane == 0) u_next = a.sched ? atomicAdd(a.sched, 1) : (int)blockIdx.x;
+    for (int j = 0; ok; ++j) {
+      int u = u_next, pub = 1;
+      if (lane == 0) {  // announce unit j (its slot is free once every reader took unit j - 8)
+        const int r = j & (UNIT_RING - 1);
+        pub = wait_bounded(smem_u32(&ctrl->unit_empty[r]), (uint32_t)(((j / UNIT_RING) & 1) ^ 1),
+                           abort_flag, err, a.wait_limit_ns)
+                  ? 1
+                  : 0;
+        if (pub) {
+          reinterpret_cast<volatile int*>(ctrl->unit_ring)[r] = u;
+          mbar_arrive(smem_u32(&ctrl->unit_full[r]));
+          if (u < total_units) u_next = a.sched ? atomicAdd(a.sched, 1) : u + (int)gridDim.x;
+        }
+      }
+      pub = __shfl_sync(0xffffffffu, pub, 0);
+      u = __shfl_sync(0xffffffffu, u, 0);
+      if (!pub) {
+        ok = false;
+        break;
+      }
+      if (u >= total_units) break;
       const Unit U = decode_unit<NMAX>(u, tile_off, row_off, a, units1, kblocks);
       const CUtensorMap* mA = U.grp ? &tmA1 : &tmA0;
       const CUtensorMap* mB = U.grp ? &tmB1 : &tmB0;
@@ -650,9 +709,14 @@ __global__ void __launch_bounds__(threads_of(Q), 1)
       // ---------------------------------------------------------------- MMA issuer
       int stage = 0;
       uint32_t phase = 0;
-      int j = 0;  // units of this CTA so far: accumulator j % ACC_STAGES
       bool ok = true, issued = false;
-      for (int u = blockIdx.x; u < total_units && ok; u += gridDim.x, ++j) {
+      for (int j = 0; ok; ++j) {  // j: units of this CTA so far (accumulator j % ACC_STAGES)
+        const int u = next_unit(j);
+        if (u < 0) {
+          ok = false;
+          break;
+        }
+        if (u >= total_units) break;
         const Unit U = decode_unit<NMAX>(u, tile_off, row_off, a, units1, kblocks);
         const int n_pad = (U.m + 15) & ~15;
         const uint32_t idesc = MX ? idesc_mx(n_pad) : F8 ? idesc_e4m3(n_pad) : idesc_bf16(n_pad);
@@ -744,7 +808,11 @@ __global__ void __launch_bounds__(threads_of(Q), 1)
     int stage = 0;
     uint32_t phase = 0;
     bool ok = true;
-    for (int u = blockIdx.x; u < total_units && ok; u += gridDim.x) {
+    for (int j = 0; ok; ++j) {
+      int u = 0;
+      if (lane == 0) u = next_unit(j);
+      u = __shfl_sync(0xffffffffu, u, 0);
+      if (u < 0 || u >= total_units) break;
       const Unit U = decode_unit<NMAX>(u, tile_off, row_off, a, units1, kblocks);
       const int wrow = U.grp ? U.fb * TL::FEAT : (a.e_begin + U.e) * a.w_rows0 + U.fb * TL::FEAT;
       int sf_row[NG];
@@ -850,8 +918,11 @@ __global__ void __launch_bounds__(threads_of(Q), 1)
     // and the 16-column chunks c0 = 16 * half, 16 * half + 32, ... of a unit.
     const int q = warp & 3;  // TMEM lane quarter this warp may access
     const int half = (warp - 2) >> 2;
-    int j = 0;
-    for (int u = blockIdx.x; u < total_units; u += gridDim.x, ++j) {
+    for (int j = 0;; ++j) {
+      int u = 0;
+      if (lane == 0) u = next_unit(j);
+      u = __shfl_sync(0xffffffffu, u, 0);
+      if (u < 0 || u >= total_units) break;
       const Unit U = decode_unit<NMAX>(u, tile_off, row_off, a, units1, kblocks);
       const int as = j % TL::ACC_STAGES;
       const uint32_t acc_par = (uint32_t)((j / TL::ACC_STAGES) & 1);
@@ -984,6 +1055,15 @@ __global__ void __launch_bounds__(threads_of(Q), 1)
                  "r"(TL::TMEM_COLS)
                  : "memory");
   }
+  if (a.sched && threadIdx.x == 0) {
+    // every unit index this CTA will ever take has been taken: the last CTA
+    // out resets the scheduler for the next launch
+    __threadfence();
+    if (atomicAdd(a.sched + 1, 1) == (int)gridDim.x - 1) {
+      atomicExch(a.sched, 0);
+      atomicExch(a.sched + 1, 0);
+    }
+  }
 }
 
 // ------------------------------------------------------------------ host side
@@ -1107,6 +1187,7 @@ moe_status run_ffn(const FfnGroup& g0, const FfnGroup* g1, int H, int I, cudaStr
   args.a1_packed = (pk && g1) ? static_cast<const uint16_t*>(g1->W13) : nullptr;
   args.wait_limit_ns = g_wait_limit_ns;
   args.stall_fill = g_stall_fill;
+  args.sched = g0.sched;  // GEMM1 and GEMM2 run one after the other on `s`
   args.offsets = g0.offsets;
   args.rows0 = g0.rows;
   args.e_begin = g0.e_begin;

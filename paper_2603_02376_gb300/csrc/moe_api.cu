@@ -153,6 +153,10 @@ struct Layout {
   bool fuse_combine = false;
   float* row_w;      // [T*k]
   float* acc;        // [T, H] or null (= the fp32 output)
+  // The expert GEMMs' dynamic unit scheduler (two ints): zeroed at the start
+  // of each forward; every launch leaves it at 0 (all of a forward's expert
+  // GEMMs run in order on the caller's stream).
+  int32_t* sched;
   size_t bytes = 0;
 };
 
@@ -207,6 +211,7 @@ Layout carve(const moe_config& c, const moe_exec& ex, void* ws) {
   L.sh_hsf = (c.I_shared && L.fp8_block) ? cv.take<uint8_t>((size_t)(c.I_shared / 128) * T)
                                          : nullptr;
   L.sh_y = (c.I_shared && !L.fuse_combine) ? cv.take<float>(T * c.H) : nullptr;
+  L.sched = cv.take<int32_t>(2);
   L.bytes = align_up(cv.off, 256);
   return L;
 }
@@ -307,6 +312,7 @@ FfnGroup routed_group(const moe_config& c, const Layout& L, const moe_weights& w
   FfnGroup g{};
   g.rows = Tc * c.k;
   g.offsets = L.offsets + (size_t)ci * (c.E + 1);
+  g.sched = L.sched;
   g.n_experts = c.E;
   g.e_begin = e0;
   g.e_end = e1;
@@ -357,6 +363,7 @@ FfnGroup dense_group(const moe_config& c, const Layout& L, const moe_weights& w,
                      const uint16_t* x) {
   FfnGroup g{};
   g.offsets = L.sh_off;
+  g.sched = L.sched;
   g.rows = c.T;
   g.n_experts = 1;
   g.e_end = 1;
@@ -765,6 +772,7 @@ moe_status moe_layer_forward(const moe_config* cfg, const moe_exec* ex, const mo
 
   cudaStream_t s = (cudaStream_t)stream;
   const int dev = current_device();
+  MOE_CUDA(cudaMemsetAsync(L.sched, 0, 2 * sizeof(int32_t), s));
 
   if (!ex->overlap) {
     cudaEvent_t* ev = reinterpret_cast<cudaEvent_t*>(ex->stage_events);

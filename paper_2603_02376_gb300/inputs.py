@@ -70,8 +70,11 @@ SKEWED = replace(DECODE, name="deepseek-v3 skewed prefill T=8192 zipf1.2", T=819
 DECODE_E32 = replace(DECODE, name="deepseek-v3 decode shape, 32 experts, T=16", T=16, E=32)
 # The prefill shape (128 rows per expert) with 32 experts, for profiler captures.
 PREFILL_E32 = replace(PREFILL, name="deepseek-v3 prefill shape, 32 experts, T=512", T=512, E=32)
+# The skewed (Zipf) batch with 32 experts: ~512 rows per expert in 256-row
+# token tiles, hot experts over several tiles, for profiler captures.
+SKEWED_E32 = replace(SKEWED, name="deepseek-v3 skewed shape, 32 experts, T=2048", T=2048, E=32)
 WORKLOADS = {"tiny": TINY, "decode": DECODE, "prefill": PREFILL, "skewed": SKEWED,
-             "decode_e32": DECODE_E32, "prefill_e32": PREFILL_E32}
+             "decode_e32": DECODE_E32, "prefill_e32": PREFILL_E32, "skewed_e32": SKEWED_E32}
 DISPATCH_SWEEP_T = (1024, 4096, 16384, 65536)
 
 _SUB = {"x": 1, "Wr": 2, "bias": 3, "W13": 4, "W2": 5, "Ws13": 6, "Ws2": 7,

@@ -439,8 +439,9 @@ def run_ours(args, wl, rank, world, local, device):
         run_w = {k_: (None if v is None else L.pack_weights(v)) for k_, v in run_w.items()}
         torch.cuda.synchronize()
     if fp8:
-        # e4m3 copies of the expert weights with per-row scales (fp8 = 1) or 128 x 128
-        # block exponents (fp8 = 2, kept per expert as [E, rows/128, cols/128]): a
+        # e4m3 copies of the expert weights with per-row scales (fp8 = 1, kept per
+        # expert as [E, rows]) or 128 x 128 block exponents (fp8 = 2, kept per
+        # expert as [E, rows/128, cols/128]): a
         # load-time step like the packing above; the bf16 tensors are dropped (the
         # oracle leg reads the e4m3 bytes)
         f8 = {"block": fp8 == 2}
@@ -449,6 +450,8 @@ def run_ours(args, wl, rank, world, local, device):
                 f8[n] = f8[sn] = None
             elif fp8 == 1:
                 f8[n], f8[sn] = L.quantize_fp8(d[n])
+                if d[n].dim() == 3:  # row scales per expert: [E, rows]
+                    f8[sn] = f8[sn].view(d[n].shape[0], -1)
             else:
                 f8[n], f8[sn] = L.quantize_fp8_weight_blocks(d[n])
                 if d[n].dim() == 3:

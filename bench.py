@@ -672,6 +672,19 @@ def run_ours(args, wl, rank, world, local, device):
         "routing": {"max_over_mean": round(float(cnt.max()) * wl.E / (wl.T * wl.k), 3),
                     "touched_experts": touched},
     }
+    # the whole layer against its roofline: max(bytes / BW, flops / P) over the
+    # measured step time, with the measured peaks and with the nominal ones
+    # (8 TB/s; 2.25 PFLOP/s bf16, twice that for e4m3)
+    B, F = float(sum(b.values())), float(sum(f.values()))
+    t_step = ms / args.steps / 1e3
+    pk = 2.0 if fp8 else 1.0
+    tb, tfb, tfs = B / (hbm * 1e9), F / (pk * tf_burst * 1e12), F / (pk * tf_sust * 1e12)
+    line["layer_roofline"] = {
+        "bytes": B, "flops": F, "t_bytes_ms": round(tb * 1e3, 4),
+        "t_flops_ms_burst": round(tfb * 1e3, 4), "t_flops_ms_sustained": round(tfs * 1e3, 4),
+        "frac_measured_peaks": round(max(tb, tfs) / t_step, 4),
+        "frac_nominal_peaks": round(max(B / 8e12, F / (pk * 2.25e15)) / t_step, 4),
+        "bound": "hbm" if tb >= tfs else "tensor"}
     if overlap:
         line["overlap"] = overlap
     if dispatch_fusion:

@@ -11,9 +11,11 @@
 //   D[f, n] = sum_k W[f, k] * X[n, k]      (both operands K-major, bf16)
 // D lives in TMEM: lane = output feature, column = token.
 //
-// Work unit = (expert e, token tile nt, feature block fb), in that order. The
-// units of every expert are enumerated on the device from the row offsets, so
-// a launch needs no host-side knowledge of the routing. A launch may carry a
+// Work unit = (expert e, token tile nt, feature block fb): experts in order,
+// inside an expert blocks of up to 8 token tiles, each block's feature blocks
+// in turn (block_order below). The units of every expert are enumerated on the
+// device from the row offsets, so a launch needs no host-side knowledge of the
+// routing. A launch may carry a
 // second operand group: one dense segment with its own weights and
 // activations (the shared expert), whose units run in the same persistent
 // grid as the routed ones. A persistent grid (one CTA per SM) runs the units:
@@ -23,7 +25,8 @@
 // round-robin; it announces each unit to the CTA's other roles through a
 // small ring in shared memory. Warp roles:
 //   warp 0     TMA producer: weight tile(s) 128 x 64 and token rows 16 x 64
-//              per stage into a STAGES-deep ring (128-byte swizzle);
+//              per stage into a STAGES-deep ring (128-byte swizzle); takes and
+//              announces the units;
 //   warp 1     MMA issuer (one thread): 4 x tcgen05.mma (K = 16 each) per stage,
 //              tcgen05.commit frees the stage, a final commit hands the
 //              accumulator to the epilogue; also owns the TMEM allocation;

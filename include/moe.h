@@ -342,7 +342,10 @@ moe_status moe_expert_ffn_fp8(int32_t rows, int32_t H, int32_t I, int32_t n_expe
                               void* stream);
 
 /*
- * FP8 quantization with block scales, for activation rows: each 1 x 128 block
+ * FP8 quantization with block scales: the paper's "quantize" stage (Section
+ * 4.3's FP8 quantize before the dispatch) at DeepSeek-V3's fine-grained
+ * granularity, with power-of-two (UE8M0) scales the tensor cores apply
+ * inside the MMA. For activation rows: each 1 x 128 block
  * of in [rows, K] bf16 gets the exponent k = the smallest integer with
  * amax <= 448 * 2^k (k = 0 for an all-zero block, clamped to [-127, 127]),
  * stored as the UE8M0 byte sf[r * sf_ld + c / 128] = k + 127, and its
@@ -369,8 +372,10 @@ moe_status moe_quantize_fp8_weight_blocks(int64_t rows, int32_t K, const uint16_
 size_t moe_expert_ffn_fp8_blocks_workspace_size(int32_t rows, int32_t I);
 
 /*
- * Grouped expert FFN with block-scaled FP8 operands (moe_expert_ffn's segments
- * and shapes). With 2^kx, 2^kw the scales of the blocks a product's terms fall in:
+ * Grouped expert FFN with block-scaled FP8 operands: the expert compute of
+ * the paper's MoE workload (GEMM1 up/gate + SwiGLU + GEMM2 down, Appendix
+ * "Workload Details") on e4m3 operands, with moe_expert_ffn's segments and
+ * shapes. With 2^kx, 2^kw the scales of the blocks a product's terms fall in:
  *   g|u[r][j] = sum_c x_q[r][c] 2^kx(r, c/128) * W13_q[e][j][c] 2^kw13(e, j/128, c/128),
  *   h[r] = bf16(silu(g) * u), h quantized by moe_quantize_fp8_blocks,
  *   y_perm[r][c] = sum_i h_q[r][i] 2^kh(r, i/128) * W2_q[e][c][i] 2^kw2(e, c/128, i/128),

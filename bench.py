@@ -540,15 +540,15 @@ def run_ours(args, wl, rank, world, local, device):
     stage_ms = traced(fuse)
     dispatch_fusion = None
     if fusable:  # the packed dispatch against the dispatch fused into GEMM1 (same batch)
-        packed = stage_ms if not fused else traced(0)
-        fz = stage_ms if fused else traced(1)
-        extra = fz["gemm1"] - packed["gemm1"]
+        pk_ms = stage_ms if not fused else traced(0)
+        fz_ms = stage_ms if fused else traced(1)
+        extra = fz_ms["gemm1"] - pk_ms["gemm1"]
         dispatch_fusion = {"active": "fused" if fused else "packed",
-                           "dispatch_ms_packed": round(packed["dispatch"], 4),
-                           "gemm1_ms_packed": round(packed["gemm1"], 4),
-                           "gemm1_ms_fused": round(fz["gemm1"], 4),
-                           "hidden_frac": round(1.0 - extra / packed["dispatch"], 3)
-                           if packed["dispatch"] > 0 else None}
+                           "dispatch_ms_packed": round(pk_ms["dispatch"], 4),
+                           "gemm1_ms_packed": round(pk_ms["gemm1"], 4),
+                           "gemm1_ms_fused": round(fz_ms["gemm1"], 4),
+                           "hidden_frac": round(1.0 - extra / pk_ms["dispatch"], 3)
+                           if pk_ms["dispatch"] > 0 else None}
 
     # --- end to end through the C ABI with host buffers: every step copies its
     # input batch in from pinned host memory and its output back out, on two

@@ -5,8 +5,12 @@ One step = one full layer forward (router -> gate/top-k -> permutation ->
 dispatch -> grouped GEMM1+SwiGLU -> grouped GEMM2 -> shared expert ->
 combine) over one batch of synthetic tokens, through the library's C ABI.
 
-    python bench.py [--gpus N] [--steps K] [--warmup W] [--workload decode]
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--workload skewed]
     python bench.py --impl reference ...     # the CPU oracle, timed on host cores
+
+The default workload is the largest single-GPU configuration: the skewed
+(Zipf 1.2, hottest expert ~15x the mean load) DeepSeek-V3 prefill batch of
+T=8192 tokens. decode (T=128) and prefill (T=4096, balanced) are flags.
 
 Prints one JSON line (rank 0). With N > 1 (torchrun) every rank runs an
 independent replica of the layer on its own tokens (no collective on the data
@@ -36,6 +40,8 @@ from paper_2603_02376_gb300 import inputs as I  # noqa: E402
 METRIC = "MoE layer tokens/sec on 1 GB300; grouped-GEMM % bf16 peak; dispatch/combine % HBM BW"
 FALLBACK_HBM_GBS = 6800.0
 FALLBACK_BF16_TFLOPS = 1900.0
+NOMINAL_HBM_GBS = 8000.0        # GB300 HBM3e, nominal (context beside the measured copy peak)
+NOMINAL_BF16_TFLOPS = 2250.0    # GB300 dense bf16, nominal
 TRAFFIC_FILE = os.path.join(ROOT, "profiles", "traffic.json")
 GEMM_SOURCES = ("paper_2603_02376_gb300/csrc/gemm_tc.cu", "paper_2603_02376_gb300/csrc/common.cuh")
 
@@ -46,7 +52,7 @@ def parse():
     p.add_argument("--steps", type=int, default=200)
     p.add_argument("--warmup", type=int, default=10)
     p.add_argument("--impl", choices=("ours", "reference"), default="ours")
-    p.add_argument("--workload", choices=tuple(I.WORKLOADS), default="decode")
+    p.add_argument("--workload", choices=tuple(I.WORKLOADS), default="skewed")
     p.add_argument("--mode", choices=("seq", "overlap-tokens", "overlap-experts"), default="seq")
     p.add_argument("--chunk-tokens", type=int, default=512)
     p.add_argument("--expert-chunks", type=int, default=8)
@@ -74,6 +80,10 @@ def parse():
     p.add_argument("--cpu-tokens", type=int, default=None,
                    help="oracle sample size (tokens); default 128, or 8 with --precision "
                         "fp8-block, whose oracle dequantizes each touched expert in full")
+    p.add_argument("--cpu-one-core-tokens", type=int, default=4,
+                   help="tokens of the single-core oracle timing (a child process with one "
+                        "BLAS thread); 0 skips it")
+    p.add_argument("--oracle-one-core", default=None, help=argparse.SUPPRESS)
     return p.parse_args()
 
 
@@ -294,30 +304,75 @@ def measured_traffic(workload, fp8=0, kernel_bytes=None):
     return None
 
 
+def kernel_roofline(bytes_, flops, t_s, hbm_gbs, tf_sust, tf_burst, src, dtype):
+    """Roofline of one kernel: its bound is whichever of bytes / (measured copy
+    bandwidth) and flops / (measured sustained dense peak of its dtype) takes
+    longer; achieved and peak are in that bound's unit and frac = achieved /
+    peak (= that time / the measured time). Both sides are also given against
+    the measured and the nominal denominators."""
+    t_b = bytes_ / (hbm_gbs * 1e9)
+    t_f = flops / (tf_sust * 1e12)
+    gbs, tfs = bytes_ / t_s / 1e9, flops / t_s / 1e12
+    nominal_tf = NOMINAL_BF16_TFLOPS * (2.0 if dtype == "e4m3" else 1.0)
+    hbm_side = {"achieved_GBs": round(gbs, 1), "frac_measured_copy": round(gbs / hbm_gbs, 4),
+                "frac_nominal_8TBs": round(gbs / NOMINAL_HBM_GBS, 4)}
+    tensor_side = {"achieved_TFLOPs": round(tfs, 1),
+                   "frac_measured_sustained": round(tfs / tf_sust, 4),
+                   "frac_measured_burst": round(tfs / tf_burst, 4),
+                   "frac_nominal": round(tfs / nominal_tf, 4)}
+    if t_f > t_b:
+        r = {"bound": "tensor", "achieved": round(tfs, 1), "peak": round(tf_sust, 1),
+             "unit": "TFLOP/s", "frac": round(tfs / tf_sust, 4),
+             "peak_source": f"{dtype} dense, sustained ({'bf16_tflops_sustained' if dtype == 'bf16' else '2 x bf16_tflops_sustained'} of {src})"}
+    else:
+        r = {"bound": "hbm", "achieved": round(gbs, 1), "peak": hbm_gbs, "unit": "GB/s",
+             "frac": round(gbs / hbm_gbs, 4), "peak_source": f"hbm_gbs of {src}"}
+    r.update({"t_bytes_ms": round(t_b * 1e3, 4), "t_flops_ms": round(t_f * 1e3, 4),
+              "t_measured_ms": round(t_s * 1e3, 4), "hbm": hbm_side, "tensor": tensor_side})
+    return r
+
+
 # ---------------------------------------------------------------- CPU oracle leg
 
-def oracle_tokens_per_s(wl, d, tokens):
-    """Time the CPU oracle on a sample of tokens; weights come from host copies.
+def cpu_model() -> str:
+    """The host CPU's model name (lscpu, else /proc/cpuinfo, else the machine type)."""
+    try:
+        out = subprocess.run(["lscpu"], capture_output=True, text=True, timeout=10).stdout
+        for line in out.splitlines():
+            if line.split(":")[0].strip() == "Model name":
+                return line.split(":", 1)[1].strip()
+    except Exception:
+        pass
+    try:
+        with open("/proc/cpuinfo") as f:
+            for line in f:
+                if line.lower().startswith("model name"):
+                    return line.split(":", 1)[1].strip()
+    except Exception:
+        pass
+    import platform
+    return platform.machine()
 
-    With d["fp8"] the oracle runs the FP8 expert form on the e4m3 weights."""
+
+def oracle_cfg(wl, n):
+    from oracle import moe_oracle as O
+    return O.LayerConfig(T=n, H=wl.H, E=wl.E, k=wl.k, I=wl.I, I_shared=wl.I_shared,
+                         n_groups=wl.n_groups, topk_groups=wl.topk_groups, gate=wl.gate,
+                         normalize=wl.normalize, route_scale=wl.route_scale)
+
+
+def time_oracle(wl, xr, Wr, b, host_of, shared, f8=None):
+    """Time the oracle's layer on token rows xr (fp64 [n, H]).
+
+    host_of(experts) -> {e: host tensors of expert e}, built before the clock
+    starts (host copies of the touched experts: bf16 W13, W2, or the FP8 forms'
+    codes and scales); shared likewise for the shared expert (or None)."""
     from oracle import moe_oracle as O
 
-    cfg = O.LayerConfig(T=len(tokens), H=wl.H, E=wl.E, k=wl.k, I=wl.I, I_shared=wl.I_shared,
-                        n_groups=wl.n_groups, topk_groups=wl.topk_groups, gate=wl.gate,
-                        normalize=wl.normalize, route_scale=wl.route_scale)
-    tok = torch.as_tensor(tokens, device=d["x"].device)
-    xr = d["x"][tok].to(torch.float64).cpu().numpy()
-    Wr = d["Wr"].cpu().numpy()
-    b = None if d["bias"] is None else d["bias"].cpu().numpy()
-    # host copies (bf16) of the experts the sample touches, made before the clock starts
+    cfg = oracle_cfg(wl, len(xr))
     idx, _ = O.gate_topk(O.router_logits(xr, Wr), b, cfg)
-    f8 = d.get("fp8")
+    host = host_of(sorted(int(e) for e in np.unique(idx)))
     if f8:
-        # (codes, scales) pairs: e4m3 bytes, then fp32 row scales or UE8M0 block exponents
-        host = {int(e): tuple(f8[n][e].cpu() for n in ("W13", "s13", "W2", "s2"))
-                for e in np.unique(idx)}
-        shared = tuple(f8[n].cpu() for n in ("Ws13", "ss13", "Ws2", "ss2")) \
-            if wl.I_shared else None
         blk = f8.get("block", False)
 
         def conv(t, i):
@@ -327,8 +382,6 @@ def oracle_tokens_per_s(wl, d, tokens):
 
         ffn = O.swiglu_ffn_fp8_blocks if blk else O.swiglu_ffn_fp8
     else:
-        host = {int(e): (d["W13"][e].cpu(), d["W2"][e].cpu()) for e in np.unique(idx)}
-        shared = (d["Ws13"].cpu(), d["Ws2"].cpu()) if wl.I_shared else None
         conv = lambda t, i: t.to(torch.float64).numpy()
         ffn = O.swiglu_ffn
 
@@ -339,20 +392,96 @@ def oracle_tokens_per_s(wl, d, tokens):
     t0 = time.perf_counter()
     O.layer_forward_tokens(xr, Wr, b, get_expert, cfg, get_shared, ffn=ffn)
     dt = time.perf_counter() - t0
-    return len(tokens) / dt, dt, len(host)
+    return len(xr) / dt, dt, len(host)
 
 
-def cpu_baseline(wl, d, n_tokens, seed=1):
+def oracle_tokens_per_s(wl, d, tokens):
+    """Time the CPU oracle on a sample of tokens; weights come from host copies.
+
+    With d["fp8"] the oracle runs the FP8 expert form on the e4m3 weights."""
+    tok = torch.as_tensor(tokens, device=d["x"].device)
+    xr = d["x"][tok].to(torch.float64).cpu().numpy()
+    Wr = d["Wr"].cpu().numpy()
+    b = None if d["bias"] is None else d["bias"].cpu().numpy()
+    f8 = d.get("fp8")
+    if f8:
+        # (codes, scales) pairs: e4m3 bytes, then fp32 row scales or UE8M0 block exponents
+        host_of = lambda es: {e: tuple(f8[n][e].cpu() for n in ("W13", "s13", "W2", "s2"))
+                              for e in es}
+        shared = tuple(f8[n].cpu() for n in ("Ws13", "ss13", "Ws2", "ss2")) \
+            if wl.I_shared else None
+    else:
+        host_of = lambda es: {e: (d["W13"][e].cpu(), d["W2"][e].cpu()) for e in es}
+        shared = (d["Ws13"].cpu(), d["Ws2"].cpu()) if wl.I_shared else None
+    return time_oracle(wl, xr, Wr, b, host_of, shared, f8)
+
+
+def oracle_one_core_child(path):
+    """Child-process body of the single-core timing (BLAS limited to one thread
+    by the parent through the environment). Reads the sampled token rows, Wr and
+    the bias from `path`; the touched experts' bf16 weights are drawn here on the
+    CPU with the workload's distributions (same shapes and work as the device
+    draw; the oracle's time does not depend on the values). Prints one JSON line."""
+    torch.set_num_threads(1)
+    z = np.load(path)
+    wl = I.WORKLOADS[str(z["workload"])]
+    b = z["bias"] if z["bias"].size else None
+
+    def host_of(es):
+        return {e: (I.randn((2 * wl.I, wl.H), 0.02, torch.bfloat16, 0, "W13", "cpu", extra=e),
+                    I.randn((wl.H, wl.I), 0.02, torch.bfloat16, 0, "W2", "cpu", extra=e))
+                for e in es}
+
+    shared = (I.randn((2 * wl.I_shared, wl.H), 0.02, torch.bfloat16, 0, "Ws13", "cpu"),
+              I.randn((wl.H, wl.I_shared), 0.02, torch.bfloat16, 0, "Ws2", "cpu")) \
+        if wl.I_shared else None
+    v, dt, ne = time_oracle(wl, z["x"], z["Wr"], b, host_of, shared)
+    print(json.dumps({"value": v, "seconds": dt, "experts": ne, "tokens": int(len(z["x"]))}))
+
+
+def oracle_one_core(wl, d, n_tokens, seed=2):
+    """The oracle on one core: a child process with every BLAS / OpenMP pool at
+    one thread, timing n_tokens sampled tokens of the batch (bf16 form only)."""
+    import tempfile
+    toks = I.sample_tokens(wl.T, n_tokens, seed)
+    xr = d["x"][toks.to(d["x"].device)].to(torch.float64).cpu().numpy()
+    b = np.zeros(0, np.float32) if d["bias"] is None else d["bias"].cpu().numpy()
+    env = dict(os.environ, OMP_NUM_THREADS="1", OPENBLAS_NUM_THREADS="1", MKL_NUM_THREADS="1")
+    with tempfile.TemporaryDirectory() as td:
+        path = os.path.join(td, "sample.npz")
+        name = next(k_ for k_, v in I.WORKLOADS.items() if v == wl)
+        np.savez(path, x=xr, Wr=d["Wr"].cpu().numpy(), bias=b, workload=name)
+        r = subprocess.run([sys.executable, os.path.abspath(__file__), "--oracle-one-core", path],
+                           capture_output=True, text=True, env=env, timeout=600)
+    if r.returncode != 0:
+        return {"error": (r.stderr.strip().splitlines() or ["child failed"])[-1][:200]}
+    o = json.loads(r.stdout.strip().splitlines()[-1])
+    return {"value": o["value"], "unit": "tokens/s", "cores": 1,
+            "sample": f"{o['tokens']} sampled tokens ({o['experts']} experts touched), "
+                      f"{o['seconds']:.1f} s, one BLAS thread; the touched experts' weights "
+                      f"drawn on the host with the workload's distributions"}
+
+
+def cpu_baseline(wl, d, n_tokens, seed=1, one_core_tokens=0):
     toks = I.sample_tokens(wl.T, n_tokens, seed).numpy()
     v, dt, ne = oracle_tokens_per_s(wl, d, toks)
     form = ("block-scaled FP8 expert form, " if d["fp8"].get("block") else
             "FP8 expert form, ") if d.get("fp8") else ""
-    return {"value": v, "unit": "tokens/s", "cores": os.cpu_count(), "kind": "oracle",
-            "sample": f"{len(toks)} of the {wl.T} tokens ({ne} experts touched), {form}numpy "
-                      f"fp64 oracle, {dt:.1f} s; BLAS threads = host cores"}
+    sampled = len(toks) < wl.T
+    r = {"value": v, "unit": "tokens/s", "cores": os.cpu_count(), "kind": "oracle",
+         "cpu_model": cpu_model(),
+         "sample": f"{'sampled: ' if sampled else ''}{len(toks)} of the {wl.T} tokens "
+                   f"({ne} experts touched), {form}numpy fp64 oracle, {dt:.1f} s; "
+                   f"BLAS threads = host cores"}
+    if one_core_tokens and not d.get("fp8"):
+        r["one_core"] = oracle_one_core(wl, d, one_core_tokens)
+    return r
 
 
 # ---------------------------------------------------------------- main arms
+
+REF_BUDGET_S = 90.0  # the reference arm's timed steps together take about this long
+
 
 def run_reference(args, wl, rank, world, device):
     if rank != 0:
@@ -362,7 +491,11 @@ def run_reference(args, wl, rank, world, device):
     if wl.balance != "none":
         L.load()
         calibrate(L, wl, d, device)
-    n = max(1, (args.cpu_tokens or 128) // 2)
+    # per-step sample: a first untimed call measures the oracle's cost per token,
+    # then each timed step takes as many tokens as keep the K steps within the budget
+    n_max = max(1, (args.cpu_tokens or 128) // 2)
+    v0, _, _ = oracle_tokens_per_s(wl, d, I.sample_tokens(wl.T, min(8, n_max), 99).numpy())
+    n = int(max(1, min(n_max, REF_BUDGET_S * v0 / max(args.steps, 1))))
     for s in range(args.warmup):
         oracle_tokens_per_s(wl, d, I.sample_tokens(wl.T, n, 100 + s).numpy())
     times = []
@@ -378,8 +511,9 @@ def run_reference(args, wl, rank, world, device):
         "vs_baseline": None, "dtype": "f64", "data": "synthetic",
         "config": config_of(wl, args),
         "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": os.cpu_count(),
-                         "kind": "oracle",
-                         "sample": f"{n} tokens per step of the {wl.T}-token batch, numpy fp64"},
+                         "kind": "oracle", "cpu_model": cpu_model(),
+                         "sample": f"sampled: {n} tokens per step of the {wl.T}-token batch, "
+                                   f"numpy fp64"},
         "e2e": {"value": value, "unit": "tokens/s", "h2d_bytes_per_step": 0,
                 "d2h_bytes_per_step": 0},
     }
@@ -626,26 +760,37 @@ def run_ours(args, wl, rank, world, local, device):
     hbm, tf_burst, tf_sust, src = peaks()
     b, f = algorithmic(wl, touched, fused, fp8, bool(fc))
     g1 = stage_ms["gemm1"] / 1e3
-    achieved = b["gemm1"] / g1 / 1e9
     # GEMM1's own bytes (the FP8 GEMM1 stage also holds the h quantization)
     R = wl.T * wl.k
     qh = (R * wl.I * 3 + scale_bytes(R, wl.I, fp8)
           + (wl.T * wl.I_shared * 3 + scale_bytes(wl.T, wl.I_shared, fp8)
              if wl.I_shared == wl.I else 0)) if fp8 else 0
     traffic = measured_traffic(wl.name, fp8, b["gemm1"] - qh)
+    pk = 2.0 if fp8 else 1.0   # e4m3 dense peak = the measured bf16 peak x the nominal 2x
     stages = {}
     for s_, t in stage_ms.items():
         e = {"ms": round(t, 4)}
         if b.get(s_):
             e["GB/s"] = round(b[s_] / (t / 1e3) / 1e9, 1)
             e["frac_hbm"] = round(b[s_] / (t / 1e3) / 1e9 / hbm, 3)
+            e["frac_hbm_nominal"] = round(b[s_] / (t / 1e3) / 1e9 / NOMINAL_HBM_GBS, 3)
         if f.get(s_):
             e["TFLOP/s"] = round(f[s_] / (t / 1e3) / 1e12, 2)
-            if fp8:  # fp8 dense peak = the measured bf16 peak x the nominal 2x ratio
-                e["frac_fp8"] = round(f[s_] / (t / 1e3) / 1e12 / (2 * tf_sust), 4)
-            else:
-                e["frac_bf16"] = round(f[s_] / (t / 1e3) / 1e12 / tf_sust, 4)
+            e["frac_fp8" if fp8 else "frac_bf16"] = round(
+                f[s_] / (t / 1e3) / 1e12 / (pk * tf_sust), 4)
         stages[s_] = e
+    roofline = kernel_roofline(b["gemm1"], f["gemm1"], g1, hbm, tf_sust * pk, tf_burst * pk,
+                               src, "e4m3" if fp8 else "bf16")
+    roofline.update({
+        "kernel": {0: "grouped GEMM1 + SwiGLU (tcgen05), routed + shared",
+                   1: "grouped GEMM1 + SwiGLU (tcgen05 kind::f8f6f4) and the h "
+                      "quantization, routed + shared",
+                   2: "grouped GEMM1 + SwiGLU (tcgen05 kind::mxf8f6f4 block_scale) "
+                      "and the h block quantization, routed + shared"}[fp8],
+        "traffic": traffic, "algorithmic_bytes": b["gemm1"], "algorithmic_flops": f["gemm1"],
+        "touched_experts": touched,
+        "note": ("the grouped GEMM1 launch also runs the shared expert's GEMM1; its bytes and "
+                 "flops are included") if wl.I_shared == wl.I else ""})
 
     line = {
         "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world,
@@ -661,20 +806,13 @@ def run_ours(args, wl, rank, world, local, device):
                 "copies": "pinned host <-> device every step, on two copy streams, "
                           "double-buffered (overlapping the neighbouring steps' layers)"},
         "gpu_launches": launches,
-        "roofline": {"bound": "hbm",
-                     "kernel": {0: "grouped GEMM1 + SwiGLU (tcgen05), routed + shared",
-                                1: "grouped GEMM1 + SwiGLU (tcgen05 kind::f8f6f4) and the h "
-                                   "quantization, routed + shared",
-                                2: "grouped GEMM1 + SwiGLU (tcgen05 kind::mxf8f6f4 block_scale) "
-                                   "and the h block quantization, routed + shared"}[fp8],
-                     "achieved": round(achieved, 1), "peak": hbm, "unit": "GB/s",
-                     "frac": round(achieved / hbm, 4), "traffic": traffic,
-                     "peak_source": f"hbm_gbs of {src}",
-                     "algorithmic_bytes": b["gemm1"], "touched_experts": touched,
-                     "note": ("the grouped GEMM1 launch also runs the shared expert's GEMM1; "
-                              "its bytes are included") if wl.I_shared == wl.I else ""},
+        "roofline": roofline,
         "clocks": clocks,
         "stages": stages,
+        "denominators": {"frac_hbm": f"measured copy {hbm} GB/s ({src}; read + write bytes)",
+                         "frac_hbm_nominal": f"nominal {NOMINAL_HBM_GBS:.0f} GB/s",
+                         "frac_bf16 / frac_fp8": f"measured sustained dense "
+                                                 f"{tf_sust} TFLOP/s (x2 for e4m3)"},
         "routing": {"max_over_mean": round(float(cnt.max()) * wl.E / (wl.T * wl.k), 3),
                     "touched_experts": touched},
     }
@@ -683,13 +821,13 @@ def run_ours(args, wl, rank, world, local, device):
     # (8 TB/s; 2.25 PFLOP/s bf16, twice that for e4m3)
     B, F = float(sum(b.values())), float(sum(f.values()))
     t_step = ms / args.steps / 1e3
-    pk = 2.0 if fp8 else 1.0
     tb, tfb, tfs = B / (hbm * 1e9), F / (pk * tf_burst * 1e12), F / (pk * tf_sust * 1e12)
     line["layer_roofline"] = {
         "bytes": B, "flops": F, "t_bytes_ms": round(tb * 1e3, 4),
         "t_flops_ms_burst": round(tfb * 1e3, 4), "t_flops_ms_sustained": round(tfs * 1e3, 4),
         "frac_measured_peaks": round(max(tb, tfs) / t_step, 4),
-        "frac_nominal_peaks": round(max(B / 8e12, F / (pk * 2.25e15)) / t_step, 4),
+        "frac_nominal_peaks": round(max(B / (NOMINAL_HBM_GBS * 1e9),
+                                        F / (pk * NOMINAL_BF16_TFLOPS * 1e12)) / t_step, 4),
         "bound": "hbm" if tb >= tfs else "tensor"}
     if overlap:
         line["overlap"] = overlap
@@ -697,7 +835,8 @@ def run_ours(args, wl, rank, world, local, device):
         line["dispatch_fusion"] = dispatch_fusion
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         n_cpu = args.cpu_tokens or (8 if args.precision == "fp8-block" else 128)
-        line["cpu_baseline"] = cpu_baseline(wl, d, n_cpu)
+        line["cpu_baseline"] = cpu_baseline(wl, d, n_cpu,
+                                            one_core_tokens=args.cpu_one_core_tokens)
     if rank == 0:
         print(json.dumps(line), flush=True)
 
@@ -848,6 +987,9 @@ def run_sweep(args, rank, world, local, device):
 
 def main():
     args = parse()
+    if args.oracle_one_core:  # child of the CPU baseline's single-core leg: no GPU
+        oracle_one_core_child(args.oracle_one_core)
+        return
     rank, world, local = dist_env()
     if world > 1:
         torch.distributed.init_process_group("gloo")

@@ -483,6 +483,18 @@ moe_status moe_testing_expert_ffn_stall(int32_t rows, int32_t H, int32_t I, int3
                                         void* ws, size_t ws_bytes, int64_t stall_fill,
                                         int64_t wait_limit_ns, void* stream);
 
+/*
+ * Testing (no counterpart in the paper): a failure injected on the host. With
+ * n >= 0, the stage calls inside the moe_layer_forward calls that follow (the
+ * routing-and-packing step of a chunk, the expert GEMMs of a chunk or expert
+ * range) pass until n of them have; the next one returns MOE_ERR_CUDA without
+ * launching anything, and the injector turns itself off. n = -1 turns it off.
+ * Process-wide. Used to check that a pipelined forward failing after it forked
+ * its pack stream still joins that stream back into the caller's stream before
+ * returning. MOE_ERR_INVALID_ARG for n < -1.
+ */
+moe_status moe_testing_fail_stage(int32_t n);
+
 /* Synchronises `stream`, then reads and clears the device error word of the
  * current device. MOE_OK, MOE_ERR_TIMEOUT or MOE_ERR_DEVICE_CHECK (or
  * MOE_ERR_CUDA if the synchronisation itself failed). */
@@ -491,7 +503,10 @@ moe_status moe_check_errors(void* stream);
 /* Number of kernels this library has launched in this process (all devices). */
 uint64_t moe_launch_count(void);
 
-/* Releases internal streams and events. Safe to call more than once. */
+/* Releases internal streams and events, and forgets the cached device address
+ * of moe_dispatch_noalloc's scratch array (the next such call looks it up
+ * again). Call it after cudaDeviceReset and before the library's next call on
+ * that device. Safe to call more than once. */
 void moe_shutdown(void);
 
 #ifdef __cplusplus

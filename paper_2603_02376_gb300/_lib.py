@@ -34,7 +34,7 @@ EXPORTS = ("moe_status_string", "moe_validate_config", "moe_workspace_size",
            "moe_stack_forward", "moe_rms_norm", "moe_graph_create_stack", "moe_graph_launch",
            "moe_graph_kernel_count", "moe_graph_destroy", "moe_quantize_fp8_blocks",
            "moe_quantize_fp8_weight_blocks", "moe_expert_ffn_fp8_blocks",
-           "moe_expert_ffn_fp8_blocks_workspace_size")
+           "moe_expert_ffn_fp8_blocks_workspace_size", "moe_testing_fail_stage")
 MOE_DISPATCH_NOALLOC_MAX_ENTRIES = 131072
 
 
@@ -127,6 +127,7 @@ def load(path: str = LIB_PATH) -> ctypes.CDLL:
         "moe_check_errors": (S, [P]),
         "moe_launch_count": (ctypes.c_uint64, []),
         "moe_shutdown": (None, []),
+        "moe_testing_fail_stage": (S, [I32]),
     }
     for name, (res, args) in sig.items():
         f = getattr(lib, name)
@@ -355,6 +356,12 @@ def moe_testing_expert_ffn_stall(rows, H, I, n_experts, x_perm, offsets, W13, W2
                                                _ptr(W13), _ptr(W2), _ptr(y_perm), _ptr(ws), nb,
                                                int(stall_fill), int(wait_limit_ns),
                                                _stream(stream))
+
+
+def moe_testing_fail_stage(n: int) -> None:
+    """Failure-injection hook: stage call n (0-based) of the forwards that follow fails
+    with MOE_ERR_CUDA on the host; -1 turns it off."""
+    _check(load().moe_testing_fail_stage(int(n)), "moe_testing_fail_stage")
 
 
 def moe_combine(cfg, y_perm, slot_row, topk_w, shared_out, out, out_fp32, stream=None) -> None:

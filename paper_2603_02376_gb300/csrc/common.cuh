@@ -23,6 +23,10 @@ int* device_error_word();
 // Number of SMs of the current device (cached per device).
 int num_sms();
 
+// Forgets the cached device addresses of moe_dispatch_noalloc's scratch array
+// (moe_shutdown; after a device reset the array lives at a new address).
+void forget_noalloc_scratch();
+
 // Status of the last launch on this thread.
 inline moe_status launch_status() {
   return cudaPeekAtLastError() == cudaSuccess ? MOE_OK : MOE_ERR_CUDA;

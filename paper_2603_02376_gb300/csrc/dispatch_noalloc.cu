@@ -15,7 +15,8 @@
 // host memory, silently use the wrong memory. So the first call on each device
 // (with that device current) asks the runtime for the real device address with
 // cudaGetSymbolAddress and caches it; make that first call before any stream
-// capture. Kernels then receive that address.
+// capture. Kernels then receive that address. moe_shutdown forgets the cached
+// addresses (after cudaDeviceReset the array is loaded again elsewhere).
 //
 // All calls on a device share the one array and it keeps the previous call's
 // contents. Nothing in it needs to start at zero: the histogram kernel writes
@@ -50,6 +51,13 @@ moe_status scratch_address(int32_t** out) {
 }
 
 }  // namespace
+
+namespace moe {
+void forget_noalloc_scratch() {
+  std::lock_guard<std::mutex> lk(g_scratch_mu);
+  for (auto& p : g_scratch_ptr) p = nullptr;
+}
+}  // namespace moe
 
 extern "C" moe_status moe_dispatch_noalloc(const moe_config* cfg, const uint16_t* x,
                                            const int32_t* topk_idx, int32_t* counts,

@@ -249,6 +249,34 @@ bool events(int d, size_t n, std::vector<cudaEvent_t>* out) {
     if ((expr) != cudaSuccess) return MOE_ERR_CUDA;     \
   } while (0)
 
+// Testing: a simulated failure of a stage call, made on the host (no CUDA call
+// fails and nothing runs on the GPU). -1 = off; n >= 0 = the stage calls of
+// the forwards that follow pass until n of them have, then the next one
+// returns MOE_ERR_CUDA and the injector switches itself off.
+std::atomic<int> g_fail_countdown{-1};
+
+moe_status injected_failure() {
+  int v = g_fail_countdown.load(std::memory_order_relaxed);
+  while (v >= 0) {
+    if (g_fail_countdown.compare_exchange_weak(v, v - 1, std::memory_order_relaxed))
+      return v == 0 ? MOE_ERR_CUDA : MOE_OK;
+  }
+  return MOE_OK;
+}
+
+// After the pipelined forward forks the pack stream off `stream`, every return
+// -- an error part-way through included -- joins it back: `stream` then waits
+// for all the work this call put on the pack stream, so none of it can still
+// be writing the caller's workspace once the caller's stream moves on, and a
+// forward captured into a CUDA graph always leaves the fork joined.
+struct JoinOnExit {
+  cudaStream_t stream, ps;
+  cudaEvent_t ev;
+  ~JoinOnExit() {
+    if (cudaEventRecord(ev, ps) == cudaSuccess) cudaStreamWaitEvent(stream, ev, 0);
+  }
+};
+
 // Router + gate + permutation (+ packing) of tokens [t0, t0+Tc) into chunk slot `ci`.
 // Records stage event i of a traced forward (no-op without tracing).
 moe_status mark(cudaEvent_t* ev, int i, cudaStream_t s) {
@@ -273,6 +301,7 @@ moe_status quantize_tokens(const moe_config& c, const Layout& L, const uint16_t*
 moe_status pack_tokens(const moe_config& c, const Layout& L, const moe_weights& w,
                        const uint16_t* x, int t0, int Tc, int ci, bool pack_rows,
                        cudaStream_t s, cudaEvent_t* ev = nullptr, bool quantize = false) {
+  MOE_TRY(injected_failure());
   moe_config cc = c;
   cc.T = Tc;
   const size_t tk = (size_t)t0 * c.k;
@@ -399,6 +428,7 @@ FfnGroup dense_group(const moe_config& c, const Layout& L, const moe_weights& w,
 moe_status experts_tokens(const moe_config& c, const Layout& L, const moe_weights& w,
                           const uint16_t* x, int t0, int Tc, int ci, int e0, int e1,
                           cudaStream_t s, cudaEvent_t* ev = nullptr) {
+  MOE_TRY(injected_failure());
   const FfnGroup g = routed_group(c, L, w, x, t0, Tc, ci, e0, e1);
   const long hint = (long)g.rows * (e1 - e0) / c.E;
   MOE_TRY(launch_expert_ffn_groups(g, nullptr, c.H, c.I, (int)hint, s,
@@ -801,12 +831,13 @@ moe_status moe_layer_forward(const moe_config* cfg, const moe_exec* ex, const mo
   if (!ps) return MOE_ERR_CUDA;
   const int n_stage = ex->chunk_axis == 0 ? L.n_chunks : ex->n_expert_chunks;
   std::vector<cudaEvent_t> ev;
-  if (!events(dev, (size_t)n_stage + 1, &ev)) return MOE_ERR_CUDA;
+  if (!events(dev, (size_t)n_stage + 2, &ev)) return MOE_ERR_CUDA;
   if (L.fp8) MOE_TRY(quantize_tokens(c, L, x, 0, c.T, s));  // before the fork: both streams read x_q
   MOE_TRY(clear_acc(c, L, s));
   // the pack stream starts after everything already queued on `stream`
   MOE_CUDA(cudaEventRecord(ev[n_stage], s));
   MOE_CUDA(cudaStreamWaitEvent(ps, ev[n_stage], 0));
+  const JoinOnExit join{s, ps, ev[n_stage + 1]};
 
   if (ex->chunk_axis == 0) {
     // Token chunks: chunk i+1 is routed and packed on the pack stream while
@@ -875,7 +906,14 @@ moe_status moe_check_errors(void* stream) {
 
 uint64_t moe_launch_count(void) { return g_launches.load(std::memory_order_relaxed); }
 
+moe_status moe_testing_fail_stage(int32_t n) {
+  if (n < -1) return MOE_ERR_INVALID_ARG;
+  g_fail_countdown.store(n, std::memory_order_relaxed);
+  return MOE_OK;
+}
+
 void moe_shutdown(void) {
+  forget_noalloc_scratch();
   std::lock_guard<std::mutex> lk(g_mu);
   int prev = 0;
   cudaGetDevice(&prev);

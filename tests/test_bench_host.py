@@ -4,7 +4,10 @@
   hand in the comments, for bf16 and for the block-scaled FP8 form;
 * the traffic captures' source hash: unchanged by comment edits, changed by a
   code edit; a capture keyed to another hash is not used;
-* the block-scaled FP8 weight generator: shapes, exponent range, no NaN code.
+* the block-scaled FP8 weight generator: shapes, exponent range, no NaN code;
+* the per-kernel roofline: its bound is the longer of bytes / bandwidth and
+  flops / peak, with fractions against the measured and nominal peaks;
+* the CPU baseline's single-core leg (a child process with one BLAS thread).
 """
 
 import json
@@ -95,6 +98,32 @@ def test_block_scaled_weight_generator():
     assert W2.shape == (2, 256, 128) and k2.shape == (2, 2, 1)
     Ws13, ks13, Ws2, ks2 = I.fp8_block_shared_weights(wl, 0, "cpu")
     assert Ws13.shape == (256, 256) and ks13.shape == (2, 2) and ks2.shape == (2, 1)
+
+
+def test_kernel_roofline_takes_the_longer_bound():
+    # 16.45 GB and 4.33 TFLOP in 3.9 ms against 6776 GB/s and 1699.8 TFLOP/s sustained:
+    # the bytes need 2.43 ms, the flops 2.55 ms, so the kernel is tensor-bound
+    r = bench.kernel_roofline(16.45e9, 4.33e12, 3.9e-3, 6776.3, 1699.8, 1910.6, "measured", "bf16")
+    assert r["bound"] == "tensor" and r["unit"] == "TFLOP/s"
+    assert r["achieved"] == pytest.approx(4.33e12 / 3.9e-3 / 1e12, rel=1e-3)
+    assert r["frac"] == pytest.approx(4.33e12 / 3.9e-3 / 1e12 / 1699.8, abs=1e-4)
+    assert r["frac"] == pytest.approx(r["t_flops_ms"] / r["t_measured_ms"], abs=1e-3)
+    assert r["hbm"]["frac_nominal_8TBs"] == pytest.approx(16.45e9 / 3.9e-3 / 1e9 / 8000, abs=1e-4)
+    # decode: 14.7 GB and 0.1 TFLOP in 1.96 ms is bandwidth-bound
+    d = bench.kernel_roofline(14.7e9, 0.1e12, 1.96e-3, 6776.3, 1699.8, 1910.6, "measured", "bf16")
+    assert d["bound"] == "hbm" and d["unit"] == "GB/s" and d["peak"] == 6776.3
+    assert d["frac"] == pytest.approx(14.7e9 / 1.96e-3 / 1e9 / 6776.3, abs=1e-4)
+    # e4m3 takes twice the bf16 peak (the caller scales it) and names its own dtype
+    e = bench.kernel_roofline(8.4e9, 4.33e12, 2.3e-3, 6776.3, 2 * 1699.8, 2 * 1910.6, "measured",
+                              "e4m3")
+    assert e["tensor"]["frac_nominal"] == pytest.approx(4.33e12 / 2.3e-3 / 1e12 / 4500, abs=1e-4)
+
+
+def test_oracle_single_core_leg_runs_in_a_child():
+    d = I.layer_inputs(I.TINY, seed=0, device="cpu")
+    r = bench.oracle_one_core(I.TINY, d, 4)
+    assert "error" not in r, r
+    assert r["cores"] == 1 and r["value"] > 0 and r["sample"].startswith("4 sampled tokens")
 
 
 if __name__ == "__main__":

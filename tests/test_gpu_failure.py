@@ -66,3 +66,52 @@ def test_stalled_wait_times_out_and_context_survives(counts, stall_fill):
         ref = h @ W2[0].double().T
         err = (y2[:e0].double() - ref).abs().max().item()
         assert err <= 1e-3 * ref.abs().max().item() + 1e-3
+
+
+@pytest.mark.parametrize("axis", [0, 1])
+def test_pipelined_forward_failing_after_the_fork_joins_its_pack_stream(axis):
+    """A pipelined forward that fails after forking its pack stream must still
+    make the caller's stream wait for the pack stream's work before returning.
+
+    The failure is injected on the host (moe_testing_fail_stage): the second
+    stage call fails with MOE_ERR_CUDA, after the first one has put routing and
+    packing work on the pack stream. Eagerly, the error comes back and the same
+    stream then runs a correct forward. Under CUDA-graph capture, ending the
+    capture succeeds only if every stream forked from the capturing stream was
+    joined back into it; the captured graph is never launched."""
+    from paper_2603_02376_gb300 import inputs as I
+
+    L.load()
+    wl = I.TINY
+    d = I.layer_inputs(wl, seed=0, device=DEV)
+    cfg = L.config_of(wl)
+    ex = L.exec_config(overlap=1, chunk_axis=axis, chunk_tokens=16, n_expert_chunks=4)
+    W = L.weights_struct(d["Wr"], d["bias"], d["W13"], d["W2"], d["Ws13"], d["Ws2"])
+    ws = torch.zeros(L.moe_workspace_size(cfg, ex), dtype=torch.uint8, device=DEV)
+    out = torch.zeros((wl.T, wl.H), dtype=torch.bfloat16, device=DEV)
+    s = torch.cuda.Stream()
+    L.moe_check_errors()
+
+    L.moe_testing_fail_stage(1)
+    with pytest.raises(L.MoeError) as exc:
+        L.moe_layer_forward(cfg, ex, W, d["x"], out, None, ws, s)
+    assert exc.value.status == L.MOE_ERR_CUDA
+    L.moe_layer_forward(cfg, ex, W, d["x"], out, None, ws, s)   # injector is off again
+    ws2 = torch.zeros_like(ws)
+    ref = torch.zeros_like(out)
+    L.moe_layer_forward(cfg, ex, W, d["x"], ref, None, ws2, s)  # a fresh workspace
+    L.moe_check_errors(s)
+    assert torch.equal(out, ref)
+
+    g = torch.cuda.CUDAGraph()
+    L.moe_testing_fail_stage(1)
+    with torch.cuda.stream(s):
+        g.capture_begin()
+        try:
+            with pytest.raises(L.MoeError):
+                L.moe_layer_forward(cfg, ex, W, d["x"], out, None, ws, s)
+        finally:
+            g.capture_end()   # raises if the pack stream was left forked
+    L.moe_testing_fail_stage(-1)
+    del g
+    torch.cuda.synchronize()

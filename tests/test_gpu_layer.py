@@ -133,7 +133,7 @@ def test_layer_tiny_full(out_fp32, fuse_combine):
     check_permutation(wl, d, gidx)
     ref, _ = O.layer_forward(f64(d["x"]), f64(d["Wr"]), None, f64(d["W13"]), f64(d["W2"]),
                              oracle_cfg(wl))
-    assert_layer_close(f64(out), ref)
+    assert_layer_close(out, ref)
 
 
 # ---------------------------------------------------------------- small grouped layers, every token
@@ -151,7 +151,7 @@ def test_layer_small_grouped_full(I_shared, T):
     check_routing(wl, dp, a, st["oracle_logits"])
     ref, _ = O.layer_forward(f64(d["x"]), f64(d["Wr"]), bias32(d["bias"]), f64(d["W13"]),
                              f64(d["W2"]), oracle_cfg(wl), f64(d["Ws13"]), f64(d["Ws2"]))
-    assert_layer_close(f64(out), ref)
+    assert_layer_close(out, ref)
     for ex in (L.exec_config(out_fp32=1), L.exec_config(out_fp32=0),
                L.exec_config(out_fp32=1, fuse_gather=0),
                L.exec_config(out_fp32=1, overlap=1, chunk_axis=0, chunk_tokens=37),
@@ -170,7 +170,7 @@ def test_layer_small_grouped_full(I_shared, T):
         gidx = check_routing(wl, d, a, st["oracle_logits"])
         ref, _ = O.layer_forward(f64(d["x"]), f64(d["Wr"]), bias32(d["bias"]), f64(d["W13"]),
                                  f64(d["W2"]), oracle_cfg(wl), f64(d["Ws13"]), f64(d["Ws2"]))
-        assert_layer_close(f64(out), ref)
+        assert_layer_close(out, ref)
     check_permutation(wl, d, gidx)
 
 
@@ -192,7 +192,7 @@ def test_layer_decode_full(big_weights, ex):
     gidx = check_routing(wl, d, a, st["oracle_logits"])
     check_permutation(wl, d, gidx)
     ref, _ = oracle_tokens(wl, d, np.arange(wl.T))
-    assert_layer_close(f64(out), ref)
+    assert_layer_close(out, ref)
 
 
 # ---------------------------------------------------------------- prefill / skewed: sampled
@@ -226,7 +226,7 @@ def test_layer_prefill_sampled(prefill_inputs, ex):
     gidx = check_routing(wl, d, a, st["oracle_logits"])
     if ex.get("overlap", 0) == 0 and ex["out_fp32"] == 1:
         check_permutation(wl, d, gidx)
-    assert_layer_close(f64(out[torch.as_tensor(toks, device=DEV)]), ref)
+    assert_layer_close(out[torch.as_tensor(toks, device=DEV)], ref)
 
 
 def test_layer_skewed_sampled(big_weights):
@@ -242,7 +242,7 @@ def test_layer_skewed_sampled(big_weights):
                L.exec_config(out_fp32=1, fuse_combine=1)):
         out, a = run_layer(wl, d, ex)
         gidx = check_routing(wl, d, a, st["oracle_logits"])
-        assert_layer_close(f64(out[torch.as_tensor(toks, device=DEV)]), ref)
+        assert_layer_close(out[torch.as_tensor(toks, device=DEV)], ref)
     check_permutation(wl, d, gidx)
 
 

@@ -5,8 +5,9 @@ serving loop with a fixed memory plan, a latency-critical path where an
 allocation may synchronise the device) can pass no workspace. This checks,
 through the C ABI, that the allocation-free variant gives exactly what the
 workspace-taking moe_dispatch gives, on two calls in a row (the second one
-reuses the library's scratch array as the first left it), and that inputs
-larger than its fixed scratch are refused.
+reuses the library's scratch array as the first left it), that repeated
+calls leave the device's free memory unchanged, and that inputs larger than
+its fixed scratch are refused.
 """
 
 import ctypes
@@ -51,6 +52,25 @@ def test_dispatch_noalloc_matches_dispatch_twice():
         L.moe_check_errors()
         for name in ref:   # integer and copy outputs: bit for bit
             assert torch.equal(got[name], ref[name]), f"call {call}: {name} differs"
+
+
+def test_dispatch_noalloc_leaves_free_device_memory_unchanged():
+    L.load()
+    T, E, k, H = 2048, 256, 8, 512
+    cfg = L.config(T, H, E, k, 128, 0, 1, 1)
+    g = torch.Generator(device=DEV).manual_seed(7)
+    x = torch.randn((T, H), generator=g, device=DEV).to(torch.bfloat16)
+    idx = torch.from_numpy(_routing(T, E, k, 99)).to(DEV)
+    out = _outputs(T, E, k, H)
+    args = (cfg, x, idx, out["counts"], out["offsets"], out["rst"], out["slot"], out["xp"])
+    L.moe_dispatch_noalloc(*args)   # the first call on the device finds the scratch array
+    torch.cuda.synchronize()
+    free0 = torch.cuda.mem_get_info()[0]
+    for _ in range(3):
+        L.moe_dispatch_noalloc(*args)
+    torch.cuda.synchronize()
+    assert torch.cuda.mem_get_info()[0] == free0
+    L.moe_check_errors()
 
 
 def test_dispatch_noalloc_rejects_inputs_beyond_its_scratch():

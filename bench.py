@@ -76,6 +76,8 @@ def parse():
                    help="the dispatch + combine data-movement sweep instead of a layer: identity "
                         "experts, H=7168, E=256, top-8 uniform routing, T in 1024..65536; one JSON "
                         "line with the HBM GB/s of the permutation, dispatch and combine kernels")
+    p.add_argument("--sweep-t", default=None,
+                   help="comma-separated token counts of the sweep (default: 1024,4096,16384,65536)")
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--cpu-tokens", type=int, default=None,
                    help="oracle sample size (tokens); default 128, or 8 with --precision "
@@ -934,7 +936,9 @@ def run_sweep(args, rank, world, local, device):
                 ms += e0.elapsed_time(e1)
         return ms / args.steps
 
-    for T in I.DISPATCH_SWEEP_T:
+    sweep_t = tuple(int(v) for v in args.sweep_t.split(",")) if args.sweep_t else \
+        I.DISPATCH_SWEEP_T
+    for T in sweep_t:
         c = L.config(T, H, E, k, 2048)
         idx, w = I.uniform_routing(T, E, k, seed=rank, device=device)
         x = I.randn((T, H), 1.0, torch.bfloat16, rank, "x", device)
@@ -975,7 +979,7 @@ def run_sweep(args, rank, world, local, device):
         "scaling": "weak", "vs_baseline": None, "dtype": "bf16 rows, fp32 combine",
         "data": "synthetic (seeded N(0,1) rows, uniform routing)",
         "config": {"workload": "dispatch+combine sweep", "H": H, "E": E, "k": k,
-                   "T": list(I.DISPATCH_SWEEP_T),
+                   "T": list(sweep_t),
                    "l2": "a 256 MB buffer is written between timed launches"},
         "peak": hbm, "peak_source": f"hbm_gbs of {src}", "sweep": rows,
         "gpu_launches": L.moe_launch_count() - n0,

@@ -275,17 +275,24 @@ __global__ void __launch_bounds__(PERM_WARPS * 32) perm_single_kernel(
 }
 
 // x_perm[slot_row[t*k + j]] = x[t] for every token t and slot j (16-byte vectors).
+// The slot rows of a token are read eight at a time before their stores, so a
+// thread has its row reads in flight together rather than one after another.
 __global__ void dispatch_rows_kernel(const uint4* __restrict__ x, int T, int vpr, int k,
                                      const int32_t* __restrict__ slot_row,
                                      uint4* __restrict__ x_perm) {
+  constexpr int KB = 8;
   const size_t total = (size_t)T * vpr;
   for (size_t i = blockIdx.x * (size_t)blockDim.x + threadIdx.x; i < total;
        i += (size_t)gridDim.x * blockDim.x) {
     const size_t t = i / vpr, v = i % vpr;
     const uint4 val = x[i];
-    for (int j = 0; j < k; ++j) {
-      const int r = slot_row[t * k + j];
-      x_perm[(size_t)r * vpr + v] = val;
+    for (int j0 = 0; j0 < k; j0 += KB) {
+      int r[KB];
+#pragma unroll
+      for (int q = 0; q < KB; ++q) r[q] = j0 + q < k ? slot_row[t * k + j0 + q] : -1;
+#pragma unroll
+      for (int q = 0; q < KB; ++q)
+        if (j0 + q < k) x_perm[(size_t)r[q] * vpr + v] = val;
     }
   }
 }
@@ -305,10 +312,14 @@ __global__ void gather_rows_kernel(const uint4* __restrict__ x, int vpr,
 }
 
 // out[t] = sum_j w[t,j] * y_perm[slot_row[t*k+j]] (+ shared[t]); 8 elements per thread-step.
+// The slots are taken four at a time: their rows and weights first, then all
+// eight 16-byte row loads, then the fused multiply-adds in slot order (the
+// same order, and so the same rounding, as one slot after another).
 __global__ void combine_kernel(const float4* __restrict__ y_perm, int T, int vpr, int k,
                                const int32_t* __restrict__ slot_row, const float* __restrict__ w,
                                const float4* __restrict__ shared, void* __restrict__ out,
                                int out_fp32, int* __restrict__ err) {
+  constexpr int KB = 4;
   const int nrows = T * k;
   const size_t total = (size_t)T * vpr;
   for (size_t i = blockIdx.x * (size_t)blockDim.x + threadIdx.x; i < total;
@@ -317,18 +328,42 @@ __global__ void combine_kernel(const float4* __restrict__ y_perm, int T, int vpr
     float acc[8];
 #pragma unroll
     for (int q = 0; q < 8; ++q) acc[q] = 0.f;
-    for (int j = 0; j < k; ++j) {
-      const int r = slot_row[t * k + j];
-      if (r < 0 || r >= nrows) {  // not a packed row: skip it and report
-        atomicExch(err, (int)MOE_ERR_DEVICE_CHECK);
-        continue;
-      }
-      const float wj = w[t * k + j];
-      const float4 y0 = y_perm[((size_t)r * vpr + v) * 2];
-      const float4 y1 = y_perm[((size_t)r * vpr + v) * 2 + 1];
-      const float yv[8] = {y0.x, y0.y, y0.z, y0.w, y1.x, y1.y, y1.z, y1.w};
+    for (int j0 = 0; j0 < k; j0 += KB) {
+      int r[KB];
+      float wj[KB];
 #pragma unroll
-      for (int q = 0; q < 8; ++q) acc[q] = fmaf(wj, yv[q], acc[q]);
+      for (int q = 0; q < KB; ++q) {
+        const int j = j0 + q;
+        r[q] = -1;
+        wj[q] = 0.f;
+        if (j < k) {
+          const int rr = slot_row[t * k + j];
+          if (rr < 0 || rr >= nrows) {  // not a packed row: skip it and report
+            atomicExch(err, (int)MOE_ERR_DEVICE_CHECK);
+          } else {
+            r[q] = rr;
+            wj[q] = w[t * k + j];
+          }
+        }
+      }
+      float4 y[KB][2];
+#pragma unroll
+      for (int q = 0; q < KB; ++q) {
+        if (r[q] >= 0) {
+          y[q][0] = y_perm[((size_t)r[q] * vpr + v) * 2];
+          y[q][1] = y_perm[((size_t)r[q] * vpr + v) * 2 + 1];
+        } else {
+          y[q][0] = y[q][1] = make_float4(0.f, 0.f, 0.f, 0.f);
+        }
+      }
+#pragma unroll
+      for (int q = 0; q < KB; ++q) {
+        if (r[q] < 0) continue;
+        const float yv[8] = {y[q][0].x, y[q][0].y, y[q][0].z, y[q][0].w,
+                             y[q][1].x, y[q][1].y, y[q][1].z, y[q][1].w};
+#pragma unroll
+        for (int e = 0; e < 8; ++e) acc[e] = fmaf(wj[q], yv[e], acc[e]);
+      }
     }
     if (shared) {
       const float4 s0 = shared[i * 2], s1 = shared[i * 2 + 1];

@@ -56,10 +56,11 @@ def parse():
     p.add_argument("--mode", choices=("seq", "overlap-tokens", "overlap-experts"), default="seq")
     p.add_argument("--chunk-tokens", type=int, default=512)
     p.add_argument("--expert-chunks", type=int, default=8)
-    p.add_argument("--fuse-gather", action="store_true",
-                   help="for decode-sized batches, gather the token rows inside GEMM1's operand "
-                        "loads (TMA gather4) instead of packing x_perm with a dispatch kernel "
-                        "(measured 1.3 %% slower at decode with the dynamic unit scheduler)")
+    p.add_argument("--dispatch", choices=("packed", "gather4", "gemm1"), default="packed",
+                   help="packed: a dispatch kernel packs x_perm before GEMM1; gather4: for "
+                        "decode-sized batches GEMM1's operand loads gather the token rows "
+                        "(TMA gather4), no x_perm; gemm1: the dispatch copy runs inside the "
+                        "GEMM1 launch (pack warps, hidden behind the shared expert's units)")
     p.add_argument("--pack", choices=("auto", "yes", "no"), default="auto",
                    help="tile-pack the expert weights at load (auto: yes for bf16, "
                         "no for fp8, which has no packed form)")
@@ -222,11 +223,12 @@ def scale_bytes(rows, n, fp8):
     return 0 if not fp8 else rows * 4 if fp8 == 1 else rows * (n // 128)
 
 
-def algorithmic(wl, touched, fused_gather=True, fp8=0, fused_combine=False):
+def algorithmic(wl, touched, fused_gather=True, fp8=0, fused_combine=False, pack_in_gemm1=False):
     """Algorithmic bytes and flops of each stage for one forward.
 
     GEMM1's token operand is counted as R*H*eb either way (packed rows read, or
     the same rows gathered from x); a fused dispatch has no copy of its own.
+    With the copy inside GEMM1 (pack_in_gemm1) its bytes move to the GEMM1 stage.
     FP8 (eb = 1; fp8 = 1 row scales, 2 block scales): the dispatch stage also
     quantizes x (bf16 read, e4m3 + scales written) and the GEMM1 stage also
     quantizes h (bf16 read, e4m3 + scales); the GEMMs read the scales of their
@@ -257,6 +259,9 @@ def algorithmic(wl, touched, fused_gather=True, fp8=0, fused_combine=False):
         if Is else 0,
         "combine": R * H * 4 + (T * H * 4 if Is else 0) + T * H * 2 + R * 8,
     }
+    if pack_in_gemm1 and not fused_gather:
+        b["gemm1"] += T * H * eb + R * H * eb
+        b["dispatch"] -= T * H * eb + R * H * eb
     if fused_combine:
         b["router"] += T * H * 4
         b["gemm2"] += T * H * 4 - R * H * 4
@@ -531,12 +536,25 @@ def packs(args, wl):
     return args.pack in ("auto", "yes")
 
 
+def dispatch_flag(args, wl):
+    """moe_exec.fuse_gather of the run: 0 packed, 1 gather4, 2 copy inside GEMM1."""
+    return {"packed": 0, "gather4": 1, "gemm1": 2}[args.dispatch]
+
+
+def dispatch_label(args, wl):
+    f = dispatch_flag(args, wl)
+    if f == 1 and wl.T * wl.k <= 24 * wl.E:
+        return "fused into GEMM1 (TMA gather4)"
+    if f == 2 and args.mode == "seq" and args.precision != "fp8-block":
+        return "inside the GEMM1 launch (pack warps write x_perm behind the shared expert)"
+    return "packed x_perm (dispatch kernel)"
+
+
 def config_of(wl, args):
     return {"workload": wl.name, "T": wl.T, "H": wl.H, "E": wl.E, "k": wl.k, "I": wl.I,
             "I_shared": wl.I_shared, "gating": ("sigmoid+bias, 8 groups keep 4, top-8, x2.5"
                                                 if wl.gate == 1 else "softmax top-k"),
-            "mode": args.mode, "dispatch": "fused into GEMM1 (TMA gather4)"
-            if (args.fuse_gather and wl.T * wl.k <= 24 * wl.E) else "packed x_perm",
+            "mode": args.mode, "dispatch": dispatch_label(args, wl),
             "weights": "tile-packed at load (moe_pack_weights)" if packs(args, wl) else "row-major",
             "precision": {"bf16": "bf16 expert GEMMs",
                           "fp8": "e4m3 expert GEMMs, per-row fp32 scales (weights quantized "
@@ -562,10 +580,13 @@ def run_ours(args, wl, rank, world, local, device):
                                "overlap-experts": dict(overlap=1, chunk_axis=1,
                                                        n_expert_chunks=args.expert_chunks)})[
         args.mode]
-    fuse = 1 if args.fuse_gather else 0
-    # the library fuses the dispatch only for decode-sized batches (<= 24 rows per expert)
-    fused = bool(fuse) and wl.T * wl.k <= 24 * wl.E
+    fuse = dispatch_flag(args, wl)
+    # the library gathers in GEMM1 only for decode-sized batches (<= 24 rows per expert)
+    fused = fuse == 1 and wl.T * wl.k <= 24 * wl.E
     fusable = wl.T * wl.k <= 24 * wl.E  # the library would fuse the dispatch on request
+    # the dispatch copy inside GEMM1: sequential forwards, bf16 or row-scaled e4m3
+    in_gemm1_ok = args.mode == "seq" and args.precision != "fp8-block"
+    in_gemm1 = fuse == 2 and in_gemm1_ok
     fp8 = {"bf16": 0, "fp8": 1, "fp8-block": 2}[args.precision]
     fc = 1 if args.fuse_combine else 0
     ex = L.exec_config(fuse_gather=fuse, fp8=fp8, fuse_combine=fc, **mode)
@@ -675,16 +696,24 @@ def run_ours(args, wl, rank, world, local, device):
 
     stage_ms = traced(fuse)
     dispatch_fusion = None
-    if fusable:  # the packed dispatch against the dispatch fused into GEMM1 (same batch)
-        pk_ms = stage_ms if not fused else traced(0)
-        fz_ms = stage_ms if fused else traced(1)
-        extra = fz_ms["gemm1"] - pk_ms["gemm1"]
-        dispatch_fusion = {"active": "fused" if fused else "packed",
+    # the packed dispatch against the dispatch fused into GEMM1 (same batch): the
+    # copy inside the GEMM1 launch at every size, TMA gather4 at decode sizes;
+    # hidden_frac = 1 - (GEMM1 fused - GEMM1 packed) / dispatch kernel
+    if in_gemm1_ok and args.layers == 1:
+        pk_ms = stage_ms if fuse == 0 else traced(0)
+        dispatch_fusion = {"active": {0: "packed", 1: "gather4" if fused else "packed",
+                                      2: "gemm1"}[fuse],
                            "dispatch_ms_packed": round(pk_ms["dispatch"], 4),
                            "gemm1_ms_packed": round(pk_ms["gemm1"], 4),
-                           "gemm1_ms_fused": round(fz_ms["gemm1"], 4),
-                           "hidden_frac": round(1.0 - extra / pk_ms["dispatch"], 3)
-                           if pk_ms["dispatch"] > 0 else None}
+                           "layer_ms_packed": round(sum(pk_ms.values()), 4)}
+        forms = [("gemm1", 2)] + ([("gather4", 1)] if fusable else [])
+        for name, flag in forms:
+            fz_ms = stage_ms if fuse == flag else traced(flag)
+            extra = fz_ms["gemm1"] + fz_ms["dispatch"] - pk_ms["gemm1"]
+            dispatch_fusion[f"gemm1_ms_{name}"] = round(fz_ms["gemm1"], 4)
+            dispatch_fusion[f"layer_ms_{name}"] = round(sum(fz_ms.values()), 4)
+            dispatch_fusion[f"hidden_frac_{name}"] = round(1.0 - extra / pk_ms["dispatch"], 3) \
+                if pk_ms["dispatch"] > 0 else None
 
     # --- end to end through the C ABI with host buffers: every step copies its
     # input batch in from pinned host memory and its output back out, on two
@@ -760,7 +789,7 @@ def run_ours(args, wl, rank, world, local, device):
                    "ms_sequential_unchunked": round(sum(stage_ms.values()), 4)}
 
     hbm, tf_burst, tf_sust, src = peaks()
-    b, f = algorithmic(wl, touched, fused, fp8, bool(fc))
+    b, f = algorithmic(wl, touched, fused, fp8, bool(fc), pack_in_gemm1=in_gemm1)
     g1 = stage_ms["gemm1"] / 1e3
     # GEMM1's own bytes (the FP8 GEMM1 stage also holds the h quantization)
     R = wl.T * wl.k

@@ -127,6 +127,15 @@ struct FfnGroup {
   // Dynamic unit scheduling (two ints, 0 before the first launch that uses them;
   // launches sharing them must run one after another): null = static.
   int* sched;
+  // Dispatch fused into GEMM1 (pack_src non-null, x = the packed rows it
+  // writes): packed row r = pack_src row pack_rst[r] (pack_src_rows rows, the
+  // activation row size); pack_next (one int) and pack_ready (one int per
+  // expert of the group) are 0 before the first launch and left at 0.
+  const void* pack_src;
+  const int32_t* pack_rst;
+  int pack_src_rows;
+  int* pack_next;
+  int* pack_ready;
 };
 
 // Routed group plus an optional dense group (the shared expert, same I) in one

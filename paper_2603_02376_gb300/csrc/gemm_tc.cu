@@ -37,7 +37,16 @@
 //              by the fused combine);
 //   warp 10    block-scaled FP8 only: the stage's UE8M0 exponents as scale
 //              images in shared memory, which the MMA thread copies to TMEM
-//              (tcgen05.cp) ahead of block_scale MMAs.
+//              (tcgen05.cp) ahead of block_scale MMAs;
+//   warps 10-13 GEMM1 with bf16 or row-scaled e4m3 operands: the dispatch
+//              fused into the launch (GemmArgs::pack_dst). They copy the
+//              token rows into the packed order, a chunk of rows at a time
+//              taken from a global counter in row (= expert) order, and count
+//              each expert's packed rows; the producer waits for an expert's
+//              count before loading its token tiles. The shared expert's
+//              units (which read x itself) come first in the unit order, so
+//              the copy runs while they compute: the paper's dispatch hidden
+//              behind the layer's own compute, inside one kernel.
 // For SwiGLU the gate and up tiles of the same 128 features are two MMAs into
 // two TMEM column ranges, so one thread holds both g and u of its feature.
 // When two accumulators fit in TMEM's 512 columns they alternate, so the
@@ -68,6 +77,8 @@ constexpr int B_BOX = 16;         // token rows per TMA box (tile remainders)
 constexpr int B_BIG = 64;         // token rows per TMA box (bulk of tiles of >= 64 rows)
 constexpr int NUM_THREADS = 320;  // 10 warps: producer, MMA, 8 epilogue
 constexpr int NUM_WARPS_MX = 11;  // block-scaled FP8: and a scale warp
+constexpr int PACK_WARPS = 4;     // GEMM1 (bf16, row-scaled e4m3): warps copying token rows
+constexpr int PACK_ROWS = 4;      // token rows per chunk a pack warp takes
 constexpr uint64_t WAIT_LIMIT_NS = 2000000000ull;  // default limit of every barrier wait
 
 
@@ -117,6 +128,15 @@ struct Tile {
   // (<= 8 KiB) and the 1 KiB alignment slack this stays under 227 KiB per CTA.
   static constexpr int STAGES_RAW = (217 * 1024 - SF_STG_BYTES) / STAGE_BYTES;
   static constexpr int STAGES = STAGES_RAW > 12 ? 12 : STAGES_RAW;
+  // Without block scales the stages are carved from one byte ring at the size
+  // each unit needs (its weight tiles plus its padded token rows): a unit with
+  // few token rows keeps more weight bytes in flight than a full-tile stage
+  // count would allow (a 16-row unit of the 256-row kernel: 6 stages, not 3).
+  // Up to SLOTS stages are in flight. Block-scaled FP8 keeps fixed stages
+  // (its scale images and TMEM scale columns are laid out per stage).
+  static constexpr bool VAR = !MX;
+  static constexpr int SLOTS = VAR ? 12 : STAGES;
+  static constexpr int RING_BYTES = VAR ? (217 * 1024) & ~1023 : STAGES * STAGE_BYTES;
   static constexpr int ACC_COLS = TWO_ACC ? 2 * NMAX : NMAX;  // one accumulator (gate | up)
   // MX: each stage's scales live in TMEM columns of their own (4 per image)
   // until the stage's MMAs complete
@@ -136,6 +156,10 @@ constexpr int UNIT_RING = 8;  // units announced ahead by the producer (a power 
 struct Ctrl {
   uint64_t full[12];
   uint64_t empty[12];
+  // byte ring (Tile::VAR): offset and size of the stage held by each slot,
+  // written by the producer before it arms the slot's full barrier
+  uint32_t slot_off[12];
+  uint32_t slot_len[12];
   uint64_t acc_full[2];
   uint64_t acc_empty[2];
   uint64_t drain;
@@ -402,6 +426,17 @@ struct GemmArgs {
   // the first launch; launches sharing them must not overlap in time. Null:
   // CTA b runs units b, b + grid, b + 2 grid, ...
   int* sched;
+  // Dispatch fused into GEMM1 (pack_dst non-null; group 0 only): packed row r
+  // of group 0 is pack_src row pack_rst[r] (pack_src_rows rows of K elements).
+  // pack_next hands out chunks of PACK_ROWS rows; pack_ready[e] counts the
+  // packed rows of expert e_begin + e. Both are 0 at the first launch; the last
+  // CTA out sets them back to 0.
+  const uint4* pack_src;
+  uint4* pack_dst;
+  const int32_t* pack_rst;
+  int pack_src_rows;
+  int* pack_next;
+  int* pack_ready;
   uint64_t wait_limit_ns;  // limit of each barrier wait
   long stall_fill;         // testing: CTA 0 never issues this fill (-1 = none), so the
                            // MMA's wait on it runs out and the abort path is exercised
@@ -478,10 +513,25 @@ __device__ __forceinline__ Unit decode_unit(int u, const int* tile_off, const in
 
 // ------------------------------------------------------------------ kernel
 
-constexpr int threads_of(int q) { return q == Q_BLOCK ? NUM_WARPS_MX * 32 : NUM_THREADS; }
+// GEMM1 launches of the bf16 and row-scaled e4m3 forms carry the pack warps
+// (idle and gone at once when the dispatch is not fused).
+__host__ __device__ constexpr bool has_pack(int mode, int q) { return mode == MODE_SWIGLU && q != Q_BLOCK; }
+__host__ __device__ constexpr int threads_of(int mode, int q) {
+  return q == Q_BLOCK ? NUM_WARPS_MX * 32 : NUM_THREADS + (has_pack(mode, q) ? PACK_WARPS * 32 : 0);
+}
+
+__device__ __forceinline__ int ld_acquire(const int* p) {
+  int v;
+  asm volatile("ld.acquire.gpu.global.b32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+  return v;
+}
+
+__device__ __forceinline__ void fence_proxy_async_global() {
+  asm volatile("fence.proxy.async.global;" ::: "memory");
+}
 
 template <int MODE, int NMAX, int Q, bool PK>
-__global__ void __launch_bounds__(threads_of(Q), 1)
+__global__ void __launch_bounds__(threads_of(MODE, Q), 1)
     grouped_gemm_kernel(const __grid_constant__ CUtensorMap tmA0,
                         const __grid_constant__ CUtensorMap tmB0,
                         const __grid_constant__ CUtensorMap tmA1,
@@ -495,7 +545,7 @@ __global__ void __launch_bounds__(threads_of(Q), 1)
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~static_cast<uintptr_t>(1023));
-  uint8_t* sf_stg = smem + TL::STAGES * TL::STAGE_BYTES;  // MX staging (SF_STG_BYTES)
+  uint8_t* sf_stg = smem + TL::RING_BYTES;  // MX staging (SF_STG_BYTES)
   Ctrl* ctrl = reinterpret_cast<Ctrl*>(sf_stg + TL::SF_STG_BYTES);
   int* tile_off = reinterpret_cast<int*>(ctrl + 1);
   int* row_off = tile_off + a.n_exp + 1;
@@ -505,7 +555,7 @@ __global__ void __launch_bounds__(threads_of(Q), 1)
   const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
 
   if (threadIdx.x == 0) {
-    for (int s = 0; s < TL::STAGES; ++s) {
+    for (int s = 0; s < TL::SLOTS; ++s) {
       mbar_init(smem_u32(&ctrl->full[s]), MX ? 2 : 1);  // MX: the producer and the scale warp
       mbar_init(smem_u32(&ctrl->empty[s]), 1);
     }
@@ -606,6 +656,8 @@ __global__ void __launch_bounds__(threads_of(Q), 1)
     int stage = 0;
     uint32_t phase = 0;
     long fills = 0;
+    long tail = 0;      // VAR: oldest fill whose stage may still be in use
+    uint32_t head = 0;  // VAR: ring offset after the newest stage
     bool ok = true;
     // lane 0 takes the next unit one unit ahead, so the atomic's round trip
     // overlaps the current unit's loads
@@ -633,6 +685,37 @@ __global__ void __launch_bounds__(threads_of(Q), 1)
       }
       if (u >= total_units) break;
       const Unit U = decode_unit<NMAX>(u, tile_off, row_off, a, units1, kblocks);
+      if (has_pack(MODE, Q) && a.pack_dst && U.grp == 0) {
+        // fused dispatch: the expert's token rows must all be packed before its
+        // token tiles are loaded (bounded wait on the pack warps' count)
+        int okp = 1;
+        if (lane == 0) {
+          const int need = row_off[U.e + 1] - row_off[U.e];
+          const int* rp = a.pack_ready + U.e;
+          if (ld_acquire(rp) < need) {
+            const uint64_t t0 = global_timer_ns();
+            while (ld_acquire(rp) < need) {
+              if (*abort_flag) {
+                okp = 0;
+                break;
+              }
+              if (global_timer_ns() - t0 > a.wait_limit_ns) {
+                *abort_flag = 1;
+                atomicExch(err, (int)MOE_ERR_TIMEOUT);
+                okp = 0;
+                break;
+              }
+              __nanosleep(128);
+            }
+          }
+          fence_proxy_async_global();  // the rows were written by generic stores; TMA reads them
+        }
+        okp = __shfl_sync(0xffffffffu, okp, 0);
+        if (!okp) {
+          ok = false;
+          break;
+        }
+      }
       const CUtensorMap* mA = U.grp ? &tmA1 : &tmA0;
       const CUtensorMap* mB = U.grp ? &tmB1 : &tmB0;
       const CUtensorMap* mBbig = U.grp ? &tmB1big : &tmB0big;
@@ -655,9 +738,10 @@ __global__ void __launch_bounds__(threads_of(Q), 1)
         }
       for (int kb = U.kb0; kb < U.kb1; ++kb) {
         const uint32_t full = smem_u32(&ctrl->full[stage]);
-        const uint32_t sa = smem_u32(smem + stage * TL::STAGE_BYTES);
-        const uint32_t sb = sa + TL::NA * TL::A_BYTES;
+        uint32_t pos = 0;  // the stage's offset in the ring
         auto issue = [&]() {  // lane 0: arm the stage barrier, load the tiles
+          const uint32_t sa = smem_u32(smem + pos);
+          const uint32_t sb = sa + TL::NA * TL::A_BYTES;
           mbar_arrive_expect_tx(full, bytes);
 #pragma unroll
           for (int t = 0; t < TL::NA; ++t) {
@@ -678,10 +762,39 @@ __global__ void __launch_bounds__(threads_of(Q), 1)
         };
         int got = 1;
         if (lane == 0) {
-          got = wait_bounded(smem_u32(&ctrl->empty[stage]), phase ^ 1, abort_flag, err,
-                             a.wait_limit_ns)
-                    ? 1
-                    : 0;
+          if constexpr (TL::VAR) {
+            // place the stage at the head, or at the ring's start when it does not
+            // fit before the end; free the oldest stages (wait for their MMAs)
+            // while one still in flight overlaps it or every slot is taken
+            pos = head + bytes <= (uint32_t)TL::RING_BYTES ? head : 0u;
+            while (true) {
+              bool clash = fills - tail >= TL::SLOTS;
+              for (long i = tail; !clash && i < fills; ++i) {
+                const int sl = (int)(i % TL::SLOTS);
+                const uint32_t o = ctrl->slot_off[sl], l = ctrl->slot_len[sl];
+                clash = pos < o + l && o < pos + bytes;
+              }
+              if (!clash) break;
+              if (!wait_bounded(smem_u32(&ctrl->empty[tail % TL::SLOTS]),
+                                (uint32_t)((tail / TL::SLOTS) & 1), abort_flag, err,
+                                a.wait_limit_ns)) {
+                got = 0;
+                break;
+              }
+              ++tail;
+            }
+            if (got) {
+              ctrl->slot_off[stage] = pos;
+              ctrl->slot_len[stage] = bytes;
+              head = pos + bytes;
+            }
+          } else {
+            got = wait_bounded(smem_u32(&ctrl->empty[stage]), phase ^ 1, abort_flag, err,
+                               a.wait_limit_ns)
+                      ? 1
+                      : 0;
+            pos = (uint32_t)(stage * TL::STAGE_BYTES);
+          }
           if (got && blockIdx.x == 0 && fills == a.stall_fill) got = 2;  // skip this fill
           if (got == 1) issue();
         }
@@ -691,6 +804,8 @@ __global__ void __launch_bounds__(threads_of(Q), 1)
           break;
         }
         if (gather && got == 1) {
+          pos = __shfl_sync(0xffffffffu, pos, 0);
+          const uint32_t sb = smem_u32(smem + pos) + TL::NA * TL::A_BYTES;
 #pragma unroll
           for (int h = 0; h < 2; ++h) {
             const int g = lane + 32 * h;
@@ -700,7 +815,7 @@ __global__ void __launch_bounds__(threads_of(Q), 1)
           }
         }
         ++fills;
-        if (++stage == TL::STAGES) {
+        if (++stage == TL::SLOTS) {
           stage = 0;
           phase ^= 1;
         }
@@ -708,11 +823,11 @@ __global__ void __launch_bounds__(threads_of(Q), 1)
     }
     if (!ok && lane == 0) {
       // let the copies already issued land before the CTA can exit
-      for (int s = 0; s < TL::STAGES; ++s) {
+      for (int s = 0; s < TL::SLOTS; ++s) {
         if (fills <= s) continue;
-        const long f = s + ((fills - 1 - s) / TL::STAGES) * TL::STAGES;  // last fill of stage s
+        const long f = s + ((fills - 1 - s) / TL::SLOTS) * TL::SLOTS;  // last fill of slot s
         if (blockIdx.x == 0 && f == a.stall_fill) continue;  // never issued
-        const uint32_t par = (uint32_t)((f / TL::STAGES) & 1);
+        const uint32_t par = (uint32_t)((f / TL::SLOTS) & 1);
         const uint64_t t0 = global_timer_ns();
         while (!mbar_try_wait(smem_u32(&ctrl->full[s]), par) &&
                global_timer_ns() - t0 < a.wait_limit_ns) {
@@ -751,7 +866,8 @@ __global__ void __launch_bounds__(threads_of(Q), 1)
             break;
           }
           tc_fence_after();
-          const uint32_t sa = smem_u32(smem + stage * TL::STAGE_BYTES);
+          const uint32_t sa =
+              smem_u32(smem + (TL::VAR ? ctrl->slot_off[stage] : stage * TL::STAGE_BYTES));
           const uint32_t sb = sa + TL::NA * TL::A_BYTES;
           if constexpr (MX) {
             // the stage's scale images -> its TMEM scale columns: A tile t at
@@ -790,7 +906,7 @@ __global__ void __launch_bounds__(threads_of(Q), 1)
           }
           issued = true;
           mma_commit(smem_u32(&ctrl->empty[stage]));
-          if (++stage == TL::STAGES) {
+          if (++stage == TL::SLOTS) {
             stage = 0;
             phase ^= 1;
           }
@@ -924,6 +1040,70 @@ __global__ void __launch_bounds__(threads_of(Q), 1)
         if (++stage == TL::STAGES) {
           stage = 0;
           phase ^= 1;
+        }
+      }
+    }
+  } else if (has_pack(MODE, Q) && warp >= 10) {
+    // ------------------------------------------------------------------ pack warps
+    // Fused dispatch: packed row r of group 0 = source row pack_rst[r]. A warp
+    // takes PACK_ROWS consecutive packed rows from the global counter, copies
+    // them with 16-byte vectors (each lane two columns of every row in flight
+    // at once), then adds the rows to their experts' counts with release
+    // semantics. Rows with a source index outside the source matrix are left
+    // unwritten and latched as MOE_ERR_DEVICE_CHECK; they are still counted.
+    if (a.pack_dst) {
+      const int r_begin = row_off[0], r_end = row_off[a.n_exp];
+      const int vpr = a.K * (F8 ? 1 : 2) / 16;  // 16-byte vectors per row
+      const int n_chunks = (r_end - r_begin + PACK_ROWS - 1) / PACK_ROWS;
+      while (!*abort_flag) {
+        int c = 0;
+        if (lane == 0) c = atomicAdd(a.pack_next, 1);
+        c = __shfl_sync(0xffffffffu, c, 0);
+        if (c >= n_chunks) break;
+        const int r0 = r_begin + c * PACK_ROWS, nr = min(PACK_ROWS, r_end - r0);
+        int src = -1;
+        if (lane < nr) {
+          const int t = a.pack_rst[r0 + lane];
+          if (t >= 0 && t < a.pack_src_rows) src = t;
+          else atomicExch(err, (int)MOE_ERR_DEVICE_CHECK);
+        }
+        int tq[PACK_ROWS];
+#pragma unroll
+        for (int q = 0; q < PACK_ROWS; ++q) tq[q] = __shfl_sync(0xffffffffu, src, q);
+        for (int v0 = lane; v0 < vpr; v0 += 64) {
+          uint4 val[PACK_ROWS][2];
+#pragma unroll
+          for (int q = 0; q < PACK_ROWS; ++q)
+#pragma unroll
+            for (int h = 0; h < 2; ++h)
+              if (tq[q] >= 0 && v0 + 32 * h < vpr)
+                val[q][h] = a.pack_src[(size_t)tq[q] * vpr + v0 + 32 * h];
+#pragma unroll
+          for (int q = 0; q < PACK_ROWS; ++q)
+#pragma unroll
+            for (int h = 0; h < 2; ++h)
+              if (tq[q] >= 0 && v0 + 32 * h < vpr)
+                a.pack_dst[(size_t)(r0 + q) * vpr + v0 + 32 * h] = val[q][h];
+        }
+        __threadfence();
+        fence_proxy_async_global();
+        __syncwarp();
+        if (lane == 0) {
+          int lo = 0, hi = a.n_exp - 1;  // the expert of row r0: last e with row_off[e] <= r0
+          while (lo < hi) {
+            const int mid = (lo + hi + 1) >> 1;
+            if (row_off[mid] <= r0) lo = mid;
+            else hi = mid - 1;
+          }
+          for (int e = lo, r = r0; r < r0 + nr; ++e) {
+            const int end = min(row_off[e + 1], r0 + nr);
+            if (end > r) {
+              asm volatile("red.release.gpu.global.add.s32 [%0], %1;" ::"l"(a.pack_ready + e),
+                           "r"(end - r)
+                           : "memory");
+              r = end;
+            }
+          }
         }
       }
     }
@@ -1077,6 +1257,10 @@ __global__ void __launch_bounds__(threads_of(Q), 1)
     if (atomicAdd(a.sched + 1, 1) == (int)gridDim.x - 1) {
       atomicExch(a.sched, 0);
       atomicExch(a.sched + 1, 0);
+      if (a.pack_dst) {  // and the fused dispatch's counters
+        atomicExch(a.pack_next, 0);
+        for (int e = 0; e < a.n_exp; ++e) atomicExch(a.pack_ready + e, 0);
+      }
     }
   }
 }
@@ -1118,7 +1302,7 @@ long g_stall_fill = -1;
 template <int MODE, int NMAX, bool MX>
 size_t gemm_smem_bytes(int n_exp) {
   using TL = Tile<MODE, NMAX, MX>;
-  return 1024 + (size_t)TL::STAGES * TL::STAGE_BYTES + TL::SF_STG_BYTES + sizeof(Ctrl) +
+  return 1024 + (size_t)TL::RING_BYTES + TL::SF_STG_BYTES + sizeof(Ctrl) +
          2 * sizeof(int) * (n_exp + 1);
 }
 
@@ -1131,7 +1315,7 @@ moe_status launch_gemm(const CUtensorMap& A0, const CUtensorMap& B0, const CUten
   if (cudaFuncSetAttribute(grouped_gemm_kernel<MODE, NMAX, Q, PK>,
                            cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) != cudaSuccess)
     return MOE_ERR_CUDA;
-  grouped_gemm_kernel<MODE, NMAX, Q, PK><<<num_sms(), threads_of(Q), smem, s>>>(A0, B0, A1, B1,
+  grouped_gemm_kernel<MODE, NMAX, Q, PK><<<num_sms(), threads_of(MODE, Q), smem, s>>>(A0, B0, A1, B1,
                                                                               B0big, B1big, args);
   note_launch();
   return launch_status();
@@ -1234,6 +1418,16 @@ moe_status run_ffn(const FfnGroup& g0, const FfnGroup* g1, int H, int I, cudaStr
     args.b_sf_ld1 = g1 ? g1->x_sf_ld : 0;
     args.b_scale_idx0 = g0.x_scale_idx;
   }
+  if (g0.pack_src) {  // the dispatch copy inside GEMM1 (needs the dynamic scheduler's reset)
+    if (gather || MX || !g0.sched || !g0.pack_rst || !g0.pack_next || !g0.pack_ready)
+      return MOE_ERR_UNSUPPORTED;
+    args.pack_src = static_cast<const uint4*>(g0.pack_src);
+    args.pack_dst = static_cast<uint4*>(const_cast<void*>(g0.x));
+    args.pack_rst = g0.pack_rst;
+    args.pack_src_rows = g0.pack_src_rows;
+    args.pack_next = g0.pack_next;
+    args.pack_ready = g0.pack_ready;
+  }
   moe_status st =
       launch_gemm<MODE_SWIGLU, NMAX, Q, PK>(a1, b1, sa1, sb1, b1big, sb1big, args, s);
   if (st != MOE_OK) return st;
@@ -1247,6 +1441,8 @@ moe_status run_ffn(const FfnGroup& g0, const FfnGroup* g1, int H, int I, cudaStr
   }
   if (after_gemm1 && cudaEventRecord(after_gemm1, s) != cudaSuccess) return MOE_ERR_CUDA;
   args.gather0 = nullptr;  // GEMM2 reads h, already in packed row order
+  args.pack_src = nullptr;
+  args.pack_dst = nullptr;
   args.a0_packed = pk ? static_cast<const uint16_t*>(g0.W2) : nullptr;
   args.a1_packed = (pk && g1) ? static_cast<const uint16_t*>(g1->W2) : nullptr;
   if (F8 && !MX) {

@@ -88,7 +88,7 @@ bool valid_exec(const moe_exec* ex, const moe_config* c) {
   if (!ex) return false;
   if (ex->overlap != 0 && ex->overlap != 1) return false;
   if (ex->out_fp32 != 0 && ex->out_fp32 != 1) return false;
-  if (ex->fuse_gather != 0 && ex->fuse_gather != 1) return false;
+  if (ex->fuse_gather < 0 || ex->fuse_gather > 2) return false;
   if (ex->fp8 < 0 || ex->fp8 > 2) return false;
   if (ex->fuse_combine != 0 && ex->fuse_combine != 1) return false;
   if (ex->overlap) {
@@ -155,8 +155,13 @@ struct Layout {
   float* acc;        // [T, H] or null (= the fp32 output)
   // The expert GEMMs' dynamic unit scheduler (two ints): zeroed at the start
   // of each forward; every launch leaves it at 0 (all of a forward's expert
-  // GEMMs run in order on the caller's stream).
+  // GEMMs run in order on the caller's stream). Followed by the dispatch fused
+  // into GEMM1 (pack_in_gemm): its chunk counter and per-expert packed-row
+  // counts, zeroed with it and likewise left at 0 by each launch.
   int32_t* sched;
+  bool pack_in_gemm = false;
+  int32_t* pack_next;   // sched + 2
+  int32_t* pack_ready;  // sched + 3, [E]
   size_t bytes = 0;
 };
 
@@ -211,7 +216,10 @@ Layout carve(const moe_config& c, const moe_exec& ex, void* ws) {
   L.sh_hsf = (c.I_shared && L.fp8_block) ? cv.take<uint8_t>((size_t)(c.I_shared / 128) * T)
                                          : nullptr;
   L.sh_y = (c.I_shared && !L.fuse_combine) ? cv.take<float>(T * c.H) : nullptr;
-  L.sched = cv.take<int32_t>(2);
+  L.sched = cv.take<int32_t>(3 + E);
+  L.pack_next = L.sched ? L.sched + 2 : nullptr;
+  L.pack_ready = L.sched ? L.sched + 3 : nullptr;
+  L.pack_in_gemm = ex.fuse_gather == 2 && !ex.overlap && ex.fp8 != 2;
   L.bytes = align_up(cv.off, 256);
   return L;
 }
@@ -359,6 +367,14 @@ FfnGroup routed_group(const moe_config& c, const Layout& L, const moe_weights& w
   const size_t xb = L.fp8 ? 1 : 2;
   if (L.x_perm) {
     g.x = static_cast<const uint8_t*>(L.x_perm) + tk * c.H * xb;
+    if (L.pack_in_gemm) {  // GEMM1 writes x_perm itself
+      g.pack_src = L.fp8 ? static_cast<const void*>(L.x_q + (size_t)t0 * c.H)
+                         : static_cast<const void*>(x + (size_t)t0 * c.H);
+      g.pack_rst = L.rst + tk;
+      g.pack_src_rows = Tc;
+      g.pack_next = L.pack_next;
+      g.pack_ready = L.pack_ready + e0;
+    }
   } else {
     g.x = L.fp8 ? static_cast<const void*>(L.x_q + (size_t)t0 * c.H)
                 : static_cast<const void*>(x + (size_t)t0 * c.H);
@@ -802,13 +818,14 @@ moe_status moe_layer_forward(const moe_config* cfg, const moe_exec* ex, const mo
 
   cudaStream_t s = (cudaStream_t)stream;
   const int dev = current_device();
-  MOE_CUDA(cudaMemsetAsync(L.sched, 0, 2 * sizeof(int32_t), s));
+  MOE_CUDA(cudaMemsetAsync(L.sched, 0, (3 + (size_t)c.E) * sizeof(int32_t), s));
 
   if (!ex->overlap) {
     cudaEvent_t* ev = reinterpret_cast<cudaEvent_t*>(ex->stage_events);
     MOE_TRY(mark(ev, MOE_EV_START, s));
     MOE_TRY(clear_acc(c, L, s));
-    MOE_TRY(pack_tokens(c, L, *w, x, 0, c.T, 0, L.x_perm != nullptr, s, ev, true));
+    MOE_TRY(pack_tokens(c, L, *w, x, 0, c.T, 0, L.x_perm != nullptr && !L.pack_in_gemm, s, ev,
+                        true));
     if (c.I_shared == c.I) {
       MOE_TRY(experts_and_shared(c, L, *w, x, s, ev));
     } else {

@@ -240,7 +240,7 @@ def fp8_prefill(fp8_layer):
 
 @pytest.mark.parametrize("ex", [dict(out_fp32=1), dict(out_fp32=0), dict(out_fp32=1, fuse_gather=0),
                                 dict(out_fp32=1, overlap=1, chunk_axis=1, n_expert_chunks=4),
-                                dict(out_fp32=0, fuse_combine=1)])
+                                dict(out_fp32=0, fuse_combine=1), dict(out_fp32=1, fuse_gather=2)])
 def test_layer_fp8_decode_full(fp8_decode, ex):
     wl = I.DECODE
     d, toks, ref, idx = fp8_decode
@@ -253,7 +253,7 @@ def test_layer_fp8_decode_full(fp8_decode, ex):
 @pytest.mark.parametrize("ex", [dict(out_fp32=1), dict(out_fp32=1, fuse_gather=0),
                                 dict(out_fp32=1, overlap=1, chunk_axis=0, chunk_tokens=512),
                                 dict(out_fp32=1, overlap=1, chunk_axis=1, n_expert_chunks=8),
-                                dict(out_fp32=1, fuse_combine=1)])
+                                dict(out_fp32=1, fuse_combine=1), dict(out_fp32=1, fuse_gather=2)])
 def test_layer_fp8_prefill_sampled(fp8_prefill, ex):
     wl = I.PREFILL
     d, toks, ref, idx = fp8_prefill

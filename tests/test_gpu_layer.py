@@ -4,6 +4,9 @@
 * decode (T=128, DeepSeek-V3 layer): every token checked.
 * prefill (T=4096, balanced) and skewed (T=8192, Zipf): a seeded sample of
   256 tokens, in the sequential mode and both two-stream pipelined modes.
+* every size also with the dispatch copy inside the GEMM1 launch
+  (fuse_gather = 2: GEMM1's pack warps write x_perm while the shared expert
+  computes; the routed tiles wait for their expert's rows).
 Routing is compared bit for bit with the oracle gate run on the GPU's own
 fp32 logits; the GPU logits stay within the fp32 summation bound; the
 permutation of the GPU routing is bit-exact; the layer output is within
@@ -122,13 +125,15 @@ def oracle_tokens(wl, d, toks):
 
 # ---------------------------------------------------------------- tiny: every token
 
+@pytest.mark.parametrize("fuse_gather", [1, 2])
 @pytest.mark.parametrize("fuse_combine", [0, 1])
 @pytest.mark.parametrize("out_fp32", [1, 0])
-def test_layer_tiny_full(out_fp32, fuse_combine):
+def test_layer_tiny_full(out_fp32, fuse_combine, fuse_gather):
     wl = I.TINY
     d = I.layer_inputs(wl, seed=0, device=DEV)
     st = prepare_routing(wl, d)
-    out, a = run_layer(wl, d, L.exec_config(out_fp32=out_fp32, fuse_combine=fuse_combine))
+    out, a = run_layer(wl, d, L.exec_config(out_fp32=out_fp32, fuse_combine=fuse_combine,
+                                            fuse_gather=fuse_gather))
     gidx = check_routing(wl, d, a, st["oracle_logits"])
     check_permutation(wl, d, gidx)
     ref, _ = O.layer_forward(f64(d["x"]), f64(d["Wr"]), None, f64(d["W13"]), f64(d["W2"]),
@@ -165,7 +170,10 @@ def test_layer_small_grouped_full(I_shared, T):
                L.exec_config(out_fp32=0, overlap=1, chunk_axis=0, chunk_tokens=37,
                              fuse_combine=1),
                L.exec_config(out_fp32=1, overlap=1, chunk_axis=1, n_expert_chunks=3,
-                             fuse_combine=1)):
+                             fuse_combine=1),
+               # the dispatch copy inside GEMM1
+               L.exec_config(out_fp32=1, fuse_gather=2),
+               L.exec_config(out_fp32=0, fuse_gather=2, fuse_combine=1)):
         out, a = run_layer(wl, d, ex)
         gidx = check_routing(wl, d, a, st["oracle_logits"])
         ref, _ = O.layer_forward(f64(d["x"]), f64(d["Wr"]), bias32(d["bias"]), f64(d["W13"]),
@@ -179,7 +187,9 @@ def test_layer_small_grouped_full(I_shared, T):
 @pytest.mark.parametrize("ex", [dict(out_fp32=1), dict(out_fp32=0), dict(out_fp32=1, fuse_gather=0),
                                 dict(out_fp32=1, overlap=1, chunk_axis=1, n_expert_chunks=4),
                                 dict(out_fp32=1, packed=1), dict(out_fp32=0, fuse_combine=1),
-                                dict(out_fp32=1, fuse_combine=1, fuse_gather=0)])
+                                dict(out_fp32=1, fuse_combine=1, fuse_gather=0),
+                                dict(out_fp32=1, fuse_gather=2),
+                                dict(out_fp32=1, fuse_gather=2, packed=1)])
 def test_layer_decode_full(big_weights, ex):
     wl = I.DECODE
     ex = dict(ex)
@@ -218,6 +228,8 @@ def prefill_inputs(big_weights):
     dict(out_fp32=1, overlap=1, chunk_axis=1, n_expert_chunks=8),
     dict(out_fp32=1, fuse_combine=1),
     dict(out_fp32=0, overlap=1, chunk_axis=0, chunk_tokens=512, fuse_combine=1),
+    dict(out_fp32=1, fuse_gather=2),
+    dict(out_fp32=0, fuse_gather=2, fuse_combine=1),
 ])
 def test_layer_prefill_sampled(prefill_inputs, ex):
     wl = I.PREFILL
@@ -239,7 +251,9 @@ def test_layer_skewed_sampled(big_weights):
     ref, _ = oracle_tokens(wl, d, toks)
     for ex in (L.exec_config(out_fp32=1), L.exec_config(out_fp32=1, fuse_gather=0),
                L.exec_config(out_fp32=1, overlap=1, chunk_axis=1),
-               L.exec_config(out_fp32=1, fuse_combine=1)):
+               L.exec_config(out_fp32=1, fuse_combine=1),
+               L.exec_config(out_fp32=1, fuse_gather=2),
+               L.exec_config(out_fp32=1, fuse_gather=2, fuse_combine=1)):
         out, a = run_layer(wl, d, ex)
         gidx = check_routing(wl, d, a, st["oracle_logits"])
         assert_layer_close(out[torch.as_tensor(toks, device=DEV)], ref)

@@ -596,7 +596,11 @@ def run_ours(args, wl, rank, world, local, device):
                          L.moe_workspace_size(cfg, L.exec_config(fuse_gather=0, fp8=fp8))),
                      dtype=torch.uint8, device=device)
     out = torch.empty((wl.T, wl.H), dtype=torch.bfloat16, device=device)
-    stream = torch.cuda.current_stream()
+    # a stream of its own: the default stream's handle is NULL, which the C ABI
+    # reads as "no aux stream given" (the library's own pack stream), so the
+    # one-stream comparison of the pipelined modes needs a non-default stream
+    stream = torch.cuda.Stream()
+    torch.cuda.synchronize()
     # the layer runs on tile-packed copies (a load-time layout transform, not part
     # of the timed step); the row-major tensors stay for the CPU oracle
     run_w = {k_: d.get(k_) for k_ in ("W13", "W2", "Ws13", "Ws2")}

@@ -419,7 +419,9 @@ moe_status moe_combine(const moe_config* cfg, const float* y_perm, const int32_t
  * x [T,H] bf16; out [T,H] bf16 or fp32 per ex->out_fp32; aux optional;
  * ws: moe_workspace_size(cfg, ex) bytes. aux_stream: the pack stream of the
  * overlapped pipeline (NULL = an internal high-priority stream); unused when
- * ex->overlap = 0. All work is ordered after prior work on `stream`, and later
+ * ex->overlap = 0. Passing `stream` itself runs the pipelined stage order on
+ * one stream; a caller on the legacy default stream (whose handle is NULL,
+ * the same value as "internal") passes cudaStreamLegacy for that. All work is ordered after prior work on `stream`, and later
  * work on `stream` is ordered after the whole layer. Calls from several host
  * threads are safe; pipelined calls on one device share internal events and
  * enqueue one at a time. Concurrent calls must not share a workspace.

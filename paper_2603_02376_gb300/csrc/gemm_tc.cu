@@ -156,10 +156,9 @@ constexpr int UNIT_RING = 8;  // units announced ahead by the producer (a power 
 struct Ctrl {
   uint64_t full[12];
   uint64_t empty[12];
-  // byte ring (Tile::VAR): offset and size of the stage held by each slot,
-  // written by the producer before it arms the slot's full barrier
+  // byte ring (Tile::VAR): offset of the stage held by each slot, written by
+  // the producer before it arms the slot's full barrier
   uint32_t slot_off[12];
-  uint32_t slot_len[12];
   uint64_t acc_full[2];
   uint64_t acc_empty[2];
   uint64_t drain;
@@ -656,8 +655,12 @@ __global__ void __launch_bounds__(threads_of(MODE, Q), 1)
     int stage = 0;
     uint32_t phase = 0;
     long fills = 0;
-    long tail = 0;      // VAR: oldest fill whose stage may still be in use
-    uint32_t head = 0;  // VAR: ring offset after the newest stage
+    // VAR ring (lane 0): stages are allocated and freed in fill order, so the
+    // bytes in use run from the oldest stage still in flight (slot tslot,
+    // offset toff, its barrier phase parity tpar) to head, wrapping once; nfl
+    // stages are in flight
+    int tslot = 0, nfl = 0;
+    uint32_t tpar = 0, toff = 0, head = 0;
     bool ok = true;
     // lane 0 takes the next unit one unit ahead, so the atomic's round trip
     // overlaps the current unit's loads
@@ -764,28 +767,43 @@ __global__ void __launch_bounds__(threads_of(MODE, Q), 1)
         if (lane == 0) {
           if constexpr (TL::VAR) {
             // place the stage at the head, or at the ring's start when it does not
-            // fit before the end; free the oldest stages (wait for their MMAs)
-            // while one still in flight overlaps it or every slot is taken
-            pos = head + bytes <= (uint32_t)TL::RING_BYTES ? head : 0u;
+            // fit before the end; while it does not fit, or every slot is taken,
+            // free the oldest stage (wait for its MMAs)
+            constexpr uint32_t RB = (uint32_t)TL::RING_BYTES;
             while (true) {
-              bool clash = fills - tail >= TL::SLOTS;
-              for (long i = tail; !clash && i < fills; ++i) {
-                const int sl = (int)(i % TL::SLOTS);
-                const uint32_t o = ctrl->slot_off[sl], l = ctrl->slot_len[sl];
-                clash = pos < o + l && o < pos + bytes;
+              bool placed = false;
+              if (nfl == 0) {
+                pos = head + bytes <= RB ? head : 0u;
+                placed = true;
+              } else if (nfl < TL::SLOTS) {
+                if (toff < head) {  // in use: [toff, head)
+                  if (head + bytes <= RB) {
+                    pos = head;
+                    placed = true;
+                  } else if (bytes <= toff) {
+                    pos = 0;
+                    placed = true;
+                  }
+                } else if (head + bytes <= toff) {  // in use: [toff, end) and [0, head)
+                  pos = head;
+                  placed = true;
+                }
               }
-              if (!clash) break;
-              if (!wait_bounded(smem_u32(&ctrl->empty[tail % TL::SLOTS]),
-                                (uint32_t)((tail / TL::SLOTS) & 1), abort_flag, err,
+              if (placed) break;
+              if (!wait_bounded(smem_u32(&ctrl->empty[tslot]), tpar, abort_flag, err,
                                 a.wait_limit_ns)) {
                 got = 0;
                 break;
               }
-              ++tail;
+              if (++tslot == TL::SLOTS) {
+                tslot = 0;
+                tpar ^= 1;
+              }
+              if (--nfl > 0) toff = ctrl->slot_off[tslot];
             }
             if (got) {
               ctrl->slot_off[stage] = pos;
-              ctrl->slot_len[stage] = bytes;
+              if (nfl++ == 0) toff = pos;
               head = pos + bytes;
             }
           } else {

@@ -312,14 +312,14 @@ __global__ void gather_rows_kernel(const uint4* __restrict__ x, int vpr,
 }
 
 // out[t] = sum_j w[t,j] * y_perm[slot_row[t*k+j]] (+ shared[t]); 8 elements per thread-step.
-// The slots are taken four at a time: their rows and weights first, then all
-// eight 16-byte row loads, then the fused multiply-adds in slot order (the
+// The slots are taken eight at a time: their rows and weights first, then all
+// sixteen 16-byte row loads, then the fused multiply-adds in slot order (the
 // same order, and so the same rounding, as one slot after another).
 __global__ void combine_kernel(const float4* __restrict__ y_perm, int T, int vpr, int k,
                                const int32_t* __restrict__ slot_row, const float* __restrict__ w,
                                const float4* __restrict__ shared, void* __restrict__ out,
                                int out_fp32, int* __restrict__ err) {
-  constexpr int KB = 4;
+  constexpr int KB = 8;
   const int nrows = T * k;
   const size_t total = (size_t)T * vpr;
   for (size_t i = blockIdx.x * (size_t)blockDim.x + threadIdx.x; i < total;

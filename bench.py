@@ -79,6 +79,9 @@ def parse():
                         "line with the HBM GB/s of the permutation, dispatch and combine kernels")
     p.add_argument("--sweep-t", default=None,
                    help="comma-separated token counts of the sweep (default: 1024,4096,16384,65536)")
+    p.add_argument("--unit-trace", action="store_true",
+                   help="after the timed run, one more forward with GEMM1's per-unit trace "
+                        "(moe_exec.unit_trace); adds a gemm1_units summary to the JSON line")
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--cpu-tokens", type=int, default=None,
                    help="oracle sample size (tokens); default 128, or 8 with --precision "
@@ -337,6 +340,39 @@ def kernel_roofline(bytes_, flops, t_s, hbm_gbs, tf_sust, tf_burst, src, dtype):
     r.update({"t_bytes_ms": round(t_b * 1e3, 4), "t_flops_ms": round(t_f * 1e3, 4),
               "t_measured_ms": round(t_s * 1e3, 4), "hbm": hbm_side, "tensor": tensor_side})
     return r
+
+
+def unit_trace_summary(rec, H, fp8=0):
+    """Summary of GEMM1's per-unit trace records [n, 5] (int64): per token-row bin
+    of the routed units (and the shared expert's), the units' count and median
+    times: wait = handed out -> first stage ready, mma = first stage ready ->
+    accumulator complete, epilogue = accumulator complete -> stored; and the
+    unit's tensor rate while its MMAs ran (2 * 2 * 128 * m * H flops)."""
+    rec = np.asarray(rec, dtype=np.int64)
+    rec = rec[(rec[:, 3] > 0) & (rec[:, 1] > 0)]
+    if len(rec) == 0:
+        return None
+    t = (rec[:, :4] - rec[:, 0].min()) / 1e3  # us
+    meta = rec[:, 4]
+    m = (meta >> 16) & 0xFFFF
+    grp = ((meta >> 32) & 0xFFFF) >= 1024
+    wait, mma, epi = t[:, 1] - t[:, 0], t[:, 2] - t[:, 1], t[:, 3] - t[:, 2]
+    tfs = 2 * 2 * 128 * m * H / np.maximum(mma, 1e-3) / 1e6   # TFLOP/s per SM
+    out = {"units": int(len(rec)), "span_us": round(float(t[:, 3].max()), 1),
+           "sms": int(len(np.unique(meta & 0xFFFF)))}
+    bins = {}
+    for lo, hi in ((0, 32), (32, 64), (64, 128), (128, 192), (192, 256)):
+        sel = (m > lo) & (m <= hi) & ~grp
+        if sel.any():
+            bins[f"routed m {lo + 1}-{hi}"] = sel
+    if grp.any():
+        bins["shared"] = grp
+    for name, sel in bins.items():
+        out[name] = {"n": int(sel.sum()), "wait_us": round(float(np.median(wait[sel])), 2),
+                     "mma_us": round(float(np.median(mma[sel])), 2),
+                     "epilogue_us": round(float(np.median(epi[sel])), 2),
+                     "TFLOPs_per_SM": round(float(np.median(tfs[sel])), 3)}
+    return out
 
 
 # ---------------------------------------------------------------- CPU oracle leg
@@ -864,6 +900,12 @@ def run_ours(args, wl, rank, world, local, device):
         "frac_nominal_peaks": round(max(B / (NOMINAL_HBM_GBS * 1e9),
                                         F / (pk * NOMINAL_BF16_TFLOPS * 1e12)) / t_step, 4),
         "bound": "hbm" if tb >= tfs else "tensor"}
+    if args.unit_trace and not ex.overlap:
+        rt = torch.zeros((1 << 16, L.UNIT_TRACE_FIELDS), dtype=torch.int64, device=device)
+        L.moe_layer_forward(cfg, L.exec_config(fuse_gather=fuse, fp8=fp8, fuse_combine=fc,
+                                               unit_trace=rt), W, d["x"], out, None, ws, stream)
+        torch.cuda.synchronize()
+        line["gemm1_units"] = unit_trace_summary(rt.cpu().numpy(), wl.H, fp8)
     if overlap:
         line["overlap"] = overlap
     if dispatch_fusion:

@@ -136,6 +136,9 @@ struct FfnGroup {
   int pack_src_rows;
   int* pack_next;
   int* pack_ready;
+  // Per-unit trace of the GEMM1 launch (moe_exec.unit_trace; null = off).
+  unsigned long long* trace;
+  int trace_cap;
 };
 
 // Routed group plus an optional dense group (the shared expert, same I) in one

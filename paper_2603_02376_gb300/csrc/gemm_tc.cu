@@ -152,6 +152,7 @@ struct Tile {
 };
 
 constexpr int UNIT_RING = 8;  // units announced ahead by the producer (a power of two)
+constexpr int TRACE_FIELDS = 5;  // per-unit trace record (GemmArgs::trace)
 
 struct Ctrl {
   uint64_t full[12];
@@ -436,6 +437,13 @@ struct GemmArgs {
   int pack_src_rows;
   int* pack_next;
   int* pack_ready;
+  // Per-unit trace (GEMM1 only; null = off): record u < trace_cap of
+  // TRACE_FIELDS uint64: the unit's announcement by the producer, its first
+  // stage ready at the MMA thread, its accumulator complete and its epilogue
+  // done (warp 2), all %globaltimer ns, then SM id | m << 16 |
+  // (expert + 1024 * group) << 32 | feature block << 48.
+  unsigned long long* trace;
+  int trace_cap;
   uint64_t wait_limit_ns;  // limit of each barrier wait
   long stall_fill;         // testing: CTA 0 never issues this fill (-1 = none), so the
                            // MMA's wait on it runs out and the abort path is exercised
@@ -527,6 +535,18 @@ __device__ __forceinline__ int ld_acquire(const int* p) {
 
 __device__ __forceinline__ void fence_proxy_async_global() {
   asm volatile("fence.proxy.async.global;" ::: "memory");
+}
+
+__device__ __forceinline__ uint32_t sm_id() {
+  uint32_t r;
+  asm volatile("mov.u32 %0, %%smid;" : "=r"(r));
+  return r;
+}
+
+// Field f of unit u's trace record (GemmArgs::trace), if tracing and u < cap.
+__device__ __forceinline__ void trace_put(const GemmArgs& a, int u, int f,
+                                          unsigned long long v) {
+  if (a.trace && u < a.trace_cap) a.trace[(size_t)u * TRACE_FIELDS + f] = v;
 }
 
 template <int MODE, int NMAX, int Q, bool PK>
@@ -676,6 +696,7 @@ __global__ void __launch_bounds__(threads_of(MODE, Q), 1)
                   : 0;
         if (pub) {
           reinterpret_cast<volatile int*>(ctrl->unit_ring)[r] = u;
+          if (u < total_units) trace_put(a, u, 0, global_timer_ns());
           mbar_arrive(smem_u32(&ctrl->unit_full[r]));
           if (u < total_units) u_next = a.sched ? atomicAdd(a.sched, 1) : u + (int)gridDim.x;
         }
@@ -884,6 +905,7 @@ __global__ void __launch_bounds__(threads_of(MODE, Q), 1)
             break;
           }
           tc_fence_after();
+          if (kb == U.kb0) trace_put(a, u, 1, global_timer_ns());
           const uint32_t sa =
               smem_u32(smem + (TL::VAR ? ctrl->slot_off[stage] : stage * TL::STAGE_BYTES));
           const uint32_t sb = sa + TL::NA * TL::A_BYTES;
@@ -1141,6 +1163,7 @@ __global__ void __launch_bounds__(threads_of(MODE, Q), 1)
       const uint32_t acc_par = (uint32_t)((j / TL::ACC_STAGES) & 1);
       if (!wait_bounded(smem_u32(&ctrl->acc_full[as]), acc_par, abort_flag, err, a.wait_limit_ns))
         break;
+      if (warp == 2 && lane == 0) trace_put(a, u, 2, global_timer_ns());
       tc_fence_after();
       const uint32_t tq = tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(as * TL::ACC_COLS);
       const int f = U.fb * TL::FEAT + q * 32 + lane;
@@ -1256,6 +1279,13 @@ __global__ void __launch_bounds__(threads_of(MODE, Q), 1)
       }
       tc_fence_before();
       __syncwarp();
+      if (warp == 2 && lane == 0) {
+        trace_put(a, u, 3, global_timer_ns());
+        trace_put(a, u, 4,
+                  (unsigned long long)sm_id() | ((unsigned long long)U.m << 16) |
+                      ((unsigned long long)(U.e + 1024 * U.grp) << 32) |
+                      ((unsigned long long)U.fb << 48));
+      }
       if (lane == 0) mbar_arrive(smem_u32(&ctrl->acc_empty[as]));
     }
   }
@@ -1446,6 +1476,8 @@ moe_status run_ffn(const FfnGroup& g0, const FfnGroup* g1, int H, int I, cudaStr
     args.pack_next = g0.pack_next;
     args.pack_ready = g0.pack_ready;
   }
+  args.trace = g0.trace;
+  args.trace_cap = g0.trace ? g0.trace_cap : 0;
   moe_status st =
       launch_gemm<MODE_SWIGLU, NMAX, Q, PK>(a1, b1, sa1, sb1, b1big, sb1big, args, s);
   if (st != MOE_OK) return st;
@@ -1461,6 +1493,7 @@ moe_status run_ffn(const FfnGroup& g0, const FfnGroup* g1, int H, int I, cudaStr
   args.gather0 = nullptr;  // GEMM2 reads h, already in packed row order
   args.pack_src = nullptr;
   args.pack_dst = nullptr;
+  args.trace = nullptr;
   args.a0_packed = pk ? static_cast<const uint16_t*>(g0.W2) : nullptr;
   args.a1_packed = (pk && g1) ? static_cast<const uint16_t*>(g1->W2) : nullptr;
   if (F8 && !MX) {

@@ -91,6 +91,7 @@ bool valid_exec(const moe_exec* ex, const moe_config* c) {
   if (ex->fuse_gather < 0 || ex->fuse_gather > 2) return false;
   if (ex->fp8 < 0 || ex->fp8 > 2) return false;
   if (ex->fuse_combine != 0 && ex->fuse_combine != 1) return false;
+  if (ex->unit_trace_cap < 0 || (ex->unit_trace && ex->unit_trace_cap == 0)) return false;
   if (ex->overlap) {
     if (ex->chunk_axis == 0) {
       if (ex->chunk_tokens < 1) return false;
@@ -443,9 +444,14 @@ FfnGroup dense_group(const moe_config& c, const Layout& L, const moe_weights& w,
 
 moe_status experts_tokens(const moe_config& c, const Layout& L, const moe_weights& w,
                           const uint16_t* x, int t0, int Tc, int ci, int e0, int e1,
-                          cudaStream_t s, cudaEvent_t* ev = nullptr) {
+                          cudaStream_t s, cudaEvent_t* ev = nullptr,
+                          const moe_exec* ex = nullptr) {
   MOE_TRY(injected_failure());
-  const FfnGroup g = routed_group(c, L, w, x, t0, Tc, ci, e0, e1);
+  FfnGroup g = routed_group(c, L, w, x, t0, Tc, ci, e0, e1);
+  if (ex && ex->unit_trace) {
+    g.trace = ex->unit_trace;
+    g.trace_cap = ex->unit_trace_cap;
+  }
   const long hint = (long)g.rows * (e1 - e0) / c.E;
   MOE_TRY(launch_expert_ffn_groups(g, nullptr, c.H, c.I, (int)hint, s,
                                    ev ? ev[MOE_EV_GEMM1] : nullptr));
@@ -469,9 +475,14 @@ moe_status shared_expert(const moe_config& c, const Layout& L, const moe_weights
 // (the shared expert's units share the persistent grid with the routed ones).
 // Requires I_shared == I; the stage events then mark the fused GEMMs.
 moe_status experts_and_shared(const moe_config& c, const Layout& L, const moe_weights& w,
-                              const uint16_t* x, cudaStream_t s, cudaEvent_t* ev) {
+                              const uint16_t* x, cudaStream_t s, cudaEvent_t* ev,
+                              const moe_exec* ex = nullptr) {
   MOE_TRY(launch_fill_range(L.sh_off, c.T, s));
-  const FfnGroup routed = routed_group(c, L, w, x, 0, c.T, 0, 0, c.E);
+  FfnGroup routed = routed_group(c, L, w, x, 0, c.T, 0, 0, c.E);
+  if (ex && ex->unit_trace) {
+    routed.trace = ex->unit_trace;
+    routed.trace_cap = ex->unit_trace_cap;
+  }
   const FfnGroup dense = dense_group(c, L, w, x);
   MOE_TRY(launch_expert_ffn_groups(routed, &dense, c.H, c.I, routed.rows, s,
                                    ev ? ev[MOE_EV_GEMM1] : nullptr));
@@ -827,9 +838,9 @@ moe_status moe_layer_forward(const moe_config* cfg, const moe_exec* ex, const mo
     MOE_TRY(pack_tokens(c, L, *w, x, 0, c.T, 0, L.x_perm != nullptr && !L.pack_in_gemm, s, ev,
                         true));
     if (c.I_shared == c.I) {
-      MOE_TRY(experts_and_shared(c, L, *w, x, s, ev));
+      MOE_TRY(experts_and_shared(c, L, *w, x, s, ev, ex));
     } else {
-      MOE_TRY(experts_tokens(c, L, *w, x, 0, c.T, 0, 0, c.E, s, ev));
+      MOE_TRY(experts_tokens(c, L, *w, x, 0, c.T, 0, 0, c.E, s, ev, ex));
       MOE_TRY(shared_expert(c, L, *w, x, s, ev));
     }
     if (L.fuse_combine)

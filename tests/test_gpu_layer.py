@@ -182,6 +182,28 @@ def test_layer_small_grouped_full(I_shared, T):
     check_permutation(wl, d, gidx)
 
 
+def test_unit_trace_records_every_gemm1_unit():
+    """moe_exec.unit_trace: one record per GEMM1 work unit, times in order, the
+    token rows of the routed records summing to T*k (one feature block: I = 128)."""
+    wl = I.Workload("small", T=100, H=256, E=16, k=4, I=128, I_shared=128, n_groups=4,
+                    topk_groups=2, gate=I.GATE_SIGMOID, normalize=1, route_scale=2.5)
+    d = I.layer_inputs(wl, seed=5, device=DEV)
+    rt = torch.zeros((256, L.UNIT_TRACE_FIELDS), dtype=torch.int64, device=DEV)
+    out, a = run_layer(wl, d, L.exec_config(out_fp32=1, unit_trace=rt))
+    rec = rt.cpu().numpy()
+    used = rec[:, 3] != 0
+    meta = rec[used, 4]
+    m, e = (meta >> 16) & 0xFFFF, (meta >> 32) & 0xFFFF
+    routed = e < 1024
+    counts = a["counts"].cpu().numpy()
+    assert used.sum() == (counts > 0).sum() + 1          # one tile per expert, one shared
+    assert m[routed].sum() == wl.T * wl.k and m[~routed].sum() == wl.T
+    np.testing.assert_array_equal(np.sort(m[routed]), np.sort(counts[counts > 0]))
+    t = rec[used, :4]
+    assert (np.diff(t, axis=1) >= 0).all()
+    assert not rec[~used].any()                         # nothing written past the units
+
+
 # ---------------------------------------------------------------- decode: every token
 
 @pytest.mark.parametrize("ex", [dict(out_fp32=1), dict(out_fp32=0), dict(out_fp32=1, fuse_gather=0),

@@ -38,7 +38,7 @@
 //   warp 10    block-scaled FP8 only: the stage's UE8M0 exponents as scale
 //              images in shared memory, which the MMA thread copies to TMEM
 //              (tcgen05.cp) ahead of block_scale MMAs;
-//   warps 10-13 GEMM1 with bf16 or row-scaled e4m3 operands: the dispatch
+//   warps 10-17 GEMM1 with bf16 or row-scaled e4m3 operands: the dispatch
 //              fused into the launch (GemmArgs::pack_dst). They copy the
 //              token rows into the packed order, a chunk of rows at a time
 //              taken from a global counter in row (= expert) order, and count
@@ -77,7 +77,7 @@ constexpr int B_BOX = 16;         // token rows per TMA box (tile remainders)
 constexpr int B_BIG = 64;         // token rows per TMA box (bulk of tiles of >= 64 rows)
 constexpr int NUM_THREADS = 320;  // 10 warps: producer, MMA, 8 epilogue
 constexpr int NUM_WARPS_MX = 11;  // block-scaled FP8: and a scale warp
-constexpr int PACK_WARPS = 4;     // GEMM1 (bf16, row-scaled e4m3): warps copying token rows
+constexpr int PACK_WARPS = 8;     // GEMM1 (bf16, row-scaled e4m3): warps copying token rows
 constexpr int PACK_ROWS = 4;      // token rows per chunk a pack warp takes
 constexpr uint64_t WAIT_LIMIT_NS = 2000000000ull;  // default limit of every barrier wait
 
@@ -157,9 +157,6 @@ constexpr int TRACE_FIELDS = 5;  // per-unit trace record (GemmArgs::trace)
 struct Ctrl {
   uint64_t full[12];
   uint64_t empty[12];
-  // byte ring (Tile::VAR): offset of the stage held by each slot, written by
-  // the producer before it arms the slot's full barrier
-  uint32_t slot_off[12];
   uint64_t acc_full[2];
   uint64_t acc_empty[2];
   uint64_t drain;
@@ -170,6 +167,49 @@ struct Ctrl {
   int unit_ring[UNIT_RING];
   uint32_t tmem_base;
   int abort_flag;
+};
+
+// Stage placement in the byte ring (Tile::VAR). Stages are placed in fill
+// order and freed in fill order: each goes at the head, or at the ring's start
+// when it does not fit before the end, after as many of the oldest stages as
+// needed are freed (or one, when every slot is taken). A stage's offset is
+// therefore a function of the sizes of the stages before it only, so the
+// producer and the MMA thread each run this allocator over the same sequence
+// of stage sizes and agree on every offset without exchanging them. The
+// offsets of the stages in flight live in registers (fixed-index shifts).
+template <int SLOTS_, int RING_>
+struct RingAlloc {
+  uint32_t off[SLOTS_];  // offsets of the stages in flight, oldest first
+  int nfl = 0;
+  uint32_t head = 0;
+  // Offset of the next stage of `bytes`; n_free = oldest stages freed first.
+  __device__ __forceinline__ uint32_t place(uint32_t bytes, int& n_free) {
+    n_free = 0;
+    while (true) {
+      if (nfl == 0) return push(head + bytes <= (uint32_t)RING_ ? head : 0u, bytes);
+      if (nfl < SLOTS_) {
+        const uint32_t toff = off[0];
+        if (toff < head) {  // in use: [toff, head)
+          if (head + bytes <= (uint32_t)RING_) return push(head, bytes);
+          if (bytes <= toff) return push(0u, bytes);
+        } else if (head + bytes <= toff) {  // in use: [toff, end) and [0, head)
+          return push(head, bytes);
+        }
+      }
+#pragma unroll
+      for (int i = 0; i + 1 < SLOTS_; ++i) off[i] = off[i + 1];
+      --nfl;
+      ++n_free;
+    }
+  }
+  __device__ __forceinline__ uint32_t push(uint32_t pos, uint32_t bytes) {
+#pragma unroll
+    for (int i = 0; i < SLOTS_; ++i)
+      if (i == nfl) off[i] = pos;
+    ++nfl;
+    head = pos + bytes;
+    return pos;
+  }
 };
 
 // ------------------------------------------------------------------ PTX wrappers
@@ -675,12 +715,11 @@ __global__ void __launch_bounds__(threads_of(MODE, Q), 1)
     int stage = 0;
     uint32_t phase = 0;
     long fills = 0;
-    // VAR ring (lane 0): stages are allocated and freed in fill order, so the
-    // bytes in use run from the oldest stage still in flight (slot tslot,
-    // offset toff, its barrier phase parity tpar) to head, wrapping once; nfl
-    // stages are in flight
-    int tslot = 0, nfl = 0;
-    uint32_t tpar = 0, toff = 0, head = 0;
+    // VAR ring (lane 0): the allocator, and the slot and barrier phase parity
+    // of the oldest stage still in flight
+    RingAlloc<TL::SLOTS, TL::RING_BYTES> ring;
+    int tslot = 0;
+    uint32_t tpar = 0;
     bool ok = true;
     // lane 0 takes the next unit one unit ahead, so the atomic's round trip
     // overlaps the current unit's loads
@@ -787,45 +826,17 @@ __global__ void __launch_bounds__(threads_of(MODE, Q), 1)
         int got = 1;
         if (lane == 0) {
           if constexpr (TL::VAR) {
-            // place the stage at the head, or at the ring's start when it does not
-            // fit before the end; while it does not fit, or every slot is taken,
-            // free the oldest stage (wait for its MMAs)
-            constexpr uint32_t RB = (uint32_t)TL::RING_BYTES;
-            while (true) {
-              bool placed = false;
-              if (nfl == 0) {
-                pos = head + bytes <= RB ? head : 0u;
-                placed = true;
-              } else if (nfl < TL::SLOTS) {
-                if (toff < head) {  // in use: [toff, head)
-                  if (head + bytes <= RB) {
-                    pos = head;
-                    placed = true;
-                  } else if (bytes <= toff) {
-                    pos = 0;
-                    placed = true;
-                  }
-                } else if (head + bytes <= toff) {  // in use: [toff, end) and [0, head)
-                  pos = head;
-                  placed = true;
-                }
-              }
-              if (placed) break;
+            // the stage's place; the stages it displaces must have been consumed
+            int n_free;
+            pos = ring.place(bytes, n_free);
+            for (int i = 0; i < n_free && got; ++i) {
               if (!wait_bounded(smem_u32(&ctrl->empty[tslot]), tpar, abort_flag, err,
-                                a.wait_limit_ns)) {
+                                a.wait_limit_ns))
                 got = 0;
-                break;
-              }
               if (++tslot == TL::SLOTS) {
                 tslot = 0;
                 tpar ^= 1;
               }
-              if (--nfl > 0) toff = ctrl->slot_off[tslot];
-            }
-            if (got) {
-              ctrl->slot_off[stage] = pos;
-              if (nfl++ == 0) toff = pos;
-              head = pos + bytes;
             }
           } else {
             got = wait_bounded(smem_u32(&ctrl->empty[stage]), phase ^ 1, abort_flag, err,
@@ -879,6 +890,7 @@ __global__ void __launch_bounds__(threads_of(MODE, Q), 1)
       int stage = 0;
       uint32_t phase = 0;
       bool ok = true, issued = false;
+      RingAlloc<TL::SLOTS, TL::RING_BYTES> ring;  // VAR: the producer's placements, replayed
       for (int j = 0; ok; ++j) {  // j: units of this CTA so far (accumulator j % ACC_STAGES)
         const int u = next_unit(j);
         if (u < 0) {
@@ -906,8 +918,12 @@ __global__ void __launch_bounds__(threads_of(MODE, Q), 1)
           }
           tc_fence_after();
           if (kb == U.kb0) trace_put(a, u, 1, global_timer_ns());
-          const uint32_t sa =
-              smem_u32(smem + (TL::VAR ? ctrl->slot_off[stage] : stage * TL::STAGE_BYTES));
+          uint32_t pos = (uint32_t)(stage * TL::STAGE_BYTES);
+          if constexpr (TL::VAR) {
+            int n_free;
+            pos = ring.place((uint32_t)(TL::NA * TL::A_BYTES + n_pad * BK * 2), n_free);
+          }
+          const uint32_t sa = smem_u32(smem + pos);
           const uint32_t sb = sa + TL::NA * TL::A_BYTES;
           if constexpr (MX) {
             // the stage's scale images -> its TMEM scale columns: A tile t at
@@ -1087,7 +1103,7 @@ __global__ void __launch_bounds__(threads_of(MODE, Q), 1)
     // ------------------------------------------------------------------ pack warps
     // Fused dispatch: packed row r of group 0 = source row pack_rst[r]. A warp
     // takes PACK_ROWS consecutive packed rows from the global counter, copies
-    // them with 16-byte vectors (each lane two columns of every row in flight
+    // them with 16-byte vectors (each lane four columns of every row in flight
     // at once), then adds the rows to their experts' counts with release
     // semantics. Rows with a source index outside the source matrix are left
     // unwritten and latched as MOE_ERR_DEVICE_CHECK; they are still counted.
@@ -1110,18 +1126,18 @@ __global__ void __launch_bounds__(threads_of(MODE, Q), 1)
         int tq[PACK_ROWS];
 #pragma unroll
         for (int q = 0; q < PACK_ROWS; ++q) tq[q] = __shfl_sync(0xffffffffu, src, q);
-        for (int v0 = lane; v0 < vpr; v0 += 64) {
-          uint4 val[PACK_ROWS][2];
+        for (int v0 = lane; v0 < vpr; v0 += 128) {
+          uint4 val[PACK_ROWS][4];
 #pragma unroll
           for (int q = 0; q < PACK_ROWS; ++q)
 #pragma unroll
-            for (int h = 0; h < 2; ++h)
+            for (int h = 0; h < 4; ++h)
               if (tq[q] >= 0 && v0 + 32 * h < vpr)
                 val[q][h] = a.pack_src[(size_t)tq[q] * vpr + v0 + 32 * h];
 #pragma unroll
           for (int q = 0; q < PACK_ROWS; ++q)
 #pragma unroll
-            for (int h = 0; h < 2; ++h)
+            for (int h = 0; h < 4; ++h)
               if (tq[q] >= 0 && v0 + 32 * h < vpr)
                 a.pack_dst[(size_t)(r0 + q) * vpr + v0 + 32 * h] = val[q][h];
         }

@@ -38,7 +38,7 @@
 //   warp 10    block-scaled FP8 only: the stage's UE8M0 exponents as scale
 //              images in shared memory, which the MMA thread copies to TMEM
 //              (tcgen05.cp) ahead of block_scale MMAs;
-//   warps 10-17 GEMM1 with bf16 or row-scaled e4m3 operands: the dispatch
+//   warps 10-13 GEMM1 with bf16 or row-scaled e4m3 operands: the dispatch
 //              fused into the launch (GemmArgs::pack_dst). They copy the
 //              token rows into the packed order, a chunk of rows at a time
 //              taken from a global counter in row (= expert) order, and count
@@ -77,7 +77,7 @@ constexpr int B_BOX = 16;         // token rows per TMA box (tile remainders)
 constexpr int B_BIG = 64;         // token rows per TMA box (bulk of tiles of >= 64 rows)
 constexpr int NUM_THREADS = 320;  // 10 warps: producer, MMA, 8 epilogue
 constexpr int NUM_WARPS_MX = 11;  // block-scaled FP8: and a scale warp
-constexpr int PACK_WARPS = 8;     // GEMM1 (bf16, row-scaled e4m3): warps copying token rows
+constexpr int PACK_WARPS = 4;     // GEMM1 (bf16, row-scaled e4m3): warps copying token rows
 constexpr int PACK_ROWS = 4;      // token rows per chunk a pack warp takes
 constexpr uint64_t WAIT_LIMIT_NS = 2000000000ull;  // default limit of every barrier wait
 
@@ -128,15 +128,6 @@ struct Tile {
   // (<= 8 KiB) and the 1 KiB alignment slack this stays under 227 KiB per CTA.
   static constexpr int STAGES_RAW = (217 * 1024 - SF_STG_BYTES) / STAGE_BYTES;
   static constexpr int STAGES = STAGES_RAW > 12 ? 12 : STAGES_RAW;
-  // Without block scales the stages are carved from one byte ring at the size
-  // each unit needs (its weight tiles plus its padded token rows): a unit with
-  // few token rows keeps more weight bytes in flight than a full-tile stage
-  // count would allow (a 16-row unit of the 256-row kernel: 6 stages, not 3).
-  // Up to SLOTS stages are in flight. Block-scaled FP8 keeps fixed stages
-  // (its scale images and TMEM scale columns are laid out per stage).
-  static constexpr bool VAR = !MX;
-  static constexpr int SLOTS = VAR ? 12 : STAGES;
-  static constexpr int RING_BYTES = VAR ? (217 * 1024) & ~1023 : STAGES * STAGE_BYTES;
   static constexpr int ACC_COLS = TWO_ACC ? 2 * NMAX : NMAX;  // one accumulator (gate | up)
   // MX: each stage's scales live in TMEM columns of their own (4 per image)
   // until the stage's MMAs complete
@@ -167,49 +158,6 @@ struct Ctrl {
   int unit_ring[UNIT_RING];
   uint32_t tmem_base;
   int abort_flag;
-};
-
-// Stage placement in the byte ring (Tile::VAR). Stages are placed in fill
-// order and freed in fill order: each goes at the head, or at the ring's start
-// when it does not fit before the end, after as many of the oldest stages as
-// needed are freed (or one, when every slot is taken). A stage's offset is
-// therefore a function of the sizes of the stages before it only, so the
-// producer and the MMA thread each run this allocator over the same sequence
-// of stage sizes and agree on every offset without exchanging them. The
-// offsets of the stages in flight live in registers (fixed-index shifts).
-template <int SLOTS_, int RING_>
-struct RingAlloc {
-  uint32_t off[SLOTS_];  // offsets of the stages in flight, oldest first
-  int nfl = 0;
-  uint32_t head = 0;
-  // Offset of the next stage of `bytes`; n_free = oldest stages freed first.
-  __device__ __forceinline__ uint32_t place(uint32_t bytes, int& n_free) {
-    n_free = 0;
-    while (true) {
-      if (nfl == 0) return push(head + bytes <= (uint32_t)RING_ ? head : 0u, bytes);
-      if (nfl < SLOTS_) {
-        const uint32_t toff = off[0];
-        if (toff < head) {  // in use: [toff, head)
-          if (head + bytes <= (uint32_t)RING_) return push(head, bytes);
-          if (bytes <= toff) return push(0u, bytes);
-        } else if (head + bytes <= toff) {  // in use: [toff, end) and [0, head)
-          return push(head, bytes);
-        }
-      }
-#pragma unroll
-      for (int i = 0; i + 1 < SLOTS_; ++i) off[i] = off[i + 1];
-      --nfl;
-      ++n_free;
-    }
-  }
-  __device__ __forceinline__ uint32_t push(uint32_t pos, uint32_t bytes) {
-#pragma unroll
-    for (int i = 0; i < SLOTS_; ++i)
-      if (i == nfl) off[i] = pos;
-    ++nfl;
-    head = pos + bytes;
-    return pos;
-  }
 };
 
 // ------------------------------------------------------------------ PTX wrappers
@@ -604,7 +552,7 @@ __global__ void __launch_bounds__(threads_of(MODE, Q), 1)
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~static_cast<uintptr_t>(1023));
-  uint8_t* sf_stg = smem + TL::RING_BYTES;  // MX staging (SF_STG_BYTES)
+  uint8_t* sf_stg = smem + TL::STAGES * TL::STAGE_BYTES;  // MX staging (SF_STG_BYTES)
   Ctrl* ctrl = reinterpret_cast<Ctrl*>(sf_stg + TL::SF_STG_BYTES);
   int* tile_off = reinterpret_cast<int*>(ctrl + 1);
   int* row_off = tile_off + a.n_exp + 1;
@@ -614,7 +562,7 @@ __global__ void __launch_bounds__(threads_of(MODE, Q), 1)
   const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
 
   if (threadIdx.x == 0) {
-    for (int s = 0; s < TL::SLOTS; ++s) {
+    for (int s = 0; s < TL::STAGES; ++s) {
       mbar_init(smem_u32(&ctrl->full[s]), MX ? 2 : 1);  // MX: the producer and the scale warp
       mbar_init(smem_u32(&ctrl->empty[s]), 1);
     }
@@ -715,11 +663,6 @@ __global__ void __launch_bounds__(threads_of(MODE, Q), 1)
     int stage = 0;
     uint32_t phase = 0;
     long fills = 0;
-    // VAR ring (lane 0): the allocator, and the slot and barrier phase parity
-    // of the oldest stage still in flight
-    RingAlloc<TL::SLOTS, TL::RING_BYTES> ring;
-    int tslot = 0;
-    uint32_t tpar = 0;
     bool ok = true;
     // lane 0 takes the next unit one unit ahead, so the atomic's round trip
     // overlaps the current unit's loads
@@ -801,10 +744,9 @@ __global__ void __launch_bounds__(threads_of(MODE, Q), 1)
         }
       for (int kb = U.kb0; kb < U.kb1; ++kb) {
         const uint32_t full = smem_u32(&ctrl->full[stage]);
-        uint32_t pos = 0;  // the stage's offset in the ring
+        const uint32_t sa = smem_u32(smem + stage * TL::STAGE_BYTES);
+        const uint32_t sb = sa + TL::NA * TL::A_BYTES;
         auto issue = [&]() {  // lane 0: arm the stage barrier, load the tiles
-          const uint32_t sa = smem_u32(smem + pos);
-          const uint32_t sb = sa + TL::NA * TL::A_BYTES;
           mbar_arrive_expect_tx(full, bytes);
 #pragma unroll
           for (int t = 0; t < TL::NA; ++t) {
@@ -825,26 +767,10 @@ __global__ void __launch_bounds__(threads_of(MODE, Q), 1)
         };
         int got = 1;
         if (lane == 0) {
-          if constexpr (TL::VAR) {
-            // the stage's place; the stages it displaces must have been consumed
-            int n_free;
-            pos = ring.place(bytes, n_free);
-            for (int i = 0; i < n_free && got; ++i) {
-              if (!wait_bounded(smem_u32(&ctrl->empty[tslot]), tpar, abort_flag, err,
-                                a.wait_limit_ns))
-                got = 0;
-              if (++tslot == TL::SLOTS) {
-                tslot = 0;
-                tpar ^= 1;
-              }
-            }
-          } else {
-            got = wait_bounded(smem_u32(&ctrl->empty[stage]), phase ^ 1, abort_flag, err,
-                               a.wait_limit_ns)
-                      ? 1
-                      : 0;
-            pos = (uint32_t)(stage * TL::STAGE_BYTES);
-          }
+          got = wait_bounded(smem_u32(&ctrl->empty[stage]), phase ^ 1, abort_flag, err,
+                             a.wait_limit_ns)
+                    ? 1
+                    : 0;
           if (got && blockIdx.x == 0 && fills == a.stall_fill) got = 2;  // skip this fill
           if (got == 1) issue();
         }
@@ -854,8 +780,6 @@ __global__ void __launch_bounds__(threads_of(MODE, Q), 1)
           break;
         }
         if (gather && got == 1) {
-          pos = __shfl_sync(0xffffffffu, pos, 0);
-          const uint32_t sb = smem_u32(smem + pos) + TL::NA * TL::A_BYTES;
 #pragma unroll
           for (int h = 0; h < 2; ++h) {
             const int g = lane + 32 * h;
@@ -865,7 +789,7 @@ __global__ void __launch_bounds__(threads_of(MODE, Q), 1)
           }
         }
         ++fills;
-        if (++stage == TL::SLOTS) {
+        if (++stage == TL::STAGES) {
           stage = 0;
           phase ^= 1;
         }
@@ -873,11 +797,11 @@ __global__ void __launch_bounds__(threads_of(MODE, Q), 1)
     }
     if (!ok && lane == 0) {
       // let the copies already issued land before the CTA can exit
-      for (int s = 0; s < TL::SLOTS; ++s) {
+      for (int s = 0; s < TL::STAGES; ++s) {
         if (fills <= s) continue;
-        const long f = s + ((fills - 1 - s) / TL::SLOTS) * TL::SLOTS;  // last fill of slot s
+        const long f = s + ((fills - 1 - s) / TL::STAGES) * TL::STAGES;  // last fill of stage s
         if (blockIdx.x == 0 && f == a.stall_fill) continue;  // never issued
-        const uint32_t par = (uint32_t)((f / TL::SLOTS) & 1);
+        const uint32_t par = (uint32_t)((f / TL::STAGES) & 1);
         const uint64_t t0 = global_timer_ns();
         while (!mbar_try_wait(smem_u32(&ctrl->full[s]), par) &&
                global_timer_ns() - t0 < a.wait_limit_ns) {
@@ -890,7 +814,6 @@ __global__ void __launch_bounds__(threads_of(MODE, Q), 1)
       int stage = 0;
       uint32_t phase = 0;
       bool ok = true, issued = false;
-      RingAlloc<TL::SLOTS, TL::RING_BYTES> ring;  // VAR: the producer's placements, replayed
       for (int j = 0; ok; ++j) {  // j: units of this CTA so far (accumulator j % ACC_STAGES)
         const int u = next_unit(j);
         if (u < 0) {
@@ -918,12 +841,7 @@ __global__ void __launch_bounds__(threads_of(MODE, Q), 1)
           }
           tc_fence_after();
           if (kb == U.kb0) trace_put(a, u, 1, global_timer_ns());
-          uint32_t pos = (uint32_t)(stage * TL::STAGE_BYTES);
-          if constexpr (TL::VAR) {
-            int n_free;
-            pos = ring.place((uint32_t)(TL::NA * TL::A_BYTES + n_pad * BK * 2), n_free);
-          }
-          const uint32_t sa = smem_u32(smem + pos);
+          const uint32_t sa = smem_u32(smem + stage * TL::STAGE_BYTES);
           const uint32_t sb = sa + TL::NA * TL::A_BYTES;
           if constexpr (MX) {
             // the stage's scale images -> its TMEM scale columns: A tile t at
@@ -962,7 +880,7 @@ __global__ void __launch_bounds__(threads_of(MODE, Q), 1)
           }
           issued = true;
           mma_commit(smem_u32(&ctrl->empty[stage]));
-          if (++stage == TL::SLOTS) {
+          if (++stage == TL::STAGES) {
             stage = 0;
             phase ^= 1;
           }
@@ -1103,7 +1021,7 @@ __global__ void __launch_bounds__(threads_of(MODE, Q), 1)
     // ------------------------------------------------------------------ pack warps
     // Fused dispatch: packed row r of group 0 = source row pack_rst[r]. A warp
     // takes PACK_ROWS consecutive packed rows from the global counter, copies
-    // them with 16-byte vectors (each lane four columns of every row in flight
+    // them with 16-byte vectors (each lane two columns of every row in flight
     // at once), then adds the rows to their experts' counts with release
     // semantics. Rows with a source index outside the source matrix are left
     // unwritten and latched as MOE_ERR_DEVICE_CHECK; they are still counted.
@@ -1126,18 +1044,18 @@ __global__ void __launch_bounds__(threads_of(MODE, Q), 1)
         int tq[PACK_ROWS];
 #pragma unroll
         for (int q = 0; q < PACK_ROWS; ++q) tq[q] = __shfl_sync(0xffffffffu, src, q);
-        for (int v0 = lane; v0 < vpr; v0 += 128) {
-          uint4 val[PACK_ROWS][4];
+        for (int v0 = lane; v0 < vpr; v0 += 64) {
+          uint4 val[PACK_ROWS][2];
 #pragma unroll
           for (int q = 0; q < PACK_ROWS; ++q)
 #pragma unroll
-            for (int h = 0; h < 4; ++h)
+            for (int h = 0; h < 2; ++h)
               if (tq[q] >= 0 && v0 + 32 * h < vpr)
                 val[q][h] = a.pack_src[(size_t)tq[q] * vpr + v0 + 32 * h];
 #pragma unroll
           for (int q = 0; q < PACK_ROWS; ++q)
 #pragma unroll
-            for (int h = 0; h < 4; ++h)
+            for (int h = 0; h < 2; ++h)
               if (tq[q] >= 0 && v0 + 32 * h < vpr)
                 a.pack_dst[(size_t)(r0 + q) * vpr + v0 + 32 * h] = val[q][h];
         }
@@ -1366,7 +1284,7 @@ long g_stall_fill = -1;
 template <int MODE, int NMAX, bool MX>
 size_t gemm_smem_bytes(int n_exp) {
   using TL = Tile<MODE, NMAX, MX>;
-  return 1024 + (size_t)TL::RING_BYTES + TL::SF_STG_BYTES + sizeof(Ctrl) +
+  return 1024 + (size_t)TL::STAGES * TL::STAGE_BYTES + TL::SF_STG_BYTES + sizeof(Ctrl) +
          2 * sizeof(int) * (n_exp + 1);
 }
 

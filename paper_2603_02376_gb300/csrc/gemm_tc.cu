@@ -356,6 +356,20 @@ __device__ __forceinline__ void tmem_ld16(uint32_t taddr, uint32_t (&r)[16]) {
       : "r"(taddr));
 }
 
+// SiLU(g) * u for the SwiGLU epilogue: g / (1 + e^-g) * u with e^-g = 2^(-g log2 e)
+// on the hardware exp2 and the quotient through the hardware reciprocal, both
+// flushing denormals (the forms without .ftz add fix-up instructions for
+// denormal inputs and results that this epilogue never needs: e^-g is
+// denormal only for g > 87, where 1 + e^-g = 1 either way). The result's error
+// is a few fp32 ulp, far below the bf16 rounding of h that follows.
+__device__ __forceinline__ float silu_mul(float g, float u) {
+  constexpr float kLog2e = 1.4426950408889634f;  // log2(e)
+  float e, r;
+  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(e) : "f"(-g * kLog2e));
+  asm("rcp.approx.ftz.f32 %0, %1;" : "=f"(r) : "f"(1.0f + e));
+  return g * r * u;
+}
+
 __device__ __forceinline__ void tmem_wait_ld() {
   asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
 }
@@ -1152,10 +1166,7 @@ __global__ void __launch_bounds__(threads_of(MODE, Q), 1)
               if (c0 + i < U.m) {
                 const float gv = __uint_as_float(g[i]) * (sa0 * sb);
                 const float uv = __uint_as_float(v[i]) * (sa1 * sb);
-                // silu(g) * u with the hardware exp2-based __expf and a fast
-                // division: their error (a few fp32 ulp) is far below the bf16
-                // rounding of h
-                const float hv = __fdividef(gv, 1.0f + __expf(-gv)) * uv;
+                const float hv = silu_mul(gv, uv);
                 static_cast<uint16_t*>(out)[o + (size_t)(c0 + i) * a.out_ld] =
                     float_to_bf16_bits(hv);
               }

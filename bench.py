@@ -826,7 +826,8 @@ def run_ours(args, wl, rank, world, local, device):
         overlap = {"ms_two_streams": round(t_ovl, 4), "ms_same_chunks_one_stream": round(t_single, 4),
                    "ms_pack_work": round(t_pack, 4),
                    "hidden_frac": round((t_single - t_ovl) / t_pack, 3) if t_pack > 0 else None,
-                   "ms_sequential_unchunked": round(sum(stage_ms.values()), 4)}
+                   "ms_sequential_unchunked": round(sum(stage_ms.values()), 4),
+                   "timeline": pipeline_timeline(L, cfg, ex, W, d["x"], out, ws, stream, wl, args)}
 
     hbm, tf_burst, tf_sust, src = peaks()
     b, f = algorithmic(wl, touched, fused, fp8, bool(fc), pack_in_gemm1=in_gemm1)
@@ -916,6 +917,32 @@ def run_ours(args, wl, rank, world, local, device):
                                             one_core_tokens=args.cpu_one_core_tokens)
     if rank == 0:
         print(json.dumps(line), flush=True)
+
+
+def pipeline_timeline(L, cfg, ex, W, x, out, ws, stream, wl, args):
+    """One pipelined forward with moe_exec.pipe_events: when each launch boundary
+    of both streams was reached, in ms after the first event (the order is the
+    one include/moe.h documents)."""
+    n = -(-wl.T // min(wl.T, args.chunk_tokens)) if ex.chunk_axis == 0 else args.expert_chunks
+    if ex.chunk_axis == 0:
+        labels = [f"pack: chunk {i} {w}" for i in range(n) for w in ("begins", "packed")]
+        comp = [f"compute: chunk {i} GEMMs {w}" for i in range(n) for w in ("begin", "end")]
+    else:
+        labels = ["pack: routing begins", "pack: routed"] + [f"pack: range {i} gathered"
+                                                             for i in range(n)]
+        comp = [f"compute: range {i} GEMMs {w}" for i in range(n) for w in ("begin", "end")]
+    labels += ["compute: shared expert begins", "compute: shared expert ends"] + comp
+    evs = [torch.cuda.Event(enable_timing=True) for _ in labels]
+    for e in evs:   # torch creates the CUDA event at its first record
+        e.record(stream)
+    torch.cuda.synchronize()
+    ext = L.exec_config(overlap=1, chunk_axis=ex.chunk_axis, chunk_tokens=ex.chunk_tokens,
+                        n_expert_chunks=ex.n_expert_chunks, fuse_gather=ex.fuse_gather,
+                        fp8=ex.fp8, fuse_combine=ex.fuse_combine, pipe_events=evs)
+    L.moe_layer_forward(cfg, ext, W, x, out, None, ws, stream)
+    torch.cuda.synchronize()
+    return sorted(((lab, round(evs[0].elapsed_time(e), 4)) for lab, e in zip(labels, evs)),
+                  key=lambda r: r[1])
 
 
 def run_stack(args, wl, rank, world, local, device, L, cfg, ex, W, d):

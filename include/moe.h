@@ -138,6 +138,17 @@ typedef struct {
    * units that did not run are left untouched. NULL = off. */
   unsigned long long* unit_trace;
   int32_t unit_trace_cap;
+  /* Optional timeline of a pipelined forward (overlap = 1; a profiling aid):
+   * n_pipe_events cudaEvent_t created by the caller with timing enabled,
+   * recorded at the launch boundaries of both streams in this order (n =
+   * number of token chunks or expert ranges): on the pack stream, before and
+   * after each chunk's routing + packing (token chunks: 2 per chunk), or
+   * before and after the routing, then after each range's gather (expert
+   * ranges: 2 + n); then on `stream`, before and after the shared expert, and
+   * before and after each chunk's or range's expert GEMMs (2 + 2 n). Events
+   * past n_pipe_events are not recorded. NULL = off; ignored when overlap = 0. */
+  void** pipe_events;
+  int32_t n_pipe_events;
 } moe_exec;
 
 /* Indices into moe_exec.stage_events: event i is recorded when stage i ends

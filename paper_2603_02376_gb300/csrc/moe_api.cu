@@ -92,6 +92,7 @@ bool valid_exec(const moe_exec* ex, const moe_config* c) {
   if (ex->fp8 < 0 || ex->fp8 > 2) return false;
   if (ex->fuse_combine != 0 && ex->fuse_combine != 1) return false;
   if (ex->unit_trace_cap < 0 || (ex->unit_trace && ex->unit_trace_cap == 0)) return false;
+  if (ex->n_pipe_events < 0 || (ex->pipe_events && ex->n_pipe_events == 0)) return false;
   if (ex->overlap) {
     if (ex->chunk_axis == 0) {
       if (ex->chunk_tokens < 1) return false;
@@ -858,6 +859,13 @@ moe_status moe_layer_forward(const moe_config* cfg, const moe_exec* ex, const mo
   cudaStream_t ps = aux_stream ? (cudaStream_t)aux_stream : pack_stream(dev);
   if (!ps) return MOE_ERR_CUDA;
   const int n_stage = ex->chunk_axis == 0 ? L.n_chunks : ex->n_expert_chunks;
+  // the caller's timeline events, recorded in the documented order
+  int n_tl = 0;
+  auto tl = [&](cudaStream_t st) -> moe_status {
+    if (!ex->pipe_events || n_tl >= ex->n_pipe_events) return MOE_OK;
+    cudaEvent_t e = static_cast<cudaEvent_t>(ex->pipe_events[n_tl++]);
+    return cudaEventRecord(e, st) == cudaSuccess ? MOE_OK : MOE_ERR_CUDA;
+  };
   std::vector<cudaEvent_t> ev;
   if (!events(dev, (size_t)n_stage + 2, &ev)) return MOE_ERR_CUDA;
   if (L.fp8) MOE_TRY(quantize_tokens(c, L, x, 0, c.T, s));  // before the fork: both streams read x_q
@@ -872,14 +880,20 @@ moe_status moe_layer_forward(const moe_config* cfg, const moe_exec* ex, const mo
     // chunk i's experts compute on `stream`.
     for (int ci = 0; ci < L.n_chunks; ++ci) {
       const int t0 = ci * L.chunk_T, Tc = c.T - t0 < L.chunk_T ? c.T - t0 : L.chunk_T;
+      MOE_TRY(tl(ps));
       MOE_TRY(pack_tokens(c, L, *w, x, t0, Tc, ci, L.x_perm != nullptr, ps));
+      MOE_TRY(tl(ps));
       MOE_CUDA(cudaEventRecord(ev[ci], ps));
     }
+    MOE_TRY(tl(s));
     MOE_TRY(shared_expert(c, L, *w, x, s));  // overlaps the first chunk's packing
+    MOE_TRY(tl(s));
     for (int ci = 0; ci < L.n_chunks; ++ci) {
       const int t0 = ci * L.chunk_T, Tc = c.T - t0 < L.chunk_T ? c.T - t0 : L.chunk_T;
       MOE_CUDA(cudaStreamWaitEvent(s, ev[ci], 0));
+      MOE_TRY(tl(s));
       MOE_TRY(experts_tokens(c, L, *w, x, t0, Tc, ci, 0, c.E, s));
+      MOE_TRY(tl(s));
       if (!L.fuse_combine) MOE_TRY(combine_tokens(c, L, t0, Tc, out, ex->out_fp32, s));
     }
     if (L.fuse_combine) MOE_TRY(finish_acc(c, L, out, ex->out_fp32, s));
@@ -889,7 +903,9 @@ moe_status moe_layer_forward(const moe_config* cfg, const moe_exec* ex, const mo
 
   // Expert ranges: route and permute all tokens once, then pack the rows of
   // expert range i+1 while range i computes; weights are streamed once.
+  MOE_TRY(tl(ps));
   MOE_TRY(pack_tokens(c, L, *w, x, 0, c.T, 0, false, ps));
+  MOE_TRY(tl(ps));
   const int nr = ex->n_expert_chunks;
   for (int r = 0; r < nr; ++r) {
     const int e0 = (int)((long)c.E * r / nr), e1 = (int)((long)c.E * (r + 1) / nr);
@@ -900,13 +916,18 @@ moe_status moe_layer_forward(const moe_config* cfg, const moe_exec* ex, const mo
     else if (L.x_perm)  // with a fused dispatch GEMM1 gathers the rows itself
       MOE_TRY(launch_gather_rows(c.H, x, L.rst, L.offsets, e0, e1,
                                  static_cast<uint16_t*>(L.x_perm), c.T * c.k, ps));
+    MOE_TRY(tl(ps));
     MOE_CUDA(cudaEventRecord(ev[r], ps));
   }
+  MOE_TRY(tl(s));
   MOE_TRY(shared_expert(c, L, *w, x, s));  // overlaps routing on the pack stream
+  MOE_TRY(tl(s));
   for (int r = 0; r < nr; ++r) {
     const int e0 = (int)((long)c.E * r / nr), e1 = (int)((long)c.E * (r + 1) / nr);
     MOE_CUDA(cudaStreamWaitEvent(s, ev[r], 0));
+    MOE_TRY(tl(s));
     MOE_TRY(experts_tokens(c, L, *w, x, 0, c.T, 0, e0, e1, s));
+    MOE_TRY(tl(s));
   }
   if (L.fuse_combine)
     MOE_TRY(finish_acc(c, L, out, ex->out_fp32, s));

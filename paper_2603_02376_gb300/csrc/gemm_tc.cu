@@ -30,11 +30,12 @@
 //   warp 1     MMA issuer (one thread): 4 x tcgen05.mma (K = 16 each) per stage,
 //              tcgen05.commit frees the stage, a final commit hands the
 //              accumulator to the epilogue; also owns the TMEM allocation;
-//   warps 2-9  epilogue, two warps per 32-lane TMEM quarter (alternate
-//              16-column chunks): tcgen05.ld the accumulator; GEMM1 applies
-//              SwiGLU and stores h in bf16 (the operand of GEMM2), GEMM2
-//              stores y in fp32 (summed by combine, or added into the output
-//              by the fused combine);
+//   warps 2-9  epilogue (warps 2-17 for GEMM2's two-tile units), two (four)
+//              warps per 32-lane TMEM quarter taking turns on 16-column
+//              chunks: tcgen05.ld the accumulator; GEMM1 applies SwiGLU and
+//              stores h in bf16 (the operand of GEMM2), GEMM2 stores y in fp32
+//              (summed by combine, or added into the output by the fused
+//              combine);
 //   warp 10    block-scaled FP8 only: the stage's UE8M0 exponents as scale
 //              images in shared memory, which the MMA thread copies to TMEM
 //              (tcgen05.cp) ahead of block_scale MMAs;
@@ -75,8 +76,8 @@ constexpr int BK = 64;            // bf16 per stage along K: one 128-byte swizzl
 constexpr int UMMA_K = 16;        // K of one tcgen05.mma kind::f16
 constexpr int B_BOX = 16;         // token rows per TMA box (tile remainders)
 constexpr int B_BIG = 64;         // token rows per TMA box (bulk of tiles of >= 64 rows)
-constexpr int NUM_THREADS = 320;  // 10 warps: producer, MMA, 8 epilogue
-constexpr int NUM_WARPS_MX = 11;  // block-scaled FP8: and a scale warp
+// Warps: 0 producer, 1 MMA issuer, then the epilogue warps (epi_warps of the
+// mode), then the block-scaled form's scale warp or GEMM1's pack warps.
 constexpr int PACK_WARPS = 4;     // GEMM1 (bf16, row-scaled e4m3): warps copying token rows
 constexpr int PACK_ROWS = 4;      // token rows per chunk a pack warp takes
 constexpr uint64_t WAIT_LIMIT_NS = 2000000000ull;  // default limit of every barrier wait
@@ -525,8 +526,17 @@ __device__ __forceinline__ Unit decode_unit(int u, const int* tile_off, const in
 // GEMM1 launches of the bf16 and row-scaled e4m3 forms carry the pack warps
 // (idle and gone at once when the dispatch is not fused).
 __host__ __device__ constexpr bool has_pack(int mode, int q) { return mode == MODE_SWIGLU && q != Q_BLOCK; }
+// Epilogue warps (a multiple of 4: each TMEM lane quarter gets the same
+// number): 16 for GEMM2's two-tile units, whose fp32 stores (256 features x
+// up to 256 tokens per unit) hold the single accumulator pair longest; 8
+// otherwise, and for the block-scaled form (its scale warp needs the
+// registers).
+__host__ __device__ constexpr int epi_warps(int mode, int q) {
+  return mode == MODE_PLAIN2 && q != Q_BLOCK ? 16 : 8;
+}
 __host__ __device__ constexpr int threads_of(int mode, int q) {
-  return q == Q_BLOCK ? NUM_WARPS_MX * 32 : NUM_THREADS + (has_pack(mode, q) ? PACK_WARPS * 32 : 0);
+  return 32 * (2 + epi_warps(mode, q) + (q == Q_BLOCK ? 1 : 0) +
+               (has_pack(mode, q) ? PACK_WARPS : 0));
 }
 
 __device__ __forceinline__ int ld_acquire(const int* p) {
@@ -563,6 +573,8 @@ __global__ void __launch_bounds__(threads_of(MODE, Q), 1)
   constexpr bool MX = Q == Q_BLOCK;  // ... with block scales applied by the MMA
   using TL = Tile<MODE, NMAX, MX>;
   constexpr bool SWIGLU = MODE == MODE_SWIGLU;
+  constexpr int EPI = epi_warps(MODE, Q);  // epilogue warps 2 .. EPI_END - 1
+  constexpr int EPI_END = 2 + EPI;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~static_cast<uintptr_t>(1023));
@@ -582,14 +594,14 @@ __global__ void __launch_bounds__(threads_of(MODE, Q), 1)
     }
     for (int s = 0; s < TL::ACC_STAGES; ++s) {
       mbar_init(smem_u32(&ctrl->acc_full[s]), 1);
-      mbar_init(smem_u32(&ctrl->acc_empty[s]), 8);  // one arrive per epilogue warp
+      mbar_init(smem_u32(&ctrl->acc_empty[s]), EPI);  // one arrive per epilogue warp
     }
     mbar_init(smem_u32(&ctrl->drain), 1);
-    // readers of each announced unit: the MMA thread, the 8 epilogue warps and
+    // readers of each announced unit: the MMA thread, the epilogue warps and
     // (block-scaled FP8) the scale warp
     for (int r = 0; r < UNIT_RING; ++r) {
       mbar_init(smem_u32(&ctrl->unit_full[r]), 1);
-      mbar_init(smem_u32(&ctrl->unit_empty[r]), MX ? 10 : 9);
+      mbar_init(smem_u32(&ctrl->unit_empty[r]), 1 + EPI + (MX ? 1 : 0));
     }
     ctrl->abort_flag = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
@@ -911,7 +923,7 @@ __global__ void __launch_bounds__(threads_of(MODE, Q), 1)
         }
       }
     }
-  } else if (MX && warp == NUM_WARPS_MX - 1) {
+  } else if (MX && warp == EPI_END) {
     // ------------------------------------------------------------------ scale warp
     // Block-scaled FP8 only. Per stage, once the slot is free: the UE8M0
     // exponents of the stage's A tiles and token rows, written as the 512-byte
@@ -1031,7 +1043,7 @@ __global__ void __launch_bounds__(threads_of(MODE, Q), 1)
         }
       }
     }
-  } else if (has_pack(MODE, Q) && warp >= 10) {
+  } else if (has_pack(MODE, Q) && warp >= EPI_END) {
     // ------------------------------------------------------------------ pack warps
     // Fused dispatch: packed row r of group 0 = source row pack_rst[r]. A warp
     // takes PACK_ROWS consecutive packed rows from the global counter, copies
@@ -1095,12 +1107,13 @@ __global__ void __launch_bounds__(threads_of(MODE, Q), 1)
         }
       }
     }
-  } else if (warp < 10) {
+  } else if (warp < EPI_END) {
     // ------------------------------------------------------------------ epilogue
-    // Two warps per TMEM lane quarter: warp w reads lanes 32 * (w % 4) .. + 31
-    // and the 16-column chunks c0 = 16 * half, 16 * half + 32, ... of a unit.
+    // EPI / 4 warps per TMEM lane quarter: warp w reads lanes 32 * (w % 4) ..
+    // + 31 and the 16-column chunks c0 = 16 * half, 16 * half + 16 * EPI / 4,
+    // ... of a unit.
     const int q = warp & 3;  // TMEM lane quarter this warp may access
-    const int half = (warp - 2) >> 2;
+    const int half = (warp - 2) >> 2;  // this warp's turn among its quarter's EPI / 4
     for (int j = 0;; ++j) {
       int u = 0;
       if (lane == 0) u = next_unit(j);
@@ -1143,7 +1156,7 @@ __global__ void __launch_bounds__(threads_of(MODE, Q), 1)
       // inside the column loop.
       auto columns = [&](auto cb_tag) {
         constexpr bool CB = decltype(cb_tag)::value;
-        for (int c0 = 16 * half; c0 < U.m; c0 += 32) {
+        for (int c0 = 16 * half; c0 < U.m; c0 += 16 * (EPI / 4)) {
           const int mc = c0 + (lane & 15);            // this lane's column of the chunk
           const bool cv = mc < U.m;
           const int br = U.row0 + (cv ? mc : 0);

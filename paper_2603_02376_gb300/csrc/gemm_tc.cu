@@ -30,12 +30,11 @@
 //   warp 1     MMA issuer (one thread): 4 x tcgen05.mma (K = 16 each) per stage,
 //              tcgen05.commit frees the stage, a final commit hands the
 //              accumulator to the epilogue; also owns the TMEM allocation;
-//   warps 2-9  epilogue (warps 2-17 for GEMM2's two-tile units), two (four)
-//              warps per 32-lane TMEM quarter taking turns on 16-column
-//              chunks: tcgen05.ld the accumulator; GEMM1 applies SwiGLU and
-//              stores h in bf16 (the operand of GEMM2), GEMM2 stores y in fp32
-//              (summed by combine, or added into the output by the fused
-//              combine);
+//   warps 2-9  epilogue, two warps per 32-lane TMEM quarter taking turns on
+//              16-column chunks: tcgen05.ld the accumulator; GEMM1 applies
+//              SwiGLU and stores h in bf16 (the operand of GEMM2), GEMM2 stores
+//              y in fp32 (summed by combine, or added into the output by the
+//              fused combine);
 //   warp 10    block-scaled FP8 only: the stage's UE8M0 exponents as scale
 //              images in shared memory, which the MMA thread copies to TMEM
 //              (tcgen05.cp) ahead of block_scale MMAs;
@@ -527,13 +526,10 @@ __device__ __forceinline__ Unit decode_unit(int u, const int* tile_off, const in
 // (idle and gone at once when the dispatch is not fused).
 __host__ __device__ constexpr bool has_pack(int mode, int q) { return mode == MODE_SWIGLU && q != Q_BLOCK; }
 // Epilogue warps (a multiple of 4: each TMEM lane quarter gets the same
-// number): 16 for GEMM2's two-tile units, whose fp32 stores (256 features x
-// up to 256 tokens per unit) hold the single accumulator pair longest; 8
-// otherwise, and for the block-scaled form (its scale warp needs the
-// registers).
-__host__ __device__ constexpr int epi_warps(int mode, int q) {
-  return mode == MODE_PLAIN2 && q != Q_BLOCK ? 16 : 8;
-}
+// number). Eight: sixteen for GEMM2's two-tile units measured the same (their
+// epilogue is bound by the SM's store bandwidth for the 256 KB of fp32 y of a
+// full unit, not by the warps issuing the stores).
+__host__ __device__ constexpr int epi_warps(int, int) { return 8; }
 __host__ __device__ constexpr int threads_of(int mode, int q) {
   return 32 * (2 + epi_warps(mode, q) + (q == Q_BLOCK ? 1 : 0) +
                (has_pack(mode, q) ? PACK_WARPS : 0));

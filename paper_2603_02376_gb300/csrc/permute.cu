@@ -412,24 +412,6 @@ int copy_grid(size_t work) {
   return (int)b;
 }
 
-// Grid of a grid-stride kernel of 256-thread blocks: one block per 256 work
-// items, at most as many as are resident at once (the kernel's occupancy per
-// SM x SMs), so the grid is one full wave rather than a full wave and a part
-// of another (the combine of a 1024-token batch: 917 K items, 4 blocks of
-// 256 threads resident per SM at its register count).
-template <class K>
-int wave_grid(K kernel, size_t work) {
-  int per_sm = 0;
-  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kernel, 256, 0) != cudaSuccess ||
-      per_sm < 1)
-    per_sm = 1;
-  size_t b = (work + 255) / 256;
-  const size_t cap = (size_t)num_sms() * per_sm;
-  if (b > cap) b = cap;
-  if (b < 1) b = 1;
-  return (int)b;
-}
-
 }  // namespace
 
 int perm_num_chunks(int T) { return (T + PERM_TOK - 1) / PERM_TOK; }
@@ -476,7 +458,7 @@ moe_status launch_dispatch_rows(int T, int H, int k, const uint16_t* x, const in
                                 uint16_t* x_perm, cudaStream_t s) {
   if (T == 0) return MOE_OK;
   const int vpr = H / 8;
-  dispatch_rows_kernel<<<wave_grid(dispatch_rows_kernel, (size_t)T * vpr), 256, 0, s>>>(
+  dispatch_rows_kernel<<<copy_grid((size_t)T * vpr), 256, 0, s>>>(
       reinterpret_cast<const uint4*>(x), T, vpr, k, slot_row, reinterpret_cast<uint4*>(x_perm));
   note_launch();
   return launch_status();
@@ -499,7 +481,7 @@ moe_status launch_combine(int T, int H, int k, const float* y_perm, const int32_
                           cudaStream_t s) {
   if (T == 0) return MOE_OK;
   const int vpr = H / 8;
-  combine_kernel<<<wave_grid(combine_kernel, (size_t)T * vpr), 256, 0, s>>>(
+  combine_kernel<<<copy_grid((size_t)T * vpr), 256, 0, s>>>(
       reinterpret_cast<const float4*>(y_perm), T, vpr, k, slot_row, w,
       reinterpret_cast<const float4*>(shared), out, out_fp32, device_error_word());
   note_launch();

@@ -1031,17 +1031,19 @@ def run_sweep(args, rank, world, local, device):
     sampler = ClockSampler(local)
 
     def timed(fn):
-        ms = 0.0
-        for i in range(args.warmup + args.steps):
+        # all launches enqueued ahead (one synchronisation at the end), so each
+        # timed kernel is already queued behind its L2 flush when its start
+        # event fires: the events bracket the kernel, not the host's launch
+        n = args.warmup + args.steps
+        ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+              for _ in range(n)]
+        for i in range(n):
             flush.fill_(i & 0xFF)
-            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-            e0.record(stream)
+            ev[i][0].record(stream)
             fn()
-            e1.record(stream)
-            torch.cuda.synchronize()
-            if i >= args.warmup:
-                ms += e0.elapsed_time(e1)
-        return ms / args.steps
+            ev[i][1].record(stream)
+        torch.cuda.synchronize()
+        return sum(ev[i][0].elapsed_time(ev[i][1]) for i in range(args.warmup, n)) / args.steps
 
     sweep_t = tuple(int(v) for v in args.sweep_t.split(",")) if args.sweep_t else \
         I.DISPATCH_SWEEP_T

@@ -297,7 +297,14 @@ def source_sha():
     return h.hexdigest()[:16]
 
 
-def measured_traffic(workload, fp8=0, kernel_bytes=None):
+def traffic_key(workload, fp8=0, pack_in_gemm1=False):
+    """Key of a GEMM1 traffic capture: the workload, the operand form, and whether
+    the launch also carried the dispatch copy (its pack warps' bytes)."""
+    return (workload + {0: "", 1: " fp8", 2: " fp8-block"}[int(fp8)]
+            + (" +dispatch in GEMM1" if pack_in_gemm1 else ""))
+
+
+def measured_traffic(workload, fp8=0, kernel_bytes=None, pack_in_gemm1=False):
     """ncu DRAM bytes per GEMM1 launch, if captured for the current kernel source.
 
     The bf16 entry holds the bytes of the full launch; the FP8 entry holds the
@@ -306,7 +313,7 @@ def measured_traffic(workload, fp8=0, kernel_bytes=None):
     try:
         with open(TRAFFIC_FILE) as f:
             t = json.load(f)
-        e = t.get(workload + {0: "", 1: " fp8", 2: " fp8-block"}[int(fp8)])
+        e = t.get(traffic_key(workload, fp8, pack_in_gemm1))
         if e and e.get("source_sha") == source_sha():
             if "dram_bytes_per_launch" in e:
                 return float(e["dram_bytes_per_launch"])
@@ -842,7 +849,7 @@ def run_ours(args, wl, rank, world, local, device):
     qh = (R * wl.I * 3 + scale_bytes(R, wl.I, fp8)
           + (wl.T * wl.I_shared * 3 + scale_bytes(wl.T, wl.I_shared, fp8)
              if wl.I_shared == wl.I else 0)) if fp8 else 0
-    traffic = measured_traffic(wl.name, fp8, b["gemm1"] - qh)
+    traffic = measured_traffic(wl.name, fp8, b["gemm1"] - qh, pack_in_gemm1=in_gemm1)
     pk = 2.0 if fp8 else 1.0   # e4m3 dense peak = the measured bf16 peak x the nominal 2x
     stages = {}
     for s_, t in stage_ms.items():

@@ -80,6 +80,7 @@ def test_traffic_capture_of_another_source_is_not_used(tmp_path, monkeypatch):
     f.write_text(json.dumps({key: {"source_sha": bench.source_sha(), "dram_bytes_per_launch": 123}}))
     assert bench.measured_traffic(key, 0) == 123.0
     assert bench.measured_traffic(key, 2) is None          # no block-scaled entry
+    assert bench.measured_traffic(key, 0, pack_in_gemm1=True) is None   # another launch form
 
 
 def test_block_scaled_weight_generator():

@@ -173,6 +173,25 @@ def test_fused_combine_workspace():
         assert f16 - f32 >= T * H * 4
 
 
+def test_exec_options_validated_on_the_host():
+    # dispatch forms 0, 1, 2 are accepted (same workspace for 0 and 2: x_perm is
+    # written either by the dispatch kernel or by GEMM1's pack warps); 3 is not;
+    # a trace buffer or timeline events need a positive count
+    c = L.config_of(I.PREFILL)
+    ws0 = L.moe_workspace_size(c, L.exec_config(fuse_gather=0))
+    assert ws0 > 0 and L.moe_workspace_size(c, L.exec_config(fuse_gather=2)) == ws0
+    assert L.moe_workspace_size(c, L.exec_config(fuse_gather=3)) == 0
+    ex = L.exec_config()
+    ex.unit_trace, ex.unit_trace_cap = 0x1000, 0
+    assert L.moe_workspace_size(c, ex) == 0
+    ex = L.exec_config()
+    ex.unit_trace_cap = -1
+    assert L.moe_workspace_size(c, ex) == 0
+    ex = L.exec_config(overlap=1)
+    ex.n_pipe_events = -1
+    assert L.moe_workspace_size(c, ex) == 0
+
+
 def test_fp8_entry_points_reject_bad_arguments_without_a_gpu(lib):
     c = L.config(**GOOD)
     z = ctypes.c_void_p(0)

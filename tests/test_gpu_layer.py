@@ -204,6 +204,36 @@ def test_unit_trace_records_every_gemm1_unit():
     assert not rec[~used].any()                         # nothing written past the units
 
 
+@pytest.mark.parametrize("axis,n", [(1, 3), (0, 37)])
+def test_pipeline_events_record_both_streams_in_order(axis, n):
+    """moe_exec.pipe_events: the documented number of events, each stream's in
+    order, the routed GEMMs after the shared expert and each after its chunk's
+    or range's packing; the output equals the forward without events."""
+    wl = I.Workload("small", T=100, H=256, E=16, k=4, I=128, I_shared=128, n_groups=4,
+                    topk_groups=2, gate=I.GATE_SIGMOID, normalize=1, route_scale=2.5)
+    d = I.layer_inputs(wl, seed=5, device=DEV)
+    kw = dict(out_fp32=1, overlap=1, chunk_axis=axis, fuse_gather=0)
+    kw.update(n_expert_chunks=n) if axis == 1 else kw.update(chunk_tokens=n)
+    chunks = n if axis == 1 else -(-wl.T // n)
+    n_pack = 2 * chunks if axis == 0 else 2 + chunks
+    evs = [torch.cuda.Event(enable_timing=True) for _ in range(n_pack + 2 + 2 * chunks)]
+    s = torch.cuda.current_stream()
+    for e in evs:
+        e.record(s)
+    torch.cuda.synchronize()
+    out, _ = run_layer(wl, d, L.exec_config(pipe_events=evs, **kw))
+    ref, _ = run_layer(wl, d, L.exec_config(**kw))
+    torch.cuda.synchronize()
+    assert torch.equal(out, ref)
+    t = [evs[0].elapsed_time(e) for e in evs]
+    pack, comp = t[:n_pack], t[n_pack:]
+    assert all(b >= a for a, b in zip(pack, pack[1:]))
+    assert all(b >= a for a, b in zip(comp, comp[1:]))
+    packed = pack[1::2] if axis == 0 else pack[2:]
+    for i in range(chunks):           # chunk / range i's GEMMs begin after its packing
+        assert comp[2 + 2 * i] >= packed[i]
+
+
 # ---------------------------------------------------------------- decode: every token
 
 @pytest.mark.parametrize("ex", [dict(out_fp32=1), dict(out_fp32=0), dict(out_fp32=1, fuse_gather=0),

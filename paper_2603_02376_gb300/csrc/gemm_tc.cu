@@ -1118,15 +1118,10 @@ __global__ void __launch_bounds__(threads_of(MODE, Q), 1)
       const Unit U = decode_unit<NMAX>(u, tile_off, row_off, a, units1, kblocks);
       const int as = j % TL::ACC_STAGES;
       const uint32_t acc_par = (uint32_t)((j / TL::ACC_STAGES) & 1);
-      if (!wait_bounded(smem_u32(&ctrl->acc_full[as]), acc_par, abort_flag, err, a.wait_limit_ns))
-        break;
-      if (warp == 2 && lane == 0) trace_put(a, u, 2, global_timer_ns());
-      tc_fence_after();
-      const uint32_t tq = tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(as * TL::ACC_COLS);
       const int f = U.fb * TL::FEAT + q * 32 + lane;
       const size_t o = (size_t)U.row0 * a.out_ld + f;
       // FP8: the scales of this thread's weight row(s); the token columns' scales
-      // are fetched per chunk below
+      // are fetched with the other per-column data below
       float sa0 = 1.f, sa1 = 1.f;
       const float* bsc = nullptr;
       const int32_t* bidx = nullptr;
@@ -1144,25 +1139,42 @@ __global__ void __launch_bounds__(threads_of(MODE, Q), 1)
       float* comb = U.grp ? a.comb_out1 : a.comb_out0;
       const int32_t* ctok = U.grp ? nullptr : a.comb_tok0;
       const float* cw = U.grp ? nullptr : a.comb_w0;
+      // What each column of the unit needs from global memory (the token's FP8
+      // scale; with the fused combine its token row and gate weight), loaded
+      // for all of this warp's 16-column chunks at once and before the
+      // accumulator is complete, so the loads overlap the unit's MMAs: lane
+      // l < 16 holds column 16 * half + 16 * (EPI / 4) * i + l of chunk i.
+      constexpr bool CBP = MODE == MODE_PLAIN || MODE == MODE_PLAIN2;  // combine possible
+      constexpr int CSTEP = 16 * (EPI / 4);
+      constexpr int NCH = (NMAX + CSTEP - 1) / CSTEP;  // chunks per warp, at most
+      float sbv[NCH], wvv[NCH];
+      int tvv[NCH];
+      const bool cbx = CBP && comb != nullptr;
+#pragma unroll
+      for (int i = 0; i < NCH; ++i) {
+        const int mc = 16 * half + CSTEP * i + (lane & 15);
+        const bool cv = mc < U.m;
+        const int br = U.row0 + (cv ? mc : 0);
+        sbv[i] = (RS && cv) ? bsc[bidx ? bidx[br] : br] : 1.f;
+        wvv[i] = (cbx && cv && cw) ? cw[br] : 1.f;
+        tvv[i] = (cbx && cv && ctok) ? ctok[br] : br;
+      }
+      if (!wait_bounded(smem_u32(&ctrl->acc_full[as]), acc_par, abort_flag, err, a.wait_limit_ns))
+        break;
+      if (warp == 2 && lane == 0) trace_put(a, u, 2, global_timer_ns());
+      tc_fence_after();
+      const uint32_t tq = tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(as * TL::ACC_COLS);
       // The unit's columns; CB (the fused combine) is a compile-time copy of the
-      // loop so the plain stores keep their unrolled form. Per 16-column chunk,
-      // lane l < 16 fetches what column c0 + l needs from global memory (the
-      // token's scale; with the combine its token row and gate weight) once,
-      // and the other lanes read it with a shuffle: no dependent global loads
-      // inside the column loop.
+      // loop so the plain stores keep their unrolled form. The other lanes read
+      // a chunk's per-column values from lanes 0-15 with a shuffle.
       auto columns = [&](auto cb_tag) {
         constexpr bool CB = decltype(cb_tag)::value;
-        for (int c0 = 16 * half; c0 < U.m; c0 += 16 * (EPI / 4)) {
-          const int mc = c0 + (lane & 15);            // this lane's column of the chunk
-          const bool cv = mc < U.m;
-          const int br = U.row0 + (cv ? mc : 0);
-          float sb_l = 1.f, w_l = 1.f;
-          int t_l = br;
-          if (RS && cv) sb_l = bsc[bidx ? bidx[br] : br];
-          if (CB && cv) {
-            if (cw) w_l = cw[br];
-            if (ctok) t_l = ctok[br];
-          }
+#pragma unroll
+        for (int ci = 0; ci < NCH; ++ci) {
+          const int c0 = 16 * half + CSTEP * ci;
+          if (c0 >= U.m) break;
+          const float sb_l = sbv[ci], w_l = wvv[ci];
+          const int t_l = tvv[ci];
           uint32_t g[16];
           tmem_ld16(tq + c0, g);
           if constexpr (SWIGLU) {

@@ -84,6 +84,8 @@ def align256(n):
     ([300, 256, 257, 0, 1, 16], 256, 256),              # multi-tile experts, tile edges
     ([4] * 60 + [0, 12, 31, 33], 512, 256),             # decode-like: small token tiles
     ([150, 100, 0, 145, 3], 512, 256),                  # 144-row tiles, experts over two tiles
+    ([128, 129, 127, 384, 0, 200], 256, 256),           # 127/128/129-row experts, 128-row tails
+    ([128, 129, 16, 144, 273, 0, 60], 384, 128),        # ... 144-row tiles, one GEMM2 tile
     ([130, 111], 7168, 2048),                           # the real layer shape
     ([1, 3, 0, 7], 7168, 2048),                         # decode: few rows per expert
 ])

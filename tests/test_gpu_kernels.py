@@ -246,6 +246,12 @@ def test_pack_weights_layout(rows, K):
     ([4] * 60 + [0, 12, 31, 33], 512, 256),             # decode-like: small token tiles
     ([0, 0, 0, 40], 384, 128),
     ([150, 100, 0, 145, 3], 512, 256),                  # 144-row tiles, experts over two tiles
+    # experts of 127/128/129 rows and multi-tile experts with 128-row tails, for
+    # 256- and 144-row tiles and one (H % 256 != 0) or two weight tiles per GEMM2 unit
+    ([128, 129, 127, 384, 0, 200], 256, 256),
+    ([128, 129, 16, 144, 273, 0, 60], 256, 256),
+    ([128, 129, 16, 144, 273, 0, 60], 384, 128),
+    ([300, 1, 128, 200], 384, 128),
     ([130, 111], 7168, 2048),                           # the real layer shape
     ([1] * 48 + [3, 7], 7168, 2048),                    # decode: few rows per expert
 ])

@@ -68,11 +68,46 @@ moe_status launch_permutation(const moe_config& c, const int32_t* idx, int32_t* 
                               int32_t* offsets, int32_t* row_src_token, int32_t* slot_row,
                               int32_t* chunk_counts, int32_t* chunk_base, cudaStream_t s,
                               const float* topk_w = nullptr, float* row_w = nullptr);
+// Tile-packed token rows: the layout in which the layer keeps the bf16
+// operands of its expert GEMMs (x_perm and h), so that a stage's token rows
+// are one contiguous bulk copy instead of a tensor-map load of n 128-byte row
+// segments (hot GEMM1 units measured 8 % faster with the packed form). The
+// packed rows of expert e (its global index), [off[e], off[e+1]), are cut into
+// tiles of `tile` rows, the expert GEMMs' token tile. Tile t of expert e
+// starts at padded row P = off[e] + 16 e + t * tile and holds n_pad = the
+// tile's rows rounded up to 16. Its columns come in blocks of 128 bytes:
+// block kb of the tile (n_pad rows x 128 bytes) is contiguous at byte
+// P * row_bytes + kb * n_pad * 128, its row i at i * 128, and the 16-byte
+// chunk j of that row at chunk j ^ (i % 8) (the 128-byte swizzle of a K-major
+// MMA operand). A buffer of `rows` packed rows holds rows + 16 E rows (each
+// expert's last tile pads at most 15). TiledRow locates packed row r of
+// expert e; chunk16 gives the 16-byte unit index of its chunk c.
+struct TiledRow {
+  size_t tile16;  // 16-byte index of the tile's first byte
+  int i;          // row within the tile
+  int n_pad;      // rows the tile stores
+  __host__ __device__ size_t chunk16(int c) const {
+    return tile16 + (size_t)(c >> 3) * n_pad * 8 + (size_t)i * 8 + ((c & 7) ^ (i & 7));
+  }
+};
+__host__ __device__ inline TiledRow tiled_row(int r, int e, int off_e, int cnt_e, int tile,
+                                              int chunks_per_row) {
+  const int l = r - off_e, t = l / tile;
+  const int m = cnt_e - t * tile < tile ? cnt_e - t * tile : tile;
+  TiledRow w;
+  w.i = l - t * tile;
+  w.n_pad = (m + 15) & ~15;
+  w.tile16 = (size_t)(off_e + 16 * e + t * tile) * chunks_per_row;
+  return w;
+}
+
 moe_status launch_dispatch_rows(int T, int H, int k, const uint16_t* x, const int32_t* slot_row,
                                 uint16_t* x_perm, cudaStream_t s);
+// x_perm[r] = x[row_src_token[r]] for the rows of experts [e_begin, e_end);
+// tile > 0 writes them in the tile-packed layout above (offsets global).
 moe_status launch_gather_rows(int H, const uint16_t* x, const int32_t* row_src_token,
                               const int32_t* offsets, int e_begin, int e_end, uint16_t* x_perm,
-                              int max_rows, cudaStream_t s);
+                              int max_rows, cudaStream_t s, int tile = 0);
 moe_status launch_combine(int T, int H, int k, const float* y_perm, const int32_t* slot_row,
                           const float* w, const float* shared, void* out, int out_fp32,
                           cudaStream_t s);
@@ -97,6 +132,12 @@ struct FfnGroup {
   const int32_t* gather;
   int x_rows;
   bool packed;  // W13 / W2 in the tile-packed layout (moe_pack_weights)
+  // bf16 token operands in the tile-packed row layout (TiledRow) with the
+  // launch's token tile: x (GEMM1's, when it is not gathered) and h (GEMM1's
+  // output, GEMM2's operand); both buffers then hold rows + 16 * n_experts rows.
+  bool x_tiled;
+  bool h_tiled;
+  int x_tile;  // the token tile x was written with (x_tiled)
   // FP8 (e4m3) form: per-row fp32 scales of x (indexed by token through
   // x_scale_idx when x holds packed copies, else by row), of W13 and W2 rows;
   // hq / hs receive GEMM2's quantized operand and its row scales.
@@ -140,6 +181,12 @@ struct FfnGroup {
   unsigned long long* trace;
   int trace_cap;
 };
+
+// The expert GEMMs' token tile for rows_hint packed rows over n_exp experts:
+// small tiles leave more of the stage ring to weights (decode ~4 rows per
+// expert -> 32; balanced prefill ~128 +- 10 % -> 144; larger or skewed loads
+// -> 256, or 224 with block-scaled FP8).
+int ffn_tile_rows(long rows_hint, int n_exp, bool fp8, bool fp8_block);
 
 // Routed group plus an optional dense group (the shared expert, same I) in one
 // pair of launches.

@@ -227,6 +227,16 @@ __device__ __forceinline__ void bulk_load_tile(uint32_t dst, const void* src, ui
       : "memory");
 }
 
+// `bytes` contiguous bytes (a multiple of 16, both addresses 16-byte aligned).
+__device__ __forceinline__ void bulk_load(uint32_t dst, const void* src, uint32_t bytes,
+                                          uint32_t bar) {
+  asm volatile(
+      "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::
+          "r"(dst),
+      "l"(reinterpret_cast<uint64_t>(src)), "r"(bytes), "r"(bar)
+      : "memory");
+}
+
 // Four rows (y0..y3) of a 2-D tensor whose map has a one-row box, landing as
 // four consecutive 128-byte rows of a swizzled tile (tile::gather4).
 __device__ __forceinline__ void tma_gather4(uint32_t dst, const CUtensorMap* map, int x, int y0,
@@ -439,6 +449,13 @@ struct GemmArgs {
   int pack_src_rows;
   int* pack_next;
   int* pack_ready;
+  // bf16 token operands in the tile-packed row layout (TiledRow, tile = NMAX):
+  // group g's token rows come from b_tiled_g by one bulk copy per stage (null:
+  // through the tensor maps), and GEMM1 writes group g's h to out_g in that
+  // layout when out_tiled_g. Padded rows: row0 + 16 * (global expert).
+  const uint8_t* b_tiled0;
+  const uint8_t* b_tiled1;
+  int out_tiled0, out_tiled1;
   // Per-unit trace (GEMM1 only; null = off): record u < trace_cap of
   // TRACE_FIELDS uint64: the unit's announcement by the producer, its first
   // stage ready at the MMA thread, its accumulator complete and its epilogue
@@ -780,7 +797,14 @@ __global__ void __launch_bounds__(threads_of(MODE, Q), 1)
             else
               tma_load_2d(sa + t * TL::A_BYTES, mA, kb * KE, r, full);
           }
-          if (!gather) {
+          const uint8_t* bt = U.grp ? a.b_tiled1 : a.b_tiled0;
+          if (bt) {  // tile-packed rows: block kb of the tile, already swizzled
+            const int eg = U.grp ? 0 : a.e_begin + U.e;
+            bulk_load(sb,
+                      bt + (size_t)(U.row0 + 16 * eg) * a.K * (F8 ? 1 : 2) +
+                          (size_t)kb * n_pad * 128,
+                      (uint32_t)n_pad * 128, full);
+          } else if (!gather) {
             for (int i = 0; i < n_big; ++i)
               tma_load_2d(sb + i * (B_BIG * BK * 2), mBbig, kb * KE, U.row0 + i * B_BIG, full);
             for (int i = n_big * (B_BIG / B_BOX); i < n_pad / B_BOX; ++i)
@@ -1066,6 +1090,33 @@ __global__ void __launch_bounds__(threads_of(MODE, Q), 1)
         int tq[PACK_ROWS];
 #pragma unroll
         for (int q = 0; q < PACK_ROWS; ++q) tq[q] = __shfl_sync(0xffffffffu, src, q);
+        // tile-packed destination: lane q < nr places row r0 + q (its expert by
+        // binary search over the clamped offsets), every lane gets the result
+        TiledRow dq[PACK_ROWS];
+        if (a.b_tiled0) {
+          unsigned long long tb = 0;
+          int ti = 0, tn = 0;
+          if (lane < nr) {
+            const int r = r0 + lane;
+            int lo = 0, hi = a.n_exp - 1;
+            while (lo < hi) {
+              const int mid = (lo + hi + 1) >> 1;
+              if (row_off[mid] <= r) lo = mid;
+              else hi = mid - 1;
+            }
+            const TiledRow w =
+                tiled_row(r, a.e_begin + lo, row_off[lo], row_off[lo + 1] - row_off[lo], NMAX, vpr);
+            tb = w.tile16;
+            ti = w.i;
+            tn = w.n_pad;
+          }
+#pragma unroll
+          for (int q = 0; q < PACK_ROWS; ++q) {
+            dq[q].tile16 = __shfl_sync(0xffffffffu, tb, q);
+            dq[q].i = __shfl_sync(0xffffffffu, ti, q);
+            dq[q].n_pad = __shfl_sync(0xffffffffu, tn, q);
+          }
+        }
         for (int v0 = lane; v0 < vpr; v0 += 64) {
           uint4 val[PACK_ROWS][2];
 #pragma unroll
@@ -1079,7 +1130,8 @@ __global__ void __launch_bounds__(threads_of(MODE, Q), 1)
 #pragma unroll
             for (int h = 0; h < 2; ++h)
               if (tq[q] >= 0 && v0 + 32 * h < vpr)
-                a.pack_dst[(size_t)(r0 + q) * vpr + v0 + 32 * h] = val[q][h];
+                a.pack_dst[a.b_tiled0 ? dq[q].chunk16(v0 + 32 * h)
+                                      : (size_t)(r0 + q) * vpr + v0 + 32 * h] = val[q][h];
         }
         __threadfence();
         fence_proxy_async_global();
@@ -1136,6 +1188,13 @@ __global__ void __launch_bounds__(threads_of(MODE, Q), 1)
       }
       void* out = U.grp ? static_cast<void*>(static_cast<float*>(a.out1) + U.split * a.split_stride)
                         : a.out0;
+      // SwiGLU with tile-packed h: this thread's element of block f / 64 of the
+      // unit's tile (the tile of n_pad rows at padded row row0 + 16 * expert)
+      const bool h_tiled = SWIGLU && (U.grp ? a.out_tiled1 : a.out_tiled0);
+      const int h_pad = (U.m + 15) & ~15;
+      const size_t h_blk = (size_t)(U.row0 + 16 * (U.grp ? 0 : a.e_begin + U.e)) * a.out_ld +
+                           (size_t)(f >> 6) * h_pad * 64 + (f & 7);
+      const int h_chk = (f & 63) >> 3;
       float* comb = U.grp ? a.comb_out1 : a.comb_out0;
       const int32_t* ctok = U.grp ? nullptr : a.comb_tok0;
       const float* cw = U.grp ? nullptr : a.comb_w0;
@@ -1188,8 +1247,13 @@ __global__ void __launch_bounds__(threads_of(MODE, Q), 1)
                 const float gv = __uint_as_float(g[i]) * (sa0 * sb);
                 const float uv = __uint_as_float(v[i]) * (sa1 * sb);
                 const float hv = silu_mul(gv, uv);
-                static_cast<uint16_t*>(out)[o + (size_t)(c0 + i) * a.out_ld] =
-                    float_to_bf16_bits(hv);
+                // tile-packed h: token column c = c0 + i is row c of the tile;
+                // this thread's feature f is element f % 8 of 16-byte chunk
+                // (f % 64) / 8 of block f / 64
+                const int c = c0 + i;
+                const size_t idx = h_tiled ? h_blk + (size_t)c * 64 + ((h_chk ^ (c & 7)) << 3)
+                                           : o + (size_t)c * a.out_ld;
+                static_cast<uint16_t*>(out)[idx] = float_to_bf16_bits(hv);
               }
             }
           } else if constexpr (MODE == MODE_PLAIN2) {
@@ -1366,6 +1430,12 @@ moe_status run_ffn(const FfnGroup& g0, const FfnGroup* g1, int H, int I, cudaStr
   const bool pk = PK;
   if (g0.packed != PK || (F8 && PK)) return MOE_ERR_UNSUPPORTED;  // packed tiles are bf16 only
   const uint64_t xr = gather ? g0.x_rows : g0.rows;
+  // tile-packed token rows: bf16 only, x written for this launch's tile
+  if (g0.x_tiled || g0.h_tiled || (g1 && (g1->x_tiled || g1->h_tiled))) {
+    if (F8 || (g0.x_tiled && (gather || g0.x_tile != NMAX)) ||
+        (g1 && g1->x_tiled && g1->x_tile != NMAX))
+      return MOE_ERR_UNSUPPORTED;
+  }
   // GEMM2's token operand: h (bf16), or its e4m3 copy hq in the FP8 form
   const void* h0 = F8 ? static_cast<const void*>(g0.hq) : static_cast<const void*>(g0.h);
   if (!make_rows_map<F8>(&a1, g0.W13, H, (uint64_t)g0.n_experts * 2 * I, BM) ||
@@ -1444,6 +1514,10 @@ moe_status run_ffn(const FfnGroup& g0, const FfnGroup* g1, int H, int I, cudaStr
   }
   args.trace = g0.trace;
   args.trace_cap = g0.trace ? g0.trace_cap : 0;
+  args.b_tiled0 = g0.x_tiled ? static_cast<const uint8_t*>(g0.x) : nullptr;
+  args.b_tiled1 = (g1 && g1->x_tiled) ? static_cast<const uint8_t*>(g1->x) : nullptr;
+  args.out_tiled0 = g0.h_tiled;
+  args.out_tiled1 = g1 && g1->h_tiled;
   moe_status st =
       launch_gemm<MODE_SWIGLU, NMAX, Q, PK>(a1, b1, sa1, sb1, b1big, sb1big, args, s);
   if (st != MOE_OK) return st;
@@ -1457,6 +1531,10 @@ moe_status run_ffn(const FfnGroup& g0, const FfnGroup* g1, int H, int I, cudaStr
   }
   if (after_gemm1 && cudaEventRecord(after_gemm1, s) != cudaSuccess) return MOE_ERR_CUDA;
   args.gather0 = nullptr;  // GEMM2 reads h, already in packed row order
+  args.b_tiled0 = g0.h_tiled ? reinterpret_cast<const uint8_t*>(g0.h) : nullptr;
+  args.b_tiled1 = (g1 && g1->h_tiled) ? reinterpret_cast<const uint8_t*>(g1->h) : nullptr;
+  args.out_tiled0 = 0;
+  args.out_tiled1 = 0;
   args.pack_src = nullptr;
   args.pack_dst = nullptr;
   args.trace = nullptr;
@@ -1504,35 +1582,40 @@ moe_status run_ffn(const FfnGroup& g0, const FfnGroup* g1, int H, int I, cudaStr
 
 }  // namespace
 
+int ffn_tile_rows(long rows_hint, int n_exp, bool fp8, bool fp8_block) {
+  const long per = rows_hint / (n_exp > 0 ? n_exp : 1);
+  if (per <= 24) return 32;
+  if (per <= 132) return 144;
+  return fp8 && fp8_block ? 224 : 256;
+}
+
 moe_status launch_expert_ffn_groups(const FfnGroup& routed, const FfnGroup* dense, int H, int I,
                                     int rows_hint, cudaStream_t s, cudaEvent_t after_gemm1) {
   if ((routed.rows == 0 || routed.e_end <= routed.e_begin) && (!dense || dense->rows == 0))
     return MOE_OK;
   const int n_exp = routed.e_end - routed.e_begin;
   const FfnGroup* g1 = (dense && dense->rows > 0) ? dense : nullptr;
-  // Token-tile size from the expected rows per expert: small tiles leave more
-  // of the stage ring to weights (decode ~4 rows/expert -> 32; balanced
-  // prefill ~128 +- 10 % -> 144; larger or skewed loads -> 256).
-  const long per = (long)rows_hint / (n_exp > 0 ? n_exp : 1);
+  // the token tile (ffn_tile_rows); block-scaled FP8's largest is 224 rows:
+  // two 224-column accumulators and the stages' scale columns share TMEM's
+  // 512 columns
+  const int tile = ffn_tile_rows(rows_hint, n_exp, routed.fp8, routed.fp8_block);
   if (routed.fp8 && routed.fp8_block) {
-    // the largest tile is 224 rows: two 224-column accumulators and the
-    // stages' scale columns share TMEM's 512 columns
-    if (per <= 24) return run_ffn<32, Q_BLOCK, false>(routed, g1, H, I, s, after_gemm1);
-    if (per <= 132) return run_ffn<144, Q_BLOCK, false>(routed, g1, H, I, s, after_gemm1);
+    if (tile == 32) return run_ffn<32, Q_BLOCK, false>(routed, g1, H, I, s, after_gemm1);
+    if (tile == 144) return run_ffn<144, Q_BLOCK, false>(routed, g1, H, I, s, after_gemm1);
     return run_ffn<224, Q_BLOCK, false>(routed, g1, H, I, s, after_gemm1);
   }
   if (routed.fp8) {
-    if (per <= 24) return run_ffn<32, Q_ROW, false>(routed, g1, H, I, s, after_gemm1);
-    if (per <= 132) return run_ffn<144, Q_ROW, false>(routed, g1, H, I, s, after_gemm1);
+    if (tile == 32) return run_ffn<32, Q_ROW, false>(routed, g1, H, I, s, after_gemm1);
+    if (tile == 144) return run_ffn<144, Q_ROW, false>(routed, g1, H, I, s, after_gemm1);
     return run_ffn<256, Q_ROW, false>(routed, g1, H, I, s, after_gemm1);
   }
   if (routed.packed) {
-    if (per <= 24) return run_ffn<32, Q_BF16, true>(routed, g1, H, I, s, after_gemm1);
-    if (per <= 132) return run_ffn<144, Q_BF16, true>(routed, g1, H, I, s, after_gemm1);
+    if (tile == 32) return run_ffn<32, Q_BF16, true>(routed, g1, H, I, s, after_gemm1);
+    if (tile == 144) return run_ffn<144, Q_BF16, true>(routed, g1, H, I, s, after_gemm1);
     return run_ffn<256, Q_BF16, true>(routed, g1, H, I, s, after_gemm1);
   }
-  if (per <= 24) return run_ffn<32, Q_BF16, false>(routed, g1, H, I, s, after_gemm1);
-  if (per <= 132) return run_ffn<144, Q_BF16, false>(routed, g1, H, I, s, after_gemm1);
+  if (tile == 32) return run_ffn<32, Q_BF16, false>(routed, g1, H, I, s, after_gemm1);
+  if (tile == 144) return run_ffn<144, Q_BF16, false>(routed, g1, H, I, s, after_gemm1);
   return run_ffn<256, Q_BF16, false>(routed, g1, H, I, s, after_gemm1);
 }
 

@@ -311,6 +311,41 @@ __global__ void gather_rows_kernel(const uint4* __restrict__ x, int vpr,
   }
 }
 
+// The same in the tile-packed layout (TiledRow): one warp per packed row, the
+// row's expert found by binary search over the range's offsets (the last e
+// with offsets[e] <= r, so empty experts are passed over), four 16-byte loads
+// of a lane in flight before its stores.
+__global__ void gather_rows_tiled_kernel(const uint4* __restrict__ x, int vpr,
+                                         const int32_t* __restrict__ row_src_token,
+                                         const int32_t* __restrict__ offsets, int e_begin,
+                                         int e_end, int tile, uint4* __restrict__ x_perm) {
+  constexpr int U = 4;
+  const int r0 = offsets[e_begin], r1 = offsets[e_end];
+  const int lane = threadIdx.x & 31;
+  const int wpb = blockDim.x >> 5;
+  const int n_warps = gridDim.x * wpb;
+  for (int r = r0 + blockIdx.x * wpb + (threadIdx.x >> 5); r < r1; r += n_warps) {
+    int lo = e_begin, hi = e_end - 1;
+    while (lo < hi) {
+      const int mid = (lo + hi + 1) >> 1;
+      if (offsets[mid] <= r) lo = mid;
+      else hi = mid - 1;
+    }
+    const int oe = offsets[lo];
+    const TiledRow w = tiled_row(r, lo, oe, offsets[lo + 1] - oe, tile, vpr);
+    const uint4* src = x + (size_t)row_src_token[r] * vpr;
+    for (int v0 = lane; v0 < vpr; v0 += 32 * U) {
+      uint4 val[U];
+#pragma unroll
+      for (int u = 0; u < U; ++u)
+        if (v0 + 32 * u < vpr) val[u] = src[v0 + 32 * u];
+#pragma unroll
+      for (int u = 0; u < U; ++u)
+        if (v0 + 32 * u < vpr) x_perm[w.chunk16(v0 + 32 * u)] = val[u];
+    }
+  }
+}
+
 // out[t] = sum_j w[t,j] * y_perm[slot_row[t*k+j]] (+ shared[t]); 8 elements per thread-step.
 // The slots are taken eight at a time: their rows and weights first, then all
 // sixteen 16-byte row loads, then the fused multiply-adds in slot order (the
@@ -466,9 +501,19 @@ moe_status launch_dispatch_rows(int T, int H, int k, const uint16_t* x, const in
 
 moe_status launch_gather_rows(int H, const uint16_t* x, const int32_t* row_src_token,
                               const int32_t* offsets, int e_begin, int e_end, uint16_t* x_perm,
-                              int max_rows, cudaStream_t s) {
+                              int max_rows, cudaStream_t s, int tile) {
   if (max_rows == 0 || e_end <= e_begin) return MOE_OK;
   const int vpr = H / 8;
+  if (tile > 0) {
+    const int per_block = 8;  // warps of a 256-thread block, one packed row each
+    long blocks = ((long)max_rows + per_block - 1) / per_block;
+    const long cap = (long)num_sms() * 16;
+    gather_rows_tiled_kernel<<<(int)(blocks < cap ? blocks : cap), 32 * per_block, 0, s>>>(
+        reinterpret_cast<const uint4*>(x), vpr, row_src_token, offsets, e_begin, e_end, tile,
+        reinterpret_cast<uint4*>(x_perm));
+    note_launch();
+    return launch_status();
+  }
   gather_rows_kernel<<<copy_grid((size_t)max_rows * vpr), 256, 0, s>>>(
       reinterpret_cast<const uint4*>(x), vpr, row_src_token, offsets, e_begin, e_end,
       reinterpret_cast<uint4*>(x_perm));

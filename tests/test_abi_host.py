@@ -228,13 +228,17 @@ def test_fp8_entry_points_reject_bad_arguments_without_a_gpu(lib):
         p, p, None, p, 1 << 40, z, z) == L.MOE_ERR_INVALID_ARG                 # no such form
     W8 = L.moe_weights(0x1000, None, 0x1000, 0x1000, 0x1000, 0x1000, 0, 0x1000, 0x1000, 0x1000, 0x1000)
     assert lib.moe_layer_forward(cb(c), cb(ex8), cb(W8), p, p, None, z, 0, z, z) == L.MOE_ERR_WORKSPACE
-    # the fp8 layout adds the quantized copies; its x_perm is half the bf16 one
+    # the fp8 layout adds the quantized copies; its x_perm is half the bf16 one,
+    # and its row-major x_perm and h have none of the bf16 tile-packed buffers'
+    # 16 padding rows per expert (16 for the shared expert's h)
     for wl in (I.DECODE, I.PREFILL):
         cw = L.config_of(wl)
         n16 = L.moe_workspace_size(cw, L.exec_config(fuse_gather=0))
         n8 = L.moe_workspace_size(cw, L.exec_config(fuse_gather=0, fp8=1))
         tk = wl.T * wl.k
-        assert n8 - n16 >= wl.T * wl.H + tk * wl.I - tk * wl.H - (1 << 16)
+        pad = 16 * wl.E * 2 * (wl.H + wl.I) + 16 * 2 * wl.I_shared
+        assert n16 >= (tk + 16 * wl.E) * 2 * (wl.H + wl.I)
+        assert n8 - n16 >= wl.T * wl.H + tk * wl.I - tk * wl.H - pad - (1 << 16)
 
 
 def test_fp8_block_entry_points_reject_bad_arguments_without_a_gpu(lib):

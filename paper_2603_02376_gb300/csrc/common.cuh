@@ -138,6 +138,9 @@ struct FfnGroup {
   bool x_tiled;
   bool h_tiled;
   int x_tile;  // the token tile x was written with (x_tiled)
+  // FP8 (row scales): hq, GEMM2's e4m3 operand, in the tile-packed layout (h
+  // itself stays row-major for the quantizer); hq then holds the padding rows
+  bool hq_tiled;
   // FP8 (e4m3) form: per-row fp32 scales of x (indexed by token through
   // x_scale_idx when x holds packed copies, else by row), of W13 and W2 rows;
   // hq / hs receive GEMM2's quantized operand and its row scales.
@@ -208,9 +211,12 @@ moe_status launch_expert_ffn(int rows, int H, int I, int n_experts, int e_begin,
                              cudaStream_t s, cudaEvent_t after_gemm1 = nullptr,
                              bool packed = false);
 
-// e4m3 row quantization of a bf16 matrix [rows, K] (K % 8 == 0).
+// e4m3 row quantization of a bf16 matrix [rows, K] (K % 8 == 0); tile > 0:
+// only the packed rows of experts [e_begin, e_end) of `offsets`, the e4m3
+// rows written in the tile-packed layout (TiledRow), K % 16 == 0.
 moe_status launch_quantize_rows(const uint16_t* in, long rows, int K, uint8_t* out, float* scale,
-                                cudaStream_t s);
+                                cudaStream_t s, const int32_t* offsets = nullptr,
+                                int e_begin = 0, int e_end = 0, int tile = 0);
 
 // e4m3 quantization of a bf16 matrix [rows, K] in 1 x 128 blocks (K % 128 == 0):
 // k = the smallest exponent with amax <= 448 * 2^k (0 for a zero block, within

@@ -1430,9 +1430,13 @@ moe_status run_ffn(const FfnGroup& g0, const FfnGroup* g1, int H, int I, cudaStr
   const bool pk = PK;
   if (g0.packed != PK || (F8 && PK)) return MOE_ERR_UNSUPPORTED;  // packed tiles are bf16 only
   const uint64_t xr = gather ? g0.x_rows : g0.rows;
-  // tile-packed token rows: bf16 only, x written for this launch's tile
-  if (g0.x_tiled || g0.h_tiled || (g1 && (g1->x_tiled || g1->h_tiled))) {
-    if (F8 || (g0.x_tiled && (gather || g0.x_tile != NMAX)) ||
+  // tile-packed token rows: bf16 (x, h) or row-scaled e4m3 (x, hq), x written
+  // for this launch's tile
+  if (g0.x_tiled || g0.h_tiled || g0.hq_tiled ||
+      (g1 && (g1->x_tiled || g1->h_tiled || g1->hq_tiled))) {
+    if (MX || (F8 && (g0.h_tiled || (g1 && g1->h_tiled))) ||
+        (!F8 && (g0.hq_tiled || (g1 && g1->hq_tiled))) ||
+        (g0.x_tiled && (gather || g0.x_tile != NMAX)) ||
         (g1 && g1->x_tiled && g1->x_tile != NMAX))
       return MOE_ERR_UNSUPPORTED;
   }
@@ -1526,13 +1530,26 @@ moe_status run_ffn(const FfnGroup& g0, const FfnGroup* g1, int H, int I, cudaStr
     if (g1)
       MOE_STATUS_TRY(launch_quantize_blocks(g1->h, g1->rows, I, g1->hq, g1->hsf, g1->h_sf_ld, s));
   } else if (F8) {  // h of every packed row -> e4m3 and its row scale: GEMM2's operand
-    MOE_STATUS_TRY(launch_quantize_rows(g0.h, g0.rows, I, g0.hq, g0.hs, s));
-    if (g1) MOE_STATUS_TRY(launch_quantize_rows(g1->h, g1->rows, I, g1->hq, g1->hs, s));
+    if (g0.hq_tiled)  // the rows of this launch's experts, tile-packed
+      MOE_STATUS_TRY(launch_quantize_rows(g0.h, g0.rows, I, g0.hq, g0.hs, s, g0.offsets,
+                                          g0.e_begin, g0.e_end, NMAX));
+    else
+      MOE_STATUS_TRY(launch_quantize_rows(g0.h, g0.rows, I, g0.hq, g0.hs, s));
+    if (g1 && g1->hq_tiled)
+      MOE_STATUS_TRY(launch_quantize_rows(g1->h, g1->rows, I, g1->hq, g1->hs, s, g1->offsets, 0,
+                                          1, NMAX));
+    else if (g1)
+      MOE_STATUS_TRY(launch_quantize_rows(g1->h, g1->rows, I, g1->hq, g1->hs, s));
   }
   if (after_gemm1 && cudaEventRecord(after_gemm1, s) != cudaSuccess) return MOE_ERR_CUDA;
   args.gather0 = nullptr;  // GEMM2 reads h, already in packed row order
-  args.b_tiled0 = g0.h_tiled ? reinterpret_cast<const uint8_t*>(g0.h) : nullptr;
-  args.b_tiled1 = (g1 && g1->h_tiled) ? reinterpret_cast<const uint8_t*>(g1->h) : nullptr;
+  args.b_tiled0 = g0.h_tiled    ? reinterpret_cast<const uint8_t*>(g0.h)
+                  : g0.hq_tiled ? static_cast<const uint8_t*>(g0.hq)
+                                : nullptr;
+  args.b_tiled1 = !g1              ? nullptr
+                  : g1->h_tiled  ? reinterpret_cast<const uint8_t*>(g1->h)
+                  : g1->hq_tiled ? static_cast<const uint8_t*>(g1->hq)
+                                 : nullptr;
   args.out_tiled0 = 0;
   args.out_tiled1 = 0;
   args.pack_src = nullptr;

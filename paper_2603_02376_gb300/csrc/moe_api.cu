@@ -162,9 +162,10 @@ struct Layout {
   // counts, zeroed with it and likewise left at 0 by each launch.
   int32_t* sched;
   bool pack_in_gemm = false;
-  // bf16 without token chunks: x_perm and h (and the shared expert's h) in the
-  // tile-packed row layout of the expert GEMMs' token tile (TiledRow), each
-  // with 16 padding rows per expert; 0 = row-major
+  // Without token chunks, bf16 or row-scaled e4m3: x_perm and GEMM2's operand
+  // (bf16 h, or e4m3 hq; and the shared expert's) in the tile-packed row
+  // layout of the expert GEMMs' token tile (TiledRow), each with 16 padding
+  // rows per expert; 0 = row-major
   int tile = 0;
   int32_t* pack_next;   // sched + 2
   int32_t* pack_ready;  // sched + 3, [E]
@@ -203,14 +204,15 @@ Layout carve(const moe_config& c, const moe_exec& ex, void* ws) {
   L.fp8_block = ex.fp8 == 2;
   const bool rows_fp8 = L.fp8 && !L.fp8_block;
   const size_t xb = L.fp8 ? 1 : 2;  // bytes per activation element
-  L.tile = (!L.fp8 && L.n_chunks == 1) ? ffn_tile_rows((long)T * k, c.E, false, false) : 0;
+  L.tile = (!L.fp8_block && L.n_chunks == 1) ? ffn_tile_rows((long)T * k, c.E, L.fp8, false)
+                                               : 0;
   const size_t pad = L.tile ? 16 * E : 0;  // padding rows of the tile-packed buffers
   L.x_q = L.fp8 ? cv.take<uint8_t>(T * c.H) : nullptr;
   L.x_s = rows_fp8 ? cv.take<float>(T) : nullptr;
   L.x_sf = L.fp8_block ? cv.take<uint8_t>((size_t)(c.H / 128) * T) : nullptr;
   L.x_perm = fuse ? nullptr : static_cast<void*>(cv.take<uint8_t>((T * k + pad) * c.H * xb));
-  L.h = cv.take<uint16_t>((T * k + pad) * c.I);
-  L.hq = L.fp8 ? cv.take<uint8_t>(T * k * c.I) : nullptr;
+  L.h = cv.take<uint16_t>((T * k + (L.fp8 ? 0 : pad)) * c.I);
+  L.hq = L.fp8 ? cv.take<uint8_t>((T * k + pad) * c.I) : nullptr;
   L.hs = rows_fp8 ? cv.take<float>(T * k) : nullptr;
   L.hsf = L.fp8_block ? cv.take<uint8_t>((size_t)(c.I / 128) * T * k) : nullptr;
   L.fuse_combine = ex.fuse_combine != 0;
@@ -218,8 +220,9 @@ Layout carve(const moe_config& c, const moe_exec& ex, void* ws) {
   L.y_perm = L.fuse_combine ? nullptr : cv.take<float>(T * k * c.H);
   L.acc = (L.fuse_combine && !ex.out_fp32) ? cv.take<float>(T * c.H) : nullptr;
   L.sh_off = cv.take<int32_t>(2);
-  L.sh_h = c.I_shared ? cv.take<uint16_t>((T + (L.tile ? 16 : 0)) * c.I_shared) : nullptr;
-  L.sh_hq = (c.I_shared && L.fp8) ? cv.take<uint8_t>(T * c.I_shared) : nullptr;
+  const size_t sh_pad = L.tile ? 16 : 0;
+  L.sh_h = c.I_shared ? cv.take<uint16_t>((T + (L.fp8 ? 0 : sh_pad)) * c.I_shared) : nullptr;
+  L.sh_hq = (c.I_shared && L.fp8) ? cv.take<uint8_t>((T + sh_pad) * c.I_shared) : nullptr;
   L.sh_hs = (c.I_shared && rows_fp8) ? cv.take<float>(T) : nullptr;
   L.sh_hsf = (c.I_shared && L.fp8_block) ? cv.take<uint8_t>((size_t)(c.I_shared / 128) * T)
                                          : nullptr;
@@ -335,7 +338,11 @@ moe_status pack_tokens(const moe_config& c, const Layout& L, const moe_weights& 
     // quantize, then dispatch the e4m3 rows: a row of H bytes is copied as
     // H / 2 two-byte units by the same copy kernel
     if (quantize) MOE_TRY(quantize_tokens(c, L, x, t0, Tc, s));
-    if (pack_rows)
+    if (pack_rows && L.tile)  // tile-packed e4m3 rows (H bytes: H / 16 chunks)
+      MOE_TRY(launch_gather_rows(c.H / 2, reinterpret_cast<const uint16_t*>(L.x_q), L.rst,
+                                 L.offsets, 0, c.E, static_cast<uint16_t*>(L.x_perm), Tc * c.k, s,
+                                 L.tile));
+    else if (pack_rows)
       MOE_TRY(launch_dispatch_rows(Tc, c.H / 2, c.k,
                                    reinterpret_cast<const uint16_t*>(L.x_q + (size_t)t0 * c.H),
                                    L.slot_row + tk,
@@ -369,7 +376,8 @@ FfnGroup routed_group(const moe_config& c, const Layout& L, const moe_weights& w
   g.W2 = w.W2;
   g.packed = w.packed != 0;
   g.h = L.h + tk * c.I;
-  g.h_tiled = L.tile > 0;  // (tiled only without token chunks: tk = 0)
+  g.h_tiled = L.tile > 0 && !L.fp8;  // (tiled only without token chunks: tk = 0)
+  g.hq_tiled = L.tile > 0 && L.fp8;
   g.x_tiled = L.tile > 0 && L.x_perm != nullptr;
   g.x_tile = L.tile;
   if (L.fuse_combine) {  // GEMM2 adds w * y into the token rows of the accumulator
@@ -430,7 +438,8 @@ FfnGroup dense_group(const moe_config& c, const Layout& L, const moe_weights& w,
   g.W13 = w.Ws13;
   g.W2 = w.Ws2;
   g.h = L.sh_h;
-  g.h_tiled = L.tile > 0;
+  g.h_tiled = L.tile > 0 && !L.fp8;
+  g.hq_tiled = L.tile > 0 && L.fp8;
   g.y = L.sh_y;
   g.comb_out = L.fuse_combine ? L.acc : nullptr;  // token rows, weight 1
   g.packed = w.packed != 0;
@@ -926,7 +935,7 @@ moe_status moe_layer_forward(const moe_config* cfg, const moe_exec* ex, const mo
     if (L.x_perm && L.fp8)  // e4m3 rows: H bytes = H / 2 two-byte units
       MOE_TRY(launch_gather_rows(c.H / 2, reinterpret_cast<const uint16_t*>(L.x_q), L.rst,
                                  L.offsets, e0, e1, static_cast<uint16_t*>(L.x_perm), c.T * c.k,
-                                 ps));
+                                 ps, L.tile));
     else if (L.x_perm)  // with a fused dispatch GEMM1 gathers the rows itself
       MOE_TRY(launch_gather_rows(c.H, x, L.rst, L.offsets, e0, e1,
                                  static_cast<uint16_t*>(L.x_perm), c.T * c.k, ps, L.tile));

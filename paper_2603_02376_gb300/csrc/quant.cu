@@ -45,6 +45,48 @@ __global__ void __launch_bounds__(Q_WARPS * 32) quantize_rows_kernel(
   }
 }
 
+// The same for the packed rows of experts [e_begin, e_end) with the e4m3 rows
+// written in the tile-packed layout (TiledRow: rows of K / 16 chunks); the
+// scales stay indexed by packed row. One warp per row; the row's expert is
+// the last e with offsets[e] <= r.
+__global__ void __launch_bounds__(Q_WARPS * 32) quantize_rows_tiled_kernel(
+    const uint4* __restrict__ in, int vpr, const int32_t* __restrict__ offsets, int e_begin,
+    int e_end, int tile, uint2* __restrict__ out, float* __restrict__ scale) {
+  const int lane = threadIdx.x % 32;
+  const long r = (long)offsets[e_begin] + (long)blockIdx.x * Q_WARPS + threadIdx.x / 32;
+  if (r >= offsets[e_end]) return;  // uniform per warp
+  int lo = e_begin, hi = e_end - 1;
+  while (lo < hi) {
+    const int mid = (lo + hi + 1) >> 1;
+    if (offsets[mid] <= r) lo = mid;
+    else hi = mid - 1;
+  }
+  const TiledRow w = tiled_row((int)r, lo, offsets[lo], offsets[lo + 1] - offsets[lo], tile,
+                               vpr / 2);
+  const uint4* src = in + r * vpr;
+  float amax = 0.f;
+  for (int v = lane; v < vpr; v += 32) {
+    const uint4 x = src[v];
+    const uint16_t* h = reinterpret_cast<const uint16_t*>(&x);
+#pragma unroll
+    for (int i = 0; i < 8; ++i) amax = fmaxf(amax, fabsf(bf16_bits_to_float(h[i])));
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) amax = fmaxf(amax, __shfl_xor_sync(0xffffffffu, amax, o));
+  const float s = amax > 0.f ? amax / 448.0f : 1.0f;
+  if (lane == 0) scale[r] = s;
+  for (int v = lane; v < vpr; v += 32) {
+    const uint4 x = src[v];
+    const uint16_t* h = reinterpret_cast<const uint16_t*>(&x);
+    uint8_t q[8];
+#pragma unroll
+    for (int i = 0; i < 8; ++i)
+      q[i] = __nv_cvt_float_to_fp8(bf16_bits_to_float(h[i]) / s, __NV_SATFINITE, __NV_E4M3);
+    // 8 bytes = half of 16-byte chunk v / 2 of the e4m3 row
+    out[w.chunk16(v >> 1) * 2 + (v & 1)] = *reinterpret_cast<const uint2*>(q);
+  }
+}
+
 // Block scales (DeepSeek-V3's fine-grained FP8: 1 x 128 blocks of activation
 // rows, 128 x 128 blocks of weights) as UE8M0 exponents: k is the smallest
 // integer with amax <= 448 * 2^k, read off amax's fp32 bits (amax = f * 2^p,
@@ -155,9 +197,18 @@ moe_status launch_quantize_weight_blocks(const uint16_t* in, long rows, int K, u
 }
 
 moe_status launch_quantize_rows(const uint16_t* in, long rows, int K, uint8_t* out, float* scale,
-                                cudaStream_t s) {
+                                cudaStream_t s, const int32_t* offsets, int e_begin, int e_end,
+                                int tile) {
   if (rows == 0) return MOE_OK;
   const long blocks = (rows + Q_WARPS - 1) / Q_WARPS;
+  if (tile > 0) {
+    if (e_end <= e_begin) return MOE_OK;
+    quantize_rows_tiled_kernel<<<(unsigned)blocks, Q_WARPS * 32, 0, s>>>(
+        reinterpret_cast<const uint4*>(in), K / 8, offsets, e_begin, e_end, tile,
+        reinterpret_cast<uint2*>(out), scale);
+    note_launch();
+    return launch_status();
+  }
   quantize_rows_kernel<<<(unsigned)blocks, Q_WARPS * 32, 0, s>>>(
       reinterpret_cast<const uint4*>(in), rows, K / 8, reinterpret_cast<uint2*>(out), scale);
   note_launch();

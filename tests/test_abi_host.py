@@ -282,14 +282,17 @@ def test_fp8_block_entry_points_reject_bad_arguments_without_a_gpu(lib):
     Wn = L.moe_weights(0x1000, None, 0x1000, 0x1000, 0x1000, 0x1000, 0, 0x1001, None, 0x1001,
                        0x1001)
     assert lib.moe_layer_forward(cb(c), cb(exb), cb(Wn), p, p, None, z, 0, z, z) == L.MOE_ERR_INVALID_ARG
-    # the block layout: per-row scale arrays replaced by exponent bytes
+    # the block layout: per-row scale arrays replaced by exponent bytes, and its
+    # row-major e4m3 x_perm and hq without the row-scaled form's tile-packing
+    # padding (16 rows per expert, 16 for the shared expert's hq)
     for wl in (I.DECODE, I.PREFILL):
         cw = L.config_of(wl)
         n8 = L.moe_workspace_size(cw, L.exec_config(fuse_gather=0, fp8=1))
         nb = L.moe_workspace_size(cw, L.exec_config(fuse_gather=0, fp8=2))
         tk = wl.T * wl.k
         extra = wl.H // 128 * wl.T + wl.I // 128 * tk + wl.I_shared // 128 * wl.T
-        assert nb - n8 == pytest.approx(extra - 4 * (wl.T + tk + wl.T), abs=4096)
+        pad = 16 * wl.E * (wl.H + wl.I) + 16 * wl.I_shared
+        assert nb - n8 == pytest.approx(extra - 4 * (wl.T + tk + wl.T) - pad, abs=4096)
 
 
 def test_empty_batch_is_a_no_op(lib):

@@ -594,8 +594,13 @@ def dispatch_label(args, wl):
     f = dispatch_flag(args, wl)
     if f == 1 and wl.T * wl.k <= 24 * wl.E:
         return "fused into GEMM1 (TMA gather4)"
+    tiled = args.mode != "overlap-tokens" and args.precision != "fp8-block"
+    rows = " in the tile-packed row layout" if tiled else ""
     if f == 2 and args.mode == "seq" and args.precision != "fp8-block":
-        return "inside the GEMM1 launch (pack warps write x_perm behind the shared expert)"
+        return ("inside the GEMM1 launch (pack warps write x_perm" + rows
+                + " behind the shared expert)")
+    if tiled:
+        return "packed x_perm in the tile-packed row layout (dispatch kernel)"
     return "packed x_perm (dispatch kernel)"
 
 
@@ -835,7 +840,11 @@ def run_ours(args, wl, rank, world, local, device):
         torch.cuda.synchronize()
         t_single = max_over_ranks(g0.elapsed_time(g1), world) / args.steps
         t_ovl = ms / args.steps
-        t_pack = sum(stage_ms[k] for k in ("router", "gate", "permute", "dispatch"))
+        # the pipelined modes pack on the pack stream with the gather kernel, not
+        # inside GEMM1: their pack work is that of the sequential forward with
+        # the packed dispatch
+        pk_ms = stage_ms if fuse != 2 else traced(0)
+        t_pack = sum(pk_ms[k] for k in ("router", "gate", "permute", "dispatch"))
         overlap = {"ms_two_streams": round(t_ovl, 4), "ms_same_chunks_one_stream": round(t_single, 4),
                    "ms_pack_work": round(t_pack, 4),
                    "hidden_frac": round((t_single - t_ovl) / t_pack, 3) if t_pack > 0 else None,

@@ -101,8 +101,11 @@ __host__ __device__ inline TiledRow tiled_row(int r, int e, int off_e, int cnt_e
   return w;
 }
 
+// tile > 0: x_perm in the tile-packed layout, slot n's expert idx[n] and the
+// packed-row offsets [E+1] placing its row.
 moe_status launch_dispatch_rows(int T, int H, int k, const uint16_t* x, const int32_t* slot_row,
-                                uint16_t* x_perm, cudaStream_t s);
+                                uint16_t* x_perm, cudaStream_t s, int tile = 0,
+                                const int32_t* idx = nullptr, const int32_t* offsets = nullptr);
 // x_perm[r] = x[row_src_token[r]] for the rows of experts [e_begin, e_end);
 // tile > 0 writes them in the tile-packed layout above (offsets global).
 moe_status launch_gather_rows(int H, const uint16_t* x, const int32_t* row_src_token,

@@ -339,18 +339,19 @@ moe_status pack_tokens(const moe_config& c, const Layout& L, const moe_weights& 
     // H / 2 two-byte units by the same copy kernel
     if (quantize) MOE_TRY(quantize_tokens(c, L, x, t0, Tc, s));
     if (pack_rows && L.tile)  // tile-packed e4m3 rows (H bytes: H / 16 chunks)
-      MOE_TRY(launch_gather_rows(c.H / 2, reinterpret_cast<const uint16_t*>(L.x_q), L.rst,
-                                 L.offsets, 0, c.E, static_cast<uint16_t*>(L.x_perm), Tc * c.k, s,
-                                 L.tile));
+      MOE_TRY(launch_dispatch_rows(Tc, c.H / 2, c.k,
+                                   reinterpret_cast<const uint16_t*>(L.x_q + (size_t)t0 * c.H),
+                                   L.slot_row + tk, static_cast<uint16_t*>(L.x_perm), s, L.tile,
+                                   L.idx + tk, L.offsets));
     else if (pack_rows)
       MOE_TRY(launch_dispatch_rows(Tc, c.H / 2, c.k,
                                    reinterpret_cast<const uint16_t*>(L.x_q + (size_t)t0 * c.H),
                                    L.slot_row + tk,
                                    static_cast<uint16_t*>(L.x_perm) + tk * c.H / 2, s));
-  } else if (pack_rows && L.tile) {
-    // tile-packed x_perm: every packed row from its token (row_src_token)
-    MOE_TRY(launch_gather_rows(c.H, x, L.rst, L.offsets, 0, c.E,
-                               static_cast<uint16_t*>(L.x_perm), Tc * c.k, s, L.tile));
+  } else if (pack_rows && L.tile) {  // tile-packed x_perm
+    MOE_TRY(launch_dispatch_rows(Tc, c.H, c.k, x + (size_t)t0 * c.H, L.slot_row + tk,
+                                 static_cast<uint16_t*>(L.x_perm), s, L.tile, L.idx + tk,
+                                 L.offsets));
   } else if (pack_rows) {
     MOE_TRY(launch_dispatch_rows(Tc, c.H, c.k, x + (size_t)t0 * c.H, L.slot_row + tk,
                                  static_cast<uint16_t*>(L.x_perm) + tk * c.H, s));

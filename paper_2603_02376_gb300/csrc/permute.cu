@@ -297,6 +297,45 @@ __global__ void dispatch_rows_kernel(const uint4* __restrict__ x, int T, int vpr
   }
 }
 
+// The same into the tile-packed layout (TiledRow): slot n = t*k + j of token t
+// goes to packed row slot_row[n] of expert idx[n] (the gate's choice); the
+// slot rows, experts and expert offsets of eight slots are read (loads the
+// lanes of a warp share, one token's chunks being consecutive threads) before
+// the eight stores.
+__global__ void dispatch_rows_tiled_kernel(const uint4* __restrict__ x, int T, int vpr, int k,
+                                           const int32_t* __restrict__ slot_row,
+                                           const int32_t* __restrict__ idx,
+                                           const int32_t* __restrict__ offsets, int tile,
+                                           uint4* __restrict__ x_perm) {
+  constexpr int KB = 8;
+  const size_t total = (size_t)T * vpr;
+  for (size_t i = blockIdx.x * (size_t)blockDim.x + threadIdx.x; i < total;
+       i += (size_t)gridDim.x * blockDim.x) {
+    const size_t t = i / vpr;
+    const int v = (int)(i % vpr);
+    const uint4 val = x[i];
+    for (int j0 = 0; j0 < k; j0 += KB) {
+      int r[KB], e[KB];
+#pragma unroll
+      for (int q = 0; q < KB; ++q) {
+        const bool ok = j0 + q < k;
+        r[q] = ok ? slot_row[t * k + j0 + q] : 0;
+        e[q] = ok ? idx[t * k + j0 + q] : 0;
+      }
+      int oe[KB], ne[KB];
+#pragma unroll
+      for (int q = 0; q < KB; ++q) {
+        oe[q] = offsets[e[q]];
+        ne[q] = offsets[e[q] + 1];
+      }
+#pragma unroll
+      for (int q = 0; q < KB; ++q)
+        if (j0 + q < k)
+          x_perm[tiled_row(r[q], e[q], oe[q], ne[q] - oe[q], tile, vpr).chunk16(v)] = val;
+    }
+  }
+}
+
 // x_perm[r] = x[row_src_token[r]] for rows of experts [e_begin, e_end).
 __global__ void gather_rows_kernel(const uint4* __restrict__ x, int vpr,
                                    const int32_t* __restrict__ row_src_token,
@@ -490,9 +529,17 @@ moe_status launch_permutation(const moe_config& c, const int32_t* idx, int32_t* 
 }
 
 moe_status launch_dispatch_rows(int T, int H, int k, const uint16_t* x, const int32_t* slot_row,
-                                uint16_t* x_perm, cudaStream_t s) {
+                                uint16_t* x_perm, cudaStream_t s, int tile, const int32_t* idx,
+                                const int32_t* offsets) {
   if (T == 0) return MOE_OK;
   const int vpr = H / 8;
+  if (tile > 0) {
+    dispatch_rows_tiled_kernel<<<copy_grid((size_t)T * vpr), 256, 0, s>>>(
+        reinterpret_cast<const uint4*>(x), T, vpr, k, slot_row, idx, offsets, tile,
+        reinterpret_cast<uint4*>(x_perm));
+    note_launch();
+    return launch_status();
+  }
   dispatch_rows_kernel<<<copy_grid((size_t)T * vpr), 256, 0, s>>>(
       reinterpret_cast<const uint4*>(x), T, vpr, k, slot_row, reinterpret_cast<uint4*>(x_perm));
   note_launch();

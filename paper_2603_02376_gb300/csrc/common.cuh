@@ -140,7 +140,7 @@ struct FfnGroup {
   // output, GEMM2's operand); both buffers then hold rows + 16 * n_experts rows.
   bool x_tiled;
   bool h_tiled;
-  int x_tile;  // the token tile x was written with (x_tiled)
+  int x_tile;  // the token tile x and h are laid out for (0 = chosen by the launch)
   // FP8 (row scales): hq, GEMM2's e4m3 operand, in the tile-packed layout (h
   // itself stays row-major for the quantizer); hq then holds the padding rows
   bool hq_tiled;

@@ -1615,7 +1615,9 @@ moe_status launch_expert_ffn_groups(const FfnGroup& routed, const FfnGroup* dens
   // the token tile (ffn_tile_rows); block-scaled FP8's largest is 224 rows:
   // two 224-column accumulators and the stages' scale columns share TMEM's
   // 512 columns
-  const int tile = ffn_tile_rows(rows_hint, n_exp, routed.fp8, routed.fp8_block);
+  // (the tile its rows were written with, for a tile-packed routed group)
+  const int tile = routed.x_tile > 0 ? routed.x_tile
+                                     : ffn_tile_rows(rows_hint, n_exp, routed.fp8, routed.fp8_block);
   if (routed.fp8 && routed.fp8_block) {
     if (tile == 32) return run_ffn<32, Q_BLOCK, false>(routed, g1, H, I, s, after_gemm1);
     if (tile == 144) return run_ffn<144, Q_BLOCK, false>(routed, g1, H, I, s, after_gemm1);

@@ -527,6 +527,24 @@ moe_status moe_testing_expert_ffn_stall(int32_t rows, int32_t H, int32_t I, int3
  */
 moe_status moe_testing_fail_stage(int32_t n);
 
+/*
+ * Testing (no counterpart in the paper): the tile-packed row layout in which
+ * the layer keeps its bf16 and row-scaled e4m3 token operands (x_perm, and
+ * GEMM2's h or hq). Writes to *out the index, in 16-byte units from the buffer's
+ * start, of 16-byte chunk c of packed row r, which belongs to expert e whose
+ * rows are [off_e, off_e + cnt_e). The rows of expert e are cut into tiles of
+ * `tile` rows; tile t starts at padded row off_e + 16 e + t tile and stores
+ * n_pad = its rows rounded up to 16; block kb (chunks 8 kb .. 8 kb + 7 of
+ * every row) of the tile is contiguous, n_pad x 8 chunks, and row i's chunk
+ * j sits at i * 8 + (j xor (i mod 8)) inside it. Host computation only (the
+ * function the kernels use). MOE_ERR_INVALID_ARG unless 0 <= e, cnt_e >= 1,
+ * off_e <= r < off_e + cnt_e, tile a positive multiple of 16,
+ * chunks_per_row a positive multiple of 8 and 0 <= c < chunks_per_row.
+ */
+moe_status moe_testing_tiled_chunk(int32_t r, int32_t e, int32_t off_e, int32_t cnt_e,
+                                   int32_t tile, int32_t chunks_per_row, int32_t c,
+                                   int64_t* out);
+
 /* Synchronises `stream`, then reads and clears the device error word of the
  * current device. MOE_OK, MOE_ERR_TIMEOUT or MOE_ERR_DEVICE_CHECK (or
  * MOE_ERR_CUDA if the synchronisation itself failed). */

@@ -34,7 +34,8 @@ EXPORTS = ("moe_status_string", "moe_validate_config", "moe_workspace_size",
            "moe_stack_forward", "moe_rms_norm", "moe_graph_create_stack", "moe_graph_launch",
            "moe_graph_kernel_count", "moe_graph_destroy", "moe_quantize_fp8_blocks",
            "moe_quantize_fp8_weight_blocks", "moe_expert_ffn_fp8_blocks",
-           "moe_expert_ffn_fp8_blocks_workspace_size", "moe_testing_fail_stage")
+           "moe_expert_ffn_fp8_blocks_workspace_size", "moe_testing_fail_stage",
+           "moe_testing_tiled_chunk")
 MOE_DISPATCH_NOALLOC_MAX_ENTRIES = 131072
 
 
@@ -130,6 +131,8 @@ def load(path: str = LIB_PATH) -> ctypes.CDLL:
         "moe_launch_count": (ctypes.c_uint64, []),
         "moe_shutdown": (None, []),
         "moe_testing_fail_stage": (S, [I32]),
+        "moe_testing_tiled_chunk": (S, [I32, I32, I32, I32, I32, I32, I32,
+                                        ctypes.POINTER(ctypes.c_int64)]),
     }
     for name, (res, args) in sig.items():
         f = getattr(lib, name)
@@ -377,6 +380,16 @@ def moe_testing_fail_stage(n: int) -> None:
     """Failure-injection hook: stage call n (0-based) of the forwards that follow fails
     with MOE_ERR_CUDA on the host; -1 turns it off."""
     _check(load().moe_testing_fail_stage(int(n)), "moe_testing_fail_stage")
+
+
+def moe_testing_tiled_chunk(r, e, off_e, cnt_e, tile, chunks_per_row, c) -> int:
+    """16-byte chunk index of chunk c of packed row r (expert e, rows [off_e, off_e + cnt_e))
+    in the layer's tile-packed token layout (host computation)."""
+    out = ctypes.c_int64()
+    _check(load().moe_testing_tiled_chunk(int(r), int(e), int(off_e), int(cnt_e), int(tile),
+                                          int(chunks_per_row), int(c), ctypes.byref(out)),
+           "moe_testing_tiled_chunk")
+    return out.value
 
 
 def moe_combine(cfg, y_perm, slot_row, topk_w, shared_out, out, out_fp32, stream=None) -> None:

@@ -979,6 +979,16 @@ moe_status moe_check_errors(void* stream) {
 
 uint64_t moe_launch_count(void) { return g_launches.load(std::memory_order_relaxed); }
 
+moe_status moe_testing_tiled_chunk(int32_t r, int32_t e, int32_t off_e, int32_t cnt_e,
+                                   int32_t tile, int32_t chunks_per_row, int32_t c,
+                                   int64_t* out) {
+  if (!out || e < 0 || off_e < 0 || cnt_e < 1 || r < off_e || r - off_e >= cnt_e || tile < 16 ||
+      tile % 16 || chunks_per_row < 8 || chunks_per_row % 8 || c < 0 || c >= chunks_per_row)
+    return MOE_ERR_INVALID_ARG;
+  *out = (int64_t)tiled_row(r, e, off_e, cnt_e, tile, chunks_per_row).chunk16(c);
+  return MOE_OK;
+}
+
 moe_status moe_testing_fail_stage(int32_t n) {
   if (n < -1) return MOE_ERR_INVALID_ARG;
   g_fail_countdown.store(n, std::memory_order_relaxed);

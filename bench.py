@@ -85,7 +85,8 @@ def parse():
                    help="comma-separated token counts of the sweep (default: 1024,4096,16384,65536)")
     p.add_argument("--unit-trace", action="store_true",
                    help="after the timed run, one more forward with GEMM1's per-unit trace "
-                        "(moe_exec.unit_trace); adds a gemm1_units summary to the JSON line")
+                        "(moe_exec.unit_trace) of GEMM1 and of GEMM2; adds gemm1_units and "
+                        "gemm2_units summaries to the JSON line")
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--cpu-tokens", type=int, default=None,
                    help="oracle sample size (tokens); default 128, or 8 with --precision "
@@ -353,12 +354,14 @@ def kernel_roofline(bytes_, flops, t_s, hbm_gbs, tf_sust, tf_burst, src, dtype):
     return r
 
 
-def unit_trace_summary(rec, H, fp8=0):
-    """Summary of GEMM1's per-unit trace records [n, 5] (int64): per token-row bin
+def unit_trace_summary(rec, H, fp8=0, flops_per_row=None):
+    """Summary of a GEMM's per-unit trace records [n, 5] (int64): per token-row bin
     of the routed units (and the shared expert's), the units' count and median
     times: wait = handed out -> first stage ready, mma = first stage ready ->
     accumulator complete, epilogue = accumulator complete -> stored; and the
-    unit's tensor rate while its MMAs ran (2 * 2 * 128 * m * H flops)."""
+    unit's tensor rate while its MMAs ran (flops_per_row * m; GEMM1's default
+    2 * 2 * 128 * H: gate and up of 128 features)."""
+    fpr = 2 * 2 * 128 * H if flops_per_row is None else flops_per_row
     rec = np.asarray(rec, dtype=np.int64)
     rec = rec[(rec[:, 3] > 0) & (rec[:, 1] > 0)]
     if len(rec) == 0:
@@ -368,7 +371,7 @@ def unit_trace_summary(rec, H, fp8=0):
     m = (meta >> 16) & 0xFFFF
     grp = ((meta >> 32) & 0xFFFF) >= 1024
     wait, mma, epi = t[:, 1] - t[:, 0], t[:, 2] - t[:, 1], t[:, 3] - t[:, 2]
-    tfs = 2 * 2 * 128 * m * H / np.maximum(mma, 1e-3) / 1e6   # TFLOP/s per SM
+    tfs = fpr * m / np.maximum(mma, 1e-3) / 1e6   # TFLOP/s per SM
     out = {"units": int(len(rec)), "span_us": round(float(t[:, 3].max()), 1),
            "sms": int(len(np.unique(meta & 0xFFFF)))}
     bins = {}
@@ -924,11 +927,17 @@ def run_ours(args, wl, rank, world, local, device):
                                         F / (pk * NOMINAL_BF16_TFLOPS * 1e12)) / t_step, 4),
         "bound": "hbm" if tb >= tfs else "tensor"}
     if args.unit_trace and not ex.overlap:
-        rt = torch.zeros((1 << 16, L.UNIT_TRACE_FIELDS), dtype=torch.int64, device=device)
-        L.moe_layer_forward(cfg, L.exec_config(fuse_gather=fuse, fp8=fp8, fuse_combine=fc,
-                                               unit_trace=rt), W, d["x"], out, None, ws, stream)
-        torch.cuda.synchronize()
-        line["gemm1_units"] = unit_trace_summary(rt.cpu().numpy(), wl.H, fp8)
+        # one extra forward per traced GEMM; GEMM2's units cover 256 output
+        # features (128 when H is not a multiple of 256) over K = I
+        feat2 = 256 if wl.H % 256 == 0 else 128
+        for gemm, key, fpr in ((1, "gemm1_units", 2 * 2 * 128 * wl.H),
+                               (2, "gemm2_units", 2 * feat2 * wl.I)):
+            rt = torch.zeros((1 << 17, L.UNIT_TRACE_FIELDS), dtype=torch.int64, device=device)
+            L.moe_layer_forward(cfg, L.exec_config(fuse_gather=fuse, fp8=fp8, fuse_combine=fc,
+                                                   unit_trace=rt, unit_trace_gemm=gemm),
+                                W, d["x"], out, None, ws, stream)
+            torch.cuda.synchronize()
+            line[key] = unit_trace_summary(rt.cpu().numpy(), wl.H, fp8, fpr)
     if overlap:
         line["overlap"] = overlap
     if dispatch_fusion:

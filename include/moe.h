@@ -126,16 +126,19 @@ typedef struct {
    * (overlap = 0) forward; NULL = no tracing. Ignored when overlap = 1. */
   void** stage_events;
   int32_t fp8, fuse_combine;
-  /* Optional per-unit trace of the grouped GEMM1 launch (no counterpart in the
+  /* Optional per-unit trace of one grouped GEMM launch (no counterpart in the
    * paper; a profiling aid): a device buffer of unit_trace_cap records of 5
-   * uint64, written by a sequential forward for GEMM1's work units
-   * u < unit_trace_cap (the shared expert's units first, then the routed
-   * experts' in expert order). Record u: the time the unit was handed to its
+   * uint64, written by a sequential forward for the work units
+   * u < unit_trace_cap of GEMM1 (unit_trace_gemm 0 or 1) or GEMM2
+   * (unit_trace_gemm 2); the shared expert's units first, then the routed
+   * experts' in expert order. Record u: the time the unit was handed to its
    * CTA, the time its first operand stage was ready for the MMAs, the time its
    * accumulator was complete, the time its epilogue had stored it (all
    * %globaltimer nanoseconds), then SM id | token rows << 16 | (expert +
-   * 1024 * (1 for the shared expert)) << 32 | feature block << 48. Records of
-   * units that did not run are left untouched. NULL = off. */
+   * 1024 * (1 for the shared expert)) << 32 | feature block << 48 (GEMM1:
+   * blocks of 128 features of h; GEMM2: of 256 output features, or 128 when
+   * H is not a multiple of 256). Records of units that did not run are left
+   * untouched. NULL = off. */
   unsigned long long* unit_trace;
   int32_t unit_trace_cap;
   /* Optional timeline of a pipelined forward (overlap = 1; a profiling aid):
@@ -149,6 +152,9 @@ typedef struct {
    * past n_pipe_events are not recorded. NULL = off; ignored when overlap = 0. */
   void** pipe_events;
   int32_t n_pipe_events;
+  /* Which GEMM unit_trace records: 0 or 1 = GEMM1, 2 = GEMM2; else
+   * MOE_ERR_INVALID_ARG. */
+  int32_t unit_trace_gemm;
 } moe_exec;
 
 /* Indices into moe_exec.stage_events: event i is recorded when stage i ends

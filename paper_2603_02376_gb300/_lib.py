@@ -58,7 +58,8 @@ class moe_exec(ctypes.Structure):
                [("stage_events", ctypes.POINTER(ctypes.c_void_p)), ("fp8", ctypes.c_int32),
                 ("fuse_combine", ctypes.c_int32), ("unit_trace", ctypes.c_void_p),
                 ("unit_trace_cap", ctypes.c_int32),
-                ("pipe_events", ctypes.POINTER(ctypes.c_void_p)), ("n_pipe_events", ctypes.c_int32)]
+                ("pipe_events", ctypes.POINTER(ctypes.c_void_p)), ("n_pipe_events", ctypes.c_int32),
+                ("unit_trace_gemm", ctypes.c_int32)]
 
 
 STAGES = ("start", "router", "gate", "permute", "dispatch", "gemm1", "gemm2", "shared_gemm1",
@@ -186,14 +187,16 @@ UNIT_TRACE_FIELDS = 5
 
 def exec_config(overlap=0, chunk_tokens=512, chunk_axis=0, n_expert_chunks=8, out_fp32=0,
                 fuse_gather=1, stage_events=None, fp8=0, fuse_combine=0, unit_trace=None,
-                pipe_events=None):
+                pipe_events=None, unit_trace_gemm=1):
     """moe_exec; stage_events: a list of MOE_N_STAGE_EVENTS torch.cuda.Event (or None);
-    unit_trace: an int64 device tensor [cap, UNIT_TRACE_FIELDS] (or None); pipe_events:
-    a list of timing torch.cuda.Event for a pipelined forward's timeline (or None)."""
+    unit_trace: an int64 device tensor [cap, UNIT_TRACE_FIELDS] (or None), filled for
+    GEMM1 (unit_trace_gemm 1) or GEMM2 (2); pipe_events: a list of timing
+    torch.cuda.Event for a pipelined forward's timeline (or None)."""
     cap = 0 if unit_trace is None else unit_trace.shape[0]
     ex = moe_exec(overlap, chunk_tokens, chunk_axis, n_expert_chunks, out_fp32, fuse_gather, None,
                   int(fp8), int(fuse_combine),
-                  None if unit_trace is None else unit_trace.data_ptr(), cap, None, 0)
+                  None if unit_trace is None else unit_trace.data_ptr(), cap, None, 0,
+                  int(unit_trace_gemm))
     if pipe_events:
         arr = (ctypes.c_void_p * len(pipe_events))(*[int(e.cuda_event) for e in pipe_events])
         ex._pipe_keepalive = arr

@@ -183,9 +183,11 @@ struct FfnGroup {
   int pack_src_rows;
   int* pack_next;
   int* pack_ready;
-  // Per-unit trace of the GEMM1 launch (moe_exec.unit_trace; null = off).
+  // Per-unit trace of the GEMM1 (trace_gemm 1) or GEMM2 (2) launch
+  // (moe_exec.unit_trace; null = off).
   unsigned long long* trace;
   int trace_cap;
+  int trace_gemm;
 };
 
 // The expert GEMMs' token tile for rows_hint packed rows over n_exp experts:

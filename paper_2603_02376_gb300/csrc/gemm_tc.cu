@@ -1516,8 +1516,9 @@ moe_status run_ffn(const FfnGroup& g0, const FfnGroup* g1, int H, int I, cudaStr
     args.pack_next = g0.pack_next;
     args.pack_ready = g0.pack_ready;
   }
-  args.trace = g0.trace;
-  args.trace_cap = g0.trace ? g0.trace_cap : 0;
+  const bool trace2 = g0.trace && g0.trace_gemm == 2;  // the trace is GEMM2's
+  args.trace = trace2 ? nullptr : g0.trace;
+  args.trace_cap = args.trace ? g0.trace_cap : 0;
   args.b_tiled0 = g0.x_tiled ? static_cast<const uint8_t*>(g0.x) : nullptr;
   args.b_tiled1 = (g1 && g1->x_tiled) ? static_cast<const uint8_t*>(g1->x) : nullptr;
   args.out_tiled0 = g0.h_tiled;
@@ -1554,7 +1555,8 @@ moe_status run_ffn(const FfnGroup& g0, const FfnGroup* g1, int H, int I, cudaStr
   args.out_tiled1 = 0;
   args.pack_src = nullptr;
   args.pack_dst = nullptr;
-  args.trace = nullptr;
+  args.trace = trace2 ? g0.trace : nullptr;
+  args.trace_cap = trace2 ? g0.trace_cap : 0;
   args.a0_packed = pk ? static_cast<const uint16_t*>(g0.W2) : nullptr;
   args.a1_packed = (pk && g1) ? static_cast<const uint16_t*>(g1->W2) : nullptr;
   if (F8 && !MX) {

@@ -92,6 +92,7 @@ bool valid_exec(const moe_exec* ex, const moe_config* c) {
   if (ex->fp8 < 0 || ex->fp8 > 2) return false;
   if (ex->fuse_combine != 0 && ex->fuse_combine != 1) return false;
   if (ex->unit_trace_cap < 0 || (ex->unit_trace && ex->unit_trace_cap == 0)) return false;
+  if (ex->unit_trace_gemm < 0 || ex->unit_trace_gemm > 2) return false;
   if (ex->n_pipe_events < 0 || (ex->pipe_events && ex->n_pipe_events == 0)) return false;
   if (ex->overlap) {
     if (ex->chunk_axis == 0) {
@@ -476,6 +477,7 @@ moe_status experts_tokens(const moe_config& c, const Layout& L, const moe_weight
   if (ex && ex->unit_trace) {
     g.trace = ex->unit_trace;
     g.trace_cap = ex->unit_trace_cap;
+    g.trace_gemm = ex->unit_trace_gemm == 2 ? 2 : 1;
   }
   const long hint = (long)g.rows * (e1 - e0) / c.E;
   MOE_TRY(launch_expert_ffn_groups(g, nullptr, c.H, c.I, (int)hint, s,
@@ -507,6 +509,7 @@ moe_status experts_and_shared(const moe_config& c, const Layout& L, const moe_we
   if (ex && ex->unit_trace) {
     routed.trace = ex->unit_trace;
     routed.trace_cap = ex->unit_trace_cap;
+    routed.trace_gemm = ex->unit_trace_gemm == 2 ? 2 : 1;
   }
   const FfnGroup dense = dense_group(c, L, w, x);
   MOE_TRY(launch_expert_ffn_groups(routed, &dense, c.H, c.I, routed.rows, s,

@@ -187,6 +187,11 @@ def test_exec_options_validated_on_the_host():
     ex = L.exec_config()
     ex.unit_trace_cap = -1
     assert L.moe_workspace_size(c, ex) == 0
+    # the traced GEMM: 0 or 1 (GEMM1) or 2 (GEMM2)
+    for g, ok in ((0, True), (1, True), (2, True), (3, False), (-1, False)):
+        ex = L.exec_config(unit_trace_gemm=g)
+        assert (L.moe_workspace_size(c, ex) == ws0 and ws0 > 0) if ok else \
+            L.moe_workspace_size(c, ex) == 0, g
     ex = L.exec_config(overlap=1)
     ex.n_pipe_events = -1
     assert L.moe_workspace_size(c, ex) == 0

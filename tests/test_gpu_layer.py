@@ -182,14 +182,16 @@ def test_layer_small_grouped_full(I_shared, T):
     check_permutation(wl, d, gidx)
 
 
-def test_unit_trace_records_every_gemm1_unit():
-    """moe_exec.unit_trace: one record per GEMM1 work unit, times in order, the
-    token rows of the routed records summing to T*k (one feature block: I = 128)."""
+@pytest.mark.parametrize("gemm", [1, 2])
+def test_unit_trace_records_every_gemm_unit(gemm):
+    """moe_exec.unit_trace: one record per work unit of the traced GEMM, times in
+    order, the token rows of the routed records summing to T*k (one feature block
+    in both GEMMs: I = 128 features of h; H = 256 output features per GEMM2 unit)."""
     wl = I.Workload("small", T=100, H=256, E=16, k=4, I=128, I_shared=128, n_groups=4,
                     topk_groups=2, gate=I.GATE_SIGMOID, normalize=1, route_scale=2.5)
     d = I.layer_inputs(wl, seed=5, device=DEV)
     rt = torch.zeros((256, L.UNIT_TRACE_FIELDS), dtype=torch.int64, device=DEV)
-    out, a = run_layer(wl, d, L.exec_config(out_fp32=1, unit_trace=rt))
+    out, a = run_layer(wl, d, L.exec_config(out_fp32=1, unit_trace=rt, unit_trace_gemm=gemm))
     rec = rt.cpu().numpy()
     used = rec[:, 3] != 0
     meta = rec[used, 4]
@@ -202,6 +204,10 @@ def test_unit_trace_records_every_gemm1_unit():
     t = rec[used, :4]
     assert (np.diff(t, axis=1) >= 0).all()
     assert not rec[~used].any()                         # nothing written past the units
+    assert not ((meta >> 48) & 0xFFFF).any()            # the single feature block
+    ref, _ = O.layer_forward(f64(d["x"]), f64(d["Wr"]), bias32(d["bias"]), f64(d["W13"]),
+                             f64(d["W2"]), oracle_cfg(wl), f64(d["Ws13"]), f64(d["Ws2"]))
+    assert_layer_close(out, ref)                        # tracing leaves the output intact
 
 
 @pytest.mark.parametrize("axis,n", [(1, 3), (0, 37)])

@@ -216,6 +216,29 @@ def check_routing_fp8(wl, d, a, toks):
                                   np.bincount(ridx.reshape(-1), minlength=wl.E))
 
 
+@pytest.mark.parametrize("T", [150, 8])
+def test_layer_fp8_one_tile_gemm2_full(T):
+    """Row-scaled FP8 with H = 384: GEMM2 (one 128-feature tile per unit) reads
+    the e4m3 copy of h in the tile-packed layout; 144- and 32-row token tiles;
+    the packed dispatch, the copy inside GEMM1 and the expert-range pipeline;
+    every token against the oracle's FP8 chain."""
+    wl = I.Workload("one-tile gemm2 fp8", T=T, H=384, E=12, k=3, I=256, I_shared=256,
+                    n_groups=4, topk_groups=2, gate=I.GATE_SIGMOID, normalize=1,
+                    route_scale=2.5)
+    d = I.layer_inputs(wl, seed=7, device=DEV, with_experts=False)
+    d["W13"], d["s13"], d["W2"], d["s2"] = I.fp8_expert_weights(wl, 7, DEV)
+    d["Ws13"], d["ss13"], d["Ws2"], d["ss2"] = I.fp8_shared_weights(wl, 7, DEV)
+    prepare_routing(wl, d)
+    toks = np.arange(wl.T)
+    ref, idx = oracle_fp8_tokens(wl, d, toks)
+    for ex in (L.exec_config(out_fp32=1, fp8=1, fuse_gather=0),
+               L.exec_config(out_fp32=1, fp8=1, fuse_gather=2),
+               L.exec_config(out_fp32=1, fp8=1, overlap=1, chunk_axis=1, n_expert_chunks=5)):
+        out, a = run_fp8_layer(wl, d, ex)
+        check_routing_fp8(wl, d, a, toks)
+        assert_layer_close(out, ref)
+
+
 @pytest.fixture(scope="module")
 def fp8_decode(fp8_layer):
     """Decode batch (T=128) on the FP8 layer, routing made well-posed, oracle on every token."""

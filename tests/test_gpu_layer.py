@@ -182,6 +182,35 @@ def test_layer_small_grouped_full(I_shared, T):
     check_permutation(wl, d, gidx)
 
 
+@pytest.mark.parametrize("T,I_shared", [(150, 256), (150, 128), (8, 256)])
+def test_layer_one_tile_gemm2_full(T, I_shared):
+    """H = 384 (not a multiple of 256): GEMM2 takes one 128-feature weight tile per
+    unit (MODE_PLAIN) and reads h in the tile-packed layout of 144-row (T = 150,
+    ~37 rows per expert) or 32-row (T = 8) token tiles; I = 256 gives GEMM1 two
+    feature blocks. The shared expert inside the routed launches (I_s = I) or in
+    its own launches (I_s = 128). Every dispatch form, the fused combine and the
+    expert-range pipeline; every token against the oracle."""
+    wl = I.Workload("one-tile gemm2", T=T, H=384, E=12, k=3, I=256, I_shared=I_shared,
+                    n_groups=4, topk_groups=2, gate=I.GATE_SIGMOID, normalize=1,
+                    route_scale=2.5)
+    d = I.layer_inputs(wl, seed=7, device=DEV)
+    st = prepare_routing(wl, d)
+    ref, _ = O.layer_forward(f64(d["x"]), f64(d["Wr"]), bias32(d["bias"]), f64(d["W13"]),
+                             f64(d["W2"]), oracle_cfg(wl), f64(d["Ws13"]), f64(d["Ws2"]))
+    dp = packed_copy(d)
+    for dd, ex in ((d, L.exec_config(out_fp32=1, fuse_gather=0)),
+                   (dp, L.exec_config(out_fp32=1, fuse_gather=0)),
+                   (dp, L.exec_config(out_fp32=1, fuse_gather=1)),
+                   (dp, L.exec_config(out_fp32=1, fuse_gather=2)),
+                   (dp, L.exec_config(out_fp32=0, fuse_gather=2, fuse_combine=1)),
+                   (dp, L.exec_config(out_fp32=1, overlap=1, chunk_axis=1, n_expert_chunks=5)),
+                   (dp, L.exec_config(out_fp32=1, overlap=1, chunk_axis=0, chunk_tokens=64))):
+        out, a = run_layer(wl, dd, ex)
+        gidx = check_routing(wl, dd, a, st["oracle_logits"])
+        assert_layer_close(out, ref)
+    check_permutation(wl, d, gidx)
+
+
 @pytest.mark.parametrize("gemm", [1, 2])
 def test_unit_trace_records_every_gemm_unit(gemm):
     """moe_exec.unit_trace: one record per work unit of the traced GEMM, times in

@@ -449,14 +449,16 @@ struct GemmArgs {
   int pack_src_rows;
   int* pack_next;
   int* pack_ready;
-  // bf16 token operands in the tile-packed row layout (TiledRow, tile = NMAX):
-  // group g's token rows come from b_tiled_g by one bulk copy per stage (null:
-  // through the tensor maps), and GEMM1 writes group g's h to out_g in that
-  // layout when out_tiled_g. Padded rows: row0 + 16 * (global expert).
+  // Token operands (bf16, or e4m3 rows) in the tile-packed row layout
+  // (TiledRow, tile = NMAX): group g's token rows come from b_tiled_g by one
+  // bulk copy per stage (null: through the tensor maps), and GEMM1 writes group
+  // g's bf16 h to out_g in that layout when out_tiled_g. A tile's first padded
+  // row: row0 + 16 * (its global expert; 0 for group 1). The buffers hold 16
+  // padding rows per expert.
   const uint8_t* b_tiled0;
   const uint8_t* b_tiled1;
   int out_tiled0, out_tiled1;
-  // Per-unit trace (GEMM1 only; null = off): record u < trace_cap of
+  // Per-unit trace of this launch (null = off): record u < trace_cap of
   // TRACE_FIELDS uint64: the unit's announcement by the producer, its first
   // stage ready at the MMA thread, its accumulator complete and its epilogue
   // done (warp 2), all %globaltimer ns, then SM id | m << 16 |

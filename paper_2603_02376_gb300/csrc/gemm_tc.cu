@@ -1242,20 +1242,27 @@ __global__ void __launch_bounds__(threads_of(MODE, Q), 1)
             uint32_t v[16];
             tmem_ld16(tq + NMAX + c0, v);
             tmem_wait_ld();
+            // the chunk's 16 SwiGLU values first, in straight-line code (16
+            // independent chains the scheduler can interleave), then the stores
+            // of the valid columns
+            uint32_t hb[16];
 #pragma unroll
             for (int i = 0; i < 16; ++i) {
               const float sb = RS ? __shfl_sync(0xffffffffu, sb_l, i) : 1.f;
+              const float gv = __uint_as_float(g[i]) * (sa0 * sb);
+              const float uv = __uint_as_float(v[i]) * (sa1 * sb);
+              hb[i] = float_to_bf16_bits(silu_mul(gv, uv));
+            }
+#pragma unroll
+            for (int i = 0; i < 16; ++i) {
               if (c0 + i < U.m) {
-                const float gv = __uint_as_float(g[i]) * (sa0 * sb);
-                const float uv = __uint_as_float(v[i]) * (sa1 * sb);
-                const float hv = silu_mul(gv, uv);
                 // tile-packed h: token column c = c0 + i is row c of the tile;
                 // this thread's feature f is element f % 8 of 16-byte chunk
                 // (f % 64) / 8 of block f / 64
                 const int c = c0 + i;
                 const size_t idx = h_tiled ? h_blk + (size_t)c * 64 + ((h_chk ^ (c & 7)) << 3)
                                            : o + (size_t)c * a.out_ld;
-                static_cast<uint16_t*>(out)[idx] = float_to_bf16_bits(hv);
+                static_cast<uint16_t*>(out)[idx] = (uint16_t)hb[i];
               }
             }
           } else if constexpr (MODE == MODE_PLAIN2) {

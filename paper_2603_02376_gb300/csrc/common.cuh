@@ -183,6 +183,12 @@ struct FfnGroup {
   int pack_src_rows;
   int* pack_next;
   int* pack_ready;
+  // Token-major copy (used when the launch also runs group 1, whose units come
+  // first): pack_slot[t * pack_k + j] is the packed row of token t's slot j.
+  // Each token row is then read once for its pack_k rows. Null: packed-row
+  // order through pack_rst.
+  const int32_t* pack_slot;
+  int pack_k;
   // Per-unit trace of the GEMM1 (trace_gemm 1) or GEMM2 (2) launch
   // (moe_exec.unit_trace; null = off).
   unsigned long long* trace;

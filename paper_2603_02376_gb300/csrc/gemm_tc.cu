@@ -449,6 +449,10 @@ struct GemmArgs {
   int pack_src_rows;
   int* pack_next;
   int* pack_ready;
+  // Token-major form (non-null): pack_next hands out chunks of tokens and
+  // token t's slot j goes to packed row pack_slot[t * pack_k + j].
+  const int32_t* pack_slot;
+  int pack_k;
   // Token operands (bf16, or e4m3 rows) in the tile-packed row layout
   // (TiledRow, tile = NMAX): group g's token rows come from b_tiled_g by one
   // bulk copy per stage (null: through the tensor maps), and GEMM1 writes group
@@ -1073,7 +1077,96 @@ __global__ void __launch_bounds__(threads_of(MODE, Q), 1)
     // at once), then adds the rows to their experts' counts with release
     // semantics. Rows with a source index outside the source matrix are left
     // unwritten and latched as MOE_ERR_DEVICE_CHECK; they are still counted.
-    if (a.pack_dst) {
+    //
+    // Token-major form (pack_slot non-null; the shared expert's units run first,
+    // so the routed units' waits for whole experts fall behind them): a warp
+    // takes TPC consecutive tokens, loads each token row once and stores it to
+    // the packed rows of all its pack_k slots, lane s holding slot s's
+    // destination; x is read once instead of once per slot. A slot row outside
+    // this launch's rows is skipped and latched as MOE_ERR_DEVICE_CHECK (its
+    // expert's count then stays short and the producer's bounded wait expires).
+    if (a.pack_dst && a.pack_slot) {
+      const int r_begin = row_off[0], r_end = row_off[a.n_exp];
+      const int vpr = a.K * (F8 ? 1 : 2) / 16;  // 16-byte vectors per row
+      const int kk = a.pack_k;                  // 1..32 (checked on the host)
+      const int tpc = min(PACK_ROWS, 32 / kk);  // tokens per chunk: tpc * kk <= 32
+      const int n_tok = a.pack_src_rows;
+      const int n_chunks = (n_tok + tpc - 1) / tpc;
+      const bool tiled = a.b_tiled0 != nullptr;
+      while (!*abort_flag) {
+        int c = 0;
+        if (lane == 0) c = atomicAdd(a.pack_next, 1);
+        c = __shfl_sync(0xffffffffu, c, 0);
+        if (c >= n_chunks) break;
+        const int t0 = c * tpc, nt = min(tpc, n_tok - t0), ns = nt * kk;
+        // lane s < ns: slot s (token t0 + s / kk, slot s % kk) -> its expert
+        // (binary search over the clamped offsets) and destination: the tile's
+        // first 16-byte unit and (row in tile | padded rows << 16), or the row's
+        // first unit (row-major); ipk < 0 marks no slot
+        int e_s = -1, ipk = -1;
+        unsigned long long d0 = 0;
+        if (lane < ns) {
+          const int r = a.pack_slot[(size_t)t0 * kk + lane];
+          if (r >= r_begin && r < r_end) {
+            int lo = 0, hi = a.n_exp - 1;
+            while (lo < hi) {
+              const int mid = (lo + hi + 1) >> 1;
+              if (row_off[mid] <= r) lo = mid;
+              else hi = mid - 1;
+            }
+            e_s = lo;
+            if (tiled) {
+              const TiledRow w = tiled_row(r, a.e_begin + lo, row_off[lo],
+                                           row_off[lo + 1] - row_off[lo], NMAX, vpr);
+              d0 = w.tile16;
+              ipk = w.i | (w.n_pad << 16);
+            } else {
+              d0 = (unsigned long long)r * vpr;
+              ipk = 0;
+            }
+          } else {
+            atomicExch(err, (int)MOE_ERR_DEVICE_CHECK);
+          }
+        }
+        // the trip count is the same for every lane (the slot destinations are
+        // shuffled inside the loop); lanes past the row's end only skip their
+        // loads and stores
+        for (int vb = 0; vb < vpr; vb += 64) {
+          const int v0 = vb + lane;
+          uint4 val[PACK_ROWS][2];
+#pragma unroll
+          for (int q = 0; q < PACK_ROWS; ++q)
+#pragma unroll
+            for (int h = 0; h < 2; ++h)
+              if (q < nt && v0 + 32 * h < vpr)
+                val[q][h] = a.pack_src[(size_t)(t0 + q) * vpr + v0 + 32 * h];
+#pragma unroll
+          for (int q = 0; q < PACK_ROWS; ++q) {
+            if (q >= nt) break;
+            for (int j = 0; j < kk; ++j) {
+              const int sl = q * kk + j;
+              const unsigned long long ds = __shfl_sync(0xffffffffu, d0, sl);
+              const int ip = __shfl_sync(0xffffffffu, ipk, sl);
+              if (ip < 0) continue;
+              TiledRow w;
+              w.tile16 = ds;
+              w.i = ip & 0xffff;
+              w.n_pad = ip >> 16;
+#pragma unroll
+              for (int h = 0; h < 2; ++h)
+                if (v0 + 32 * h < vpr)
+                  a.pack_dst[tiled ? w.chunk16(v0 + 32 * h) : ds + v0 + 32 * h] = val[q][h];
+            }
+          }
+        }
+        __threadfence();
+        fence_proxy_async_global();
+        __syncwarp();
+        if (e_s >= 0)
+          asm volatile("red.release.gpu.global.add.s32 [%0], %1;" ::"l"(a.pack_ready + e_s), "r"(1)
+                       : "memory");
+      }
+    } else if (a.pack_dst) {
       const int r_begin = row_off[0], r_end = row_off[a.n_exp];
       const int vpr = a.K * (F8 ? 1 : 2) / 16;  // 16-byte vectors per row
       const int n_chunks = (r_end - r_begin + PACK_ROWS - 1) / PACK_ROWS;
@@ -1524,6 +1617,12 @@ moe_status run_ffn(const FfnGroup& g0, const FfnGroup* g1, int H, int I, cudaStr
     args.pack_src_rows = g0.pack_src_rows;
     args.pack_next = g0.pack_next;
     args.pack_ready = g0.pack_ready;
+    // token-major only behind the shared expert's units: without them the
+    // routed units would wait for the whole copy instead of expert by expert
+    if (g1 && g0.pack_slot && g0.pack_k >= 1 && g0.pack_k <= 32) {
+      args.pack_slot = g0.pack_slot;
+      args.pack_k = g0.pack_k;
+    }
   }
   const bool trace2 = g0.trace && g0.trace_gemm == 2;  // the trace is GEMM2's
   args.trace = trace2 ? nullptr : g0.trace;

@@ -399,6 +399,8 @@ FfnGroup routed_group(const moe_config& c, const Layout& L, const moe_weights& w
       g.pack_src_rows = Tc;
       g.pack_next = L.pack_next;
       g.pack_ready = L.pack_ready + e0;
+      g.pack_slot = L.slot_row + tk;  // token-major copy when the shared expert runs first
+      g.pack_k = c.k;
     }
   } else {
     g.x = L.fp8 ? static_cast<const void*>(L.x_q + (size_t)t0 * c.H)

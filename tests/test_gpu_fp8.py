@@ -239,6 +239,30 @@ def test_layer_fp8_one_tile_gemm2_full(T):
         assert_layer_close(out, ref)
 
 
+@pytest.mark.parametrize("H,E,k,T", [(128, 8, 2, 70), (256, 40, 32, 33)])
+def test_layer_fp8_copy_in_gemm1_token_major_full(H, E, k, T):
+    """Row-scaled FP8 with the e4m3 dispatch copy inside GEMM1 (token-major, the
+    shared expert in the launch): rows of 8 and 16 16-byte vectors (H = 128 and
+    256 e4m3 bytes), k = 2 and 32; every token against the oracle's FP8 chain."""
+    wl = I.Workload("fp8 token-major copy", T=T, H=H, E=E, k=k, I=128, I_shared=128,
+                    gate=I.GATE_SIGMOID, normalize=1, route_scale=2.5)
+    d = I.layer_inputs(wl, seed=13, device=DEV, with_experts=False)
+    d["W13"], d["s13"], d["W2"], d["s2"] = I.fp8_expert_weights(wl, 13, DEV)
+    d["Ws13"], d["ss13"], d["Ws2"], d["ss2"] = I.fp8_shared_weights(wl, 13, DEV)
+    prepare_routing(wl, d)
+    toks = np.arange(wl.T)
+    ref, idx = oracle_fp8_tokens(wl, d, toks)
+    outs = []
+    for ex in (L.exec_config(out_fp32=1, fp8=1, fuse_gather=0),
+               L.exec_config(out_fp32=1, fp8=1, fuse_gather=2)):
+        out, a = run_fp8_layer(wl, d, ex)
+        check_routing_fp8(wl, d, a, toks)
+        assert_layer_close(out, ref)
+        outs.append(out)
+    # the same e4m3 bytes in the same rows as the dispatch kernel's
+    assert float((outs[1] - outs[0]).abs().max()) <= 1e-5 * float(np.abs(ref).max())
+
+
 @pytest.fixture(scope="module")
 def fp8_decode(fp8_layer):
     """Decode batch (T=128) on the FP8 layer, routing made well-posed, oracle on every token."""

@@ -211,6 +211,40 @@ def test_layer_one_tile_gemm2_full(T, I_shared):
     check_permutation(wl, d, gidx)
 
 
+@pytest.mark.parametrize("H,E,k,T", [(128, 8, 2, 70), (128, 12, 6, 50), (256, 40, 32, 33)])
+def test_layer_copy_in_gemm1_token_major_full(H, E, k, T):
+    """The dispatch copy inside GEMM1 with the shared expert in the same launch
+    copies token-major (each token row read once for its k slots): rows of 16
+    16-byte vectors (H = 128, fewer than a warp's lanes), k = 2 and 6 (chunks of
+    four tokens, 8 and 24 slots), k = 32 (one token, 32 slots per chunk);
+    row-major and tile-packed weights; every token against the oracle, and
+    against the same layer with the rows packed by the dispatch kernel (the
+    copy moves the same bytes to the same rows, so the outputs agree to within
+    fp32 rounding of |out|, far below the layer tolerance at these small
+    outputs)."""
+    wl = I.Workload("token-major copy", T=T, H=H, E=E, k=k, I=128, I_shared=128,
+                    gate=I.GATE_SIGMOID, normalize=1, route_scale=2.5)
+    d = I.layer_inputs(wl, seed=11, device=DEV)
+    st = prepare_routing(wl, d)
+    ref, _ = O.layer_forward(f64(d["x"]), f64(d["Wr"]), bias32(d["bias"]), f64(d["W13"]),
+                             f64(d["W2"]), oracle_cfg(wl), f64(d["Ws13"]), f64(d["Ws2"]))
+    dp = packed_copy(d)
+    base = {}
+    for name, dd, ex in (("rows", d, L.exec_config(out_fp32=1, fuse_gather=0)),
+                         ("packed", dp, L.exec_config(out_fp32=1, fuse_gather=0)),
+                         ("rows", d, L.exec_config(out_fp32=1, fuse_gather=2)),
+                         ("packed", dp, L.exec_config(out_fp32=1, fuse_gather=2))):
+        out, a = run_layer(wl, dd, ex)
+        gidx = check_routing(wl, dd, a, st["oracle_logits"])
+        assert_layer_close(out, ref)
+        if name in base:
+            lim = 1e-5 * float(np.abs(ref).max())
+            assert float((out - base[name]).abs().max()) <= lim
+        else:
+            base[name] = out
+    check_permutation(wl, d, gidx)
+
+
 @pytest.mark.parametrize("gemm", [1, 2])
 def test_unit_trace_records_every_gemm_unit(gemm):
     """moe_exec.unit_trace: one record per work unit of the traced GEMM, times in

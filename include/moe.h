@@ -90,11 +90,14 @@ typedef struct {
  *    k-block costs more than the copy once tiles hold ~128 rows).
  *    2 = the dispatch copy runs inside the GEMM1 launch, at every batch size
  *    (sequential forward, bf16 or row-scaled FP8; otherwise as 0): warps of
- *    GEMM1 write x_perm in expert order while the shared expert's units, which
- *    read x directly and come first, compute; each routed expert's token tiles
- *    are loaded once all its rows are written (a bounded wait; on expiry
- *    MOE_ERR_TIMEOUT is latched). This is the single-kernel form of the paper's
- *    dispatch hidden behind the layer's own compute (Section 4.3).
+ *    GEMM1 write x_perm while the shared expert's units, which read x directly
+ *    and come first, compute; each routed expert's token tiles are loaded once
+ *    all its rows are written (a bounded wait; on expiry MOE_ERR_TIMEOUT is
+ *    latched). With the shared expert in the same launch (I_shared == I) the
+ *    copy is token-major, each token row read once for its k packed rows;
+ *    otherwise it goes in expert order, so the first experts' tiles can start
+ *    early. This is the single-kernel form of the paper's dispatch hidden
+ *    behind the layer's own compute (Section 4.3).
  *  fp8 0 = bf16 expert GEMMs; 1 = FP8 (e4m3) expert GEMMs, the quantized
  *    pipeline of the paper's MoE workload (Section 4.3 lists an FP8 quantize
  *    stage before the dispatch): after the gate every token row x[t] is

@@ -40,13 +40,16 @@
 //              (tcgen05.cp) ahead of block_scale MMAs;
 //   warps 10-13 GEMM1 with bf16 or row-scaled e4m3 operands: the dispatch
 //              fused into the launch (GemmArgs::pack_dst). They copy the
-//              token rows into the packed order, a chunk of rows at a time
-//              taken from a global counter in row (= expert) order, and count
-//              each expert's packed rows; the producer waits for an expert's
-//              count before loading its token tiles. The shared expert's
-//              units (which read x itself) come first in the unit order, so
-//              the copy runs while they compute: the paper's dispatch hidden
-//              behind the layer's own compute, inside one kernel.
+//              token rows into the packed order, a chunk at a time taken from
+//              a global counter: a few tokens, each row read once and written
+//              to its k packed rows, when the launch also runs the shared
+//              expert; else a few packed rows in row (= expert) order. They
+//              count each expert's packed rows; the producer waits for an
+//              expert's count before loading its token tiles. The shared
+//              expert's units (which read x itself) come first in the unit
+//              order, so the copy runs while they compute: the paper's
+//              dispatch hidden behind the layer's own compute, inside one
+//              kernel.
 // For SwiGLU the gate and up tiles of the same 128 features are two MMAs into
 // two TMEM column ranges, so one thread holds both g and u of its feature.
 // When two accumulators fit in TMEM's 512 columns they alternate, so the

@@ -537,7 +537,7 @@ def cpu_baseline(wl, d, n_tokens, seed=1, one_core_tokens=0):
 
 # ---------------------------------------------------------------- main arms
 
-REF_BUDGET_S = 90.0  # the reference arm's timed steps together take about this long
+REF_TIMED_S = 90.0  # the reference arm's timed steps together take about this long
 
 
 def run_reference(args, wl, rank, world, device):
@@ -549,10 +549,10 @@ def run_reference(args, wl, rank, world, device):
         L.load()
         calibrate(L, wl, d, device)
     # per-step sample: a first untimed call measures the oracle's cost per token,
-    # then each timed step takes as many tokens as keep the K steps within the budget
+    # then each timed step takes as many tokens as keep the K steps near REF_TIMED_S
     n_max = max(1, (args.cpu_tokens or 128) // 2)
     v0, _, _ = oracle_tokens_per_s(wl, d, I.sample_tokens(wl.T, min(8, n_max), 99).numpy())
-    n = int(max(1, min(n_max, REF_BUDGET_S * v0 / max(args.steps, 1))))
+    n = int(max(1, min(n_max, REF_TIMED_S * v0 / max(args.steps, 1))))
     for s in range(args.warmup):
         oracle_tokens_per_s(wl, d, I.sample_tokens(wl.T, n, 100 + s).numpy())
     times = []
